@@ -1,0 +1,245 @@
+"""ST-Lite reference oracle -- TEST INFRASTRUCTURE ONLY.
+
+Thin ctypes wrapper around ``stlite_oracle.c``: a plain, slow, fp64 CPU
+restatement of the ST-Lite compression procedure (Algorithm 1 of arXiv
+2603.00188; Eqs. 2, 4-9).  Only the test suite, the package smoke check and
+the benchmark's CPU-baseline leg may import this module.  It shares no code
+with the CUDA library and never imports it.
+
+Arrays: ``q`` [w, Hq, d] and ``k`` [N, Hkv, d] as float64 (exact copies of the
+bf16/fp32 inputs).  Frames are three int32 arrays (offset, grid_h, grid_w);
+the last frame is the current frame.  Per-head results are [Hkv, N].
+
+Every function here is pinned by ``tests/test_oracle_pins.py`` to closed
+forms, invariants, hand-computed fixtures (``tests/golden/``) and brute force.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+from concurrent.futures import ThreadPoolExecutor
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "stlite_oracle.c")
+_SO = os.path.join(_HERE, "libstlite_oracle.so")
+_lib = None
+
+_dp = ctypes.POINTER(ctypes.c_double)
+_ip = ctypes.POINTER(ctypes.c_int32)
+_bp = ctypes.POINTER(ctypes.c_uint8)
+_i32 = ctypes.c_int32
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle with gcc (plain -O2, IEEE semantics kept)."""
+    if force or not os.path.exists(_SO) or os.path.getmtime(_SO) < os.path.getmtime(_SRC):
+        tmp = _SO + ".tmp%d" % os.getpid()
+        subprocess.check_call(["gcc", "-O2", "-std=c11", "-fPIC", "-shared", _SRC, "-o", tmp, "-lm"])
+        os.replace(tmp, _SO)
+    return _SO
+
+
+def _load():
+    global _lib
+    if _lib is None:
+        build()
+        lib = ctypes.CDLL(_SO)
+        lib.orc_budget.restype = _i32
+        lib.orc_budget.argtypes = [_i32, ctypes.c_double, _i32]
+        lib.orc_abase.restype = None
+        lib.orc_abase.argtypes = [_dp, _dp, _i32, _i32, _i32, _i32, _i32, _i32, _dp]
+        lib.orc_css_phi_token.restype = ctypes.c_double
+        lib.orc_css_phi_token.argtypes = [_dp, _i32, _i32, _i32, _i32, _i32, _i32, _i32, _i32]
+        lib.orc_css_phi.restype = None
+        lib.orc_css_phi.argtypes = [_dp, _i32, _i32, _i32, _i32, _i32, _ip, _ip, _ip, _dp]
+        lib.orc_tsg_rho_token.restype = ctypes.c_double
+        lib.orc_tsg_rho_token.argtypes = [_dp, _i32, _i32, _i32, _i32, _i32, _i32]
+        lib.orc_tsg_rho.restype = None
+        lib.orc_tsg_rho.argtypes = [_dp, _i32, _i32, _i32, _i32, _i32, _ip, _ip, _ip, _dp]
+        lib.orc_tsg_gate.restype = _i32
+        lib.orc_tsg_gate.argtypes = [_dp, _i32, _i32, _ip, _ip, _ip, _i32, _i32, _dp, _bp]
+        lib.orc_combine.restype = None
+        lib.orc_combine.argtypes = [_dp, _dp, _bp, _i32, _i32, _ip, _ip, _ip, ctypes.c_double, _i32, _dp]
+        lib.orc_topk.restype = None
+        lib.orc_topk.argtypes = [_dp, _i32, _i32, _ip]
+        lib.orc_gather.restype = None
+        lib.orc_gather.argtypes = [_bp, _bp, _i32, _i32, _i32, _i32, _ip, _i32, _bp, _bp]
+        _lib = lib
+    return _lib
+
+
+def _d(a):
+    return a.ctypes.data_as(_dp)
+
+
+def _c64(a):
+    return np.ascontiguousarray(a, dtype=np.float64)
+
+
+def _frames(frames):
+    off, gh, gw = (np.ascontiguousarray(x, dtype=np.int32) for x in frames)
+    assert off.shape == gh.shape == gw.shape
+    return off, gh, gw
+
+
+def _per_head(fn, hkv, threads):
+    if threads and threads > 1 and hkv > 1:
+        with ThreadPoolExecutor(max_workers=min(threads, hkv)) as ex:
+            list(ex.map(fn, range(hkv)))
+    else:
+        for h in range(hkv):
+            fn(h)
+
+
+def budget(n: int, beta: float, k_override: int = 0) -> int:
+    """B = floor(beta * N) (Sec. 2.1), >= 1; k_override > 0 replaces it."""
+    return int(_load().orc_budget(int(n), float(beta), int(k_override)))
+
+
+def abase(q, k, threads: int = 1) -> np.ndarray:
+    """Eq. 2 window score per KV head (mean over the G query heads of a group)."""
+    lib = _load()
+    q, k = _c64(q), _c64(k)
+    w, hq, d = q.shape
+    n, hkv, d2 = k.shape
+    assert d == d2 and hq % hkv == 0
+    out = np.zeros((hkv, n), dtype=np.float64)
+
+    def run(h):
+        lib.orc_abase(_d(q), _d(k), n, w, hq, hkv, d, h, out[h].ctypes.data_as(_dp))
+
+    _per_head(run, hkv, threads)
+    return out
+
+
+def css_phi(k, frames, threads: int = 1) -> np.ndarray:
+    """Eqs. 4-5: Phi = 1 - mean Moore-neighbour cosine; NaN for text tokens."""
+    lib = _load()
+    k = _c64(k)
+    n, hkv, d = k.shape
+    off, gh, gw = _frames(frames)
+    out = np.zeros((hkv, n), dtype=np.float64)
+
+    def run(h):
+        lib.orc_css_phi(_d(k), n, hkv, d, h, len(off), off.ctypes.data_as(_ip),
+                        gh.ctypes.data_as(_ip), gw.ctypes.data_as(_ip), out[h].ctypes.data_as(_dp))
+
+    _per_head(run, hkv, threads)
+    return out
+
+
+def css_phi_token(k, h: int, off: int, gh: int, gw: int, u: int, v: int) -> float:
+    """Phi of the single visual token (u, v) of the frame at ``off``."""
+    k = _c64(k)
+    n, hkv, d = k.shape
+    return float(_load().orc_css_phi_token(_d(k), hkv, d, h, off, gh, gw, u, v))
+
+
+def tsg_rho(k, frames, threads: int = 1) -> np.ndarray:
+    """Eq. 6: rho_i = max cosine to the current frame; NaN outside the pool."""
+    lib = _load()
+    k = _c64(k)
+    n, hkv, d = k.shape
+    off, gh, gw = _frames(frames)
+    out = np.zeros((hkv, n), dtype=np.float64)
+
+    def run(h):
+        lib.orc_tsg_rho(_d(k), n, hkv, d, h, len(off), off.ctypes.data_as(_ip),
+                        gh.ctypes.data_as(_ip), gw.ctypes.data_as(_ip), out[h].ctypes.data_as(_dp))
+
+    _per_head(run, hkv, threads)
+    return out
+
+
+def tsg_rho_token(k, h: int, i: int, frames) -> float:
+    """rho of the single token i against the current (last) frame."""
+    k = _c64(k)
+    n, hkv, d = k.shape
+    off, gh, gw = _frames(frames)
+    return float(_load().orc_tsg_rho_token(_d(k), hkv, d, h, i, int(off[-1]), int(gh[-1] * gw[-1])))
+
+
+def tsg_gate(rho, frames, budget_b: int, tsg_enable: int = 1):
+    """Eqs. 7-8: tau = min(B,|pool|)-th smallest rho; M = [rho <= tau].
+
+    Returns (tau [Hkv], gate [Hkv, N] uint8, pool_size)."""
+    lib = _load()
+    rho = _c64(rho)
+    hkv, n = rho.shape
+    off, gh, gw = _frames(frames)
+    tau = np.zeros(hkv, dtype=np.float64)
+    gate = np.zeros((hkv, n), dtype=np.uint8)
+    pool = 0
+    for h in range(hkv):
+        t = ctypes.c_double()
+        pool = lib.orc_tsg_gate(rho[h].ctypes.data_as(_dp), n, len(off), off.ctypes.data_as(_ip),
+                                gh.ctypes.data_as(_ip), gw.ctypes.data_as(_ip), int(budget_b),
+                                int(tsg_enable), ctypes.byref(t), gate[h].ctypes.data_as(_bp))
+        tau[h] = t.value
+    return tau, gate, int(pool)
+
+
+def combine(a, phi, gate, frames, alpha: float = 1.0, css_enable: int = 1) -> np.ndarray:
+    """Eq. 9: S = A (text); S = M * (A + alpha * Phi) (visual)."""
+    lib = _load()
+    a, phi = _c64(a), _c64(phi)
+    gate = np.ascontiguousarray(gate, dtype=np.uint8)
+    hkv, n = a.shape
+    off, gh, gw = _frames(frames)
+    out = np.zeros((hkv, n), dtype=np.float64)
+    for h in range(hkv):
+        lib.orc_combine(a[h].ctypes.data_as(_dp), phi[h].ctypes.data_as(_dp), gate[h].ctypes.data_as(_bp),
+                        n, len(off), off.ctypes.data_as(_ip), gh.ctypes.data_as(_ip),
+                        gw.ctypes.data_as(_ip), float(alpha), int(css_enable), out[h].ctypes.data_as(_dp))
+    return out
+
+
+def topk(s, budget_b: int) -> np.ndarray:
+    """Top-B by (S desc, index asc), returned in ascending index order: [Hkv, B]."""
+    lib = _load()
+    s = _c64(s)
+    hkv, n = s.shape
+    b = min(int(budget_b), n)
+    out = np.zeros((hkv, b), dtype=np.int32)
+    for h in range(hkv):
+        lib.orc_topk(s[h].ctypes.data_as(_dp), n, int(budget_b), out[h].ctypes.data_as(_ip))
+    return out
+
+
+def gather(k, v, idx):
+    """K'[r,h,:] = K[idx[h,r],h,:] (and V), byte-exact for any element type."""
+    lib = _load()
+    k = np.ascontiguousarray(k)
+    v = np.ascontiguousarray(v)
+    assert k.shape == v.shape and k.dtype == v.dtype
+    n, hkv, d = k.shape
+    idx = np.ascontiguousarray(idx, dtype=np.int32)
+    b = idx.shape[1]
+    ko = np.zeros((b, hkv, d), dtype=k.dtype)
+    vo = np.zeros((b, hkv, d), dtype=v.dtype)
+    kb, vb = k.view(np.uint8), v.view(np.uint8)
+    for h in range(hkv):
+        lib.orc_gather(kb.ctypes.data_as(_bp), vb.ctypes.data_as(_bp), hkv, d, k.itemsize, h,
+                       idx[h].ctypes.data_as(_ip), b, ko.view(np.uint8).ctypes.data_as(_bp),
+                       vo.view(np.uint8).ctypes.data_as(_bp))
+    return ko, vo
+
+
+def compress_layer(q, k, frames, beta: float = 0.2, k_override: int = 0, alpha: float = 1.0,
+                   tsg_enable: int = 1, css_enable: int = 1, threads: int = 1) -> dict:
+    """Algorithm 1 for one layer: every stage in the paper's order."""
+    n = k.shape[0]
+    b = budget(n, beta, k_override)
+    a = abase(q, k, threads)
+    phi = css_phi(k, frames, threads)
+    if tsg_enable:
+        rho = tsg_rho(k, frames, threads)
+    else:
+        rho = np.full_like(a, np.nan)
+    tau, gate, pool = tsg_gate(rho, frames, b, tsg_enable)
+    s = combine(a, phi, gate, frames, alpha, css_enable)
+    idx = topk(s, b)
+    return dict(budget=b, a=a, phi=phi, rho=rho, tau=tau, gate=gate, pool=pool, s=s, idx=idx)

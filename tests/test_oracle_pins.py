@@ -1,0 +1,437 @@
+"""Pins for the CPU oracle: closed forms, invariants, hand-derived fixtures and
+brute force on tiny inputs (none of them re-types the oracle's own formula).
+
+Each test names the paper passage it pins: Eq. 2 (window score), Eqs. 4-5
+(CSS), Eqs. 6-8 (TSG), Eq. 9 (integrated score), Sec. 2.1 (budget, top-B) and
+Algorithm 1 (whole procedure).
+"""
+import itertools
+import math
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2603_00188_gb300 import synth
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def frames_of(*spans):
+    """spans: (offset, gh, gw) per frame."""
+    off = np.array([s[0] for s in spans], np.int32)
+    gh = np.array([s[1] for s in spans], np.int32)
+    gw = np.array([s[2] for s in spans], np.int32)
+    return off, gh, gw
+
+
+# ------------------------------------------------------------------ budget
+
+@pytest.mark.parametrize("n,beta,expect", [
+    (1152, 0.2, 230), (23680, 0.1, 2368), (23680, 0.2, 4736), (23680, 0.3, 7104),
+    (23680, 0.4, 9472), (53600, 0.2, 10720), (132800, 0.1, 13280), (10, 1.0, 10),
+    (10, 0.01, 1), (7, 0.5, 3),
+])
+def test_budget_floor(n, beta, expect):
+    # Sec. 2.1: B = floor(beta * L); integer values worked by hand.
+    assert oracle.budget(n, beta) == expect
+
+
+def test_budget_override():
+    assert oracle.budget(1152, 0.2, 231) == 231    # ceil(0.2 * 1152) via override
+    assert oracle.budget(10, 0.2, 50) == 10
+
+
+# ------------------------------------------------------- window score, Eq. 2
+
+def test_abase_closed_form_single_head():
+    # w = 1, G = 1, q = e_0 and k_j = sqrt(d) * x_j * e_0, so q.k_j / sqrt(d) = x_j
+    # and A_j = exp(x_j) / sum exp(x).  Catches a missing or wrong 1/sqrt(d).
+    d, n = 16, 7
+    x = np.array([0.3, -1.2, 2.0, 0.0, 0.7, -0.4, 1.1])
+    q = np.zeros((1, 1, d)); q[0, 0, 0] = 1.0
+    k = np.zeros((n, 1, d)); k[:, 0, 0] = math.sqrt(d) * x
+    a = oracle.abase(q, k)
+    z = sum(math.exp(t) for t in x)
+    np.testing.assert_allclose(a[0], [math.exp(t) / z for t in x], rtol=1e-13)
+
+
+def test_abase_equal_keys_uniform():
+    # All keys identical: every softmax row is uniform, so A_j = w / N.
+    rng = np.random.default_rng(1)
+    w, hq, hkv, d, n = 5, 6, 2, 8, 11
+    q = rng.standard_normal((w, hq, d))
+    k = np.repeat(rng.standard_normal((1, hkv, d)), n, axis=0)
+    a = oracle.abase(q, k)
+    np.testing.assert_allclose(a, np.full((hkv, n), w / n), rtol=1e-12)
+
+
+def test_abase_sums_to_window():
+    # Each softmax row sums to 1; w rows summed, G heads averaged -> sum_j A = w.
+    rng = np.random.default_rng(2)
+    w, hq, hkv, d, n = 4, 6, 3, 16, 40
+    a = oracle.abase(rng.standard_normal((w, hq, d)) * 2, rng.standard_normal((n, hkv, d)))
+    np.testing.assert_allclose(a.sum(axis=1), np.full(hkv, w), rtol=1e-12)
+    assert (a > 0).all()
+
+
+def test_abase_gqa_grouping():
+    # Query head g belongs to KV head g // G: perturbing query head 2 (G=2)
+    # moves A of KV head 1 only.
+    rng = np.random.default_rng(3)
+    w, hq, hkv, d, n = 3, 4, 2, 8, 9
+    q = rng.standard_normal((w, hq, d)); k = rng.standard_normal((n, hkv, d))
+    a0 = oracle.abase(q, k)
+    q2 = q.copy(); q2[:, 2] += rng.standard_normal((w, d))
+    a1 = oracle.abase(q2, k)
+    np.testing.assert_array_equal(a0[0], a1[0])
+    assert np.abs(a0[1] - a1[1]).max() > 1e-3
+
+
+def test_abase_gqa_mean_closed_form():
+    # G = 2 query heads with logits x (head 0) and y (head 1), w = 1:
+    # A = (softmax(x) + softmax(y)) / 2, built from hand-chosen logits.
+    d = 4
+    x = np.array([0.5, -0.5, 1.5]); y = np.array([2.0, 0.0, -1.0])
+    q = np.zeros((1, 2, d)); q[0, 0, 0] = 1.0; q[0, 1, 1] = 1.0
+    k = np.zeros((3, 1, d)); k[:, 0, 0] = 2 * x; k[:, 0, 1] = 2 * y   # sqrt(4) = 2
+    sx = np.exp(x) / np.exp(x).sum(); sy = np.exp(y) / np.exp(y).sum()
+    np.testing.assert_allclose(oracle.abase(q, k)[0], (sx + sy) / 2, rtol=1e-13)
+
+
+def test_abase_library_softmax():
+    # Special case that reduces to a library routine: torch.softmax in float64.
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(4)
+    w, hq, hkv, d, n = 6, 4, 1, 32, 50
+    q = rng.standard_normal((w, hq, d)); k = rng.standard_normal((n, hkv, d)) * 1.5
+    logits = torch.einsum("rgd,nd->rgn", torch.from_numpy(q), torch.from_numpy(k[:, 0])) / math.sqrt(d)
+    ref = torch.softmax(logits, dim=-1).sum(dim=0).mean(dim=0).numpy()
+    np.testing.assert_allclose(oracle.abase(q, k)[0], ref, rtol=1e-12)
+
+
+# ------------------------------------------------------------- CSS, Eqs. 4-5
+
+def _read_fixture(name):
+    rows = []
+    with open(os.path.join(GOLDEN, name)) as f:
+        for line in f:
+            line = line.split("#")[0].strip()
+            if line:
+                rows.append(line)
+    return rows
+
+
+def _closed(expr):
+    return float(eval(expr, {"sqrt": math.sqrt, "__builtins__": {}}))
+
+
+def test_css_handworked_fixture():
+    rows = _read_fixture("css_handworked_2x3.txt")
+    k = np.zeros((6, 1, 2)); expect = np.zeros(6)
+    for r in rows:
+        parts = r.split()
+        u, v = int(parts[1]), int(parts[2])
+        k[u * 3 + v, 0] = [float(parts[3]), float(parts[4])]
+        expect[u * 3 + v] = _closed(" ".join(parts[5:]))
+    phi = oracle.css_phi(k, frames_of((0, 2, 3)))
+    np.testing.assert_allclose(phi[0], expect, rtol=0, atol=1e-14)
+
+
+def test_css_checkerboard_fixture():
+    rows = _read_fixture("css_checkerboard_3x4.txt")
+    expect = np.array([[_closed(t) for t in r.split()] for r in rows])
+    gh, gw, d = 3, 4, 5
+    k = np.zeros((gh * gw, 1, d))
+    for u in range(gh):
+        for v in range(gw):
+            k[u * gw + v, 0, 0] = (-1) ** (u + v)
+    phi = oracle.css_phi(k, frames_of((0, gh, gw)))
+    np.testing.assert_allclose(phi[0].reshape(gh, gw), expect, atol=1e-14)
+
+
+def test_css_equal_keys_zero():
+    rng = np.random.default_rng(5)
+    k = np.repeat(rng.standard_normal((1, 2, 16)), 30, axis=0)
+    phi = oracle.css_phi(k, frames_of((0, 5, 6)))
+    np.testing.assert_allclose(phi, 0.0, atol=1e-14)
+
+
+def test_css_orthonormal_one():
+    # Distinct basis vectors: every cosine 0 -> Phi = 1 everywhere.
+    gh, gw = 4, 5
+    k = np.eye(gh * gw)[:, None, :] * np.arange(1, gh * gw + 1)[:, None, None]  # magnitudes differ
+    phi = oracle.css_phi(k, frames_of((0, gh, gw)))
+    np.testing.assert_allclose(phi[0], 1.0, atol=1e-15)
+
+
+def test_css_planted_rectangle_closed_form():
+    # Identical keys r on a 2x3 rectangle, distinct basis vectors elsewhere:
+    # rectangle cell Phi = 1 - (#rectangle neighbours)/|N|, background Phi = 1.
+    gh, gw, d = 6, 7, 64
+    k = np.eye(d)[: gh * gw][:, None, :].copy()
+    r = np.zeros(d); r[-1] = 2.5
+    rect = [(u, v) for u in range(2, 4) for v in range(3, 6)]
+    for (u, v) in rect:
+        k[u * gw + v, 0] = r
+    phi = oracle.css_phi(k, frames_of((0, gh, gw)))[0].reshape(gh, gw)
+    for u in range(gh):
+        for v in range(gw):
+            nb = [(u + a, v + b) for a in (-1, 0, 1) for b in (-1, 0, 1)
+                  if (a or b) and 0 <= u + a < gh and 0 <= v + b < gw]
+            if (u, v) in rect:
+                expect = 1 - sum((p in rect) for p in nb) / len(nb)
+            else:
+                expect = 1.0
+            assert abs(phi[u, v] - expect) < 1e-14, (u, v)
+
+
+def test_css_edge_cases_and_frame_isolation():
+    rng = np.random.default_rng(6)
+    # 1x1 grid: no neighbour -> Phi = 0; text tokens -> NaN.
+    k = rng.standard_normal((10, 1, 8))
+    fr = frames_of((0, 1, 1), (3, 2, 2))
+    phi = oracle.css_phi(k, fr)[0]
+    assert phi[0] == 0.0
+    assert np.isnan(phi[[1, 2, 7, 8, 9]]).all()
+    # 1xW grid: each cell sees only its left/right neighbours.
+    k2 = np.zeros((3, 1, 2)); k2[:, 0] = [[1, 0], [1, 1], [0, 1]]
+    p2 = oracle.css_phi(k2, frames_of((0, 1, 3)))[0]
+    s = 1 / math.sqrt(2)
+    np.testing.assert_allclose(p2, [1 - s, 1 - s, 1 - s], atol=1e-15)
+    # frames do not see each other: changing frame 1 leaves frame 0 alone
+    k3 = k.copy(); k3[3:7] = rng.standard_normal((4, 1, 8))
+    np.testing.assert_array_equal(oracle.css_phi(k3, fr)[0][:3], phi[:3])
+
+
+def test_css_magnitude_invariance():
+    rng = np.random.default_rng(7)
+    k = rng.standard_normal((24, 2, 16))
+    fr = frames_of((0, 4, 6))
+    scale = rng.uniform(0.1, 10, size=(24, 2, 1))
+    np.testing.assert_allclose(oracle.css_phi(k * scale, fr), oracle.css_phi(k, fr), atol=1e-13)
+
+
+def test_css_zero_vector():
+    # Reading: norms clamp at 1e-8, so a zero key has cosine 0 with every neighbour.
+    k = np.ones((4, 1, 3)); k[0] = 0.0
+    phi = oracle.css_phi(k, frames_of((0, 2, 2)))[0]
+    assert phi[0] == 1.0
+    np.testing.assert_allclose(phi[1:], 1 - 2 / 3, atol=1e-15)
+
+
+# ------------------------------------------------------------- TSG, Eqs. 6-8
+
+def test_rho_angles_closed_form():
+    # 2-D keys at angles; rho_i = max_j cos(theta_i - phi_j) by trigonometry.
+    rng = np.random.default_rng(8)
+    th = rng.uniform(-math.pi, math.pi, 6)     # historical frame, 2x3
+    ph = rng.uniform(-math.pi, math.pi, 4)     # current frame, 2x2
+    mags = rng.uniform(0.5, 3, 10)
+    ang = np.concatenate([th, ph])
+    k = np.stack([np.cos(ang), np.sin(ang)], -1)[:, None, :] * mags[:, None, None]
+    fr = frames_of((0, 2, 3), (6, 2, 2))
+    rho = oracle.tsg_rho(k, fr)[0]
+    expect = [max(math.cos(t - p) for p in ph) for t in th]
+    np.testing.assert_allclose(rho[:6], expect, atol=1e-14)
+    assert np.isnan(rho[6:]).all()
+
+
+def test_rho_duplicate_and_orthogonal():
+    rng = np.random.default_rng(9)
+    d = 32
+    cur = rng.standard_normal((4, 1, d))
+    ortho = np.eye(d)[8:12][:, None, :]           # orthogonal to the current frame below
+    cur_o = np.eye(d)[:4][:, None, :] * 3
+    # frame 0 = copy of current (rho = 1); frame 1 orthogonal (rho = 0)
+    k = np.concatenate([cur, np.zeros((1, 1, d)), cur, np.zeros((1, 1, d))])
+    fr = frames_of((0, 2, 2), (5, 2, 2))
+    np.testing.assert_allclose(oracle.tsg_rho(k, fr)[0][:4], 1.0, atol=1e-14)
+    k2 = np.concatenate([ortho, cur_o])
+    fr2 = frames_of((0, 2, 2), (4, 2, 2))
+    np.testing.assert_allclose(oracle.tsg_rho(k2, fr2)[0][:4], 0.0, atol=1e-15)
+
+
+def test_rho_single_frame_and_scale():
+    rng = np.random.default_rng(10)
+    k = rng.standard_normal((20, 2, 8))
+    assert np.isnan(oracle.tsg_rho(k, frames_of((2, 3, 3)))).all()   # F = 1: empty pool
+    fr = frames_of((0, 2, 3), (6, 1, 4), (12, 2, 2))
+    r1 = oracle.tsg_rho(k, fr)
+    r2 = oracle.tsg_rho(k * 7.5, fr)
+    np.testing.assert_allclose(r1, r2, atol=1e-14)
+    # pool = frames 0 and 1 only; text and current frame are NaN
+    pool = np.zeros(20, bool); pool[0:6] = True; pool[6:10] = True
+    assert np.isfinite(r1[:, pool]).all() and np.isnan(r1[:, ~pool]).all()
+
+
+def test_tau_rank_property():
+    # tau is the min(B, |pool|)-th smallest pool value:
+    # #{rho < tau} < m <= #{rho <= tau}; gate = [rho <= tau] on the pool only.
+    rng = np.random.default_rng(11)
+    fr = frames_of((0, 3, 4), (14, 2, 5), (30, 2, 2))
+    n = 36
+    rho = np.full((2, n), np.nan)
+    pool = np.r_[0:12, 14:24]
+    rho[:, pool] = np.round(rng.uniform(0, 1, (2, pool.size)), 1)   # many ties
+    for b in (1, 5, 13, 22, 40):
+        tau, gate, psz = oracle.tsg_gate(rho, fr, b)
+        assert psz == 22
+        m = min(b, 22)
+        for h in range(2):
+            vals = rho[h, pool]
+            assert (vals < tau[h]).sum() < m <= (vals <= tau[h]).sum()
+            assert tau[h] in vals
+            expect = np.ones(n, np.uint8); expect[pool] = vals <= tau[h]
+            np.testing.assert_array_equal(gate[h], expect)
+        if b >= 22:
+            assert (gate == 1).all()   # B >= |pool| admits the whole pool
+
+
+def test_gate_disabled_or_empty_pool():
+    rho = np.random.default_rng(12).uniform(size=(1, 10))
+    tau, gate, _ = oracle.tsg_gate(rho, frames_of((0, 2, 2), (5, 1, 2)), 1, tsg_enable=0)
+    assert np.isnan(tau).all() and (gate == 1).all()
+    tau, gate, psz = oracle.tsg_gate(np.full((1, 10), np.nan), frames_of((2, 2, 2)), 3)
+    assert psz == 0 and np.isnan(tau).all() and (gate == 1).all()
+
+
+# ------------------------------------------------------- integrated score, Eq. 9
+
+def test_combine_cases():
+    fr = frames_of((0, 1, 3), (4, 1, 2))      # tokens 3, 6, 7 are text
+    a = np.array([[0.1, 0.2, 0.3, 0.4, 0.5, 0.6, 0.7, 0.8]])
+    phi = np.array([[1.0, 0.5, 0.25, np.nan, 2.0, 0.0, np.nan, np.nan]])
+    gate = np.array([[1, 0, 1, 1, 1, 1, 1, 1]], np.uint8)
+    s = oracle.combine(a, phi, gate, fr, alpha=1.0)
+    np.testing.assert_allclose(s[0], [1.1, 0.0, 0.55, 0.4, 2.5, 0.6, 0.7, 0.8], atol=1e-15)
+    s2 = oracle.combine(a, phi, gate, fr, alpha=0.5)
+    np.testing.assert_allclose(s2[0], [0.6, 0.0, 0.425, 0.4, 1.5, 0.6, 0.7, 0.8], atol=1e-15)
+    s3 = oracle.combine(a, phi, gate, fr, alpha=1.0, css_enable=0)
+    np.testing.assert_allclose(s3[0], [0.1, 0.0, 0.3, 0.4, 0.5, 0.6, 0.7, 0.8], atol=1e-15)
+
+
+# ----------------------------------------------------------- top-B, Sec. 2.1
+
+def _dominates(s, keep):
+    """The kept set of size B: every kept token outranks every dropped one,
+    where i outranks j iff s_i > s_j or (s_i == s_j and i < j)."""
+    drop = [j for j in range(len(s)) if j not in keep]
+    return all((s[i] > s[j]) or (s[i] == s[j] and i < j) for i in keep for j in drop)
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_topk_brute_force(seed):
+    rng = np.random.default_rng(100 + seed)
+    n = 8
+    s = rng.integers(0, 4, size=(1, n)).astype(np.float64) / 2      # heavy ties
+    for b in range(1, n + 1):
+        got = oracle.topk(s, b)[0]
+        valid = [c for c in itertools.combinations(range(n), b) if _dominates(s[0], set(c))]
+        assert len(valid) == 1
+        np.testing.assert_array_equal(got, valid[0])
+
+
+def test_topk_invariants_large():
+    rng = np.random.default_rng(13)
+    s = rng.standard_normal((3, 5000)); s[:, ::7] = 0.25          # planted ties
+    idx = oracle.topk(s, 1234)
+    for h in range(3):
+        row = idx[h]
+        assert len(row) == 1234 and (np.diff(row) > 0).all() and row.min() >= 0 and row.max() < 5000
+        thr = np.sort(s[h])[::-1][1233]
+        assert (s[h, row] >= thr).all()
+        assert (s[h][np.setdiff1d(np.arange(5000), row)] <= thr).all()
+
+
+# --------------------------------------------------------------------- gather
+
+def test_gather_bytes():
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(14)
+    k = torch.from_numpy(rng.standard_normal((50, 3, 128)).astype(np.float32)).to(torch.bfloat16)
+    v = torch.from_numpy(rng.standard_normal((50, 3, 128)).astype(np.float32)).to(torch.bfloat16)
+    kk, vv = k.view(torch.int16).numpy(), v.view(torch.int16).numpy()
+    idx = np.sort(np.stack([rng.choice(50, 17, replace=False) for _ in range(3)]), axis=1).astype(np.int32)
+    ko, vo = oracle.gather(kk, vv, idx)
+    for h in range(3):
+        np.testing.assert_array_equal(ko[:, h], kk[idx[h], h])
+        np.testing.assert_array_equal(vo[:, h], vv[idx[h], h])
+
+
+# ------------------------------------------------------- Algorithm 1, end to end
+
+def _tiny_traj(seed=0, n_steps=4, gh=4, gw=5, nt=3, hq=4, hkv=2, d=16, w=3):
+    return synth.trajectory(n_steps=n_steps, gh=gh, gw=gw, n_text=nt, hq=hq, hkv=hkv, d=d, w=w,
+                            n_boxes=(1, 2), box_hw=((1, 1), (2, 2)), seed=(900, seed))
+
+
+def test_end_to_end_beta_one_keeps_all():
+    wl = _tiny_traj()
+    out = oracle.compress_layer(wl.q, wl.k, wl.frames, beta=1.0)
+    assert out["budget"] == wl.n
+    np.testing.assert_array_equal(out["idx"], np.tile(np.arange(wl.n), (2, 1)))
+
+
+def test_end_to_end_single_frame_tsg_noop():
+    # One frame: TSG has an empty pool and must not change anything (CSS only).
+    wl = _tiny_traj(n_steps=1)
+    a = oracle.compress_layer(wl.q, wl.k, wl.frames, beta=0.3, tsg_enable=1)
+    b = oracle.compress_layer(wl.q, wl.k, wl.frames, beta=0.3, tsg_enable=0)
+    np.testing.assert_array_equal(a["idx"], b["idx"])
+    assert (a["gate"] == 1).all()
+
+
+def test_end_to_end_snapkv_base():
+    # alpha = 0 and TSG off: the retained set is top-B of A_base (library argsort).
+    wl = _tiny_traj(seed=3)
+    out = oracle.compress_layer(wl.q, wl.k, wl.frames, beta=0.25, tsg_enable=0, css_enable=0)
+    for h in range(2):
+        order = np.lexsort((np.arange(wl.n), -out["a"][h]))   # S desc, index asc
+        np.testing.assert_array_equal(out["idx"][h], np.sort(order[: out["budget"]]))
+
+
+def test_end_to_end_exact_budget_and_gate_invariants():
+    wl = _tiny_traj(seed=4, n_steps=5)
+    out = oracle.compress_layer(wl.q, wl.k, wl.frames, beta=0.2)
+    b = out["budget"]
+    off, gh, gw = wl.frames
+    cur = np.arange(off[-1], off[-1] + gh[-1] * gw[-1])
+    for h in range(2):
+        assert len(np.unique(out["idx"][h])) == b
+        assert (out["gate"][h][cur] == 1).all()
+        assert out["gate"][h].sum() - (wl.n - out["pool"]) >= min(b, out["pool"])
+
+
+def test_tiny_ref_duplicate_frame_gated():
+    # Frame 3 (current) = frame 2 + N(0, 0.01^2): frame 2's rho is ~1 and the
+    # m = 230 lowest-rho pool tokens come from frames 0-1, so TSG gates all of frame 2.
+    wl = synth.tiny_ref()
+    b = oracle.budget(wl.n, 0.2)
+    rho = oracle.tsg_rho(wl.k, wl.frames, threads=4)
+    tau, gate, pool = oracle.tsg_gate(rho, wl.frames, b)
+    assert pool == 768 and b == 230
+    f2 = np.arange(2 * 288, 2 * 288 + 256)
+    assert (rho[:, f2] > 0.99).all()
+    assert (gate[:, f2] == 0).all()
+    assert (tau < 0.6).all()
+
+
+def test_salient_rectangle_kept():
+    # CSS purpose (Sec. 3.1): on a uniform background a small element with
+    # different keys has Phi ~ 1 on its cells and ring, ~0 elsewhere, so at a
+    # budget just above the element+ring size all element cells are kept.
+    rng = np.random.default_rng(15)
+    gh, gw, d, hq, hkv, w = 8, 8, 32, 2, 1, 2
+    base = rng.standard_normal(d)
+    k = np.tile(base, (gh * gw, 1)) + 1e-3 * rng.standard_normal((gh * gw, d))
+    elem = [(3, 3), (3, 4)]
+    other = rng.standard_normal(d)
+    for (u, v) in elem:
+        k[u * gw + v] = other
+    k = k[:, None, :]
+    q = rng.standard_normal((w, hq, d)) * 0.1
+    out = oracle.compress_layer(q, k, frames_of((0, gh, gw)), beta=0.25)   # B = 16
+    kept = set(out["idx"][0].tolist())
+    assert all(u * gw + v in kept for (u, v) in elem)
