@@ -1,0 +1,190 @@
+/*
+ * stlite.h -- C ABI of libstlite.so, the GB300 (sm_103a) implementation of the
+ * ST-Lite per-layer KV-cache compression pass (arXiv 2603.00188, Algorithm 1).
+ *
+ * One call compresses one layer of one sequence (or, for the _varlen entry,
+ * one layer of a packed batch).  The pass has five steps:
+ *   1. window scoring       A_base, Sec. 2.1 Eq. (2)
+ *   2. TSG redundancy gate  rho, tau, M_time, Sec. 3.2 Eqs. (6)-(8)
+ *   3. CSS saliency         Phi, Sec. 3.1 Eqs. (4)-(5)
+ *   4. flat budget + top-B  S, I_keep, Sec. 2.1 and Sec. 3.3 Eq. (9)
+ *   5. compaction           K' = K[I_keep], V' = V[I_keep] (Algorithm 1)
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * Tensors.  Every tensor argument is a DEVICE pointer owned by the caller,
+ *   16-byte aligned, densely packed in the layout given beside it:
+ *     q      [w][Hq][d]        window queries (the last w query positions)
+ *     k, v   [N][Hkv][d]       one layer's cached keys / values
+ *     per-head outputs [Hkv][N] (float32 or uint8), idx [Hkv][B] (int32)
+ *     k_out, v_out [B][Hkv][d] compacted cache
+ *   Element type of q/k/v/k_out/v_out is shape->dtype (bf16 or fp32).
+ *   Query head g serves KV head g / (Hq/Hkv) (grouped-query attention).
+ * Frames.  stlite_frames holds HOST arrays.  Frame f owns the contiguous
+ *   visual span [offset[f], offset[f] + grid_h[f]*grid_w[f]) laid out
+ *   row-major on its patch grid (u = row, v = column); frames are sorted,
+ *   disjoint, inside [0, N), at most STLITE_MAX_FRAMES.  The LAST frame is the
+ *   current frame; every token outside a frame is a text token.
+ * Workspace.  ws is caller-allocated device memory of at least the size that
+ *   stlite_workspace_size() reports for the same shape/frames/params.  It
+ *   must be zero-filled before its first use (its first word is a device
+ *   error word, see stlite_device_status).  Calls on one stream may share a
+ *   workspace; concurrent calls on different streams need their own.
+ * Streams.  `stream` is a cudaStream_t passed as void* (NULL = legacy
+ *   default stream).  Every call only enqueues work: it returns after the
+ *   launches, without synchronising; outputs are valid once the stream has
+ *   reached that point.  No call allocates device memory.
+ * Errors.  All arguments are validated on the host before anything is
+ *   enqueued; a failed check returns STLITE_EINVAL / STLITE_EUNSUPPORTED /
+ *   STLITE_EWORKSPACE and enqueues nothing.  A launch failure returns
+ *   STLITE_ECUDA.  Kernels never trap: a bounded wait that runs out records
+ *   STLITE_ETIMEOUT in the workspace error word, read by stlite_device_status.
+ *   No call aborts the process; every call is thread-safe.
+ * Numbers.  bf16 inputs are multiplied exactly and accumulated in fp32
+ *   (tensor cores); fp32 inputs use fp32 FMA.  Softmax and cosines are fp32.
+ */
+#ifndef STLITE_H_
+#define STLITE_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#if defined(__GNUC__)
+#define STLITE_API __attribute__((visibility("default")))
+#else
+#define STLITE_API
+#endif
+
+#define STLITE_MAX_FRAMES 256
+#define STLITE_HEAD_DIM 128
+
+typedef enum {
+  STLITE_OK = 0,
+  STLITE_EINVAL = 1,       /* malformed argument (null, negative, overlapping frames, ...) */
+  STLITE_EUNSUPPORTED = 2, /* well-formed but outside what this build handles (d != 128, ...) */
+  STLITE_EWORKSPACE = 3,   /* workspace smaller than stlite_workspace_size() */
+  STLITE_ECUDA = 4,        /* a CUDA runtime call or kernel launch failed */
+  STLITE_ETIMEOUT = 5      /* a kernel's bounded wait ran out (device error word) */
+} stlite_status;
+
+typedef enum { STLITE_BF16 = 0, STLITE_F32 = 1 } stlite_dtype;
+
+typedef struct {
+  int32_t n_tokens;   /* N: cached tokens of the layer, >= 1 */
+  int32_t n_q_heads;  /* Hq: query heads, a multiple of n_kv_heads */
+  int32_t n_kv_heads; /* Hkv: key/value heads */
+  int32_t head_dim;   /* d: must be STLITE_HEAD_DIM */
+  int32_t window;     /* w: observation-window queries (delta of Eq. 2), 1..256 */
+  int32_t dtype;      /* stlite_dtype of q, k, v, k_out, v_out */
+} stlite_shape;
+
+typedef struct {
+  int32_t n_frames;       /* F >= 0; frame F-1 is the current frame */
+  const int32_t* offset;  /* host [F]: first token of each frame's visual span */
+  const int32_t* grid_h;  /* host [F]: patch-grid rows (>= 1) */
+  const int32_t* grid_w;  /* host [F]: patch-grid columns (>= 1) */
+} stlite_frames;
+
+typedef struct {
+  double beta;        /* compression ratio in (0, 1]: B = floor(beta * N) (Sec. 2.1) */
+  int32_t k_override; /* > 0: use this B instead (clamped to N); 0: use beta */
+  float alpha;        /* CSS weight of Eq. (9), >= 0 (paper default 1) */
+  int32_t tsg_enable; /* 1: apply the TSG gate of Eq. (8); 0: M_time = 1 everywhere */
+  int32_t css_enable; /* 1: add alpha * Phi (Eq. 9); 0: as alpha = 0 */
+} stlite_params;
+
+/* Flat per-layer budget (Sec. 2.1, Algorithm 1 initialisation):
+ * k_override > 0 ? min(k_override, N) : clamp(floor(beta * N + 1e-9), 1, N).
+ * Returns -1 if N < 1 or beta is not in (0, 1] (when k_override <= 0). */
+STLITE_API int32_t stlite_budget(int32_t n_tokens, double beta, int32_t k_override);
+
+/* Bytes of workspace every call below needs for this problem. */
+STLITE_API stlite_status stlite_workspace_size(const stlite_shape* shape, const stlite_frames* frames,
+                                    const stlite_params* params, size_t* bytes);
+
+/* Step 1, Eq. (2): a_base[h][j] = (1/G) sum_{g in group h} sum_{r<w}
+ * softmax_j(q[r][g] . k[j][h] / sqrt(d)), all N keys, no mask.
+ * a_base: device float [Hkv][N]. */
+STLITE_API stlite_status stlite_score(const stlite_shape* shape, const void* q, const void* k, float* a_base,
+                           void* ws, size_t ws_bytes, void* stream);
+
+/* Step 2, Eqs. (6)-(8): for every historical visual token i (frames 0..F-2)
+ * rho[h][i] = max over current-frame tokens j of cos(k_i, k_j), cos = a.b /
+ * (max(|a|,1e-8) max(|b|,1e-8)); tau[h] = the min(budget, |pool|)-th smallest
+ * rho; gate[h][i] = rho <= tau.  Outside the pool rho is NaN and gate is 1.
+ * With F < 2 (empty pool) tau is NaN and every gate is 1.
+ * rho: device float [Hkv][N]; tau: device float [Hkv]; gate: device uint8
+ * [Hkv][N]; budget >= 1. */
+STLITE_API stlite_status stlite_gate_frames(const stlite_shape* shape, const stlite_frames* frames,
+                                 const void* k, int32_t budget, float* rho, float* tau,
+                                 uint8_t* gate, void* ws, size_t ws_bytes, void* stream);
+
+/* Step 3, Eqs. (4)-(5): for every visual token, Phi = 1 - mean cosine to its
+ * in-grid 3x3 Moore neighbours in the same frame (0 when it has none); text
+ * tokens get NaN.  phi: device float [Hkv][N]. */
+STLITE_API stlite_status stlite_spatial_saliency(const stlite_shape* shape, const stlite_frames* frames,
+                                      const void* k, float* phi, void* ws, size_t ws_bytes,
+                                      void* stream);
+
+/* Step 4, Eq. (9) and Top_B: S = a_base for text tokens, S = gate * (a_base +
+ * alpha * phi) for visual tokens (phi ignored when css_enable = 0; gate may be
+ * NULL = all ones); idx[h][:] = the budget tokens of largest S, equal S ranked
+ * by lower index, written in ascending index order.  score_out (nullable):
+ * device float [Hkv][N] receives S. */
+STLITE_API stlite_status stlite_select_topk(const stlite_shape* shape, const stlite_frames* frames,
+                                 const stlite_params* params, const float* a_base,
+                                 const float* phi, const uint8_t* gate, int32_t budget,
+                                 int32_t* idx, float* score_out, void* ws, size_t ws_bytes,
+                                 void* stream);
+
+/* Step 5: k_out[r][h][:] = k[idx[h][r]][h][:] and the same for v, bit-exact.
+ * idx: device int32 [Hkv][budget].  The kernel checks every index: a row whose
+ * index lies outside [0, N) is left unwritten. */
+STLITE_API stlite_status stlite_compact(const stlite_shape* shape, int32_t budget, const int32_t* idx,
+                             const void* k, const void* v, void* k_out, void* v_out,
+                             void* stream);
+
+/* Steps 1-5 fused for one layer (Algorithm 1).  idx_out: device int32
+ * [Hkv][B] receives I_keep per head in ascending order; budget_out (nullable,
+ * HOST) receives B; k_out/v_out: device [B][Hkv][d].  Runs norms, TSG (when
+ * tsg_enable and F >= 2), window scoring, CSS (when css_enable), selection
+ * and compaction, all on `stream`. */
+STLITE_API stlite_status stlite_compress_layer(const stlite_shape* shape, const stlite_frames* frames,
+                                    const stlite_params* params, const void* q, const void* k,
+                                    const void* v, void* k_out, void* v_out, int32_t* idx_out,
+                                    int32_t* budget_out, void* ws, size_t ws_bytes, void* stream);
+
+/* Reads and clears the workspace's device error word (synchronises `stream`).
+ * *status receives STLITE_OK or the first error a kernel recorded since the
+ * last read (STLITE_ETIMEOUT). */
+STLITE_API stlite_status stlite_device_status(void* ws, void* stream, stlite_status* status);
+
+/* Per-kernel timing (instrumentation; not part of Algorithm 1).
+ * stlite_timing_enable(1) makes every later launch by this library, on a
+ * stream that is not being captured into a graph, record a pair of CUDA
+ * events around itself on its stream.  stlite_timing_read() waits for the
+ * recorded events, writes one entry per kernel name (number of launches and
+ * summed device time in ms) into `out` (up to `capacity` entries; *count
+ * receives the number of distinct kernels) and clears the record.  Both are
+ * process-wide and thread-safe. */
+typedef struct {
+  char name[32];
+  int32_t launches;
+  double total_ms;
+} stlite_kernel_time;
+STLITE_API stlite_status stlite_timing_enable(int32_t on);
+STLITE_API stlite_status stlite_timing_read(stlite_kernel_time* out, int32_t capacity,
+                                            int32_t* count);
+
+/* Human-readable name of a status code (static storage). */
+STLITE_API const char* stlite_status_string(stlite_status status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* STLITE_H_ */

@@ -1,0 +1,449 @@
+// C ABI of libstlite.so: argument validation, workspace planning and the
+// launch sequence of each entry point.  Declarations and the contract of
+// every call are in include/stlite.h.
+#include <math.h>
+#include <string.h>
+
+#include <atomic>
+#include <map>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "../../include/stlite.h"
+#include "kernels.cuh"
+
+using namespace stl;
+
+namespace {
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+stlite_status check_shape(const stlite_shape* s) {
+  if (!s) return STLITE_EINVAL;
+  if (s->n_tokens < 1 || s->n_q_heads < 1 || s->n_kv_heads < 1 || s->window < 1 ||
+      s->head_dim < 1)
+    return STLITE_EINVAL;
+  if (s->n_q_heads % s->n_kv_heads != 0) return STLITE_EINVAL;
+  if (s->dtype != STLITE_BF16 && s->dtype != STLITE_F32) return STLITE_EINVAL;
+  if (s->head_dim != STLITE_HEAD_DIM) return STLITE_EUNSUPPORTED;
+  if (s->window > 256) return STLITE_EUNSUPPORTED;
+  const long long R = (long long)s->window * (s->n_q_heads / s->n_kv_heads);
+  if (R > 512) return STLITE_EUNSUPPORTED;
+  if ((long long)s->n_tokens * s->n_kv_heads > (1LL << 30)) return STLITE_EUNSUPPORTED;
+  return STLITE_OK;
+}
+
+stlite_status build_frames(const stlite_shape* s, const stlite_frames* fr, FrameTable* ft) {
+  memset(ft, 0, sizeof(*ft));
+  ft->n_tokens = s->n_tokens;
+  if (!fr) return STLITE_EINVAL;
+  const int F = fr->n_frames;
+  if (F < 0) return STLITE_EINVAL;
+  if (F > STLITE_MAX_FRAMES) return STLITE_EUNSUPPORTED;
+  if (F > 0 && (!fr->offset || !fr->grid_h || !fr->grid_w)) return STLITE_EINVAL;
+  long long prev_end = 0;
+  for (int f = 0; f < F; ++f) {
+    const long long off = fr->offset[f], gh = fr->grid_h[f], gw = fr->grid_w[f];
+    if (off < 0 || gh < 1 || gw < 1) return STLITE_EINVAL;
+    if (off < prev_end) return STLITE_EINVAL;  // sorted and disjoint
+    if (off + gh * gw > s->n_tokens) return STLITE_EINVAL;
+    prev_end = off + gh * gw;
+    ft->off[f] = (int32_t)off;
+    ft->gh[f] = (int32_t)gh;
+    ft->gw[f] = (int32_t)gw;
+  }
+  ft->n_frames = F;
+  ft->tile0[0] = 0;
+  for (int f = 0; f + 1 < F; ++f)
+    ft->tile0[f + 1] = ft->tile0[f] + (ft->gh[f] * ft->gw[f] + kTsgTile - 1) / kTsgTile;
+  if (F > 0) {
+    ft->cur_off = ft->off[F - 1];
+    ft->cur_len = ft->gh[F - 1] * ft->gw[F - 1];
+  }
+  return STLITE_OK;
+}
+
+stlite_status check_params(const stlite_params* pr) {
+  if (!pr) return STLITE_EINVAL;
+  if (pr->k_override < 0) return STLITE_EINVAL;
+  if (pr->k_override == 0 && !(pr->beta > 0.0 && pr->beta <= 1.0)) return STLITE_EINVAL;
+  if (!(pr->alpha >= 0.f) || !isfinite(pr->alpha)) return STLITE_EINVAL;
+  return STLITE_OK;
+}
+
+Problem to_problem(const stlite_shape* s) {
+  Problem p;
+  p.n = s->n_tokens;
+  p.hq = s->n_q_heads;
+  p.hkv = s->n_kv_heads;
+  p.w = s->window;
+  p.dtype = s->dtype == STLITE_BF16 ? kBF16 : kF32;
+  return p;
+}
+
+bool use_tensor_cores(const Problem& p) { return p.dtype == kBF16; }
+
+stlite_status cuda_status(cudaError_t e) { return e == cudaSuccess ? STLITE_OK : STLITE_ECUDA; }
+
+}  // namespace
+
+namespace stl {
+
+// Workspace regions, each 256-byte aligned.
+WsPlan plan_workspace(const Problem& p, const FrameTable& ft) {
+  WsPlan w;
+  const size_t hn = (size_t)p.hkv * p.n;
+  if (use_tensor_cores(p)) {
+    w.nsplit = umma_score_nsplit(p);
+    w.nchunk = ft.n_frames >= 2 ? (ft.cur_len + 255) / 256 : 1;  // 256-column slices
+  } else {
+    int per_head = (304 + p.hkv - 1) / p.hkv;
+    int max_split = (p.n + 63) / 64;
+    w.nsplit = per_head < max_split ? per_head : max_split;
+    w.nchunk = 1;
+  }
+  if (w.nchunk < 1) w.nchunk = 1;
+  size_t o = 0;
+  auto take = [&](size_t bytes) {
+    size_t at = o;
+    o = align_up(o + bytes, 256);
+    return at;
+  };
+  w.err = take(4);
+  w.rn = take(hn * 4);
+  w.rowpart = take((size_t)p.hkv * w.nsplit * p.R() * 8 + (size_t)p.hkv * p.R() * 4);
+  w.a_base = take(hn * 4);
+  w.phi = take(hn * 4);
+  w.rho = take(hn * 4);
+  w.rho_part = take((size_t)w.nchunk * hn * 4);
+  w.tau = take((size_t)p.hkv * 4);
+  w.gate = take(hn);
+  w.score = take(hn * 4);
+  w.total = o;
+  return w;
+}
+
+// ---- per-kernel timing ----------------------------------------------------
+namespace {
+struct TimingRecord {
+  const char* name;
+  cudaEvent_t start, stop;
+};
+std::atomic<int> g_timing_on{0};
+std::mutex g_timing_mu;
+std::vector<TimingRecord> g_records;
+std::vector<cudaEvent_t> g_event_pool;
+
+cudaEvent_t take_event() {
+  {
+    std::lock_guard<std::mutex> lk(g_timing_mu);
+    if (!g_event_pool.empty()) {
+      cudaEvent_t e = g_event_pool.back();
+      g_event_pool.pop_back();
+      return e;
+    }
+  }
+  cudaEvent_t e = nullptr;
+  if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+  return e;
+}
+
+bool stream_capturing(cudaStream_t st) {
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  return cudaStreamIsCapturing(st, &cs) == cudaSuccess && cs != cudaStreamCaptureStatusNone;
+}
+}  // namespace
+
+TimingScope::TimingScope(const char* name, cudaStream_t st) : name_(name), st_(st), start_(nullptr) {
+  if (!g_timing_on.load(std::memory_order_relaxed) || stream_capturing(st)) return;
+  start_ = take_event();
+  if (start_ && cudaEventRecord(start_, st_) != cudaSuccess) start_ = nullptr;
+}
+
+TimingScope::~TimingScope() {
+  if (!start_) return;
+  cudaEvent_t stop = take_event();
+  if (!stop || cudaEventRecord(stop, st_) != cudaSuccess) return;
+  std::lock_guard<std::mutex> lk(g_timing_mu);
+  g_records.push_back({name_, start_, stop});
+}
+
+}  // namespace stl
+
+namespace {
+
+struct Ctx {
+  Problem p;
+  FrameTable ft;
+  WsPlan plan;
+  uint8_t* ws;
+  uint32_t* err;
+  cudaStream_t st;
+  template <typename T>
+  T* at(size_t off) const {
+    return reinterpret_cast<T*>(ws + off);
+  }
+};
+
+stlite_status prepare(const stlite_shape* shape, const stlite_frames* frames, void* ws,
+                      size_t ws_bytes, void* stream, Ctx* c) {
+  stlite_status s = check_shape(shape);
+  if (s != STLITE_OK) return s;
+  stlite_frames none = {0, nullptr, nullptr, nullptr};
+  if ((s = build_frames(shape, frames ? frames : &none, &c->ft)) != STLITE_OK) return s;
+  c->p = to_problem(shape);
+  c->plan = plan_workspace(c->p, c->ft);
+  if (!ws || !aligned16(ws)) return STLITE_EINVAL;
+  if (ws_bytes < c->plan.total) return STLITE_EWORKSPACE;
+  c->ws = static_cast<uint8_t*>(ws);
+  c->err = c->at<uint32_t>(c->plan.err);
+  c->st = static_cast<cudaStream_t>(stream);
+  return STLITE_OK;
+}
+
+cudaError_t run_norms(const Ctx& c, const void* k) {
+  return launch_inv_norms(c.p, k, c.at<float>(c.plan.rn), c.st);
+}
+
+cudaError_t run_score(const Ctx& c, const void* q, const void* k, float* a_base) {
+  float2* rp = c.at<float2>(c.plan.rowpart);
+  if (use_tensor_cores(c.p)) return launch_score_umma(c.p, q, k, rp, c.plan.nsplit, a_base, c.err, c.st);
+  return launch_score(c.p, q, k, rp, c.plan.nsplit, a_base, c.err, c.st);
+}
+
+cudaError_t run_tsg(const Ctx& c, const void* k) {
+  float* rp = c.at<float>(c.plan.rho_part);
+  const float* rn = c.at<float>(c.plan.rn);
+  if (use_tensor_cores(c.p))
+    return launch_tsg_umma(c.p, c.ft, k, rn, rp, umma_tsg_nchunk(c.ft), c.err, c.st);
+  return launch_tsg(c.p, c.ft, k, rn, rp, 1, c.err, c.st);
+}
+
+}  // namespace
+
+extern "C" {
+
+int32_t stlite_budget(int32_t n_tokens, double beta, int32_t k_override) {
+  if (n_tokens < 1) return -1;
+  if (k_override > 0) return k_override < n_tokens ? k_override : n_tokens;
+  if (!(beta > 0.0 && beta <= 1.0)) return -1;
+  long long b = (long long)floor(beta * (double)n_tokens + 1e-9);
+  if (b < 1) b = 1;
+  if (b > n_tokens) b = n_tokens;
+  return (int32_t)b;
+}
+
+stlite_status stlite_workspace_size(const stlite_shape* shape, const stlite_frames* frames,
+                                    const stlite_params* params, size_t* bytes) {
+  if (!bytes) return STLITE_EINVAL;
+  stlite_status s = check_shape(shape);
+  if (s != STLITE_OK) return s;
+  if (params && (s = check_params(params)) != STLITE_OK) return s;
+  stlite_frames none = {0, nullptr, nullptr, nullptr};
+  FrameTable ft;
+  if ((s = build_frames(shape, frames ? frames : &none, &ft)) != STLITE_OK) return s;
+  *bytes = plan_workspace(to_problem(shape), ft).total;
+  return STLITE_OK;
+}
+
+stlite_status stlite_score(const stlite_shape* shape, const void* q, const void* k, float* a_base,
+                           void* ws, size_t ws_bytes, void* stream) {
+  Ctx c;
+  stlite_status s = prepare(shape, nullptr, ws, ws_bytes, stream, &c);
+  if (s != STLITE_OK) return s;
+  if (!q || !k || !a_base || !aligned16(q) || !aligned16(k) || !aligned16(a_base)) return STLITE_EINVAL;
+  return cuda_status(run_score(c, q, k, a_base));
+}
+
+stlite_status stlite_gate_frames(const stlite_shape* shape, const stlite_frames* frames,
+                                 const void* k, int32_t budget, float* rho, float* tau,
+                                 uint8_t* gate, void* ws, size_t ws_bytes, void* stream) {
+  Ctx c;
+  stlite_status s = prepare(shape, frames, ws, ws_bytes, stream, &c);
+  if (s != STLITE_OK) return s;
+  if (!k || !rho || !tau || !gate || !aligned16(k) || !aligned16(rho) || !aligned16(tau) ||
+      !aligned16(gate))
+    return STLITE_EINVAL;
+  if (budget < 1 || budget > c.p.n) return STLITE_EINVAL;
+  cudaError_t e = run_norms(c, k);
+  if (e == cudaSuccess) e = run_tsg(c, k);
+  if (e != cudaSuccess) return STLITE_ECUDA;
+  SelectArgs a = {};
+  a.mode = kSelGate;
+  a.budget = budget;
+  a.nchunk = c.plan.nchunk;
+  a.tsg_enable = 1;
+  a.rho_part = c.at<float>(c.plan.rho_part);
+  a.rn = c.at<float>(c.plan.rn);
+  a.rho = rho;
+  a.tau = tau;
+  a.gate = gate;
+  return cuda_status(launch_select(c.p, c.ft, a, c.st));
+}
+
+stlite_status stlite_spatial_saliency(const stlite_shape* shape, const stlite_frames* frames,
+                                      const void* k, float* phi, void* ws, size_t ws_bytes,
+                                      void* stream) {
+  Ctx c;
+  stlite_status s = prepare(shape, frames, ws, ws_bytes, stream, &c);
+  if (s != STLITE_OK) return s;
+  if (!k || !phi || !aligned16(k) || !aligned16(phi)) return STLITE_EINVAL;
+  cudaError_t e = run_norms(c, k);
+  if (e == cudaSuccess) e = launch_css(c.p, c.ft, k, c.at<float>(c.plan.rn), phi, c.st);
+  return cuda_status(e);
+}
+
+stlite_status stlite_select_topk(const stlite_shape* shape, const stlite_frames* frames,
+                                 const stlite_params* params, const float* a_base,
+                                 const float* phi, const uint8_t* gate, int32_t budget,
+                                 int32_t* idx, float* score_out, void* ws, size_t ws_bytes,
+                                 void* stream) {
+  Ctx c;
+  stlite_status s = prepare(shape, frames, ws, ws_bytes, stream, &c);
+  if (s != STLITE_OK) return s;
+  if ((s = check_params(params)) != STLITE_OK) return s;
+  if (!a_base || !idx || !aligned16(a_base) || !aligned16(idx)) return STLITE_EINVAL;
+  if (params->css_enable && (!phi || !aligned16(phi))) return STLITE_EINVAL;
+  if ((gate && !aligned16(gate)) || (score_out && !aligned16(score_out))) return STLITE_EINVAL;
+  if (budget < 1 || budget > c.p.n) return STLITE_EINVAL;
+  SelectArgs a = {};
+  a.mode = kSelTopk;
+  a.budget = budget;
+  a.css_enable = params->css_enable ? 1 : 0;
+  a.alpha = params->alpha;
+  a.a_base = a_base;
+  a.phi = params->css_enable ? phi : nullptr;
+  a.gate = const_cast<uint8_t*>(gate);
+  a.score = score_out ? score_out : c.at<float>(c.plan.score);
+  a.idx = idx;
+  return cuda_status(launch_select(c.p, c.ft, a, c.st));
+}
+
+stlite_status stlite_compact(const stlite_shape* shape, int32_t budget, const int32_t* idx,
+                             const void* k, const void* v, void* k_out, void* v_out,
+                             void* stream) {
+  stlite_status s = check_shape(shape);
+  if (s != STLITE_OK) return s;
+  if (!idx || !k || !v || !k_out || !v_out) return STLITE_EINVAL;
+  if (!aligned16(idx) || !aligned16(k) || !aligned16(v) || !aligned16(k_out) || !aligned16(v_out))
+    return STLITE_EINVAL;
+  if (budget < 1 || budget > shape->n_tokens) return STLITE_EINVAL;
+  Problem p = to_problem(shape);
+  return cuda_status(
+      launch_gather(p, budget, idx, k, v, k_out, v_out, static_cast<cudaStream_t>(stream)));
+}
+
+stlite_status stlite_compress_layer(const stlite_shape* shape, const stlite_frames* frames,
+                                    const stlite_params* params, const void* q, const void* k,
+                                    const void* v, void* k_out, void* v_out, int32_t* idx_out,
+                                    int32_t* budget_out, void* ws, size_t ws_bytes,
+                                    void* stream) {
+  Ctx c;
+  stlite_status s = prepare(shape, frames, ws, ws_bytes, stream, &c);
+  if (s != STLITE_OK) return s;
+  if ((s = check_params(params)) != STLITE_OK) return s;
+  if (!q || !k || !v || !k_out || !v_out || !idx_out) return STLITE_EINVAL;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(k_out) || !aligned16(v_out) ||
+      !aligned16(idx_out))
+    return STLITE_EINVAL;
+  const int32_t budget = stlite_budget(c.p.n, params->beta, params->k_override);
+  if (budget < 1) return STLITE_EINVAL;
+  if (budget_out) *budget_out = budget;
+  const bool tsg = params->tsg_enable && c.ft.n_frames >= 2;
+  float* a_base = c.at<float>(c.plan.a_base);
+  float* phi = c.at<float>(c.plan.phi);
+  cudaError_t e = run_norms(c, k);
+  if (e == cudaSuccess && tsg) e = run_tsg(c, k);
+  if (e == cudaSuccess) e = run_score(c, q, k, a_base);
+  if (e == cudaSuccess && params->css_enable) e = launch_css(c.p, c.ft, k, c.at<float>(c.plan.rn), phi, c.st);
+  if (e != cudaSuccess) return STLITE_ECUDA;
+  SelectArgs a = {};
+  a.mode = (tsg ? kSelGate : 0) | kSelTopk;
+  a.budget = budget;
+  a.nchunk = c.plan.nchunk;
+  a.tsg_enable = tsg ? 1 : 0;
+  a.css_enable = params->css_enable ? 1 : 0;
+  a.alpha = params->alpha;
+  a.rho_part = c.at<float>(c.plan.rho_part);
+  a.rn = c.at<float>(c.plan.rn);
+  a.rho = c.at<float>(c.plan.rho);
+  a.tau = c.at<float>(c.plan.tau);
+  a.gate = tsg ? c.at<uint8_t>(c.plan.gate) : nullptr;
+  a.a_base = a_base;
+  a.phi = params->css_enable ? phi : nullptr;
+  a.score = c.at<float>(c.plan.score);
+  a.idx = idx_out;
+  if ((e = launch_select(c.p, c.ft, a, c.st)) != cudaSuccess) return STLITE_ECUDA;
+  return cuda_status(launch_gather(c.p, budget, idx_out, k, v, k_out, v_out, c.st));
+}
+
+stlite_status stlite_device_status(void* ws, void* stream, stlite_status* status) {
+  if (!ws || !status || !aligned16(ws)) return STLITE_EINVAL;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  uint32_t word = 0;
+  if (cudaMemcpyAsync(&word, ws, 4, cudaMemcpyDeviceToHost, st) != cudaSuccess) return STLITE_ECUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return STLITE_ECUDA;
+  if (cudaMemsetAsync(ws, 0, 4, st) != cudaSuccess) return STLITE_ECUDA;
+  *status = (word & kErrTimeout) ? STLITE_ETIMEOUT : STLITE_OK;
+  return STLITE_OK;
+}
+
+stlite_status stlite_timing_enable(int32_t on) {
+  g_timing_on.store(on ? 1 : 0);
+  return STLITE_OK;
+}
+
+stlite_status stlite_timing_read(stlite_kernel_time* out, int32_t capacity, int32_t* count) {
+  if (!count || capacity < 0 || (capacity > 0 && !out)) return STLITE_EINVAL;
+  std::vector<TimingRecord> recs;
+  {
+    std::lock_guard<std::mutex> lk(g_timing_mu);
+    recs.swap(g_records);
+  }
+  std::map<std::string, std::pair<int, double>> agg;
+  bool ok = true;
+  for (auto& r : recs) {
+    float ms = 0.f;
+    if (cudaEventSynchronize(r.stop) != cudaSuccess || cudaEventElapsedTime(&ms, r.start, r.stop) != cudaSuccess)
+      ok = false;
+    auto& a = agg[r.name];
+    a.first += 1;
+    a.second += ms;
+  }
+  {
+    std::lock_guard<std::mutex> lk(g_timing_mu);
+    for (auto& r : recs) {
+      g_event_pool.push_back(r.start);
+      g_event_pool.push_back(r.stop);
+    }
+  }
+  int i = 0;
+  for (auto& kv : agg) {
+    if (i < capacity) {
+      memset(out[i].name, 0, sizeof(out[i].name));
+      strncpy(out[i].name, kv.first.c_str(), sizeof(out[i].name) - 1);
+      out[i].launches = kv.second.first;
+      out[i].total_ms = kv.second.second;
+    }
+    ++i;
+  }
+  *count = i;
+  return ok ? STLITE_OK : STLITE_ECUDA;
+}
+
+const char* stlite_status_string(stlite_status status) {
+  switch (status) {
+    case STLITE_OK: return "ok";
+    case STLITE_EINVAL: return "invalid argument";
+    case STLITE_EUNSUPPORTED: return "unsupported shape or layout";
+    case STLITE_EWORKSPACE: return "workspace too small";
+    case STLITE_ECUDA: return "CUDA launch or runtime error";
+    case STLITE_ETIMEOUT: return "a kernel wait timed out";
+  }
+  return "unknown status";
+}
+
+}  // extern "C"

@@ -1,0 +1,658 @@
+// Tensor-core (tcgen05 + TMA) kernels for bf16 caches:
+//   k_tsg_umma       TSG redundancy, Eq. 6: historical keys x current-frame
+//                    keys on the tensor cores, scale-and-row-max epilogue.
+//   k_rowstats_umma  window score pass 1 (Eq. 2): per query row running max
+//                    and sum of exponentials over a split of the keys.
+//   k_colsum_umma    window score pass 2: per key sum over query rows of the
+//                    softmax probabilities.
+//
+// All three share one structure: warp 0 issues TMA loads of 128-byte-swizzled
+// key tiles, warp 1 issues tcgen05.mma into TMEM (fp32 accumulators), warps
+// 2-9 (two groups of four, one warp per TMEM lane quarter) drain TMEM with
+// tcgen05.ld and run the fp32 epilogue.  Every mbarrier wait is bounded.
+#include <cudaTypedefs.h>
+
+#include "kernels.cuh"
+#include "ptx.cuh"
+
+namespace stl {
+
+constexpr int kThreads = 320;  // 10 warps
+constexpr float kLog2eF = 1.4426950408889634f;
+
+__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
+  uint32_t a = smem_u32(p);
+  return p + ((1024u - (a & 1023u)) & 1023u);
+}
+
+// Q rows of KV head h into shared memory in the K-major 128B-swizzle layout
+// [2 K-halves][rows][128 B]; row r = window row * G + group member; rows past
+// R are zero.
+__device__ __forceinline__ void load_q_sw128(uint8_t* sq, int rows, const __nv_bfloat16* q,
+                                             const Problem& p, int h) {
+  const int G = p.G(), R = p.R();
+  for (int e = threadIdx.x; e < rows * 16; e += blockDim.x) {
+    int row = e >> 4, c16 = e & 15, kb = c16 >> 3, cc = c16 & 7;
+    uint4 val = make_uint4(0, 0, 0, 0);
+    if (row < R) {
+      int wr = row / G, g = row - wr * G;
+      val = __ldg(reinterpret_cast<const uint4*>(q + ((size_t)wr * p.hq + h * G + g) * kD + c16 * 8));
+    }
+    *reinterpret_cast<uint4*>(sq + (size_t)kb * rows * 128 + row * 128 + ((cc ^ (row & 7)) << 4)) = val;
+  }
+  fence_proxy_async_smem();
+}
+
+// Lane 0 polls the barrier; the verdict is broadcast so that the whole warp
+// leaves converged (the tcgen05.ld that follows is .sync.aligned).
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, uint32_t* err,
+                                          volatile uint32_t* abort_flag) {
+  int ok = 1;
+  if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, err, abort_flag) ? 1 : 0;
+  return __shfl_sync(0xffffffffu, ok, 0) != 0;
+}
+
+// First token of TSG row tile t and the end of its frame's visual span.
+__device__ __forceinline__ void tsg_tile(const FrameTable& ft, int t, int& tok0, int& fend) {
+  int lo = 0, hi = ft.n_frames - 2, f = 0;
+  while (lo <= hi) {
+    int mid = (lo + hi) >> 1;
+    if (ft.tile0[mid] <= t) {
+      f = mid;
+      lo = mid + 1;
+    } else {
+      hi = mid - 1;
+    }
+  }
+  tok0 = ft.off[f] + (t - ft.tile0[f]) * kTsgTile;
+  fend = ft.off[f] + ft.gh[f] * ft.gw[f];
+}
+
+// =========================================================================
+// TSG.  CTA (x, chunk, h): current-frame columns [512*chunk, 512*chunk+512)
+// of head h stay in shared memory (128 KB); historical row tiles of 128
+// tokens stream through two 32 KB stages.  TMEM holds the 128 x 512 fp32
+// product as two 256-column accumulator stages; epilogue group g owns stage g
+// and writes slice 2*chunk+g of rho_part: max_j acc_ij * rn_j.  Columns past
+// the current frame carry rn = NaN, which fmaxf ignores.
+constexpr int kTsgB = 0;                  // [2][512][128 B]
+constexpr int kTsgA = 131072;             // [2 stages][2][128][128 B]
+constexpr int kTsgRn = 196608;            // float[512]
+constexpr int kTsgBar = 198656;           // 10 mbarriers + slot + abort
+constexpr int kTsgSmem = kTsgBar + 128 + 1024;
+
+__global__ void __launch_bounds__(kThreads, 1)
+    k_tsg_umma(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ FrameTable ft,
+               const float* __restrict__ rn, float* __restrict__ rho_part, int hkv,
+               uint32_t* err) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = align1024(smem_raw);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int chunk = blockIdx.y, h = blockIdx.z, n = ft.n_tokens;
+  const int n_tiles = ft.tile0[ft.n_frames - 1];
+  const int col0 = chunk * 512;
+  const int valid = min(512, ft.cur_len - col0);
+  const int nst = valid > 256 ? 2 : 1;
+  const uint32_t sB = smem_u32(sm + kTsgB), sA = smem_u32(sm + kTsgA);
+  float* rn_s = reinterpret_cast<float*>(sm + kTsgRn);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + kTsgBar);
+  const uint32_t b_afull = smem_u32(&bars[0]), b_aempty = smem_u32(&bars[2]);
+  const uint32_t b_bfull = smem_u32(&bars[4]), b_accfull = smem_u32(&bars[5]);
+  const uint32_t b_accempty = smem_u32(&bars[7]), b_done = smem_u32(&bars[9]);
+  uint32_t* slot = reinterpret_cast<uint32_t*>(sm + kTsgBar + 80);
+  volatile uint32_t* abort_flag = slot + 1;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(b_afull + 8 * i, 1);
+      mbar_init(b_aempty + 8 * i, 1);
+      mbar_init(b_accfull + 8 * i, 1);
+      mbar_init(b_accempty + 8 * i, 4);
+    }
+    mbar_init(b_bfull, 1);
+    mbar_init(b_done, 1);
+    *abort_flag = 0u;
+    fence_mbar_init();
+    tma_prefetch_desc(&kmap);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(slot), 512);
+    tmem_relinquish();
+  }
+  for (int c = (int)threadIdx.x - 64; c < 512; c += kThreads - 64)
+    if (c >= 0) rn_s[c] = c < valid ? rn[(size_t)h * n + ft.cur_off + col0 + c] : CUDART_NAN_F;
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      mbar_arrive_expect_tx(b_bfull, 131072);
+      for (int kb = 0; kb < 2; ++kb)
+        for (int rb = 0; rb < 4; ++rb)
+          tma_load_3d(sB + kb * 65536 + rb * 16384, &kmap, b_bfull, kb * 64, h,
+                      ft.cur_off + col0 + rb * 128);
+      int it = 0, issued[2] = {0, 0};
+      for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++it) {
+        const int s = it & 1;
+        const uint32_t u = (uint32_t)(it >> 1);
+        if (!mbar_wait(b_aempty + 8 * s, (u & 1u) ^ 1u, err, abort_flag)) break;
+        int tok0, fend;
+        tsg_tile(ft, t, tok0, fend);
+        mbar_arrive_expect_tx(b_afull + 8 * s, 32768);
+        tma_load_3d(sA + s * 32768, &kmap, b_afull + 8 * s, 0, h, tok0);
+        tma_load_3d(sA + s * 32768 + 16384, &kmap, b_afull + 8 * s, 64, h, tok0);
+        ++issued[s];
+      }
+      if (*abort_flag) {  // drain copies still in flight before the CTA exits
+        mbar_wait_drain(b_bfull, 0);
+        for (int s = 0; s < 2; ++s)
+          if (issued[s]) mbar_wait_drain(b_afull + 8 * s, (uint32_t)(issued[s] - 1) & 1u);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      bool ok = mbar_wait(b_bfull, 0, err, abort_flag);
+      int it = 0;
+      for (int t = blockIdx.x; ok && t < n_tiles; t += gridDim.x, ++it) {
+        const int s = it & 1;
+        const uint32_t u = (uint32_t)(it >> 1);
+        if (!mbar_wait(b_afull + 8 * s, u & 1u, err, abort_flag)) break;
+        tc_fence_after();
+        for (int g = 0; g < nst && ok; ++g) {
+          if (!mbar_wait(b_accempty + 8 * g, ((uint32_t)it & 1u) ^ 1u, err, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const int ncols = (min(256, valid - g * 256) + 15) & ~15;
+          const uint32_t idesc = idesc_bf16(128, ncols);
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const uint32_t kb = k >> 2, koff = (k & 3) * 32;
+            uint64_t ad = desc_sw128(sA + s * 32768 + kb * 16384 + koff);
+            uint64_t bd = desc_sw128(sB + kb * 65536 + g * 256 * 128 + koff);
+            umma_bf16(tmem + g * 256, ad, bd, idesc, k > 0 ? 1u : 0u);
+          }
+          umma_commit(b_accfull + 8 * g);
+        }
+        if (!ok) break;
+        umma_commit(b_aempty + 8 * s);
+      }
+      umma_commit(b_done);
+      mbar_wait_drain(b_done, 0);
+    }
+  } else {
+    const int g = (warp - 2) >> 2, quarter = warp & 3;
+    if (g < nst) {
+      const int valid_g = min(256, valid - g * 256);
+      const uint32_t tbase = tmem + ((uint32_t)(quarter * 32) << 16) + g * 256;
+      const float* rg = rn_s + g * 256;
+      int it = 0;
+      for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++it) {
+        if (!warp_wait(b_accfull + 8 * g, (uint32_t)it & 1u, err, abort_flag)) break;
+        tc_fence_after();
+        float mx = -CUDART_INF_F;
+        for (int c = 0; c < 8; ++c) {
+          if (c * 32 >= valid_g) break;
+          float v[32];
+          tmem_ld32(tbase + c * 32, v);
+          const float4* r4 = reinterpret_cast<const float4*>(rg + c * 32);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            float4 r = r4[i];
+            mx = fmaxf(mx, v[4 * i] * r.x);
+            mx = fmaxf(mx, v[4 * i + 1] * r.y);
+            mx = fmaxf(mx, v[4 * i + 2] * r.z);
+            mx = fmaxf(mx, v[4 * i + 3] * r.w);
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(b_accempty + 8 * g);
+        int tok0, fend;
+        tsg_tile(ft, t, tok0, fend);
+        const int tok = tok0 + quarter * 32 + lane;
+        if (tok < fend) rho_part[((size_t)(2 * chunk + g) * hkv + h) * n + tok] = mx;
+      }
+    }
+  }
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// =========================================================================
+// Window score pass 1.  CTA (split, h): Q of head h (R rows, MT M-tiles of
+// 128) stays in shared memory as the A operand; key tiles of KN = 256/MT
+// keys stream as the B operand.  TMEM: two stages of MT*KN <= 256 columns;
+// epilogue group g handles the key tiles with it % 2 == g and keeps, per
+// query row, the running max m (raw dot units) and l = sum 2^((x - m) c).
+// The two groups merge at the end; part[h][split][r] = (m c, l).
+constexpr int kRsStage = 2;
+
+struct RsLayout {
+  int MT, KN, q_bytes, k_stage_bytes, off_k, off_bar, off_xch, total;
+};
+__host__ __device__ inline RsLayout rs_layout(int R) {
+  RsLayout L;
+  L.MT = R <= 128 ? 1 : (R <= 256 ? 2 : 4);
+  L.KN = 256 / L.MT;
+  L.q_bytes = L.MT * 128 * 256;
+  L.k_stage_bytes = L.KN * 256;
+  L.off_k = L.q_bytes;
+  L.off_bar = L.off_k + kRsStage * L.k_stage_bytes;
+  L.off_xch = L.off_bar + 128;
+  L.total = L.off_xch + L.MT * 128 * 8 + 1024;
+  return L;
+}
+
+__device__ __forceinline__ void online_merge(float& m, float& l, float m2, float l2, float c) {
+  float mn = fmaxf(m, m2);
+  if (mn == -CUDART_INF_F) return;
+  float a = (m == -CUDART_INF_F) ? 0.f : l * exp2f((m - mn) * c);
+  float b = (m2 == -CUDART_INF_F) ? 0.f : l2 * exp2f((m2 - mn) * c);
+  m = mn;
+  l = a + b;
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    k_rowstats_umma(const __grid_constant__ CUtensorMap kmap, const __nv_bfloat16* __restrict__ q,
+                    Problem p, int nsplit, float2* __restrict__ part, uint32_t* err) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = align1024(smem_raw);
+  const RsLayout L = rs_layout(p.R());
+  const int MT = L.MT, KN = L.KN, R = p.R();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int split = blockIdx.x, h = blockIdx.y, n = p.n;
+  const int per = (((n + nsplit - 1) / nsplit) + KN - 1) / KN * KN;
+  const int j0 = split * per, j1 = min(n, j0 + per);
+  const int ntiles = j1 > j0 ? (j1 - j0 + KN - 1) / KN : 0;
+  const uint32_t sQ = smem_u32(sm), sK = smem_u32(sm + L.off_k);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + L.off_bar);
+  const uint32_t b_kfull = smem_u32(&bars[0]), b_kempty = smem_u32(&bars[2]);
+  const uint32_t b_accfull = smem_u32(&bars[4]), b_accempty = smem_u32(&bars[6]);
+  const uint32_t b_done = smem_u32(&bars[8]);
+  uint32_t* slot = reinterpret_cast<uint32_t*>(sm + L.off_bar + 80);
+  volatile uint32_t* abort_flag = slot + 1;
+  float2* xch = reinterpret_cast<float2*>(sm + L.off_xch);
+  const float c = kLog2eF * rsqrtf((float)kD);
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(b_kfull + 8 * i, 1);
+      mbar_init(b_kempty + 8 * i, 1);
+      mbar_init(b_accfull + 8 * i, 1);
+      mbar_init(b_accempty + 8 * i, 4);
+    }
+    mbar_init(b_done, 1);
+    *abort_flag = 0u;
+    fence_mbar_init();
+    tma_prefetch_desc(&kmap);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(slot), 512);
+    tmem_relinquish();
+  }
+  load_q_sw128(sm, MT * 128, q, p, h);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *slot;
+
+  // per-thread row state for up to 4 M-tiles (epilogue warps)
+  float m_st[4], l_st[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    m_st[i] = -CUDART_INF_F;
+    l_st[i] = 0.f;
+  }
+  const int g = warp >= 2 ? (warp - 2) >> 2 : 0, quarter = warp & 3;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int issued[2] = {0, 0};
+      for (int it = 0; it < ntiles; ++it) {
+        const int s = it & 1;
+        const uint32_t u = (uint32_t)(it >> 1);
+        if (!mbar_wait(b_kempty + 8 * s, (u & 1u) ^ 1u, err, abort_flag)) break;
+        const int tok = j0 + it * KN;
+        mbar_arrive_expect_tx(b_kfull + 8 * s, (uint32_t)L.k_stage_bytes);
+        tma_load_3d(sK + s * L.k_stage_bytes, &kmap, b_kfull + 8 * s, 0, h, tok);
+        tma_load_3d(sK + s * L.k_stage_bytes + KN * 128, &kmap, b_kfull + 8 * s, 64, h, tok);
+        ++issued[s];
+      }
+      if (*abort_flag)
+        for (int s = 0; s < 2; ++s)
+          if (issued[s]) mbar_wait_drain(b_kfull + 8 * s, (uint32_t)(issued[s] - 1) & 1u);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      const uint32_t idesc = idesc_bf16(128, KN);
+      for (int it = 0; it < ntiles; ++it) {
+        const int s = it & 1;
+        const uint32_t u = (uint32_t)(it >> 1);
+        if (!mbar_wait(b_kfull + 8 * s, u & 1u, err, abort_flag)) break;
+        if (!mbar_wait(b_accempty + 8 * s, (u & 1u) ^ 1u, err, abort_flag)) break;
+        tc_fence_after();
+        for (int mt = 0; mt < MT; ++mt) {
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const uint32_t kb = k >> 2, koff = (k & 3) * 32;
+            uint64_t ad = desc_sw128(sQ + kb * (MT * 128 * 128) + mt * 128 * 128 + koff);
+            uint64_t bd = desc_sw128(sK + s * L.k_stage_bytes + kb * (KN * 128) + koff);
+            umma_bf16(tmem + s * 256 + mt * KN, ad, bd, idesc, k > 0 ? 1u : 0u);
+          }
+        }
+        umma_commit(b_accfull + 8 * s);
+        umma_commit(b_kempty + 8 * s);
+      }
+      umma_commit(b_done);
+      mbar_wait_drain(b_done, 0);
+    }
+  } else {
+    const uint32_t lanebase = tmem + ((uint32_t)(quarter * 32) << 16);
+    for (int it = g; it < ntiles; it += 2) {
+      const uint32_t u = (uint32_t)(it >> 1);
+      if (!warp_wait(b_accfull + 8 * g, u & 1u, err, abort_flag)) break;
+      tc_fence_after();
+      const int tok = j0 + it * KN;
+      for (int mt = 0; mt < MT; ++mt) {
+        float m = m_st[mt], l = l_st[mt];
+        for (int cg = 0; cg < KN / 32; ++cg) {
+          const int kbase = tok + cg * 32;
+          if (kbase >= j1) break;
+          float v[32];
+          tmem_ld32(lanebase + g * 256 + mt * KN + cg * 32, v);
+          const int nv = min(32, j1 - kbase);
+          float mc = -CUDART_INF_F;
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (i < nv) mc = fmaxf(mc, v[i]);
+          const float mn = fmaxf(m, mc);
+          const float mnc = mn * c;
+          float sacc = 0.f;
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (i < nv) sacc += exp2f(fmaf(v[i], c, -mnc));
+          l = (m == -CUDART_INF_F ? 0.f : l * exp2f((m - mn) * c)) + sacc;
+          m = mn;
+        }
+        m_st[mt] = m;
+        l_st[mt] = l;
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(b_accempty + 8 * g);
+    }
+  }
+  // merge the two epilogue groups, then write (m * c, l) per query row
+  if (warp >= 2 && g == 1)
+    for (int mt = 0; mt < MT; ++mt) xch[mt * 128 + quarter * 32 + lane] = make_float2(m_st[mt], l_st[mt]);
+  tc_fence_before();
+  __syncthreads();
+  if (warp >= 2 && g == 0) {
+    for (int mt = 0; mt < MT; ++mt) {
+      const int row = mt * 128 + quarter * 32 + lane;
+      float2 o = xch[row];
+      float m = m_st[mt], l = l_st[mt];
+      online_merge(m, l, o.x, o.y, c);
+      if (row < R) part[((size_t)h * nsplit + split) * R + row] = make_float2(m * c, l);
+    }
+  }
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// =========================================================================
+// Window score pass 2.  CTA (x, h): key tiles of 128 tokens are the A operand
+// (M = 128, one key per TMEM lane), Q of head h (NQ = R rounded up to 32
+// rows) is the B operand.  Each thread sums 2^(x_r c + bias_r) over the R
+// query rows of its key.  TMEM: two stages of NQ columns when NQ <= 256
+// (epilogue group g takes the tiles with it % 2 == g), else one stage.
+struct CsLayout {
+  int NQ, nstage, tmem_cols, q_bytes, off_k, off_bias, off_bar, total;
+};
+__host__ __device__ inline CsLayout cs_layout(int R) {
+  CsLayout L;
+  L.NQ = (R + 31) & ~31;
+  L.nstage = L.NQ <= 256 ? 2 : 1;
+  L.tmem_cols = 32;
+  while (L.tmem_cols < L.nstage * L.NQ) L.tmem_cols <<= 1;
+  L.q_bytes = L.NQ * 256;
+  L.off_k = L.q_bytes;
+  L.off_bias = L.off_k + 2 * 32768;
+  L.off_bar = L.off_bias + L.NQ * 4;
+  L.total = L.off_bar + 128 + 1024;
+  return L;
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    k_colsum_umma(const __grid_constant__ CUtensorMap kmap, const __nv_bfloat16* __restrict__ q,
+                  Problem p, const float* __restrict__ bias, float* __restrict__ a_base,
+                  uint32_t* err) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = align1024(smem_raw);
+  const CsLayout L = cs_layout(p.R());
+  const int NQ = L.NQ, nstage = L.nstage, R = p.R(), n = p.n;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, h = blockIdx.y;
+  const int ntiles_all = (n + 127) / 128;
+  const uint32_t sQ = smem_u32(sm), sK = smem_u32(sm + L.off_k);
+  float* bias_s = reinterpret_cast<float*>(sm + L.off_bias);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + L.off_bar);
+  const uint32_t b_kfull = smem_u32(&bars[0]), b_kempty = smem_u32(&bars[2]);
+  const uint32_t b_accfull = smem_u32(&bars[4]), b_accempty = smem_u32(&bars[6]);
+  const uint32_t b_done = smem_u32(&bars[8]);
+  uint32_t* slot = reinterpret_cast<uint32_t*>(sm + L.off_bar + 80);
+  volatile uint32_t* abort_flag = slot + 1;
+  const float c = kLog2eF * rsqrtf((float)kD);
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(b_kfull + 8 * i, 1);
+      mbar_init(b_kempty + 8 * i, 1);
+      mbar_init(b_accfull + 8 * i, 1);
+      mbar_init(b_accempty + 8 * i, 4);
+    }
+    mbar_init(b_done, 1);
+    *abort_flag = 0u;
+    fence_mbar_init();
+    tma_prefetch_desc(&kmap);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(slot), (uint32_t)L.tmem_cols);
+    tmem_relinquish();
+  }
+  load_q_sw128(sm, NQ, q, p, h);
+  for (int r = threadIdx.x; r < NQ; r += blockDim.x)
+    bias_s[r] = r < R ? bias[(size_t)h * R + r] : -CUDART_INF_F;
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *slot;
+  int ntiles = 0;
+  for (int t = blockIdx.x; t < ntiles_all; t += gridDim.x) ++ntiles;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int issued[2] = {0, 0};
+      for (int it = 0; it < ntiles; ++it) {
+        const int s = it & 1;
+        const uint32_t u = (uint32_t)(it >> 1);
+        if (!mbar_wait(b_kempty + 8 * s, (u & 1u) ^ 1u, err, abort_flag)) break;
+        const int tok = (blockIdx.x + it * gridDim.x) * 128;
+        mbar_arrive_expect_tx(b_kfull + 8 * s, 32768);
+        tma_load_3d(sK + s * 32768, &kmap, b_kfull + 8 * s, 0, h, tok);
+        tma_load_3d(sK + s * 32768 + 16384, &kmap, b_kfull + 8 * s, 64, h, tok);
+        ++issued[s];
+      }
+      if (*abort_flag)
+        for (int s = 0; s < 2; ++s)
+          if (issued[s]) mbar_wait_drain(b_kfull + 8 * s, (uint32_t)(issued[s] - 1) & 1u);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      for (int it = 0; it < ntiles; ++it) {
+        const int s = it & 1, as = it % nstage;
+        const uint32_t u = (uint32_t)(it >> 1), ua = (uint32_t)(it / nstage);
+        if (!mbar_wait(b_kfull + 8 * s, u & 1u, err, abort_flag)) break;
+        if (!mbar_wait(b_accempty + 8 * as, (ua & 1u) ^ 1u, err, abort_flag)) break;
+        tc_fence_after();
+        for (int nb = 0; nb < NQ; nb += 256) {
+          const int nn = min(256, NQ - nb);
+          const uint32_t idesc = idesc_bf16(128, nn);
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const uint32_t kb = k >> 2, koff = (k & 3) * 32;
+            uint64_t ad = desc_sw128(sK + s * 32768 + kb * 16384 + koff);
+            uint64_t bd = desc_sw128(sQ + kb * (NQ * 128) + nb * 128 + koff);
+            umma_bf16(tmem + as * NQ + nb, ad, bd, idesc, k > 0 ? 1u : 0u);
+          }
+        }
+        umma_commit(b_accfull + 8 * as);
+        umma_commit(b_kempty + 8 * s);
+      }
+      umma_commit(b_done);
+      mbar_wait_drain(b_done, 0);
+    }
+  } else {
+    const int g = (warp - 2) >> 2, quarter = warp & 3;
+    if (g < nstage) {
+      const uint32_t tbase = tmem + ((uint32_t)(quarter * 32) << 16) + g * NQ;
+      for (int it = g; it < ntiles; it += nstage) {
+        const uint32_t ua = (uint32_t)(it / nstage);
+        if (!warp_wait(b_accfull + 8 * g, ua & 1u, err, abort_flag)) break;
+        tc_fence_after();
+        float acc = 0.f;
+        for (int cg = 0; cg < NQ / 32; ++cg) {
+          float v[32];
+          tmem_ld32(tbase + cg * 32, v);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const int r = cg * 32 + i;
+            if (r < R) acc += exp2f(fmaf(v[i], c, bias_s[r]));
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(b_accempty + 8 * g);
+        const int tok = (blockIdx.x + it * gridDim.x) * 128 + quarter * 32 + lane;
+        if (tok < n) a_base[(size_t)h * n + tok] = acc;
+      }
+    }
+  }
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, (uint32_t)L.tmem_cols);
+  }
+}
+
+// =========================================================================
+// host side
+
+static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult qr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &qr) == cudaSuccess &&
+        qr == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  }
+  return fn;
+}
+
+// K [N][Hkv][128] bf16 as a 3-D tensor (d, head, token); box = 64 x 1 x rows
+// with the 128-byte swizzle, out-of-range tokens read as zero.
+static cudaError_t make_kmap(CUtensorMap* m, const void* k, int n, int hkv, int rows) {
+  auto fn = encode_fn();
+  if (!fn) return cudaErrorNotSupported;
+  cuuint64_t dims[3] = {(cuuint64_t)kD, (cuuint64_t)hkv, (cuuint64_t)n};
+  cuuint64_t strides[2] = {(cuuint64_t)kD * 2, (cuuint64_t)hkv * kD * 2};
+  cuuint32_t box[3] = {64, 1, (cuuint32_t)rows};
+  cuuint32_t es[3] = {1, 1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(k), dims, strides, box,
+                  es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+static int sm_count() {
+  int dev = 0, c = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&c, cudaDevAttrMultiProcessorCount, dev);
+  return c > 0 ? c : 148;
+}
+
+int umma_tsg_nchunk(const FrameTable& ft) {
+  return ft.n_frames >= 2 ? (ft.cur_len + 511) / 512 : 0;
+}
+
+int umma_score_nsplit(const Problem& p) {
+  const RsLayout L = rs_layout(p.R());
+  int per_head = (148 + p.hkv - 1) / p.hkv;
+  int max_split = (p.n + L.KN - 1) / L.KN;
+  return per_head < max_split ? per_head : max_split;
+}
+
+cudaError_t launch_tsg_umma(const Problem& p, const FrameTable& ft, const void* k, const float* rn,
+                            float* rho_part, int nchunk, uint32_t* err, cudaStream_t st) {
+  if (ft.n_frames < 2) return cudaSuccess;
+  const int n_tiles = ft.tile0[ft.n_frames - 1];
+  if (n_tiles == 0 || ft.cur_len == 0) return cudaSuccess;
+  CUtensorMap map;
+  cudaError_t e = make_kmap(&map, k, p.n, p.hkv, 128);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(k_tsg_umma, cudaFuncAttributeMaxDynamicSharedMemorySize, kTsgSmem);
+  if (e != cudaSuccess) return e;
+  int groups = nchunk * p.hkv;
+  int gx = (sm_count() + groups - 1) / groups;
+  if (gx > n_tiles) gx = n_tiles;
+  if (gx < 1) gx = 1;
+  dim3 grid(gx, nchunk, p.hkv);
+  TimingScope ts("tsg_umma", st);
+  k_tsg_umma<<<grid, kThreads, kTsgSmem, st>>>(map, ft, rn, rho_part, p.hkv, err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_score_umma(const Problem& p, const void* q, const void* k, float2* rowpart,
+                              int nsplit, float* a_base, uint32_t* err, cudaStream_t st) {
+  const int R = p.R();
+  if (R > 512) return cudaErrorNotSupported;
+  const RsLayout L1 = rs_layout(R);
+  const CsLayout L2 = cs_layout(R);
+  CUtensorMap m1, m2;
+  cudaError_t e = make_kmap(&m1, k, p.n, p.hkv, L1.KN);
+  if (e != cudaSuccess) return e;
+  if ((e = make_kmap(&m2, k, p.n, p.hkv, 128)) != cudaSuccess) return e;
+  if ((e = cudaFuncSetAttribute(k_rowstats_umma, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                L1.total)) != cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(k_colsum_umma, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                L2.total)) != cudaSuccess)
+    return e;
+  float* bias = reinterpret_cast<float*>(rowpart + (size_t)p.hkv * nsplit * R);
+  {
+    TimingScope ts("rowstats_umma", st);
+    k_rowstats_umma<<<dim3(nsplit, p.hkv), kThreads, L1.total, st>>>(
+        m1, (const __nv_bfloat16*)q, p, nsplit, rowpart, err);
+  }
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  if ((e = launch_row_bias(p, rowpart, nsplit, bias, st)) != cudaSuccess) return e;
+  int tiles = (p.n + 127) / 128;
+  int gx = (sm_count() + p.hkv - 1) / p.hkv;
+  if (gx > tiles) gx = tiles;
+  TimingScope ts("colsum_umma", st);
+  k_colsum_umma<<<dim3(gx, p.hkv), kThreads, L2.total, st>>>(m2, (const __nv_bfloat16*)q, p,
+                                                              bias, a_base, err);
+  return cudaGetLastError();
+}
+
+}  // namespace stl

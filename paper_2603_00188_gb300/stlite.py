@@ -1,0 +1,235 @@
+"""Python binding of libstlite.so (ctypes; argument marshalling only).
+
+Every function here has the name of the C entry point it calls (declared in
+``include/stlite.h``) and forwards torch CUDA tensors as raw device pointers
+on the current torch stream.  No computation happens in Python: if the
+library is not built this module raises at import time.
+
+    from paper_2603_00188_gb300 import stlite
+    k_out, v_out, idx = stlite.compress_layer(q, k, v, frames, beta=0.2)
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+import torch
+
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libstlite.so")
+if not os.path.exists(_LIB_PATH):
+    raise ImportError("libstlite.so is not built (run paper_2603_00188_gb300.build.build()): %s" % _LIB_PATH)
+_lib = ctypes.CDLL(_LIB_PATH)
+
+STLITE_OK, STLITE_EINVAL, STLITE_EUNSUPPORTED, STLITE_EWORKSPACE, STLITE_ECUDA, STLITE_ETIMEOUT = range(6)
+STLITE_BF16, STLITE_F32 = 0, 1
+MAX_FRAMES = 256
+EXPORTED = ("stlite_budget", "stlite_workspace_size", "stlite_score", "stlite_gate_frames",
+            "stlite_spatial_saliency", "stlite_select_topk", "stlite_compact",
+            "stlite_compress_layer", "stlite_device_status", "stlite_timing_enable", "stlite_timing_read",
+            "stlite_status_string")
+
+
+class Shape(ctypes.Structure):
+    _fields_ = [("n_tokens", ctypes.c_int32), ("n_q_heads", ctypes.c_int32),
+                ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("window", ctypes.c_int32), ("dtype", ctypes.c_int32)]
+
+
+class Frames(ctypes.Structure):
+    _fields_ = [("n_frames", ctypes.c_int32), ("offset", ctypes.POINTER(ctypes.c_int32)),
+                ("grid_h", ctypes.POINTER(ctypes.c_int32)), ("grid_w", ctypes.POINTER(ctypes.c_int32))]
+
+
+class Params(ctypes.Structure):
+    _fields_ = [("beta", ctypes.c_double), ("k_override", ctypes.c_int32), ("alpha", ctypes.c_float),
+                ("tsg_enable", ctypes.c_int32), ("css_enable", ctypes.c_int32)]
+
+
+class KernelTime(ctypes.Structure):
+    _fields_ = [("name", ctypes.c_char * 32), ("launches", ctypes.c_int32), ("total_ms", ctypes.c_double)]
+
+
+_P = ctypes.c_void_p
+_S = ctypes.c_int32
+_sig = {
+    "stlite_budget": (ctypes.c_int32, [ctypes.c_int32, ctypes.c_double, ctypes.c_int32]),
+    "stlite_workspace_size": (_S, [ctypes.POINTER(Shape), ctypes.POINTER(Frames), ctypes.POINTER(Params),
+                                   ctypes.POINTER(ctypes.c_size_t)]),
+    "stlite_score": (_S, [ctypes.POINTER(Shape), _P, _P, _P, _P, ctypes.c_size_t, _P]),
+    "stlite_gate_frames": (_S, [ctypes.POINTER(Shape), ctypes.POINTER(Frames), _P, ctypes.c_int32, _P, _P, _P,
+                                _P, ctypes.c_size_t, _P]),
+    "stlite_spatial_saliency": (_S, [ctypes.POINTER(Shape), ctypes.POINTER(Frames), _P, _P, _P,
+                                     ctypes.c_size_t, _P]),
+    "stlite_select_topk": (_S, [ctypes.POINTER(Shape), ctypes.POINTER(Frames), ctypes.POINTER(Params), _P, _P,
+                                _P, ctypes.c_int32, _P, _P, _P, ctypes.c_size_t, _P]),
+    "stlite_compact": (_S, [ctypes.POINTER(Shape), ctypes.c_int32, _P, _P, _P, _P, _P, _P]),
+    "stlite_compress_layer": (_S, [ctypes.POINTER(Shape), ctypes.POINTER(Frames), ctypes.POINTER(Params), _P,
+                                   _P, _P, _P, _P, _P, ctypes.POINTER(ctypes.c_int32), _P, ctypes.c_size_t, _P]),
+    "stlite_device_status": (_S, [_P, _P, ctypes.POINTER(ctypes.c_int32)]),
+    "stlite_timing_enable": (_S, [ctypes.c_int32]),
+    "stlite_timing_read": (_S, [ctypes.POINTER(KernelTime), ctypes.c_int32, ctypes.POINTER(ctypes.c_int32)]),
+    "stlite_status_string": (ctypes.c_char_p, [ctypes.c_int32]),
+}
+for _name, (_res, _args) in _sig.items():
+    _f = getattr(_lib, _name)
+    _f.restype = _res
+    _f.argtypes = _args
+
+
+class StliteError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__("%s: %s (%d)" % (where, _lib.stlite_status_string(status).decode(), status))
+
+
+def _check(status: int, where: str):
+    if status != STLITE_OK:
+        raise StliteError(status, where)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def make_shape(q, k) -> Shape:
+    w, hq, d = q.shape
+    n, hkv, d2 = k.shape
+    if d != d2:
+        raise ValueError("q and k head_dim differ")
+    dt = {torch.bfloat16: STLITE_BF16, torch.float32: STLITE_F32}[k.dtype]
+    return Shape(n, hq, hkv, d, w, dt)
+
+
+class FrameSpec:
+    """Host frame descriptor (offset, grid_h, grid_w), kept alive with its ctypes view."""
+
+    def __init__(self, offset, grid_h, grid_w):
+        self.offset = np.ascontiguousarray(offset, dtype=np.int32)
+        self.grid_h = np.ascontiguousarray(grid_h, dtype=np.int32)
+        self.grid_w = np.ascontiguousarray(grid_w, dtype=np.int32)
+        ip = ctypes.POINTER(ctypes.c_int32)
+        self.c = Frames(len(self.offset), self.offset.ctypes.data_as(ip), self.grid_h.ctypes.data_as(ip),
+                        self.grid_w.ctypes.data_as(ip))
+
+
+def _frames(frames) -> FrameSpec:
+    if isinstance(frames, FrameSpec):
+        return frames
+    return FrameSpec(*frames)
+
+
+def make_params(beta=0.2, k_override=0, alpha=1.0, tsg_enable=1, css_enable=1) -> Params:
+    return Params(float(beta), int(k_override), float(alpha), int(tsg_enable), int(css_enable))
+
+
+# ----------------------------------------------------------------- entries
+
+def stlite_budget(n_tokens: int, beta: float, k_override: int = 0) -> int:
+    return int(_lib.stlite_budget(int(n_tokens), float(beta), int(k_override)))
+
+
+def stlite_workspace_size(shape: Shape, frames, params: Params | None = None) -> int:
+    fs = _frames(frames)
+    out = ctypes.c_size_t()
+    _check(_lib.stlite_workspace_size(ctypes.byref(shape), ctypes.byref(fs.c),
+                                      ctypes.byref(params) if params is not None else None,
+                                      ctypes.byref(out)), "stlite_workspace_size")
+    return int(out.value)
+
+
+def workspace(shape: Shape, frames, params: Params | None = None, device="cuda"):
+    """Zero-filled workspace tensor of the size the library asks for."""
+    return torch.zeros(stlite_workspace_size(shape, frames, params), dtype=torch.uint8, device=device)
+
+
+def stlite_score(q, k, a_base, ws, stream=None):
+    sh = make_shape(q, k)
+    _check(_lib.stlite_score(ctypes.byref(sh), _ptr(q), _ptr(k), _ptr(a_base), _ptr(ws), ws.numel(),
+                             _stream(stream)), "stlite_score")
+
+
+def stlite_gate_frames(q, k, frames, budget, rho, tau, gate, ws, stream=None):
+    sh = make_shape(q, k)
+    fs = _frames(frames)
+    _check(_lib.stlite_gate_frames(ctypes.byref(sh), ctypes.byref(fs.c), _ptr(k), int(budget), _ptr(rho),
+                                   _ptr(tau), _ptr(gate), _ptr(ws), ws.numel(), _stream(stream)),
+           "stlite_gate_frames")
+
+
+def stlite_spatial_saliency(q, k, frames, phi, ws, stream=None):
+    sh = make_shape(q, k)
+    fs = _frames(frames)
+    _check(_lib.stlite_spatial_saliency(ctypes.byref(sh), ctypes.byref(fs.c), _ptr(k), _ptr(phi), _ptr(ws),
+                                        ws.numel(), _stream(stream)), "stlite_spatial_saliency")
+
+
+def stlite_select_topk(q, k, frames, params, a_base, phi, gate, budget, idx, score_out, ws, stream=None):
+    sh = make_shape(q, k)
+    fs = _frames(frames)
+    _check(_lib.stlite_select_topk(ctypes.byref(sh), ctypes.byref(fs.c), ctypes.byref(params), _ptr(a_base),
+                                   _ptr(phi), _ptr(gate), int(budget), _ptr(idx), _ptr(score_out), _ptr(ws),
+                                   ws.numel(), _stream(stream)), "stlite_select_topk")
+
+
+def stlite_compact(q, k, v, budget, idx, k_out, v_out, stream=None):
+    sh = make_shape(q, k)
+    _check(_lib.stlite_compact(ctypes.byref(sh), int(budget), _ptr(idx), _ptr(k), _ptr(v), _ptr(k_out),
+                               _ptr(v_out), _stream(stream)), "stlite_compact")
+
+
+def stlite_compress_layer(q, k, v, frames, params, k_out, v_out, idx_out, ws, stream=None) -> int:
+    sh = make_shape(q, k)
+    fs = _frames(frames)
+    b = ctypes.c_int32(0)
+    _check(_lib.stlite_compress_layer(ctypes.byref(sh), ctypes.byref(fs.c), ctypes.byref(params), _ptr(q),
+                                      _ptr(k), _ptr(v), _ptr(k_out), _ptr(v_out), _ptr(idx_out),
+                                      ctypes.byref(b), _ptr(ws), ws.numel(), _stream(stream)),
+           "stlite_compress_layer")
+    return int(b.value)
+
+
+def stlite_device_status(ws, stream=None) -> int:
+    st = ctypes.c_int32(0)
+    _check(_lib.stlite_device_status(_ptr(ws), _stream(stream), ctypes.byref(st)), "stlite_device_status")
+    return int(st.value)
+
+
+def stlite_timing_enable(on: bool = True):
+    _check(_lib.stlite_timing_enable(1 if on else 0), "stlite_timing_enable")
+
+
+def stlite_timing_read() -> dict:
+    """{kernel name: (launches, total device ms)} since the last read."""
+    cap = 64
+    buf = (KernelTime * cap)()
+    cnt = ctypes.c_int32(0)
+    _check(_lib.stlite_timing_read(buf, cap, ctypes.byref(cnt)), "stlite_timing_read")
+    return {buf[i].name.decode(): (int(buf[i].launches), float(buf[i].total_ms)) for i in range(min(cnt.value, cap))}
+
+
+# ------------------------------------------------------- convenience layer
+
+def compress_layer(q, k, v, frames, beta=0.2, k_override=0, alpha=1.0, tsg_enable=1, css_enable=1,
+                   ws=None, stream=None):
+    """Allocates outputs (and a workspace if none is given) and runs
+    stlite_compress_layer.  Returns (k_out, v_out, idx)."""
+    fs = _frames(frames)
+    params = make_params(beta, k_override, alpha, tsg_enable, css_enable)
+    sh = make_shape(q, k)
+    b = stlite_budget(sh.n_tokens, beta, k_override)
+    if b < 1:
+        raise StliteError(STLITE_EINVAL, "stlite_budget")
+    if ws is None:
+        ws = workspace(sh, fs, params, device=k.device)
+    k_out = torch.empty((b, sh.n_kv_heads, sh.head_dim), dtype=k.dtype, device=k.device)
+    v_out = torch.empty_like(k_out)
+    idx = torch.empty((sh.n_kv_heads, b), dtype=torch.int32, device=k.device)
+    stlite_compress_layer(q, k, v, fs, params, k_out, v_out, idx, ws, stream)
+    return k_out, v_out, idx

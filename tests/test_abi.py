@@ -1,0 +1,105 @@
+"""C-ABI library checks that need no GPU: the library builds and loads, it
+exports every symbol ``include/stlite.h`` declares, and the host-side
+validation rejects malformed calls before anything is enqueued."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2603_00188_gb300 import build as pkg_build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def st():
+    pkg_build.build()
+    from paper_2603_00188_gb300 import stlite
+    return stlite
+
+
+def header_functions():
+    text = open(os.path.join(ROOT, "include", "stlite.h")).read()
+    return sorted(set(re.findall(r"STLITE_API\s+[\w\s\*]+?\b(stlite_\w+)\s*\(", text)))
+
+
+def test_exports_match_header(st):
+    declared = header_functions()
+    assert len(declared) >= 10
+    assert sorted(st.EXPORTED) == declared
+    lib = ctypes.CDLL(st._LIB_PATH)
+    for name in declared:
+        assert hasattr(lib, name), name
+
+
+@pytest.mark.parametrize("n,beta,ko", [(1152, 0.2, 0), (23680, 0.1, 0), (23680, 0.3, 0), (53600, 0.2, 0),
+                                       (132800, 0.1, 0), (10, 1.0, 0), (10, 0.01, 0), (1152, 0.2, 231),
+                                       (5, 0.2, 99), (7, 0.5, 0)])
+def test_budget_matches_oracle(st, n, beta, ko):
+    assert st.stlite_budget(n, beta, ko) == oracle.budget(n, beta, ko)
+
+
+def test_budget_rejects(st):
+    assert st.stlite_budget(0, 0.2, 0) == -1
+    assert st.stlite_budget(10, 0.0, 0) == -1
+    assert st.stlite_budget(10, 1.5, 0) == -1
+
+
+def test_status_strings(st):
+    for s in range(6):
+        assert st._lib.stlite_status_string(s)
+    assert st._lib.stlite_status_string(1).decode() == "invalid argument"
+
+
+def _shape(st, n=100, hq=4, hkv=2, d=128, w=4, dt=0):
+    return st.Shape(n, hq, hkv, d, w, dt)
+
+
+def test_workspace_size_and_validation(st):
+    fr = st.FrameSpec([0, 30], [4, 5], [5, 6])
+    assert st.stlite_workspace_size(_shape(st), fr) > 0
+    bad = [
+        (_shape(st, hq=5), fr, st.STLITE_EINVAL),                 # Hq % Hkv
+        (_shape(st, d=64), fr, st.STLITE_EUNSUPPORTED),           # head_dim
+        (_shape(st, w=0), fr, st.STLITE_EINVAL),
+        (_shape(st, w=300), fr, st.STLITE_EUNSUPPORTED),
+        (_shape(st, dt=7), fr, st.STLITE_EINVAL),
+        (_shape(st), st.FrameSpec([0, 10], [4, 5], [5, 6]), st.STLITE_EINVAL),   # overlap
+        (_shape(st), st.FrameSpec([30, 0], [4, 5], [5, 6]), st.STLITE_EINVAL),   # unsorted
+        (_shape(st), st.FrameSpec([0, 90], [4, 5], [5, 6]), st.STLITE_EINVAL),   # past N
+        (_shape(st), st.FrameSpec([0], [0], [5]), st.STLITE_EINVAL),             # empty grid
+        (_shape(st), st.FrameSpec(np.zeros(257), np.ones(257), np.ones(257)), st.STLITE_EUNSUPPORTED),
+    ]
+    for sh, f, code in bad:
+        with pytest.raises(st.StliteError) as e:
+            st.stlite_workspace_size(sh, f)
+        assert e.value.status == code
+
+
+def test_entry_points_reject_before_launch(st):
+    """Malformed pointers and sizes are refused on the host (no GPU needed)."""
+    lib = st._lib
+    sh = _shape(st)
+    fr = st.FrameSpec([0, 30], [4, 5], [5, 6])
+    prm = st.make_params(0.2)
+    need = st.stlite_workspace_size(sh, fr, prm)
+    P = ctypes.c_void_p
+    good = P(0x10000)
+    mis = P(0x10008)          # not 16-byte aligned
+    assert lib.stlite_score(ctypes.byref(sh), None, good, good, good, need, None) == st.STLITE_EINVAL
+    assert lib.stlite_score(ctypes.byref(sh), mis, good, good, good, need, None) == st.STLITE_EINVAL
+    assert lib.stlite_score(ctypes.byref(sh), good, good, good, good, need - 1, None) == st.STLITE_EWORKSPACE
+    assert lib.stlite_gate_frames(ctypes.byref(sh), ctypes.byref(fr.c), good, 0, good, good, good, good,
+                                  need, None) == st.STLITE_EINVAL
+    bad_prm = st.make_params(beta=0.0)
+    assert lib.stlite_compress_layer(ctypes.byref(sh), ctypes.byref(fr.c), ctypes.byref(bad_prm), good, good,
+                                     good, good, good, good, None, good, need, None) == st.STLITE_EINVAL
+    neg_alpha = st.make_params(alpha=-1.0)
+    assert lib.stlite_select_topk(ctypes.byref(sh), ctypes.byref(fr.c), ctypes.byref(neg_alpha), good, good,
+                                  None, 5, good, None, good, need, None) == st.STLITE_EINVAL
+    assert lib.stlite_compact(ctypes.byref(sh), 0, good, good, good, good, good, None) == st.STLITE_EINVAL
+    assert lib.stlite_compact(ctypes.byref(sh), 101, good, good, good, good, good, None) == st.STLITE_EINVAL
+    assert lib.stlite_device_status(None, None, None) == st.STLITE_EINVAL

@@ -1,0 +1,262 @@
+"""GPU vs oracle parity, stage by stage and end to end, through the C ABI.
+
+Workloads: the seeded synthetic trajectories of ``synth`` at sizes the fp64
+oracle finishes in seconds (several 128-token tiles, ragged tails: 36x36
+frames = 10.1 row tiles and a 1296-column current frame = 2.53 chunks of
+512; w*G = 448, 224 and 96 query rows), the fp32 tiny reference, and edge
+cases.  Full-size configurations are checked in test_full_size_gpu.py.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2603_00188_gb300 import synth
+from parity import (A_FLOOR, A_RTOL, CACHE, COS_ATOL, a_bound, assert_within, check_kept_sets, cos_bound,
+                    exact64, gate_flip_tokens, pool_mask, to_device, visual_mask)
+
+pytestmark = pytest.mark.gpu
+
+WORKLOADS = {
+    "tiny_ref_fp32": lambda: synth.tiny_ref(),
+    "uitars_3f": lambda: synth.scaled("uitars", 3),
+    "traj50_4f": lambda: synth.scaled("traj50", 4),
+    "small_3f": lambda: synth.scaled("small", 3, beta=0.4),
+    "long_3f": lambda: synth.scaled("long", 3, beta=0.1),
+}
+THREADS = 8
+
+
+@pytest.fixture(scope="module")
+def st():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2603_00188_gb300 import build
+    build.build()
+    from paper_2603_00188_gb300 import stlite
+    return stlite
+
+
+def load(name):
+    def make():
+        wl = WORKLOADS[name]()
+        q, k, v = to_device(wl)
+        q64, k64 = exact64(q), exact64(k)
+        b = oracle.budget(wl.n, wl.beta)
+        ref = oracle.compress_layer(q64, k64, wl.frames, beta=wl.beta, threads=THREADS)
+        return wl, q64, k64, b, ref
+    wl, q64, k64, b, ref = CACHE.get(name, make)
+    q, k, v = to_device(wl)
+    return wl, (q, k, v), q64, k64, b, ref
+
+
+def s_tol(x):
+    return A_RTOL * abs(x) + A_FLOOR + COS_ATOL * 2
+
+
+@pytest.mark.parametrize("name", list(WORKLOADS))
+def test_score(st, name):
+    wl, (q, k, v), q64, k64, b, ref = load(name)
+    sh = st.make_shape(q, k)
+    ws = st.workspace(sh, wl.frames)
+    a = torch.empty((sh.n_kv_heads, sh.n_tokens), dtype=torch.float32, device="cuda")
+    st.stlite_score(q, k, a, ws)
+    torch.cuda.synchronize()
+    ag = a.cpu().numpy()
+    for h in range(sh.n_kv_heads):
+        assert_within(ag[h], ref["a"][h], a_bound(ref["a"][h]), "A_base head %d" % h)
+    np.testing.assert_allclose(ag.astype(np.float64).sum(1), wl.q.shape[0], rtol=1e-4)
+    assert st.stlite_device_status(ws) == st.STLITE_OK
+
+
+@pytest.mark.parametrize("name", list(WORKLOADS))
+def test_css(st, name):
+    wl, (q, k, v), q64, k64, b, ref = load(name)
+    sh = st.make_shape(q, k)
+    ws = st.workspace(sh, wl.frames)
+    phi = torch.empty((sh.n_kv_heads, sh.n_tokens), dtype=torch.float32, device="cuda")
+    st.stlite_spatial_saliency(q, k, wl.frames, phi, ws)
+    torch.cuda.synchronize()
+    pg = phi.cpu().numpy()
+    vis = visual_mask(wl.n, wl.frames)
+    assert np.isnan(pg[:, ~vis]).all()
+    assert_within(pg[:, vis], ref["phi"][:, vis], cos_bound(ref["phi"][:, vis]), "Phi")
+
+
+@pytest.mark.parametrize("name", list(WORKLOADS))
+def test_gate(st, name):
+    wl, (q, k, v), q64, k64, b, ref = load(name)
+    sh = st.make_shape(q, k)
+    ws = st.workspace(sh, wl.frames)
+    H, n = sh.n_kv_heads, sh.n_tokens
+    rho = torch.empty((H, n), dtype=torch.float32, device="cuda")
+    tau = torch.empty((H,), dtype=torch.float32, device="cuda")
+    gate = torch.empty((H, n), dtype=torch.uint8, device="cuda")
+    st.stlite_gate_frames(q, k, wl.frames, b, rho, tau, gate, ws)
+    torch.cuda.synchronize()
+    rg, tg, gg = rho.cpu().numpy(), tau.cpu().numpy(), gate.cpu().numpy()
+    pool = pool_mask(n, wl.frames)
+    assert np.isnan(rg[:, ~pool]).all() and (gg[:, ~pool] == 1).all()
+    assert_within(rg[:, pool], ref["rho"][:, pool], cos_bound(ref["rho"][:, pool]), "rho")
+    # staged: the oracle's threshold and gate on the GPU's own rho are exact
+    t2, g2, _ = oracle.tsg_gate(rg.astype(np.float64), wl.frames, b)
+    np.testing.assert_array_equal(t2, tg.astype(np.float64))
+    np.testing.assert_array_equal(g2, gg)
+    # against the oracle's own rho: flips only at the threshold
+    for h in range(H):
+        assert abs(tg[h] - ref["tau"][h]) <= A_RTOL * abs(ref["tau"][h]) + COS_ATOL
+        gate_flip_tokens(gg[h], ref["gate"][h], ref["rho"][h], ref["tau"][h])
+
+
+@pytest.mark.parametrize("name", list(WORKLOADS))
+def test_select_and_compact(st, name):
+    wl, (q, k, v), q64, k64, b, ref = load(name)
+    sh = st.make_shape(q, k)
+    prm = st.make_params(wl.beta)
+    ws = st.workspace(sh, wl.frames, prm)
+    H, n = sh.n_kv_heads, sh.n_tokens
+    a = torch.empty((H, n), dtype=torch.float32, device="cuda")
+    phi = torch.empty_like(a)
+    rho = torch.empty_like(a)
+    tau = torch.empty((H,), dtype=torch.float32, device="cuda")
+    gate = torch.empty((H, n), dtype=torch.uint8, device="cuda")
+    st.stlite_score(q, k, a, ws)
+    st.stlite_spatial_saliency(q, k, wl.frames, phi, ws)
+    st.stlite_gate_frames(q, k, wl.frames, b, rho, tau, gate, ws)
+    idx = torch.empty((H, b), dtype=torch.int32, device="cuda")
+    score = torch.empty_like(a)
+    st.stlite_select_topk(q, k, wl.frames, prm, a, phi, gate, b, idx, score, ws)
+    ko = torch.empty((b, H, sh.head_dim), dtype=k.dtype, device="cuda")
+    vo = torch.empty_like(ko)
+    st.stlite_compact(q, k, v, b, idx, ko, vo)
+    torch.cuda.synchronize()
+    ig, sg = idx.cpu().numpy(), score.cpu().numpy()
+    # S from the GPU's own stage outputs, recomputed by the oracle
+    s2 = oracle.combine(a.cpu().numpy(), phi.cpu().numpy(), gate.cpu().numpy(), wl.frames)
+    assert_within(sg, s2, A_RTOL * np.abs(s2) + 2 * COS_ATOL, "S")
+    # staged exactness: oracle top-B on the GPU's S equals the GPU's idx
+    np.testing.assert_array_equal(oracle.topk(sg.astype(np.float64), b), ig)
+    # compaction is a bit copy
+    raw = torch.int16 if k.dtype == torch.bfloat16 else torch.int32
+    ko2, vo2 = oracle.gather(k.view(raw).cpu().numpy(), v.view(raw).cpu().numpy(), ig)
+    np.testing.assert_array_equal(ko.view(raw).cpu().numpy(), ko2)
+    np.testing.assert_array_equal(vo.view(raw).cpu().numpy(), vo2)
+
+
+@pytest.mark.parametrize("name", list(WORKLOADS))
+def test_end_to_end(st, name):
+    wl, (q, k, v), q64, k64, b, ref = load(name)
+    ko, vo, idx = st.compress_layer(q, k, v, wl.frames, beta=wl.beta)
+    torch.cuda.synchronize()
+    ig = idx.cpu().numpy()
+    H = k.shape[1]
+    assert ig.shape == (H, b)
+    # fused call == staged calls (same kernels, deterministic)
+    sh = st.make_shape(q, k)
+    prm = st.make_params(wl.beta)
+    ws = st.workspace(sh, wl.frames, prm)
+    a = torch.empty((H, wl.n), dtype=torch.float32, device="cuda")
+    phi, rho = torch.empty_like(a), torch.empty_like(a)
+    tau = torch.empty((H,), dtype=torch.float32, device="cuda")
+    gate = torch.empty((H, wl.n), dtype=torch.uint8, device="cuda")
+    st.stlite_score(q, k, a, ws)
+    st.stlite_spatial_saliency(q, k, wl.frames, phi, ws)
+    st.stlite_gate_frames(q, k, wl.frames, b, rho, tau, gate, ws)
+    idx2 = torch.empty_like(idx)
+    st.stlite_select_topk(q, k, wl.frames, prm, a, phi, gate, b, idx2, None, ws)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(idx2.cpu().numpy(), ig)
+    # against the oracle: kept sets equal up to threshold swaps and gate flips
+    gg = gate.cpu().numpy()
+    for h in range(H):
+        flips = gate_flip_tokens(gg[h], ref["gate"][h], ref["rho"][h], ref["tau"][h])
+        check_kept_sets(ig[h], ref["idx"][h], ref["s"][h], b, s_tol, allowed_extra=flips)
+    raw = torch.int16 if k.dtype == torch.bfloat16 else torch.int32
+    ko2, vo2 = oracle.gather(k.view(raw).cpu().numpy(), v.view(raw).cpu().numpy(), ig)
+    np.testing.assert_array_equal(ko.view(raw).cpu().numpy(), ko2)
+    np.testing.assert_array_equal(vo.view(raw).cpu().numpy(), vo2)
+
+
+# ------------------------------------------------------------------ edge cases
+
+def _run_edge(st, wl, beta, k_override=0, tsg=1, css=1, alpha=1.0):
+    q, k, v = to_device(wl)
+    q64, k64 = exact64(q), exact64(k)
+    ko, vo, idx = st.compress_layer(q, k, v, wl.frames, beta=beta, k_override=k_override, tsg_enable=tsg,
+                                    css_enable=css, alpha=alpha)
+    torch.cuda.synchronize()
+    ref = oracle.compress_layer(q64, k64, wl.frames, beta=beta, k_override=k_override, tsg_enable=tsg,
+                                css_enable=css, alpha=alpha, threads=THREADS)
+    ig = idx.cpu().numpy()
+    b = ref["budget"]
+    assert ig.shape[1] == b
+    for h in range(k.shape[1]):
+        flips = set()
+        if tsg and len(wl.frames[0]) >= 2:
+            flips = set(np.nonzero(np.abs(ref["rho"][h] - ref["tau"][h]) <= 1e-3 * abs(ref["tau"][h]) + COS_ATOL)[0].tolist())
+        check_kept_sets(ig[h], ref["idx"][h], ref["s"][h], b, s_tol, allowed_extra=flips)
+    raw = torch.int16 if k.dtype == torch.bfloat16 else torch.int32
+    ko2, _ = oracle.gather(k.view(raw).cpu().numpy(), v.view(raw).cpu().numpy(), ig)
+    np.testing.assert_array_equal(ko.view(raw).cpu().numpy(), ko2)
+    return ig, ref
+
+
+def test_edge_single_frame(st):
+    wl = synth.trajectory(n_steps=1, gh=20, gw=30, n_text=17, seed=(700,))
+    _run_edge(st, wl, 0.2)
+
+
+def test_edge_no_frames_text_only(st):
+    wl = synth.trajectory(n_steps=1, gh=2, gw=2, n_text=301, seed=(701,))
+    wl.offset, wl.grid_h, wl.grid_w = (np.zeros(0, np.int32),) * 3
+    ig, ref = _run_edge(st, wl, 0.3)
+    # text only: S = A_base, so top-B of the window score
+    for h in range(ig.shape[0]):
+        np.testing.assert_array_equal(ig[h], ref["idx"][h])
+
+
+def test_edge_beta_one_and_override(st):
+    wl = synth.scaled("traj50", 2)
+    ig, _ = _run_edge(st, wl, 1.0)
+    assert (ig == np.arange(wl.n)[None, :]).all()
+    _run_edge(st, wl, 0.2, k_override=wl.n - 3)
+    _run_edge(st, wl, 0.2, k_override=1)
+
+
+def test_edge_flags(st):
+    wl = synth.scaled("small", 2)
+    _run_edge(st, wl, 0.25, tsg=0)
+    _run_edge(st, wl, 0.25, css=0)
+    _run_edge(st, wl, 0.25, tsg=0, css=0)
+    _run_edge(st, wl, 0.25, alpha=0.5)
+
+
+def test_edge_ragged_small(st):
+    # N not a multiple of anything, 1x1 and 1xW grids, frames separated by text
+    rng = np.random.default_rng(5)
+    n, hq, hkv, w = 997, 12, 2, 7
+    q = rng.standard_normal((w, hq, 128), dtype=np.float32)
+    k = rng.standard_normal((n, hkv, 128), dtype=np.float32)
+    k[400:500] = k[600:700] + 0.01 * rng.standard_normal((100, hkv, 128), dtype=np.float32)
+    v = rng.standard_normal((n, hkv, 128), dtype=np.float32)
+    wl = synth.Workload("ragged", q, k, v, np.array([3, 10, 41, 400, 600], np.int32),
+                        np.array([1, 1, 7, 10, 10], np.int32), np.array([1, 13, 9, 10, 10], np.int32), beta=0.15)
+    _run_edge(st, wl, 0.15)
+    wl.dtype = "f32"
+    _run_edge(st, wl, 0.15)
+
+
+def test_edge_exact_duplicate_ties(st):
+    # exact duplicate frames: equal rho at the threshold and equal S (ties by index)
+    wl = synth.scaled("long", 4, beta=0.1)
+    _run_edge(st, wl, 0.1)
+
+
+def test_repeat_deterministic(st):
+    wl = synth.scaled("uitars", 2)
+    q, k, v = to_device(wl)
+    outs = [st.compress_layer(q, k, v, wl.frames, beta=0.2) for _ in range(3)]
+    torch.cuda.synchronize()
+    for o in outs[1:]:
+        for x, y in zip(o, outs[0]):
+            assert torch.equal(x, y)
