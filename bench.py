@@ -1,0 +1,458 @@
+#!/usr/bin/env python
+"""Benchmark of the ST-Lite per-layer KV-cache compression pass on GB300.
+
+Workload (one "step"): the 28-layer, 50-step GUI trajectory at UI-TARS-1.5-7B
+head shape -- 50 frames of 32x32 patches + 48 text tokens per step
+(N = 53,600 tokens), 28 query / 4 KV heads, head_dim 128, bf16, window
+w = 32, flat budget beta = 20% (B = 10,720 per head and layer).  A step runs
+the whole pass (window score, TSG, CSS, top-B, compaction) on all 28 layers.
+Synthetic seeded inputs (``synth.trajectory_50``); the 28 layers' K/V
+(3.07 GB) exceed the 129 MB L2, so every layer is read cold.
+
+Metric: KV tokens compressed per second per layer = N * layers / step time.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl stlite|reference]
+
+Under torchrun each rank compresses its own trajectory (weak scaling, no
+data-path collective); rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import threading
+import time
+from concurrent.futures import ThreadPoolExecutor
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "KV tokens compressed/sec per layer at beta=20%"
+UNIT = "tokens/s/layer"
+LAYERS = 28
+N_TOK, N_STEPS, GH, GW, N_TEXT = 53600, 50, 32, 32, 48
+HQ, HKV, D, W, BETA = 28, 4, 128, 32, 0.2
+WORKLOAD = "traj50_32x32+48text_28layers_bf16_beta0.2"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="stlite", choices=["stlite", "reference"])
+    ap.add_argument("--layers", type=int, default=LAYERS)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return dict(hbm=d["hbm_gbs"], bf16=d["bf16_tflops"], bf16_sus=d["bf16_tflops_sustained"],
+                    sm_mhz=d.get("sm_max_mhz", 2070.0), source="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, sm_mhz=2070.0, source="fallback")
+
+
+# --------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi sampling (every 100 ms) of SM clock and throttle reasons."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        self.gpu = gpu_index
+        self.p = None
+
+    def start(self):
+        try:
+            self.p = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.FIELDS,
+                                       "--format=csv,noheader,nounits", "-lms", "100"],
+                                      stdout=self.f, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.p = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.p is None:
+            return dict(sm_mhz=None, sm_max_mhz=None, reasons=["nvidia-smi unavailable"], samples=0)
+        time.sleep(0.15)
+        self.p.terminate()
+        self.p.wait()
+        self.f.flush()
+        with open(self.f.name) as f:
+            rows = [r.strip().split(", ") for r in f if r.strip()]
+        os.unlink(self.f.name)
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            if len(r) < 9:
+                continue
+            try:
+                sm.append(float(r[1]))
+                mx = float(r[2])
+            except ValueError:
+                continue
+            for nm, v in zip(names, r[5:9]):
+                if v.strip() == "Active":
+                    reasons.add(nm)
+        return dict(sm_mhz=statistics.median(sm) if sm else None, sm_max_mhz=mx, reasons=sorted(reasons),
+                    samples=len(sm))
+
+
+# ------------------------------------------------------------------- workload
+
+def gen_layers(layers: int, seed: int):
+    from paper_2603_00188_gb300 import synth
+    with ThreadPoolExecutor(max_workers=min(8, os.cpu_count() or 1)) as ex:
+        return list(ex.map(lambda l: synth.trajectory_50(l, seed=seed), range(layers)))
+
+
+def alg_bytes_per_layer(budget: int) -> float:
+    """Read K once, read the kept V rows, write the kept K and V rows."""
+    s = N_TOK * HKV * D * 2
+    kept = budget * HKV * D * 2
+    return s + kept + 2 * kept
+
+
+def tsg_flops_per_layer() -> float:
+    n_hist = (N_STEPS - 1) * GH * GW
+    return 2.0 * n_hist * GH * GW * D * HKV
+
+
+def score_flops_per_layer() -> float:
+    return 2 * (2.0 * W * (HQ // HKV) * N_TOK * D * HKV)
+
+
+def exps_per_layer() -> float:
+    return 2.0 * W * (HQ // HKV) * N_TOK * HKV
+
+
+# --------------------------------------------------------------- oracle arm
+
+def oracle_sample(wl, pool_stride: int = 16, q_heads: int = HQ // HKV):
+    """Times the oracle on KV head 0 of one layer: the window score of
+    `q_heads` of the head's G query heads, CSS, the TSG threshold and gate,
+    integrated score and top-B in full, and rho on every pool_stride-th
+    historical token.  Returns the seconds extrapolated to the whole layer
+    (all query heads, every historical token, all KV heads), the measured
+    seconds, and a description of the sample."""
+    import oracle
+    G = HQ // HKV
+    q64 = wl.q.astype(np.float64)
+    k64 = wl.k.astype(np.float64)
+    off, gh, gw = wl.frames
+    b = oracle.budget(wl.n, wl.beta)
+    kh = np.ascontiguousarray(k64[:, :1])
+    qh = np.ascontiguousarray(q64[:, :q_heads])
+    t0 = time.perf_counter()
+    a = oracle.abase(qh, kh)
+    t1 = time.perf_counter()
+    phi = oracle.css_phi(kh, wl.frames)
+    t2 = time.perf_counter()
+    pool = np.concatenate([np.arange(o, o + x * y) for o, x, y in zip(off[:-1], gh[:-1], gw[:-1])])
+    sample = pool[::pool_stride]
+    rho = np.full((1, wl.n), np.nan)
+    for i in sample:
+        rho[0, i] = oracle.tsg_rho_token(kh, 0, int(i), wl.frames)
+    t3 = time.perf_counter()
+    rho[0, pool] = np.nan_to_num(rho[0, pool], nan=0.5)   # unsampled tokens: placeholder values
+    tau, gate, _ = oracle.tsg_gate(rho, wl.frames, b)
+    s = oracle.combine(a, phi, gate, wl.frames)
+    oracle.topk(s, b)
+    t4 = time.perf_counter()
+    per_head = (t1 - t0) * (G / q_heads) + (t2 - t1) + (t3 - t2) * (len(pool) / len(sample)) + (t4 - t3)
+    note = ("oracle on KV head 0 of one layer: window score of %d/%d query heads, CSS, gate and top-B in "
+            "full, rho on 1/%d of the %d historical tokens; extrapolated to all query heads, all historical "
+            "tokens and %d KV heads" % (q_heads, G, pool_stride, len(pool), HKV))
+    return per_head * HKV, t4 - t0, note
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    sys.stdout.flush()
+    from paper_2603_00188_gb300 import synth
+    import oracle
+    oracle.build()
+    vals = []
+    note = ""
+    wls = gen_layers(2, seed=0)
+    for wl in wls:   # the bf16-rounded inputs the GPU arm sees
+        import torch
+        wl.q = torch.from_numpy(wl.q).to(torch.bfloat16).float().numpy()
+        wl.k = torch.from_numpy(wl.k).to(torch.bfloat16).float().numpy()
+    for step in range(args.warmup + args.steps):
+        t_layer, _, note = oracle_sample(wls[step % len(wls)], pool_stride=256, q_heads=1)
+        if step >= args.warmup:
+            vals.append(N_TOK / t_layer)
+    value = statistics.mean(vals)
+    line = dict(impl="reference", metric=METRIC, value=value, unit=UNIT, n_gpus=args.gpus, steps=args.steps,
+                warmup=args.warmup, ms_per_step=1e3 * N_TOK * LAYERS / value, higher_is_better=True,
+                scaling="weak", vs_baseline=None, dtype="f64", data="synthetic",
+                config=dict(workload=WORKLOAD, layers=LAYERS, n_tokens=N_TOK, beta=BETA),
+                cpu_baseline=dict(value=value, unit=UNIT, cores=1, kind="oracle", sample=note),
+                e2e=dict(value=value, unit=UNIT, h2d_bytes_per_step=0, d2h_bytes_per_step=0))
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------- GPU arm
+
+def src_digest():
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2603_00188_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode() + f.read())
+    return h.hexdigest()[:16]
+
+
+def traffic_for(kernel: str):
+    """Per-launch DRAM bytes of `kernel` from the committed ncu summary, if it
+    was taken on the current sources."""
+    p = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    if d.get("src_digest") != src_digest():
+        return None
+    e = d.get("kernels", {}).get(kernel)
+    return None if e is None else e.get("dram_bytes_per_launch_full")
+
+
+def run_gpu(args):
+    import torch
+    import torch.distributed as dist
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    from paper_2603_00188_gb300 import build as pkg_build
+    if rank == 0:
+        pkg_build.build()
+    if world > 1:
+        dist.barrier()
+    from paper_2603_00188_gb300 import stlite
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    peaks = load_peaks()
+    L = args.layers
+    wls = gen_layers(L, seed=rank)
+    fs = stlite.FrameSpec(*wls[0].frames)
+    host = []
+    for wl in wls:
+        host.append(tuple(torch.from_numpy(x).to(torch.bfloat16).pin_memory() for x in (wl.q, wl.k, wl.v)))
+    qs = [h[0].to(dev) for h in host]
+    ks = [h[1].to(dev) for h in host]
+    vs = [h[2].to(dev) for h in host]
+    prm = stlite.make_params(BETA)
+    sh = stlite.make_shape(qs[0], ks[0])
+    budget = stlite.stlite_budget(N_TOK, BETA)
+    ws = stlite.workspace(sh, fs, prm, device=dev)
+    kos = [torch.empty((budget, HKV, D), dtype=torch.bfloat16, device=dev) for _ in range(L)]
+    vos = [torch.empty_like(kos[0]) for _ in range(L)]
+    idxs = [torch.empty((HKV, budget), dtype=torch.int32, device=dev) for _ in range(L)]
+    stream = torch.cuda.Stream(device=dev)
+
+    def step(st=None):
+        for l in range(L):
+            stlite.stlite_compress_layer(qs[l], ks[l], vs[l], fs, prm, kos[l], vos[l], idxs[l], ws, st)
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            step(stream)
+    stream.synchronize()
+    assert stlite.stlite_device_status(ws, stream) == stlite.STLITE_OK
+
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        step(stream)
+    # ---- timed region: K graph replays of the full 28-layer step.  The clock
+    # sampler runs from one second of untimed replays (steady clocks) to the end.
+    clocks = ClockSampler(local)
+    clocks.start()
+    t_warm = time.perf_counter()
+    with torch.cuda.stream(stream):
+        while True:
+            for _ in range(max(3, args.warmup)):
+                graph.replay()
+            stream.synchronize()
+            if time.perf_counter() - t_warm > 1.0:
+                break
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(args.steps):
+            graph.replay()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    clk = clocks.stop()
+    ms = e0.elapsed_time(e1) / args.steps
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    assert stlite.stlite_device_status(ws, stream) == stlite.STLITE_OK
+    value = world * N_TOK * L / (ms * 1e-3)
+
+    # ---- per-kernel device time (CUDA events around each launch, eager replay)
+    stlite.stlite_timing_read()
+    stlite.stlite_timing_enable(True)
+    with torch.cuda.stream(stream):
+        for _ in range(args.steps):
+            step(stream)
+    stream.synchronize()
+    stlite.stlite_timing_enable(False)
+    ktimes = stlite.stlite_timing_read()
+    per_step_launches = sum(c for c, _ in ktimes.values()) // args.steps
+    kernels = {k: dict(launches_per_step=c // args.steps, ms_per_launch=t / c, share=None)
+               for k, (c, t) in ktimes.items()}
+    tot = sum(t for _, t in ktimes.values())
+    for k, (c, t) in ktimes.items():
+        kernels[k]["share"] = t / tot
+    dom = max(ktimes, key=lambda k: ktimes[k][1])
+    t_dom = ktimes[dom][1] / ktimes[dom][0] * 1e-3
+    if dom.startswith("tsg"):
+        ach = tsg_flops_per_layer() / t_dom / 1e12
+        roof = dict(bound="tensor", achieved=ach, peak=peaks["bf16_sus"], unit="TFLOP/s",
+                    frac=ach / peaks["bf16_sus"], kernel=dom,
+                    work="2*N_hist*N_cur*d*H_kv = %.3g FLOP per launch (one layer)" % tsg_flops_per_layer())
+    elif dom.startswith(("colsum", "rowstats")):
+        mufu_peak = 152 * 16 * peaks["sm_mhz"] * 1e6 / 1e12  # T exp/s
+        ach = exps_per_layer() / 2 / t_dom / 1e12
+        roof = dict(bound="alu", achieved=ach, peak=mufu_peak, unit="Texp/s", frac=ach / mufu_peak, kernel=dom,
+                    work="w*G*N*H_kv = %.3g exp2 per launch" % (exps_per_layer() / 2))
+    else:
+        ach = alg_bytes_per_layer(budget) / t_dom / 1e9
+        roof = dict(bound="hbm", achieved=ach, peak=peaks["hbm"], unit="GB/s", frac=ach / peaks["hbm"], kernel=dom)
+    roof["traffic"] = traffic_for(dom)
+    roof["peak_source"] = peaks["source"] + (" sustained" if roof["unit"] == "TFLOP/s" else "")
+
+    # ---- end to end: host (pinned) inputs -> device -> compress -> host outputs
+    e2e = None
+    if not args.no_e2e:
+        h_out = [(torch.empty(kos[0].shape, dtype=torch.bfloat16).pin_memory(),
+                  torch.empty(vos[0].shape, dtype=torch.bfloat16).pin_memory(),
+                  torch.empty(idxs[0].shape, dtype=torch.int32).pin_memory()) for _ in range(L)]
+        cp_in, cp_out = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
+        ev_in = [torch.cuda.Event() for _ in range(L)]
+        ev_done = [torch.cuda.Event() for _ in range(L)]
+        bi = sum(t.numel() * t.element_size() for h in host for t in h)
+        bo = sum(t.numel() * t.element_size() for h in h_out for t in h)
+
+        def e2e_step():
+            for l in range(L):
+                with torch.cuda.stream(cp_in):
+                    qs[l].copy_(host[l][0], non_blocking=True)
+                    ks[l].copy_(host[l][1], non_blocking=True)
+                    vs[l].copy_(host[l][2], non_blocking=True)
+                    ev_in[l].record(cp_in)
+            for l in range(L):
+                stream.wait_event(ev_in[l])
+                stlite.stlite_compress_layer(qs[l], ks[l], vs[l], fs, prm, kos[l], vos[l], idxs[l], ws, stream)
+                ev_done[l].record(stream)
+                cp_out.wait_event(ev_done[l])
+                with torch.cuda.stream(cp_out):
+                    h_out[l][0].copy_(kos[l], non_blocking=True)
+                    h_out[l][1].copy_(vos[l], non_blocking=True)
+                    h_out[l][2].copy_(idxs[l], non_blocking=True)
+            stream.wait_stream(cp_out)
+
+        for _ in range(args.warmup):
+            e2e_step()
+            cp_in.wait_stream(stream)
+        torch.cuda.synchronize()
+        barrier()
+        f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        f0.record(stream)
+        cp_in.wait_stream(stream)
+        for _ in range(args.steps):
+            e2e_step()
+            cp_in.wait_stream(stream)
+        f1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        ms_e2e = f0.elapsed_time(f1) / args.steps
+        if world > 1:
+            t = torch.tensor([ms_e2e], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ms_e2e = float(t.item())
+        # the final host copy equals the device result
+        assert torch.equal(h_out[0][2], idxs[0].cpu())
+        e2e = dict(value=world * N_TOK * L / (ms_e2e * 1e-3), unit=UNIT, h2d_bytes_per_step=bi,
+                   d2h_bytes_per_step=bo, ms_per_step=ms_e2e)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        oracle.build()
+        wl0 = wls[0]
+        wl0.q, wl0.k = host[0][0].float().numpy(), host[0][1].float().numpy()   # the bf16 inputs
+        t_layer, t_raw, note = oracle_sample(wl0, pool_stride=16)
+        cpu = dict(value=N_TOK / t_layer, unit=UNIT, cores=1, kind="oracle", sample=note,
+                   measured_s=round(t_raw, 2))
+
+    if rank == 0:
+        line = dict(metric=METRIC, value=value, unit=UNIT, n_gpus=world, steps=args.steps, warmup=args.warmup,
+                    ms_per_step=ms, higher_is_better=True, scaling="weak", vs_baseline=None, dtype="bf16",
+                    data="synthetic",
+                    config=dict(workload=WORKLOAD, layers=L, n_tokens=N_TOK, frames=N_STEPS, grid="%dx%d" % (GH, GW),
+                                text_per_step=N_TEXT, q_heads=HQ, kv_heads=HKV, head_dim=D, window=W, beta=BETA,
+                                budget=budget, l2="inputs larger than L2 (%.2f GB K/V per step)" %
+                                (2 * L * N_TOK * HKV * D * 2 / 1e9),
+                                timing="CUDA graph of one step, replayed", parallelism="dp%d" % world),
+                    hbm=dict(achieved_gbs=alg_bytes_per_layer(budget) * L / (ms * 1e-3) / 1e9,
+                             peak_gbs=peaks["hbm"],
+                             frac=alg_bytes_per_layer(budget) * L / (ms * 1e-3) / 1e9 / peaks["hbm"],
+                             bytes_per_layer=alg_bytes_per_layer(budget)),
+                    tensor=dict(achieved_tflops=(tsg_flops_per_layer() + score_flops_per_layer()) * L / (ms * 1e-3) / 1e12,
+                                peak_tflops=peaks["bf16_sus"]),
+                    roofline=roof, kernels=kernels, gpu_launches=per_step_launches * args.steps,
+                    clocks=dict(sm_mhz=clk["sm_mhz"], sm_max_mhz=clk["sm_max_mhz"], reasons=clk["reasons"],
+                                samples=clk["samples"]),
+                    e2e=e2e, cpu_baseline=cpu)
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

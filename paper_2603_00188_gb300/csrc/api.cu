@@ -33,6 +33,7 @@ stlite_status check_shape(const stlite_shape* s) {
   const long long R = (long long)s->window * (s->n_q_heads / s->n_kv_heads);
   if (R > 512) return STLITE_EUNSUPPORTED;
   if ((long long)s->n_tokens * s->n_kv_heads > (1LL << 30)) return STLITE_EUNSUPPORTED;
+  if (s->n_tokens > select_max_tokens()) return STLITE_EUNSUPPORTED;
   return STLITE_OK;
 }
 
@@ -291,8 +292,8 @@ stlite_status stlite_spatial_saliency(const stlite_shape* shape, const stlite_fr
   stlite_status s = prepare(shape, frames, ws, ws_bytes, stream, &c);
   if (s != STLITE_OK) return s;
   if (!k || !phi || !aligned16(k) || !aligned16(phi)) return STLITE_EINVAL;
-  cudaError_t e = run_norms(c, k);
-  if (e == cudaSuccess) e = launch_css(c.p, c.ft, k, c.at<float>(c.plan.rn), phi, c.st);
+  cudaError_t e = launch_css(c.p, c.ft, k, phi, c.at<float>(c.plan.rn), c.st);
+  if (e == cudaSuccess) e = launch_fill_text_nan(c.p, c.ft, phi, c.st);
   return cuda_status(e);
 }
 
@@ -355,10 +356,15 @@ stlite_status stlite_compress_layer(const stlite_shape* shape, const stlite_fram
   const bool tsg = params->tsg_enable && c.ft.n_frames >= 2;
   float* a_base = c.at<float>(c.plan.a_base);
   float* phi = c.at<float>(c.plan.phi);
-  cudaError_t e = run_norms(c, k);
+  // CSS also produces the inverse key norms TSG needs; without CSS a plain
+  // norms pass provides them.
+  cudaError_t e = cudaSuccess;
+  if (params->css_enable)
+    e = launch_css(c.p, c.ft, k, phi, c.at<float>(c.plan.rn), c.st);
+  else if (tsg)
+    e = run_norms(c, k);
   if (e == cudaSuccess && tsg) e = run_tsg(c, k);
   if (e == cudaSuccess) e = run_score(c, q, k, a_base);
-  if (e == cudaSuccess && params->css_enable) e = launch_css(c.p, c.ft, k, c.at<float>(c.plan.rn), phi, c.st);
   if (e != cudaSuccess) return STLITE_ECUDA;
   SelectArgs a = {};
   a.mode = (tsg ? kSelGate : 0) | kSelTopk;

@@ -73,9 +73,14 @@ cudaError_t launch_score(const Problem& p, const void* q, const void* k, float2*
 cudaError_t launch_tsg(const Problem& p, const FrameTable& ft, const void* k, const float* rn,
                        float* rho_part, int nchunk, uint32_t* err, cudaStream_t st);
 
-// CSS saliency Phi (Eqs. 4-5).
-cudaError_t launch_css(const Problem& p, const FrameTable& ft, const void* k, const float* rn,
-                       float* phi, cudaStream_t st);
+// CSS saliency Phi (Eqs. 4-5) of every visual token; also writes the
+// inverse key norms rn of every visual token.  Text entries are not touched.
+cudaError_t launch_css(const Problem& p, const FrameTable& ft, const void* k, float* phi, float* rn,
+                       cudaStream_t st);
+// phi[h][j] = NaN for every text token j.
+cudaError_t launch_fill_text_nan(const Problem& p, const FrameTable& ft, float* phi, cudaStream_t st);
+// Largest N the selection kernel handles.
+int select_max_tokens();
 
 // Selection: mode bit 1 = finish rho, tau and gate (Eqs. 6-8); mode bit 2 =
 // integrated score and top-B (Eq. 9, Sec. 2.1).

@@ -1,79 +1,37 @@
-// Selection kernels.  One 1024-thread CTA per KV head.
+// Selection kernel.  One cluster of kSelCta CTAs per KV head; CTA c owns the
+// contiguous token range [c*chunk, (c+1)*chunk) and keeps its radix keys in
+// shared memory for every pass.
 //   kSelGate: rho_i = |k_i|^-1 * max over slices of rho_part (Eq. 6), tau =
-//             the min(B, |pool|)-th smallest rho (Eq. 7) by radix select,
-//             gate = rho <= tau (Eq. 8).
-//   kSelTopk: S from Eq. 9, then the B-th largest S by radix select and an
-//             ordered stream compaction that emits the kept indices in
-//             ascending order, equal scores resolved towards lower indices.
-// Both selections are exact: keys are the order-preserving uint32 images of
-// the fp32 values, resolved 8 bits per pass.
+//             the min(B, |pool|)-th smallest rho (Eq. 7), gate = rho <= tau
+//             (Eq. 8).
+//   kSelTopk: S from Eq. 9, then the B-th largest S and an ordered stream
+//             compaction that emits the kept indices in ascending order,
+//             equal scores resolved towards lower indices.
+// Both selections are exact radix selects on the order-preserving uint32
+// images of the fp32 values, 8 bits per pass.  Each pass builds a per-CTA
+// histogram with warp-aggregated shared atomics, then every CTA sums the
+// cluster's histograms through distributed shared memory and picks the same
+// digit; one cluster barrier per pass.
+#include <cooperative_groups.h>
+
 #include "kernels.cuh"
+
+namespace cg = cooperative_groups;
 
 namespace stl {
 
+constexpr int kSelCta = 8;
 constexpr int kSelThreads = 1024;
+constexpr int kSelMaxChunk = 46080;  // keys per CTA held in shared memory (180 KB)
 
-// Visits every token of the historical pool (visual tokens of frames
-// 0..F-2), block-strided inside each frame span.
-template <class Fn>
-__device__ __forceinline__ void for_pool(const FrameTable& ft, Fn fn) {
-  for (int f = 0; f + 1 < ft.n_frames; ++f) {
-    const int b = ft.off[f], e = b + ft.gh[f] * ft.gw[f];
-    for (int i = b + threadIdx.x; i < e; i += blockDim.x) fn(i);
-  }
-}
-template <class Fn>
-__device__ __forceinline__ void for_all(int n, Fn fn) {
-  for (int j = threadIdx.x; j < n; j += blockDim.x) fn(j);
-}
-
-// k-th largest (1-indexed) of the keys produced by `visit`; returns the key
-// T and, in *need, how many elements equal to T belong to the top k.
-template <class Visit>
-__device__ uint32_t radix_select_desc(Visit visit, uint32_t k, uint32_t* hist, uint32_t* sel,
-                                      uint32_t* need_out) {
-  uint32_t prefix = 0, mask = 0, need = k;
-  const int tid = threadIdx.x, lane = tid & 31;
-  for (int shift = 24; shift >= 0; shift -= 8) {
-    for (int b = tid; b < 256; b += blockDim.x) hist[b] = 0;
-    __syncthreads();
-    visit([&](uint32_t key) {
-      if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
-    });
-    __syncthreads();
-    if (tid < 32) {
-      uint32_t c[8], s = 0;
-#pragma unroll
-      for (int b = 0; b < 8; ++b) {
-        c[b] = hist[lane * 8 + b];
-        s += c[b];
-      }
-      uint32_t incl = s;  // sum over lanes >= lane
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        uint32_t v = __shfl_down_sync(0xffffffffu, incl, o);
-        if (lane + o < 32) incl += v;
-      }
-      uint32_t above = incl - s;
-#pragma unroll
-      for (int b = 7; b >= 0; --b) {
-        if (above < need && need <= above + c[b]) {
-          sel[0] = (uint32_t)(lane * 8 + b);
-          sel[1] = above;
-        }
-        above += c[b];
-      }
-    }
-    __syncthreads();
-    const uint32_t d = sel[0];
-    need -= sel[1];
-    prefix |= d << shift;
-    mask |= 0xffu << shift;
-    __syncthreads();
-  }
-  *need_out = need;
-  return prefix;
-}
+struct SelShared {
+  uint32_t whist[kSelThreads / 32][256];  // per-warp histograms (no cross-warp atomics)
+  uint32_t hist[2][256];  // this CTA's histogram, double-buffered by pass parity
+  uint32_t tot[256];      // cluster-wide histogram of the current pass
+  uint32_t bcast[4];
+  uint32_t warp_tot[32];
+  uint32_t counts[2];     // (greater, equal) of this CTA for the compaction
+};
 
 // Exclusive block-wide prefix sum of v; *total receives the block sum.
 __device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* warp_tot,
@@ -103,44 +61,119 @@ __device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* w
   return before + x - v;
 }
 
-__global__ void __launch_bounds__(kSelThreads) k_select(Problem p,
-                                                        const __grid_constant__ FrameTable ft,
-                                                        SelectArgs a) {
-  __shared__ uint32_t hist[256];
-  __shared__ uint32_t sel[2];
-  __shared__ uint32_t warp_tot[32];
-  const int h = blockIdx.x, n = p.n;
+// k-th largest (1-indexed) key over the whole cluster; key 0 marks an empty
+// slot.  Returns the key T; *need_out = how many keys equal to T belong to
+// the top k.
+__device__ uint32_t cluster_select_desc(cg::cluster_group& cl, const uint32_t* keys, int len,
+                                        uint32_t k, SelShared& sh, int& pass,
+                                        uint32_t* need_out) {
+  uint32_t prefix = 0, mask = 0, need = k;
+  const int tid = threadIdx.x, lane = tid & 31;
+  const int len_r = (len + blockDim.x - 1) / blockDim.x * blockDim.x;
+  const int nw = blockDim.x >> 5, wid = tid >> 5;
+  uint32_t* wh = sh.whist[wid];
+  for (int shift = 24; shift >= 0; shift -= 8, ++pass) {
+    uint32_t* hb = sh.hist[pass & 1];
+    for (int b = lane; b < 256; b += 32) wh[b] = 0u;
+    __syncwarp();
+    for (int i = tid; i < len_r; i += blockDim.x) {
+      const uint32_t key = i < len ? keys[i] : 0u;
+      const bool valid = key != 0u && (key & mask) == prefix;
+      const uint32_t bin = (key >> shift) & 255u;
+      const uint32_t grp = __match_any_sync(0xffffffffu, valid ? bin : 0x100u + lane);
+      if (valid && lane == __ffs(grp) - 1) wh[bin] += (uint32_t)__popc(grp);
+      __syncwarp();
+    }
+    __syncthreads();
+    for (int b = tid; b < 256; b += blockDim.x) {
+      uint32_t t = 0;
+      for (int w = 0; w < nw; ++w) t += sh.whist[w][b];
+      hb[b] = t;
+    }
+    cl.sync();
+    for (int b = tid; b < 256; b += blockDim.x) {
+      uint32_t t = 0;
+#pragma unroll
+      for (int r = 0; r < kSelCta; ++r) t += cl.map_shared_rank(hb, r)[b];
+      sh.tot[b] = t;
+    }
+    __syncthreads();
+    if (tid < 32) {
+      uint32_t c[8], s = 0;
+#pragma unroll
+      for (int b = 0; b < 8; ++b) {
+        c[b] = sh.tot[lane * 8 + b];
+        s += c[b];
+      }
+      uint32_t incl = s;  // sum over lanes >= lane
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        uint32_t v = __shfl_down_sync(0xffffffffu, incl, o);
+        if (lane + o < 32) incl += v;
+      }
+      uint32_t above = incl - s;
+#pragma unroll
+      for (int b = 7; b >= 0; --b) {
+        if (above < need && need <= above + c[b]) {
+          sh.bcast[0] = (uint32_t)(lane * 8 + b);
+          sh.bcast[1] = above;
+        }
+        above += c[b];
+      }
+    }
+    __syncthreads();
+    need -= sh.bcast[1];
+    prefix |= sh.bcast[0] << shift;
+    mask |= 0xffu << shift;
+    __syncthreads();
+  }
+  *need_out = need;
+  return prefix;
+}
+
+__global__ void __cluster_dims__(kSelCta, 1, 1) __launch_bounds__(kSelThreads)
+    k_select(Problem p, const __grid_constant__ FrameTable ft, SelectArgs a) {
+  extern __shared__ uint32_t keys[];
+  __shared__ SelShared sh;
+  cg::cluster_group cl = cg::this_cluster();
+  const int c = (int)cl.block_rank(), h = blockIdx.y, n = p.n, tid = threadIdx.x;
+  const int chunk = (n + kSelCta - 1) / kSelCta;
+  const int j0 = min(n, c * chunk), j1 = min(n, j0 + chunk), len = j1 - j0;
   const size_t hn = (size_t)h * n;
+  int pass = 0;
 
   if (a.mode & kSelGate) {
     float* rho = a.rho + hn;
     uint8_t* gate = a.gate + hn;
-    for_all(n, [&](int j) {
-      rho[j] = CUDART_NAN_F;
-      gate[j] = 1;
-    });
+    for (int i = tid; i < len; i += blockDim.x) {
+      rho[j0 + i] = CUDART_NAN_F;
+      gate[j0 + i] = 1;
+      keys[i] = 0u;
+    }
     __syncthreads();
     int pool = 0;
     for (int f = 0; f + 1 < ft.n_frames; ++f) pool += ft.gh[f] * ft.gw[f];
-    if (pool > 0) {
-      for_pool(ft, [&](int i) {
+    for (int f = 0; f + 1 < ft.n_frames; ++f) {
+      const int lo = max(ft.off[f], j0), hi = min(ft.off[f] + ft.gh[f] * ft.gw[f], j1);
+      for (int i = lo + tid; i < hi; i += blockDim.x) {
         float mx = -CUDART_INF_F;
-        for (int c = 0; c < a.nchunk; ++c) mx = fmaxf(mx, a.rho_part[((size_t)c * p.hkv + h) * n + i]);
-        rho[i] = mx * a.rn[hn + i];
-      });
+        for (int s = 0; s < a.nchunk; ++s) mx = fmaxf(mx, a.rho_part[((size_t)s * p.hkv + h) * n + i]);
+        const float r = mx * a.rn[hn + i];
+        rho[i] = r;
+        keys[i - j0] = ~float_key(r);  // m-th smallest == m-th largest complement
+      }
     }
     __syncthreads();
     if (pool > 0 && a.tsg_enable) {
-      const uint32_t m = (uint32_t)min(a.budget, pool);
       uint32_t need;
-      // m-th smallest rho == m-th largest of the complemented keys
-      const uint32_t kt = radix_select_desc(
-          [&](auto add) { for_pool(ft, [&](int i) { add(~float_key(rho[i])); }); }, m, hist, sel,
-          &need);
+      const uint32_t kt = cluster_select_desc(cl, keys, len, (uint32_t)min(a.budget, pool), sh, pass, &need);
       const float tau = key_float(~kt);
-      for_pool(ft, [&](int i) { gate[i] = rho[i] <= tau ? 1 : 0; });
-      if (threadIdx.x == 0) a.tau[h] = tau;
-    } else if (threadIdx.x == 0) {
+      for (int f = 0; f + 1 < ft.n_frames; ++f) {
+        const int lo = max(ft.off[f], j0), hi = min(ft.off[f] + ft.gh[f] * ft.gw[f], j1);
+        for (int i = lo + tid; i < hi; i += blockDim.x) gate[i] = rho[i] <= tau ? 1 : 0;
+      }
+      if (c == 0 && tid == 0) a.tau[h] = tau;
+    } else if (c == 0 && tid == 0) {
       a.tau[h] = CUDART_NAN_F;
     }
     __syncthreads();
@@ -152,40 +185,71 @@ __global__ void __launch_bounds__(kSelThreads) k_select(Problem p,
     const uint8_t* gt = a.gate ? a.gate + hn : nullptr;
     float* sc = a.score + hn;
     const float alpha = a.css_enable ? a.alpha : 0.f;
-    for_all(n, [&](int j) {
+    for (int i = tid; i < len; i += blockDim.x) {
+      const int j = j0 + i;
       float s = ab[j];
       if (find_frame(ft, j) >= 0) {
-        float x = s + (alpha != 0.f ? alpha * ph[j] : 0.f);
+        const float x = s + (alpha != 0.f ? alpha * ph[j] : 0.f);
         s = (gt == nullptr || gt[j]) ? x : 0.f;
       }
-      sc[j] = s + 0.0f;
-    });
+      s += 0.0f;
+      sc[j] = s;
+      keys[i] = float_key(s);
+    }
     __syncthreads();
     uint32_t need;
-    const uint32_t T = radix_select_desc(
-        [&](auto add) { for_all(n, [&](int j) { add(float_key(sc[j])); }); },
-        (uint32_t)a.budget, hist, sel, &need);
-    // ordered compaction: kept = key > T, plus the first `need` keys == T
+    const uint32_t T = cluster_select_desc(cl, keys, len, (uint32_t)a.budget, sh, pass, &need);
+    // this CTA's counts, then its offsets from the lower-ranked CTAs
+    uint32_t g_loc = 0, e_loc = 0;
+    for (int i = tid; i < len; i += blockDim.x) {
+      g_loc += keys[i] > T;
+      e_loc += keys[i] == T;
+    }
+    uint32_t tot;
+    block_exclusive_scan(g_loc | (e_loc << 16), sh.warp_tot, &tot);
+    if (tid == 0) {
+      sh.counts[0] = tot & 0xffffu;
+      sh.counts[1] = tot >> 16;
+    }
+    cl.sync();
+    if (tid == 0) {
+      uint32_t gb = 0, eb = 0;
+      for (int r = 0; r < c; ++r) {
+        const uint32_t* rc = cl.map_shared_rank(sh.counts, r);
+        gb += rc[0];
+        eb += rc[1];
+      }
+      sh.bcast[2] = gb;
+      sh.bcast[3] = eb;
+    }
+    __syncthreads();
+    uint32_t run_gt = sh.bcast[2], run_eq = sh.bcast[3];
     int32_t* out = a.idx + (size_t)h * a.budget;
-    uint32_t run_gt = 0, run_eq = 0;
-    for (int base = 0; base < n; base += blockDim.x) {
-      const int j = base + threadIdx.x;
-      const uint32_t key = j < n ? float_key(sc[j]) : 0u;
-      const bool g = j < n && key > T, e = j < n && key == T;
-      uint32_t tot;
-      const uint32_t ex = block_exclusive_scan((g ? 1u : 0u) | (e ? 0x10000u : 0u), warp_tot, &tot);
+    for (int base = 0; base < len; base += blockDim.x) {
+      const int i = base + tid;
+      const uint32_t key = i < len ? keys[i] : 0u;
+      const bool g = i < len && key > T, e = i < len && key == T;
+      const uint32_t ex = block_exclusive_scan((g ? 1u : 0u) | (e ? 0x10000u : 0u), sh.warp_tot, &tot);
       const uint32_t gt_before = run_gt + (ex & 0xffffu), eq_before = run_eq + (ex >> 16);
-      if (g || (e && eq_before < need)) out[gt_before + min(eq_before, need)] = j;
+      if (g || (e && eq_before < need)) out[gt_before + min(eq_before, need)] = j0 + i;
       run_gt += tot & 0xffffu;
       run_eq += tot >> 16;
     }
   }
+  cl.sync();  // no CTA leaves while a peer may still read its shared memory
 }
+
+int select_max_tokens() { return kSelCta * kSelMaxChunk; }
 
 cudaError_t launch_select(const Problem& p, const FrameTable& ft, const SelectArgs& a,
                           cudaStream_t st) {
+  const int chunk = (p.n + kSelCta - 1) / kSelCta;
+  if (chunk > kSelMaxChunk) return cudaErrorNotSupported;
+  const size_t smem = (size_t)chunk * 4;
+  cudaError_t e = cudaFuncSetAttribute(k_select, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)(kSelMaxChunk * 4));
+  if (e != cudaSuccess) return e;
   TimingScope ts(a.mode & kSelGate ? (a.mode & kSelTopk ? "select_gate_topk" : "select_gate") : "select_topk", st);
-  k_select<<<p.hkv, kSelThreads, 0, st>>>(p, ft, a);
+  k_select<<<dim3(kSelCta, p.hkv), kSelThreads, smem, st>>>(p, ft, a);
   return cudaGetLastError();
 }
 

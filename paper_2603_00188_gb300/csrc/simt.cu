@@ -8,80 +8,239 @@ namespace stl {
 constexpr float kLog2e = 1.4426950408889634f;
 
 // ---------------------------------------------------------------- norms
-// rn[h][j] = 1 / max(|k_{j,h}|, 1e-8).  One warp per (token, head); lane l
-// holds elements 4l..4l+3.
+// (unpack16 is shared with the CSS kernel so that both compute a norm with
+// the same sequence of operations: fmaf over elements 0..127 in order.)
+template <typename T>
+__device__ __forceinline__ void unpack16(const uint4& w, float (&f)[16 / sizeof(T)]) {
+  if constexpr (sizeof(T) == 2) {
+    f[0] = __uint_as_float(w.x << 16);
+    f[1] = __uint_as_float(w.x & 0xffff0000u);
+    f[2] = __uint_as_float(w.y << 16);
+    f[3] = __uint_as_float(w.y & 0xffff0000u);
+    f[4] = __uint_as_float(w.z << 16);
+    f[5] = __uint_as_float(w.z & 0xffff0000u);
+    f[6] = __uint_as_float(w.w << 16);
+    f[7] = __uint_as_float(w.w & 0xffff0000u);
+  } else {
+    f[0] = __uint_as_float(w.x);
+    f[1] = __uint_as_float(w.y);
+    f[2] = __uint_as_float(w.z);
+    f[3] = __uint_as_float(w.w);
+  }
+}
+
+// rn[h][j] = 1 / max(|k_{j,h}|, 1e-8), one thread per (token, head) row.
 template <typename T>
 __global__ void __launch_bounds__(256) k_inv_norms(const T* __restrict__ k, int n, int hkv,
                                                    float* __restrict__ rn) {
-  int gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  int lane = threadIdx.x & 31;
-  if (gw >= n * hkv) return;
-  int j = gw / hkv, h = gw - j * hkv;
-  float4 x = Elem<T>::load4(k + ((size_t)j * hkv + h) * kD + lane * 4);
-  float s = warp_sum(dot4(x, x));
-  if (lane == 0) rn[(size_t)h * n + j] = 1.0f / fmaxf(sqrtf(s), 1e-8f);
+  constexpr int kChunks = kD * (int)sizeof(T) / 16;
+  constexpr int kPer = 16 / (int)sizeof(T);
+  const long long rows = (long long)n * hkv;
+  for (long long r = (long long)blockIdx.x * blockDim.x + threadIdx.x; r < rows;
+       r += (long long)gridDim.x * blockDim.x) {
+    const uint4* src = reinterpret_cast<const uint4*>(k + r * kD);
+    uint4 w[kChunks];
+#pragma unroll
+    for (int c = 0; c < kChunks; ++c) w[c] = __ldg(src + c);
+    float sn = 0.f;
+#pragma unroll
+    for (int c = 0; c < kChunks; ++c) {
+      float x[kPer];
+      unpack16<T>(w[c], x);
+#pragma unroll
+      for (int t = 0; t < kPer; ++t) sn = fmaf(x[t], x[t], sn);
+    }
+    const long long j = r / hkv, h = r - j * hkv;
+    rn[h * n + j] = 1.0f / fmaxf(sqrtf(sn), 1e-8f);
+  }
 }
 
 cudaError_t launch_inv_norms(const Problem& p, const void* k, float* rn, cudaStream_t st) {
-  long long warps = (long long)p.n * p.hkv;
-  int blocks = (int)((warps + 7) / 8);
+  long long rows = (long long)p.n * p.hkv;
+  long long blocks = (rows + 255) / 256;
+  if (blocks > 152 * 8) blocks = 152 * 8;
   TimingScope ts("inv_norms", st);
   if (p.dtype == kBF16)
-    k_inv_norms<<<blocks, 256, 0, st>>>((const __nv_bfloat16*)k, p.n, p.hkv, rn);
+    k_inv_norms<<<(int)blocks, 256, 0, st>>>((const __nv_bfloat16*)k, p.n, p.hkv, rn);
   else
-    k_inv_norms<<<blocks, 256, 0, st>>>((const float*)k, p.n, p.hkv, rn);
+    k_inv_norms<<<(int)blocks, 256, 0, st>>>((const float*)k, p.n, p.hkv, rn);
   return cudaGetLastError();
 }
 
 // ---------------------------------------------------------------- CSS
-// Eqs. 4-5.  One warp per (token, head).  Text tokens get NaN; a visual token
-// with no in-grid neighbour gets 0.
+// Eqs. 4-5 on 2-D tiles of one frame's patch grid.  A CTA (tile, frame, head)
+// stages the tile's keys plus a one-cell halo in shared memory (rows padded
+// by 16 bytes, so 8 threads reading 8 different keys hit 8 distinct bank
+// groups), computes every key's inverse norm once and every unordered
+// neighbour pair once (the E, S, SE, SW pairs of each cell), then sums the
+// eight directions of each output cell.  It also writes the inverse norms of
+// its output cells (used by TSG).
+constexpr int kCssThreads = 256;
+constexpr int kCssBudget = 100 * 1024;  // shared-memory bytes per CTA
+constexpr int kCssMaxCols = 64;         // output columns per tile
+
 template <typename T>
-__global__ void __launch_bounds__(256) k_css(const T* __restrict__ k, const float* __restrict__ rn,
-                                             const __grid_constant__ FrameTable ft, int hkv,
-                                             float* __restrict__ phi) {
-  int n = ft.n_tokens;
-  int gw_ = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  int lane = threadIdx.x & 31;
-  if (gw_ >= n * hkv) return;
-  int j = gw_ / hkv, h = gw_ - j * hkv;
-  int f = find_frame(ft, j);
-  if (f < 0) {
-    if (lane == 0) phi[(size_t)h * n + j] = CUDART_NAN_F;
-    return;
+struct CssGeom {
+  static constexpr int kStride = kD * (int)sizeof(T) + 16;   // padded key row
+  static constexpr int kCellBytes = kStride + 5 * 4;         // key + rn + 4 pair dots
+  static constexpr int kCap = kCssBudget / kCellBytes;       // cells per CTA
+  // output tile of CB columns x RB rows, loaded as (RB+2) x (CB+2) cells
+  __host__ __device__ static void tile(int gh, int gw, int& RB, int& CB) {
+    CB = gw < kCssMaxCols ? gw : kCssMaxCols;
+    RB = kCap / (CB + 2) - 2;
+    if (RB < 1) RB = 1;
+    if (RB > gh) RB = gh;
   }
-  int off = ft.off[f], gh = ft.gh[f], gw = ft.gw[f];
-  int local = j - off, u = local / gw, v = local - u * gw;
-  float4 c = Elem<T>::load4(k + ((size_t)j * hkv + h) * kD + lane * 4);
-  float rc = rn[(size_t)h * n + j];
-  float sum = 0.f;
-  int cnt = 0;
+  __host__ __device__ static int tiles(int gh, int gw) {
+    int RB, CB;
+    tile(gh, gw, RB, CB);
+    return ((gh + RB - 1) / RB) * ((gw + CB - 1) / CB);
+  }
+};
+
+template <typename T>
+__global__ void __launch_bounds__(kCssThreads) k_css(const T* __restrict__ k,
+                                                     const __grid_constant__ FrameTable ft, int hkv,
+                                                     float* __restrict__ phi,
+                                                     float* __restrict__ rn_out) {
+  using Gm = CssGeom<T>;
+  constexpr int kChunks = kD * (int)sizeof(T) / 16;
+  constexpr int kPer = 16 / (int)sizeof(T);
+  extern __shared__ float4 css_smem[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>(css_smem);
+  const int f = blockIdx.y, h = blockIdx.z, n = ft.n_tokens, tid = threadIdx.x;
+  if (f >= ft.n_frames) return;
+  const int gh = ft.gh[f], gw = ft.gw[f], off = ft.off[f];
+  int RB, CB;
+  Gm::tile(gh, gw, RB, CB);
+  const int tv = (gw + CB - 1) / CB;
+  if ((int)blockIdx.x >= ((gh + RB - 1) / RB) * tv) return;
+  const int u0 = ((int)blockIdx.x / tv) * RB, v0 = ((int)blockIdx.x % tv) * CB;
+  const int TW = CB + 2, TH = RB + 2, cells = TW * TH;
+  uint8_t* keys = sm;
+  float* rn = reinterpret_cast<float*>(sm + (size_t)cells * Gm::kStride);
+  float* dE = rn + cells;
+  float* dS = dE + cells;
+  float* dSE = dS + cells;
+  float* dSW = dSE + cells;
+  // stage the tile (local cell (a, b) = grid cell (u0 - 1 + a, v0 - 1 + b))
+  // with asynchronous 16-byte copies; cells outside the grid stay unloaded
+  for (int e = tid; e < cells * kChunks; e += blockDim.x) {
+    const int cell = e / kChunks, ch = e - cell * kChunks;
+    const int u = u0 - 1 + cell / TW, v = v0 - 1 + cell % TW;
+    if (u < 0 || u >= gh || v < 0 || v >= gw) continue;
+    const T* src = k + ((size_t)(off + u * gw + v) * hkv + h) * kD + ch * kPer;
+    const uint32_t dst = static_cast<uint32_t>(__cvta_generic_to_shared(keys + (size_t)cell * Gm::kStride + 16 * ch));
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+  }
+  asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+  __syncthreads();
+  // one thread per cell: its norm and its E, S, SE, SW pair dots in one sweep
+  // (a missing partner reads the cell itself and is discarded)
+  for (int cell = tid; cell < cells; cell += blockDim.x) {
+    const int a = cell / TW, b = cell % TW;
+    const int u = u0 - 1 + a, v = v0 - 1 + b;
+    if (u < 0 || u >= gh || v < 0 || v >= gw) continue;
+    const bool fwd = a <= RB && u + 1 < gh;
+    const bool hasE = b + 1 < TW && v + 1 < gw;
+    const bool hasS = fwd;
+    const bool hasSE = fwd && b + 1 < TW && v + 1 < gw;
+    const bool hasSW = fwd && b >= 1 && v >= 1;
+    const uint8_t* p0 = keys + (size_t)cell * Gm::kStride;
+    const uint8_t* pE = hasE ? p0 + Gm::kStride : p0;
+    const uint8_t* pS = hasS ? p0 + (size_t)TW * Gm::kStride : p0;
+    const uint8_t* pSE = hasSE ? p0 + (size_t)(TW + 1) * Gm::kStride : p0;
+    const uint8_t* pSW = hasSW ? p0 + (size_t)(TW - 1) * Gm::kStride : p0;
+    float sn = 0.f, sE = 0.f, sS = 0.f, sSE = 0.f, sSW = 0.f;
+#pragma unroll 4
+    for (int c = 0; c < kChunks; ++c) {
+      float x[kPer], y[kPer];
+      unpack16<T>(*reinterpret_cast<const uint4*>(p0 + 16 * c), x);
 #pragma unroll
-  for (int du = -1; du <= 1; ++du) {
+      for (int t = 0; t < kPer; ++t) sn = fmaf(x[t], x[t], sn);
+      unpack16<T>(*reinterpret_cast<const uint4*>(pE + 16 * c), y);
 #pragma unroll
-    for (int dv = -1; dv <= 1; ++dv) {
-      if (du == 0 && dv == 0) continue;
-      int pu = u + du, pv = v + dv;
-      if (pu < 0 || pu >= gh || pv < 0 || pv >= gw) continue;
-      int nb = off + pu * gw + pv;
-      float4 x = Elem<T>::load4(k + ((size_t)nb * hkv + h) * kD + lane * 4);
-      float dot = warp_sum(dot4(c, x));
-      sum += dot * rc * rn[(size_t)h * n + nb];
-      ++cnt;
+      for (int t = 0; t < kPer; ++t) sE = fmaf(x[t], y[t], sE);
+      unpack16<T>(*reinterpret_cast<const uint4*>(pS + 16 * c), y);
+#pragma unroll
+      for (int t = 0; t < kPer; ++t) sS = fmaf(x[t], y[t], sS);
+      unpack16<T>(*reinterpret_cast<const uint4*>(pSE + 16 * c), y);
+#pragma unroll
+      for (int t = 0; t < kPer; ++t) sSE = fmaf(x[t], y[t], sSE);
+      unpack16<T>(*reinterpret_cast<const uint4*>(pSW + 16 * c), y);
+#pragma unroll
+      for (int t = 0; t < kPer; ++t) sSW = fmaf(x[t], y[t], sSW);
     }
+    rn[cell] = 1.0f / fmaxf(sqrtf(sn), 1e-8f);
+    dE[cell] = sE;
+    dS[cell] = sS;
+    dSE[cell] = sSE;
+    dSW[cell] = sSW;
   }
-  if (lane == 0) phi[(size_t)h * n + j] = cnt ? 1.0f - sum / (float)cnt : 0.0f;
+  __syncthreads();
+  for (int o = tid; o < RB * CB; o += blockDim.x) {
+    const int u = u0 + o / CB, v = v0 + o % CB;
+    if (u >= gh || v >= gw) continue;
+    const int c = (o / CB + 1) * TW + (o % CB + 1);
+    const float r0 = rn[c];
+    float sum = 0.f;
+    int cnt = 0;
+    const bool up = u > 0, dn = u + 1 < gh, lf = v > 0, rt = v + 1 < gw;
+    if (rt) { sum += dE[c] * r0 * rn[c + 1]; ++cnt; }
+    if (lf) { sum += dE[c - 1] * rn[c - 1] * r0; ++cnt; }
+    if (dn) { sum += dS[c] * r0 * rn[c + TW]; ++cnt; }
+    if (up) { sum += dS[c - TW] * rn[c - TW] * r0; ++cnt; }
+    if (dn && rt) { sum += dSE[c] * r0 * rn[c + TW + 1]; ++cnt; }
+    if (up && lf) { sum += dSE[c - TW - 1] * rn[c - TW - 1] * r0; ++cnt; }
+    if (dn && lf) { sum += dSW[c] * r0 * rn[c + TW - 1]; ++cnt; }
+    if (up && rt) { sum += dSW[c - TW + 1] * rn[c - TW + 1] * r0; ++cnt; }
+    const int j = off + u * gw + v;
+    phi[(size_t)h * n + j] = cnt ? 1.0f - sum / (float)cnt : 0.0f;
+    rn_out[(size_t)h * n + j] = r0;
+  }
 }
 
-cudaError_t launch_css(const Problem& p, const FrameTable& ft, const void* k, const float* rn,
-                       float* phi, cudaStream_t st) {
-  long long warps = (long long)p.n * p.hkv;
-  int blocks = (int)((warps + 7) / 8);
+// Phi of text tokens is undefined: NaN (only the staged entry point writes it).
+__global__ void k_fill_text_nan(const __grid_constant__ FrameTable ft, int hkv, float* __restrict__ phi) {
+  const int n = ft.n_tokens;
+  for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e < (long long)n * hkv;
+       e += (long long)gridDim.x * blockDim.x) {
+    const int j = (int)(e % n);
+    if (find_frame(ft, j) < 0) phi[e] = CUDART_NAN_F;
+  }
+}
+
+template <typename T>
+static cudaError_t css_launch_t(const Problem& p, const FrameTable& ft, const void* k, float* phi,
+                                float* rn, cudaStream_t st) {
+  using Gm = CssGeom<T>;
+  int tmax = 0, cmax = 0;
+  for (int f = 0; f < ft.n_frames; ++f) {
+    int RB, CB;
+    Gm::tile(ft.gh[f], ft.gw[f], RB, CB);
+    tmax = max(tmax, Gm::tiles(ft.gh[f], ft.gw[f]));
+    cmax = max(cmax, (RB + 2) * (CB + 2));
+  }
+  if (tmax == 0) return cudaSuccess;
+  const size_t smem = (size_t)cmax * Gm::kCellBytes;
+  cudaError_t e = cudaFuncSetAttribute(k_css<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
   TimingScope ts("css", st);
-  if (p.dtype == kBF16)
-    k_css<<<blocks, 256, 0, st>>>((const __nv_bfloat16*)k, rn, ft, p.hkv, phi);
-  else
-    k_css<<<blocks, 256, 0, st>>>((const float*)k, rn, ft, p.hkv, phi);
+  k_css<T><<<dim3(tmax, ft.n_frames, p.hkv), kCssThreads, smem, st>>>((const T*)k, ft, p.hkv, phi, rn);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_css(const Problem& p, const FrameTable& ft, const void* k, float* phi, float* rn,
+                       cudaStream_t st) {
+  if (p.dtype == kBF16) return css_launch_t<__nv_bfloat16>(p, ft, k, phi, rn, st);
+  return css_launch_t<float>(p, ft, k, phi, rn, st);
+}
+
+cudaError_t launch_fill_text_nan(const Problem& p, const FrameTable& ft, float* phi, cudaStream_t st) {
+  long long tot = (long long)p.n * p.hkv;
+  long long blocks = (tot + 255) / 256;
+  if (blocks > 152 * 8) blocks = 152 * 8;
+  k_fill_text_nan<<<(int)blocks, 256, 0, st>>>(ft, p.hkv, phi);
   return cudaGetLastError();
 }
 

@@ -194,18 +194,40 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!warp_wait(b_accfull + 8 * g, (uint32_t)it & 1u, err, abort_flag)) break;
         tc_fence_after();
         float mx = -CUDART_INF_F;
-        for (int c = 0; c < 8; ++c) {
-          if (c * 32 >= valid_g) break;
-          float v[32];
-          tmem_ld32(tbase + c * 32, v);
-          const float4* r4 = reinterpret_cast<const float4*>(rg + c * 32);
+        if (valid_g == 256) {
+          // full stage: no masked column, packed products and 3-input max
+          float m0 = -CUDART_INF_F, m1 = -CUDART_INF_F;
+#pragma unroll 1
+          for (int c = 0; c < 4; ++c) {
+            float v[64];
+            tmem_ld64(tbase + c * 64, v);
+            const float4* r4 = reinterpret_cast<const float4*>(rg + c * 64);
 #pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            float4 r = r4[i];
-            mx = fmaxf(mx, v[4 * i] * r.x);
-            mx = fmaxf(mx, v[4 * i + 1] * r.y);
-            mx = fmaxf(mx, v[4 * i + 2] * r.z);
-            mx = fmaxf(mx, v[4 * i + 3] * r.w);
+            for (int i = 0; i < 16; ++i) {
+              const float4 r = r4[i];
+              float p0, p1, p2, p3;
+              mul2(v[4 * i], v[4 * i + 1], r.x, r.y, p0, p1);
+              mul2(v[4 * i + 2], v[4 * i + 3], r.z, r.w, p2, p3);
+              m0 = max3(m0, p0, p1);
+              m1 = max3(m1, p2, p3);
+            }
+          }
+          mx = fmaxf(m0, m1);
+        } else {
+          // ragged stage: columns past the frame carry rn = NaN, ignored by fmaxf
+          for (int c = 0; c < 8; ++c) {
+            if (c * 32 >= valid_g) break;
+            float v[32];
+            tmem_ld32(tbase + c * 32, v);
+            const float4* r4 = reinterpret_cast<const float4*>(rg + c * 32);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+              float4 r = r4[i];
+              mx = fmaxf(mx, v[4 * i] * r.x);
+              mx = fmaxf(mx, v[4 * i + 1] * r.y);
+              mx = fmaxf(mx, v[4 * i + 2] * r.z);
+              mx = fmaxf(mx, v[4 * i + 3] * r.w);
+            }
           }
         }
         tc_fence_before();
@@ -259,13 +281,15 @@ __device__ __forceinline__ void online_merge(float& m, float& l, float m2, float
   l = a + b;
 }
 
+template <int MT>
 __global__ void __launch_bounds__(kThreads, 1)
     k_rowstats_umma(const __grid_constant__ CUtensorMap kmap, const __nv_bfloat16* __restrict__ q,
                     Problem p, int nsplit, float2* __restrict__ part, uint32_t* err) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = align1024(smem_raw);
   const RsLayout L = rs_layout(p.R());
-  const int MT = L.MT, KN = L.KN, R = p.R();
+  constexpr int KN = 256 / MT;
+  const int R = p.R();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int split = blockIdx.x, h = blockIdx.y, n = p.n;
   const int per = (((n + nsplit - 1) / nsplit) + KN - 1) / KN * KN;
@@ -304,9 +328,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = *slot;
 
   // per-thread row state for up to 4 M-tiles (epilogue warps)
-  float m_st[4], l_st[4];
+  float m_st[MT], l_st[MT];
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
+  for (int i = 0; i < MT; ++i) {
     m_st[i] = -CUDART_INF_F;
     l_st[i] = 0.f;
   }
@@ -360,26 +384,51 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!warp_wait(b_accfull + 8 * g, u & 1u, err, abort_flag)) break;
       tc_fence_after();
       const int tok = j0 + it * KN;
+#pragma unroll
       for (int mt = 0; mt < MT; ++mt) {
         float m = m_st[mt], l = l_st[mt];
-        for (int cg = 0; cg < KN / 32; ++cg) {
-          const int kbase = tok + cg * 32;
+#pragma unroll 1
+        for (int cg = 0; cg < KN / 64; ++cg) {
+          const int kbase = tok + cg * 64;
           if (kbase >= j1) break;
-          float v[32];
-          tmem_ld32(lanebase + g * 256 + mt * KN + cg * 32, v);
-          const int nv = min(32, j1 - kbase);
-          float mc = -CUDART_INF_F;
+          float v[64];
+          tmem_ld64(lanebase + g * 256 + mt * KN + cg * 64, v);
+          const int nv = min(64, j1 - kbase);
+          if (nv == 64) {
+            // indices 0..63: c0 takes 0, 2..3, 6..7, ..., 62..63; c1 takes 1, 4..5, ..., 60..61
+            float c0 = v[0], c1 = v[1];
 #pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (i < nv) mc = fmaxf(mc, v[i]);
-          const float mn = fmaxf(m, mc);
-          const float mnc = mn * c;
-          float sacc = 0.f;
+            for (int i = 2; i < 62; i += 4) {
+              c0 = max3(c0, v[i], v[i + 1]);
+              c1 = max3(c1, v[i + 2], v[i + 3]);
+            }
+            c0 = max3(c0, v[62], v[63]);
+            const float mn = fmaxf(m, fmaxf(c0, c1));
+            const float mnc = mn * c;
+            float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
 #pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (i < nv) sacc += exp2f(fmaf(v[i], c, -mnc));
-          l = (m == -CUDART_INF_F ? 0.f : l * exp2f((m - mn) * c)) + sacc;
-          m = mn;
+            for (int i = 0; i < 64; i += 4) {
+              s0 += ex2_approx(fmaf(v[i], c, -mnc));
+              s1 += ex2_approx(fmaf(v[i + 1], c, -mnc));
+              s2 += ex2_approx(fmaf(v[i + 2], c, -mnc));
+              s3 += ex2_approx(fmaf(v[i + 3], c, -mnc));
+            }
+            l = (m == -CUDART_INF_F ? 0.f : l * ex2_approx((m - mn) * c)) + ((s0 + s1) + (s2 + s3));
+            m = mn;
+          } else {
+            float mc = -CUDART_INF_F;
+#pragma unroll
+            for (int i = 0; i < 64; ++i)
+              if (i < nv) mc = fmaxf(mc, v[i]);
+            const float mn = fmaxf(m, mc);
+            const float mnc = mn * c;
+            float sacc = 0.f;
+#pragma unroll
+            for (int i = 0; i < 64; ++i)
+              if (i < nv) sacc += ex2_approx(fmaf(v[i], c, -mnc));
+            l = (m == -CUDART_INF_F ? 0.f : l * ex2_approx((m - mn) * c)) + sacc;
+            m = mn;
+          }
         }
         m_st[mt] = m;
         l_st[mt] = l;
@@ -390,11 +439,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
   // merge the two epilogue groups, then write (m * c, l) per query row
-  if (warp >= 2 && g == 1)
+  if (warp >= 2 && g == 1) {
+#pragma unroll
     for (int mt = 0; mt < MT; ++mt) xch[mt * 128 + quarter * 32 + lane] = make_float2(m_st[mt], l_st[mt]);
+  }
   tc_fence_before();
   __syncthreads();
   if (warp >= 2 && g == 0) {
+#pragma unroll
     for (int mt = 0; mt < MT; ++mt) {
       const int row = mt * 128 + quarter * 32 + lane;
       float2 o = xch[row];
@@ -434,8 +486,8 @@ __host__ __device__ inline CsLayout cs_layout(int R) {
 
 __global__ void __launch_bounds__(kThreads, 1)
     k_colsum_umma(const __grid_constant__ CUtensorMap kmap, const __nv_bfloat16* __restrict__ q,
-                  Problem p, const float* __restrict__ bias, float* __restrict__ a_base,
-                  uint32_t* err) {
+                  Problem p, const float2* __restrict__ part, int nsplit,
+                  float* __restrict__ a_base, uint32_t* err) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = align1024(smem_raw);
   const CsLayout L = cs_layout(p.R());
@@ -469,8 +521,23 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_relinquish();
   }
   load_q_sw128(sm, NQ, q, p, h);
-  for (int r = threadIdx.x; r < NQ; r += blockDim.x)
-    bias_s[r] = r < R ? bias[(size_t)h * R + r] : -CUDART_INF_F;
+  // merge pass 1's per-split row statistics: bias_r = -m_r - log2(G l_r), so
+  // that 2^(x c + bias_r) is the softmax probability divided by G
+  for (int r = threadIdx.x; r < NQ; r += blockDim.x) {
+    float b = -CUDART_INF_F;
+    if (r < R) {
+      const float2* pp = part + (size_t)h * nsplit * R + r;
+      float m = -CUDART_INF_F;
+      for (int s = 0; s < nsplit; ++s) m = fmaxf(m, pp[(size_t)s * R].x);
+      float l = 0.f;
+      for (int s = 0; s < nsplit; ++s) {
+        const float2 v = pp[(size_t)s * R];
+        if (v.y > 0.f) l += v.y * exp2f(v.x - m);
+      }
+      b = -m - log2f((float)p.G() * l);
+    }
+    bias_s[r] = b;
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -528,16 +595,36 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t ua = (uint32_t)(it / nstage);
         if (!warp_wait(b_accfull + 8 * g, ua & 1u, err, abort_flag)) break;
         tc_fence_after();
-        float acc = 0.f;
-        for (int cg = 0; cg < NQ / 32; ++cg) {
-          float v[32];
-          tmem_ld32(tbase + cg * 32, v);
+        float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+#pragma unroll 1
+        for (int cg = 0; cg < NQ / 64; ++cg) {
+          float v[64];
+          tmem_ld64(tbase + cg * 64, v);
+          const float4* b4 = reinterpret_cast<const float4*>(bias_s + cg * 64);
+          if (cg * 64 + 64 <= R) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const int r = cg * 32 + i;
-            if (r < R) acc += exp2f(fmaf(v[i], c, bias_s[r]));
+            for (int i = 0; i < 16; ++i) {
+              const float4 b = b4[i];
+              a0 += ex2_approx(fmaf(v[4 * i], c, b.x));
+              a1 += ex2_approx(fmaf(v[4 * i + 1], c, b.y));
+              a2 += ex2_approx(fmaf(v[4 * i + 2], c, b.z));
+              a3 += ex2_approx(fmaf(v[4 * i + 3], c, b.w));
+            }
+          } else {
+#pragma unroll
+            for (int i = 0; i < 64; ++i)
+              if (cg * 64 + i < R) a0 += ex2_approx(fmaf(v[i], c, bias_s[cg * 64 + i]));
           }
         }
+        if (NQ % 64) {
+          const int cb = NQ - 32;
+          float v[32];
+          tmem_ld32(tbase + cb, v);
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (cb + i < R) a1 += ex2_approx(fmaf(v[i], c, bias_s[cb + i]));
+        }
+        const float acc = (a0 + a1) + (a2 + a3);
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(b_accempty + 8 * g);
@@ -632,26 +719,25 @@ cudaError_t launch_score_umma(const Problem& p, const void* q, const void* k, fl
   cudaError_t e = make_kmap(&m1, k, p.n, p.hkv, L1.KN);
   if (e != cudaSuccess) return e;
   if ((e = make_kmap(&m2, k, p.n, p.hkv, 128)) != cudaSuccess) return e;
-  if ((e = cudaFuncSetAttribute(k_rowstats_umma, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                L1.total)) != cudaSuccess)
+  auto rs_kernel = L1.MT == 1 ? k_rowstats_umma<1> : (L1.MT == 2 ? k_rowstats_umma<2> : k_rowstats_umma<4>);
+  if ((e = cudaFuncSetAttribute(rs_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, L1.total)) !=
+      cudaSuccess)
     return e;
   if ((e = cudaFuncSetAttribute(k_colsum_umma, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 L2.total)) != cudaSuccess)
     return e;
-  float* bias = reinterpret_cast<float*>(rowpart + (size_t)p.hkv * nsplit * R);
   {
     TimingScope ts("rowstats_umma", st);
-    k_rowstats_umma<<<dim3(nsplit, p.hkv), kThreads, L1.total, st>>>(
-        m1, (const __nv_bfloat16*)q, p, nsplit, rowpart, err);
+    rs_kernel<<<dim3(nsplit, p.hkv), kThreads, L1.total, st>>>(m1, (const __nv_bfloat16*)q, p, nsplit,
+                                                               rowpart, err);
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  if ((e = launch_row_bias(p, rowpart, nsplit, bias, st)) != cudaSuccess) return e;
   int tiles = (p.n + 127) / 128;
   int gx = (sm_count() + p.hkv - 1) / p.hkv;
   if (gx > tiles) gx = tiles;
   TimingScope ts("colsum_umma", st);
   k_colsum_umma<<<dim3(gx, p.hkv), kThreads, L2.total, st>>>(m2, (const __nv_bfloat16*)q, p,
-                                                              bias, a_base, err);
+                                                              rowpart, nsplit, a_base, err);
   return cudaGetLastError();
 }
 
