@@ -158,6 +158,27 @@ STLITE_API stlite_status stlite_compress_layer(const stlite_shape* shape, const 
                                     const void* v, void* k_out, void* v_out, int32_t* idx_out,
                                     int32_t* budget_out, void* ws, size_t ws_bytes, void* stream);
 
+/* Window score (same result as stlite_score) for callers that cannot
+ * allocate device memory and so cannot provide a workspace -- for example
+ * code running inside an allocator or memory-pool callback, or a process
+ * whose device memory is fully reserved by another runtime.  The paper has no
+ * counterpart: this is a deployment convenience.  Its scratch (an error word
+ * and the per-split softmax row statistics) is one fixed 2 MiB device array
+ * inside the library, which every GPU that loads the library holds until
+ * exit; problems whose scratch, 256 + Hkv*S*w*G*8 + Hkv*w*G*4 bytes (S = the
+ * library's key splits, at most ceil(304/Hkv)), exceeds it are rejected with
+ * STLITE_EUNSUPPORTED.  The call allocates nothing.  Its first call on each
+ * device resolves that device's scratch address (cudaGetSymbolAddress), so
+ * make the first call on a device before any stream capture.  All calls
+ * share the array, which keeps the last call's contents (each call clears
+ * its error word; the statistics are fully rewritten): calls that overlap on
+ * the GPU -- issued to one device on different streams, or from several
+ * threads -- race on it.  Kernel timeouts of this path are not reported (its
+ * error word is internal).
+ * q, k, a_base: as for stlite_score. */
+STLITE_API stlite_status stlite_score_noalloc(const stlite_shape* shape, const void* q, const void* k,
+                                              float* a_base, void* stream);
+
 /* Reads and clears the workspace's device error word (synchronises `stream`).
  * *status receives STLITE_OK or the first error a kernel recorded since the
  * last read (STLITE_ETIMEOUT). */

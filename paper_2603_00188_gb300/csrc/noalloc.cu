@@ -1,0 +1,79 @@
+// stlite_score_noalloc: the window-score call (same kernels as stlite_score)
+// for callers that cannot allocate device memory -- e.g. code running inside
+// an allocator or memory-pool callback, a host with a fixed, fully reserved
+// device budget, or a runtime that forbids cudaMalloc while it owns the
+// device -- and therefore cannot provide the usual workspace.  Its scratch
+// (the device error word and the per-split row statistics of the two-pass
+// softmax) lives in one file-scope device array instead.
+#include <mutex>
+
+#include "../../include/stlite.h"
+#include "kernels.cuh"
+
+using namespace stl;
+
+namespace {
+
+constexpr size_t kScratchBytes = 2u << 20;  // 2 MiB, held by every device that loads the library
+constexpr size_t kErrBytes = 256;           // error word, then the row statistics
+constexpr int kMaxDevices = 64;
+
+// Device-side scratch.  In host code this name is only a stand-in for the
+// symbol: the device address comes from cudaGetSymbolAddress below.
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kScratchBytes];
+
+std::mutex g_setup_mu;
+void* g_scratch_addr[kMaxDevices] = {};
+
+// Once per device, with that device current: resolve the scratch address.
+cudaError_t scratch_address(void** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lk(g_setup_mu);
+  if (!g_scratch_addr[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess) return e;
+    g_scratch_addr[dev] = p;
+  }
+  *out = g_scratch_addr[dev];
+  return cudaSuccess;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+}  // namespace
+
+extern "C" stlite_status stlite_score_noalloc(const stlite_shape* s, const void* q, const void* k,
+                                              float* a_base, void* stream) {
+  if (!s || !q || !k || !a_base) return STLITE_EINVAL;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(a_base)) return STLITE_EINVAL;
+  if (s->n_tokens < 1 || s->n_q_heads < 1 || s->n_kv_heads < 1 || s->window < 1 || s->head_dim < 1)
+    return STLITE_EINVAL;
+  if (s->n_q_heads % s->n_kv_heads != 0) return STLITE_EINVAL;
+  if (s->dtype != STLITE_BF16 && s->dtype != STLITE_F32) return STLITE_EINVAL;
+  if (s->head_dim != STLITE_HEAD_DIM || s->window > 256) return STLITE_EUNSUPPORTED;
+  if ((long long)s->window * (s->n_q_heads / s->n_kv_heads) > 512) return STLITE_EUNSUPPORTED;
+  Problem p;
+  p.n = s->n_tokens;
+  p.hq = s->n_q_heads;
+  p.hkv = s->n_kv_heads;
+  p.w = s->window;
+  p.dtype = s->dtype == STLITE_BF16 ? kBF16 : kF32;
+  FrameTable ft = {};
+  ft.n_tokens = p.n;
+  const WsPlan plan = plan_workspace(p, ft);
+  const size_t stats = (size_t)p.hkv * plan.nsplit * p.R() * 8 + (size_t)p.hkv * p.R() * 4;
+  if (kErrBytes + stats > kScratchBytes) return STLITE_EUNSUPPORTED;  // beyond the fixed scratch
+  void* base = nullptr;
+  if (scratch_address(&base) != cudaSuccess) return STLITE_ECUDA;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  uint32_t* err = static_cast<uint32_t*>(base);
+  float2* rowpart = reinterpret_cast<float2*>(static_cast<unsigned char*>(base) + kErrBytes);
+  if (cudaMemsetAsync(err, 0, sizeof(uint32_t), st) != cudaSuccess) return STLITE_ECUDA;
+  cudaError_t e = p.dtype == kBF16 ? launch_score_umma(p, q, k, rowpart, plan.nsplit, a_base, err, st)
+                                   : launch_score(p, q, k, rowpart, plan.nsplit, a_base, err, st);
+  return e == cudaSuccess ? STLITE_OK : STLITE_ECUDA;
+}

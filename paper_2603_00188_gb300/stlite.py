@@ -27,7 +27,7 @@ MAX_FRAMES = 256
 EXPORTED = ("stlite_budget", "stlite_workspace_size", "stlite_score", "stlite_gate_frames",
             "stlite_spatial_saliency", "stlite_select_topk", "stlite_compact",
             "stlite_compress_layer", "stlite_device_status", "stlite_timing_enable", "stlite_timing_read",
-            "stlite_status_string")
+            "stlite_status_string", "stlite_score_noalloc")
 
 
 class Shape(ctypes.Structure):
@@ -70,6 +70,7 @@ _sig = {
     "stlite_timing_enable": (_S, [ctypes.c_int32]),
     "stlite_timing_read": (_S, [ctypes.POINTER(KernelTime), ctypes.c_int32, ctypes.POINTER(ctypes.c_int32)]),
     "stlite_status_string": (ctypes.c_char_p, [ctypes.c_int32]),
+    "stlite_score_noalloc": (_S, [ctypes.POINTER(Shape), _P, _P, _P, _P]),
 }
 for _name, (_res, _args) in _sig.items():
     _f = getattr(_lib, _name)
@@ -199,6 +200,14 @@ def stlite_device_status(ws, stream=None) -> int:
     st = ctypes.c_int32(0)
     _check(_lib.stlite_device_status(_ptr(ws), _stream(stream), ctypes.byref(st)), "stlite_device_status")
     return int(st.value)
+
+
+def stlite_score_noalloc(q, k, a_base, stream=None):
+    """Window score without a workspace (for callers that cannot allocate
+    device memory); see include/stlite.h."""
+    sh = make_shape(q, k)
+    _check(_lib.stlite_score_noalloc(ctypes.byref(sh), _ptr(q), _ptr(k), _ptr(a_base), _stream(stream)),
+           "stlite_score_noalloc")
 
 
 def stlite_timing_enable(on: bool = True):
