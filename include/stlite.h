@@ -179,6 +179,30 @@ STLITE_API stlite_status stlite_compress_layer(const stlite_shape* shape, const 
 STLITE_API stlite_status stlite_score_noalloc(const stlite_shape* shape, const void* q, const void* k,
                                               float* a_base, void* stream);
 
+/* One layer's tensors for stlite_compress_layers (all device pointers, laid
+ * out as for stlite_compress_layer). */
+typedef struct {
+  const void* q;    /* [w][Hq][d] window queries of this layer */
+  const void* k;    /* [N][Hkv][d] */
+  const void* v;    /* [N][Hkv][d] */
+  void* k_out;      /* [B][Hkv][d] */
+  void* v_out;      /* [B][Hkv][d] */
+  int32_t* idx_out; /* [Hkv][B], ascending per head */
+} stlite_layer_io;
+
+/* Algorithm 1 for n_layers layers of one sequence (one frame layout, one
+ * budget), each layer compressed independently with its own window queries;
+ * the result for every layer equals stlite_compress_layer's.  Every step
+ * runs as one launch covering up to 32 layers at a time, so small per-layer
+ * stages (the selections, the compaction) fill the GPU.  layers: HOST array
+ * [n_layers].  ws: n_layers times stlite_workspace_size() bytes (layer l uses
+ * the l-th slice; the first word of the whole workspace is the error word).
+ * budget_out (nullable, HOST) receives B. */
+STLITE_API stlite_status stlite_compress_layers(const stlite_shape* shape, const stlite_frames* frames,
+                                                const stlite_params* params, int32_t n_layers,
+                                                const stlite_layer_io* layers, int32_t* budget_out,
+                                                void* ws, size_t ws_bytes, void* stream);
+
 /* Reads and clears the workspace's device error word (synchronises `stream`).
  * *status receives STLITE_OK or the first error a kernel recorded since the
  * last read (STLITE_ETIMEOUT). */

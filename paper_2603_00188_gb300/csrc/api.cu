@@ -34,6 +34,7 @@ stlite_status check_shape(const stlite_shape* s) {
   if (R > 512) return STLITE_EUNSUPPORTED;
   if ((long long)s->n_tokens * s->n_kv_heads > (1LL << 30)) return STLITE_EUNSUPPORTED;
   if (s->n_tokens > select_max_tokens()) return STLITE_EUNSUPPORTED;
+  if (s->n_kv_heads > 4096) return STLITE_EUNSUPPORTED;
   return STLITE_OK;
 }
 
@@ -75,13 +76,14 @@ stlite_status check_params(const stlite_params* pr) {
   return STLITE_OK;
 }
 
-Problem to_problem(const stlite_shape* s) {
+Problem to_problem(const stlite_shape* s, int L) {
   Problem p;
   p.n = s->n_tokens;
   p.hq = s->n_q_heads;
   p.hkv = s->n_kv_heads;
   p.w = s->window;
   p.dtype = s->dtype == STLITE_BF16 ? kBF16 : kF32;
+  p.L = L;
   return p;
 }
 
@@ -93,19 +95,13 @@ stlite_status cuda_status(cudaError_t e) { return e == cudaSuccess ? STLITE_OK :
 
 namespace stl {
 
-// Workspace regions, each 256-byte aligned.
+// One layer's workspace region; regions of consecutive layers follow each
+// other.  Every buffer is 256-byte aligned.
 WsPlan plan_workspace(const Problem& p, const FrameTable& ft) {
   WsPlan w;
   const size_t hn = (size_t)p.hkv * p.n;
-  if (use_tensor_cores(p)) {
-    w.nsplit = umma_score_nsplit(p);
-    w.nchunk = ft.n_frames >= 2 ? (ft.cur_len + 255) / 256 : 1;  // 256-column slices
-  } else {
-    int per_head = (304 + p.hkv - 1) / p.hkv;
-    int max_split = (p.n + 63) / 64;
-    w.nsplit = per_head < max_split ? per_head : max_split;
-    w.nchunk = 1;
-  }
+  w.nsplit = score_nsplit_max(p);
+  w.nchunk = use_tensor_cores(p) && ft.n_frames >= 2 ? (ft.cur_len + 255) / 256 : 1;
   if (w.nchunk < 1) w.nchunk = 1;
   size_t o = 0;
   auto take = [&](size_t bytes) {
@@ -176,6 +172,8 @@ TimingScope::~TimingScope() {
 
 namespace {
 
+// One launch context: a batch of L (<= kMaxLayers) layers whose workspace
+// regions start at `ws`.
 struct Ctx {
   Problem p;
   FrameTable ft;
@@ -184,43 +182,91 @@ struct Ctx {
   uint32_t* err;
   cudaStream_t st;
   template <typename T>
-  T* at(size_t off) const {
-    return reinterpret_cast<T*>(ws + off);
+  Strided<T> view(size_t off) const {
+    return strided(reinterpret_cast<T*>(ws + off), plan.total);
   }
 };
 
-stlite_status prepare(const stlite_shape* shape, const stlite_frames* frames, void* ws,
-                      size_t ws_bytes, void* stream, Ctx* c) {
+stlite_status prepare(const stlite_shape* shape, const stlite_frames* frames, void* ws, size_t ws_bytes,
+                      int n_layers, void* stream, Ctx* c) {
   stlite_status s = check_shape(shape);
   if (s != STLITE_OK) return s;
   stlite_frames none = {0, nullptr, nullptr, nullptr};
   if ((s = build_frames(shape, frames ? frames : &none, &c->ft)) != STLITE_OK) return s;
-  c->p = to_problem(shape);
+  c->p = to_problem(shape, 1);
   c->plan = plan_workspace(c->p, c->ft);
   if (!ws || !aligned16(ws)) return STLITE_EINVAL;
-  if (ws_bytes < c->plan.total) return STLITE_EWORKSPACE;
+  if (ws_bytes / (size_t)n_layers < c->plan.total) return STLITE_EWORKSPACE;
   c->ws = static_cast<uint8_t*>(ws);
-  c->err = c->at<uint32_t>(c->plan.err);
+  c->err = reinterpret_cast<uint32_t*>(c->ws + c->plan.err);
   c->st = static_cast<cudaStream_t>(stream);
   return STLITE_OK;
 }
 
-cudaError_t run_norms(const Ctx& c, const void* k) {
-  return launch_inv_norms(c.p, k, c.at<float>(c.plan.rn), c.st);
+LayerPtrs single_layer(const void* q, const void* k, const void* v, void* ko, void* vo, int32_t* idx) {
+  LayerPtrs io;
+  memset(&io, 0, sizeof(io));
+  io.q[0] = q;
+  io.k[0] = k;
+  io.v[0] = v;
+  io.k_out[0] = ko;
+  io.v_out[0] = vo;
+  io.idx[0] = idx;
+  return io;
 }
 
-cudaError_t run_score(const Ctx& c, const void* q, const void* k, float* a_base) {
-  float2* rp = c.at<float2>(c.plan.rowpart);
-  if (use_tensor_cores(c.p)) return launch_score_umma(c.p, q, k, rp, c.plan.nsplit, a_base, c.err, c.st);
-  return launch_score(c.p, q, k, rp, c.plan.nsplit, a_base, c.err, c.st);
+template <typename T>
+Strided<T> one(T* p) {
+  return strided(p, 0);
 }
 
-cudaError_t run_tsg(const Ctx& c, const void* k) {
-  float* rp = c.at<float>(c.plan.rho_part);
-  const float* rn = c.at<float>(c.plan.rn);
-  if (use_tensor_cores(c.p))
-    return launch_tsg_umma(c.p, c.ft, k, rn, rp, umma_tsg_nchunk(c.ft), c.err, c.st);
-  return launch_tsg(c.p, c.ft, k, rn, rp, 1, c.err, c.st);
+cudaError_t run_score(const Ctx& c, const LayerPtrs& io, Strided<float> a_base) {
+  Strided<float2> rp = c.view<float2>(c.plan.rowpart);
+  const int ns = score_nsplit(c.p);
+  if (use_tensor_cores(c.p)) return launch_score_umma(c.p, io, rp, ns, a_base, c.err, c.st);
+  return launch_score(c.p, io, rp, ns, a_base, c.err, c.st);
+}
+
+cudaError_t run_tsg(const Ctx& c, const LayerPtrs& io) {
+  Strided<const float> rn = c.view<const float>(c.plan.rn);
+  Strided<float> rp = c.view<float>(c.plan.rho_part);
+  if (use_tensor_cores(c.p)) return launch_tsg_umma(c.p, c.ft, io, rn, rp, c.err, c.st);
+  return launch_tsg(c.p, c.ft, io, rn, rp, c.err, c.st);
+}
+
+// Algorithm 1 for a batch of layers (steps 1-5), every stage one launch.
+stlite_status compress_batch(const Ctx& c, const stlite_params* params, const LayerPtrs& io, int32_t budget) {
+  const bool tsg = params->tsg_enable && c.ft.n_frames >= 2;
+  Strided<float> a_base = c.view<float>(c.plan.a_base);
+  Strided<float> phi = c.view<float>(c.plan.phi);
+  // CSS also produces the inverse key norms TSG needs; without CSS a plain
+  // norms pass provides them.
+  cudaError_t e = cudaSuccess;
+  if (params->css_enable)
+    e = launch_css(c.p, c.ft, io, phi, c.view<float>(c.plan.rn), c.st);
+  else if (tsg)
+    e = launch_inv_norms(c.p, io, c.view<float>(c.plan.rn), c.st);
+  if (e == cudaSuccess && tsg) e = run_tsg(c, io);
+  if (e == cudaSuccess) e = run_score(c, io, a_base);
+  if (e != cudaSuccess) return STLITE_ECUDA;
+  SelectArgs a = {};
+  a.mode = (tsg ? kSelGate : 0) | kSelTopk;
+  a.budget = budget;
+  a.nchunk = c.plan.nchunk;
+  a.tsg_enable = tsg ? 1 : 0;
+  a.css_enable = params->css_enable ? 1 : 0;
+  a.alpha = params->alpha;
+  a.rho_part = c.view<const float>(c.plan.rho_part);
+  a.rn = c.view<const float>(c.plan.rn);
+  a.rho = c.view<float>(c.plan.rho);
+  a.tau = c.view<float>(c.plan.tau);
+  a.gate = tsg ? c.view<uint8_t>(c.plan.gate) : strided<uint8_t>(nullptr, 0);
+  a.a_base = c.view<const float>(c.plan.a_base);
+  a.phi = params->css_enable ? c.view<const float>(c.plan.phi) : strided<const float>(nullptr, 0);
+  a.score = c.view<float>(c.plan.score);
+  for (int l = 0; l < c.p.L; ++l) a.idx[l] = io.idx[l];
+  if ((e = launch_select(c.p, c.ft, a, c.st)) != cudaSuccess) return STLITE_ECUDA;
+  return cuda_status(launch_gather(c.p, budget, io, c.st));
 }
 
 }  // namespace
@@ -246,42 +292,43 @@ stlite_status stlite_workspace_size(const stlite_shape* shape, const stlite_fram
   stlite_frames none = {0, nullptr, nullptr, nullptr};
   FrameTable ft;
   if ((s = build_frames(shape, frames ? frames : &none, &ft)) != STLITE_OK) return s;
-  *bytes = plan_workspace(to_problem(shape), ft).total;
+  *bytes = plan_workspace(to_problem(shape, 1), ft).total;
   return STLITE_OK;
 }
 
 stlite_status stlite_score(const stlite_shape* shape, const void* q, const void* k, float* a_base,
                            void* ws, size_t ws_bytes, void* stream) {
   Ctx c;
-  stlite_status s = prepare(shape, nullptr, ws, ws_bytes, stream, &c);
+  stlite_status s = prepare(shape, nullptr, ws, ws_bytes, 1, stream, &c);
   if (s != STLITE_OK) return s;
   if (!q || !k || !a_base || !aligned16(q) || !aligned16(k) || !aligned16(a_base)) return STLITE_EINVAL;
-  return cuda_status(run_score(c, q, k, a_base));
+  return cuda_status(run_score(c, single_layer(q, k, nullptr, nullptr, nullptr, nullptr), one(a_base)));
 }
 
 stlite_status stlite_gate_frames(const stlite_shape* shape, const stlite_frames* frames,
                                  const void* k, int32_t budget, float* rho, float* tau,
                                  uint8_t* gate, void* ws, size_t ws_bytes, void* stream) {
   Ctx c;
-  stlite_status s = prepare(shape, frames, ws, ws_bytes, stream, &c);
+  stlite_status s = prepare(shape, frames, ws, ws_bytes, 1, stream, &c);
   if (s != STLITE_OK) return s;
   if (!k || !rho || !tau || !gate || !aligned16(k) || !aligned16(rho) || !aligned16(tau) ||
       !aligned16(gate))
     return STLITE_EINVAL;
   if (budget < 1 || budget > c.p.n) return STLITE_EINVAL;
-  cudaError_t e = run_norms(c, k);
-  if (e == cudaSuccess) e = run_tsg(c, k);
+  const LayerPtrs io = single_layer(nullptr, k, nullptr, nullptr, nullptr, nullptr);
+  cudaError_t e = launch_inv_norms(c.p, io, c.view<float>(c.plan.rn), c.st);
+  if (e == cudaSuccess) e = run_tsg(c, io);
   if (e != cudaSuccess) return STLITE_ECUDA;
   SelectArgs a = {};
   a.mode = kSelGate;
   a.budget = budget;
   a.nchunk = c.plan.nchunk;
   a.tsg_enable = 1;
-  a.rho_part = c.at<float>(c.plan.rho_part);
-  a.rn = c.at<float>(c.plan.rn);
-  a.rho = rho;
-  a.tau = tau;
-  a.gate = gate;
+  a.rho_part = c.view<const float>(c.plan.rho_part);
+  a.rn = c.view<const float>(c.plan.rn);
+  a.rho = one(rho);
+  a.tau = one(tau);
+  a.gate = one(gate);
   return cuda_status(launch_select(c.p, c.ft, a, c.st));
 }
 
@@ -289,10 +336,11 @@ stlite_status stlite_spatial_saliency(const stlite_shape* shape, const stlite_fr
                                       const void* k, float* phi, void* ws, size_t ws_bytes,
                                       void* stream) {
   Ctx c;
-  stlite_status s = prepare(shape, frames, ws, ws_bytes, stream, &c);
+  stlite_status s = prepare(shape, frames, ws, ws_bytes, 1, stream, &c);
   if (s != STLITE_OK) return s;
   if (!k || !phi || !aligned16(k) || !aligned16(phi)) return STLITE_EINVAL;
-  cudaError_t e = launch_css(c.p, c.ft, k, phi, c.at<float>(c.plan.rn), c.st);
+  const LayerPtrs io = single_layer(nullptr, k, nullptr, nullptr, nullptr, nullptr);
+  cudaError_t e = launch_css(c.p, c.ft, io, one(phi), c.view<float>(c.plan.rn), c.st);
   if (e == cudaSuccess) e = launch_fill_text_nan(c.p, c.ft, phi, c.st);
   return cuda_status(e);
 }
@@ -303,7 +351,7 @@ stlite_status stlite_select_topk(const stlite_shape* shape, const stlite_frames*
                                  int32_t* idx, float* score_out, void* ws, size_t ws_bytes,
                                  void* stream) {
   Ctx c;
-  stlite_status s = prepare(shape, frames, ws, ws_bytes, stream, &c);
+  stlite_status s = prepare(shape, frames, ws, ws_bytes, 1, stream, &c);
   if (s != STLITE_OK) return s;
   if ((s = check_params(params)) != STLITE_OK) return s;
   if (!a_base || !idx || !aligned16(a_base) || !aligned16(idx)) return STLITE_EINVAL;
@@ -315,11 +363,11 @@ stlite_status stlite_select_topk(const stlite_shape* shape, const stlite_frames*
   a.budget = budget;
   a.css_enable = params->css_enable ? 1 : 0;
   a.alpha = params->alpha;
-  a.a_base = a_base;
-  a.phi = params->css_enable ? phi : nullptr;
-  a.gate = const_cast<uint8_t*>(gate);
-  a.score = score_out ? score_out : c.at<float>(c.plan.score);
-  a.idx = idx;
+  a.a_base = one(a_base);
+  a.phi = params->css_enable ? one(phi) : strided<const float>(nullptr, 0);
+  a.gate = one(const_cast<uint8_t*>(gate));
+  a.score = score_out ? one(score_out) : c.view<float>(c.plan.score);
+  a.idx[0] = idx;
   return cuda_status(launch_select(c.p, c.ft, a, c.st));
 }
 
@@ -332,9 +380,9 @@ stlite_status stlite_compact(const stlite_shape* shape, int32_t budget, const in
   if (!aligned16(idx) || !aligned16(k) || !aligned16(v) || !aligned16(k_out) || !aligned16(v_out))
     return STLITE_EINVAL;
   if (budget < 1 || budget > shape->n_tokens) return STLITE_EINVAL;
-  Problem p = to_problem(shape);
-  return cuda_status(
-      launch_gather(p, budget, idx, k, v, k_out, v_out, static_cast<cudaStream_t>(stream)));
+  const Problem p = to_problem(shape, 1);
+  const LayerPtrs io = single_layer(nullptr, k, v, k_out, v_out, const_cast<int32_t*>(idx));
+  return cuda_status(launch_gather(p, budget, io, static_cast<cudaStream_t>(stream)));
 }
 
 stlite_status stlite_compress_layer(const stlite_shape* shape, const stlite_frames* frames,
@@ -342,48 +390,49 @@ stlite_status stlite_compress_layer(const stlite_shape* shape, const stlite_fram
                                     const void* v, void* k_out, void* v_out, int32_t* idx_out,
                                     int32_t* budget_out, void* ws, size_t ws_bytes,
                                     void* stream) {
+  stlite_layer_io io = {q, k, v, k_out, v_out, idx_out};
+  return stlite_compress_layers(shape, frames, params, 1, &io, budget_out, ws, ws_bytes, stream);
+}
+
+stlite_status stlite_compress_layers(const stlite_shape* shape, const stlite_frames* frames,
+                                     const stlite_params* params, int32_t n_layers,
+                                     const stlite_layer_io* layers, int32_t* budget_out, void* ws,
+                                     size_t ws_bytes, void* stream) {
+  if (n_layers < 1 || !layers) return STLITE_EINVAL;
   Ctx c;
-  stlite_status s = prepare(shape, frames, ws, ws_bytes, stream, &c);
+  stlite_status s = prepare(shape, frames, ws, ws_bytes, n_layers, stream, &c);
   if (s != STLITE_OK) return s;
   if ((s = check_params(params)) != STLITE_OK) return s;
-  if (!q || !k || !v || !k_out || !v_out || !idx_out) return STLITE_EINVAL;
-  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(k_out) || !aligned16(v_out) ||
-      !aligned16(idx_out))
-    return STLITE_EINVAL;
+  for (int l = 0; l < n_layers; ++l) {
+    const stlite_layer_io& x = layers[l];
+    if (!x.q || !x.k || !x.v || !x.k_out || !x.v_out || !x.idx_out) return STLITE_EINVAL;
+    if (!aligned16(x.q) || !aligned16(x.k) || !aligned16(x.v) || !aligned16(x.k_out) ||
+        !aligned16(x.v_out) || !aligned16(x.idx_out))
+      return STLITE_EINVAL;
+  }
   const int32_t budget = stlite_budget(c.p.n, params->beta, params->k_override);
   if (budget < 1) return STLITE_EINVAL;
   if (budget_out) *budget_out = budget;
-  const bool tsg = params->tsg_enable && c.ft.n_frames >= 2;
-  float* a_base = c.at<float>(c.plan.a_base);
-  float* phi = c.at<float>(c.plan.phi);
-  // CSS also produces the inverse key norms TSG needs; without CSS a plain
-  // norms pass provides them.
-  cudaError_t e = cudaSuccess;
-  if (params->css_enable)
-    e = launch_css(c.p, c.ft, k, phi, c.at<float>(c.plan.rn), c.st);
-  else if (tsg)
-    e = run_norms(c, k);
-  if (e == cudaSuccess && tsg) e = run_tsg(c, k);
-  if (e == cudaSuccess) e = run_score(c, q, k, a_base);
-  if (e != cudaSuccess) return STLITE_ECUDA;
-  SelectArgs a = {};
-  a.mode = (tsg ? kSelGate : 0) | kSelTopk;
-  a.budget = budget;
-  a.nchunk = c.plan.nchunk;
-  a.tsg_enable = tsg ? 1 : 0;
-  a.css_enable = params->css_enable ? 1 : 0;
-  a.alpha = params->alpha;
-  a.rho_part = c.at<float>(c.plan.rho_part);
-  a.rn = c.at<float>(c.plan.rn);
-  a.rho = c.at<float>(c.plan.rho);
-  a.tau = c.at<float>(c.plan.tau);
-  a.gate = tsg ? c.at<uint8_t>(c.plan.gate) : nullptr;
-  a.a_base = a_base;
-  a.phi = params->css_enable ? phi : nullptr;
-  a.score = c.at<float>(c.plan.score);
-  a.idx = idx_out;
-  if ((e = launch_select(c.p, c.ft, a, c.st)) != cudaSuccess) return STLITE_ECUDA;
-  return cuda_status(launch_gather(c.p, budget, idx_out, k, v, k_out, v_out, c.st));
+  // one launch per stage for up to kMaxLayers layers at a time
+  for (int l0 = 0; l0 < n_layers; l0 += kMaxLayers) {
+    const int L = n_layers - l0 < kMaxLayers ? n_layers - l0 : kMaxLayers;
+    Ctx cb = c;
+    cb.p.L = L;
+    cb.ws = c.ws + (size_t)l0 * c.plan.total;
+    LayerPtrs io;
+    memset(&io, 0, sizeof(io));
+    for (int l = 0; l < L; ++l) {
+      const stlite_layer_io& x = layers[l0 + l];
+      io.q[l] = x.q;
+      io.k[l] = x.k;
+      io.v[l] = x.v;
+      io.k_out[l] = x.k_out;
+      io.v_out[l] = x.v_out;
+      io.idx[l] = x.idx_out;
+    }
+    if ((s = compress_batch(cb, params, io, budget)) != STLITE_OK) return s;
+  }
+  return STLITE_OK;
 }
 
 stlite_status stlite_device_status(void* ws, void* stream, stlite_status* status) {

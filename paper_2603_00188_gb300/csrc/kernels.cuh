@@ -1,5 +1,8 @@
 // Internal launch interface between the C ABI (api.cu) and the kernels.
-// Every launcher enqueues on `st` and returns the launch status.
+// Every launcher enqueues on `st` and returns the launch status.  A launch
+// covers a batch of L layers that share one frame layout (the layers of one
+// model on one sequence); per-layer tensors are reached through LayerPtrs
+// and per-layer workspace buffers through Strided views.
 #pragma once
 
 #include <cuda.h>
@@ -12,21 +15,51 @@ namespace stl {
 
 enum DType { kBF16 = 0, kF32 = 1 };
 
+constexpr int kMaxLayers = 32;  // layers per launch
+
 struct Problem {
   int n;       // tokens
   int hq;      // query heads
   int hkv;     // KV heads
   int w;       // window queries
   int dtype;   // DType
+  int L;       // layers in the launch
   __host__ __device__ int G() const { return hq / hkv; }
   __host__ __device__ int R() const { return w * (hq / hkv); }  // query rows per KV head
 };
 
-// ---- workspace plan (byte offsets into the caller's workspace) ----------
+// Per-layer device tensors of one launch.
+struct LayerPtrs {
+  const void* q[kMaxLayers];
+  const void* k[kMaxLayers];
+  const void* v[kMaxLayers];
+  void* k_out[kMaxLayers];
+  void* v_out[kMaxLayers];
+  int32_t* idx[kMaxLayers];
+};
+
+// A per-layer buffer: layer l starts `stride` bytes after layer l-1.
+template <typename T>
+struct Strided {
+  T* base;
+  size_t stride;
+  __host__ __device__ T* at(int l) const {
+    return reinterpret_cast<T*>(reinterpret_cast<uintptr_t>(base) + (size_t)l * stride);
+  }
+};
+template <typename T>
+inline Strided<T> strided(T* base, size_t stride) {
+  Strided<T> s;
+  s.base = base;
+  s.stride = stride;
+  return s;
+}
+
+// ---- workspace plan (byte offsets into one layer's workspace region) ------
 struct WsPlan {
-  size_t err;        // uint32 error word
+  size_t err;        // uint32 error word (layer 0's is the one used)
   size_t rn;         // float [Hkv][N] inverse key norms
-  size_t rowpart;    // float2 [Hkv][nsplit][R] partial (max, sum) per query row
+  size_t rowpart;    // float2 [Hkv][nsplit][R] per-split (max, sum) per query row, then float [Hkv][R]
   size_t a_base;     // float [Hkv][N]
   size_t phi;        // float [Hkv][N]
   size_t rho;        // float [Hkv][N]
@@ -34,9 +67,9 @@ struct WsPlan {
   size_t tau;        // float [Hkv]
   size_t gate;       // uint8 [Hkv][N]
   size_t score;      // float [Hkv][N]
-  size_t total;
-  int nsplit;        // key splits of the row-statistics pass
-  int nchunk;        // current-frame column chunks of the TSG pass
+  size_t total;      // bytes of one layer's region
+  int nsplit;        // largest key-split count of the row-statistics pass
+  int nchunk;        // 256-column slices of rho_part
 };
 WsPlan plan_workspace(const Problem& p, const FrameTable& ft);
 
@@ -58,29 +91,36 @@ class TimingScope {
 };
 
 // ---- launchers ----------------------------------------------------------
-cudaError_t launch_inv_norms(const Problem& p, const void* k, float* rn, cudaStream_t st);
+// rn[l][h][j] = 1 / max(|k_l[j,h]|, 1e-8) for every token.
+cudaError_t launch_inv_norms(const Problem& p, const LayerPtrs& io, Strided<float> rn, cudaStream_t st);
 
-// bias[h][r] = -m_r - log2(G l_r) from the per-split row statistics.
-cudaError_t launch_row_bias(const Problem& p, const float2* part, int nsplit, float* bias,
+// Window score (Eq. 2): row statistics then column sums.  rowpart holds, per
+// layer, [Hkv][nsplit][R] float2 followed by [Hkv][R] float (row bias).
+cudaError_t launch_score(const Problem& p, const LayerPtrs& io, Strided<float2> rowpart, int nsplit,
+                         Strided<float> a_base, uint32_t* err, cudaStream_t st);
+cudaError_t launch_score_umma(const Problem& p, const LayerPtrs& io, Strided<float2> rowpart,
+                              int nsplit, Strided<float> a_base, uint32_t* err, cudaStream_t st);
+// Key splits of window-score pass 1 for this batch, and the largest value it
+// takes for any batch size (which sizes the workspace).
+int score_nsplit(const Problem& p);
+int score_nsplit_max(const Problem& p);
+
+// TSG partial row maxima: rho_part[l][s][h][i] = max over the current-frame
+// columns of 256-column slice s of k_i.k_j * rn_j, for historical visual
+// tokens i (Eq. 6 before the 1/|k_i| factor).
+cudaError_t launch_tsg(const Problem& p, const FrameTable& ft, const LayerPtrs& io,
+                       Strided<const float> rn, Strided<float> rho_part, uint32_t* err,
+                       cudaStream_t st);
+cudaError_t launch_tsg_umma(const Problem& p, const FrameTable& ft, const LayerPtrs& io,
+                            Strided<const float> rn, Strided<float> rho_part, uint32_t* err,
                             cudaStream_t st);
 
-// Window score: row statistics then column sums (Eq. 2).
-cudaError_t launch_score(const Problem& p, const void* q, const void* k, float2* rowpart,
-                         int nsplit, float* a_base, uint32_t* err, cudaStream_t st);
-
-// TSG partial row maxima: rho_part[c][h][i] = max_{j in chunk c} k_i.k_j * rn_j
-// for historical visual tokens i (Eq. 6 before the 1/|k_i| factor).
-cudaError_t launch_tsg(const Problem& p, const FrameTable& ft, const void* k, const float* rn,
-                       float* rho_part, int nchunk, uint32_t* err, cudaStream_t st);
-
-// CSS saliency Phi (Eqs. 4-5) of every visual token; also writes the
-// inverse key norms rn of every visual token.  Text entries are not touched.
-cudaError_t launch_css(const Problem& p, const FrameTable& ft, const void* k, float* phi, float* rn,
-                       cudaStream_t st);
-// phi[h][j] = NaN for every text token j.
+// CSS saliency Phi (Eqs. 4-5) of every visual token; also writes the inverse
+// key norms rn of every visual token.  Text entries are not touched.
+cudaError_t launch_css(const Problem& p, const FrameTable& ft, const LayerPtrs& io,
+                       Strided<float> phi, Strided<float> rn, cudaStream_t st);
+// phi[h][j] = NaN for every text token j (one layer).
 cudaError_t launch_fill_text_nan(const Problem& p, const FrameTable& ft, float* phi, cudaStream_t st);
-// Largest N the selection kernel handles.
-int select_max_tokens();
 
 // Selection: mode bit 1 = finish rho, tau and gate (Eqs. 6-8); mode bit 2 =
 // integrated score and top-B (Eq. 9, Sec. 2.1).
@@ -93,30 +133,23 @@ struct SelectArgs {
   int tsg_enable;
   int css_enable;
   float alpha;
-  const float* rho_part;  // [nchunk][Hkv][N]
-  const float* rn;        // [Hkv][N]
-  float* rho;             // out [Hkv][N]
-  float* tau;             // out [Hkv]
-  uint8_t* gate;          // out (kSelGate) / in (kSelTopk, nullable) [Hkv][N]
-  const float* a_base;    // [Hkv][N]
-  const float* phi;       // [Hkv][N] (nullable if !css_enable)
-  float* score;           // out [Hkv][N]
-  int32_t* idx;           // out [Hkv][budget]
+  Strided<const float> rho_part;  // [nchunk][Hkv][N]
+  Strided<const float> rn;        // [Hkv][N]
+  Strided<float> rho;             // out [Hkv][N]
+  Strided<float> tau;             // out [Hkv]
+  Strided<uint8_t> gate;          // out (kSelGate) / in (kSelTopk; null base = all ones)
+  Strided<const float> a_base;    // [Hkv][N]
+  Strided<const float> phi;       // [Hkv][N] (null base when !css_enable)
+  Strided<float> score;           // out [Hkv][N]
+  int32_t* idx[kMaxLayers];       // out per layer [Hkv][budget]
 };
 cudaError_t launch_select(const Problem& p, const FrameTable& ft, const SelectArgs& a,
                           cudaStream_t st);
+// Largest N the selection kernel handles.
+int select_max_tokens();
 
-cudaError_t launch_gather(const Problem& p, int budget, const int32_t* idx, const void* k,
-                          const void* v, void* k_out, void* v_out, cudaStream_t st);
-
-// Tensor-core (tcgen05) paths for bf16; return cudaErrorNotSupported when the
-// shape is outside what they handle.
-cudaError_t launch_score_umma(const Problem& p, const void* q, const void* k, float2* rowpart,
-                              int nsplit, float* a_base, uint32_t* err, cudaStream_t st);
-cudaError_t launch_tsg_umma(const Problem& p, const FrameTable& ft, const void* k,
-                            const float* rn, float* rho_part, int nchunk, uint32_t* err,
-                            cudaStream_t st);
-int umma_score_nsplit(const Problem& p);
-int umma_tsg_nchunk(const FrameTable& ft);
+// k_out[l][r][h][:] = k_l[idx[l][h][r]][h][:] and the same for v (idx, k,
+// v, k_out, v_out from io).
+cudaError_t launch_gather(const Problem& p, int budget, const LayerPtrs& io, cudaStream_t st);
 
 }  // namespace stl

@@ -62,6 +62,7 @@ extern "C" stlite_status stlite_score_noalloc(const stlite_shape* s, const void*
   p.hkv = s->n_kv_heads;
   p.w = s->window;
   p.dtype = s->dtype == STLITE_BF16 ? kBF16 : kF32;
+  p.L = 1;
   FrameTable ft = {};
   ft.n_tokens = p.n;
   const WsPlan plan = plan_workspace(p, ft);
@@ -73,7 +74,13 @@ extern "C" stlite_status stlite_score_noalloc(const stlite_shape* s, const void*
   uint32_t* err = static_cast<uint32_t*>(base);
   float2* rowpart = reinterpret_cast<float2*>(static_cast<unsigned char*>(base) + kErrBytes);
   if (cudaMemsetAsync(err, 0, sizeof(uint32_t), st) != cudaSuccess) return STLITE_ECUDA;
-  cudaError_t e = p.dtype == kBF16 ? launch_score_umma(p, q, k, rowpart, plan.nsplit, a_base, err, st)
-                                   : launch_score(p, q, k, rowpart, plan.nsplit, a_base, err, st);
+  LayerPtrs io = {};
+  io.q[0] = q;
+  io.k[0] = k;
+  const int nsplit = score_nsplit(p);
+  const Strided<float2> parts = strided(rowpart, 0);
+  const Strided<float> out = strided(a_base, 0);
+  cudaError_t e = p.dtype == kBF16 ? launch_score_umma(p, io, parts, nsplit, out, err, st)
+                                   : launch_score(p, io, parts, nsplit, out, err, st);
   return e == cudaSuccess ? STLITE_OK : STLITE_ECUDA;
 }

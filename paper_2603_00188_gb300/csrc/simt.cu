@@ -1,15 +1,16 @@
 // CUDA-core kernels: inverse key norms, CSS saliency, and the fp32 versions
 // of window scoring and TSG (fp32 inputs cannot use the bf16 tensor-core
-// path without losing the exactness of the products).
+// path without losing the exactness of the products).  Every kernel covers a
+// batch of layers: the layer index is the high part of one grid dimension.
 #include "kernels.cuh"
 
 namespace stl {
 
 constexpr float kLog2e = 1.4426950408889634f;
 
-// ---------------------------------------------------------------- norms
-// (unpack16 is shared with the CSS kernel so that both compute a norm with
-// the same sequence of operations: fmaf over elements 0..127 in order.)
+// 16 bytes of keys -> floats (8 bf16 or 4 fp32).  Shared by the norm and CSS
+// kernels, so that both compute a key's norm with the same sequence of
+// operations (fmaf over elements 0..127 in order) and agree bit for bit.
 template <typename T>
 __device__ __forceinline__ void unpack16(const uint4& w, float (&f)[16 / sizeof(T)]) {
   if constexpr (sizeof(T) == 2) {
@@ -29,12 +30,17 @@ __device__ __forceinline__ void unpack16(const uint4& w, float (&f)[16 / sizeof(
   }
 }
 
-// rn[h][j] = 1 / max(|k_{j,h}|, 1e-8), one thread per (token, head) row.
+// ---------------------------------------------------------------- norms
+// rn[l][h][j] = 1 / max(|k_l[j,h]|, 1e-8); one thread per (token, head) row,
+// grid.y = layer.
 template <typename T>
-__global__ void __launch_bounds__(256) k_inv_norms(const T* __restrict__ k, int n, int hkv,
-                                                   float* __restrict__ rn) {
+__global__ void __launch_bounds__(256) k_inv_norms(const __grid_constant__ LayerPtrs io, int n, int hkv,
+                                                   Strided<float> rn_all) {
   constexpr int kChunks = kD * (int)sizeof(T) / 16;
   constexpr int kPer = 16 / (int)sizeof(T);
+  const int l = blockIdx.y;
+  const T* k = static_cast<const T*>(io.k[l]);
+  float* rn = rn_all.at(l);
   const long long rows = (long long)n * hkv;
   for (long long r = (long long)blockIdx.x * blockDim.x + threadIdx.x; r < rows;
        r += (long long)gridDim.x * blockDim.x) {
@@ -55,26 +61,29 @@ __global__ void __launch_bounds__(256) k_inv_norms(const T* __restrict__ k, int 
   }
 }
 
-cudaError_t launch_inv_norms(const Problem& p, const void* k, float* rn, cudaStream_t st) {
+cudaError_t launch_inv_norms(const Problem& p, const LayerPtrs& io, Strided<float> rn, cudaStream_t st) {
   long long rows = (long long)p.n * p.hkv;
   long long blocks = (rows + 255) / 256;
-  if (blocks > 152 * 8) blocks = 152 * 8;
+  long long cap = (152 * 8 + p.L - 1) / p.L;
+  if (blocks > cap) blocks = cap;
   TimingScope ts("inv_norms", st);
+  dim3 grid((unsigned)blocks, p.L);
   if (p.dtype == kBF16)
-    k_inv_norms<<<(int)blocks, 256, 0, st>>>((const __nv_bfloat16*)k, p.n, p.hkv, rn);
+    k_inv_norms<__nv_bfloat16><<<grid, 256, 0, st>>>(io, p.n, p.hkv, rn);
   else
-    k_inv_norms<<<(int)blocks, 256, 0, st>>>((const float*)k, p.n, p.hkv, rn);
+    k_inv_norms<float><<<grid, 256, 0, st>>>(io, p.n, p.hkv, rn);
   return cudaGetLastError();
 }
 
 // ---------------------------------------------------------------- CSS
-// Eqs. 4-5 on 2-D tiles of one frame's patch grid.  A CTA (tile, frame, head)
-// stages the tile's keys plus a one-cell halo in shared memory (rows padded
-// by 16 bytes, so 8 threads reading 8 different keys hit 8 distinct bank
-// groups), computes every key's inverse norm once and every unordered
-// neighbour pair once (the E, S, SE, SW pairs of each cell), then sums the
-// eight directions of each output cell.  It also writes the inverse norms of
-// its output cells (used by TSG).
+// Eqs. 4-5 on 2-D tiles of one frame's patch grid.  A CTA (tile, frame,
+// layer*Hkv + head) stages the tile's keys plus a one-cell halo in shared
+// memory with asynchronous copies (key rows padded by 16 bytes, so 8 threads
+// reading 8 different keys hit 8 distinct bank groups).  One thread per cell
+// then computes the cell's norm and its E, S, SE, SW pair dots in one sweep,
+// so every unordered neighbour pair is computed once; finally each output
+// cell sums its eight directions.  The inverse norms of the output cells are
+// written too (TSG uses them).
 constexpr int kCssThreads = 256;
 constexpr int kCssBudget = 100 * 1024;  // shared-memory bytes per CTA
 constexpr int kCssMaxCols = 64;         // output columns per tile
@@ -99,17 +108,20 @@ struct CssGeom {
 };
 
 template <typename T>
-__global__ void __launch_bounds__(kCssThreads) k_css(const T* __restrict__ k,
+__global__ void __launch_bounds__(kCssThreads) k_css(const __grid_constant__ LayerPtrs io,
                                                      const __grid_constant__ FrameTable ft, int hkv,
-                                                     float* __restrict__ phi,
-                                                     float* __restrict__ rn_out) {
+                                                     Strided<float> phi_all, Strided<float> rn_all) {
   using Gm = CssGeom<T>;
   constexpr int kChunks = kD * (int)sizeof(T) / 16;
   constexpr int kPer = 16 / (int)sizeof(T);
   extern __shared__ float4 css_smem[];
   uint8_t* sm = reinterpret_cast<uint8_t*>(css_smem);
-  const int f = blockIdx.y, h = blockIdx.z, n = ft.n_tokens, tid = threadIdx.x;
+  const int f = blockIdx.y, l = blockIdx.z / hkv, h = blockIdx.z % hkv, n = ft.n_tokens;
+  const int tid = threadIdx.x;
   if (f >= ft.n_frames) return;
+  const T* k = static_cast<const T*>(io.k[l]);
+  float* phi = phi_all.at(l);
+  float* rn_out = rn_all.at(l);
   const int gh = ft.gh[f], gw = ft.gw[f], off = ft.off[f];
   int RB, CB;
   Gm::tile(gh, gw, RB, CB);
@@ -123,14 +135,15 @@ __global__ void __launch_bounds__(kCssThreads) k_css(const T* __restrict__ k,
   float* dS = dE + cells;
   float* dSE = dS + cells;
   float* dSW = dSE + cells;
-  // stage the tile (local cell (a, b) = grid cell (u0 - 1 + a, v0 - 1 + b))
-  // with asynchronous 16-byte copies; cells outside the grid stay unloaded
+  // stage the tile (local cell (a, b) = grid cell (u0 - 1 + a, v0 - 1 + b));
+  // cells outside the grid stay unloaded and are never read
   for (int e = tid; e < cells * kChunks; e += blockDim.x) {
     const int cell = e / kChunks, ch = e - cell * kChunks;
     const int u = u0 - 1 + cell / TW, v = v0 - 1 + cell % TW;
     if (u < 0 || u >= gh || v < 0 || v >= gw) continue;
     const T* src = k + ((size_t)(off + u * gw + v) * hkv + h) * kD + ch * kPer;
-    const uint32_t dst = static_cast<uint32_t>(__cvta_generic_to_shared(keys + (size_t)cell * Gm::kStride + 16 * ch));
+    const uint32_t dst =
+        static_cast<uint32_t>(__cvta_generic_to_shared(keys + (size_t)cell * Gm::kStride + 16 * ch));
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
   }
   asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
@@ -143,12 +156,11 @@ __global__ void __launch_bounds__(kCssThreads) k_css(const T* __restrict__ k,
     if (u < 0 || u >= gh || v < 0 || v >= gw) continue;
     const bool fwd = a <= RB && u + 1 < gh;
     const bool hasE = b + 1 < TW && v + 1 < gw;
-    const bool hasS = fwd;
     const bool hasSE = fwd && b + 1 < TW && v + 1 < gw;
     const bool hasSW = fwd && b >= 1 && v >= 1;
     const uint8_t* p0 = keys + (size_t)cell * Gm::kStride;
     const uint8_t* pE = hasE ? p0 + Gm::kStride : p0;
-    const uint8_t* pS = hasS ? p0 + (size_t)TW * Gm::kStride : p0;
+    const uint8_t* pS = fwd ? p0 + (size_t)TW * Gm::kStride : p0;
     const uint8_t* pSE = hasSE ? p0 + (size_t)(TW + 1) * Gm::kStride : p0;
     const uint8_t* pSW = hasSW ? p0 + (size_t)(TW - 1) * Gm::kStride : p0;
     float sn = 0.f, sE = 0.f, sS = 0.f, sSE = 0.f, sSW = 0.f;
@@ -211,8 +223,8 @@ __global__ void k_fill_text_nan(const __grid_constant__ FrameTable ft, int hkv, 
 }
 
 template <typename T>
-static cudaError_t css_launch_t(const Problem& p, const FrameTable& ft, const void* k, float* phi,
-                                float* rn, cudaStream_t st) {
+static cudaError_t css_launch_t(const Problem& p, const FrameTable& ft, const LayerPtrs& io,
+                                Strided<float> phi, Strided<float> rn, cudaStream_t st) {
   using Gm = CssGeom<T>;
   int tmax = 0, cmax = 0;
   for (int f = 0; f < ft.n_frames; ++f) {
@@ -226,14 +238,14 @@ static cudaError_t css_launch_t(const Problem& p, const FrameTable& ft, const vo
   cudaError_t e = cudaFuncSetAttribute(k_css<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   TimingScope ts("css", st);
-  k_css<T><<<dim3(tmax, ft.n_frames, p.hkv), kCssThreads, smem, st>>>((const T*)k, ft, p.hkv, phi, rn);
+  k_css<T><<<dim3(tmax, ft.n_frames, p.L * p.hkv), kCssThreads, smem, st>>>(io, ft, p.hkv, phi, rn);
   return cudaGetLastError();
 }
 
-cudaError_t launch_css(const Problem& p, const FrameTable& ft, const void* k, float* phi, float* rn,
-                       cudaStream_t st) {
-  if (p.dtype == kBF16) return css_launch_t<__nv_bfloat16>(p, ft, k, phi, rn, st);
-  return css_launch_t<float>(p, ft, k, phi, rn, st);
+cudaError_t launch_css(const Problem& p, const FrameTable& ft, const LayerPtrs& io, Strided<float> phi,
+                       Strided<float> rn, cudaStream_t st) {
+  if (p.dtype == kBF16) return css_launch_t<__nv_bfloat16>(p, ft, io, phi, rn, st);
+  return css_launch_t<float>(p, ft, io, phi, rn, st);
 }
 
 cudaError_t launch_fill_text_nan(const Problem& p, const FrameTable& ft, float* phi, cudaStream_t st) {
@@ -245,21 +257,24 @@ cudaError_t launch_fill_text_nan(const Problem& p, const FrameTable& ft, float* 
 }
 
 // ------------------------------------------------------- row statistics
-// Window score, first pass: for every query row r of KV head h (r = window
-// row * G + group member) the running maximum m and sum l of
+// Window score, first pass (fp32): for every query row r of KV head h (r =
+// window row * G + group member) the running maximum m and sum l of
 // 2^(x - m), x = q.k * log2(e)/sqrt(d), over the keys of one split.
+// grid = (split, layer*Hkv + head, row chunk).
 constexpr int kRsRows = 256;   // query rows per block
 constexpr int kRsKeys = 64;    // keys per smem tile
 constexpr int kRsSmem = (kRsRows * (kD + 1) + kRsKeys * kD) * 4;
 
 template <typename T>
-__global__ void __launch_bounds__(kRsRows) k_rowstats_simt(const T* __restrict__ q,
-                                                           const T* __restrict__ k, Problem p,
-                                                           int nsplit, float2* __restrict__ part) {
+__global__ void __launch_bounds__(kRsRows) k_rowstats_simt(const __grid_constant__ LayerPtrs io, Problem p,
+                                                           int nsplit, Strided<float2> part_all) {
   extern __shared__ float sm[];
   float* qs = sm;                       // [kRsRows][kD+1]
   float* ks = sm + kRsRows * (kD + 1);  // [kRsKeys][kD]
-  const int s = blockIdx.x, h = blockIdx.y, r0 = blockIdx.z * kRsRows;
+  const int s = blockIdx.x, l = blockIdx.y / p.hkv, h = blockIdx.y % p.hkv, r0 = blockIdx.z * kRsRows;
+  const T* q = static_cast<const T*>(io.q[l]);
+  const T* k = static_cast<const T*>(io.k[l]);
+  float2* part = part_all.at(l);
   const int G = p.G(), R = p.R(), tid = threadIdx.x;
   const float c = kLog2e * rsqrtf((float)kD);
   for (int e = tid; e < kRsRows * kD; e += blockDim.x) {
@@ -273,7 +288,7 @@ __global__ void __launch_bounds__(kRsRows) k_rowstats_simt(const T* __restrict__
   }
   int per = (p.n + nsplit - 1) / nsplit;
   int j0 = s * per, j1 = min(p.n, j0 + per);
-  float m = -CUDART_INF_F, l = 0.f;
+  float m = -CUDART_INF_F, lsum = 0.f;
   for (int jt = j0; jt < j1; jt += kRsKeys) {
     __syncthreads();
     for (int e = tid; e < kRsKeys * kD; e += blockDim.x) {
@@ -293,53 +308,58 @@ __global__ void __launch_bounds__(kRsRows) k_rowstats_simt(const T* __restrict__
       }
       float x = (d0 + d1) * c;
       if (x > m) {
-        l = l * exp2f(m - x) + 1.0f;
+        lsum = lsum * exp2f(m - x) + 1.0f;
         m = x;
       } else {
-        l += exp2f(x - m);
+        lsum += exp2f(x - m);
       }
     }
   }
-  if (r0 + tid < R) part[((size_t)h * nsplit + s) * R + r0 + tid] = make_float2(m, l);
+  if (r0 + tid < R) part[((size_t)h * nsplit + s) * R + r0 + tid] = make_float2(m, lsum);
 }
 
 // Merge the splits: bias[h][r] = -m_r - log2(G * l_r), so that
-// 2^(x + bias) = softmax probability / G.
-__global__ void k_row_bias(const float2* __restrict__ part, Problem p, int nsplit,
-                           float* __restrict__ bias) {
-  int R = p.R();
+// 2^(x + bias) = softmax probability / G.  grid.y = layer.
+__global__ void k_row_bias(Problem p, int nsplit, Strided<float2> part_all) {
+  const int R = p.R(), l = blockIdx.y;
+  const float2* part = part_all.at(l);
+  float* bias = reinterpret_cast<float*>(part_all.at(l) + (size_t)p.hkv * nsplit * R);
   int e = blockIdx.x * blockDim.x + threadIdx.x;
   if (e >= p.hkv * R) return;
   int h = e / R, r = e - h * R;
   const float2* pp = part + (size_t)h * nsplit * R + r;
   float m = -CUDART_INF_F;
   for (int s = 0; s < nsplit; ++s) m = fmaxf(m, pp[(size_t)s * R].x);
-  float l = 0.f;
+  float lsum = 0.f;
   for (int s = 0; s < nsplit; ++s) {
     float2 v = pp[(size_t)s * R];
-    if (v.y > 0.f) l += v.y * exp2f(v.x - m);
+    if (v.y > 0.f) lsum += v.y * exp2f(v.x - m);
   }
-  bias[e] = -m - log2f((float)p.G() * l);
+  bias[e] = -m - log2f((float)p.G() * lsum);
 }
 
 // ---------------------------------------------------------- column sums
-// Window score, second pass: a[h][j] = sum_r 2^(x_rj + bias_r).  One thread
-// per key; the key tile is kept (padded) in shared memory.
+// Window score, second pass (fp32): a[h][j] = sum_r 2^(x_rj + bias_r).  One
+// thread per key; the key tile is kept (padded) in shared memory.
+// grid = (key tile, layer*Hkv + head).
 constexpr int kCsKeys = 128;
 constexpr int kCsRows = 32;
 constexpr int kCsMaxR = 1024;
 constexpr int kCsSmem = (kCsKeys * (kD + 1) + kCsRows * kD + kCsMaxR) * 4;
 
 template <typename T>
-__global__ void __launch_bounds__(kCsKeys) k_colsum_simt(const T* __restrict__ q,
-                                                         const T* __restrict__ k, Problem p,
-                                                         const float* __restrict__ bias,
-                                                         float* __restrict__ a_base) {
+__global__ void __launch_bounds__(kCsKeys) k_colsum_simt(const __grid_constant__ LayerPtrs io, Problem p,
+                                                         int nsplit, Strided<float2> part_all,
+                                                         Strided<float> a_all) {
   extern __shared__ float sm[];
   float* ks = sm;                            // [kCsKeys][kD+1]
   float* qs = ks + kCsKeys * (kD + 1);       // [kCsRows][kD]
   float* bs = qs + kCsRows * kD;             // [R]
-  const int h = blockIdx.y, j0 = blockIdx.x * kCsKeys, tid = threadIdx.x;
+  const int l = blockIdx.y / p.hkv, h = blockIdx.y % p.hkv, j0 = blockIdx.x * kCsKeys, tid = threadIdx.x;
+  const T* q = static_cast<const T*>(io.q[l]);
+  const T* k = static_cast<const T*>(io.k[l]);
+  const float* bias = reinterpret_cast<const float*>(part_all.at(l) + (size_t)p.hkv * nsplit * p.R());
+  float* a_base = a_all.at(l);
   const int G = p.G(), R = p.R();
   const float c = kLog2e * rsqrtf((float)kD);
   for (int e = tid; e < kCsKeys * kD; e += blockDim.x) {
@@ -377,61 +397,60 @@ __global__ void __launch_bounds__(kCsKeys) k_colsum_simt(const T* __restrict__ q
   if (j0 + tid < p.n) a_base[(size_t)h * p.n + j0 + tid] = acc;
 }
 
-cudaError_t launch_row_bias(const Problem& p, const float2* part, int nsplit, float* bias,
-                            cudaStream_t st) {
-  int tot = p.hkv * p.R();
-  TimingScope ts("row_bias", st);
-  k_row_bias<<<(tot + 127) / 128, 128, 0, st>>>(part, p, nsplit, bias);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_score(const Problem& p, const void* q, const void* k, float2* rowpart,
-                         int nsplit, float* a_base, uint32_t* err, cudaStream_t st) {
+cudaError_t launch_score(const Problem& p, const LayerPtrs& io, Strided<float2> rowpart, int nsplit,
+                         Strided<float> a_base, uint32_t* err, cudaStream_t st) {
   (void)err;
+  if (p.R() > kCsMaxR) return cudaErrorNotSupported;
   cudaFuncSetAttribute(k_rowstats_simt<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, kRsSmem);
   cudaFuncSetAttribute(k_rowstats_simt<__nv_bfloat16>, cudaFuncAttributeMaxDynamicSharedMemorySize, kRsSmem);
   cudaFuncSetAttribute(k_colsum_simt<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, kCsSmem);
   cudaFuncSetAttribute(k_colsum_simt<__nv_bfloat16>, cudaFuncAttributeMaxDynamicSharedMemorySize, kCsSmem);
-  if (p.R() > kCsMaxR) return cudaErrorNotSupported;
-  dim3 g1(nsplit, p.hkv, (p.R() + kRsRows - 1) / kRsRows);
-  float* bias = reinterpret_cast<float*>(rowpart + (size_t)p.hkv * nsplit * p.R());
-  dim3 g2((p.n + kCsKeys - 1) / kCsKeys, p.hkv);
+  dim3 g1(nsplit, p.L * p.hkv, (p.R() + kRsRows - 1) / kRsRows);
+  dim3 g2((p.n + kCsKeys - 1) / kCsKeys, p.L * p.hkv);
   {
-  TimingScope ts("rowstats_simt", st);
-  if (p.dtype == kBF16) {
-    k_rowstats_simt<<<g1, kRsRows, kRsSmem, st>>>((const __nv_bfloat16*)q, (const __nv_bfloat16*)k, p, nsplit, rowpart);
-  } else {
-    k_rowstats_simt<<<g1, kRsRows, kRsSmem, st>>>((const float*)q, (const float*)k, p, nsplit, rowpart);
-  }
+    TimingScope ts("rowstats_simt", st);
+    if (p.dtype == kBF16)
+      k_rowstats_simt<__nv_bfloat16><<<g1, kRsRows, kRsSmem, st>>>(io, p, nsplit, rowpart);
+    else
+      k_rowstats_simt<float><<<g1, kRsRows, kRsSmem, st>>>(io, p, nsplit, rowpart);
   }
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  if ((e = launch_row_bias(p, rowpart, nsplit, bias, st)) != cudaSuccess) return e;
-  TimingScope ts("colsum_simt", st);
-  if (p.dtype == kBF16) {
-    k_colsum_simt<<<g2, kCsKeys, kCsSmem, st>>>((const __nv_bfloat16*)q, (const __nv_bfloat16*)k, p, bias, a_base);
-  } else {
-    k_colsum_simt<<<g2, kCsKeys, kCsSmem, st>>>((const float*)q, (const float*)k, p, bias, a_base);
+  {
+    TimingScope ts("row_bias", st);
+    int tot = p.hkv * p.R();
+    k_row_bias<<<dim3((tot + 127) / 128, p.L), 128, 0, st>>>(p, nsplit, rowpart);
   }
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  TimingScope ts("colsum_simt", st);
+  if (p.dtype == kBF16)
+    k_colsum_simt<__nv_bfloat16><<<g2, kCsKeys, kCsSmem, st>>>(io, p, nsplit, rowpart, a_base);
+  else
+    k_colsum_simt<float><<<g2, kCsKeys, kCsSmem, st>>>(io, p, nsplit, rowpart, a_base);
   return cudaGetLastError();
 }
 
 // ------------------------------------------------------------------ TSG
 // fp32 path of Eq. 6: one thread per historical token, current-frame keys
-// streamed through shared memory.  Writes chunk 0 of rho_part.
+// streamed through shared memory.  Writes slice 0 of rho_part (the fp32 path
+// has a single slice).  grid = (row tile, layer*Hkv + head).
 constexpr int kTsKeys = 64;
 constexpr int kTsSmem = (kTsgTile * (kD + 1) + kTsKeys * kD + kTsKeys) * 4;
 
 template <typename T>
-__global__ void __launch_bounds__(kTsgTile) k_tsg_simt(const T* __restrict__ k,
-                                                       const float* __restrict__ rn,
-                                                       const __grid_constant__ FrameTable ft,
-                                                       int hkv, float* __restrict__ rho_part) {
+__global__ void __launch_bounds__(kTsgTile) k_tsg_simt(const __grid_constant__ LayerPtrs io,
+                                                       const __grid_constant__ FrameTable ft, int hkv,
+                                                       Strided<const float> rn_all,
+                                                       Strided<float> rho_all) {
   extern __shared__ float sm[];
   float* hs = sm;                              // [128][kD+1]
   float* cs = hs + kTsgTile * (kD + 1);        // [kTsKeys][kD]
   float* cr = cs + kTsKeys * kD;               // [kTsKeys]
-  const int t = blockIdx.x, h = blockIdx.y, tid = threadIdx.x, n = ft.n_tokens;
+  const int t = blockIdx.x, l = blockIdx.y / hkv, h = blockIdx.y % hkv, tid = threadIdx.x;
+  const int n = ft.n_tokens;
+  const T* k = static_cast<const T*>(io.k[l]);
+  const float* rn = rn_all.at(l);
+  float* rho_part = rho_all.at(l);
   // tile -> historical frame
   int f = 0;
   while (f + 1 < ft.n_frames - 1 && ft.tile0[f + 1] <= t) ++f;
@@ -468,20 +487,19 @@ __global__ void __launch_bounds__(kTsgTile) k_tsg_simt(const T* __restrict__ k,
   if (i0 + tid < fend) rho_part[(size_t)h * n + i0 + tid] = best;
 }
 
-cudaError_t launch_tsg(const Problem& p, const FrameTable& ft, const void* k, const float* rn,
-                       float* rho_part, int nchunk, uint32_t* err, cudaStream_t st) {
+cudaError_t launch_tsg(const Problem& p, const FrameTable& ft, const LayerPtrs& io, Strided<const float> rn,
+                       Strided<float> rho_part, uint32_t* err, cudaStream_t st) {
   (void)err;
-  (void)nchunk;
   cudaFuncSetAttribute(k_tsg_simt<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTsSmem);
   cudaFuncSetAttribute(k_tsg_simt<__nv_bfloat16>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTsSmem);
   int tiles = ft.n_frames >= 2 ? ft.tile0[ft.n_frames - 1] : 0;
   if (tiles == 0) return cudaSuccess;
-  dim3 g(tiles, p.hkv);
+  dim3 g(tiles, p.L * p.hkv);
   TimingScope ts("tsg_simt", st);
   if (p.dtype == kBF16)
-    k_tsg_simt<<<g, kTsgTile, kTsSmem, st>>>((const __nv_bfloat16*)k, rn, ft, p.hkv, rho_part);
+    k_tsg_simt<__nv_bfloat16><<<g, kTsgTile, kTsSmem, st>>>(io, ft, p.hkv, rn, rho_part);
   else
-    k_tsg_simt<<<g, kTsgTile, kTsSmem, st>>>((const float*)k, rn, ft, p.hkv, rho_part);
+    k_tsg_simt<float><<<g, kTsgTile, kTsSmem, st>>>(io, ft, p.hkv, rn, rho_part);
   return cudaGetLastError();
 }
 

@@ -25,6 +25,11 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return p + ((1024u - (a & 1023u)) & 1023u);
 }
 
+// Per-layer tensor maps of K (one launch covers up to kMaxLayers layers).
+struct KMaps {
+  CUtensorMap m[kMaxLayers];
+};
+
 // Q rows of KV head h into shared memory in the K-major 128B-swizzle layout
 // [2 K-halves][rows][128 B]; row r = window row * G + group member; rows past
 // R are zero.
@@ -82,13 +87,15 @@ constexpr int kTsgBar = 198656;           // 10 mbarriers + slot + abort
 constexpr int kTsgSmem = kTsgBar + 128 + 1024;
 
 __global__ void __launch_bounds__(kThreads, 1)
-    k_tsg_umma(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ FrameTable ft,
-               const float* __restrict__ rn, float* __restrict__ rho_part, int hkv,
-               uint32_t* err) {
+    k_tsg_umma(const __grid_constant__ KMaps maps, const __grid_constant__ FrameTable ft,
+               Strided<const float> rn_all, Strided<float> rho_all, int hkv, uint32_t* err) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = align1024(smem_raw);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int chunk = blockIdx.y, h = blockIdx.z, n = ft.n_tokens;
+  const int chunk = blockIdx.y, l = blockIdx.z / hkv, h = blockIdx.z % hkv, n = ft.n_tokens;
+  const CUtensorMap& kmap = maps.m[l];
+  const float* rn = rn_all.at(l);
+  float* rho_part = rho_all.at(l);
   const int n_tiles = ft.tile0[ft.n_frames - 1];
   const int col0 = chunk * 512;
   const int valid = min(512, ft.cur_len - col0);
@@ -254,10 +261,32 @@ __global__ void __launch_bounds__(kThreads, 1)
 // epilogue group g handles the key tiles with it % 2 == g and keeps, per
 // query row, the running max m (raw dot units) and l = sum 2^((x - m) c).
 // The two groups merge at the end; part[h][split][r] = (m c, l).
-constexpr int kRsStage = 2;
+constexpr int kMaxKStages = 4;        // key-tile ring depth (as shared memory allows)
+constexpr int kScoreSmemCap = 200 * 1024;
+
+// barrier block of the score kernels: kfull[S], kempty[S], accfull[2],
+// accempty[2], done, then the TMEM slot and the abort flag
+struct ScoreBars {
+  uint32_t kfull, kempty, accfull, accempty, done;
+  uint32_t* slot;
+  volatile uint32_t* abort_flag;
+};
+__device__ __forceinline__ ScoreBars score_bars(uint8_t* base) {
+  ScoreBars b;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(base);
+  b.kfull = smem_u32(&bars[0]);
+  b.kempty = smem_u32(&bars[kMaxKStages]);
+  b.accfull = smem_u32(&bars[2 * kMaxKStages]);
+  b.accempty = smem_u32(&bars[2 * kMaxKStages + 2]);
+  b.done = smem_u32(&bars[2 * kMaxKStages + 4]);
+  b.slot = reinterpret_cast<uint32_t*>(base + (2 * kMaxKStages + 5) * 8);
+  b.abort_flag = b.slot + 1;
+  return b;
+}
+constexpr int kScoreBarBytes = 128;
 
 struct RsLayout {
-  int MT, KN, q_bytes, k_stage_bytes, off_k, off_bar, off_xch, total;
+  int MT, KN, q_bytes, k_stage_bytes, kstages, off_k, off_bar, off_xch, total;
 };
 __host__ __device__ inline RsLayout rs_layout(int R) {
   RsLayout L;
@@ -265,9 +294,13 @@ __host__ __device__ inline RsLayout rs_layout(int R) {
   L.KN = 256 / L.MT;
   L.q_bytes = L.MT * 128 * 256;
   L.k_stage_bytes = L.KN * 256;
+  const int fixed = L.q_bytes + kScoreBarBytes + L.MT * 128 * 8 + 1024;
+  L.kstages = (kScoreSmemCap - fixed) / L.k_stage_bytes;
+  if (L.kstages > kMaxKStages) L.kstages = kMaxKStages;
+  if (L.kstages < 2) L.kstages = 2;
   L.off_k = L.q_bytes;
-  L.off_bar = L.off_k + kRsStage * L.k_stage_bytes;
-  L.off_xch = L.off_bar + 128;
+  L.off_bar = L.off_k + L.kstages * L.k_stage_bytes;
+  L.off_xch = L.off_bar + kScoreBarBytes;
   L.total = L.off_xch + L.MT * 128 * 8 + 1024;
   return L;
 }
@@ -283,32 +316,37 @@ __device__ __forceinline__ void online_merge(float& m, float& l, float m2, float
 
 template <int MT>
 __global__ void __launch_bounds__(kThreads, 1)
-    k_rowstats_umma(const __grid_constant__ CUtensorMap kmap, const __nv_bfloat16* __restrict__ q,
-                    Problem p, int nsplit, float2* __restrict__ part, uint32_t* err) {
+    k_rowstats_umma(const __grid_constant__ KMaps maps, const __grid_constant__ LayerPtrs io, Problem p,
+                    int nsplit, Strided<float2> part_all, uint32_t* err) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = align1024(smem_raw);
   const RsLayout L = rs_layout(p.R());
   constexpr int KN = 256 / MT;
   const int R = p.R();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int split = blockIdx.x, h = blockIdx.y, n = p.n;
+  const int split = blockIdx.x, layer = blockIdx.y / p.hkv, h = blockIdx.y % p.hkv, n = p.n;
+  const CUtensorMap& kmap = maps.m[layer];
+  const __nv_bfloat16* q = static_cast<const __nv_bfloat16*>(io.q[layer]);
+  float2* part = part_all.at(layer);
   const int per = (((n + nsplit - 1) / nsplit) + KN - 1) / KN * KN;
   const int j0 = split * per, j1 = min(n, j0 + per);
   const int ntiles = j1 > j0 ? (j1 - j0 + KN - 1) / KN : 0;
   const uint32_t sQ = smem_u32(sm), sK = smem_u32(sm + L.off_k);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + L.off_bar);
-  const uint32_t b_kfull = smem_u32(&bars[0]), b_kempty = smem_u32(&bars[2]);
-  const uint32_t b_accfull = smem_u32(&bars[4]), b_accempty = smem_u32(&bars[6]);
-  const uint32_t b_done = smem_u32(&bars[8]);
-  uint32_t* slot = reinterpret_cast<uint32_t*>(sm + L.off_bar + 80);
-  volatile uint32_t* abort_flag = slot + 1;
+  const ScoreBars bb = score_bars(sm + L.off_bar);
+  const uint32_t b_kfull = bb.kfull, b_kempty = bb.kempty, b_accfull = bb.accfull;
+  const uint32_t b_accempty = bb.accempty, b_done = bb.done;
+  uint32_t* slot = bb.slot;
+  volatile uint32_t* abort_flag = bb.abort_flag;
+  const int S = L.kstages;
   float2* xch = reinterpret_cast<float2*>(sm + L.off_xch);
   const float c = kLog2eF * rsqrtf((float)kD);
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < S; ++i) {
       mbar_init(b_kfull + 8 * i, 1);
       mbar_init(b_kempty + 8 * i, 1);
+    }
+    for (int i = 0; i < 2; ++i) {
       mbar_init(b_accfull + 8 * i, 1);
       mbar_init(b_accempty + 8 * i, 4);
     }
@@ -338,10 +376,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     if (lane == 0) {
-      int issued[2] = {0, 0};
+      int issued[kMaxKStages] = {0, 0, 0, 0};
       for (int it = 0; it < ntiles; ++it) {
-        const int s = it & 1;
-        const uint32_t u = (uint32_t)(it >> 1);
+        const int s = it % S;
+        const uint32_t u = (uint32_t)(it / S);
         if (!mbar_wait(b_kempty + 8 * s, (u & 1u) ^ 1u, err, abort_flag)) break;
         const int tok = j0 + it * KN;
         mbar_arrive_expect_tx(b_kfull + 8 * s, (uint32_t)L.k_stage_bytes);
@@ -350,17 +388,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         ++issued[s];
       }
       if (*abort_flag)
-        for (int s = 0; s < 2; ++s)
+        for (int s = 0; s < S; ++s)
           if (issued[s]) mbar_wait_drain(b_kfull + 8 * s, (uint32_t)(issued[s] - 1) & 1u);
     }
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16(128, KN);
       for (int it = 0; it < ntiles; ++it) {
-        const int s = it & 1;
-        const uint32_t u = (uint32_t)(it >> 1);
+        const int s = it % S, as = it & 1;
+        const uint32_t u = (uint32_t)(it / S), ua = (uint32_t)(it >> 1);
         if (!mbar_wait(b_kfull + 8 * s, u & 1u, err, abort_flag)) break;
-        if (!mbar_wait(b_accempty + 8 * s, (u & 1u) ^ 1u, err, abort_flag)) break;
+        if (!mbar_wait(b_accempty + 8 * as, (ua & 1u) ^ 1u, err, abort_flag)) break;
         tc_fence_after();
         for (int mt = 0; mt < MT; ++mt) {
 #pragma unroll
@@ -368,10 +406,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t kb = k >> 2, koff = (k & 3) * 32;
             uint64_t ad = desc_sw128(sQ + kb * (MT * 128 * 128) + mt * 128 * 128 + koff);
             uint64_t bd = desc_sw128(sK + s * L.k_stage_bytes + kb * (KN * 128) + koff);
-            umma_bf16(tmem + s * 256 + mt * KN, ad, bd, idesc, k > 0 ? 1u : 0u);
+            umma_bf16(tmem + as * 256 + mt * KN, ad, bd, idesc, k > 0 ? 1u : 0u);
           }
         }
-        umma_commit(b_accfull + 8 * s);
+        umma_commit(b_accfull + 8 * as);
         umma_commit(b_kempty + 8 * s);
       }
       umma_commit(b_done);
@@ -468,7 +506,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 // query rows of its key.  TMEM: two stages of NQ columns when NQ <= 256
 // (epilogue group g takes the tiles with it % 2 == g), else one stage.
 struct CsLayout {
-  int NQ, nstage, tmem_cols, q_bytes, off_k, off_bias, off_bar, total;
+  int NQ, nstage, kstages, tmem_cols, q_bytes, off_k, off_bias, off_bar, total;
 };
 __host__ __device__ inline CsLayout cs_layout(int R) {
   CsLayout L;
@@ -477,37 +515,47 @@ __host__ __device__ inline CsLayout cs_layout(int R) {
   L.tmem_cols = 32;
   while (L.tmem_cols < L.nstage * L.NQ) L.tmem_cols <<= 1;
   L.q_bytes = L.NQ * 256;
+  const int fixed = L.q_bytes + L.NQ * 4 + kScoreBarBytes + 1024;
+  L.kstages = (kScoreSmemCap - fixed) / 32768;
+  if (L.kstages > kMaxKStages) L.kstages = kMaxKStages;
+  if (L.kstages < 2) L.kstages = 2;
   L.off_k = L.q_bytes;
-  L.off_bias = L.off_k + 2 * 32768;
+  L.off_bias = L.off_k + L.kstages * 32768;
   L.off_bar = L.off_bias + L.NQ * 4;
-  L.total = L.off_bar + 128 + 1024;
+  L.total = L.off_bar + kScoreBarBytes + 1024;
   return L;
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
-    k_colsum_umma(const __grid_constant__ CUtensorMap kmap, const __nv_bfloat16* __restrict__ q,
-                  Problem p, const float2* __restrict__ part, int nsplit,
-                  float* __restrict__ a_base, uint32_t* err) {
+    k_colsum_umma(const __grid_constant__ KMaps maps, const __grid_constant__ LayerPtrs io, Problem p,
+                  Strided<float2> part_all, int nsplit, Strided<float> a_all, uint32_t* err) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = align1024(smem_raw);
   const CsLayout L = cs_layout(p.R());
   const int NQ = L.NQ, nstage = L.nstage, R = p.R(), n = p.n;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, h = blockIdx.y;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int layer = blockIdx.y / p.hkv, h = blockIdx.y % p.hkv;
+  const CUtensorMap& kmap = maps.m[layer];
+  const __nv_bfloat16* q = static_cast<const __nv_bfloat16*>(io.q[layer]);
+  const float2* part = part_all.at(layer);
+  float* a_base = a_all.at(layer);
   const int ntiles_all = (n + 127) / 128;
   const uint32_t sQ = smem_u32(sm), sK = smem_u32(sm + L.off_k);
   float* bias_s = reinterpret_cast<float*>(sm + L.off_bias);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + L.off_bar);
-  const uint32_t b_kfull = smem_u32(&bars[0]), b_kempty = smem_u32(&bars[2]);
-  const uint32_t b_accfull = smem_u32(&bars[4]), b_accempty = smem_u32(&bars[6]);
-  const uint32_t b_done = smem_u32(&bars[8]);
-  uint32_t* slot = reinterpret_cast<uint32_t*>(sm + L.off_bar + 80);
-  volatile uint32_t* abort_flag = slot + 1;
+  const ScoreBars bb = score_bars(sm + L.off_bar);
+  const uint32_t b_kfull = bb.kfull, b_kempty = bb.kempty, b_accfull = bb.accfull;
+  const uint32_t b_accempty = bb.accempty, b_done = bb.done;
+  uint32_t* slot = bb.slot;
+  volatile uint32_t* abort_flag = bb.abort_flag;
+  const int S = L.kstages;
   const float c = kLog2eF * rsqrtf((float)kD);
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < S; ++i) {
       mbar_init(b_kfull + 8 * i, 1);
       mbar_init(b_kempty + 8 * i, 1);
+    }
+    for (int i = 0; i < 2; ++i) {
       mbar_init(b_accfull + 8 * i, 1);
       mbar_init(b_accempty + 8 * i, 4);
     }
@@ -547,10 +595,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     if (lane == 0) {
-      int issued[2] = {0, 0};
+      int issued[kMaxKStages] = {0, 0, 0, 0};
       for (int it = 0; it < ntiles; ++it) {
-        const int s = it & 1;
-        const uint32_t u = (uint32_t)(it >> 1);
+        const int s = it % S;
+        const uint32_t u = (uint32_t)(it / S);
         if (!mbar_wait(b_kempty + 8 * s, (u & 1u) ^ 1u, err, abort_flag)) break;
         const int tok = (blockIdx.x + it * gridDim.x) * 128;
         mbar_arrive_expect_tx(b_kfull + 8 * s, 32768);
@@ -559,14 +607,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         ++issued[s];
       }
       if (*abort_flag)
-        for (int s = 0; s < 2; ++s)
+        for (int s = 0; s < S; ++s)
           if (issued[s]) mbar_wait_drain(b_kfull + 8 * s, (uint32_t)(issued[s] - 1) & 1u);
     }
   } else if (warp == 1) {
     if (lane == 0) {
       for (int it = 0; it < ntiles; ++it) {
-        const int s = it & 1, as = it % nstage;
-        const uint32_t u = (uint32_t)(it >> 1), ua = (uint32_t)(it / nstage);
+        const int s = it % S, as = it % nstage;
+        const uint32_t u = (uint32_t)(it / S), ua = (uint32_t)(it / nstage);
         if (!mbar_wait(b_kfull + 8 * s, u & 1u, err, abort_flag)) break;
         if (!mbar_wait(b_accempty + 8 * as, (ua & 1u) ^ 1u, err, abort_flag)) break;
         tc_fence_after();
@@ -678,47 +726,88 @@ static int sm_count() {
   return c > 0 ? c : 148;
 }
 
-int umma_tsg_nchunk(const FrameTable& ft) {
-  return ft.n_frames >= 2 ? (ft.cur_len + 511) / 512 : 0;
+// CTAs per work unit (1..cap): one wave when the units are fewer than the
+// SMs, else the split among 1..4 that fills whole waves best.
+static int pick_split(int units, int cap, int slots) {
+  if (cap < 1) cap = 1;
+  if (units < slots) {
+    int s = (slots + units - 1) / units;
+    return s < cap ? s : cap;
+  }
+  int best = 1;
+  double best_eff = 0.0;
+  for (int s = 1; s <= 4 && s <= cap; ++s) {
+    const long long ctas = (long long)units * s;
+    const long long waves = (ctas + slots - 1) / slots;
+    const double eff = (double)ctas / (double)(waves * slots);
+    if (eff > best_eff + 0.02) {
+      best = s;
+      best_eff = eff;
+    }
+  }
+  return best;
 }
 
-int umma_score_nsplit(const Problem& p) {
-  const RsLayout L = rs_layout(p.R());
-  int per_head = (148 + p.hkv - 1) / p.hkv;
-  int max_split = (p.n + L.KN - 1) / L.KN;
-  return per_head < max_split ? per_head : max_split;
+static cudaError_t make_kmaps(KMaps* maps, const LayerPtrs& io, int L, int n, int hkv, int rows) {
+  for (int l = 0; l < L; ++l) {
+    cudaError_t e = make_kmap(&maps->m[l], io.k[l], n, hkv, rows);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
-cudaError_t launch_tsg_umma(const Problem& p, const FrameTable& ft, const void* k, const float* rn,
-                            float* rho_part, int nchunk, uint32_t* err, cudaStream_t st) {
+// Key splits of window-score pass 1.  They fix how the fp32 row sums are
+// grouped, so they depend on the problem shape only -- not on the batch
+// size or the device -- and a layer gives the same bits alone or batched:
+// one wave of a nominal 152-SM GB300 for one layer, more waves for batches.
+static int score_tiles(const Problem& p) {
+  const int kn = p.dtype == kBF16 ? rs_layout(p.R()).KN : 64;
+  return (p.n + kn - 1) / kn;
+}
+
+int score_nsplit_max(const Problem& p) {
+  const int slots = p.dtype == kBF16 ? 152 : 2 * 152;
+  const int tiles = score_tiles(p);
+  int s = pick_split(p.hkv, tiles, slots);
+  // at least ~24 key tiles per split, so that a CTA's set-up (Q load,
+  // barrier and TMEM set-up, pipeline fill) stays small next to its work
+  const int fat = (tiles + 23) / 24;
+  if (p.dtype == kBF16 && s > fat) s = fat;
+  return s < 1 ? 1 : s;
+}
+
+int score_nsplit(const Problem& p) { return score_nsplit_max(p); }
+
+cudaError_t launch_tsg_umma(const Problem& p, const FrameTable& ft, const LayerPtrs& io,
+                            Strided<const float> rn, Strided<float> rho_part, uint32_t* err,
+                            cudaStream_t st) {
   if (ft.n_frames < 2) return cudaSuccess;
   const int n_tiles = ft.tile0[ft.n_frames - 1];
   if (n_tiles == 0 || ft.cur_len == 0) return cudaSuccess;
-  CUtensorMap map;
-  cudaError_t e = make_kmap(&map, k, p.n, p.hkv, 128);
+  const int nchunk = (ft.cur_len + 511) / 512;
+  KMaps local;
+  cudaError_t e = make_kmaps(&local, io, p.L, p.n, p.hkv, 128);
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(k_tsg_umma, cudaFuncAttributeMaxDynamicSharedMemorySize, kTsgSmem);
   if (e != cudaSuccess) return e;
-  int groups = nchunk * p.hkv;
-  int gx = (sm_count() + groups - 1) / groups;
-  if (gx > n_tiles) gx = n_tiles;
-  if (gx < 1) gx = 1;
-  dim3 grid(gx, nchunk, p.hkv);
+  const int groups = nchunk * p.L * p.hkv;
+  const int gx = pick_split(groups, n_tiles, sm_count());
+  dim3 grid(gx, nchunk, p.L * p.hkv);
   TimingScope ts("tsg_umma", st);
-  k_tsg_umma<<<grid, kThreads, kTsgSmem, st>>>(map, ft, rn, rho_part, p.hkv, err);
+  k_tsg_umma<<<grid, kThreads, kTsgSmem, st>>>(local, ft, rn, rho_part, p.hkv, err);
   return cudaGetLastError();
 }
 
-cudaError_t launch_score_umma(const Problem& p, const void* q, const void* k, float2* rowpart,
-                              int nsplit, float* a_base, uint32_t* err, cudaStream_t st) {
+cudaError_t launch_score_umma(const Problem& p, const LayerPtrs& io, Strided<float2> rowpart, int nsplit,
+                              Strided<float> a_base, uint32_t* err, cudaStream_t st) {
   const int R = p.R();
   if (R > 512) return cudaErrorNotSupported;
   const RsLayout L1 = rs_layout(R);
   const CsLayout L2 = cs_layout(R);
-  CUtensorMap m1, m2;
-  cudaError_t e = make_kmap(&m1, k, p.n, p.hkv, L1.KN);
+  KMaps m1, m2;
+  cudaError_t e = make_kmaps(&m1, io, p.L, p.n, p.hkv, L1.KN);
   if (e != cudaSuccess) return e;
-  if ((e = make_kmap(&m2, k, p.n, p.hkv, 128)) != cudaSuccess) return e;
+  if ((e = make_kmaps(&m2, io, p.L, p.n, p.hkv, 128)) != cudaSuccess) return e;
   auto rs_kernel = L1.MT == 1 ? k_rowstats_umma<1> : (L1.MT == 2 ? k_rowstats_umma<2> : k_rowstats_umma<4>);
   if ((e = cudaFuncSetAttribute(rs_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, L1.total)) !=
       cudaSuccess)
@@ -728,16 +817,13 @@ cudaError_t launch_score_umma(const Problem& p, const void* q, const void* k, fl
     return e;
   {
     TimingScope ts("rowstats_umma", st);
-    rs_kernel<<<dim3(nsplit, p.hkv), kThreads, L1.total, st>>>(m1, (const __nv_bfloat16*)q, p, nsplit,
-                                                               rowpart, err);
+    rs_kernel<<<dim3(nsplit, p.L * p.hkv), kThreads, L1.total, st>>>(m1, io, p, nsplit, rowpart, err);
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  int tiles = (p.n + 127) / 128;
-  int gx = (sm_count() + p.hkv - 1) / p.hkv;
-  if (gx > tiles) gx = tiles;
+  const int tiles = (p.n + 127) / 128;
+  const int gx = pick_split(p.L * p.hkv, tiles, sm_count());
   TimingScope ts("colsum_umma", st);
-  k_colsum_umma<<<dim3(gx, p.hkv), kThreads, L2.total, st>>>(m2, (const __nv_bfloat16*)q, p,
-                                                              rowpart, nsplit, a_base, err);
+  k_colsum_umma<<<dim3(gx, p.L * p.hkv), kThreads, L2.total, st>>>(m2, io, p, rowpart, nsplit, a_base, err);
   return cudaGetLastError();
 }
 

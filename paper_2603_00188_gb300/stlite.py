@@ -27,7 +27,7 @@ MAX_FRAMES = 256
 EXPORTED = ("stlite_budget", "stlite_workspace_size", "stlite_score", "stlite_gate_frames",
             "stlite_spatial_saliency", "stlite_select_topk", "stlite_compact",
             "stlite_compress_layer", "stlite_device_status", "stlite_timing_enable", "stlite_timing_read",
-            "stlite_status_string", "stlite_score_noalloc")
+            "stlite_status_string", "stlite_score_noalloc", "stlite_compress_layers")
 
 
 class Shape(ctypes.Structure):
@@ -44,6 +44,11 @@ class Frames(ctypes.Structure):
 class Params(ctypes.Structure):
     _fields_ = [("beta", ctypes.c_double), ("k_override", ctypes.c_int32), ("alpha", ctypes.c_float),
                 ("tsg_enable", ctypes.c_int32), ("css_enable", ctypes.c_int32)]
+
+
+class LayerIO(ctypes.Structure):
+    _fields_ = [("q", ctypes.c_void_p), ("k", ctypes.c_void_p), ("v", ctypes.c_void_p),
+                ("k_out", ctypes.c_void_p), ("v_out", ctypes.c_void_p), ("idx_out", ctypes.c_void_p)]
 
 
 class KernelTime(ctypes.Structure):
@@ -71,6 +76,9 @@ _sig = {
     "stlite_timing_read": (_S, [ctypes.POINTER(KernelTime), ctypes.c_int32, ctypes.POINTER(ctypes.c_int32)]),
     "stlite_status_string": (ctypes.c_char_p, [ctypes.c_int32]),
     "stlite_score_noalloc": (_S, [ctypes.POINTER(Shape), _P, _P, _P, _P]),
+    "stlite_compress_layers": (_S, [ctypes.POINTER(Shape), ctypes.POINTER(Frames), ctypes.POINTER(Params),
+                                    ctypes.c_int32, ctypes.POINTER(LayerIO), ctypes.POINTER(ctypes.c_int32), _P,
+                                    ctypes.c_size_t, _P]),
 }
 for _name, (_res, _args) in _sig.items():
     _f = getattr(_lib, _name)
@@ -193,6 +201,20 @@ def stlite_compress_layer(q, k, v, frames, params, k_out, v_out, idx_out, ws, st
                                       _ptr(k), _ptr(v), _ptr(k_out), _ptr(v_out), _ptr(idx_out),
                                       ctypes.byref(b), _ptr(ws), ws.numel(), _stream(stream)),
            "stlite_compress_layer")
+    return int(b.value)
+
+
+def stlite_compress_layers(layers, frames, params, ws, stream=None) -> int:
+    """layers: list of (q, k, v, k_out, v_out, idx_out) device tensors, one
+    tuple per layer (same shapes); ws: n_layers * stlite_workspace_size bytes."""
+    q0, k0 = layers[0][0], layers[0][1]
+    sh = make_shape(q0, k0)
+    fs = _frames(frames)
+    arr = (LayerIO * len(layers))(*[LayerIO(*(t.data_ptr() for t in lay)) for lay in layers])
+    b = ctypes.c_int32(0)
+    _check(_lib.stlite_compress_layers(ctypes.byref(sh), ctypes.byref(fs.c), ctypes.byref(params), len(layers),
+                                       arr, ctypes.byref(b), _ptr(ws), ws.numel(), _stream(stream)),
+           "stlite_compress_layers")
     return int(b.value)
 
 

@@ -260,3 +260,41 @@ def test_repeat_deterministic(st):
     for o in outs[1:]:
         for x, y in zip(o, outs[0]):
             assert torch.equal(x, y)
+
+
+# ------------------------------------------------------------ batched layers
+
+def _batched_vs_single(st, wls):
+    dev = [to_device(wl) for wl in wls]
+    wl0 = wls[0]
+    sh = st.make_shape(dev[0][0], dev[0][1])
+    prm = st.make_params(wl0.beta)
+    b = st.stlite_budget(wl0.n, wl0.beta)
+    H = sh.n_kv_heads
+    single = [st.compress_layer(q, k, v, wl0.frames, beta=wl0.beta) for (q, k, v) in dev]
+    outs = []
+    for (q, k, v) in dev:
+        ko = torch.empty((b, H, 128), dtype=k.dtype, device="cuda")
+        outs.append((q, k, v, ko, torch.empty_like(ko), torch.empty((H, b), dtype=torch.int32, device="cuda")))
+    ws = torch.zeros(len(wls) * st.stlite_workspace_size(sh, wl0.frames, prm), dtype=torch.uint8, device="cuda")
+    assert st.stlite_compress_layers(outs, wl0.frames, prm, ws) == b
+    torch.cuda.synchronize()
+    assert st.stlite_device_status(ws) == st.STLITE_OK
+    for (ko1, vo1, i1), (_, _, _, ko2, vo2, i2) in zip(single, outs):
+        assert torch.equal(i1, i2)
+        assert torch.equal(ko1, ko2) and torch.equal(vo1, vo2)
+
+
+def test_compress_layers_equals_single_bf16(st):
+    _batched_vs_single(st, [synth.scaled("traj50", 3, seed=s) for s in range(3)])
+
+
+def test_compress_layers_equals_single_fp32(st):
+    _batched_vs_single(st, [synth.tiny_ref(seed=s) for s in range(2)])
+
+
+def test_compress_layers_more_than_one_launch(st):
+    # 34 layers: two launches of up to 32 layers each
+    wls = [synth.trajectory(n_steps=3, gh=5, gw=7, n_text=4, hq=8, hkv=2, w=4, beta=0.3, seed=(800, s))
+           for s in range(34)]
+    _batched_vs_single(st, wls)
