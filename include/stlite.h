@@ -204,8 +204,9 @@ STLITE_API stlite_status stlite_compress_layers(const stlite_shape* shape, const
                                                 void* ws, size_t ws_bytes, void* stream);
 
 /* Reads and clears the workspace's device error word (synchronises `stream`).
- * *status receives STLITE_OK or the first error a kernel recorded since the
- * last read (STLITE_ETIMEOUT). */
+ * *status receives STLITE_OK, STLITE_ETIMEOUT if a kernel's bounded wait ran
+ * out since the last read, or STLITE_ECUDA if a kernel found its launch
+ * configuration unusable (it then returned without touching its outputs). */
 STLITE_API stlite_status stlite_device_status(void* ws, void* stream, stlite_status* status);
 
 /* Per-kernel timing (instrumentation; not part of Algorithm 1).

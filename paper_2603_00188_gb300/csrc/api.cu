@@ -61,6 +61,9 @@ stlite_status build_frames(const stlite_shape* s, const stlite_frames* fr, Frame
   ft->tile0[0] = 0;
   for (int f = 0; f + 1 < F; ++f)
     ft->tile0[f + 1] = ft->tile0[f] + (ft->gh[f] * ft->gw[f] + kTsgTile - 1) / kTsgTile;
+  ft->ctile0[0] = 0;
+  for (int f = 0; f < F; ++f)
+    ft->ctile0[f + 1] = ft->ctile0[f] + (ft->gh[f] * ft->gw[f] + kTsgTile - 1) / kTsgTile;
   if (F > 0) {
     ft->cur_off = ft->off[F - 1];
     ft->cur_len = ft->gh[F - 1] * ft->gw[F - 1];
@@ -109,8 +112,10 @@ WsPlan plan_workspace(const Problem& p, const FrameTable& ft) {
     o = align_up(o + bytes, 256);
     return at;
   };
+  w.cur_pad = ft.n_frames > 0 ? (ft.cur_len + 3) / 4 * 4 : 4;
   w.err = take(4);
   w.rn = take(hn * 4);
+  w.rn_cur = take((size_t)p.hkv * w.cur_pad * 4);
   w.rowpart = take((size_t)p.hkv * w.nsplit * p.R() * 8 + (size_t)p.hkv * p.R() * 4);
   w.a_base = take(hn * 4);
   w.phi = take(hn * 4);
@@ -119,6 +124,7 @@ WsPlan plan_workspace(const Problem& p, const FrameTable& ft) {
   w.tau = take((size_t)p.hkv * 4);
   w.gate = take(hn);
   w.score = take(hn * 4);
+  w.dots = take(4 * hn * 4);
   w.total = o;
   return w;
 }
@@ -220,6 +226,29 @@ Strided<T> one(T* p) {
   return strided(p, 0);
 }
 
+// CSS (Eqs. 4-5) into phi, plus the inverse key norms rn / rn_cur that TSG
+// uses.  bf16 caches whose grids are at most 127 wide take the tensor-core
+// kernel; otherwise the CUDA-core one.
+cudaError_t run_css(const Ctx& c, const LayerPtrs& io, Strided<float> phi) {
+  Strided<float> rn = c.view<float>(c.plan.rn), rc = c.view<float>(c.plan.rn_cur);
+  if (use_tensor_cores(c.p) && css_umma_supported(c.ft)) {
+    const size_t hn4 = (size_t)c.p.hkv * c.p.n * 4;
+    Strided<float> dE = c.view<float>(c.plan.dots), dS = c.view<float>(c.plan.dots + hn4);
+    Strided<float> dSE = c.view<float>(c.plan.dots + 2 * hn4), dSW = c.view<float>(c.plan.dots + 3 * hn4);
+    return launch_css_umma(c.p, c.ft, io, phi, rn, rc, c.plan.cur_pad, dE, dS, dSE, dSW, c.err, c.st);
+  }
+  return launch_css(c.p, c.ft, io, phi, rn, rc, c.plan.cur_pad, c.st);
+}
+
+// The inverse norms alone: from the CSS kernel when that is the tensor-core
+// one (so that every path sees the same bits), else from the norms kernel
+// (whose arithmetic matches the CUDA-core CSS kernel's).
+cudaError_t run_norms(const Ctx& c, const LayerPtrs& io) {
+  if (use_tensor_cores(c.p) && css_umma_supported(c.ft)) return run_css(c, io, c.view<float>(c.plan.phi));
+  return launch_inv_norms(c.p, c.ft, io, c.view<float>(c.plan.rn), c.view<float>(c.plan.rn_cur), c.plan.cur_pad,
+                          c.st);
+}
+
 cudaError_t run_score(const Ctx& c, const LayerPtrs& io, Strided<float> a_base) {
   Strided<float2> rp = c.view<float2>(c.plan.rowpart);
   const int ns = score_nsplit(c.p);
@@ -230,7 +259,8 @@ cudaError_t run_score(const Ctx& c, const LayerPtrs& io, Strided<float> a_base) 
 cudaError_t run_tsg(const Ctx& c, const LayerPtrs& io) {
   Strided<const float> rn = c.view<const float>(c.plan.rn);
   Strided<float> rp = c.view<float>(c.plan.rho_part);
-  if (use_tensor_cores(c.p)) return launch_tsg_umma(c.p, c.ft, io, rn, rp, c.err, c.st);
+  if (use_tensor_cores(c.p))
+    return launch_tsg_umma(c.p, c.ft, io, c.view<const float>(c.plan.rn_cur), c.plan.cur_pad, rp, c.err, c.st);
   return launch_tsg(c.p, c.ft, io, rn, rp, c.err, c.st);
 }
 
@@ -243,9 +273,9 @@ stlite_status compress_batch(const Ctx& c, const stlite_params* params, const La
   // norms pass provides them.
   cudaError_t e = cudaSuccess;
   if (params->css_enable)
-    e = launch_css(c.p, c.ft, io, phi, c.view<float>(c.plan.rn), c.st);
+    e = run_css(c, io, phi);
   else if (tsg)
-    e = launch_inv_norms(c.p, io, c.view<float>(c.plan.rn), c.st);
+    e = run_norms(c, io);
   if (e == cudaSuccess && tsg) e = run_tsg(c, io);
   if (e == cudaSuccess) e = run_score(c, io, a_base);
   if (e != cudaSuccess) return STLITE_ECUDA;
@@ -316,7 +346,7 @@ stlite_status stlite_gate_frames(const stlite_shape* shape, const stlite_frames*
     return STLITE_EINVAL;
   if (budget < 1 || budget > c.p.n) return STLITE_EINVAL;
   const LayerPtrs io = single_layer(nullptr, k, nullptr, nullptr, nullptr, nullptr);
-  cudaError_t e = launch_inv_norms(c.p, io, c.view<float>(c.plan.rn), c.st);
+  cudaError_t e = run_norms(c, io);
   if (e == cudaSuccess) e = run_tsg(c, io);
   if (e != cudaSuccess) return STLITE_ECUDA;
   SelectArgs a = {};
@@ -340,7 +370,7 @@ stlite_status stlite_spatial_saliency(const stlite_shape* shape, const stlite_fr
   if (s != STLITE_OK) return s;
   if (!k || !phi || !aligned16(k) || !aligned16(phi)) return STLITE_EINVAL;
   const LayerPtrs io = single_layer(nullptr, k, nullptr, nullptr, nullptr, nullptr);
-  cudaError_t e = launch_css(c.p, c.ft, io, one(phi), c.view<float>(c.plan.rn), c.st);
+  cudaError_t e = run_css(c, io, one(phi));
   if (e == cudaSuccess) e = launch_fill_text_nan(c.p, c.ft, phi, c.st);
   return cuda_status(e);
 }
@@ -442,7 +472,7 @@ stlite_status stlite_device_status(void* ws, void* stream, stlite_status* status
   if (cudaMemcpyAsync(&word, ws, 4, cudaMemcpyDeviceToHost, st) != cudaSuccess) return STLITE_ECUDA;
   if (cudaStreamSynchronize(st) != cudaSuccess) return STLITE_ECUDA;
   if (cudaMemsetAsync(ws, 0, 4, st) != cudaSuccess) return STLITE_ECUDA;
-  *status = (word & kErrTimeout) ? STLITE_ETIMEOUT : STLITE_OK;
+  *status = (word & kErrTimeout) ? STLITE_ETIMEOUT : (word ? STLITE_ECUDA : STLITE_OK);
   return STLITE_OK;
 }
 

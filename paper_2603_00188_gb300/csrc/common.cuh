@@ -13,7 +13,8 @@ constexpr int kMaxFrames = 256;    // frames per sequence
 constexpr int kTsgTile = 128;      // historical tokens per TSG row tile
 
 // Device error word bits (first 32-bit word of the workspace).
-constexpr uint32_t kErrTimeout = 1u;
+constexpr uint32_t kErrTimeout = 1u;  // a bounded wait ran out
+constexpr uint32_t kErrLaunch = 2u;   // a kernel found its launch configuration unusable
 
 // Bounded waits give up after this many nanoseconds of %globaltimer.
 constexpr uint64_t kWaitLimitNs = 1000000000ull;
@@ -32,6 +33,7 @@ struct FrameTable {
   int32_t gh[kMaxFrames];
   int32_t gw[kMaxFrames];
   int32_t tile0[kMaxFrames + 1];
+  int32_t ctile0[kMaxFrames + 1];  // first 128-token CSS tile of every frame (all frames)
 };
 
 // Frame holding token j, or -1 for a text token (binary search on offsets).

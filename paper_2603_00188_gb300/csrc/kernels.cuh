@@ -59,6 +59,7 @@ inline Strided<T> strided(T* base, size_t stride) {
 struct WsPlan {
   size_t err;        // uint32 error word (layer 0's is the one used)
   size_t rn;         // float [Hkv][N] inverse key norms
+  size_t rn_cur;     // float [Hkv][cur_pad] inverse norms of the current frame (16-byte rows)
   size_t rowpart;    // float2 [Hkv][nsplit][R] per-split (max, sum) per query row, then float [Hkv][R]
   size_t a_base;     // float [Hkv][N]
   size_t phi;        // float [Hkv][N]
@@ -67,9 +68,11 @@ struct WsPlan {
   size_t tau;        // float [Hkv]
   size_t gate;       // uint8 [Hkv][N]
   size_t score;      // float [Hkv][N]
+  size_t dots;       // float [4][Hkv][N]: E, S, SE, SW neighbour dots (tensor-core CSS)
   size_t total;      // bytes of one layer's region
   int nsplit;        // largest key-split count of the row-statistics pass
   int nchunk;        // 256-column slices of rho_part
+  int cur_pad;       // current-frame length rounded up to 4
 };
 WsPlan plan_workspace(const Problem& p, const FrameTable& ft);
 
@@ -91,8 +94,11 @@ class TimingScope {
 };
 
 // ---- launchers ----------------------------------------------------------
-// rn[l][h][j] = 1 / max(|k_l[j,h]|, 1e-8) for every token.
-cudaError_t launch_inv_norms(const Problem& p, const LayerPtrs& io, Strided<float> rn, cudaStream_t st);
+// rn[l][h][j] = 1 / max(|k_l[j,h]|, 1e-8) for every token; the current
+// frame's values are also written to rn_cur[l][h][j - cur_off] (row stride
+// cur_pad).
+cudaError_t launch_inv_norms(const Problem& p, const FrameTable& ft, const LayerPtrs& io, Strided<float> rn,
+                             Strided<float> rn_cur, int cur_pad, cudaStream_t st);
 
 // Window score (Eq. 2): row statistics then column sums.  rowpart holds, per
 // layer, [Hkv][nsplit][R] float2 followed by [Hkv][R] float (row bias).
@@ -112,13 +118,23 @@ cudaError_t launch_tsg(const Problem& p, const FrameTable& ft, const LayerPtrs& 
                        Strided<const float> rn, Strided<float> rho_part, uint32_t* err,
                        cudaStream_t st);
 cudaError_t launch_tsg_umma(const Problem& p, const FrameTable& ft, const LayerPtrs& io,
-                            Strided<const float> rn, Strided<float> rho_part, uint32_t* err,
-                            cudaStream_t st);
+                            Strided<const float> rn_cur, int cur_pad, Strided<float> rho_part,
+                            uint32_t* err, cudaStream_t st);
 
 // CSS saliency Phi (Eqs. 4-5) of every visual token; also writes the inverse
-// key norms rn of every visual token.  Text entries are not touched.
+// key norms of every visual token to rn (and of the current frame's to
+// rn_cur, as launch_inv_norms).  Text entries are not touched.
 cudaError_t launch_css(const Problem& p, const FrameTable& ft, const LayerPtrs& io,
-                       Strided<float> phi, Strided<float> rn, cudaStream_t st);
+                       Strided<float> phi, Strided<float> rn, Strided<float> rn_cur, int cur_pad,
+                       cudaStream_t st);
+// Tensor-core CSS (bf16, every grid at most 127 wide): per-token squared-norm
+// and E/S/SE/SW dots on the tensor cores, then Phi; writes rn and rn_cur as
+// launch_css does.
+bool css_umma_supported(const FrameTable& ft);
+cudaError_t launch_css_umma(const Problem& p, const FrameTable& ft, const LayerPtrs& io, Strided<float> phi,
+                            Strided<float> rn, Strided<float> rn_cur, int cur_pad, Strided<float> dE,
+                            Strided<float> dS, Strided<float> dSE, Strided<float> dSW, uint32_t* err,
+                            cudaStream_t st);
 // phi[h][j] = NaN for every text token j (one layer).
 cudaError_t launch_fill_text_nan(const Problem& p, const FrameTable& ft, float* phi, cudaStream_t st);
 

@@ -158,6 +158,36 @@ __device__ __forceinline__ void for_spans(const FrameTable& ft, int f0, int f1, 
   }
 }
 
+// Same visiting order, four tokens per thread at a time: load(i) for all four
+// is issued before use(i, value) runs for any, so their latencies overlap.
+template <class Load, class Use>
+__device__ __forceinline__ void for_spans4(const FrameTable& ft, int f0, int f1, int j0, int j1, Load load,
+                                           Use use) {
+  int lo = f0, hi = f1 - 1, first = f1;
+  while (lo <= hi) {
+    const int mid = (lo + hi) >> 1;
+    if (ft.off[mid] + ft.gh[mid] * ft.gw[mid] > j0) {
+      first = mid;
+      hi = mid - 1;
+    } else {
+      lo = mid + 1;
+    }
+  }
+  const int B = blockDim.x;
+  for (int f = first; f < f1 && ft.off[f] < j1; ++f) {
+    const int a = max(ft.off[f], j0), b = min(ft.off[f] + ft.gh[f] * ft.gw[f], j1);
+    for (int i0 = a + (int)threadIdx.x; i0 < b; i0 += 4 * B) {
+      decltype(load(i0)) v[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        if (i0 + u * B < b) v[u] = load(i0 + u * B);
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        if (i0 + u * B < b) use(i0 + u * B, v[u]);
+    }
+  }
+}
+
 __global__ void __launch_bounds__(kSelThreads) k_select(Problem p, const __grid_constant__ FrameTable ft,
                                                         SelectArgs a) {
   extern __shared__ uint32_t keys[];
@@ -185,19 +215,24 @@ __global__ void __launch_bounds__(kSelThreads) k_select(Problem p, const __grid_
     int pool = 0;
     for (int f = 0; f + 1 < F; ++f) pool += ft.gh[f] * ft.gw[f];
     const size_t slice = (size_t)p.hkv * n;
-    for_spans(ft, 0, F - 1, j0, j1, [&](int i) {
-      const float* src = rp + hn + i;
-      float m0 = -CUDART_INF_F, m1 = -CUDART_INF_F;
-      int s = 0;
-      for (; s + 1 < a.nchunk; s += 2) {
-        m0 = fmaxf(m0, __ldg(src + (size_t)s * slice));
-        m1 = fmaxf(m1, __ldg(src + (size_t)(s + 1) * slice));
-      }
-      if (s < a.nchunk) m0 = fmaxf(m0, __ldg(src + (size_t)s * slice));
-      const float r = fmaxf(m0, m1) * __ldg(rn + i);
-      rho[i] = r;
-      keys[i - j0] = ~float_key(r);  // m-th smallest == m-th largest complement
-    });
+    for_spans4(
+        ft, 0, F - 1, j0, j1,
+        [&](int i) {
+          const float* src = rp + hn + i;
+          float m0 = -CUDART_INF_F, m1 = -CUDART_INF_F;
+          int s = 0;
+          for (; s + 1 < a.nchunk; s += 2) {
+            m0 = fmaxf(m0, __ldg(src + (size_t)s * slice));
+            m1 = fmaxf(m1, __ldg(src + (size_t)(s + 1) * slice));
+          }
+          if (s < a.nchunk) m0 = fmaxf(m0, __ldg(src + (size_t)s * slice));
+          return make_float2(fmaxf(m0, m1), __ldg(rn + i));
+        },
+        [&](int i, float2 v) {
+          const float r = v.x * v.y;
+          rho[i] = r;
+          keys[i - j0] = ~float_key(r);  // m-th smallest == m-th largest complement
+        });
     __syncthreads();
     if (pool > 0 && a.tsg_enable) {
       uint32_t need;
@@ -218,18 +253,33 @@ __global__ void __launch_bounds__(kSelThreads) k_select(Problem p, const __grid_
     float* sc = a.score.at(l) + hn;
     const float alpha = a.css_enable ? a.alpha : 0.f;
     // text tokens: S = A_base; visual tokens are overwritten below
-    for (int i = tid; i < len; i += blockDim.x) {
-      const float s = __ldg(ab + j0 + i) + 0.0f;
-      sc[j0 + i] = s;
-      keys[i] = float_key(s);
+    for (int i0 = tid; i0 < len; i0 += 4 * blockDim.x) {
+      float v[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        if (i0 + u * (int)blockDim.x < len) v[u] = __ldg(ab + j0 + i0 + u * blockDim.x);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int i = i0 + u * blockDim.x;
+        if (i < len) {
+          const float s = v[u] + 0.0f;
+          sc[j0 + i] = s;
+          keys[i] = float_key(s);
+        }
+      }
     }
     __syncthreads();
-    for_spans(ft, 0, F, j0, j1, [&](int j) {
-      const float x = __ldg(ab + j) + (alpha != 0.f ? alpha * __ldg(ph + j) : 0.f);
-      const float s = ((gt == nullptr || gt[j]) ? x : 0.f) + 0.0f;
-      sc[j] = s;
-      keys[j - j0] = float_key(s);
-    });
+    for_spans4(
+        ft, 0, F, j0, j1,
+        [&](int j) {
+          const float x = __ldg(ab + j) + (alpha != 0.f ? alpha * __ldg(ph + j) : 0.f);
+          return (gt == nullptr || gt[j]) ? x : 0.f;
+        },
+        [&](int j, float x) {
+          const float s = x + 0.0f;
+          sc[j] = s;
+          keys[j - j0] = float_key(s);
+        });
     __syncthreads();
     uint32_t need;
     const uint32_t T = cluster_select_desc(cl, keys, len, (uint32_t)a.budget, sh, pass, &need);

@@ -35,7 +35,8 @@ __device__ __forceinline__ void unpack16(const uint4& w, float (&f)[16 / sizeof(
 // grid.y = layer.
 template <typename T>
 __global__ void __launch_bounds__(256) k_inv_norms(const __grid_constant__ LayerPtrs io, int n, int hkv,
-                                                   Strided<float> rn_all) {
+                                                   Strided<float> rn_all, Strided<float> rc_all, int cur_off,
+                                                   int cur_len, int cur_pad) {
   constexpr int kChunks = kD * (int)sizeof(T) / 16;
   constexpr int kPer = 16 / (int)sizeof(T);
   const int l = blockIdx.y;
@@ -57,11 +58,14 @@ __global__ void __launch_bounds__(256) k_inv_norms(const __grid_constant__ Layer
       for (int t = 0; t < kPer; ++t) sn = fmaf(x[t], x[t], sn);
     }
     const long long j = r / hkv, h = r - j * hkv;
-    rn[h * n + j] = 1.0f / fmaxf(sqrtf(sn), 1e-8f);
+    const float v = 1.0f / fmaxf(sqrtf(sn), 1e-8f);
+    rn[h * n + j] = v;
+    if (j >= cur_off && j < cur_off + cur_len) rc_all.at(l)[h * cur_pad + (j - cur_off)] = v;
   }
 }
 
-cudaError_t launch_inv_norms(const Problem& p, const LayerPtrs& io, Strided<float> rn, cudaStream_t st) {
+cudaError_t launch_inv_norms(const Problem& p, const FrameTable& ft, const LayerPtrs& io, Strided<float> rn,
+                             Strided<float> rn_cur, int cur_pad, cudaStream_t st) {
   long long rows = (long long)p.n * p.hkv;
   long long blocks = (rows + 255) / 256;
   long long cap = (152 * 8 + p.L - 1) / p.L;
@@ -69,9 +73,9 @@ cudaError_t launch_inv_norms(const Problem& p, const LayerPtrs& io, Strided<floa
   TimingScope ts("inv_norms", st);
   dim3 grid((unsigned)blocks, p.L);
   if (p.dtype == kBF16)
-    k_inv_norms<__nv_bfloat16><<<grid, 256, 0, st>>>(io, p.n, p.hkv, rn);
+    k_inv_norms<__nv_bfloat16><<<grid, 256, 0, st>>>(io, p.n, p.hkv, rn, rn_cur, ft.cur_off, ft.cur_len, cur_pad);
   else
-    k_inv_norms<float><<<grid, 256, 0, st>>>(io, p.n, p.hkv, rn);
+    k_inv_norms<float><<<grid, 256, 0, st>>>(io, p.n, p.hkv, rn, rn_cur, ft.cur_off, ft.cur_len, cur_pad);
   return cudaGetLastError();
 }
 
@@ -110,7 +114,8 @@ struct CssGeom {
 template <typename T>
 __global__ void __launch_bounds__(kCssThreads) k_css(const __grid_constant__ LayerPtrs io,
                                                      const __grid_constant__ FrameTable ft, int hkv,
-                                                     Strided<float> phi_all, Strided<float> rn_all) {
+                                                     Strided<float> phi_all, Strided<float> rn_all,
+                                                     Strided<float> rc_all, int cur_pad) {
   using Gm = CssGeom<T>;
   constexpr int kChunks = kD * (int)sizeof(T) / 16;
   constexpr int kPer = 16 / (int)sizeof(T);
@@ -209,6 +214,7 @@ __global__ void __launch_bounds__(kCssThreads) k_css(const __grid_constant__ Lay
     const int j = off + u * gw + v;
     phi[(size_t)h * n + j] = cnt ? 1.0f - sum / (float)cnt : 0.0f;
     rn_out[(size_t)h * n + j] = r0;
+    if (f == ft.n_frames - 1) rc_all.at(l)[(size_t)h * cur_pad + (j - off)] = r0;
   }
 }
 
@@ -224,7 +230,8 @@ __global__ void k_fill_text_nan(const __grid_constant__ FrameTable ft, int hkv, 
 
 template <typename T>
 static cudaError_t css_launch_t(const Problem& p, const FrameTable& ft, const LayerPtrs& io,
-                                Strided<float> phi, Strided<float> rn, cudaStream_t st) {
+                                Strided<float> phi, Strided<float> rn, Strided<float> rn_cur, int cur_pad,
+                                cudaStream_t st) {
   using Gm = CssGeom<T>;
   int tmax = 0, cmax = 0;
   for (int f = 0; f < ft.n_frames; ++f) {
@@ -238,14 +245,15 @@ static cudaError_t css_launch_t(const Problem& p, const FrameTable& ft, const La
   cudaError_t e = cudaFuncSetAttribute(k_css<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   TimingScope ts("css", st);
-  k_css<T><<<dim3(tmax, ft.n_frames, p.L * p.hkv), kCssThreads, smem, st>>>(io, ft, p.hkv, phi, rn);
+  k_css<T><<<dim3(tmax, ft.n_frames, p.L * p.hkv), kCssThreads, smem, st>>>(io, ft, p.hkv, phi, rn, rn_cur,
+                                                                             cur_pad);
   return cudaGetLastError();
 }
 
 cudaError_t launch_css(const Problem& p, const FrameTable& ft, const LayerPtrs& io, Strided<float> phi,
-                       Strided<float> rn, cudaStream_t st) {
-  if (p.dtype == kBF16) return css_launch_t<__nv_bfloat16>(p, ft, io, phi, rn, st);
-  return css_launch_t<float>(p, ft, io, phi, rn, st);
+                       Strided<float> rn, Strided<float> rn_cur, int cur_pad, cudaStream_t st) {
+  if (p.dtype == kBF16) return css_launch_t<__nv_bfloat16>(p, ft, io, phi, rn, rn_cur, cur_pad, st);
+  return css_launch_t<float>(p, ft, io, phi, rn, rn_cur, cur_pad, st);
 }
 
 cudaError_t launch_fill_text_nan(const Problem& p, const FrameTable& ft, float* phi, cudaStream_t st) {

@@ -81,20 +81,26 @@ __device__ __forceinline__ void tsg_tile(const FrameTable& ft, int t, int& tok0,
 // and writes slice 2*chunk+g of rho_part: max_j acc_ij * rn_j.  Columns past
 // the current frame carry rn = NaN, which fmaxf ignores.
 constexpr int kTsgB = 0;                  // [2][512][128 B]
-constexpr int kTsgA = 131072;             // [2 stages][2][128][128 B]
-constexpr int kTsgRn = 196608;            // float[512]
-constexpr int kTsgBar = 198656;           // 10 mbarriers + slot + abort
-constexpr int kTsgSmem = kTsgBar + 128 + 1024;
+constexpr int kTsgAStages = 3;
+constexpr int kTsgA = 131072;                              // [3 stages][2][128][128 B]
+constexpr int kTsgRn = kTsgA + kTsgAStages * 32768;        // float[512]
+constexpr int kTsgBar = kTsgRn + 2048;                     // 12 mbarriers + slot + abort
+constexpr int kTsgUsed = kTsgBar + 128;                    // bytes after 1024-alignment
+constexpr int kTsgSmem = 232448;                           // the per-CTA maximum; the rest is alignment slack
 
 __global__ void __launch_bounds__(kThreads, 1)
     k_tsg_umma(const __grid_constant__ KMaps maps, const __grid_constant__ FrameTable ft,
-               Strided<const float> rn_all, Strided<float> rho_all, int hkv, uint32_t* err) {
+               Strided<const float> rc_all, int cur_pad, Strided<float> rho_all, int hkv, uint32_t* err) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = align1024(smem_raw);
+  if ((int)(sm - smem_raw) + kTsgUsed > kTsgSmem) {  // uniform: the layout would not fit
+    if (threadIdx.x == 0) record_error(err, kErrLaunch);
+    return;
+  }
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int chunk = blockIdx.y, l = blockIdx.z / hkv, h = blockIdx.z % hkv, n = ft.n_tokens;
   const CUtensorMap& kmap = maps.m[l];
-  const float* rn = rn_all.at(l);
+  const float* rn_cur = rc_all.at(l) + (size_t)h * cur_pad;  // 16-byte aligned rows
   float* rho_part = rho_all.at(l);
   const int n_tiles = ft.tile0[ft.n_frames - 1];
   const int col0 = chunk * 512;
@@ -103,16 +109,20 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t sB = smem_u32(sm + kTsgB), sA = smem_u32(sm + kTsgA);
   float* rn_s = reinterpret_cast<float*>(sm + kTsgRn);
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + kTsgBar);
-  const uint32_t b_afull = smem_u32(&bars[0]), b_aempty = smem_u32(&bars[2]);
-  const uint32_t b_bfull = smem_u32(&bars[4]), b_accfull = smem_u32(&bars[5]);
-  const uint32_t b_accempty = smem_u32(&bars[7]), b_done = smem_u32(&bars[9]);
-  uint32_t* slot = reinterpret_cast<uint32_t*>(sm + kTsgBar + 80);
+  const uint32_t b_afull = smem_u32(&bars[0]), b_aempty = smem_u32(&bars[kTsgAStages]);
+  const uint32_t b_bfull = smem_u32(&bars[2 * kTsgAStages]);
+  const uint32_t b_accfull = smem_u32(&bars[2 * kTsgAStages + 1]);
+  const uint32_t b_accempty = smem_u32(&bars[2 * kTsgAStages + 3]);
+  const uint32_t b_done = smem_u32(&bars[2 * kTsgAStages + 5]);
+  uint32_t* slot = reinterpret_cast<uint32_t*>(sm + kTsgBar + (2 * kTsgAStages + 6) * 8);
   volatile uint32_t* abort_flag = slot + 1;
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < kTsgAStages; ++i) {
       mbar_init(b_afull + 8 * i, 1);
       mbar_init(b_aempty + 8 * i, 1);
+    }
+    for (int i = 0; i < 2; ++i) {
       mbar_init(b_accfull + 8 * i, 1);
       mbar_init(b_accempty + 8 * i, 4);
     }
@@ -126,8 +136,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_alloc(smem_u32(slot), 512);
     tmem_relinquish();
   }
+  // inverse norms of this chunk's current-frame columns (NaN past the frame)
   for (int c = (int)threadIdx.x - 64; c < 512; c += kThreads - 64)
-    if (c >= 0) rn_s[c] = c < valid ? rn[(size_t)h * n + ft.cur_off + col0 + c] : CUDART_NAN_F;
+    if (c >= 0) rn_s[c] = c < valid ? rn_cur[col0 + c] : CUDART_NAN_F;
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -140,10 +151,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int rb = 0; rb < 4; ++rb)
           tma_load_3d(sB + kb * 65536 + rb * 16384, &kmap, b_bfull, kb * 64, h,
                       ft.cur_off + col0 + rb * 128);
-      int it = 0, issued[2] = {0, 0};
+      int it = 0, issued[kTsgAStages] = {0, 0, 0};
       for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++it) {
-        const int s = it & 1;
-        const uint32_t u = (uint32_t)(it >> 1);
+        const int s = it % kTsgAStages;
+        const uint32_t u = (uint32_t)(it / kTsgAStages);
         if (!mbar_wait(b_aempty + 8 * s, (u & 1u) ^ 1u, err, abort_flag)) break;
         int tok0, fend;
         tsg_tile(ft, t, tok0, fend);
@@ -154,7 +165,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (*abort_flag) {  // drain copies still in flight before the CTA exits
         mbar_wait_drain(b_bfull, 0);
-        for (int s = 0; s < 2; ++s)
+        for (int s = 0; s < kTsgAStages; ++s)
           if (issued[s]) mbar_wait_drain(b_afull + 8 * s, (uint32_t)(issued[s] - 1) & 1u);
       }
     }
@@ -163,8 +174,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = mbar_wait(b_bfull, 0, err, abort_flag);
       int it = 0;
       for (int t = blockIdx.x; ok && t < n_tiles; t += gridDim.x, ++it) {
-        const int s = it & 1;
-        const uint32_t u = (uint32_t)(it >> 1);
+        const int s = it % kTsgAStages;
+        const uint32_t u = (uint32_t)(it / kTsgAStages);
         if (!mbar_wait(b_afull + 8 * s, u & 1u, err, abort_flag)) break;
         tc_fence_after();
         for (int g = 0; g < nst && ok; ++g) {
@@ -422,55 +433,65 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!warp_wait(b_accfull + 8 * g, u & 1u, err, abort_flag)) break;
       tc_fence_after();
       const int tok = j0 + it * KN;
-#pragma unroll
-      for (int mt = 0; mt < MT; ++mt) {
+      // a tile is always four 64-column chunks (MT m-tiles x KN/64 key
+      // chunks); chunk q+1 loads from TMEM while chunk q is reduced
+      uint32_t b0[64], b1[64];
+      auto online = [&](const uint32_t (&b)[64], int q) {
+        const int mt = q / (KN / 64), kbase = tok + (q % (KN / 64)) * 64;
+        const int nv = min(64, j1 - kbase);
+        if (nv <= 0) return;
         float m = m_st[mt], l = l_st[mt];
-#pragma unroll 1
-        for (int cg = 0; cg < KN / 64; ++cg) {
-          const int kbase = tok + cg * 64;
-          if (kbase >= j1) break;
-          float v[64];
-          tmem_ld64(lanebase + g * 256 + mt * KN + cg * 64, v);
-          const int nv = min(64, j1 - kbase);
-          if (nv == 64) {
-            // indices 0..63: c0 takes 0, 2..3, 6..7, ..., 62..63; c1 takes 1, 4..5, ..., 60..61
-            float c0 = v[0], c1 = v[1];
+        if (nv == 64) {
+          // indices 0..63: c0 takes 0, 2..3, 6..7, ..., 62..63; c1 takes 1, 4..5, ..., 60..61
+          float c0 = __uint_as_float(b[0]), c1 = __uint_as_float(b[1]);
 #pragma unroll
-            for (int i = 2; i < 62; i += 4) {
-              c0 = max3(c0, v[i], v[i + 1]);
-              c1 = max3(c1, v[i + 2], v[i + 3]);
-            }
-            c0 = max3(c0, v[62], v[63]);
-            const float mn = fmaxf(m, fmaxf(c0, c1));
-            const float mnc = mn * c;
-            float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-#pragma unroll
-            for (int i = 0; i < 64; i += 4) {
-              s0 += ex2_approx(fmaf(v[i], c, -mnc));
-              s1 += ex2_approx(fmaf(v[i + 1], c, -mnc));
-              s2 += ex2_approx(fmaf(v[i + 2], c, -mnc));
-              s3 += ex2_approx(fmaf(v[i + 3], c, -mnc));
-            }
-            l = (m == -CUDART_INF_F ? 0.f : l * ex2_approx((m - mn) * c)) + ((s0 + s1) + (s2 + s3));
-            m = mn;
-          } else {
-            float mc = -CUDART_INF_F;
-#pragma unroll
-            for (int i = 0; i < 64; ++i)
-              if (i < nv) mc = fmaxf(mc, v[i]);
-            const float mn = fmaxf(m, mc);
-            const float mnc = mn * c;
-            float sacc = 0.f;
-#pragma unroll
-            for (int i = 0; i < 64; ++i)
-              if (i < nv) sacc += ex2_approx(fmaf(v[i], c, -mnc));
-            l = (m == -CUDART_INF_F ? 0.f : l * ex2_approx((m - mn) * c)) + sacc;
-            m = mn;
+          for (int i = 2; i < 62; i += 4) {
+            c0 = max3(c0, __uint_as_float(b[i]), __uint_as_float(b[i + 1]));
+            c1 = max3(c1, __uint_as_float(b[i + 2]), __uint_as_float(b[i + 3]));
           }
+          c0 = max3(c0, __uint_as_float(b[62]), __uint_as_float(b[63]));
+          const float mn = fmaxf(m, fmaxf(c0, c1));
+          const float mnc = mn * c;
+          float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+          for (int i = 0; i < 64; i += 4) {
+            s0 += ex2_approx(fmaf(__uint_as_float(b[i]), c, -mnc));
+            s1 += ex2_approx(fmaf(__uint_as_float(b[i + 1]), c, -mnc));
+            s2 += ex2_approx(fmaf(__uint_as_float(b[i + 2]), c, -mnc));
+            s3 += ex2_approx(fmaf(__uint_as_float(b[i + 3]), c, -mnc));
+          }
+          l = (m == -CUDART_INF_F ? 0.f : l * ex2_approx((m - mn) * c)) + ((s0 + s1) + (s2 + s3));
+          m = mn;
+        } else {
+          float mc = -CUDART_INF_F;
+#pragma unroll
+          for (int i = 0; i < 64; ++i)
+            if (i < nv) mc = fmaxf(mc, __uint_as_float(b[i]));
+          const float mn = fmaxf(m, mc);
+          const float mnc = mn * c;
+          float sacc = 0.f;
+#pragma unroll
+          for (int i = 0; i < 64; ++i)
+            if (i < nv) sacc += ex2_approx(fmaf(__uint_as_float(b[i]), c, -mnc));
+          l = (m == -CUDART_INF_F ? 0.f : l * ex2_approx((m - mn) * c)) + sacc;
+          m = mn;
         }
         m_st[mt] = m;
         l_st[mt] = l;
-      }
+      };
+      const uint32_t tb = lanebase + g * 256;
+      tmem_ld64_issue(tb, b0);
+      tmem_ld64_wait(b0);
+      tmem_ld64_issue(tb + 64, b1);
+      online(b0, 0);
+      tmem_ld64_wait(b1);
+      tmem_ld64_issue(tb + 128, b0);
+      online(b1, 1);
+      tmem_ld64_wait(b0);
+      tmem_ld64_issue(tb + 192, b1);
+      online(b0, 2);
+      tmem_ld64_wait(b1);
+      online(b1, 3);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(b_accempty + 8 * g);
@@ -689,6 +710,232 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // =========================================================================
+// CSS on the tensor cores (bf16).  CTA (x, layer*Hkv + head) walks 128-token
+// tiles of the frames' visual spans.  For a tile starting at token t0 of a
+// frame with grid width gw, B = keys of tokens [t0, t0 + NB), NB =
+// roundup16(128 + gw + 1) <= 256, and A = its first 128 rows; one tcgen05
+// MMA gives every dot product a row needs: D[i][i] (squared norm),
+// D[i][i+1] (E), D[i][i+gw-1] (SW), D[i][i+gw] (S), D[i][i+gw+1] (SE).  Each
+// epilogue thread drains its TMEM row window in 32-column chunks, parks each
+// chunk in its own row of a padded shared buffer and picks the five
+// diagonals; k_css_phi then forms Phi from the per-token dots (Eqs. 4-5).
+constexpr int kCssBStage = 65536;                        // [2 halves][256 rows][128 B]
+constexpr int kCssStgRow = 36;                           // floats per staged row (16-byte rows, no conflicts)
+constexpr int kCssStg = 2 * kCssBStage;                  // 8 warps x [32][36] floats
+constexpr int kCssBar = kCssStg + 8 * 32 * kCssStgRow * 4;
+constexpr int kCssUmmaSmem = kCssBar + 128 + 1024;
+constexpr int kCssMaxGw = 127;                           // NB <= 256
+
+struct CssDots {
+  Strided<float> rn, dE, dS, dSE, dSW, rn_cur;
+  int cur_pad;
+};
+
+__device__ __forceinline__ void css_tile(const FrameTable& ft, int t, int& f, int& t0) {
+  int lo = 0, hi = ft.n_frames - 1;
+  f = 0;
+  while (lo <= hi) {
+    const int mid = (lo + hi) >> 1;
+    if (ft.ctile0[mid] <= t) {
+      f = mid;
+      lo = mid + 1;
+    } else {
+      hi = mid - 1;
+    }
+  }
+  t0 = ft.off[f] + (t - ft.ctile0[f]) * 128;
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    k_css_umma(const __grid_constant__ KMaps maps, const __grid_constant__ FrameTable ft, int hkv,
+               CssDots out, uint32_t* err) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = align1024(smem_raw);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int l = blockIdx.y / hkv, h = blockIdx.y % hkv, n = ft.n_tokens;
+  const CUtensorMap& kmap = maps.m[l];
+  const int ntiles_all = ft.ctile0[ft.n_frames];
+  const uint32_t sB = smem_u32(sm);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + kCssBar);
+  const uint32_t b_kfull = smem_u32(&bars[0]), b_kempty = smem_u32(&bars[2]);
+  const uint32_t b_accfull = smem_u32(&bars[4]), b_accempty = smem_u32(&bars[6]);
+  const uint32_t b_done = smem_u32(&bars[8]);
+  uint32_t* slot = reinterpret_cast<uint32_t*>(sm + kCssBar + 80);
+  volatile uint32_t* abort_flag = slot + 1;
+  int ntiles = 0;
+  for (int t = blockIdx.x; t < ntiles_all; t += gridDim.x) ++ntiles;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(b_kfull + 8 * i, 1);
+      mbar_init(b_kempty + 8 * i, 1);
+      mbar_init(b_accfull + 8 * i, 1);
+      mbar_init(b_accempty + 8 * i, 4);
+    }
+    mbar_init(b_done, 1);
+    *abort_flag = 0u;
+    fence_mbar_init();
+    tma_prefetch_desc(&kmap);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(slot), 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int issued[2] = {0, 0};
+      for (int it = 0; it < ntiles; ++it) {
+        const int s = it & 1;
+        const uint32_t u = (uint32_t)(it >> 1);
+        if (!mbar_wait(b_kempty + 8 * s, (u & 1u) ^ 1u, err, abort_flag)) break;
+        int f, t0;
+        css_tile(ft, blockIdx.x + it * gridDim.x, f, t0);
+        mbar_arrive_expect_tx(b_kfull + 8 * s, kCssBStage);
+        for (int kb = 0; kb < 2; ++kb)
+          for (int half = 0; half < 2; ++half)
+            tma_load_3d(sB + s * kCssBStage + kb * 32768 + half * 16384, &kmap, b_kfull + 8 * s, kb * 64, h,
+                        t0 + half * 128);
+        ++issued[s];
+      }
+      if (*abort_flag)
+        for (int s = 0; s < 2; ++s)
+          if (issued[s]) mbar_wait_drain(b_kfull + 8 * s, (uint32_t)(issued[s] - 1) & 1u);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      for (int it = 0; it < ntiles; ++it) {
+        const int s = it & 1;
+        const uint32_t u = (uint32_t)(it >> 1);
+        if (!mbar_wait(b_kfull + 8 * s, u & 1u, err, abort_flag)) break;
+        if (!mbar_wait(b_accempty + 8 * s, (u & 1u) ^ 1u, err, abort_flag)) break;
+        tc_fence_after();
+        int f, t0;
+        css_tile(ft, blockIdx.x + it * gridDim.x, f, t0);
+        const int nb = (128 + ft.gw[f] + 1 + 15) & ~15;
+        const uint32_t idesc = idesc_bf16(128, nb);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const uint32_t kb = k >> 2, koff = (k & 3) * 32;
+          const uint64_t d = desc_sw128(sB + s * kCssBStage + kb * 32768 + koff);
+          umma_bf16(tmem + s * 256, d, d, idesc, k > 0 ? 1u : 0u);
+        }
+        umma_commit(b_accfull + 8 * s);
+        umma_commit(b_kempty + 8 * s);
+      }
+      umma_commit(b_done);
+      mbar_wait_drain(b_done, 0);
+    }
+  } else {
+    const int g = (warp - 2) >> 2, quarter = warp & 3;
+    float* stg = reinterpret_cast<float*>(sm + kCssStg) + (size_t)(warp - 2) * 32 * kCssStgRow + lane * kCssStgRow;
+    const uint32_t tbase = tmem + ((uint32_t)(quarter * 32) << 16) + g * 256 + quarter * 32;
+    float* rn_o = out.rn.at(l) + (size_t)h * n;
+    float* e_o = out.dE.at(l) + (size_t)h * n;
+    float* s_o = out.dS.at(l) + (size_t)h * n;
+    float* se_o = out.dSE.at(l) + (size_t)h * n;
+    float* sw_o = out.dSW.at(l) + (size_t)h * n;
+    float* rc_o = out.rn_cur.at(l) + (size_t)h * out.cur_pad;
+    for (int it = g; it < ntiles; it += 2) {
+      const uint32_t ua = (uint32_t)(it >> 1);
+      if (!warp_wait(b_accfull + 8 * g, ua & 1u, err, abort_flag)) break;
+      tc_fence_after();
+      int f, t0;
+      css_tile(ft, blockIdx.x + it * gridDim.x, f, t0);
+      const int gw = ft.gw[f];
+      const int dd[5] = {0, 1, gw - 1, gw, gw + 1};
+      float val[5] = {0.f, 0.f, 0.f, 0.f, 0.f};
+      const int nch = (32 + gw + 1 + 31) >> 5;  // row i needs columns i .. i+gw+1
+      // park a 32-column chunk in this lane's staging row and pick the
+      // diagonals that fall in it
+      auto pick = [&](const uint32_t (&w)[32], int c) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+          *reinterpret_cast<uint4*>(stg + 4 * k) = make_uint4(w[4 * k], w[4 * k + 1], w[4 * k + 2], w[4 * k + 3]);
+#pragma unroll
+        for (int q = 0; q < 5; ++q) {
+          const int idx = lane + dd[q] - 32 * c;
+          if (idx >= 0 && idx < 32) val[q] = stg[idx];
+        }
+      };
+      if (nch <= 3) {
+        // every load of the window in flight at once (grids up to 63 wide)
+        uint32_t w0[32], w1[32], w2[32];
+        tmem_ld32_issue(tbase, w0);
+        if (nch > 1) tmem_ld32_issue(tbase + 32, w1);
+        if (nch > 2) tmem_ld32_issue(tbase + 64, w2);
+        tmem_wait_regs96(w0, w1, w2);
+        pick(w0, 0);
+        if (nch > 1) pick(w1, 1);
+        if (nch > 2) pick(w2, 2);
+      } else {
+        for (int c = 0; c < nch; ++c) {
+          uint32_t w0[32], w1[32], w2[32];
+          tmem_ld32_issue(tbase + c * 32, w0);
+          tmem_wait_regs96(w0, w1, w2);
+          pick(w0, c);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(b_accempty + 8 * g);
+      const int tok = t0 + quarter * 32 + lane;
+      if (tok < ft.off[f] + ft.gh[f] * gw) {
+        const float r = 1.0f / fmaxf(sqrtf(val[0]), 1e-8f);
+        rn_o[tok] = r;
+        e_o[tok] = val[1];
+        sw_o[tok] = val[2];
+        s_o[tok] = val[3];
+        se_o[tok] = val[4];
+        if (f == ft.n_frames - 1) rc_o[tok - ft.cur_off] = r;
+      }
+    }
+  }
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// Phi from the per-token dots: the eight in-grid Moore neighbours of (u, v)
+// are E, W, S, N, SE, NW, SW, NE; W's dot is E of the left neighbour, N's is
+// S of the upper one, NW's is SE of the upper-left one and NE's is SW of the
+// upper-right one.  grid = (cell block, frame, layer*Hkv + head).
+__global__ void __launch_bounds__(256) k_css_phi(const __grid_constant__ FrameTable ft, int hkv, CssDots d,
+                                                 Strided<float> phi_all) {
+  const int f = blockIdx.y, l = blockIdx.z / hkv, h = blockIdx.z % hkv, n = ft.n_tokens;
+  if (f >= ft.n_frames) return;
+  const int gh = ft.gh[f], gw = ft.gw[f], off = ft.off[f];
+  const int cell = blockIdx.x * blockDim.x + threadIdx.x;
+  if (cell >= gh * gw) return;
+  const size_t hn = (size_t)h * n;
+  const float* rn = d.rn.at(l) + hn;
+  const float* e = d.dE.at(l) + hn;
+  const float* s = d.dS.at(l) + hn;
+  const float* se = d.dSE.at(l) + hn;
+  const float* sw = d.dSW.at(l) + hn;
+  const int u = cell / gw, v = cell - u * gw, j = off + cell;
+  const bool up = u > 0, dn = u + 1 < gh, lf = v > 0, rt = v + 1 < gw;
+  const float r0 = __ldg(rn + j);
+  float sum = 0.f;
+  int cnt = 0;
+  if (rt) { sum += __ldg(e + j) * r0 * __ldg(rn + j + 1); ++cnt; }
+  if (lf) { sum += __ldg(e + j - 1) * __ldg(rn + j - 1) * r0; ++cnt; }
+  if (dn) { sum += __ldg(s + j) * r0 * __ldg(rn + j + gw); ++cnt; }
+  if (up) { sum += __ldg(s + j - gw) * __ldg(rn + j - gw) * r0; ++cnt; }
+  if (dn && rt) { sum += __ldg(se + j) * r0 * __ldg(rn + j + gw + 1); ++cnt; }
+  if (up && lf) { sum += __ldg(se + j - gw - 1) * __ldg(rn + j - gw - 1) * r0; ++cnt; }
+  if (dn && lf) { sum += __ldg(sw + j) * r0 * __ldg(rn + j + gw - 1); ++cnt; }
+  if (up && rt) { sum += __ldg(sw + j - gw + 1) * __ldg(rn + j - gw + 1) * r0; ++cnt; }
+  phi_all.at(l)[hn + j] = cnt ? 1.0f - sum / (float)cnt : 0.0f;
+}
+
+// =========================================================================
 // host side
 
 static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -779,8 +1026,8 @@ int score_nsplit_max(const Problem& p) {
 int score_nsplit(const Problem& p) { return score_nsplit_max(p); }
 
 cudaError_t launch_tsg_umma(const Problem& p, const FrameTable& ft, const LayerPtrs& io,
-                            Strided<const float> rn, Strided<float> rho_part, uint32_t* err,
-                            cudaStream_t st) {
+                            Strided<const float> rn_cur, int cur_pad, Strided<float> rho_part,
+                            uint32_t* err, cudaStream_t st) {
   if (ft.n_frames < 2) return cudaSuccess;
   const int n_tiles = ft.tile0[ft.n_frames - 1];
   if (n_tiles == 0 || ft.cur_len == 0) return cudaSuccess;
@@ -794,7 +1041,7 @@ cudaError_t launch_tsg_umma(const Problem& p, const FrameTable& ft, const LayerP
   const int gx = pick_split(groups, n_tiles, sm_count());
   dim3 grid(gx, nchunk, p.L * p.hkv);
   TimingScope ts("tsg_umma", st);
-  k_tsg_umma<<<grid, kThreads, kTsgSmem, st>>>(local, ft, rn, rho_part, p.hkv, err);
+  k_tsg_umma<<<grid, kThreads, kTsgSmem, st>>>(local, ft, rn_cur, cur_pad, rho_part, p.hkv, err);
   return cudaGetLastError();
 }
 
@@ -824,6 +1071,45 @@ cudaError_t launch_score_umma(const Problem& p, const LayerPtrs& io, Strided<flo
   const int gx = pick_split(p.L * p.hkv, tiles, sm_count());
   TimingScope ts("colsum_umma", st);
   k_colsum_umma<<<dim3(gx, p.L * p.hkv), kThreads, L2.total, st>>>(m2, io, p, rowpart, nsplit, a_base, err);
+  return cudaGetLastError();
+}
+
+bool css_umma_supported(const FrameTable& ft) {
+  for (int f = 0; f < ft.n_frames; ++f)
+    if (ft.gw[f] > kCssMaxGw) return false;
+  return true;
+}
+
+cudaError_t launch_css_umma(const Problem& p, const FrameTable& ft, const LayerPtrs& io, Strided<float> phi,
+                            Strided<float> rn, Strided<float> rn_cur, int cur_pad, Strided<float> dE,
+                            Strided<float> dS, Strided<float> dSE, Strided<float> dSW, uint32_t* err,
+                            cudaStream_t st) {
+  const int tiles = ft.ctile0[ft.n_frames];
+  if (tiles == 0) return cudaSuccess;
+  KMaps maps;
+  cudaError_t e = make_kmaps(&maps, io, p.L, p.n, p.hkv, 128);
+  if (e != cudaSuccess) return e;
+  if ((e = cudaFuncSetAttribute(k_css_umma, cudaFuncAttributeMaxDynamicSharedMemorySize, kCssUmmaSmem)) !=
+      cudaSuccess)
+    return e;
+  CssDots d;
+  d.rn = rn;
+  d.dE = dE;
+  d.dS = dS;
+  d.dSE = dSE;
+  d.dSW = dSW;
+  d.rn_cur = rn_cur;
+  d.cur_pad = cur_pad;
+  const int gx = pick_split(p.L * p.hkv, tiles, sm_count());
+  {
+    TimingScope ts("css_umma", st);
+    k_css_umma<<<dim3(gx, p.L * p.hkv), kThreads, kCssUmmaSmem, st>>>(maps, ft, p.hkv, d, err);
+  }
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  int cmax = 1;
+  for (int f = 0; f < ft.n_frames; ++f) cmax = max(cmax, ft.gh[f] * ft.gw[f]);
+  TimingScope ts("css_phi", st);
+  k_css_phi<<<dim3((cmax + 255) / 256, ft.n_frames, p.L * p.hkv), 256, 0, st>>>(ft, p.hkv, d, phi);
   return cudaGetLastError();
 }
 
