@@ -144,6 +144,54 @@ def exps_per_layer() -> float:
     return 2.0 * W * (HQ // HKV) * N_TOK * HKV
 
 
+def mufu_peak_texp(peaks) -> float:
+    """ex2 throughput of the SM's special-function units: 32 results per
+    clock per SM on GB300 (ncu counts one xu warp-instruction per SM-clock
+    as its peak), 152 SMs, at the maximum SM clock."""
+    return 152 * 32 * peaks["sm_mhz"] * 1e6 / 1e12
+
+
+def kernel_roofline(name: str, t_launch: float, layers: int, budget: int, peaks) -> dict:
+    """Roofline of one launch of `name` (which covers `layers` layers):
+    algorithmic work per layer x layers / measured launch time, against the
+    bound that limits it.  Algorithmic bytes count each operand once (what a
+    perfectly fused kernel must move), not the intermediates this design
+    writes."""
+    tok_head = N_TOK * HKV
+    kbytes = tok_head * D * 2                      # every key once, bf16
+    kept = budget * HKV * D * 2                    # kept rows of K (or V)
+    if name.startswith("tsg"):
+        work = tsg_flops_per_layer()
+        ach = work * layers / t_launch / 1e12
+        return dict(bound="tensor", achieved=ach, peak=peaks["bf16"], unit="TFLOP/s", frac=ach / peaks["bf16"],
+                    frac_of_sustained=ach / peaks["bf16_sus"],
+                    work="2*N_hist*N_cur*d*H_kv = %.4g FLOP per layer x %d layers" % (work, layers))
+    if name.startswith(("rowstats", "colsum", "css_umma")):
+        # every key once; colsum and CSS also write one fp32 value per token and head
+        out = 0 if name.startswith("rowstats") else tok_head * 4
+        work = kbytes + out
+        ach = work * layers / t_launch / 1e9
+        d = dict(bound="hbm", achieved=ach, peak=peaks["hbm"], unit="GB/s", frac=ach / peaks["hbm"],
+                 work="%.4g bytes per layer (keys once%s) x %d layers"
+                      % (work, ", fp32 output per token and head" if out else "", layers))
+        if name.startswith(("rowstats", "colsum")):
+            ex = exps_per_layer() / 2 * layers / t_launch / 1e12
+            d["mufu"] = dict(achieved=ex, peak=mufu_peak_texp(peaks), unit="Texp/s",
+                             frac=ex / mufu_peak_texp(peaks))
+        return d
+    if name.startswith("css_phi"):
+        work = tok_head * (5 * 4 + 4)              # five dot products in, Phi out
+    elif name.startswith("select"):
+        work = tok_head * 3 * 4 + budget * HKV * 4  # A, Phi, rho in; indices out
+    elif name.startswith("gather"):
+        work = 4 * kept + budget * HKV * 4         # kept K, V rows in and out; indices
+    else:
+        work = kbytes
+    ach = work * layers / t_launch / 1e9
+    return dict(bound="hbm", achieved=ach, peak=peaks["hbm"], unit="GB/s", frac=ach / peaks["hbm"],
+                work="%.4g bytes per layer x %d layers" % (work, layers))
+
+
 # --------------------------------------------------------------- oracle arm
 
 def oracle_sample(wl, pool_stride: int = 16, q_heads: int = HQ // HKV):
@@ -343,29 +391,11 @@ def run_gpu(args):
     for k, (c, t) in ktimes.items():
         kernels[k]["share"] = t / tot
     dom = max(ktimes, key=lambda k: ktimes[k][1])
-    t_dom = ktimes[dom][1] / ktimes[dom][0] * 1e-3
-    lpl = L  # layers per launch (one batched call per step)
-    if dom.startswith("tsg"):
-        ach = tsg_flops_per_layer() * lpl / t_dom / 1e12
-        roof = dict(bound="tensor", achieved=ach, peak=peaks["bf16_sus"], unit="TFLOP/s",
-                    frac=ach / peaks["bf16_sus"], kernel=dom,
-                    work="2*N_hist*N_cur*d*H_kv = %.4g FLOP per layer x %d layers per launch"
-                         % (tsg_flops_per_layer(), lpl))
-    elif dom.startswith(("colsum", "rowstats")):
-        mufu_peak = 152 * 16 * peaks["sm_mhz"] * 1e6 / 1e12  # T exp2/s
-        ach = exps_per_layer() / 2 * lpl / t_dom / 1e12
-        roof = dict(bound="alu", achieved=ach, peak=mufu_peak, unit="Texp/s", frac=ach / mufu_peak, kernel=dom,
-                    work="w*G*N*H_kv = %.4g exp2 per layer x %d layers per launch" % (exps_per_layer() / 2, lpl))
-    elif dom.startswith("css"):
-        ach = N_TOK * HKV * D * 2 * lpl / t_dom / 1e9
-        roof = dict(bound="hbm", achieved=ach, peak=peaks["hbm"], unit="GB/s", frac=ach / peaks["hbm"], kernel=dom,
-                    work="reads every key once: N*H_kv*d*2 bytes per layer x %d layers per launch" % lpl)
-    else:
-        ach = alg_bytes_per_layer(budget) * lpl / t_dom / 1e9
-        roof = dict(bound="hbm", achieved=ach, peak=peaks["hbm"], unit="GB/s", frac=ach / peaks["hbm"], kernel=dom,
-                    work="S*(1+3*beta) bytes per layer x %d layers per launch" % lpl)
+    for k, (c, t) in ktimes.items():
+        kernels[k]["roofline"] = kernel_roofline(k, t / c * 1e-3, L, budget, peaks)
+    roof = dict(kernels[dom]["roofline"], kernel=dom)
     roof["traffic"] = traffic_for(dom)
-    roof["peak_source"] = peaks["source"] + (" sustained" if roof["unit"] == "TFLOP/s" else "")
+    roof["peak_source"] = peaks["source"] + (" burst" if roof["unit"] == "TFLOP/s" else "")
 
     # ---- end to end: host (pinned) inputs -> device -> compress -> host outputs
     e2e = None
@@ -450,7 +480,7 @@ def run_gpu(args):
                              frac=alg_bytes_per_layer(budget) * L / (ms * 1e-3) / 1e9 / peaks["hbm"],
                              bytes_per_layer=alg_bytes_per_layer(budget)),
                     tensor=dict(achieved_tflops=(tsg_flops_per_layer() + score_flops_per_layer()) * L / (ms * 1e-3) / 1e12,
-                                peak_tflops=peaks["bf16_sus"]),
+                                peak_tflops=peaks["bf16"]),
                     roofline=roof, kernels=kernels, gpu_launches=per_step_launches * args.steps,
                     clocks=dict(sm_mhz=clk["sm_mhz"], sm_max_mhz=clk["sm_max_mhz"], reasons=clk["reasons"],
                                 samples=clk["samples"]),

@@ -230,6 +230,31 @@ __device__ __forceinline__ void mul2(float a0, float a1, float b0, float b1, flo
       : "f"(a0), "f"(a1), "f"(b0), "f"(b1));
 }
 
+// Packed fused multiply-add, two lanes: (d0, d1) = (a0*b0 + c0, a1*b1 + c1),
+// each rounded as a scalar fmaf.
+__device__ __forceinline__ void fma2(float a0, float a1, float b0, float b1, float c0, float c1, float& d0,
+                                     float& d1) {
+  asm("{\n\t.reg .b64 x, y, z, w;\n\t"
+      "mov.b64 x, {%2, %3};\n\t"
+      "mov.b64 y, {%4, %5};\n\t"
+      "mov.b64 z, {%6, %7};\n\t"
+      "fma.rn.f32x2 w, x, y, z;\n\t"
+      "mov.b64 {%0, %1}, w;\n\t}"
+      : "=f"(d0), "=f"(d1)
+      : "f"(a0), "f"(a1), "f"(b0), "f"(b1), "f"(c0), "f"(c1));
+}
+
+// Packed addition, two lanes: (a0, a1) += (b0, b1), each rounded as a scalar add.
+__device__ __forceinline__ void add2(float& a0, float& a1, float b0, float b1) {
+  asm("{\n\t.reg .b64 x, y, z;\n\t"
+      "mov.b64 x, {%0, %1};\n\t"
+      "mov.b64 y, {%2, %3};\n\t"
+      "add.rn.f32x2 z, x, y;\n\t"
+      "mov.b64 {%0, %1}, z;\n\t}"
+      : "+f"(a0), "+f"(a1)
+      : "f"(b0), "f"(b1));
+}
+
 // max(a, b, c) in one instruction (inputs here are never NaN).
 __device__ __forceinline__ float max3(float a, float b, float c) {
   float d;

@@ -455,10 +455,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
 #pragma unroll
           for (int i = 0; i < 64; i += 4) {
-            s0 += ex2_approx(fmaf(__uint_as_float(b[i]), c, -mnc));
-            s1 += ex2_approx(fmaf(__uint_as_float(b[i + 1]), c, -mnc));
-            s2 += ex2_approx(fmaf(__uint_as_float(b[i + 2]), c, -mnc));
-            s3 += ex2_approx(fmaf(__uint_as_float(b[i + 3]), c, -mnc));
+            float x0, x1, x2, x3;
+            fma2(__uint_as_float(b[i]), __uint_as_float(b[i + 1]), c, c, -mnc, -mnc, x0, x1);
+            fma2(__uint_as_float(b[i + 2]), __uint_as_float(b[i + 3]), c, c, -mnc, -mnc, x2, x3);
+            add2(s0, s1, ex2_approx(x0), ex2_approx(x1));
+            add2(s2, s3, ex2_approx(x2), ex2_approx(x3));
           }
           l = (m == -CUDART_INF_F ? 0.f : l * ex2_approx((m - mn) * c)) + ((s0 + s1) + (s2 + s3));
           m = mn;
@@ -674,10 +675,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
               const float4 b = b4[i];
-              a0 += ex2_approx(fmaf(v[4 * i], c, b.x));
-              a1 += ex2_approx(fmaf(v[4 * i + 1], c, b.y));
-              a2 += ex2_approx(fmaf(v[4 * i + 2], c, b.z));
-              a3 += ex2_approx(fmaf(v[4 * i + 3], c, b.w));
+              float x0, x1, x2, x3;
+              fma2(v[4 * i], v[4 * i + 1], c, c, b.x, b.y, x0, x1);
+              fma2(v[4 * i + 2], v[4 * i + 3], c, c, b.z, b.w, x2, x3);
+              add2(a0, a1, ex2_approx(x0), ex2_approx(x1));
+              add2(a2, a3, ex2_approx(x2), ex2_approx(x3));
             }
           } else {
 #pragma unroll
@@ -976,14 +978,16 @@ static int sm_count() {
 // CTAs per work unit (1..cap): one wave when the units are fewer than the
 // SMs, else the split among 1..4 that fills whole waves best.
 static int pick_split(int units, int cap, int slots) {
+  // Splits s of each unit so that units * s CTAs (one per SM) fill whole
+  // waves as nearly as possible; among equal fills the fewest CTAs win.
   if (cap < 1) cap = 1;
-  if (units < slots) {
-    int s = (slots + units - 1) / units;
-    return s < cap ? s : cap;
-  }
+  const int even = (slots + units - 1) / units;
+  int smax = 4 * even;
+  if (smax < 4) smax = 4;
+  if (smax > cap) smax = cap;
   int best = 1;
   double best_eff = 0.0;
-  for (int s = 1; s <= 4 && s <= cap; ++s) {
+  for (int s = 1; s <= smax; ++s) {
     const long long ctas = (long long)units * s;
     const long long waves = (ctas + slots - 1) / slots;
     const double eff = (double)ctas / (double)(waves * slots);
