@@ -100,7 +100,12 @@ __device__ uint32_t cluster_select_desc(cg::cluster_group& cl, const uint32_t* k
     cl.sync();
     for (int b = tid; b < 256; b += blockDim.x) {
       uint32_t t = 0;
-      for (int r = 0; r < ncta; ++r) t += cl.map_shared_rank(hb, r)[b];
+      for (int r0 = 0; r0 < ncta; r0 += 4) {  // four remote reads in flight
+        uint32_t v[4];
+#pragma unroll
+        for (int r = 0; r < 4; ++r) v[r] = r0 + r < ncta ? cl.map_shared_rank(hb, r0 + r)[b] : 0u;
+        t += (v[0] + v[1]) + (v[2] + v[3]);
+      }
       sh.tot[b] = t;
     }
     __syncthreads();
@@ -137,58 +142,56 @@ __device__ uint32_t cluster_select_desc(cg::cluster_group& cl, const uint32_t* k
   return prefix;
 }
 
-// Calls fn(i) for the tokens of [j0, j1) inside a frame's visual span, for
-// the frames [f0, f1), block-strided.  Only frames that overlap [j0, j1) are
-// visited (binary search for the first; the frame loop is uniform).
-template <class Fn>
-__device__ __forceinline__ void for_spans(const FrameTable& ft, int f0, int f1, int j0, int j1, Fn fn) {
-  int lo = f0, hi = f1 - 1, first = f1;
-  while (lo <= hi) {  // first frame whose span ends after j0
+// Inputs of one pool token's rho: the row maxima of the TSG slices (folded
+// into four) and 1/|k_i|.
+struct RhoIn {
+  float s[4];
+  float rn;
+};
+
+// Token kinds of the flat loops.
+constexpr int kTokText = 0;  // not inside any frame's visual span
+constexpr int kTokPool = 1;  // visual token of a historical frame (the TSG pool)
+constexpr int kTokCur = 2;   // visual token of the current (last) frame
+
+// Visits the tokens j0 + threadIdx.x + k * blockDim.x of [j0, j1) in
+// batches of U per thread: load(t, kind) runs for the whole batch before
+// use(t, kind, value) runs for any of it, so the batch's memory latencies
+// overlap.  Each thread tracks the frame of its (increasing) tokens.
+template <int U, class Load, class Use>
+__device__ __forceinline__ void for_tokens(const FrameTable& ft, int j0, int j1, Load load, Use use) {
+  const int B = blockDim.x, F = ft.n_frames;
+  int f = -1, lo = 0, hi = F - 1;
+  while (lo <= hi) {  // last frame starting at or before j0
     const int mid = (lo + hi) >> 1;
-    if (ft.off[mid] + ft.gh[mid] * ft.gw[mid] > j0) {
-      first = mid;
-      hi = mid - 1;
-    } else {
+    if (ft.off[mid] <= j0) {
+      f = mid;
       lo = mid + 1;
+    } else {
+      hi = mid - 1;
     }
   }
-  for (int f = first; f < f1 && ft.off[f] < j1; ++f) {
-    const int a = max(ft.off[f], j0), b = min(ft.off[f] + ft.gh[f] * ft.gw[f], j1);
-    for (int i = a + (int)threadIdx.x; i < b; i += blockDim.x) fn(i);
+  for (int base = j0 + (int)threadIdx.x; base < j1; base += U * B) {
+    int kind[U];
+    decltype(load(0, 0)) v[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int t = base + u * B;
+      kind[u] = -1;
+      if (t < j1) {
+        while (f + 1 < F && ft.off[f + 1] <= t) ++f;
+        const bool vis = f >= 0 && t < ft.off[f] + ft.gh[f] * ft.gw[f];
+        kind[u] = vis ? (f + 1 < F ? kTokPool : kTokCur) : kTokText;
+        v[u] = load(t, kind[u]);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+      if (kind[u] >= 0) use(base + u * B, kind[u], v[u]);
   }
 }
 
-// Same visiting order, four tokens per thread at a time: load(i) for all four
-// is issued before use(i, value) runs for any, so their latencies overlap.
-template <class Load, class Use>
-__device__ __forceinline__ void for_spans4(const FrameTable& ft, int f0, int f1, int j0, int j1, Load load,
-                                           Use use) {
-  int lo = f0, hi = f1 - 1, first = f1;
-  while (lo <= hi) {
-    const int mid = (lo + hi) >> 1;
-    if (ft.off[mid] + ft.gh[mid] * ft.gw[mid] > j0) {
-      first = mid;
-      hi = mid - 1;
-    } else {
-      lo = mid + 1;
-    }
-  }
-  const int B = blockDim.x;
-  for (int f = first; f < f1 && ft.off[f] < j1; ++f) {
-    const int a = max(ft.off[f], j0), b = min(ft.off[f] + ft.gh[f] * ft.gw[f], j1);
-    for (int i0 = a + (int)threadIdx.x; i0 < b; i0 += 4 * B) {
-      decltype(load(i0)) v[4];
-#pragma unroll
-      for (int u = 0; u < 4; ++u)
-        if (i0 + u * B < b) v[u] = load(i0 + u * B);
-#pragma unroll
-      for (int u = 0; u < 4; ++u)
-        if (i0 + u * B < b) use(i0 + u * B, v[u]);
-    }
-  }
-}
-
-__global__ void __launch_bounds__(kSelThreads) k_select(Problem p, const __grid_constant__ FrameTable ft,
+__global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __grid_constant__ FrameTable ft,
                                                         SelectArgs a) {
   extern __shared__ uint32_t keys[];
   __shared__ SelShared sh;
@@ -200,97 +203,116 @@ __global__ void __launch_bounds__(kSelThreads) k_select(Problem p, const __grid_
   const size_t hn = (size_t)h * n;
   const int F = ft.n_frames;
   int pass = 0;
+  int pool = 0;
+  for (int f = 0; f + 1 < F; ++f) pool += ft.gh[f] * ft.gw[f];
+  // tau comes from a selection only when there is a pool and TSG is on;
+  // otherwise tau = NaN and every gate stays open
+  const bool gate_sel = (a.mode & kSelGate) && pool > 0 && a.tsg_enable;
+  float tau = CUDART_NAN_F;
+  uint8_t* gate = a.gate.base ? a.gate.at(l) + hn : nullptr;
 
   if (a.mode & kSelGate) {
     float* rho = a.rho.at(l) + hn;
-    uint8_t* gate = a.gate.at(l) + hn;
-    const float* rp = a.rho_part.at(l);
+    const float* rp = a.rho_part.at(l) + hn;
     const float* rn = a.rn.at(l) + hn;
-    for (int i = tid; i < len; i += blockDim.x) {
-      rho[j0 + i] = CUDART_NAN_F;
-      gate[j0 + i] = 1;
-      keys[i] = 0u;
-    }
-    __syncthreads();
-    int pool = 0;
-    for (int f = 0; f + 1 < F; ++f) pool += ft.gh[f] * ft.gw[f];
     const size_t slice = (size_t)p.hkv * n;
-    for_spans4(
-        ft, 0, F - 1, j0, j1,
-        [&](int i) {
-          const float* src = rp + hn + i;
-          float m0 = -CUDART_INF_F, m1 = -CUDART_INF_F;
-          int s = 0;
-          for (; s + 1 < a.nchunk; s += 2) {
-            m0 = fmaxf(m0, __ldg(src + (size_t)s * slice));
-            m1 = fmaxf(m1, __ldg(src + (size_t)(s + 1) * slice));
+    const int nsl = a.nchunk;
+    // rho of every token: pool tokens from the TSG slices and 1/|k_i|, NaN
+    // elsewhere; the selection keys are complements (m-th smallest rho ==
+    // m-th largest key), 0 marks a token outside the pool
+    for_tokens<2>(
+        ft, j0, j1,
+        [&](int t, int kind) {
+          // independent loads (no max between them), so that all of a
+          // batch's slices are in flight together
+          RhoIn r;
+#pragma unroll
+          for (int s = 0; s < 4; ++s) r.s[s] = -CUDART_INF_F;
+          r.rn = CUDART_NAN_F;
+          if (kind == kTokPool) {
+            const float* src = rp + t;
+#pragma unroll
+            for (int s = 0; s < 4; ++s)
+              if (s < nsl) r.s[s] = __ldg(src + (size_t)s * slice);
+            for (int s = 4; s < nsl; ++s) r.s[3] = fmaxf(r.s[3], __ldg(src + (size_t)s * slice));
+            r.rn = __ldg(rn + t);
           }
-          if (s < a.nchunk) m0 = fmaxf(m0, __ldg(src + (size_t)s * slice));
-          return make_float2(fmaxf(m0, m1), __ldg(rn + i));
+          return r;
         },
-        [&](int i, float2 v) {
-          const float r = v.x * v.y;
-          rho[i] = r;
-          keys[i - j0] = ~float_key(r);  // m-th smallest == m-th largest complement
+        [&](int t, int kind, const RhoIn& v) {
+          const float m = fmaxf(fmaxf(v.s[0], v.s[1]), fmaxf(v.s[2], v.s[3]));
+          const float r = kind == kTokPool ? m * v.rn : CUDART_NAN_F;
+          rho[t] = r;
+          keys[t - j0] = kind == kTokPool ? ~float_key(r) : 0u;
         });
     __syncthreads();
-    if (pool > 0 && a.tsg_enable) {
+    if (gate_sel) {
       uint32_t need;
       const uint32_t kt = cluster_select_desc(cl, keys, len, (uint32_t)min(a.budget, pool), sh, pass, &need);
-      const float tau = key_float(~kt);
-      for_spans(ft, 0, F - 1, j0, j1, [&](int i) { gate[i] = key_float(~keys[i - j0]) <= tau ? 1 : 0; });
-      if (c == 0 && tid == 0) a.tau.at(l)[h] = tau;
-    } else if (c == 0 && tid == 0) {
-      a.tau.at(l)[h] = CUDART_NAN_F;
+      tau = key_float(~kt);
     }
-    __syncthreads();
+    if (c == 0 && tid == 0) a.tau.at(l)[h] = tau;
+    if (!(a.mode & kSelTopk)) {
+      // gate only: Eq. 8 on the pool, open elsewhere
+      for_tokens<2>(
+          ft, j0, j1, [&](int, int) { return 0; },
+          [&](int t, int kind, int) {
+            gate[t] = (kind == kTokPool && gate_sel) ? (key_float(~keys[t - j0]) <= tau ? 1 : 0) : 1;
+          });
+    }
   }
 
   if (a.mode & kSelTopk) {
     const float* ab = a.a_base.at(l) + hn;
     const float* ph = a.phi.base ? a.phi.at(l) + hn : nullptr;
-    const uint8_t* gt = a.gate.base ? a.gate.at(l) + hn : nullptr;
+    const uint8_t* gt = gate;
     float* sc = a.score.at(l) + hn;
     const float alpha = a.css_enable ? a.alpha : 0.f;
-    // text tokens: S = A_base; visual tokens are overwritten below
-    for (int i0 = tid; i0 < len; i0 += 4 * blockDim.x) {
-      float v[4];
-#pragma unroll
-      for (int u = 0; u < 4; ++u)
-        if (i0 + u * (int)blockDim.x < len) v[u] = __ldg(ab + j0 + i0 + u * blockDim.x);
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int i = i0 + u * blockDim.x;
-        if (i < len) {
-          const float s = v[u] + 0.0f;
-          sc[j0 + i] = s;
-          keys[i] = float_key(s);
-        }
-      }
-    }
-    __syncthreads();
-    for_spans4(
-        ft, 0, F, j0, j1,
-        [&](int j) {
-          const float x = __ldg(ab + j) + (alpha != 0.f ? alpha * __ldg(ph + j) : 0.f);
-          return (gt == nullptr || gt[j]) ? x : 0.f;
+    const bool fused = (a.mode & kSelGate) != 0;  // gate decided here from the rho keys
+    // Eq. 9: S = A_base for text tokens; for visual tokens S = A_base +
+    // alpha * Phi where the gate is open and 0 where it is closed
+    for_tokens<2>(
+        ft, j0, j1,
+        [&](int t, int kind) {
+          const float A = __ldg(ab + t);
+          const float P = (kind != kTokText && alpha != 0.f) ? __ldg(ph + t) : 0.f;
+          const float G = (kind != kTokText && !fused && gt != nullptr) ? (float)gt[t] : 1.f;
+          return make_float3(A, P, G);
         },
-        [&](int j, float x) {
-          const float s = x + 0.0f;
-          sc[j] = s;
-          keys[j - j0] = float_key(s);
+        [&](int t, int kind, float3 v) {
+          float s;
+          if (kind == kTokText) {
+            s = v.x + 0.0f;
+            if (fused) gate[t] = 1;
+          } else {
+            bool g = v.z != 0.f;
+            if (fused) {
+              g = !(kind == kTokPool && gate_sel) || key_float(~keys[t - j0]) <= tau;
+              gate[t] = g ? 1 : 0;
+            }
+            const float x = alpha != 0.f ? __fmaf_rn(alpha, v.y, v.x) : v.x;
+            s = (g ? x : 0.f) + 0.0f;
+          }
+          sc[t] = s;
+          keys[t - j0] = float_key(s);
         });
     __syncthreads();
     uint32_t need;
     const uint32_t T = cluster_select_desc(cl, keys, len, (uint32_t)a.budget, sh, pass, &need);
-    // this CTA's counts, then its offsets from the lower-ranked CTAs
+    // Ordered compaction.  Thread tid owns the contiguous run [r0, r1) of
+    // this CTA's keys (odd run length: conflict-free shared reads); one
+    // block scan gives its (greater, equal) counts before the run, the
+    // cluster's lower ranks add theirs.
+    const int per = ((len + (int)blockDim.x - 1) / (int)blockDim.x) | 1;
+    const int r0 = min(len, tid * per), r1 = min(len, r0 + per);
     uint32_t g_loc = 0, e_loc = 0;
-    for (int i = tid; i < len; i += blockDim.x) {
-      g_loc += keys[i] > T;
-      e_loc += keys[i] == T;
+    for (int i = r0; i < r1; ++i) {
+      const uint32_t k = keys[i];
+      g_loc += k > T;
+      e_loc += k == T;
     }
     uint32_t tot;
-    block_exclusive_scan(g_loc | (e_loc << 16), sh.warp_tot, &tot);
+    const uint32_t ex = block_exclusive_scan(g_loc | (e_loc << 16), sh.warp_tot, &tot);
     if (tid == 0) {
       sh.counts[0] = tot & 0xffffu;
       sh.counts[1] = tot >> 16;
@@ -307,17 +329,19 @@ __global__ void __launch_bounds__(kSelThreads) k_select(Problem p, const __grid_
       sh.bcast[3] = eb;
     }
     __syncthreads();
-    uint32_t run_gt = sh.bcast[2], run_eq = sh.bcast[3];
+    uint32_t gt_before = sh.bcast[2] + (ex & 0xffffu), eq_before = sh.bcast[3] + (ex >> 16);
     int32_t* out = a.idx[l] + (size_t)h * a.budget;
-    for (int base = 0; base < len; base += blockDim.x) {
-      const int i = base + tid;
-      const uint32_t key = i < len ? keys[i] : 0u;
-      const bool g = i < len && key > T, e = i < len && key == T;
-      const uint32_t ex = block_exclusive_scan((g ? 1u : 0u) | (e ? 0x10000u : 0u), sh.warp_tot, &tot);
-      const uint32_t gt_before = run_gt + (ex & 0xffffu), eq_before = run_eq + (ex >> 16);
-      if (g || (e && eq_before < need)) out[gt_before + min(eq_before, need)] = j0 + i;
-      run_gt += tot & 0xffffu;
-      run_eq += tot >> 16;
+    // kept: every key > T, and the first `need` keys == T in index order;
+    // a kept token's slot = kept tokens before it
+    for (int i = r0; i < r1; ++i) {
+      const uint32_t k = keys[i];
+      if (k > T) {
+        out[gt_before + min(eq_before, need)] = j0 + i;
+        ++gt_before;
+      } else if (k == T) {
+        if (eq_before < need) out[gt_before + eq_before] = j0 + i;
+        ++eq_before;
+      }
     }
   }
   cl.sync();  // no CTA leaves while a peer may still read its shared memory
@@ -325,29 +349,54 @@ __global__ void __launch_bounds__(kSelThreads) k_select(Problem p, const __grid_
 
 int select_max_tokens() { return kSelMaxCluster * kSelMaxChunk; }
 
-cudaError_t launch_select(const Problem& p, const FrameTable& ft, const SelectArgs& a, cudaStream_t st) {
-  // smallest cluster whose CTAs hold their keys in shared memory, grown
-  // (up to 8) while the launch does not fill one wave of the SMs
-  int cl = 1;
-  while ((p.n + cl - 1) / cl > kSelMaxChunk) cl <<= 1;
-  if (cl > kSelMaxCluster) return cudaErrorNotSupported;
-  while (cl < kSelMaxCluster && p.L * p.hkv * cl * 2 <= 152) cl <<= 1;
-  const int chunk = (p.n + cl - 1) / cl;
-  cudaError_t e = cudaFuncSetAttribute(k_select, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)(kSelMaxChunk * 4));
-  if (e != cudaSuccess) return e;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(cl, p.L * p.hkv, 1);
-  cfg.blockDim = dim3(kSelThreads, 1, 1);
-  cfg.dynamicSmemBytes = (size_t)chunk * 4;
-  cfg.stream = st;
-  cudaLaunchAttribute attr[1];
+static void select_config(cudaLaunchConfig_t* cfg, cudaLaunchAttribute* attr, const Problem& p, int cl,
+                          cudaStream_t st) {
+  *cfg = cudaLaunchConfig_t{};
+  cfg->gridDim = dim3(cl, p.L * p.hkv, 1);
+  cfg->blockDim = dim3(kSelThreads, 1, 1);
+  cfg->dynamicSmemBytes = (size_t)((p.n + cl - 1) / cl) * 4;
+  cfg->stream = st;
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = cl;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg->attrs = attr;
+  cfg->numAttrs = 1;
+}
+
+cudaError_t launch_select(const Problem& p, const FrameTable& ft, const SelectArgs& a, cudaStream_t st) {
+  // Cluster size: the CTAs of a cluster split one (layer, head)'s tokens.
+  // Each CTA is latency-bound on its own chunk, so the estimated time is
+  // (waves of co-resident clusters) x (chunk length); the smallest cluster
+  // with the lowest estimate wins (fewer CTAs per cluster barrier).
+  cudaError_t e = cudaFuncSetAttribute(k_select, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)(kSelMaxChunk * 4));
+  if (e != cudaSuccess) return e;
+  // all of the SM's configurable memory as shared memory: the CTAs' keys
+  // are what limits how many clusters are resident
+  e = cudaFuncSetAttribute(k_select, cudaFuncAttributePreferredSharedMemoryCarveout,
+                           (int)cudaSharedmemCarveoutMaxShared);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg;
+  cudaLaunchAttribute attr[1];
+  int cl = 0;
+  long long best = 0;
+  for (int c = 1; c <= kSelMaxCluster; c <<= 1) {
+    const int ch = (p.n + c - 1) / c;
+    if (ch > kSelMaxChunk) continue;
+    select_config(&cfg, attr, p, c, st);
+    int fit = 0;
+    if ((e = cudaOccupancyMaxActiveClusters(&fit, k_select, &cfg)) != cudaSuccess) return e;
+    if (fit < 1) continue;
+    const long long units = (long long)p.L * p.hkv;
+    const long long est = (units + fit - 1) / fit * ch;
+    if (cl == 0 || est < best) {
+      cl = c;
+      best = est;
+    }
+  }
+  if (cl == 0) return cudaErrorNotSupported;
+  select_config(&cfg, attr, p, cl, st);
   TimingScope ts(a.mode & kSelGate ? (a.mode & kSelTopk ? "select_gate_topk" : "select_gate") : "select_topk", st);
   e = cudaLaunchKernelEx(&cfg, k_select, p, ft, a);
   if (e != cudaSuccess) return e;
