@@ -214,7 +214,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         float mx = -CUDART_INF_F;
         if (valid_g == 256) {
           // full stage: no masked column, packed products and 3-input max
-          float m0 = -CUDART_INF_F, m1 = -CUDART_INF_F;
+          // into eight independent running maxima (short dependency chains)
+          float m[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) m[i] = -CUDART_INF_F;
 #pragma unroll 1
           for (int c = 0; c < 4; ++c) {
             float v[64];
@@ -226,11 +229,11 @@ __global__ void __launch_bounds__(kThreads, 1)
               float p0, p1, p2, p3;
               mul2(v[4 * i], v[4 * i + 1], r.x, r.y, p0, p1);
               mul2(v[4 * i + 2], v[4 * i + 3], r.z, r.w, p2, p3);
-              m0 = max3(m0, p0, p1);
-              m1 = max3(m1, p2, p3);
+              m[(2 * i) & 7] = max3(m[(2 * i) & 7], p0, p1);
+              m[(2 * i + 1) & 7] = max3(m[(2 * i + 1) & 7], p2, p3);
             }
           }
-          mx = fmaxf(m0, m1);
+          mx = fmaxf(fmaxf(max3(m[0], m[1], m[2]), max3(m[3], m[4], m[5])), fmaxf(m[6], m[7]));
         } else {
           // ragged stage: columns past the frame carry rn = NaN, ignored by fmaxf
           for (int c = 0; c < 8; ++c) {
@@ -302,7 +305,7 @@ struct RsLayout {
 __host__ __device__ inline RsLayout rs_layout(int R) {
   RsLayout L;
   L.MT = R <= 128 ? 1 : (R <= 256 ? 2 : 4);
-  L.KN = 256 / L.MT;
+  L.KN = L.MT <= 2 ? 256 : 128;  // keys per tile = MMA N of one (m-tile, key tile) item
   L.q_bytes = L.MT * 128 * 256;
   L.k_stage_bytes = L.KN * 256;
   const int fixed = L.q_bytes + kScoreBarBytes + L.MT * 128 * 8 + 1024;
@@ -332,7 +335,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = align1024(smem_raw);
   const RsLayout L = rs_layout(p.R());
-  constexpr int KN = 256 / MT;
+  constexpr int KN = MT <= 2 ? 256 : 128;
   const int R = p.R();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int split = blockIdx.x, layer = blockIdx.y / p.hkv, h = blockIdx.y % p.hkv, n = p.n;
@@ -342,6 +345,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int per = (((n + nsplit - 1) / nsplit) + KN - 1) / KN * KN;
   const int j0 = split * per, j1 = min(n, j0 + per);
   const int ntiles = j1 > j0 ? (j1 - j0 + KN - 1) / KN : 0;
+  const int nitems = ntiles * MT;
   const uint32_t sQ = smem_u32(sm), sK = smem_u32(sm + L.off_k);
   const ScoreBars bb = score_bars(sm + L.off_bar);
   const uint32_t b_kfull = bb.kfull, b_kempty = bb.kempty, b_accfull = bb.accfull;
@@ -359,7 +363,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(b_accfull + 8 * i, 1);
-      mbar_init(b_accempty + 8 * i, 4);
+      mbar_init(b_accempty + 8 * i, 8);  // both epilogue groups
     }
     mbar_init(b_done, 1);
     *abort_flag = 0u;
@@ -376,12 +380,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *slot;
 
-  // per-thread row state for up to 4 M-tiles (epilogue warps)
-  float m_st[MT], l_st[MT];
+  // Work items u = t * MT + mt: m-tile mt of Q against key tile t, into
+  // TMEM slot u % 2 (KN columns).  Both epilogue groups drain every item,
+  // group g taking key columns [g*KN/2, (g+1)*KN/2), so that one item drains
+  // while the MMA fills the other slot.  Each group keeps a row state per
+  // m-tile, (running max m in raw dot units, l = sum 2^((x - m) c)); the two
+  // groups' states are merged at the end.
+  float ms[MT], ls[MT];
 #pragma unroll
   for (int i = 0; i < MT; ++i) {
-    m_st[i] = -CUDART_INF_F;
-    l_st[i] = 0.f;
+    ms[i] = -CUDART_INF_F;
+    ls[i] = 0.f;
   }
   const int g = warp >= 2 ? (warp - 2) >> 2 : 0, quarter = warp & 3;
 
@@ -405,52 +414,69 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1) {
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16(128, KN);
-      for (int it = 0; it < ntiles; ++it) {
-        const int s = it % S, as = it & 1;
-        const uint32_t u = (uint32_t)(it / S), ua = (uint32_t)(it >> 1);
-        if (!mbar_wait(b_kfull + 8 * s, u & 1u, err, abort_flag)) break;
-        if (!mbar_wait(b_accempty + 8 * as, (ua & 1u) ^ 1u, err, abort_flag)) break;
-        tc_fence_after();
-        for (int mt = 0; mt < MT; ++mt) {
+      bool ok = true;
+      int u = 0;
+      for (int it = 0; ok && it < ntiles; ++it) {
+        const int s = it % S;
+        if (!mbar_wait(b_kfull + 8 * s, (uint32_t)(it / S) & 1u, err, abort_flag)) break;
+        for (int mt = 0; mt < MT; ++mt, ++u) {
+          const int as = u & 1;
+          if (!mbar_wait(b_accempty + 8 * as, ((uint32_t)(u >> 1) & 1u) ^ 1u, err, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
 #pragma unroll
           for (int k = 0; k < 8; ++k) {
             const uint32_t kb = k >> 2, koff = (k & 3) * 32;
             uint64_t ad = desc_sw128(sQ + kb * (MT * 128 * 128) + mt * 128 * 128 + koff);
             uint64_t bd = desc_sw128(sK + s * L.k_stage_bytes + kb * (KN * 128) + koff);
-            umma_bf16(tmem + as * 256 + mt * KN, ad, bd, idesc, k > 0 ? 1u : 0u);
+            umma_bf16(tmem + as * 256, ad, bd, idesc, k > 0 ? 1u : 0u);
           }
+          umma_commit(b_accfull + 8 * as);
         }
-        umma_commit(b_accfull + 8 * as);
+        if (!ok) break;
         umma_commit(b_kempty + 8 * s);
       }
       umma_commit(b_done);
       mbar_wait_drain(b_done, 0);
     }
   } else {
-    const uint32_t lanebase = tmem + ((uint32_t)(quarter * 32) << 16);
-    for (int it = g; it < ntiles; it += 2) {
-      const uint32_t u = (uint32_t)(it >> 1);
-      if (!warp_wait(b_accfull + 8 * g, u & 1u, err, abort_flag)) break;
+    constexpr int HALF = KN / 2;  // key columns per group and item
+    const uint32_t lanebase = tmem + ((uint32_t)(quarter * 32) << 16) + g * HALF;
+    for (int u = 0; u < nitems; ++u) {
+      const int as = u & 1;
+      if (!warp_wait(b_accfull + 8 * as, (uint32_t)(u >> 1) & 1u, err, abort_flag)) break;
       tc_fence_after();
-      const int tok = j0 + it * KN;
-      // a tile is always four 64-column chunks (MT m-tiles x KN/64 key
-      // chunks); chunk q+1 loads from TMEM while chunk q is reduced
-      uint32_t b0[64], b1[64];
+      const int t = u / MT, mt = u % MT;
+      float m = ms[0], l = ls[0];
+#pragma unroll
+      for (int i = 1; i < MT; ++i)
+        if (mt == i) {
+          m = ms[i];
+          l = ls[i];
+        }
+      const int tok = j0 + t * KN + g * HALF;
+      // 64-column chunks in key order; chunk q+1 loads from TMEM while
+      // chunk q is reduced
       auto online = [&](const uint32_t (&b)[64], int q) {
-        const int mt = q / (KN / 64), kbase = tok + (q % (KN / 64)) * 64;
+        const int kbase = tok + q * 64;
         const int nv = min(64, j1 - kbase);
         if (nv <= 0) return;
-        float m = m_st[mt], l = l_st[mt];
         if (nv == 64) {
-          // indices 0..63: c0 takes 0, 2..3, 6..7, ..., 62..63; c1 takes 1, 4..5, ..., 60..61
-          float c0 = __uint_as_float(b[0]), c1 = __uint_as_float(b[1]);
+          // chunk maximum over four independent chains: chain r starts at
+          // element r and takes pairs 4 + 2r + 8i, 5 + 2r + 8i (i = 0..7)
+          float cm[4];
 #pragma unroll
-          for (int i = 2; i < 62; i += 4) {
-            c0 = max3(c0, __uint_as_float(b[i]), __uint_as_float(b[i + 1]));
-            c1 = max3(c1, __uint_as_float(b[i + 2]), __uint_as_float(b[i + 3]));
+          for (int r = 0; r < 4; ++r) cm[r] = __uint_as_float(b[r]);
+#pragma unroll
+          for (int i = 4; i < 64; i += 8) {
+#pragma unroll
+            for (int r = 0; r < 4; ++r)
+              if (i + 2 * r + 1 < 64)
+                cm[r] = max3(cm[r], __uint_as_float(b[i + 2 * r]), __uint_as_float(b[i + 2 * r + 1]));
           }
-          c0 = max3(c0, __uint_as_float(b[62]), __uint_as_float(b[63]));
-          const float mn = fmaxf(m, fmaxf(c0, c1));
+          const float mn = fmaxf(m, fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3])));
           const float mnc = mn * c;
           float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
 #pragma unroll
@@ -477,31 +503,35 @@ __global__ void __launch_bounds__(kThreads, 1)
           l = (m == -CUDART_INF_F ? 0.f : l * ex2_approx((m - mn) * c)) + sacc;
           m = mn;
         }
-        m_st[mt] = m;
-        l_st[mt] = l;
       };
-      const uint32_t tb = lanebase + g * 256;
+      const uint32_t tb = lanebase + as * 256;
+      uint32_t b0[64];
       tmem_ld64_issue(tb, b0);
       tmem_ld64_wait(b0);
-      tmem_ld64_issue(tb + 64, b1);
-      online(b0, 0);
-      tmem_ld64_wait(b1);
-      tmem_ld64_issue(tb + 128, b0);
-      online(b1, 1);
-      tmem_ld64_wait(b0);
-      tmem_ld64_issue(tb + 192, b1);
-      online(b0, 2);
-      tmem_ld64_wait(b1);
-      online(b1, 3);
+      if (HALF == 128) {
+        uint32_t b1[64];
+        tmem_ld64_issue(tb + 64, b1);
+        online(b0, 0);
+        tmem_ld64_wait(b1);
+        online(b1, 1);
+      } else {
+        online(b0, 0);
+      }
+#pragma unroll
+      for (int i = 0; i < MT; ++i)
+        if (mt == i) {
+          ms[i] = m;
+          ls[i] = l;
+        }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(b_accempty + 8 * g);
+      if (lane == 0) mbar_arrive(b_accempty + 8 * as);
     }
   }
-  // merge the two epilogue groups, then write (m * c, l) per query row
+  // merge the two groups' states, then write (m * c, l) per query row
   if (warp >= 2 && g == 1) {
 #pragma unroll
-    for (int mt = 0; mt < MT; ++mt) xch[mt * 128 + quarter * 32 + lane] = make_float2(m_st[mt], l_st[mt]);
+    for (int mt = 0; mt < MT; ++mt) xch[mt * 128 + quarter * 32 + lane] = make_float2(ms[mt], ls[mt]);
   }
   tc_fence_before();
   __syncthreads();
@@ -509,8 +539,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
     for (int mt = 0; mt < MT; ++mt) {
       const int row = mt * 128 + quarter * 32 + lane;
-      float2 o = xch[row];
-      float m = m_st[mt], l = l_st[mt];
+      const float2 o = xch[row];
+      float m = ms[mt], l = ls[mt];
       online_merge(m, l, o.x, o.y, c);
       if (row < R) part[((size_t)h * nsplit + split) * R + row] = make_float2(m * c, l);
     }
