@@ -558,8 +558,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 // query rows of its key.  TMEM: two stages of NQ columns when NQ <= 256
 // (epilogue group g takes the tiles with it % 2 == g), else one stage.
 struct CsLayout {
-  int NQ, nstage, kstages, tmem_cols, q_bytes, off_k, off_bias, off_bar, total;
+  int NQ, nstage, kstages, tmem_cols, q_bytes, off_k, off_bias, off_bar, off_xch, total;
 };
+constexpr int kCsXchBytes = 2 * 128 * 4 + 64;  // two partial-sum buffers, then xfull[2], xempty[2]
 __host__ __device__ inline CsLayout cs_layout(int R) {
   CsLayout L;
   L.NQ = (R + 31) & ~31;
@@ -567,14 +568,15 @@ __host__ __device__ inline CsLayout cs_layout(int R) {
   L.tmem_cols = 32;
   while (L.tmem_cols < L.nstage * L.NQ) L.tmem_cols <<= 1;
   L.q_bytes = L.NQ * 256;
-  const int fixed = L.q_bytes + L.NQ * 4 + kScoreBarBytes + 1024;
+  const int fixed = L.q_bytes + L.NQ * 4 + kScoreBarBytes + kCsXchBytes + 1024;
   L.kstages = (kScoreSmemCap - fixed) / 32768;
   if (L.kstages > kMaxKStages) L.kstages = kMaxKStages;
   if (L.kstages < 2) L.kstages = 2;
   L.off_k = L.q_bytes;
   L.off_bias = L.off_k + L.kstages * 32768;
   L.off_bar = L.off_bias + L.NQ * 4;
-  L.total = L.off_bar + kScoreBarBytes + 1024;
+  L.off_xch = L.off_bar + kScoreBarBytes;
+  L.total = L.off_xch + kCsXchBytes + 1024;
   return L;
 }
 
@@ -601,6 +603,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile uint32_t* abort_flag = bb.abort_flag;
   const int S = L.kstages;
   const float c = kLog2eF * rsqrtf((float)kD);
+  float* xch = reinterpret_cast<float*>(sm + L.off_xch);
+  uint64_t* xbars = reinterpret_cast<uint64_t*>(sm + L.off_xch + 2 * 128 * 4);
+  const uint32_t b_xfull = smem_u32(&xbars[0]), b_xempty = smem_u32(&xbars[2]);
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < S; ++i) {
@@ -609,7 +614,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(b_accfull + 8 * i, 1);
-      mbar_init(b_accempty + 8 * i, 4);
+      mbar_init(b_accempty + 8 * i, 8);  // both epilogue groups
+      mbar_init(b_xfull + 8 * i, 4);
+      mbar_init(b_xempty + 8 * i, 4);
     }
     mbar_init(b_done, 1);
     *abort_flag = 0u;
@@ -688,48 +695,70 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_wait_drain(b_done, 0);
     }
   } else {
-    const int g = (warp - 2) >> 2, quarter = warp & 3;
-    if (g < nstage) {
-      const uint32_t tbase = tmem + ((uint32_t)(quarter * 32) << 16) + g * NQ;
-      for (int it = g; it < ntiles; it += nstage) {
-        const uint32_t ua = (uint32_t)(it / nstage);
-        if (!warp_wait(b_accfull + 8 * g, ua & 1u, err, abort_flag)) break;
-        tc_fence_after();
-        float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+    // Both groups drain every tile: group 0 the query columns [0, sp),
+    // group 1 [sp, NQ); columns of padded rows carry bias = -inf, so they
+    // add exact zeros.  Group 1 passes its partial sum to group 0 through
+    // a double-buffered shared array (xfull / xempty barriers).
+    const int g = (warp - 2) >> 2, quarter = warp & 3, row = quarter * 32 + lane;
+    const int sp = min(NQ, ((NQ >> 1) + 63) & ~63);
+    const int c0 = g == 0 ? 0 : sp, c1 = g == 0 ? sp : NQ;
+    const uint32_t lanebase = tmem + ((uint32_t)(quarter * 32) << 16);
+    for (int it = 0; it < ntiles; ++it) {
+      const int as = it % nstage;
+      const uint32_t ua = (uint32_t)(it / nstage);
+      if (!warp_wait(b_accfull + 8 * as, ua & 1u, err, abort_flag)) break;
+      tc_fence_after();
+      const uint32_t tbase = lanebase + as * NQ;
+      float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+      int cb = c0;
 #pragma unroll 1
-        for (int cg = 0; cg < NQ / 64; ++cg) {
-          float v[64];
-          tmem_ld64(tbase + cg * 64, v);
-          const float4* b4 = reinterpret_cast<const float4*>(bias_s + cg * 64);
-          if (cg * 64 + 64 <= R) {
+      for (; cb + 64 <= c1; cb += 64) {
+        float v[64];
+        tmem_ld64(tbase + cb, v);
+        const float4* b4 = reinterpret_cast<const float4*>(bias_s + cb);
 #pragma unroll
-            for (int i = 0; i < 16; ++i) {
-              const float4 b = b4[i];
-              float x0, x1, x2, x3;
-              fma2(v[4 * i], v[4 * i + 1], c, c, b.x, b.y, x0, x1);
-              fma2(v[4 * i + 2], v[4 * i + 3], c, c, b.z, b.w, x2, x3);
-              add2(a0, a1, ex2_approx(x0), ex2_approx(x1));
-              add2(a2, a3, ex2_approx(x2), ex2_approx(x3));
-            }
-          } else {
-#pragma unroll
-            for (int i = 0; i < 64; ++i)
-              if (cg * 64 + i < R) a0 += ex2_approx(fmaf(v[i], c, bias_s[cg * 64 + i]));
-          }
+        for (int i = 0; i < 16; ++i) {
+          const float4 b = b4[i];
+          float x0, x1, x2, x3;
+          fma2(v[4 * i], v[4 * i + 1], c, c, b.x, b.y, x0, x1);
+          fma2(v[4 * i + 2], v[4 * i + 3], c, c, b.z, b.w, x2, x3);
+          add2(a0, a1, ex2_approx(x0), ex2_approx(x1));
+          add2(a2, a3, ex2_approx(x2), ex2_approx(x3));
         }
-        if (NQ % 64) {
-          const int cb = NQ - 32;
-          float v[32];
-          tmem_ld32(tbase + cb, v);
+      }
+      if (c1 - cb == 32) {
+        float v[32];
+        tmem_ld32(tbase + cb, v);
+        const float4* b4 = reinterpret_cast<const float4*>(bias_s + cb);
 #pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (cb + i < R) a1 += ex2_approx(fmaf(v[i], c, bias_s[cb + i]));
+        for (int i = 0; i < 8; ++i) {
+          const float4 b = b4[i];
+          float x0, x1, x2, x3;
+          fma2(v[4 * i], v[4 * i + 1], c, c, b.x, b.y, x0, x1);
+          fma2(v[4 * i + 2], v[4 * i + 3], c, c, b.z, b.w, x2, x3);
+          add2(a0, a1, ex2_approx(x0), ex2_approx(x1));
+          add2(a2, a3, ex2_approx(x2), ex2_approx(x3));
         }
-        const float acc = (a0 + a1) + (a2 + a3);
-        tc_fence_before();
+      }
+      float acc = (a0 + a1) + (a2 + a3);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(b_accempty + 8 * as);
+      const int xb = it & 1;
+      const uint32_t ux = (uint32_t)(it >> 1);
+      if (g == 1) {
+        if (!warp_wait(b_xempty + 8 * xb, (ux & 1u) ^ 1u, err, abort_flag)) break;
+        __syncwarp();  // the lanes' accesses follow lane 0's acquire
+        xch[xb * 128 + row] = acc;
         __syncwarp();
-        if (lane == 0) mbar_arrive(b_accempty + 8 * g);
-        const int tok = (blockIdx.x + it * gridDim.x) * 128 + quarter * 32 + lane;
+        if (lane == 0) mbar_arrive(b_xfull + 8 * xb);
+      } else {
+        if (!warp_wait(b_xfull + 8 * xb, ux & 1u, err, abort_flag)) break;
+        __syncwarp();
+        acc += xch[xb * 128 + row];
+        __syncwarp();
+        if (lane == 0) mbar_arrive(b_xempty + 8 * xb);
+        const int tok = (blockIdx.x + it * gridDim.x) * 128 + row;
         if (tok < n) a_base[(size_t)h * n + tok] = acc;
       }
     }
