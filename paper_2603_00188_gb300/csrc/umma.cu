@@ -780,12 +780,22 @@ __global__ void __launch_bounds__(kThreads, 1)
 // epilogue thread drains its TMEM row window in 32-column chunks, parks each
 // chunk in its own row of a padded shared buffer and picks the five
 // diagonals; k_css_phi then forms Phi from the per-token dots (Eqs. 4-5).
-constexpr int kCssBStage = 65536;                        // [2 halves][256 rows][128 B]
+// B stages hold cap_rows key rows ([2 halves][cap_rows][128 B]), loaded as
+// 64-row TMA boxes: the widest frame of the launch sets cap_rows =
+// roundup64(roundup16(128 + gw + 1)), and as many stages as fit (2 to 4).
 constexpr int kCssStgRow = 36;                           // floats per staged row (16-byte rows, no conflicts)
-constexpr int kCssStg = 2 * kCssBStage;                  // 8 warps x [32][36] floats
-constexpr int kCssBar = kCssStg + 8 * 32 * kCssStgRow * 4;
-constexpr int kCssUmmaSmem = kCssBar + 128 + 1024;
+constexpr int kCssStgBytes = 8 * 32 * kCssStgRow * 4;    // 8 warps x [32][36] floats
+constexpr int kCssBarBytes = 128;                        // kfull[4], kempty[4], accfull[2], accempty[2], done, slot, abort
+constexpr int kCssSmemMax = 232448;
 constexpr int kCssMaxGw = 127;                           // NB <= 256
+constexpr int kCssMaxStages = 4;
+
+struct CssGeom {
+  int cap_rows;     // key rows per B stage (multiple of 64)
+  int stage_bytes;  // 2 * cap_rows * 128
+  int stages;       // B stages in the ring
+  int smem;         // dynamic shared memory of the launch
+};
 
 struct CssDots {
   Strided<float> rn, dE, dS, dSE, dSW, rn_cur;
@@ -809,27 +819,36 @@ __device__ __forceinline__ void css_tile(const FrameTable& ft, int t, int& f, in
 
 __global__ void __launch_bounds__(kThreads, 1)
     k_css_umma(const __grid_constant__ KMaps maps, const __grid_constant__ FrameTable ft, int hkv,
-               CssDots out, uint32_t* err) {
+               CssDots out, CssGeom geo, uint32_t* err) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = align1024(smem_raw);
+  const int S = geo.stages, SB = geo.stage_bytes, half_bytes = geo.cap_rows * 128;
+  const int off_stg = S * SB, off_bar = off_stg + kCssStgBytes;
+  if ((int)(sm - smem_raw) + off_bar + kCssBarBytes > geo.smem) {  // uniform: the layout would not fit
+    if (threadIdx.x == 0) record_error(err, kErrLaunch);
+    return;
+  }
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int l = blockIdx.y / hkv, h = blockIdx.y % hkv, n = ft.n_tokens;
   const CUtensorMap& kmap = maps.m[l];
   const int ntiles_all = ft.ctile0[ft.n_frames];
   const uint32_t sB = smem_u32(sm);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + kCssBar);
-  const uint32_t b_kfull = smem_u32(&bars[0]), b_kempty = smem_u32(&bars[2]);
-  const uint32_t b_accfull = smem_u32(&bars[4]), b_accempty = smem_u32(&bars[6]);
-  const uint32_t b_done = smem_u32(&bars[8]);
-  uint32_t* slot = reinterpret_cast<uint32_t*>(sm + kCssBar + 80);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + off_bar);
+  const uint32_t b_kfull = smem_u32(&bars[0]), b_kempty = smem_u32(&bars[kCssMaxStages]);
+  const uint32_t b_accfull = smem_u32(&bars[2 * kCssMaxStages]);
+  const uint32_t b_accempty = smem_u32(&bars[2 * kCssMaxStages + 2]);
+  const uint32_t b_done = smem_u32(&bars[2 * kCssMaxStages + 4]);
+  uint32_t* slot = reinterpret_cast<uint32_t*>(sm + off_bar + (2 * kCssMaxStages + 5) * 8);
   volatile uint32_t* abort_flag = slot + 1;
   int ntiles = 0;
   for (int t = blockIdx.x; t < ntiles_all; t += gridDim.x) ++ntiles;
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < S; ++i) {
       mbar_init(b_kfull + 8 * i, 1);
       mbar_init(b_kempty + 8 * i, 1);
+    }
+    for (int i = 0; i < 2; ++i) {
       mbar_init(b_accfull + 8 * i, 1);
       mbar_init(b_accempty + 8 * i, 4);
     }
@@ -849,31 +868,31 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     if (lane == 0) {
-      int issued[2] = {0, 0};
+      int issued[kCssMaxStages] = {0, 0, 0, 0};
       for (int it = 0; it < ntiles; ++it) {
-        const int s = it & 1;
-        const uint32_t u = (uint32_t)(it >> 1);
+        const int s = it % S;
+        const uint32_t u = (uint32_t)(it / S);
         if (!mbar_wait(b_kempty + 8 * s, (u & 1u) ^ 1u, err, abort_flag)) break;
         int f, t0;
         css_tile(ft, blockIdx.x + it * gridDim.x, f, t0);
-        mbar_arrive_expect_tx(b_kfull + 8 * s, kCssBStage);
+        const int nbox = (((128 + ft.gw[f] + 1 + 15) & ~15) + 63) / 64;  // 64-row boxes covering NB rows
+        mbar_arrive_expect_tx(b_kfull + 8 * s, (uint32_t)(2 * nbox * 64 * 128));
         for (int kb = 0; kb < 2; ++kb)
-          for (int half = 0; half < 2; ++half)
-            tma_load_3d(sB + s * kCssBStage + kb * 32768 + half * 16384, &kmap, b_kfull + 8 * s, kb * 64, h,
-                        t0 + half * 128);
+          for (int r = 0; r < nbox; ++r)
+            tma_load_3d(sB + s * SB + kb * half_bytes + r * 8192, &kmap, b_kfull + 8 * s, kb * 64, h,
+                        t0 + r * 64);
         ++issued[s];
       }
       if (*abort_flag)
-        for (int s = 0; s < 2; ++s)
+        for (int s = 0; s < S; ++s)
           if (issued[s]) mbar_wait_drain(b_kfull + 8 * s, (uint32_t)(issued[s] - 1) & 1u);
     }
   } else if (warp == 1) {
     if (lane == 0) {
       for (int it = 0; it < ntiles; ++it) {
-        const int s = it & 1;
-        const uint32_t u = (uint32_t)(it >> 1);
-        if (!mbar_wait(b_kfull + 8 * s, u & 1u, err, abort_flag)) break;
-        if (!mbar_wait(b_accempty + 8 * s, (u & 1u) ^ 1u, err, abort_flag)) break;
+        const int s = it % S, as = it & 1;
+        if (!mbar_wait(b_kfull + 8 * s, (uint32_t)(it / S) & 1u, err, abort_flag)) break;
+        if (!mbar_wait(b_accempty + 8 * as, ((uint32_t)(it >> 1) & 1u) ^ 1u, err, abort_flag)) break;
         tc_fence_after();
         int f, t0;
         css_tile(ft, blockIdx.x + it * gridDim.x, f, t0);
@@ -882,10 +901,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
           const uint32_t kb = k >> 2, koff = (k & 3) * 32;
-          const uint64_t d = desc_sw128(sB + s * kCssBStage + kb * 32768 + koff);
-          umma_bf16(tmem + s * 256, d, d, idesc, k > 0 ? 1u : 0u);
+          const uint64_t d = desc_sw128(sB + s * SB + kb * half_bytes + koff);
+          umma_bf16(tmem + as * 256, d, d, idesc, k > 0 ? 1u : 0u);
         }
-        umma_commit(b_accfull + 8 * s);
+        umma_commit(b_accfull + 8 * as);
         umma_commit(b_kempty + 8 * s);
       }
       umma_commit(b_done);
@@ -893,7 +912,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     const int g = (warp - 2) >> 2, quarter = warp & 3;
-    float* stg = reinterpret_cast<float*>(sm + kCssStg) + (size_t)(warp - 2) * 32 * kCssStgRow + lane * kCssStgRow;
+    float* stg = reinterpret_cast<float*>(sm + off_stg) + (size_t)(warp - 2) * 32 * kCssStgRow + lane * kCssStgRow;
     const uint32_t tbase = tmem + ((uint32_t)(quarter * 32) << 16) + g * 256 + quarter * 32;
     float* rn_o = out.rn.at(l) + (size_t)h * n;
     float* e_o = out.dE.at(l) + (size_t)h * n;
@@ -1150,9 +1169,18 @@ cudaError_t launch_css_umma(const Problem& p, const FrameTable& ft, const LayerP
   const int tiles = ft.ctile0[ft.n_frames];
   if (tiles == 0) return cudaSuccess;
   KMaps maps;
-  cudaError_t e = make_kmaps(&maps, io, p.L, p.n, p.hkv, 128);
+  cudaError_t e = make_kmaps(&maps, io, p.L, p.n, p.hkv, 64);
   if (e != cudaSuccess) return e;
-  if ((e = cudaFuncSetAttribute(k_css_umma, cudaFuncAttributeMaxDynamicSharedMemorySize, kCssUmmaSmem)) !=
+  CssGeom geo;
+  int nb_max = 0;
+  for (int f = 0; f < ft.n_frames; ++f) nb_max = max(nb_max, (128 + ft.gw[f] + 1 + 15) & ~15);
+  geo.cap_rows = (nb_max + 63) / 64 * 64;
+  geo.stage_bytes = 2 * geo.cap_rows * 128;
+  geo.smem = kCssSmemMax;
+  geo.stages = (kCssSmemMax - 1024 - kCssStgBytes - kCssBarBytes) / geo.stage_bytes;
+  if (geo.stages > kCssMaxStages) geo.stages = kCssMaxStages;
+  if (geo.stages < 2) return cudaErrorNotSupported;
+  if ((e = cudaFuncSetAttribute(k_css_umma, cudaFuncAttributeMaxDynamicSharedMemorySize, geo.smem)) !=
       cudaSuccess)
     return e;
   CssDots d;
@@ -1166,7 +1194,7 @@ cudaError_t launch_css_umma(const Problem& p, const FrameTable& ft, const LayerP
   const int gx = pick_split(p.L * p.hkv, tiles, sm_count());
   {
     TimingScope ts("css_umma", st);
-    k_css_umma<<<dim3(gx, p.L * p.hkv), kThreads, kCssUmmaSmem, st>>>(maps, ft, p.hkv, d, err);
+    k_css_umma<<<dim3(gx, p.L * p.hkv), kThreads, geo.smem, st>>>(maps, ft, p.hkv, d, geo, err);
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   int cmax = 1;
