@@ -393,8 +393,9 @@ def run_gpu(args):
     dom = max(ktimes, key=lambda k: ktimes[k][1])
     for k, (c, t) in ktimes.items():
         kernels[k]["roofline"] = kernel_roofline(k, t / c * 1e-3, L, budget, peaks)
+        kernels[k]["roofline"]["traffic"] = traffic_for(k) if L == LAYERS else None
     roof = dict(kernels[dom]["roofline"], kernel=dom)
-    roof["traffic"] = traffic_for(dom)
+    roof["traffic"] = traffic_for(dom) if L == LAYERS else None
     roof["peak_source"] = peaks["source"] + (" burst" if roof["unit"] == "TFLOP/s" else "")
 
     # ---- end to end: host (pinned) inputs -> device -> compress -> host outputs
