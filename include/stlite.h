@@ -20,6 +20,12 @@
  *     k_out, v_out [B][Hkv][d] compacted cache
  *   Element type of q/k/v/k_out/v_out is shape->dtype (bf16 or fp32).
  *   Query head g serves KV head g / (Hq/Hkv) (grouped-query attention).
+ *   Exception: v may instead be page-locked HOST memory (cudaHostAlloc,
+ *   cudaMallocHost or cudaHostRegister), which kernels address directly under
+ *   unified addressing.  Only the compaction reads v, and only the B kept
+ *   rows per head, so values kept on the host cost B rows of host-link
+ *   traffic per head instead of a copy of all N (stlite_compact,
+ *   stlite_compress_layer and stlite_compress_layers).
  * Frames.  stlite_frames holds HOST arrays.  Frame f owns the contiguous
  *   visual span [offset[f], offset[f] + grid_h[f]*grid_w[f]) laid out
  *   row-major on its patch grid (u = row, v = column); frames are sorted,

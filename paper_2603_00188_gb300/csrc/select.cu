@@ -436,7 +436,7 @@ __global__ void __launch_bounds__(256) k_gather(const __grid_constant__ LayerPtr
         if (src >= 0 && src < n) {
           const size_t s = ((size_t)src * hkv + h) * CPR + c;
           kv[u] = __ldg(k + s);
-          vv[u] = __ldg(v + s);
+          vv[u] = v[s];  // plain load: v may be page-locked host memory
           ok[u] = true;
         }
       }

@@ -298,3 +298,35 @@ def test_compress_layers_more_than_one_launch(st):
     wls = [synth.trajectory(n_steps=3, gh=5, gw=7, n_text=4, hq=8, hkv=2, w=4, beta=0.3, seed=(800, s))
            for s in range(34)]
     _batched_vs_single(st, wls)
+
+
+# ------------------------------------------------- values in page-locked host memory
+
+def test_host_resident_values(st):
+    """v may live in page-locked host memory (only the kept rows are read):
+    the outputs equal those of a device-resident v, for the single-layer and
+    the batched entry, bf16 and fp32."""
+    for wls in ([synth.scaled("traj50", 3, seed=s) for s in range(2)], [synth.tiny_ref(seed=5)]):
+        wl0 = wls[0]
+        dev = [to_device(wl) for wl in wls]
+        ref = [st.compress_layer(q, k, v, wl0.frames, beta=wl0.beta) for (q, k, v) in dev]
+        hv = [v.cpu().pin_memory() for (_, _, v) in dev]
+        torch.cuda.synchronize()
+        one = [st.compress_layer(q, k, v_h, wl0.frames, beta=wl0.beta) for (q, k, _), v_h in zip(dev, hv)]
+        sh = st.make_shape(dev[0][0], dev[0][1])
+        prm = st.make_params(wl0.beta)
+        b = st.stlite_budget(wl0.n, wl0.beta)
+        H = sh.n_kv_heads
+        outs = []
+        for (q, k, _), v_h in zip(dev, hv):
+            ko = torch.empty((b, H, sh.head_dim), dtype=k.dtype, device="cuda")
+            outs.append((q, k, v_h, ko, torch.empty_like(ko), torch.empty((H, b), dtype=torch.int32, device="cuda")))
+        ws = torch.zeros(len(wls) * st.stlite_workspace_size(sh, wl0.frames, prm), dtype=torch.uint8,
+                         device="cuda")
+        assert st.stlite_compress_layers(outs, wl0.frames, prm, ws) == b
+        torch.cuda.synchronize()
+        assert st.stlite_device_status(ws) == st.STLITE_OK
+        for (k1, v1, i1), (k2, v2, i2), (_, _, _, k3, v3, i3) in zip(ref, one, outs):
+            assert torch.equal(i1, i2) and torch.equal(i1, i3)
+            assert torch.equal(k1, k2) and torch.equal(k1, k3)
+            assert torch.equal(v1, v2) and torch.equal(v1, v3)
