@@ -479,13 +479,18 @@ __global__ void __launch_bounds__(kThreads, 1)
           const float mn = fmaxf(m, fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3])));
           const float mnc = mn * c;
           float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+          // three phases (exponent arguments, exponentials, sums), so that
+          // independent work separates dependent instructions
+          float x[64];
+#pragma unroll
+          for (int i = 0; i < 64; i += 2)
+            fma2(__uint_as_float(b[i]), __uint_as_float(b[i + 1]), c, c, -mnc, -mnc, x[i], x[i + 1]);
+#pragma unroll
+          for (int i = 0; i < 64; ++i) x[i] = ex2_approx(x[i]);
 #pragma unroll
           for (int i = 0; i < 64; i += 4) {
-            float x0, x1, x2, x3;
-            fma2(__uint_as_float(b[i]), __uint_as_float(b[i + 1]), c, c, -mnc, -mnc, x0, x1);
-            fma2(__uint_as_float(b[i + 2]), __uint_as_float(b[i + 3]), c, c, -mnc, -mnc, x2, x3);
-            add2(s0, s1, ex2_approx(x0), ex2_approx(x1));
-            add2(s2, s3, ex2_approx(x2), ex2_approx(x3));
+            add2(s0, s1, x[i], x[i + 1]);
+            add2(s2, s3, x[i + 2], x[i + 3]);
           }
           l = (m == -CUDART_INF_F ? 0.f : l * ex2_approx((m - mn) * c)) + ((s0 + s1) + (s2 + s3));
           m = mn;
@@ -716,14 +721,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         float v[64];
         tmem_ld64(tbase + cb, v);
         const float4* b4 = reinterpret_cast<const float4*>(bias_s + cb);
+        // three phases over the chunk (exponent arguments, exponentials,
+        // sums), so that independent work separates dependent instructions
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           const float4 b = b4[i];
-          float x0, x1, x2, x3;
-          fma2(v[4 * i], v[4 * i + 1], c, c, b.x, b.y, x0, x1);
-          fma2(v[4 * i + 2], v[4 * i + 3], c, c, b.z, b.w, x2, x3);
-          add2(a0, a1, ex2_approx(x0), ex2_approx(x1));
-          add2(a2, a3, ex2_approx(x2), ex2_approx(x3));
+          fma2(v[4 * i], v[4 * i + 1], c, c, b.x, b.y, v[4 * i], v[4 * i + 1]);
+          fma2(v[4 * i + 2], v[4 * i + 3], c, c, b.z, b.w, v[4 * i + 2], v[4 * i + 3]);
+        }
+#pragma unroll
+        for (int i = 0; i < 64; ++i) v[i] = ex2_approx(v[i]);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          add2(a0, a1, v[4 * i], v[4 * i + 1]);
+          add2(a2, a3, v[4 * i + 2], v[4 * i + 3]);
         }
       }
       if (c1 - cb == 32) {
