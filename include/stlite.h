@@ -2,8 +2,9 @@
  * stlite.h -- C ABI of libstlite.so, the GB300 (sm_103a) implementation of the
  * ST-Lite per-layer KV-cache compression pass (arXiv 2603.00188, Algorithm 1).
  *
- * One call compresses one layer of one sequence (or, for the _varlen entry,
- * one layer of a packed batch).  The pass has five steps:
+ * One call compresses one layer of one sequence (stlite_compress_layer), a
+ * batch of layers of one sequence (stlite_compress_layers), or one layer of
+ * a packed batch of sequences (stlite_compress_varlen).  The pass has five steps:
  *   1. window scoring       A_base, Sec. 2.1 Eq. (2)
  *   2. TSG redundancy gate  rho, tau, M_time, Sec. 3.2 Eqs. (6)-(8)
  *   3. CSS saliency         Phi, Sec. 3.1 Eqs. (4)-(5)
@@ -208,6 +209,37 @@ STLITE_API stlite_status stlite_compress_layers(const stlite_shape* shape, const
                                                 const stlite_params* params, int32_t n_layers,
                                                 const stlite_layer_io* layers, int32_t* budget_out,
                                                 void* ws, size_t ws_bytes, void* stream);
+
+/* A packed batch of sequences of different lengths and frame layouts (one
+ * layer): Algorithm 1 for each sequence on its own, with its own budget
+ * B_s = stlite_budget(N_s, beta, k_override).
+ * shape: n_tokens = the total packed length; the other fields are shared.
+ * cu_seqlens: HOST int32 [n_seqs + 1], cu_seqlens[0] = 0, non-decreasing by at
+ *   least 1, cu_seqlens[n_seqs] = n_tokens: sequence s owns packed tokens
+ *   [cu_seqlens[s], cu_seqlens[s + 1]).
+ * frames: HOST array [n_seqs]; frames[s] describes sequence s with offsets
+ *   relative to the sequence's first token.
+ * q: [n_seqs][w][Hq][d] (each sequence's window queries); k, v: packed
+ *   [n_tokens][Hkv][d].
+ * k_out, v_out: packed [sum_s B_s][Hkv][d] in sequence order; idx_out: the
+ *   blocks [Hkv][B_s] of the sequences one after another (block s starts at
+ *   element Hkv * sum_{r<s} B_r), indices relative to the sequence start.
+ * cu_budget_out (nullable, HOST int32 [n_seqs + 1]) receives the prefix sums
+ *   of B_s.  ws: at least stlite_workspace_size_varlen bytes; the sequences
+ *   run one after another on `stream` and share it.  The result for each
+ *   sequence equals stlite_compress_layer's on that sequence alone. */
+STLITE_API stlite_status stlite_compress_varlen(const stlite_shape* shape, int32_t n_seqs,
+                                                const int32_t* cu_seqlens, const stlite_frames* frames,
+                                                const stlite_params* params, const void* q, const void* k,
+                                                const void* v, void* k_out, void* v_out, int32_t* idx_out,
+                                                int32_t* cu_budget_out, void* ws, size_t ws_bytes,
+                                                void* stream);
+
+/* Workspace bytes stlite_compress_varlen needs: the largest of the
+ * sequences' stlite_workspace_size. */
+STLITE_API stlite_status stlite_workspace_size_varlen(const stlite_shape* shape, int32_t n_seqs,
+                                                      const int32_t* cu_seqlens, const stlite_frames* frames,
+                                                      const stlite_params* params, size_t* bytes);
 
 /* Reads and clears the workspace's device error word (synchronises `stream`).
  * *status receives STLITE_OK, STLITE_ETIMEOUT if a kernel's bounded wait ran

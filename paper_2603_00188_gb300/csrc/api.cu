@@ -465,6 +465,78 @@ stlite_status stlite_compress_layers(const stlite_shape* shape, const stlite_fra
   return STLITE_OK;
 }
 
+// Packed batches (stlite_compress_varlen): per-sequence shapes.
+static stlite_status varlen_shapes(const stlite_shape* shape, int32_t n_seqs, const int32_t* cu,
+                                   const stlite_frames* frames, size_t* ws_max) {
+  if (!shape || n_seqs < 1 || !cu || !frames) return STLITE_EINVAL;
+  stlite_status s = check_shape(shape);
+  if (s != STLITE_OK) return s;
+  if (cu[0] != 0 || cu[n_seqs] != shape->n_tokens) return STLITE_EINVAL;
+  size_t mx = 0;
+  for (int i = 0; i < n_seqs; ++i) {
+    if (cu[i + 1] <= cu[i]) return STLITE_EINVAL;
+    stlite_shape ss = *shape;
+    ss.n_tokens = cu[i + 1] - cu[i];
+    if ((s = check_shape(&ss)) != STLITE_OK) return s;
+    FrameTable ft;
+    if ((s = build_frames(&ss, &frames[i], &ft)) != STLITE_OK) return s;
+    const size_t b = plan_workspace(to_problem(&ss, 1), ft).total;
+    if (b > mx) mx = b;
+  }
+  *ws_max = mx;
+  return STLITE_OK;
+}
+
+stlite_status stlite_workspace_size_varlen(const stlite_shape* shape, int32_t n_seqs, const int32_t* cu_seqlens,
+                                           const stlite_frames* frames, const stlite_params* params,
+                                           size_t* bytes) {
+  if (!bytes) return STLITE_EINVAL;
+  stlite_status s;
+  if (params && (s = check_params(params)) != STLITE_OK) return s;
+  return varlen_shapes(shape, n_seqs, cu_seqlens, frames, bytes);
+}
+
+stlite_status stlite_compress_varlen(const stlite_shape* shape, int32_t n_seqs, const int32_t* cu_seqlens,
+                                     const stlite_frames* frames, const stlite_params* params, const void* q,
+                                     const void* k, const void* v, void* k_out, void* v_out, int32_t* idx_out,
+                                     int32_t* cu_budget_out, void* ws, size_t ws_bytes, void* stream) {
+  size_t ws_need = 0;
+  stlite_status s = varlen_shapes(shape, n_seqs, cu_seqlens, frames, &ws_need);
+  if (s != STLITE_OK) return s;
+  if ((s = check_params(params)) != STLITE_OK) return s;
+  if (!q || !k || !v || !k_out || !v_out || !idx_out) return STLITE_EINVAL;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(k_out) || !aligned16(v_out) ||
+      !aligned16(idx_out))
+    return STLITE_EINVAL;
+  if (!ws || !aligned16(ws)) return STLITE_EINVAL;
+  if (ws_bytes < ws_need) return STLITE_EWORKSPACE;
+  // every budget is checked before anything is enqueued
+  for (int i = 0; i < n_seqs; ++i)
+    if (stlite_budget(cu_seqlens[i + 1] - cu_seqlens[i], params->beta, params->k_override) < 1)
+      return STLITE_EINVAL;
+  const size_t e = shape->dtype == STLITE_BF16 ? 2 : 4;
+  const size_t row = (size_t)shape->n_kv_heads * shape->head_dim * e;  // one token of k / v
+  const size_t qseq = (size_t)shape->window * shape->n_q_heads * shape->head_dim * e;
+  size_t cum = 0;
+  if (cu_budget_out) cu_budget_out[0] = 0;
+  for (int i = 0; i < n_seqs; ++i) {
+    stlite_shape ss = *shape;
+    ss.n_tokens = cu_seqlens[i + 1] - cu_seqlens[i];
+    Ctx c;
+    if ((s = prepare(&ss, &frames[i], ws, ws_bytes, 1, stream, &c)) != STLITE_OK) return s;
+    const int32_t b = stlite_budget(ss.n_tokens, params->beta, params->k_override);
+    const size_t t0 = (size_t)cu_seqlens[i];
+    const LayerPtrs io =
+        single_layer(static_cast<const uint8_t*>(q) + i * qseq, static_cast<const uint8_t*>(k) + t0 * row,
+                     static_cast<const uint8_t*>(v) + t0 * row, static_cast<uint8_t*>(k_out) + cum * row,
+                     static_cast<uint8_t*>(v_out) + cum * row, idx_out + (size_t)shape->n_kv_heads * cum);
+    if ((s = compress_batch(c, params, io, b)) != STLITE_OK) return s;
+    cum += (size_t)b;
+    if (cu_budget_out) cu_budget_out[i + 1] = (int32_t)cum;
+  }
+  return STLITE_OK;
+}
+
 stlite_status stlite_device_status(void* ws, void* stream, stlite_status* status) {
   if (!ws || !status || !aligned16(ws)) return STLITE_EINVAL;
   cudaStream_t st = static_cast<cudaStream_t>(stream);

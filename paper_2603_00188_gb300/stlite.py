@@ -27,7 +27,8 @@ MAX_FRAMES = 256
 EXPORTED = ("stlite_budget", "stlite_workspace_size", "stlite_score", "stlite_gate_frames",
             "stlite_spatial_saliency", "stlite_select_topk", "stlite_compact",
             "stlite_compress_layer", "stlite_device_status", "stlite_timing_enable", "stlite_timing_read",
-            "stlite_status_string", "stlite_score_noalloc", "stlite_compress_layers")
+            "stlite_status_string", "stlite_score_noalloc", "stlite_compress_layers", "stlite_compress_varlen",
+            "stlite_workspace_size_varlen")
 
 
 class Shape(ctypes.Structure):
@@ -79,6 +80,12 @@ _sig = {
     "stlite_compress_layers": (_S, [ctypes.POINTER(Shape), ctypes.POINTER(Frames), ctypes.POINTER(Params),
                                     ctypes.c_int32, ctypes.POINTER(LayerIO), ctypes.POINTER(ctypes.c_int32), _P,
                                     ctypes.c_size_t, _P]),
+    "stlite_compress_varlen": (_S, [ctypes.POINTER(Shape), ctypes.c_int32, ctypes.POINTER(ctypes.c_int32),
+                                    ctypes.POINTER(Frames), ctypes.POINTER(Params), _P, _P, _P, _P, _P, _P,
+                                    ctypes.POINTER(ctypes.c_int32), _P, ctypes.c_size_t, _P]),
+    "stlite_workspace_size_varlen": (_S, [ctypes.POINTER(Shape), ctypes.c_int32, ctypes.POINTER(ctypes.c_int32),
+                                          ctypes.POINTER(Frames), ctypes.POINTER(Params),
+                                          ctypes.POINTER(ctypes.c_size_t)]),
 }
 for _name, (_res, _args) in _sig.items():
     _f = getattr(_lib, _name)
@@ -216,6 +223,40 @@ def stlite_compress_layers(layers, frames, params, ws, stream=None) -> int:
                                        arr, ctypes.byref(b), _ptr(ws), ws.numel(), _stream(stream)),
            "stlite_compress_layers")
     return int(b.value)
+
+
+def _varlen_args(cu_seqlens, frames_list):
+    cu = np.ascontiguousarray(cu_seqlens, dtype=np.int32)
+    specs = [_frames(f) for f in frames_list]
+    arr = (Frames * len(specs))(*[f.c for f in specs])
+    return cu, specs, arr
+
+
+def stlite_workspace_size_varlen(shape: Shape, cu_seqlens, frames_list, params: Params | None = None) -> int:
+    cu, specs, arr = _varlen_args(cu_seqlens, frames_list)
+    out = ctypes.c_size_t()
+    _check(_lib.stlite_workspace_size_varlen(ctypes.byref(shape), len(specs),
+                                             cu.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)), arr,
+                                             ctypes.byref(params) if params is not None else None,
+                                             ctypes.byref(out)), "stlite_workspace_size_varlen")
+    return int(out.value)
+
+
+def stlite_compress_varlen(q, k, v, cu_seqlens, frames_list, params, k_out, v_out, idx_out, ws, stream=None):
+    """Packed batch of sequences (one layer): q [n_seqs][w][Hq][d], k/v packed
+    [N][Hkv][d], cu_seqlens (n_seqs + 1 offsets), one frame descriptor per
+    sequence (offsets relative to the sequence).  Returns the budget prefix
+    sums (n_seqs + 1)."""
+    n_seqs = len(frames_list)
+    sh = make_shape(q[0] if q.dim() == 4 else q, k)
+    cu, specs, arr = _varlen_args(cu_seqlens, frames_list)
+    cb = np.zeros(n_seqs + 1, dtype=np.int32)
+    ip = ctypes.POINTER(ctypes.c_int32)
+    _check(_lib.stlite_compress_varlen(ctypes.byref(sh), n_seqs, cu.ctypes.data_as(ip), arr, ctypes.byref(params),
+                                       _ptr(q), _ptr(k), _ptr(v), _ptr(k_out), _ptr(v_out), _ptr(idx_out),
+                                       cb.ctypes.data_as(ip), _ptr(ws), ws.numel(), _stream(stream)),
+           "stlite_compress_varlen")
+    return cb
 
 
 def stlite_device_status(ws, stream=None) -> int:

@@ -103,3 +103,22 @@ def test_entry_points_reject_before_launch(st):
     assert lib.stlite_compact(ctypes.byref(sh), 0, good, good, good, good, good, None) == st.STLITE_EINVAL
     assert lib.stlite_compact(ctypes.byref(sh), 101, good, good, good, good, good, None) == st.STLITE_EINVAL
     assert lib.stlite_device_status(None, None, None) == st.STLITE_EINVAL
+
+
+def test_varlen_validation(st):
+    """stlite_compress_varlen / stlite_workspace_size_varlen reject malformed
+    packed batches on the host (no GPU needed)."""
+    sh = _shape(st, n=300, hq=4, hkv=2, w=4)
+    fr = [st.FrameSpec([0], [5], [8]), st.FrameSpec([10], [4], [6]), st.FrameSpec([], [], [])]
+    prm = st.make_params(0.2)
+    ok = st.stlite_workspace_size_varlen(sh, [0, 100, 200, 300], fr, prm)
+    assert ok > 0
+    # the largest sequence sets the size
+    assert ok == max(st.stlite_workspace_size(_shape(st, n=100, hq=4, hkv=2, w=4), f, prm) for f in fr)
+    for cu in ([0, 100, 200, 299], [1, 100, 200, 300], [0, 100, 100, 300], [0, 200, 100, 300]):
+        with pytest.raises(st.StliteError):
+            st.stlite_workspace_size_varlen(sh, cu, fr, prm)
+    # a frame outside its own sequence
+    bad = [st.FrameSpec([0], [10], [11]), fr[1], fr[2]]
+    with pytest.raises(st.StliteError):
+        st.stlite_workspace_size_varlen(sh, [0, 100, 200, 300], bad, prm)

@@ -330,3 +330,53 @@ def test_host_resident_values(st):
             assert torch.equal(i1, i2) and torch.equal(i1, i3)
             assert torch.equal(k1, k2) and torch.equal(k1, k3)
             assert torch.equal(v1, v2) and torch.equal(v1, v3)
+
+
+# ------------------------------------------------------- packed batch of sequences
+
+def _varlen_vs_single(st, wls):
+    dev = [to_device(wl) for wl in wls]
+    cu = np.concatenate([[0], np.cumsum([wl.n for wl in wls])]).astype(np.int32)
+    q = torch.stack([d[0] for d in dev])
+    k = torch.cat([d[1] for d in dev])
+    v = torch.cat([d[2] for d in dev])
+    beta = wls[0].beta
+    prm = st.make_params(beta)
+    budgets = [st.stlite_budget(wl.n, beta) for wl in wls]
+    H, D = k.shape[1], k.shape[2]
+    tot = sum(budgets)
+    ko = torch.empty((tot, H, D), dtype=k.dtype, device="cuda")
+    vo = torch.empty_like(ko)
+    ix = torch.empty((H * tot,), dtype=torch.int32, device="cuda")
+    sh = st.make_shape(dev[0][0], k)
+    ws = torch.zeros(st.stlite_workspace_size_varlen(sh, cu, [wl.frames for wl in wls], prm), dtype=torch.uint8,
+                     device="cuda")
+    cb = st.stlite_compress_varlen(q, k, v, cu, [wl.frames for wl in wls], prm, ko, vo, ix, ws)
+    torch.cuda.synchronize()
+    assert st.stlite_device_status(ws) == st.STLITE_OK
+    assert list(cb) == list(np.concatenate([[0], np.cumsum(budgets)]))
+    for s, (wl, (qs, ks, vs)) in enumerate(zip(wls, dev)):
+        k1, v1, i1 = st.compress_layer(qs, ks, vs, wl.frames, beta=beta)
+        b0, b1 = cb[s], cb[s + 1]
+        assert torch.equal(ix[H * b0:H * b1].view(H, b1 - b0), i1)
+        assert torch.equal(ko[b0:b1], k1) and torch.equal(vo[b0:b1], v1)
+    return cb
+
+
+def test_varlen_small_backbone_batch(st):
+    # the batch-8 smaller-backbone configuration: 12-20 frames of 24x42 per sequence
+    _varlen_vs_single(st, [synth.small_backbone_seq(s, beta=0.1) for s in range(8)])
+
+
+def test_varlen_ragged_fp32_and_oracle(st):
+    # three sequences of different frame layouts (fp32), one of them a single frame;
+    # the packed call equals per-sequence calls, and those match the oracle
+    wls = [synth.trajectory(n_steps=3, gh=5, gw=7, n_text=4, hq=8, hkv=2, w=4, beta=0.3, seed=(900, 0),
+                            dtype="fp32"),
+           synth.trajectory(n_steps=1, gh=6, gw=3, n_text=9, hq=8, hkv=2, w=4, beta=0.3, seed=(900, 1),
+                            dtype="fp32"),
+           synth.trajectory(n_steps=4, gh=3, gw=9, n_text=2, hq=8, hkv=2, w=4, beta=0.3, seed=(900, 2),
+                            dtype="fp32")]
+    _varlen_vs_single(st, wls)
+    for wl in wls:
+        _run_edge(st, wl, wl.beta)
