@@ -233,8 +233,8 @@ def oracle_sample(wl, pool_stride: int = 16, q_heads: int = HQ // HKV):
 
 
 def run_reference(args):
-    rank = int(os.environ.get("RANK", "0"))
-    if rank != 0:
+    _, rank, _ = dist_env()
+    if rank != 0:   # under torchrun rank 0 alone times the oracle; the others exit 0
         return
     sys.stdout.flush()
     from paper_2603_00188_gb300 import synth
@@ -286,13 +286,37 @@ def traffic_for(kernel: str):
     return None if e is None else e.get("dram_bytes_per_launch_full")
 
 
+# ------------------------------------------------------------ multi-rank glue
+
+def dist_env():
+    """(world, rank, local_rank) from the torchrun environment (1, 0, 0 alone)."""
+    return (int(os.environ.get("WORLD_SIZE", "1")), int(os.environ.get("RANK", "0")),
+            int(os.environ.get("LOCAL_RANK", "0")))
+
+
+def max_over_ranks(ms: float, device, world: int) -> float:
+    """The slowest rank's time: every rank processed its own units, so the job
+    took as long as its slowest rank."""
+    if world == 1:
+        return ms
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(world: int, layers: int, ms: float) -> float:
+    """Whole-job tokens per second per layer: every rank compresses its own
+    trajectory of `layers` layers of N_TOK tokens (weak scaling)."""
+    return world * N_TOK * layers / (ms * 1e-3)
+
+
 def run_gpu(args):
     import torch
     import torch.distributed as dist
 
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    world, rank, local = dist_env()
     if world > 1:
         os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
@@ -368,12 +392,9 @@ def run_gpu(args):
     barrier()
     clk = clocks.stop()
     ms = e0.elapsed_time(e1) / args.steps
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ms, dev, world)
     assert stlite.stlite_device_status(ws, stream) == stlite.STLITE_OK
-    value = world * N_TOK * L / (ms * 1e-3)
+    value = job_throughput(world, L, ms)
 
     # ---- per-kernel device time (CUDA events around each launch, eager replay)
     stlite.stlite_timing_read()
@@ -466,16 +487,13 @@ def run_gpu(args):
         torch.cuda.synchronize()
         barrier()
         ms_e2e = f0.elapsed_time(f1) / args.steps
-        if world > 1:
-            t = torch.tensor([ms_e2e], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ms_e2e = float(t.item())
+        ms_e2e = max_over_ranks(ms_e2e, dev, world)
         # the host copies hold the device results of the last step
         last = sets[(args.steps - 1) % 2]
         for l in (0, L - 1):
             assert torch.equal(last["h_out"][l][2], idxs[l].cpu())
             assert torch.equal(last["h_out"][l][1], vos[l].cpu())
-        e2e = dict(value=world * N_TOK * L / (ms_e2e * 1e-3), unit=UNIT, h2d_bytes_per_step=bi,
+        e2e = dict(value=job_throughput(world, L, ms_e2e), unit=UNIT, h2d_bytes_per_step=bi,
                    d2h_bytes_per_step=bo, ms_per_step=ms_e2e,
                    note="q and k copied; v read in place from page-locked host memory (kept rows only)")
 

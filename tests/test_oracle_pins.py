@@ -435,3 +435,38 @@ def test_salient_rectangle_kept():
     out = oracle.compress_layer(q, k, frames_of((0, gh, gw)), beta=0.25)   # B = 16
     kept = set(out["idx"][0].tolist())
     assert all(u * gw + v in kept for (u, v) in elem)
+
+
+def _text_reversal(n, frames):
+    """Permutation that reverses the order of the text tokens (positions
+    outside every frame) and leaves every visual token in place: new
+    position p holds old token perm[p]."""
+    off, gh, gw = frames
+    vis = np.zeros(n, bool)
+    for o, a, b in zip(off, gh, gw):
+        vis[o:o + a * b] = True
+    text = np.nonzero(~vis)[0]
+    perm = np.arange(n)
+    perm[text] = text[::-1]
+    return perm
+
+
+def test_end_to_end_text_permutation_equivariance():
+    # Nothing in Algorithm 1 depends on where a text token sits (no positional
+    # term; CSS and TSG only see visual tokens): reordering the text tokens
+    # reorders A_base and S the same way, leaves Phi, rho and tau unchanged,
+    # and maps the kept set through the permutation.
+    wl = _tiny_traj(seed=6, n_steps=4, nt=5)
+    perm = _text_reversal(wl.n, wl.frames)
+    assert (perm != np.arange(wl.n)).any()
+    a = oracle.compress_layer(wl.q, wl.k, wl.frames, beta=0.3)
+    b = oracle.compress_layer(wl.q, wl.k[perm], wl.frames, beta=0.3)
+    np.testing.assert_allclose(b["a"], a["a"][:, perm], rtol=1e-12, atol=1e-15)
+    np.testing.assert_allclose(b["s"], a["s"][:, perm], rtol=1e-12, atol=1e-15)
+    np.testing.assert_array_equal(b["phi"], a["phi"][:, perm])
+    np.testing.assert_array_equal(b["gate"], a["gate"][:, perm])
+    np.testing.assert_array_equal(np.isnan(b["rho"]), np.isnan(a["rho"]))
+    np.testing.assert_array_equal(b["tau"], a["tau"])
+    inv = np.argsort(perm)
+    for h in range(2):
+        np.testing.assert_array_equal(b["idx"][h], np.sort(inv[a["idx"][h]]))

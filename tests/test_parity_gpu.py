@@ -380,3 +380,26 @@ def test_varlen_ragged_fp32_and_oracle(st):
     _varlen_vs_single(st, wls)
     for wl in wls:
         _run_edge(st, wl, wl.beta)
+
+
+def test_text_permutation_equivariance(st):
+    # Reordering the text tokens reorders the GPU's kept set the same way
+    # (up to swaps at the B-th score, where fp32 sums in a different key order
+    # may round differently).
+    wl = synth.scaled("traj50", 3)
+    q, k, v = to_device(wl)
+    off, gh, gw = wl.frames
+    vis = visual_mask(wl.n, wl.frames)
+    text = np.nonzero(~vis)[0]
+    perm = np.arange(wl.n)
+    perm[text] = text[::-1]
+    pt = torch.from_numpy(perm).cuda()
+    _, _, ia = st.compress_layer(q, k, v, wl.frames, beta=wl.beta)
+    _, _, ib = st.compress_layer(q, k[pt].contiguous(), v[pt].contiguous(), wl.frames, beta=wl.beta)
+    torch.cuda.synchronize()
+    ref = oracle.compress_layer(exact64(q), exact64(k), wl.frames, beta=wl.beta, threads=THREADS)
+    ia, ib = ia.cpu().numpy(), ib.cpu().numpy()
+    b = ref["budget"]
+    for h in range(k.shape[1]):
+        flips = set(np.nonzero(np.abs(ref["rho"][h] - ref["tau"][h]) <= 1e-3 * abs(ref["tau"][h]) + COS_ATOL)[0].tolist())
+        check_kept_sets(np.sort(perm[ib[h]]), ia[h], ref["s"][h], b, s_tol, allowed_extra=flips)
