@@ -67,6 +67,7 @@ def _load():
         lib.orc_topk.argtypes = [_dp, _i32, _i32, _ip]
         lib.orc_gather.restype = None
         lib.orc_gather.argtypes = [_bp, _bp, _i32, _i32, _i32, _i32, _ip, _i32, _bp, _bp]
+        lib.orc_decode_row.argtypes = [_dp, _dp, _dp, _i32, _i32, _i32, _i32, _i32, _i32, _dp]
         _lib = lib
     return _lib
 
@@ -243,3 +244,19 @@ def compress_layer(q, k, frames, beta: float = 0.2, k_override: int = 0, alpha: 
     s = combine(a, phi, gate, frames, alpha, css_enable)
     idx = topk(s, b)
     return dict(budget=b, a=a, phi=phi, rho=rho, tau=tau, gate=gate, pool=pool, s=s, idx=idx)
+
+
+def decode_attention(q, k, v) -> np.ndarray:
+    """Attention of every query row over the whole cache (the decoder's use of
+    the compressed cache): out[r][g] = sum_j softmax_j(q_{r,g}.k_{j,g/G}/sqrt(d))
+    v_{j,g/G}.  q [w][Hq][d], k and v [n][Hkv][d]; returns [w][Hq][d] float64."""
+    lib = _load()
+    q, k, v = _c64(q), _c64(k), _c64(v)
+    w, hq, d = q.shape
+    n, hkv, d2 = k.shape
+    assert d == d2 and v.shape == k.shape and hq % hkv == 0
+    out = np.zeros((w, hq, d), dtype=np.float64)
+    for r in range(w):
+        for g in range(hq):
+            lib.orc_decode_row(_d(q), _d(k), _d(v), n, hq, hkv, d, r, g, out[r, g].ctypes.data_as(_dp))
+    return out

@@ -292,3 +292,32 @@ void orc_compress_head(const double* q, const double* k, int32_t n, int32_t w, i
   orc_combine(a, phi, gate, n, n_frames, off, gh, gw, alpha, css_enable, s);
   orc_topk(s, n, budget, idx_out);
 }
+
+/* ------------------------------------ consumer: decode over the cache */
+
+/* Scaled dot-product attention of one query row over a KV cache, the
+ * operation a decoder runs at every generated token (the consumer of the
+ * compressed cache: the efficiency study's decode latency compares the full
+ * and the compressed cache).  For query head g of window row r:
+ *   out = sum_j softmax_j(q_{r,g} . k_{j,h} / sqrt(d)) v_{j,h},  h = g / G,
+ * over all n cached tokens, with the softmax materialised in full. */
+void orc_decode_row(const double* q, const double* k, const double* v, int32_t n, int32_t hq,
+                    int32_t hkv, int32_t d, int32_t r, int32_t g, double* out) {
+  const int32_t G = hq / hkv, h = g / G;
+  const double* qrow = q + ((size_t)r * hq + g) * d;
+  double* logit = (double*)malloc(sizeof(double) * (size_t)(n > 0 ? n : 1));
+  double mx = -INFINITY;
+  for (int32_t j = 0; j < n; ++j) {
+    logit[j] = dot(qrow, key_row(k, hkv, d, j, h), d) / sqrt((double)d);
+    if (logit[j] > mx) mx = logit[j];
+  }
+  double z = 0.0;
+  for (int32_t j = 0; j < n; ++j) z += exp(logit[j] - mx);
+  for (int32_t e = 0; e < d; ++e) out[e] = 0.0;
+  for (int32_t j = 0; j < n; ++j) {
+    const double p = exp(logit[j] - mx) / z;
+    const double* vrow = key_row(v, hkv, d, j, h);
+    for (int32_t e = 0; e < d; ++e) out[e] += p * vrow[e];
+  }
+  free(logit);
+}

@@ -470,3 +470,51 @@ def test_end_to_end_text_permutation_equivariance():
     inv = np.argsort(perm)
     for h in range(2):
         np.testing.assert_array_equal(b["idx"][h], np.sort(inv[a["idx"][h]]))
+
+
+# ------------------------------------------- consumer: decode over the cache
+
+def test_decode_single_and_equal_keys():
+    rng = np.random.default_rng(21)
+    d, hq, hkv = 8, 4, 2
+    q = rng.standard_normal((2, hq, d))
+    v = rng.standard_normal((5, hkv, d))
+    # one cached token: the output is its value row, whatever the query
+    out = oracle.decode_attention(q, rng.standard_normal((1, hkv, d)), v[:1])
+    for g in range(hq):
+        np.testing.assert_allclose(out[:, g], np.broadcast_to(v[0, g // 2], (2, d)), rtol=0, atol=1e-15)
+    # equal keys: uniform weights, the output is the mean value row of the head
+    k = np.tile(rng.standard_normal((1, hkv, d)), (5, 1, 1))
+    out = oracle.decode_attention(q, k, v)
+    for g in range(hq):
+        np.testing.assert_allclose(out[:, g], np.broadcast_to(v[:, g // 2].mean(0), (2, d)), rtol=1e-13,
+                                   atol=1e-15)
+
+
+def test_decode_dominant_key_and_weights_sum_to_one():
+    rng = np.random.default_rng(22)
+    d, hq, hkv, n = 16, 2, 1, 7
+    q = rng.standard_normal((1, hq, d))
+    k = rng.standard_normal((n, hkv, d)) * 0.01
+    k[3, 0] = 100.0 * q[0, 0] / np.linalg.norm(q[0, 0])   # dominates head 0's softmax
+    v = rng.standard_normal((n, hkv, d))
+    out = oracle.decode_attention(q, k, v)
+    np.testing.assert_allclose(out[0, 0], v[3, 0], rtol=0, atol=1e-12)
+    # constant value rows: convex weights return the constant exactly (up to rounding)
+    out = oracle.decode_attention(q, k, np.full((n, hkv, d), 2.5))
+    np.testing.assert_allclose(out, 2.5, rtol=1e-14)
+
+
+def test_decode_library_attention():
+    # the textbook case against the library routine (fp64 CPU scaled-dot-product attention)
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(23)
+    w, hq, hkv, n, d = 3, 6, 2, 40, 32
+    q, k, v = rng.standard_normal((w, hq, d)), rng.standard_normal((n, hkv, d)), rng.standard_normal((n, hkv, d))
+    out = oracle.decode_attention(q, k, v)
+    G = hq // hkv
+    tq = torch.from_numpy(q).permute(1, 0, 2)                                     # [hq][w][d]
+    tk = torch.from_numpy(k).permute(1, 0, 2).repeat_interleave(G, 0)              # [hq][n][d]
+    tv = torch.from_numpy(v).permute(1, 0, 2).repeat_interleave(G, 0)
+    ref = torch.nn.functional.scaled_dot_product_attention(tq, tk, tv).permute(1, 0, 2).numpy()
+    np.testing.assert_allclose(out, ref, rtol=1e-12, atol=1e-14)
