@@ -241,6 +241,23 @@ STLITE_API stlite_status stlite_workspace_size_varlen(const stlite_shape* shape,
                                                       const int32_t* cu_seqlens, const stlite_frames* frames,
                                                       const stlite_params* params, size_t* bytes);
 
+/* Consumer of the compressed cache: attention of query rows over a KV cache,
+ * the operation a decoder runs for every generated token (the paper's
+ * efficiency study compares decode latency with the full and the compressed
+ * cache):  out[r][g][:] = sum_j softmax_j(q[r][g] . k[j][h] / sqrt(d)) v[j][h][:]
+ * with h = g / (Hq/Hkv), over all n cached rows, no mask.
+ * shape: n_tokens = cache rows n (N for the full cache, B after
+ *   compaction), window = query rows w, Hq / Hkv <= 16.
+ * q [w][Hq][d], k and v [n][Hkv][d] (device, shape->dtype); out: device float
+ *   [w][Hq][d].  ws: at least stlite_decode_workspace_size bytes (split
+ *   partials; need not be zeroed). */
+STLITE_API stlite_status stlite_decode_attention(const stlite_shape* shape, const void* q, const void* k,
+                                                 const void* v, float* out, void* ws, size_t ws_bytes,
+                                                 void* stream);
+
+/* Workspace bytes of stlite_decode_attention for this shape. */
+STLITE_API stlite_status stlite_decode_workspace_size(const stlite_shape* shape, size_t* bytes);
+
 /* Reads and clears the workspace's device error word (synchronises `stream`).
  * *status receives STLITE_OK, STLITE_ETIMEOUT if a kernel's bounded wait ran
  * out since the last read, or STLITE_ECUDA if a kernel found its launch

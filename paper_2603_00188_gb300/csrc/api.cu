@@ -537,6 +537,35 @@ stlite_status stlite_compress_varlen(const stlite_shape* shape, int32_t n_seqs, 
   return STLITE_OK;
 }
 
+// Decode attention over a (compressed) cache.
+static stlite_status check_decode(const stlite_shape* shape) {
+  stlite_status s = check_shape(shape);
+  if (s != STLITE_OK) return s;
+  if (shape->n_q_heads / shape->n_kv_heads > kDecMaxG) return STLITE_EUNSUPPORTED;
+  return STLITE_OK;
+}
+
+stlite_status stlite_decode_workspace_size(const stlite_shape* shape, size_t* bytes) {
+  if (!bytes) return STLITE_EINVAL;
+  stlite_status s = check_decode(shape);
+  if (s != STLITE_OK) return s;
+  *bytes = decode_workspace_bytes(shape->n_tokens, shape->n_q_heads, shape->n_kv_heads, shape->window);
+  return STLITE_OK;
+}
+
+stlite_status stlite_decode_attention(const stlite_shape* shape, const void* q, const void* k, const void* v,
+                                      float* out, void* ws, size_t ws_bytes, void* stream) {
+  stlite_status s = check_decode(shape);
+  if (s != STLITE_OK) return s;
+  if (!q || !k || !v || !out || !ws) return STLITE_EINVAL;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(out) || !aligned16(ws)) return STLITE_EINVAL;
+  if (ws_bytes < decode_workspace_bytes(shape->n_tokens, shape->n_q_heads, shape->n_kv_heads, shape->window))
+    return STLITE_EWORKSPACE;
+  return cuda_status(launch_decode(shape->dtype == STLITE_BF16 ? kBF16 : kF32, q, k, v, shape->n_tokens,
+                                   shape->n_q_heads, shape->n_kv_heads, shape->window, out, ws,
+                                   static_cast<cudaStream_t>(stream)));
+}
+
 stlite_status stlite_device_status(void* ws, void* stream, stlite_status* status) {
   if (!ws || !status || !aligned16(ws)) return STLITE_EINVAL;
   cudaStream_t st = static_cast<cudaStream_t>(stream);

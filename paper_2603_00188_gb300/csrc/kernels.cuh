@@ -168,4 +168,12 @@ int select_max_tokens();
 // v, k_out, v_out from io).
 cudaError_t launch_gather(const Problem& p, int budget, const LayerPtrs& io, cudaStream_t st);
 
+// ---- consumer: decode attention over a (compressed) cache -----------------
+constexpr int kDecMaxG = 16;  // query heads per KV head
+int decode_splits(int n, int hkv, int w);
+size_t decode_workspace_bytes(int n, int hq, int hkv, int w);
+// out [w][hq][128] fp32; q [w][hq][128], k/v [n][hkv][128] of dtype dt.
+cudaError_t launch_decode(DType dt, const void* q, const void* k, const void* v, int n, int hq, int hkv, int w,
+                          float* out, void* ws, cudaStream_t st);
+
 }  // namespace stl

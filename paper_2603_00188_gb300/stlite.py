@@ -28,7 +28,7 @@ EXPORTED = ("stlite_budget", "stlite_workspace_size", "stlite_score", "stlite_ga
             "stlite_spatial_saliency", "stlite_select_topk", "stlite_compact",
             "stlite_compress_layer", "stlite_device_status", "stlite_timing_enable", "stlite_timing_read",
             "stlite_status_string", "stlite_score_noalloc", "stlite_compress_layers", "stlite_compress_varlen",
-            "stlite_workspace_size_varlen")
+            "stlite_workspace_size_varlen", "stlite_decode_attention", "stlite_decode_workspace_size")
 
 
 class Shape(ctypes.Structure):
@@ -86,6 +86,8 @@ _sig = {
     "stlite_workspace_size_varlen": (_S, [ctypes.POINTER(Shape), ctypes.c_int32, ctypes.POINTER(ctypes.c_int32),
                                           ctypes.POINTER(Frames), ctypes.POINTER(Params),
                                           ctypes.POINTER(ctypes.c_size_t)]),
+    "stlite_decode_attention": (_S, [ctypes.POINTER(Shape), _P, _P, _P, _P, _P, ctypes.c_size_t, _P]),
+    "stlite_decode_workspace_size": (_S, [ctypes.POINTER(Shape), ctypes.POINTER(ctypes.c_size_t)]),
 }
 for _name, (_res, _args) in _sig.items():
     _f = getattr(_lib, _name)
@@ -257,6 +259,29 @@ def stlite_compress_varlen(q, k, v, cu_seqlens, frames_list, params, k_out, v_ou
                                        cb.ctypes.data_as(ip), _ptr(ws), ws.numel(), _stream(stream)),
            "stlite_compress_varlen")
     return cb
+
+
+def stlite_decode_workspace_size(shape: Shape) -> int:
+    out = ctypes.c_size_t()
+    _check(_lib.stlite_decode_workspace_size(ctypes.byref(shape), ctypes.byref(out)), "stlite_decode_workspace_size")
+    return int(out.value)
+
+
+def stlite_decode_attention(q, k, v, out, ws, stream=None):
+    """Attention of the query rows q [w][Hq][d] over the cache k, v [n][Hkv][d]
+    (full or compacted) into out [w][Hq][d] float32."""
+    sh = make_shape(q, k)
+    _check(_lib.stlite_decode_attention(ctypes.byref(sh), _ptr(q), _ptr(k), _ptr(v), _ptr(out), _ptr(ws),
+                                        ws.numel(), _stream(stream)), "stlite_decode_attention")
+
+
+def decode_attention(q, k, v, stream=None):
+    """Allocates the output and the workspace and runs stlite_decode_attention."""
+    sh = make_shape(q, k)
+    ws = torch.empty(stlite_decode_workspace_size(sh), dtype=torch.uint8, device=k.device)
+    out = torch.empty(q.shape, dtype=torch.float32, device=k.device)
+    stlite_decode_attention(q, k, v, out, ws, stream)
+    return out
 
 
 def stlite_device_status(ws, stream=None) -> int:

@@ -1,0 +1,66 @@
+"""Decode attention over a full and a compressed cache (the consumer of the
+compressed cache) through the C ABI, against the fp64 oracle."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2603_00188_gb300 import synth
+from parity import exact64, to_device
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def st():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2603_00188_gb300 import build
+    build.build()
+    from paper_2603_00188_gb300 import stlite
+    return stlite
+
+
+def _close(got, ref, v64):
+    # fp32 scores and sums: |g - o| <= 1e-3 |o| + 2e-4 max|v| (the output is a
+    # convex combination of value rows, so max|v| bounds it)
+    tol = 1e-3 * np.abs(ref) + 2e-4 * np.abs(v64).max()
+    bad = np.abs(got - ref) > tol
+    assert not bad.any(), ("decode mismatch", int(bad.sum()), float(np.abs(got - ref).max()))
+
+
+@pytest.mark.parametrize("w,hq,hkv,n,dtype", [(1, 28, 4, 1000, torch.bfloat16), (3, 28, 4, 257, torch.bfloat16),
+                                              (2, 16, 1, 33, torch.bfloat16), (1, 4, 4, 1, torch.bfloat16),
+                                              (2, 12, 2, 513, torch.float32), (1, 8, 2, 31, torch.float32)])
+def test_decode_matches_oracle(st, w, hq, hkv, n, dtype):
+    g = torch.Generator().manual_seed(n * 7 + hq)
+    q = torch.randn((w, hq, 128), generator=g).to(dtype).cuda()
+    k = torch.randn((n, hkv, 128), generator=g).to(dtype).cuda()
+    v = torch.randn((n, hkv, 128), generator=g).to(dtype).cuda()
+    out = st.decode_attention(q, k, v)
+    torch.cuda.synchronize()
+    ref = oracle.decode_attention(exact64(q), exact64(k), exact64(v))
+    _close(out.cpu().numpy().astype(np.float64), ref, exact64(v))
+
+
+def test_decode_over_compressed_cache(st):
+    # compress one layer, then decode a probe row over the compacted rows
+    wl = synth.scaled("traj50", 4)
+    q, k, v = to_device(wl)
+    ko, vo, idx = st.compress_layer(q, k, v, wl.frames, beta=wl.beta)
+    probe = q[-1:].contiguous()                      # the last window row as the next query
+    full = st.decode_attention(probe, k, v)
+    comp = st.decode_attention(probe, ko, vo)
+    torch.cuda.synchronize()
+    _close(comp.cpu().numpy().astype(np.float64),
+           oracle.decode_attention(exact64(probe), exact64(ko), exact64(vo)), exact64(vo))
+    _close(full.cpu().numpy().astype(np.float64),
+           oracle.decode_attention(exact64(probe), exact64(k), exact64(v)), exact64(v))
+    assert ko.shape[0] == idx.shape[1] < k.shape[0]
+
+
+def test_decode_rejects(st):
+    q = torch.zeros((1, 32, 128), dtype=torch.bfloat16, device="cuda")
+    k = torch.zeros((10, 1, 128), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(st.StliteError):
+        st.decode_attention(q, k, k)                  # 32 query heads per KV head > 16
