@@ -53,6 +53,7 @@ def parse():
     ap.add_argument("--layers", type=int, default=LAYERS)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-decode", action="store_true", help="skip the decode-over-the-cache measurement")
     return ap.parse_args()
 
 
@@ -419,6 +420,49 @@ def run_gpu(args):
     roof["traffic"] = traffic_for(dom) if L == LAYERS else None
     roof["peak_source"] = peaks["source"] + (" burst" if roof["unit"] == "TFLOP/s" else "")
 
+    # ---- consumer: one decode step (a query row per layer) over the full and
+    # the compressed caches of all layers, each step one CUDA graph
+    decode = None
+    if not args.no_decode:
+        probes = [qs[l][-1:].contiguous() for l in range(L)]    # the last window row as the next query
+        dsh = stlite.make_shape(probes[0], ks[0])
+        dws = torch.empty(stlite.stlite_decode_workspace_size(dsh), dtype=torch.uint8, device=dev)
+        douts = [torch.empty((1, HQ, D), dtype=torch.float32, device=dev) for _ in range(L)]
+
+        def decode_ms(kk, vv):
+            def one():
+                for l in range(L):
+                    stlite.stlite_decode_attention(probes[l], kk[l], vv[l], douts[l], dws, stream)
+            with torch.cuda.stream(stream):
+                for _ in range(3):
+                    one()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                one()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            reps = max(10, args.steps)
+            with torch.cuda.stream(stream):
+                for _ in range(3):
+                    g.replay()
+                a.record(stream)
+                for _ in range(reps):
+                    g.replay()
+                b.record(stream)
+            torch.cuda.synchronize()
+            return a.elapsed_time(b) / reps
+
+        t_full = decode_ms(ks, vs)
+        t_comp = decode_ms(kos, vos)
+        row = HKV * D * 2 * 2   # one cached token's key and value rows, bf16
+        decode = dict(layers=L, cache_rows_full=N_TOK, cache_rows_compressed=budget,
+                      full_us_per_step=t_full * 1e3, compressed_us_per_step=t_comp * 1e3,
+                      speedup=t_full / t_comp,
+                      full_gbs=N_TOK * row * L / (t_full * 1e-3) / 1e9,
+                      compressed_gbs=budget * row * L / (t_comp * 1e-3) / 1e9,
+                      peak_gbs=peaks["hbm"],
+                      note="one query row per layer attends over every cached row (keys and values read once); "
+                           "full = N rows, compressed = the B kept rows")
+
     # ---- end to end: host (pinned) inputs -> device -> compress -> host outputs.
     # Q and K of every layer are copied to the device (every stage reads all
     # keys); V stays in page-locked host memory, from which the compaction
@@ -526,7 +570,7 @@ def run_gpu(args):
                     roofline=roof, kernels=kernels, gpu_launches=per_step_launches * args.steps,
                     clocks=dict(sm_mhz=clk["sm_mhz"], sm_max_mhz=clk["sm_max_mhz"], reasons=clk["reasons"],
                                 samples=clk["samples"]),
-                    e2e=e2e, cpu_baseline=cpu)
+                    e2e=e2e, cpu_baseline=cpu, decode=decode)
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()

@@ -18,7 +18,7 @@
 
 namespace stl {
 
-constexpr int kDecThreads = 128;  // 4 warps
+constexpr int kDecThreads = 256;  // 8 warps
 constexpr float kDecLog2e = 1.4426950408889634f;
 constexpr int kDecWarps = kDecThreads / 32;
 
@@ -51,7 +51,7 @@ __device__ __forceinline__ float weight(float a, float m) { return a == -CUDART_
 // Dynamic shared memory: qs[G][128] (query rows times log2(e)/sqrt(d)), then
 // per warp o[G][128] and (m, l)[G].
 template <typename T, int GM>
-__global__ void __launch_bounds__(kDecThreads) k_decode_split(const T* __restrict__ q, const T* __restrict__ k,
+__global__ void __launch_bounds__(kDecThreads, 2) k_decode_split(const T* __restrict__ q, const T* __restrict__ k,
                                                               const T* __restrict__ v, int n, int hq, int hkv,
                                                               int per, float* part_o, float2* part_ml) {
   extern __shared__ float4 dec_smem[];
@@ -85,7 +85,7 @@ __global__ void __launch_bounds__(kDecThreads) k_decode_split(const T* __restric
     for (int g = 0; g < GM; ++g) s[g] = 0.f;
     if (t < j1) {
       const T* kr = k + (size_t)t * rs + (size_t)h * kD;
-#pragma unroll 4
+#pragma unroll 8
       for (int c = 0; c < kD; c += 8) {
         float kf[8];
         load8(kr + c, kf);
@@ -115,18 +115,27 @@ __global__ void __launch_bounds__(kDecThreads) k_decode_split(const T* __restric
         m[g] = mn;
       }
     }
-    // value rows: lane owns dimensions 4*lane .. 4*lane + 3
+    // value rows: lane owns dimensions 4*lane .. 4*lane + 3; eight rows'
+    // loads are in flight before their products
     const int cnt = min(32, j1 - base);
-    for (int tt = 0; tt < cnt; ++tt) {
-      const float4 vv = Elem<T>::load4(v + (size_t)(base + tt) * rs + (size_t)h * kD + 4 * lane);
+    for (int t0 = 0; t0 < cnt; t0 += 8) {
+      float4 vv[8];
 #pragma unroll
-      for (int g = 0; g < GM; ++g) {
-        if (g < G) {
-          const float pg = __shfl_sync(0xffffffffu, p[g], tt);
-          o[g][0] = fmaf(pg, vv.x, o[g][0]);
-          o[g][1] = fmaf(pg, vv.y, o[g][1]);
-          o[g][2] = fmaf(pg, vv.z, o[g][2]);
-          o[g][3] = fmaf(pg, vv.w, o[g][3]);
+      for (int u = 0; u < 8; ++u)
+        if (t0 + u < cnt) vv[u] = Elem<T>::load4(v + (size_t)(base + t0 + u) * rs + (size_t)h * kD + 4 * lane);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        if (t0 + u < cnt) {
+#pragma unroll
+          for (int g = 0; g < GM; ++g) {
+            if (g < G) {
+              const float pg = __shfl_sync(0xffffffffu, p[g], t0 + u);
+              o[g][0] = fmaf(pg, vv[u].x, o[g][0]);
+              o[g][1] = fmaf(pg, vv[u].y, o[g][1]);
+              o[g][2] = fmaf(pg, vv[u].z, o[g][2]);
+              o[g][3] = fmaf(pg, vv[u].w, o[g][3]);
+            }
+          }
         }
       }
     }
@@ -141,8 +150,9 @@ __global__ void __launch_bounds__(kDecThreads) k_decode_split(const T* __restric
     }
   }
   __syncthreads();
-  const int c = threadIdx.x;  // one dimension per thread
-  for (int g = 0; g < G; ++g) {
+  // one (query head, dimension) pair per thread and step
+  for (int e = threadIdx.x; e < G * kD; e += kDecThreads) {
+    const int g = e / kD, c = e % kD;
     float M = -CUDART_INF_F;
     for (int w = 0; w < kDecWarps; ++w) M = fmaxf(M, wml[w * G + g].x);
     float L = 0.f, O = 0.f;
@@ -158,29 +168,67 @@ __global__ void __launch_bounds__(kDecThreads) k_decode_split(const T* __restric
   (void)nsplit;
 }
 
-// out[r][g][c] = merge over the splits.  grid (hq, w), one thread per dimension.
+// out[r][g][c] = merge over the splits.  grid (hq, w), one thread per
+// dimension: the splits' weights exp2(m_s - M) and the normaliser are formed
+// once in shared memory, then every thread sums its dimension over the splits
+// with eight partial loads in flight.
+constexpr int kDecMaxSplits = 1024;
 __global__ void __launch_bounds__(kD) k_decode_combine(const float* part_o, const float2* part_ml, int nsplit,
                                                        int hq, int w, float* out) {
-  const int g = blockIdx.x, r = blockIdx.y, c = threadIdx.x;
-  float M = -CUDART_INF_F;
-  for (int s = 0; s < nsplit; ++s) M = fmaxf(M, part_ml[((size_t)s * w + r) * hq + g].x);
-  float L = 0.f, O = 0.f;
-  for (int s = 0; s < nsplit; ++s) {
-    const size_t slot = ((size_t)s * w + r) * hq + g;
-    const float a = weight(part_ml[slot].x, M);
-    L = fmaf(part_ml[slot].y, a, L);
-    O = fmaf(part_o[slot * kD + c], a, O);
+  __shared__ float wts[kDecMaxSplits];
+  __shared__ float red[kD / 32];
+  __shared__ float bc[2];
+  const int g = blockIdx.x, r = blockIdx.y, c = threadIdx.x, lane = c & 31, wp = c >> 5;
+  float mx = -CUDART_INF_F;
+  for (int s = c; s < nsplit; s += kD) mx = fmaxf(mx, part_ml[((size_t)s * w + r) * hq + g].x);
+  mx = warp_max(mx);
+  if (lane == 0) red[wp] = mx;
+  __syncthreads();
+  if (c == 0) {
+    float M = red[0];
+    for (int i = 1; i < kD / 32; ++i) M = fmaxf(M, red[i]);
+    bc[0] = M;
   }
-  out[((size_t)r * hq + g) * kD + c] = O / L;
+  __syncthreads();
+  const float M = bc[0];
+  float ls = 0.f;
+  for (int s = c; s < nsplit; s += kD) {
+    const float2 ml = part_ml[((size_t)s * w + r) * hq + g];
+    const float a = weight(ml.x, M);
+    wts[s] = a;
+    ls = fmaf(ml.y, a, ls);
+  }
+  ls = warp_sum(ls);
+  __syncthreads();  // red is reused
+  if (lane == 0) red[wp] = ls;
+  __syncthreads();
+  if (c == 0) {
+    float L = 0.f;
+    for (int i = 0; i < kD / 32; ++i) L += red[i];
+    bc[1] = L;
+  }
+  __syncthreads();
+  float O = 0.f;
+  int s = 0;
+  for (; s + 8 <= nsplit; s += 8) {
+    float x[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) x[u] = part_o[(((size_t)(s + u) * w + r) * hq + g) * kD + c];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) O = fmaf(x[u], wts[s + u], O);
+  }
+  for (; s < nsplit; ++s) O = fmaf(part_o[(((size_t)s * w + r) * hq + g) * kD + c], wts[s], O);
+  out[((size_t)r * hq + g) * kD + c] = O / bc[1];
 }
 
 int decode_splits(int n, int hkv, int w) {
   int dev = 0, sms = 152;
   if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  // about four CTAs per SM, each with at least 128 cached rows
-  long long s = (4LL * sms + (long long)hkv * w - 1) / ((long long)hkv * w);
-  const long long cap = (n + 127) / 128;
+  // about two CTAs per SM, each with at least 256 cached rows
+  long long s = (2LL * sms + (long long)hkv * w - 1) / ((long long)hkv * w);
+  const long long cap = (n + 255) / 256;
   if (s > cap) s = cap;
+  if (s > kDecMaxSplits) s = kDecMaxSplits;
   if (s < 1) s = 1;
   return (int)s;
 }
@@ -200,9 +248,12 @@ cudaError_t launch_decode(DType dt, const void* q, const void* k, const void* v,
   const size_t smem = (size_t)G * kD * 4 + (size_t)kDecWarps * G * kD * 4 + (size_t)kDecWarps * G * 8;
   dim3 grid(nsplit, hkv, w);
   // register arrays sized for the group: G <= 4, <= 8 or <= 16 query heads
+  cudaError_t fe = cudaSuccess;
   auto run = [&](auto tag, auto gm) {
     using T = decltype(tag);
     constexpr int GM = decltype(gm)::value;
+    fe = cudaFuncSetAttribute(k_decode_split<T, GM>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (fe != cudaSuccess) return;
     k_decode_split<T, GM><<<grid, kDecThreads, smem, st>>>(static_cast<const T*>(q), static_cast<const T*>(k),
                                                            static_cast<const T*>(v), n, hq, hkv, per, part_o,
                                                            part_ml);
@@ -222,6 +273,7 @@ cudaError_t launch_decode(DType dt, const void* q, const void* k, const void* v,
       else run(float(), G16());
     }
   }
+  if (fe != cudaSuccess) return fe;
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   TimingScope ts("decode_combine", st);
