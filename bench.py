@@ -287,6 +287,28 @@ def traffic_for(kernel: str):
     return None if e is None else e.get("dram_bytes_per_launch_full")
 
 
+# ------------------------------------------------------- critical hit rate
+
+def gpu_critical_hit_rate(stlite, q_probe, k, idx_keep, stream=None):
+    """Per KV head, the share of a probe query's B most-attended tokens that
+    the compressed cache kept: the probe's window score over every cached key
+    (Eq. 2 with the probe as the only window row, stlite_score) and its Top_B
+    (stlite_select_topk with no gate and no CSS: S = A) run in the library's
+    kernels; only the set intersection is a torch op."""
+    import torch
+    n, hkv = k.shape[0], k.shape[1]
+    b = idx_keep.shape[1]
+    none = ([], [], [])
+    prm = stlite.make_params(1.0, k_override=b, alpha=0.0, tsg_enable=0, css_enable=0)
+    sh = stlite.make_shape(q_probe, k)
+    ws = stlite.workspace(sh, none, prm, device=k.device)
+    a = torch.empty((hkv, n), dtype=torch.float32, device=k.device)
+    top = torch.empty((hkv, b), dtype=torch.int32, device=k.device)
+    stlite.stlite_score(q_probe, k, a, ws, stream)
+    stlite.stlite_select_topk(q_probe, k, none, prm, a, None, None, b, top, None, ws, stream)
+    return torch.stack([torch.isin(idx_keep[h], top[h]).sum() for h in range(hkv)]).double() / b
+
+
 # ------------------------------------------------------------ multi-rank glue
 
 def dist_env():
@@ -453,6 +475,8 @@ def run_gpu(args):
 
         t_full = decode_ms(ks, vs)
         t_comp = decode_ms(kos, vos)
+        # critical hit rate of the same probe rows: mean over layers and KV heads
+        chr_ = torch.stack([gpu_critical_hit_rate(stlite, probes[l], ks[l], idxs[l], stream) for l in range(L)])
         row = HKV * D * 2 * 2   # one cached token's key and value rows, bf16
         decode = dict(layers=L, cache_rows_full=N_TOK, cache_rows_compressed=budget,
                       full_us_per_step=t_full * 1e3, compressed_us_per_step=t_comp * 1e3,
@@ -460,8 +484,10 @@ def run_gpu(args):
                       full_gbs=N_TOK * row * L / (t_full * 1e-3) / 1e9,
                       compressed_gbs=budget * row * L / (t_comp * 1e-3) / 1e9,
                       peak_gbs=peaks["hbm"],
-                      note="one query row per layer attends over every cached row (keys and values read once); "
-                           "full = N rows, compressed = the B kept rows")
+                      critical_hit_rate=float(chr_.mean()), critical_hit_rate_min=float(chr_.min()),
+                      note="one query row per layer (the last window row) attends over every cached row (keys and "
+                           "values read once); full = N rows, compressed = the B kept rows; critical hit rate = "
+                           "share of that probe's B most-attended tokens kept (synthetic inputs)")
 
     # ---- end to end: host (pinned) inputs -> device -> compress -> host outputs.
     # Q and K of every layer are copied to the device (every stage reads all

@@ -260,3 +260,17 @@ def decode_attention(q, k, v) -> np.ndarray:
         for g in range(hq):
             lib.orc_decode_row(_d(q), _d(k), _d(v), n, hq, hkv, d, r, g, out[r, g].ctypes.data_as(_dp))
     return out
+
+
+def critical_hit_rate(idx_keep, q_probe, k) -> np.ndarray:
+    """Share of the probe query's B most-attended tokens (per KV head: its
+    window score with the probe as the only window row, Eq. 2 with w = 1)
+    that the compressed cache kept: |I_keep & Top_B(A_probe)| / B."""
+    idx_keep = np.asarray(idx_keep)
+    hkv, b = idx_keep.shape
+    a = abase(q_probe, k)
+    out = np.zeros(hkv, dtype=np.float64)
+    for h in range(hkv):
+        top = topk(a[h:h + 1], b)[0]
+        out[h] = len(np.intersect1d(top, idx_keep[h])) / b
+    return out

@@ -518,3 +518,20 @@ def test_decode_library_attention():
     tv = torch.from_numpy(v).permute(1, 0, 2).repeat_interleave(G, 0)
     ref = torch.nn.functional.scaled_dot_product_attention(tq, tk, tv).permute(1, 0, 2).numpy()
     np.testing.assert_allclose(out, ref, rtol=1e-12, atol=1e-14)
+
+
+def test_critical_hit_rate_cases():
+    wl = _tiny_traj(seed=8, n_steps=3, w=1)
+    # kept set = Top_B of the probe's own attention (alpha = 0, TSG off, the
+    # probe as the only window row): every critical token is kept
+    out = oracle.compress_layer(wl.q, wl.k, wl.frames, beta=0.3, tsg_enable=0, css_enable=0)
+    np.testing.assert_array_equal(oracle.critical_hit_rate(out["idx"], wl.q, wl.k), 1.0)
+    # beta = 1 keeps everything
+    out = oracle.compress_layer(wl.q, wl.k, wl.frames, beta=1.0)
+    np.testing.assert_array_equal(oracle.critical_hit_rate(out["idx"], wl.q, wl.k), 1.0)
+    # the complement of the critical set scores 0
+    b = oracle.budget(wl.n, 0.3)
+    a = oracle.abase(wl.q, wl.k)
+    top = oracle.topk(a, b)
+    rest = np.stack([np.setdiff1d(np.arange(wl.n), top[h])[:b] for h in range(a.shape[0])])
+    np.testing.assert_array_equal(oracle.critical_hit_rate(rest, wl.q, wl.k), 0.0)

@@ -403,3 +403,26 @@ def test_text_permutation_equivariance(st):
     for h in range(k.shape[1]):
         flips = set(np.nonzero(np.abs(ref["rho"][h] - ref["tau"][h]) <= 1e-3 * abs(ref["tau"][h]) + COS_ATOL)[0].tolist())
         check_kept_sets(np.sort(perm[ib[h]]), ia[h], ref["s"][h], b, s_tol, allowed_extra=flips)
+
+
+# ------------------------------------------------------------ critical hit rate
+
+def test_critical_hit_rate(st):
+    import bench
+    # consistency: alpha = 0, TSG off, the probe as the only window row -> the
+    # kept set is exactly the probe's Top_B, so the GPU's rate is 1
+    wl = synth.trajectory(n_steps=3, gh=8, gw=9, n_text=5, hq=8, hkv=2, w=1, beta=0.25, seed=(950,))
+    q, k, v = to_device(wl)
+    _, _, idx = st.compress_layer(q, k, v, wl.frames, beta=wl.beta, tsg_enable=0, css_enable=0, alpha=0.0)
+    assert torch.equal(bench.gpu_critical_hit_rate(st, q, k, idx), torch.ones(2, dtype=torch.float64, device="cuda"))
+    # the full method on a 4-frame trajectory: the GPU's rate against the
+    # oracle's (both kept sets and both top sets may differ by swaps at their
+    # thresholds; each swap moves the rate by at most 1/B)
+    wl = synth.scaled("traj50", 4)
+    q, k, v = to_device(wl)
+    _, _, idx = st.compress_layer(q, k, v, wl.frames, beta=wl.beta)
+    probe = q[-1:].contiguous()
+    got = bench.gpu_critical_hit_rate(st, probe, k, idx).cpu().numpy()
+    ref_keep = oracle.compress_layer(exact64(q), exact64(k), wl.frames, beta=wl.beta, threads=THREADS)["idx"]
+    ref = oracle.critical_hit_rate(ref_keep, exact64(probe), exact64(k))
+    assert np.all(np.abs(got - ref) <= 4.0 / idx.shape[1]), (got, ref)
