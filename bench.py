@@ -448,7 +448,7 @@ def run_gpu(args):
     if not args.no_decode:
         probes = [qs[l][-1:].contiguous() for l in range(L)]    # the last window row as the next query
         dsh = stlite.make_shape(probes[0], ks[0])
-        dws = torch.empty(stlite.stlite_decode_workspace_size(dsh), dtype=torch.uint8, device=dev)
+        dws = torch.zeros(stlite.stlite_decode_workspace_size(dsh), dtype=torch.uint8, device=dev)
         douts = [torch.empty((1, HQ, D), dtype=torch.float32, device=dev) for _ in range(L)]
 
         def decode_ms(kk, vv):
@@ -475,6 +475,7 @@ def run_gpu(args):
 
         t_full = decode_ms(ks, vs)
         t_comp = decode_ms(kos, vos)
+        assert stlite.stlite_device_status(dws, stream) == stlite.STLITE_OK
         # critical hit rate of the same probe rows: mean over layers and KV heads
         chr_ = torch.stack([gpu_critical_hit_rate(stlite, probes[l], ks[l], idxs[l], stream) for l in range(L)])
         row = HKV * D * 2 * 2   # one cached token's key and value rows, bf16

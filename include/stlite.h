@@ -250,7 +250,9 @@ STLITE_API stlite_status stlite_workspace_size_varlen(const stlite_shape* shape,
  *   compaction), window = query rows w, Hq / Hkv <= 16.
  * q [w][Hq][d], k and v [n][Hkv][d] (device, shape->dtype); out: device float
  *   [w][Hq][d].  ws: at least stlite_decode_workspace_size bytes (split
- *   partials; need not be zeroed). */
+ *   partials), zero-filled before its first use: its first word is the
+ *   device error word that stlite_device_status reads (a bounded wait that
+ *   ran out records STLITE_ETIMEOUT there). */
 STLITE_API stlite_status stlite_decode_attention(const stlite_shape* shape, const void* q, const void* k,
                                                  const void* v, float* out, void* ws, size_t ws_bytes,
                                                  void* stream);

@@ -15,6 +15,7 @@
 #include <type_traits>
 
 #include "kernels.cuh"
+#include "ptx.cuh"
 
 namespace stl {
 
@@ -168,6 +169,225 @@ __global__ void __launch_bounds__(kDecThreads, 2) k_decode_split(const T* __rest
   (void)nsplit;
 }
 
+// ---------------------------------------------------------------------------
+// bf16 caches: key and value tiles of 64 cached rows stream through a ring of
+// shared-memory stages by TMA (128-byte swizzle, the layout of the tensor-core
+// kernels); warp 16 issues the copies, warps 0-15 consume each tile in three
+// phases separated by a named barrier, each key and value element read once
+// per tile:
+//   1. scores: thread (row t = tid % 64, slice sl = tid / 64) dots dimensions
+//      16 sl .. 16 sl + 15 of its row's key with every query head of the
+//      group (a warp's lanes share the slice, so query reads are broadcasts);
+//      the eight slices' partial scores are summed through shared memory;
+//   2. online softmax: warp w updates (max, sum) of query head w and turns
+//      the tile's scores into probabilities;
+//   3. values: thread (dimension pair dp = tid % 64, row slice ts = tid / 64)
+//      accumulates p * v over rows ts, ts + 8, ... for every query head; the
+//      eight row slices are summed once, after the last tile.
+// Scores and probabilities are kept row-slice-major: entry (g, t) at
+// g * 64 + (t % 8) * 8 + t / 8.
+// Every mbarrier wait is made by one thread and its outcome shared through
+// shared memory after the named barrier, so all consumer warps take the same
+// path and always meet at every barrier.
+constexpr int kDecTile = 64;                         // cached rows per tile
+constexpr int kDecStages = 4;
+constexpr int kDecHalf = kDecTile * 128;             // one 64-dimension half of a tile: 64 rows x 128 B
+constexpr int kDecStageBytes = 4 * kDecHalf;         // keys (two halves), then values (two halves)
+constexpr int kDecConsumers = 512;                   // warps 0-15
+constexpr int kDecQGroups = kDecConsumers / 64;      // query groups of 64 threads
+constexpr int kDecTmaThreads = kDecConsumers + 32;   // + warp 16 (copies)
+constexpr int kDecQPitch = kD + 4;                   // floats per staged query row
+constexpr int kDecTmaSmem = 1024 + kDecStages * kDecStageBytes + kDecMaxG * kDecQPitch * 4 +
+                            9 * kDecMaxG * kDecTile * 4 + 3 * kDecMaxG * 4 + 128;
+
+__device__ __forceinline__ void consumer_sync() { asm volatile("bar.sync 1, 512;" ::: "memory"); }
+
+// Element e (0..127) of row t of a swizzled [2][64][128 B] tile.
+__device__ __forceinline__ uint32_t tile_off(int t, int e) {
+  const int kb = e >> 6, c = (e >> 3) & 7;
+  return (uint32_t)(kb * kDecHalf + t * 128 + ((c ^ (t & 7)) << 4) + (e & 7) * 2);
+}
+
+template <int GM>
+__global__ void __launch_bounds__(kDecTmaThreads, 1)
+    k_decode_tma(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
+                 const __nv_bfloat16* __restrict__ q, int n, int hq, int hkv, int per, float* part_o,
+                 float2* part_ml, uint32_t* err) {
+  extern __shared__ uint8_t dec_raw[];
+  uint8_t* sm = dec_raw + ((1024u - (smem_u32(dec_raw) & 1023u)) & 1023u);
+  const int split = blockIdx.x, h = blockIdx.y, r = blockIdx.z;
+  const int G = hq / hkv;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  float* qs = reinterpret_cast<float*>(sm + kDecStages * kDecStageBytes);  // [GM][kDecQPitch]
+  float* ps = qs + GM * kDecQPitch;                                           // [GM][64]
+  float* part = ps + GM * kDecTile;                                          // [8][GM][64]
+  float* st_m = part + 8 * GM * kDecTile;
+  float* st_l = st_m + GM;
+  float* st_a = st_l + GM;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(st_a + GM + (GM & 1));      // 8-byte aligned
+  const uint32_t b_full = smem_u32(&bars[0]), b_empty = smem_u32(&bars[kDecStages]);
+  volatile uint32_t* flag = reinterpret_cast<volatile uint32_t*>(&bars[2 * kDecStages]);
+  volatile uint32_t* abort_flag = flag + 1;
+  const uint32_t s0 = smem_u32(sm);
+  const int j0 = min(n, split * per), j1 = min(n, j0 + per);
+  const int ntiles = (j1 - j0 + kDecTile - 1) / kDecTile;
+
+  if (tid == 0) {
+    for (int i = 0; i < kDecStages; ++i) {
+      mbar_init(b_full + 8 * i, 1);
+      mbar_init(b_empty + 8 * i, 1);
+    }
+    *abort_flag = 0u;
+    fence_mbar_init();
+  }
+  // query rows of the group, times log2(e)/sqrt(d); running (max, sum)
+  const float scale = kDecLog2e * rsqrtf((float)kD);
+  for (int e = tid; e < G * kD; e += kDecTmaThreads)
+    qs[(e / kD) * kDecQPitch + e % kD] = __bfloat162float(q[((size_t)r * hq + h * G) * kD + e]) * scale;
+  for (int g = tid; g < GM; g += kDecTmaThreads) {
+    st_m[g] = -CUDART_INF_F;
+    st_l[g] = 0.f;
+  }
+  __syncthreads();
+
+  if (warp == kDecConsumers / 32) {
+    if (lane == 0) {
+      int issued[kDecStages] = {0, 0, 0, 0};
+      for (int it = 0; it < ntiles; ++it) {
+        const int s = it % kDecStages;
+        if (!mbar_wait(b_empty + 8 * s, ((uint32_t)(it / kDecStages) & 1u) ^ 1u, err, abort_flag)) break;
+        const uint32_t dst = s0 + s * kDecStageBytes;
+        const int row = j0 + it * kDecTile;
+        mbar_arrive_expect_tx(b_full + 8 * s, (uint32_t)kDecStageBytes);
+        tma_load_3d(dst, &kmap, b_full + 8 * s, 0, h, row);
+        tma_load_3d(dst + kDecHalf, &kmap, b_full + 8 * s, 64, h, row);
+        tma_load_3d(dst + 2 * kDecHalf, &vmap, b_full + 8 * s, 0, h, row);
+        tma_load_3d(dst + 3 * kDecHalf, &vmap, b_full + 8 * s, 64, h, row);
+        ++issued[s];
+      }
+      if (*abort_flag)  // drain copies still in flight before the CTA exits
+        for (int s = 0; s < kDecStages; ++s)
+          if (issued[s]) mbar_wait_drain(b_full + 8 * s, (uint32_t)(issued[s] - 1) & 1u);
+    }
+    return;
+  }
+
+  // ---------------------------------------------------------- consumers
+  float o[GM][2];  // dimensions 2*dp, 2*dp + 1 over this thread's row slice
+#pragma unroll
+  for (int g = 0; g < GM; ++g) o[g][0] = o[g][1] = 0.f;
+  const int dp = tid & 63, ts = tid >> 6;   // phase 3 roles
+  const int t1 = tid & 63, sl = tid >> 6;   // phase 1 roles
+  for (int it = 0; it < ntiles; ++it) {
+    const int s = it % kDecStages;
+    if (tid == 0) *flag = mbar_wait(b_full + 8 * s, (uint32_t)(it / kDecStages) & 1u, err, abort_flag) ? 1u : 0u;
+    consumer_sync();
+    if (*flag == 0u) break;  // the same value for every consumer thread
+    const uint8_t* kt = sm + s * kDecStageBytes;
+    const uint8_t* vt = kt + 2 * kDecHalf;
+    const int base = j0 + it * kDecTile;
+    // phase 1: row t1, dimensions 16 sl .. 16 sl + 15, every query head
+    {
+      float kf[16];
+#pragma unroll
+      for (int m = 0; m < 2; ++m) {
+        const uint4 u = *reinterpret_cast<const uint4*>(kt + tile_off(t1, 16 * sl + 8 * m));
+        const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          kf[8 * m + 2 * i] = __uint_as_float(w4[i] << 16);
+          kf[8 * m + 2 * i + 1] = __uint_as_float(w4[i] & 0xffff0000u);
+        }
+      }
+#pragma unroll
+      for (int g = 0; g < GM; ++g) {
+        if (g < G) {
+          float x0 = 0.f, x1 = 0.f;
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const float4 a = *reinterpret_cast<const float4*>(qs + g * kDecQPitch + 16 * sl + 4 * j);
+            float& x = (j & 1) ? x1 : x0;
+            x = fmaf(kf[4 * j], a.x, fmaf(kf[4 * j + 1], a.y, fmaf(kf[4 * j + 2], a.z, fmaf(kf[4 * j + 3], a.w, x))));
+          }
+          part[(sl * GM + g) * kDecTile + t1] = x0 + x1;
+        }
+      }
+    }
+    consumer_sync();
+    // phase 1b: sum the slices; scores of rows past the range are -inf
+    for (int e = tid; e < G * kDecTile; e += kDecConsumers) {
+      const int g = e / kDecTile, t = e % kDecTile;
+      float x = 0.f;
+#pragma unroll
+      for (int q8 = 0; q8 < 8; ++q8) x += part[(q8 * GM + g) * kDecTile + t];
+      ps[g * kDecTile + (t & 7) * 8 + (t >> 3)] = base + t < j1 ? x : -CUDART_INF_F;
+    }
+    consumer_sync();
+    // phase 2: online softmax of query head g over the tile's 64 rows
+    for (int g = warp; g < G; g += kDecConsumers / 32) {
+      const int i0 = (lane & 7) * 8 + (lane >> 3), i1 = i0 + 4;  // rows lane and lane + 32
+      const float x0 = ps[g * kDecTile + i0], x1 = ps[g * kDecTile + i1];
+      const float mo = st_m[g];
+      const float mn = fmaxf(mo, warp_max(fmaxf(x0, x1)));
+      const float p0 = weight(x0, mn), p1 = weight(x1, mn);
+      const float sum = warp_sum(p0 + p1);
+      ps[g * kDecTile + i0] = p0;
+      ps[g * kDecTile + i1] = p1;
+      if (lane == 0) {
+        const float a = weight(mo, mn);
+        st_a[g] = a;
+        st_l[g] = st_l[g] * a + sum;
+        st_m[g] = mn;
+      }
+    }
+    consumer_sync();
+    // phase 3: rows ts + 8 k, dimensions 2 dp and 2 dp + 1, every query head
+    {
+      float2 vv[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const uint32_t w = *reinterpret_cast<const uint32_t*>(vt + tile_off(ts + 8 * k, 2 * dp));
+        vv[k] = make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
+      }
+#pragma unroll
+      for (int g = 0; g < GM; ++g) {
+        if (g < G) {
+          const float a = st_a[g];
+          const float4 pa = *reinterpret_cast<const float4*>(ps + g * kDecTile + ts * 8);
+          const float4 pb = *reinterpret_cast<const float4*>(ps + g * kDecTile + ts * 8 + 4);
+          const float pp[8] = {pa.x, pa.y, pa.z, pa.w, pb.x, pb.y, pb.z, pb.w};
+          float y0 = o[g][0] * a, y1 = o[g][1] * a;
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            y0 = fmaf(pp[k], vv[k].x, y0);
+            y1 = fmaf(pp[k], vv[k].y, y1);
+          }
+          o[g][0] = y0;
+          o[g][1] = y1;
+        }
+      }
+    }
+    consumer_sync();  // every consumer is done with this stage
+    if (tid == 0) mbar_arrive(b_empty + 8 * s);
+  }
+  // sum the eight row slices (through the first stage buffer, now idle),
+  // then write this split's partial per query head
+  float* red = reinterpret_cast<float*>(sm);  // [8 slices][GM][128]
+#pragma unroll
+  for (int g = 0; g < GM; ++g)
+    if (g < G) *reinterpret_cast<float2*>(red + ((size_t)ts * GM + g) * kD + 2 * dp) = make_float2(o[g][0], o[g][1]);
+  consumer_sync();
+  for (int e = tid; e < G * kD; e += kDecConsumers) {
+    const int g = e / kD, c = e % kD;
+    float x = 0.f;
+#pragma unroll
+    for (int q8 = 0; q8 < 8; ++q8) x += red[((size_t)q8 * GM + g) * kD + c];
+    const size_t slot = ((size_t)split * gridDim.z + r) * hq + h * G + g;
+    part_o[slot * kD + c] = x;
+    if (c == 0) part_ml[slot] = make_float2(st_m[g], st_l[g]);
+  }
+}
+
 // out[r][g][c] = merge over the splits.  grid (hq, w), one thread per
 // dimension: the splits' weights exp2(m_s - M) and the normaliser are formed
 // once in shared memory, then every thread sums its dimension over the splits
@@ -224,8 +444,8 @@ __global__ void __launch_bounds__(kD) k_decode_combine(const float* part_o, cons
 int decode_splits(int n, int hkv, int w) {
   int dev = 0, sms = 152;
   if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  // about two CTAs per SM, each with at least 256 cached rows
-  long long s = (2LL * sms + (long long)hkv * w - 1) / ((long long)hkv * w);
+  // one wave of one CTA per SM, each with at least 256 cached rows
+  long long s = ((long long)sms + (long long)hkv * w - 1) / ((long long)hkv * w);
   const long long cap = (n + 255) / 256;
   if (s > cap) s = cap;
   if (s > kDecMaxSplits) s = kDecMaxSplits;
@@ -233,49 +453,62 @@ int decode_splits(int n, int hkv, int w) {
   return (int)s;
 }
 
+// Workspace: the error word (first 256 bytes), then the split partials.
 size_t decode_workspace_bytes(int n, int hq, int hkv, int w) {
   const size_t slots = (size_t)decode_splits(n, hkv, w) * w * hq;
-  return slots * kD * sizeof(float) + slots * sizeof(float2) + 256;
+  return 256 + slots * kD * sizeof(float) + slots * sizeof(float2);
 }
 
 cudaError_t launch_decode(DType dt, const void* q, const void* k, const void* v, int n, int hq, int hkv, int w,
                           float* out, void* ws, cudaStream_t st) {
   const int nsplit = decode_splits(n, hkv, w);
-  const int per = ((n + nsplit - 1) / nsplit + 31) / 32 * 32;
-  float* part_o = static_cast<float*>(ws);
+  uint32_t* err = static_cast<uint32_t*>(ws);
+  float* part_o = reinterpret_cast<float*>(static_cast<uint8_t*>(ws) + 256);
   float2* part_ml = reinterpret_cast<float2*>(part_o + (size_t)nsplit * w * hq * kD);
   const int G = hq / hkv;
-  const size_t smem = (size_t)G * kD * 4 + (size_t)kDecWarps * G * kD * 4 + (size_t)kDecWarps * G * 8;
   dim3 grid(nsplit, hkv, w);
-  // register arrays sized for the group: G <= 4, <= 8 or <= 16 query heads
-  cudaError_t fe = cudaSuccess;
-  auto run = [&](auto tag, auto gm) {
-    using T = decltype(tag);
-    constexpr int GM = decltype(gm)::value;
-    fe = cudaFuncSetAttribute(k_decode_split<T, GM>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (fe != cudaSuccess) return;
-    k_decode_split<T, GM><<<grid, kDecThreads, smem, st>>>(static_cast<const T*>(q), static_cast<const T*>(k),
-                                                           static_cast<const T*>(v), n, hq, hkv, per, part_o,
-                                                           part_ml);
-  };
-  {
+  cudaError_t e = cudaSuccess;
+  if (dt == kBF16) {
+    const int per = ((n + nsplit - 1) / nsplit + kDecTile - 1) / kDecTile * kDecTile;
+    CUtensorMap km, vm;
+    if ((e = make_row_map(&km, k, n, hkv, kDecTile)) != cudaSuccess) return e;
+    if ((e = make_row_map(&vm, v, n, hkv, kDecTile)) != cudaSuccess) return e;
+    auto run = [&](auto gm) {
+      constexpr int GM = decltype(gm)::value;
+      e = cudaFuncSetAttribute(k_decode_tma<GM>, cudaFuncAttributeMaxDynamicSharedMemorySize, kDecTmaSmem);
+      if (e != cudaSuccess) return;
+      k_decode_tma<GM><<<grid, kDecTmaThreads, kDecTmaSmem, st>>>(
+          km, vm, static_cast<const __nv_bfloat16*>(q), n, hq, hkv, per, part_o, part_ml, err);
+    };
     TimingScope ts("decode_split", st);
-    using G4 = std::integral_constant<int, 4>;
-    using G8 = std::integral_constant<int, 8>;
-    using G16 = std::integral_constant<int, 16>;
-    if (dt == kBF16) {
-      if (G <= 4) run(__nv_bfloat16(), G4());
-      else if (G <= 8) run(__nv_bfloat16(), G8());
-      else run(__nv_bfloat16(), G16());
-    } else {
-      if (G <= 4) run(float(), G4());
-      else if (G <= 8) run(float(), G8());
-      else run(float(), G16());
-    }
+    if (G <= 4)
+      run(std::integral_constant<int, 4>());
+    else if (G <= 8)
+      run(std::integral_constant<int, 8>());
+    else
+      run(std::integral_constant<int, 16>());
+  } else {
+    const int per = ((n + nsplit - 1) / nsplit + 31) / 32 * 32;
+    const size_t smem = (size_t)G * kD * 4 + (size_t)kDecWarps * G * kD * 4 + (size_t)kDecWarps * G * 8;
+    auto run = [&](auto gm) {
+      constexpr int GM = decltype(gm)::value;
+      e = cudaFuncSetAttribute(k_decode_split<float, GM>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (e != cudaSuccess) return;
+      k_decode_split<float, GM><<<grid, kDecThreads, smem, st>>>(static_cast<const float*>(q),
+                                                                 static_cast<const float*>(k),
+                                                                 static_cast<const float*>(v), n, hq, hkv, per,
+                                                                 part_o, part_ml);
+    };
+    TimingScope ts("decode_split", st);
+    if (G <= 4)
+      run(std::integral_constant<int, 4>());
+    else if (G <= 8)
+      run(std::integral_constant<int, 8>());
+    else
+      run(std::integral_constant<int, 16>());
   }
-  if (fe != cudaSuccess) return fe;
-  cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
   TimingScope ts("decode_combine", st);
   k_decode_combine<<<dim3(hq, w), kD, 0, st>>>(part_o, part_ml, nsplit, hq, w, out);
   return cudaGetLastError();

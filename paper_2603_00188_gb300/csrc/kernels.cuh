@@ -168,6 +168,10 @@ int select_max_tokens();
 // v, k_out, v_out from io).
 cudaError_t launch_gather(const Problem& p, int budget, const LayerPtrs& io, cudaStream_t st);
 
+// 3-D TMA map (d, head, row) over a bf16 [n][hkv][128] tensor with boxes of
+// 64 x 1 x rows and the 128-byte swizzle.
+cudaError_t make_row_map(CUtensorMap* m, const void* base, int n, int hkv, int rows);
+
 // ---- consumer: decode attention over a (compressed) cache -----------------
 constexpr int kDecMaxG = 16;  // query heads per KV head
 int decode_splits(int n, int hkv, int w);

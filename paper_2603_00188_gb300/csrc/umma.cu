@@ -1057,6 +1057,10 @@ static cudaError_t make_kmap(CUtensorMap* m, const void* k, int n, int hkv, int 
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
+cudaError_t make_row_map(CUtensorMap* m, const void* base, int n, int hkv, int rows) {
+  return make_kmap(m, base, n, hkv, rows);
+}
+
 static int sm_count() {
   int dev = 0, c = 148;
   cudaGetDevice(&dev);

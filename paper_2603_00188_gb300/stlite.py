@@ -278,7 +278,7 @@ def stlite_decode_attention(q, k, v, out, ws, stream=None):
 def decode_attention(q, k, v, stream=None):
     """Allocates the output and the workspace and runs stlite_decode_attention."""
     sh = make_shape(q, k)
-    ws = torch.empty(stlite_decode_workspace_size(sh), dtype=torch.uint8, device=k.device)
+    ws = torch.zeros(stlite_decode_workspace_size(sh), dtype=torch.uint8, device=k.device)
     out = torch.empty(q.shape, dtype=torch.float32, device=k.device)
     stlite_decode_attention(q, k, v, out, ws, stream)
     return out

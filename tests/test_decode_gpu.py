@@ -31,14 +31,19 @@ def _close(got, ref, v64):
 
 @pytest.mark.parametrize("w,hq,hkv,n,dtype", [(1, 28, 4, 1000, torch.bfloat16), (3, 28, 4, 257, torch.bfloat16),
                                               (2, 16, 1, 33, torch.bfloat16), (1, 4, 4, 1, torch.bfloat16),
+                                              (1, 28, 4, 20000, torch.bfloat16), (2, 6, 2, 130, torch.bfloat16),
                                               (2, 12, 2, 513, torch.float32), (1, 8, 2, 31, torch.float32)])
 def test_decode_matches_oracle(st, w, hq, hkv, n, dtype):
     g = torch.Generator().manual_seed(n * 7 + hq)
     q = torch.randn((w, hq, 128), generator=g).to(dtype).cuda()
     k = torch.randn((n, hkv, 128), generator=g).to(dtype).cuda()
     v = torch.randn((n, hkv, 128), generator=g).to(dtype).cuda()
-    out = st.decode_attention(q, k, v)
+    sh = st.make_shape(q, k)
+    ws = torch.zeros(st.stlite_decode_workspace_size(sh), dtype=torch.uint8, device="cuda")
+    out = torch.empty((w, hq, 128), dtype=torch.float32, device="cuda")
+    st.stlite_decode_attention(q, k, v, out, ws)
     torch.cuda.synchronize()
+    assert st.stlite_device_status(ws) == st.STLITE_OK
     ref = oracle.decode_attention(exact64(q), exact64(k), exact64(v))
     _close(out.cpu().numpy().astype(np.float64), ref, exact64(v))
 
