@@ -26,6 +26,13 @@ CONFIGS = {
     "small_s0_b10": (lambda: synth.small_backbone_seq(0, beta=0.1), True),
     "small_s5_b40": (lambda: synth.small_backbone_seq(5, beta=0.4), True),
     "long_l0": (lambda: synth.long_horizon(0), False),
+    # the frame-table limit: 256 frames (2x3 grids, one text token after each)
+    "max_frames_256": (lambda: synth.trajectory(n_steps=256, gh=2, gw=3, n_text=1, hq=4, hkv=2, w=4, beta=0.3,
+                                                n_boxes=(1, 2), box_hw=((1, 1), (2, 2)), seed=(990,)), True),
+    # the largest cache the selection holds on chip: 393,216 tokens
+    # (256 frames of 32x48, one KV head)
+    "max_tokens_393216": (lambda: synth.trajectory(n_steps=256, gh=32, gw=48, n_text=0, hq=2, hkv=1, w=2,
+                                                   beta=0.1, seed=(991,)), False),
 }
 
 

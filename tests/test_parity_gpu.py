@@ -372,11 +372,11 @@ def test_varlen_ragged_fp32_and_oracle(st):
     # three sequences of different frame layouts (fp32), one of them a single frame;
     # the packed call equals per-sequence calls, and those match the oracle
     wls = [synth.trajectory(n_steps=3, gh=5, gw=7, n_text=4, hq=8, hkv=2, w=4, beta=0.3, seed=(900, 0),
-                            dtype="fp32"),
+                            dtype="f32"),
            synth.trajectory(n_steps=1, gh=6, gw=3, n_text=9, hq=8, hkv=2, w=4, beta=0.3, seed=(900, 1),
-                            dtype="fp32"),
+                            dtype="f32"),
            synth.trajectory(n_steps=4, gh=3, gw=9, n_text=2, hq=8, hkv=2, w=4, beta=0.3, seed=(900, 2),
-                            dtype="fp32")]
+                            dtype="f32")]
     _varlen_vs_single(st, wls)
     for wl in wls:
         _run_edge(st, wl, wl.beta)
