@@ -56,11 +56,11 @@ def _load():
         lib.orc_css_phi.restype = None
         lib.orc_css_phi.argtypes = [_dp, _i32, _i32, _i32, _i32, _i32, _ip, _ip, _ip, _dp]
         lib.orc_tsg_rho_token.restype = ctypes.c_double
-        lib.orc_tsg_rho_token.argtypes = [_dp, _i32, _i32, _i32, _i32, _i32, _i32]
+        lib.orc_tsg_rho_token.argtypes = [_dp, _i32, _i32, _i32, _i32, _i32, _i32, _i32]
         lib.orc_tsg_rho.restype = None
-        lib.orc_tsg_rho.argtypes = [_dp, _i32, _i32, _i32, _i32, _i32, _ip, _ip, _ip, _dp]
+        lib.orc_tsg_rho.argtypes = [_dp, _i32, _i32, _i32, _i32, _i32, _ip, _ip, _ip, _i32, _dp]
         lib.orc_tsg_gate.restype = _i32
-        lib.orc_tsg_gate.argtypes = [_dp, _i32, _i32, _ip, _ip, _ip, _i32, _i32, _dp, _bp]
+        lib.orc_tsg_gate.argtypes = [_dp, _i32, _i32, _ip, _ip, _ip, _i32, _i32, _i32, ctypes.c_double, _dp, _bp]
         lib.orc_combine.restype = None
         lib.orc_combine.argtypes = [_dp, _dp, _bp, _i32, _i32, _ip, _ip, _ip, ctypes.c_double, _i32, _dp]
         lib.orc_topk.restype = None
@@ -139,8 +139,13 @@ def css_phi_token(k, h: int, off: int, gh: int, gw: int, u: int, v: int) -> floa
     return float(_load().orc_css_phi_token(_d(k), hkv, d, h, off, gh, gw, u, v))
 
 
-def tsg_rho(k, frames, threads: int = 1) -> np.ndarray:
-    """Eq. 6: rho_i = max cosine to the current frame; NaN outside the pool."""
+TSG_COSINE, TSG_DOT, TSG_NEG_L2 = 0, 1, 2
+
+
+def tsg_rho(k, frames, threads: int = 1, metric: int = TSG_COSINE) -> np.ndarray:
+    """Eq. 6: rho_i = max similarity to the current frame (cosine; or, for the
+    similarity-metric ablation, dot product / negative squared L2 distance);
+    NaN outside the pool."""
     lib = _load()
     k = _c64(k)
     n, hkv, d = k.shape
@@ -149,22 +154,23 @@ def tsg_rho(k, frames, threads: int = 1) -> np.ndarray:
 
     def run(h):
         lib.orc_tsg_rho(_d(k), n, hkv, d, h, len(off), off.ctypes.data_as(_ip),
-                        gh.ctypes.data_as(_ip), gw.ctypes.data_as(_ip), out[h].ctypes.data_as(_dp))
+                        gh.ctypes.data_as(_ip), gw.ctypes.data_as(_ip), int(metric), out[h].ctypes.data_as(_dp))
 
     _per_head(run, hkv, threads)
     return out
 
 
-def tsg_rho_token(k, h: int, i: int, frames) -> float:
+def tsg_rho_token(k, h: int, i: int, frames, metric: int = TSG_COSINE) -> float:
     """rho of the single token i against the current (last) frame."""
     k = _c64(k)
     n, hkv, d = k.shape
     off, gh, gw = _frames(frames)
-    return float(_load().orc_tsg_rho_token(_d(k), hkv, d, h, i, int(off[-1]), int(gh[-1] * gw[-1])))
+    return float(_load().orc_tsg_rho_token(_d(k), hkv, d, h, i, int(off[-1]), int(gh[-1] * gw[-1]), int(metric)))
 
 
-def tsg_gate(rho, frames, budget_b: int, tsg_enable: int = 1):
-    """Eqs. 7-8: tau = min(B,|pool|)-th smallest rho; M = [rho <= tau].
+def tsg_gate(rho, frames, budget_b: int, tsg_enable: int = 1, fixed_tau=None):
+    """Eqs. 7-8: tau = min(B,|pool|)-th smallest rho; M = [rho <= tau].  With
+    fixed_tau (the fixed-threshold control) tau is that constant instead.
 
     Returns (tau [Hkv], gate [Hkv, N] uint8, pool_size)."""
     lib = _load()
@@ -178,7 +184,9 @@ def tsg_gate(rho, frames, budget_b: int, tsg_enable: int = 1):
         t = ctypes.c_double()
         pool = lib.orc_tsg_gate(rho[h].ctypes.data_as(_dp), n, len(off), off.ctypes.data_as(_ip),
                                 gh.ctypes.data_as(_ip), gw.ctypes.data_as(_ip), int(budget_b),
-                                int(tsg_enable), ctypes.byref(t), gate[h].ctypes.data_as(_bp))
+                                int(tsg_enable), 0 if fixed_tau is None else 1,
+                                0.0 if fixed_tau is None else float(fixed_tau), ctypes.byref(t),
+                                gate[h].ctypes.data_as(_bp))
         tau[h] = t.value
     return tau, gate, int(pool)
 
@@ -229,18 +237,29 @@ def gather(k, v, idx):
     return ko, vo
 
 
+BASE_WINDOW, BASE_UNIFORM = 0, 1
+
+
 def compress_layer(q, k, frames, beta: float = 0.2, k_override: int = 0, alpha: float = 1.0,
-                   tsg_enable: int = 1, css_enable: int = 1, threads: int = 1) -> dict:
-    """Algorithm 1 for one layer: every stage in the paper's order."""
+                   tsg_enable: int = 1, css_enable: int = 1, threads: int = 1, tsg_metric: int = TSG_COSINE,
+                   fixed_tau=None, base_scorer: int = BASE_WINDOW) -> dict:
+    """Algorithm 1 for one layer: every stage in the paper's order.  The
+    keyword variants are the paper's ablations: TSG similarity metric, a fixed
+    gate threshold, and the uniform base prior (A = w/N for every token, the
+    same total as the window score)."""
     n = k.shape[0]
+    w = q.shape[0]
     b = budget(n, beta, k_override)
-    a = abase(q, k, threads)
+    if base_scorer == BASE_UNIFORM:
+        a = np.full((k.shape[1], n), w / n, dtype=np.float64)
+    else:
+        a = abase(q, k, threads)
     phi = css_phi(k, frames, threads)
     if tsg_enable:
-        rho = tsg_rho(k, frames, threads)
+        rho = tsg_rho(k, frames, threads, metric=tsg_metric)
     else:
         rho = np.full_like(a, np.nan)
-    tau, gate, pool = tsg_gate(rho, frames, b, tsg_enable)
+    tau, gate, pool = tsg_gate(rho, frames, b, tsg_enable, fixed_tau=fixed_tau)
     s = combine(a, phi, gate, frames, alpha, css_enable)
     idx = topk(s, b)
     return dict(budget=b, a=a, phi=phi, rho=rho, tau=tau, gate=gate, pool=pool, s=s, idx=idx)

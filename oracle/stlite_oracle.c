@@ -147,12 +147,25 @@ void orc_css_phi(const double* k, int32_t n, int32_t hkv, int32_t d, int32_t h,
 /* ----------------------------------------------- TSG redundancy (Eq. 6) */
 
 /* rho_i = max over current-frame visual keys k_j of cos(k_i, k_j) (Sec. 3.2). */
+/* TSG similarity of two keys.  metric 0: cosine (Eq. 6, the method);
+ * 1: dot product; 2: negative squared L2 distance -|a - b|^2 (the two
+ * alternatives of the similarity-metric ablation). */
+static double tsg_similarity(const double* a, const double* b, int32_t d, int32_t metric) {
+  if (metric == 1) return dot(a, b, d);
+  if (metric == 2) {
+    double s = 0.0;
+    for (int32_t e = 0; e < d; ++e) s += (a[e] - b[e]) * (a[e] - b[e]);
+    return -s;
+  }
+  return cosine(a, b, d);
+}
+
 double orc_tsg_rho_token(const double* k, int32_t hkv, int32_t d, int32_t h, int32_t i,
-                         int32_t cur_off, int32_t cur_len) {
+                         int32_t cur_off, int32_t cur_len, int32_t metric) {
   double best = -INFINITY;
   const double* ki = key_row(k, hkv, d, i, h);
   for (int32_t j = cur_off; j < cur_off + cur_len; ++j) {
-    double c = cosine(ki, key_row(k, hkv, d, j, h), d);
+    double c = tsg_similarity(ki, key_row(k, hkv, d, j, h), d, metric);
     if (c > best) best = c;
   }
   return best;
@@ -162,14 +175,14 @@ double orc_tsg_rho_token(const double* k, int32_t hkv, int32_t d, int32_t h, int
  * 0..F-2, Algorithm 1 ComputeScores); NaN for every other token (R7). */
 void orc_tsg_rho(const double* k, int32_t n, int32_t hkv, int32_t d, int32_t h,
                  int32_t n_frames, const int32_t* off, const int32_t* gh, const int32_t* gw,
-                 double* rho_out) {
+                 int32_t metric, double* rho_out) {
   for (int32_t j = 0; j < n; ++j) rho_out[j] = NAN;
   if (n_frames < 2) return;
   int32_t cf = n_frames - 1;
   int32_t cur_off = off[cf], cur_len = gh[cf] * gw[cf];
   for (int32_t f = 0; f < cf; ++f)
     for (int32_t i = off[f]; i < off[f] + gh[f] * gw[f]; ++i)
-      rho_out[i] = orc_tsg_rho_token(k, hkv, d, h, i, cur_off, cur_len);
+      rho_out[i] = orc_tsg_rho_token(k, hkv, d, h, i, cur_off, cur_len, metric);
 }
 
 /* ---------------------------------------- TSG threshold and gate (7-8) */
@@ -184,14 +197,23 @@ static int cmp_double_asc(const void* a, const void* b) {
  * for historical visual tokens; the current frame is exempt (M = 1, Sec. 3.3);
  * text tokens carry M = 1 (they are never gated).  With an empty pool or TSG
  * disabled every M is 1 and tau is reported as NaN.  Returns |T_pool|. */
+/* tau and the gate (Eqs. 7-8).  fixed_gate != 0 replaces the adaptive tau by
+ * the constant fixed_tau (the fixed-threshold control of the necessity
+ * study: every pool token with similarity above it is gated). */
 int32_t orc_tsg_gate(const double* rho, int32_t n, int32_t n_frames, const int32_t* off,
                      const int32_t* gh, const int32_t* gw, int32_t budget, int32_t tsg_enable,
-                     double* tau_out, uint8_t* gate_out) {
+                     int32_t fixed_gate, double fixed_tau, double* tau_out, uint8_t* gate_out) {
   for (int32_t j = 0; j < n; ++j) gate_out[j] = 1;
   *tau_out = NAN;
   int32_t pool = 0;
   for (int32_t f = 0; f + 1 < n_frames; ++f) pool += gh[f] * gw[f];
   if (!tsg_enable || pool == 0) return pool;
+  if (fixed_gate) {
+    *tau_out = fixed_tau;
+    for (int32_t f = 0; f + 1 < n_frames; ++f)
+      for (int32_t i = off[f]; i < off[f] + gh[f] * gw[f]; ++i) gate_out[i] = rho[i] <= fixed_tau;
+    return pool;
+  }
   double* sorted = (double*)malloc(sizeof(double) * (size_t)pool);
   int32_t t = 0;
   for (int32_t f = 0; f + 1 < n_frames; ++f)
@@ -285,10 +307,10 @@ void orc_compress_head(const double* q, const double* k, int32_t n, int32_t w, i
   orc_abase(q, k, n, w, hq, hkv, d, h, a);
   orc_css_phi(k, n, hkv, d, h, n_frames, off, gh, gw, phi);
   if (tsg_enable)
-    orc_tsg_rho(k, n, hkv, d, h, n_frames, off, gh, gw, rho);
+    orc_tsg_rho(k, n, hkv, d, h, n_frames, off, gh, gw, 0, rho);
   else
     for (int32_t j = 0; j < n; ++j) rho[j] = NAN;
-  orc_tsg_gate(rho, n, n_frames, off, gh, gw, budget, tsg_enable, tau, gate);
+  orc_tsg_gate(rho, n, n_frames, off, gh, gw, budget, tsg_enable, 0, 0.0, tau, gate);
   orc_combine(a, phi, gate, n, n_frames, off, gh, gw, alpha, css_enable, s);
   orc_topk(s, n, budget, idx_out);
 }

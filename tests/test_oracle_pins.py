@@ -535,3 +535,65 @@ def test_critical_hit_rate_cases():
     top = oracle.topk(a, b)
     rest = np.stack([np.setdiff1d(np.arange(wl.n), top[h])[:b] for h in range(a.shape[0])])
     np.testing.assert_array_equal(oracle.critical_hit_rate(rest, wl.q, wl.k), 0.0)
+
+
+# ------------------------------------------------------ ablation variants
+
+def _two_frame_keys(hist, cur, d=16):
+    """Keys of two 1 x n frames (historical then current) in R^d from short
+    explicit vectors (zero-padded); one KV head."""
+    rows = [np.pad(np.asarray(v, float), (0, d - len(v))) for v in list(hist) + list(cur)]
+    k = np.asarray(rows)[:, None, :]
+    frames = frames_of((0, 1, len(hist)), (len(hist), 1, len(cur)))
+    return k, frames
+
+
+def test_rho_dot_and_neg_l2_closed_form():
+    k, fr = _two_frame_keys(hist=[[3, 0], [0, 2], [1, 1]], cur=[[2, 0], [0, 1], [4, 0]])
+    dot = oracle.tsg_rho(k, fr, metric=oracle.TSG_DOT)[0]
+    l2 = oracle.tsg_rho(k, fr, metric=oracle.TSG_NEG_L2)[0]
+    # dot: max(6, 0, 12) = 12; max(0, 2, 0) = 2; max(2, 1, 4) = 4
+    np.testing.assert_array_equal(dot[:3], [12.0, 2.0, 4.0])
+    # -|a-b|^2: (3,0) vs (2,0),(0,1),(4,0): 1, 10, 1 -> -1; (0,2): 8, 1, 20 -> -1; (1,1): 2, 1, 10 -> -1
+    np.testing.assert_array_equal(l2[:3], [-1.0, -1.0, -1.0])
+    assert np.isnan(dot[3:]).all() and np.isnan(l2[3:]).all()
+    # homogeneity: scaling every key by c scales both by c^2 (cosine is invariant)
+    np.testing.assert_allclose(oracle.tsg_rho(2.5 * k, fr, metric=oracle.TSG_DOT)[0][:3], 6.25 * dot[:3])
+    np.testing.assert_allclose(oracle.tsg_rho(2.5 * k, fr, metric=oracle.TSG_NEG_L2)[0][:3], 6.25 * l2[:3])
+
+
+def test_rho_neg_l2_duplicate_is_zero():
+    wl = _tiny_traj(seed=9, n_steps=3)
+    k = wl.k.copy()
+    off, gh, gw = wl.frames
+    P = gh[0] * gw[0]
+    k[off[-1]:off[-1] + P] = k[off[0]:off[0] + P]          # current frame = a copy of frame 0
+    rho = oracle.tsg_rho(k, wl.frames, metric=oracle.TSG_NEG_L2)
+    np.testing.assert_array_equal(rho[:, off[0]:off[0] + P], 0.0)
+    assert (rho[:, off[1]:off[1] + P] < 0).all()
+
+
+def test_fixed_threshold_gate():
+    wl = _tiny_traj(seed=10, n_steps=4)
+    rho = oracle.tsg_rho(wl.k, wl.frames)
+    pool = np.isfinite(rho[0])
+    for t in (0.85, -2.0, 2.0):
+        tau, gate, _ = oracle.tsg_gate(rho, wl.frames, 5, fixed_tau=t)
+        np.testing.assert_array_equal(tau, t)
+        for h in range(rho.shape[0]):
+            np.testing.assert_array_equal(gate[h][pool], (rho[h][pool] <= t).astype(np.uint8))
+            assert (gate[h][~pool] == 1).all()
+    # a threshold below every rho closes the whole pool; one above admits it all
+    _, g_lo, _ = oracle.tsg_gate(rho, wl.frames, 5, fixed_tau=-2.0)
+    _, g_hi, _ = oracle.tsg_gate(rho, wl.frames, 5, fixed_tau=2.0)
+    assert (g_lo[:, pool] == 0).all() and (g_hi[:, pool] == 1).all()
+
+
+def test_uniform_base_prior():
+    wl = _tiny_traj(seed=11, n_steps=3)
+    out = oracle.compress_layer(wl.q, wl.k, wl.frames, beta=0.3, tsg_enable=0, css_enable=0,
+                                base_scorer=oracle.BASE_UNIFORM)
+    # every S equal: Top_B is the first B indices (ties by lower index)
+    b = out["budget"]
+    np.testing.assert_array_equal(out["a"], wl.q.shape[0] / wl.n)
+    np.testing.assert_array_equal(out["idx"], np.tile(np.arange(b), (2, 1)))
