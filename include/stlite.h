@@ -96,12 +96,25 @@ typedef struct {
   const int32_t* grid_w;  /* host [F]: patch-grid columns (>= 1) */
 } stlite_frames;
 
+/* TSG similarity (Eq. 6 uses cosine; the others are the paper's
+ * similarity-metric ablation) and base scorers (Eq. 2's window score; the
+ * uniform prior of the base-scoring ablation). */
+typedef enum { STLITE_TSG_COSINE = 0, STLITE_TSG_DOT = 1, STLITE_TSG_NEG_L2 = 2 } stlite_tsg_metric;
+typedef enum { STLITE_BASE_WINDOW = 0, STLITE_BASE_UNIFORM = 1 } stlite_base_scorer;
+
 typedef struct {
   double beta;        /* compression ratio in (0, 1]: B = floor(beta * N) (Sec. 2.1) */
   int32_t k_override; /* > 0: use this B instead (clamped to N); 0: use beta */
   float alpha;        /* CSS weight of Eq. (9), >= 0 (paper default 1) */
   int32_t tsg_enable; /* 1: apply the TSG gate of Eq. (8); 0: M_time = 1 everywhere */
   int32_t css_enable; /* 1: add alpha * Phi (Eq. 9); 0: as alpha = 0 */
+  /* Ablation variants; all zero = the method as published. */
+  int32_t tsg_metric;  /* stlite_tsg_metric: rho_i = max_j of cos(k_i, k_j), k_i . k_j, or
+                          -|k_i - k_j|^2 over the current frame's keys */
+  int32_t tsg_fixed;   /* 0: adaptive tau of Eq. (7); 1: tau = tsg_fixed_tau for every head
+                          (the fixed-threshold control: pool tokens with rho > tau are gated) */
+  float tsg_fixed_tau; /* used when tsg_fixed = 1; finite */
+  int32_t base_scorer; /* stlite_base_scorer: A_base of Eq. (2), or A = w/N for every token */
 } stlite_params;
 
 /* Flat per-layer budget (Sec. 2.1, Algorithm 1 initialisation):
@@ -137,7 +150,8 @@ STLITE_API stlite_status stlite_spatial_saliency(const stlite_shape* shape, cons
                                       const void* k, float* phi, void* ws, size_t ws_bytes,
                                       void* stream);
 
-/* Step 4, Eq. (9) and Top_B: S = a_base for text tokens, S = gate * (a_base +
+/* Step 4, Eq. (9) and Top_B (base_scorer = STLITE_BASE_UNIFORM replaces a_base,
+ * which may then be NULL, by w/N for every token): S = a_base for text tokens, S = gate * (a_base +
  * alpha * phi) for visual tokens (phi ignored when css_enable = 0; gate may be
  * NULL = all ones); idx[h][:] = the budget tokens of largest S, equal S ranked
  * by lower index, written in ascending index order.  score_out (nullable):

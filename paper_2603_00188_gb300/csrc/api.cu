@@ -76,6 +76,10 @@ stlite_status check_params(const stlite_params* pr) {
   if (pr->k_override < 0) return STLITE_EINVAL;
   if (pr->k_override == 0 && !(pr->beta > 0.0 && pr->beta <= 1.0)) return STLITE_EINVAL;
   if (!(pr->alpha >= 0.f) || !isfinite(pr->alpha)) return STLITE_EINVAL;
+  if (pr->tsg_metric < STLITE_TSG_COSINE || pr->tsg_metric > STLITE_TSG_NEG_L2) return STLITE_EINVAL;
+  if (pr->tsg_fixed != 0 && pr->tsg_fixed != 1) return STLITE_EINVAL;
+  if (pr->tsg_fixed && !isfinite(pr->tsg_fixed_tau)) return STLITE_EINVAL;
+  if (pr->base_scorer != STLITE_BASE_WINDOW && pr->base_scorer != STLITE_BASE_UNIFORM) return STLITE_EINVAL;
   return STLITE_OK;
 }
 
@@ -256,12 +260,22 @@ cudaError_t run_score(const Ctx& c, const LayerPtrs& io, Strided<float> a_base) 
   return launch_score(c.p, io, rp, ns, a_base, c.err, c.st);
 }
 
-cudaError_t run_tsg(const Ctx& c, const LayerPtrs& io) {
+cudaError_t run_tsg(const Ctx& c, const LayerPtrs& io, int metric) {
   Strided<const float> rn = c.view<const float>(c.plan.rn);
   Strided<float> rp = c.view<float>(c.plan.rho_part);
   if (use_tensor_cores(c.p))
-    return launch_tsg_umma(c.p, c.ft, io, c.view<const float>(c.plan.rn_cur), c.plan.cur_pad, rp, c.err, c.st);
-  return launch_tsg(c.p, c.ft, io, rn, rp, c.err, c.st);
+    return launch_tsg_umma(c.p, c.ft, io, c.view<const float>(c.plan.rn_cur), c.plan.cur_pad, rp, metric, c.err,
+                           c.st);
+  return launch_tsg(c.p, c.ft, io, rn, rp, metric, c.err, c.st);
+}
+
+// The ablation fields of the parameters, for the selection kernel.
+void select_variants(SelectArgs& a, const stlite_params* params, const Problem& p) {
+  a.tsg_metric = params->tsg_metric;
+  a.tsg_fixed = params->tsg_fixed;
+  a.tsg_fixed_tau = params->tsg_fixed_tau;
+  a.base_uniform = params->base_scorer == STLITE_BASE_UNIFORM ? 1 : 0;
+  a.a_uniform = (float)p.w / (float)p.n;  // the window score's total, spread evenly
 }
 
 // Algorithm 1 for a batch of layers (steps 1-5), every stage one launch.
@@ -276,8 +290,8 @@ stlite_status compress_batch(const Ctx& c, const stlite_params* params, const La
     e = run_css(c, io, phi);
   else if (tsg)
     e = run_norms(c, io);
-  if (e == cudaSuccess && tsg) e = run_tsg(c, io);
-  if (e == cudaSuccess) e = run_score(c, io, a_base);
+  if (e == cudaSuccess && tsg) e = run_tsg(c, io, params->tsg_metric);
+  if (e == cudaSuccess && params->base_scorer == STLITE_BASE_WINDOW) e = run_score(c, io, a_base);
   if (e != cudaSuccess) return STLITE_ECUDA;
   SelectArgs a = {};
   a.mode = (tsg ? kSelGate : 0) | kSelTopk;
@@ -286,6 +300,7 @@ stlite_status compress_batch(const Ctx& c, const stlite_params* params, const La
   a.tsg_enable = tsg ? 1 : 0;
   a.css_enable = params->css_enable ? 1 : 0;
   a.alpha = params->alpha;
+  select_variants(a, params, c.p);
   a.rho_part = c.view<const float>(c.plan.rho_part);
   a.rn = c.view<const float>(c.plan.rn);
   a.rho = c.view<float>(c.plan.rho);
@@ -347,7 +362,7 @@ stlite_status stlite_gate_frames(const stlite_shape* shape, const stlite_frames*
   if (budget < 1 || budget > c.p.n) return STLITE_EINVAL;
   const LayerPtrs io = single_layer(nullptr, k, nullptr, nullptr, nullptr, nullptr);
   cudaError_t e = run_norms(c, io);
-  if (e == cudaSuccess) e = run_tsg(c, io);
+  if (e == cudaSuccess) e = run_tsg(c, io, kTsgCosine);
   if (e != cudaSuccess) return STLITE_ECUDA;
   SelectArgs a = {};
   a.mode = kSelGate;
@@ -384,7 +399,8 @@ stlite_status stlite_select_topk(const stlite_shape* shape, const stlite_frames*
   stlite_status s = prepare(shape, frames, ws, ws_bytes, 1, stream, &c);
   if (s != STLITE_OK) return s;
   if ((s = check_params(params)) != STLITE_OK) return s;
-  if (!a_base || !idx || !aligned16(a_base) || !aligned16(idx)) return STLITE_EINVAL;
+  const bool uniform = params->base_scorer == STLITE_BASE_UNIFORM;
+  if ((!uniform && !a_base) || (a_base && !aligned16(a_base)) || !idx || !aligned16(idx)) return STLITE_EINVAL;
   if (params->css_enable && (!phi || !aligned16(phi))) return STLITE_EINVAL;
   if ((gate && !aligned16(gate)) || (score_out && !aligned16(score_out))) return STLITE_EINVAL;
   if (budget < 1 || budget > c.p.n) return STLITE_EINVAL;
@@ -393,6 +409,7 @@ stlite_status stlite_select_topk(const stlite_shape* shape, const stlite_frames*
   a.budget = budget;
   a.css_enable = params->css_enable ? 1 : 0;
   a.alpha = params->alpha;
+  select_variants(a, params, c.p);
   a.a_base = one(a_base);
   a.phi = params->css_enable ? one(phi) : strided<const float>(nullptr, 0);
   a.gate = one(const_cast<uint8_t*>(gate));

@@ -114,11 +114,14 @@ int score_nsplit_max(const Problem& p);
 // TSG partial row maxima: rho_part[l][s][h][i] = max over the current-frame
 // columns of 256-column slice s of k_i.k_j * rn_j, for historical visual
 // tokens i (Eq. 6 before the 1/|k_i| factor).
+// metric: kTsgCosine / kTsgDot / kTsgNegL2.  The slices hold max_j of
+// k_i.k_j * rn_j (cosine), k_i.k_j (dot) or 2 k_i.k_j - |k_j|^2 (negative L2);
+// the selection kernel finishes rho with the row's own term.
 cudaError_t launch_tsg(const Problem& p, const FrameTable& ft, const LayerPtrs& io,
-                       Strided<const float> rn, Strided<float> rho_part, uint32_t* err,
+                       Strided<const float> rn, Strided<float> rho_part, int metric, uint32_t* err,
                        cudaStream_t st);
 cudaError_t launch_tsg_umma(const Problem& p, const FrameTable& ft, const LayerPtrs& io,
-                            Strided<const float> rn_cur, int cur_pad, Strided<float> rho_part,
+                            Strided<const float> rn_cur, int cur_pad, Strided<float> rho_part, int metric,
                             uint32_t* err, cudaStream_t st);
 
 // CSS saliency Phi (Eqs. 4-5) of every visual token; also writes the inverse
@@ -142,6 +145,10 @@ cudaError_t launch_fill_text_nan(const Problem& p, const FrameTable& ft, float* 
 // integrated score and top-B (Eq. 9, Sec. 2.1).
 constexpr int kSelGate = 1;
 constexpr int kSelTopk = 2;
+// TSG similarity (Eq. 6: cosine; dot product and negative squared L2 are the
+// similarity-metric ablation).
+constexpr int kTsgCosine = 0, kTsgDot = 1, kTsgNegL2 = 2;
+
 struct SelectArgs {
   int mode;
   int budget;
@@ -149,6 +156,11 @@ struct SelectArgs {
   int tsg_enable;
   int css_enable;
   float alpha;
+  int tsg_metric;      // kTsgCosine / kTsgDot / kTsgNegL2: how rho is finished from the slices
+  int tsg_fixed;       // 1: tau = tsg_fixed_tau instead of the adaptive select (Eq. 7)
+  float tsg_fixed_tau;
+  int base_uniform;    // 1: A = a_uniform for every token instead of a_base
+  float a_uniform;
   Strided<const float> rho_part;  // [nchunk][Hkv][N]
   Strided<const float> rn;        // [Hkv][N]
   Strided<float> rho;             // out [Hkv][N]

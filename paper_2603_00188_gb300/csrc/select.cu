@@ -240,16 +240,24 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
           return r;
         },
         [&](int t, int kind, const RhoIn& v) {
+          // finish Eq. 6 with the row's own term: times 1/|k_i| (cosine),
+          // nothing (dot), minus |k_i|^2 (negative squared L2)
           const float m = fmaxf(fmaxf(v.s[0], v.s[1]), fmaxf(v.s[2], v.s[3]));
-          const float r = kind == kTokPool ? m * v.rn : CUDART_NAN_F;
+          const float own = a.tsg_metric == kTsgCosine ? m * v.rn
+                            : (a.tsg_metric == kTsgDot ? m : m - 1.f / (v.rn * v.rn));
+          const float r = kind == kTokPool ? own : CUDART_NAN_F;
           rho[t] = r;
           keys[t - j0] = kind == kTokPool ? ~float_key(r) : 0u;
         });
     __syncthreads();
     if (gate_sel) {
-      uint32_t need;
-      const uint32_t kt = cluster_select_desc(cl, keys, len, (uint32_t)min(a.budget, pool), sh, pass, &need);
-      tau = key_float(~kt);
+      if (a.tsg_fixed) {
+        tau = a.tsg_fixed_tau;  // fixed-threshold control: no selection
+      } else {
+        uint32_t need;
+        const uint32_t kt = cluster_select_desc(cl, keys, len, (uint32_t)min(a.budget, pool), sh, pass, &need);
+        tau = key_float(~kt);
+      }
     }
     if (c == 0 && tid == 0) a.tau.at(l)[h] = tau;
     if (!(a.mode & kSelTopk)) {
@@ -263,7 +271,7 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
   }
 
   if (a.mode & kSelTopk) {
-    const float* ab = a.a_base.at(l) + hn;
+    const float* ab = a.base_uniform ? nullptr : a.a_base.at(l) + hn;
     const float* ph = a.phi.base ? a.phi.at(l) + hn : nullptr;
     const uint8_t* gt = gate;
     float* sc = a.score.at(l) + hn;
@@ -274,7 +282,7 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
     for_tokens<2>(
         ft, j0, j1,
         [&](int t, int kind) {
-          const float A = __ldg(ab + t);
+          const float A = ab ? __ldg(ab + t) : a.a_uniform;
           const float P = (kind != kTokText && alpha != 0.f) ? __ldg(ph + t) : 0.f;
           const float G = (kind != kTokText && !fused && gt != nullptr) ? (float)gt[t] : 1.f;
           return make_float3(A, P, G);

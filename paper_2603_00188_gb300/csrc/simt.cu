@@ -443,17 +443,18 @@ cudaError_t launch_score(const Problem& p, const LayerPtrs& io, Strided<float2> 
 // streamed through shared memory.  Writes slice 0 of rho_part (the fp32 path
 // has a single slice).  grid = (row tile, layer*Hkv + head).
 constexpr int kTsKeys = 64;
-constexpr int kTsSmem = (kTsgTile * (kD + 1) + kTsKeys * kD + kTsKeys) * 4;
+constexpr int kTsSmem = (kTsgTile * (kD + 1) + kTsKeys * kD + 2 * kTsKeys) * 4;
 
 template <typename T>
 __global__ void __launch_bounds__(kTsgTile) k_tsg_simt(const __grid_constant__ LayerPtrs io,
                                                        const __grid_constant__ FrameTable ft, int hkv,
                                                        Strided<const float> rn_all,
-                                                       Strided<float> rho_all) {
+                                                       Strided<float> rho_all, int metric) {
   extern __shared__ float sm[];
   float* hs = sm;                              // [128][kD+1]
   float* cs = hs + kTsgTile * (kD + 1);        // [kTsKeys][kD]
-  float* cr = cs + kTsKeys * kD;               // [kTsKeys]
+  float* cr = cs + kTsKeys * kD;               // [kTsKeys] scale of each current key
+  float* co = cr + kTsKeys;                    // [kTsKeys] offset: value = dot * scale + offset
   const int t = blockIdx.x, l = blockIdx.y / hkv, h = blockIdx.y % hkv, tid = threadIdx.x;
   const int n = ft.n_tokens;
   const T* k = static_cast<const T*>(io.k[l]);
@@ -477,8 +478,13 @@ __global__ void __launch_bounds__(kTsgTile) k_tsg_simt(const __grid_constant__ L
       int j = ft.cur_off + jt + jj;
       cs[e] = (jt + jj < ft.cur_len) ? Elem<T>::load1(k + ((size_t)j * hkv + h) * kD + c) : 0.f;
     }
-    for (int jj = tid; jj < kTsKeys; jj += blockDim.x)
-      cr[jj] = (jt + jj < ft.cur_len) ? rn[(size_t)h * n + ft.cur_off + jt + jj] : 0.f;
+    for (int jj = tid; jj < kTsKeys; jj += blockDim.x) {
+      // cosine: dot * rn_j; dot: dot; negative L2 (without the row's own
+      // -|k_i|^2): 2 dot - |k_j|^2
+      const float r = (jt + jj < ft.cur_len) ? rn[(size_t)h * n + ft.cur_off + jt + jj] : 0.f;
+      cr[jj] = metric == kTsgCosine ? r : (metric == kTsgDot ? 1.f : 2.f);
+      co[jj] = metric == kTsgNegL2 ? -1.f / (r * r) : 0.f;
+    }
     __syncthreads();
     int nk = min(kTsKeys, ft.cur_len - jt);
     for (int jj = 0; jj < nk; ++jj) {
@@ -489,14 +495,14 @@ __global__ void __launch_bounds__(kTsgTile) k_tsg_simt(const __grid_constant__ L
         d0 = fmaf(hr[c], kr[c], d0);
         d1 = fmaf(hr[c + 1], kr[c + 1], d1);
       }
-      best = fmaxf(best, (d0 + d1) * cr[jj]);
+      best = fmaxf(best, fmaf(d0 + d1, cr[jj], co[jj]));
     }
   }
   if (i0 + tid < fend) rho_part[(size_t)h * n + i0 + tid] = best;
 }
 
 cudaError_t launch_tsg(const Problem& p, const FrameTable& ft, const LayerPtrs& io, Strided<const float> rn,
-                       Strided<float> rho_part, uint32_t* err, cudaStream_t st) {
+                       Strided<float> rho_part, int metric, uint32_t* err, cudaStream_t st) {
   (void)err;
   cudaFuncSetAttribute(k_tsg_simt<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTsSmem);
   cudaFuncSetAttribute(k_tsg_simt<__nv_bfloat16>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTsSmem);
@@ -505,9 +511,9 @@ cudaError_t launch_tsg(const Problem& p, const FrameTable& ft, const LayerPtrs& 
   dim3 g(tiles, p.L * p.hkv);
   TimingScope ts("tsg_simt", st);
   if (p.dtype == kBF16)
-    k_tsg_simt<__nv_bfloat16><<<g, kTsgTile, kTsSmem, st>>>(io, ft, p.hkv, rn, rho_part);
+    k_tsg_simt<__nv_bfloat16><<<g, kTsgTile, kTsSmem, st>>>(io, ft, p.hkv, rn, rho_part, metric);
   else
-    k_tsg_simt<float><<<g, kTsgTile, kTsSmem, st>>>(io, ft, p.hkv, rn, rho_part);
+    k_tsg_simt<float><<<g, kTsgTile, kTsSmem, st>>>(io, ft, p.hkv, rn, rho_part, metric);
   return cudaGetLastError();
 }
 

@@ -88,6 +88,10 @@ constexpr int kTsgBar = kTsgRn + 2048;                     // 12 mbarriers + slo
 constexpr int kTsgUsed = kTsgBar + 128;                    // bytes after 1024-alignment
 constexpr int kTsgSmem = 232448;                           // the per-CTA maximum; the rest is alignment slack
 
+// METRIC kTsgCosine: acc_ij * rn_j; kTsgDot: acc_ij; kTsgNegL2: 2 acc_ij -
+// |k_j|^2 (the row's own -|k_i|^2 is added by the selection kernel).  The
+// per-column term sits in rn_s (rn_j, 1, or -|k_j|^2), NaN past the frame.
+template <int METRIC>
 __global__ void __launch_bounds__(kThreads, 1)
     k_tsg_umma(const __grid_constant__ KMaps maps, const __grid_constant__ FrameTable ft,
                Strided<const float> rc_all, int cur_pad, Strided<float> rho_all, int hkv, uint32_t* err) {
@@ -137,8 +141,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_relinquish();
   }
   // inverse norms of this chunk's current-frame columns (NaN past the frame)
-  for (int c = (int)threadIdx.x - 64; c < 512; c += kThreads - 64)
-    if (c >= 0) rn_s[c] = c < valid ? rn_cur[col0 + c] : CUDART_NAN_F;
+  for (int c = (int)threadIdx.x - 64; c < 512; c += kThreads - 64) {
+    if (c >= 0) {
+      float v = CUDART_NAN_F;
+      if (c < valid) {
+        const float r = rn_cur[col0 + c];
+        v = METRIC == kTsgCosine ? r : (METRIC == kTsgDot ? 1.f : -1.f / (r * r));
+      }
+      rn_s[c] = v;
+    }
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -227,8 +239,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int i = 0; i < 16; ++i) {
               const float4 r = r4[i];
               float p0, p1, p2, p3;
-              mul2(v[4 * i], v[4 * i + 1], r.x, r.y, p0, p1);
-              mul2(v[4 * i + 2], v[4 * i + 3], r.z, r.w, p2, p3);
+              if (METRIC == kTsgNegL2) {
+                fma2(v[4 * i], v[4 * i + 1], 2.f, 2.f, r.x, r.y, p0, p1);
+                fma2(v[4 * i + 2], v[4 * i + 3], 2.f, 2.f, r.z, r.w, p2, p3);
+              } else {
+                mul2(v[4 * i], v[4 * i + 1], r.x, r.y, p0, p1);
+                mul2(v[4 * i + 2], v[4 * i + 3], r.z, r.w, p2, p3);
+              }
               m[(2 * i) & 7] = max3(m[(2 * i) & 7], p0, p1);
               m[(2 * i + 1) & 7] = max3(m[(2 * i + 1) & 7], p2, p3);
             }
@@ -244,10 +261,17 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int i = 0; i < 8; ++i) {
               float4 r = r4[i];
-              mx = fmaxf(mx, v[4 * i] * r.x);
-              mx = fmaxf(mx, v[4 * i + 1] * r.y);
-              mx = fmaxf(mx, v[4 * i + 2] * r.z);
-              mx = fmaxf(mx, v[4 * i + 3] * r.w);
+              if (METRIC == kTsgNegL2) {
+                mx = fmaxf(mx, fmaf(v[4 * i], 2.f, r.x));
+                mx = fmaxf(mx, fmaf(v[4 * i + 1], 2.f, r.y));
+                mx = fmaxf(mx, fmaf(v[4 * i + 2], 2.f, r.z));
+                mx = fmaxf(mx, fmaf(v[4 * i + 3], 2.f, r.w));
+              } else {
+                mx = fmaxf(mx, v[4 * i] * r.x);
+                mx = fmaxf(mx, v[4 * i + 1] * r.y);
+                mx = fmaxf(mx, v[4 * i + 2] * r.z);
+                mx = fmaxf(mx, v[4 * i + 3] * r.w);
+              }
             }
           }
         }
@@ -1123,7 +1147,7 @@ int score_nsplit_max(const Problem& p) {
 int score_nsplit(const Problem& p) { return score_nsplit_max(p); }
 
 cudaError_t launch_tsg_umma(const Problem& p, const FrameTable& ft, const LayerPtrs& io,
-                            Strided<const float> rn_cur, int cur_pad, Strided<float> rho_part,
+                            Strided<const float> rn_cur, int cur_pad, Strided<float> rho_part, int metric,
                             uint32_t* err, cudaStream_t st) {
   if (ft.n_frames < 2) return cudaSuccess;
   const int n_tiles = ft.tile0[ft.n_frames - 1];
@@ -1132,13 +1156,14 @@ cudaError_t launch_tsg_umma(const Problem& p, const FrameTable& ft, const LayerP
   KMaps local;
   cudaError_t e = make_kmaps(&local, io, p.L, p.n, p.hkv, 128);
   if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(k_tsg_umma, cudaFuncAttributeMaxDynamicSharedMemorySize, kTsgSmem);
+  auto kern = metric == kTsgDot ? k_tsg_umma<kTsgDot> : (metric == kTsgNegL2 ? k_tsg_umma<kTsgNegL2> : k_tsg_umma<kTsgCosine>);
+  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kTsgSmem);
   if (e != cudaSuccess) return e;
   const int groups = nchunk * p.L * p.hkv;
   const int gx = pick_split(groups, n_tiles, sm_count());
   dim3 grid(gx, nchunk, p.L * p.hkv);
   TimingScope ts("tsg_umma", st);
-  k_tsg_umma<<<grid, kThreads, kTsgSmem, st>>>(local, ft, rn_cur, cur_pad, rho_part, p.hkv, err);
+  kern<<<grid, kThreads, kTsgSmem, st>>>(local, ft, rn_cur, cur_pad, rho_part, p.hkv, err);
   return cudaGetLastError();
 }
 

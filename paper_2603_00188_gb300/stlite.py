@@ -44,7 +44,12 @@ class Frames(ctypes.Structure):
 
 class Params(ctypes.Structure):
     _fields_ = [("beta", ctypes.c_double), ("k_override", ctypes.c_int32), ("alpha", ctypes.c_float),
-                ("tsg_enable", ctypes.c_int32), ("css_enable", ctypes.c_int32)]
+                ("tsg_enable", ctypes.c_int32), ("css_enable", ctypes.c_int32), ("tsg_metric", ctypes.c_int32),
+                ("tsg_fixed", ctypes.c_int32), ("tsg_fixed_tau", ctypes.c_float), ("base_scorer", ctypes.c_int32)]
+
+
+STLITE_TSG_COSINE, STLITE_TSG_DOT, STLITE_TSG_NEG_L2 = 0, 1, 2
+STLITE_BASE_WINDOW, STLITE_BASE_UNIFORM = 0, 1
 
 
 class LayerIO(ctypes.Structure):
@@ -143,8 +148,13 @@ def _frames(frames) -> FrameSpec:
     return FrameSpec(*frames)
 
 
-def make_params(beta=0.2, k_override=0, alpha=1.0, tsg_enable=1, css_enable=1) -> Params:
-    return Params(float(beta), int(k_override), float(alpha), int(tsg_enable), int(css_enable))
+def make_params(beta=0.2, k_override=0, alpha=1.0, tsg_enable=1, css_enable=1, tsg_metric=STLITE_TSG_COSINE,
+                fixed_tau=None, base_scorer=STLITE_BASE_WINDOW) -> Params:
+    """Parameters of the pass; the last three select the paper's ablation
+    variants (TSG similarity metric, a fixed gate threshold, the uniform base
+    prior) and default to the method as published."""
+    return Params(float(beta), int(k_override), float(alpha), int(tsg_enable), int(css_enable), int(tsg_metric),
+                  0 if fixed_tau is None else 1, 0.0 if fixed_tau is None else float(fixed_tau), int(base_scorer))
 
 
 # ----------------------------------------------------------------- entries
@@ -314,11 +324,11 @@ def stlite_timing_read() -> dict:
 # ------------------------------------------------------- convenience layer
 
 def compress_layer(q, k, v, frames, beta=0.2, k_override=0, alpha=1.0, tsg_enable=1, css_enable=1,
-                   ws=None, stream=None):
+                   ws=None, stream=None, tsg_metric=STLITE_TSG_COSINE, fixed_tau=None, base_scorer=STLITE_BASE_WINDOW):
     """Allocates outputs (and a workspace if none is given) and runs
     stlite_compress_layer.  Returns (k_out, v_out, idx)."""
     fs = _frames(frames)
-    params = make_params(beta, k_override, alpha, tsg_enable, css_enable)
+    params = make_params(beta, k_override, alpha, tsg_enable, css_enable, tsg_metric, fixed_tau, base_scorer)
     sh = make_shape(q, k)
     b = stlite_budget(sh.n_tokens, beta, k_override)
     if b < 1:

@@ -179,14 +179,16 @@ def test_end_to_end(st, name):
 
 # ------------------------------------------------------------------ edge cases
 
-def _run_edge(st, wl, beta, k_override=0, tsg=1, css=1, alpha=1.0):
+def _run_edge(st, wl, beta, k_override=0, tsg=1, css=1, alpha=1.0, **variant):
+    """variant: tsg_metric / fixed_tau / base_scorer, the same names for the
+    library and the oracle."""
     q, k, v = to_device(wl)
     q64, k64 = exact64(q), exact64(k)
     ko, vo, idx = st.compress_layer(q, k, v, wl.frames, beta=beta, k_override=k_override, tsg_enable=tsg,
-                                    css_enable=css, alpha=alpha)
+                                    css_enable=css, alpha=alpha, **variant)
     torch.cuda.synchronize()
     ref = oracle.compress_layer(q64, k64, wl.frames, beta=beta, k_override=k_override, tsg_enable=tsg,
-                                css_enable=css, alpha=alpha, threads=THREADS)
+                                css_enable=css, alpha=alpha, threads=THREADS, **variant)
     ig = idx.cpu().numpy()
     b = ref["budget"]
     assert ig.shape[1] == b
@@ -426,3 +428,28 @@ def test_critical_hit_rate(st):
     ref_keep = oracle.compress_layer(exact64(q), exact64(k), wl.frames, beta=wl.beta, threads=THREADS)["idx"]
     ref = oracle.critical_hit_rate(ref_keep, exact64(probe), exact64(k))
     assert np.all(np.abs(got - ref) <= 4.0 / idx.shape[1]), (got, ref)
+
+
+# ----------------------------------------------------- the paper's ablation variants
+
+@pytest.mark.parametrize("name", ["uitars_3f", "tiny_ref_fp32"])
+@pytest.mark.parametrize("metric", [1, 2])
+def test_variant_tsg_metric(st, name, metric):
+    # TSG similarity: dot product (1) and negative squared L2 distance (2)
+    wl = WORKLOADS[name]()
+    _run_edge(st, wl, wl.beta, tsg_metric=metric)
+
+
+@pytest.mark.parametrize("name", ["traj50_4f", "tiny_ref_fp32"])
+def test_variant_fixed_threshold(st, name):
+    # fixed-threshold control: gate every pool token with cosine above 0.85
+    wl = WORKLOADS[name]()
+    ig, ref = _run_edge(st, wl, wl.beta, fixed_tau=0.85)
+    assert (ref["tau"] == 0.85).all()
+
+
+@pytest.mark.parametrize("name", ["small_3f", "tiny_ref_fp32"])
+def test_variant_uniform_base(st, name):
+    # uniform base prior: A = w/N for every token (the score passes are skipped)
+    wl = WORKLOADS[name]()
+    _run_edge(st, wl, wl.beta, base_scorer=1)
