@@ -224,6 +224,36 @@ STLITE_API stlite_status stlite_compress_layers(const stlite_shape* shape, const
                                                 const stlite_layer_io* layers, int32_t* budget_out,
                                                 void* ws, size_t ws_bytes, void* stream);
 
+/* stlite_compress_layers with a budget of its own for every layer: layer l
+ * keeps budgets[l] tokens per KV head and its result equals
+ * stlite_compress_layer's with k_override = budgets[l].  This is the
+ * flat-versus-hierarchical ablation (appendix "CSS/TSG Interaction
+ * Analysis", the budget-allocation table; Sec. 3.3 states the flat default):
+ * the scoring is unchanged and only B^(l) varies across layers.  params->beta and
+ * params->k_override are ignored.
+ * budgets: HOST int32 [n_layers], each in [1, n_tokens]; k_out / v_out of
+ *   layer l hold budgets[l] rows and idx_out [Hkv][budgets[l]].
+ * Returns STLITE_EINVAL for a NULL array or an out-of-range budget, checked
+ * before anything is enqueued. */
+STLITE_API stlite_status stlite_compress_layers_budgets(const stlite_shape* shape, const stlite_frames* frames,
+                                                        const stlite_params* params, int32_t n_layers,
+                                                        const stlite_layer_io* layers, const int32_t* budgets,
+                                                        void* ws, size_t ws_bytes, void* stream);
+
+/* Hierarchical per-layer budgets from per-layer attention mass (appendix
+ * "Failure Mode Derivations", F2, the noise-dominated allocation
+ * proposition): B^(l) = S^(l) / sum_l' S^(l') * B_total.  The real shares
+ * are made integer as the budgets in [1, n_tokens] that add up to B_total and
+ * are nearest to the shares in squared distance (ties to the lower layer);
+ * without clamping this is rounding by largest remainder.  Host only.
+ * layer_mass: HOST [n_layers], each finite and > 0 (S^(l): e.g. the sum of a
+ *   layer's window scores A_base over its heads and prefix keys).
+ * total_budget: B_total in [n_layers, n_layers * n_tokens].
+ * budgets: HOST int32 [n_layers] out.
+ * Returns STLITE_EINVAL for invalid arguments (nothing written). */
+STLITE_API stlite_status stlite_hierarchical_budgets(int32_t n_layers, const double* layer_mass, int64_t total_budget,
+                                                     int32_t n_tokens, int32_t* budgets);
+
 /* A packed batch of sequences of different lengths and frame layouts (one
  * layer): Algorithm 1 for each sequence on its own, with its own budget
  * B_s = stlite_budget(N_s, beta, k_override).

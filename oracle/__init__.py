@@ -100,6 +100,31 @@ def budget(n: int, beta: float, k_override: int = 0) -> int:
     return int(_load().orc_budget(int(n), float(beta), int(k_override)))
 
 
+def hierarchical_budgets(layer_mass, total_budget: int, n_tokens: int) -> list:
+    """Hierarchical allocation of the F2 proposition (appendix "Failure Mode
+    Derivations"): layer l gets the real share B^(l) = S^(l) / sum S * B_total.
+    Budgets must be whole tokens in [1, N] adding up to B_total; the reading
+    taken is the integer vector nearest to the shares in squared distance
+    (ties to the lower layer), found by single-token moves from the clamped
+    floors, which is exact for a separable convex objective."""
+    mass = [float(x) for x in layer_mass]
+    n_layers = len(mass)
+    tot = 0.0
+    for m in mass:  # left to right, no compensated summation
+        tot += m
+    share = [m / tot * float(total_budget) for m in mass]
+    b = [min(max(int(np.floor(x)), 1), int(n_tokens)) for x in share]
+    while sum(b) < total_budget:
+        room = [l for l in range(n_layers) if b[l] < n_tokens]
+        l = max(room, key=lambda i: share[i] - b[i])
+        b[l] += 1
+    while sum(b) > total_budget:
+        room = [l for l in range(n_layers) if b[l] > 1]
+        l = max(room, key=lambda i: b[i] - share[i])
+        b[l] -= 1
+    return b
+
+
 def abase(q, k, threads: int = 1) -> np.ndarray:
     """Eq. 2 window score per KV head (mean over the G query heads of a group)."""
     lib = _load()

@@ -5,6 +5,7 @@
 #include <string.h>
 
 #include <atomic>
+#include <cmath>
 #include <map>
 #include <mutex>
 #include <string>
@@ -279,7 +280,8 @@ void select_variants(SelectArgs& a, const stlite_params* params, const Problem& 
 }
 
 // Algorithm 1 for a batch of layers (steps 1-5), every stage one launch.
-stlite_status compress_batch(const Ctx& c, const stlite_params* params, const LayerPtrs& io, int32_t budget) {
+// Layer l keeps io.budget[l] tokens per KV head.
+stlite_status compress_batch(const Ctx& c, const stlite_params* params, const LayerPtrs& io) {
   const bool tsg = params->tsg_enable && c.ft.n_frames >= 2;
   Strided<float> a_base = c.view<float>(c.plan.a_base);
   Strided<float> phi = c.view<float>(c.plan.phi);
@@ -295,7 +297,7 @@ stlite_status compress_batch(const Ctx& c, const stlite_params* params, const La
   if (e != cudaSuccess) return STLITE_ECUDA;
   SelectArgs a = {};
   a.mode = (tsg ? kSelGate : 0) | kSelTopk;
-  a.budget = budget;
+  for (int l = 0; l < c.p.L; ++l) a.budget[l] = io.budget[l];
   a.nchunk = c.plan.nchunk;
   a.tsg_enable = tsg ? 1 : 0;
   a.css_enable = params->css_enable ? 1 : 0;
@@ -311,7 +313,7 @@ stlite_status compress_batch(const Ctx& c, const stlite_params* params, const La
   a.score = c.view<float>(c.plan.score);
   for (int l = 0; l < c.p.L; ++l) a.idx[l] = io.idx[l];
   if ((e = launch_select(c.p, c.ft, a, c.st)) != cudaSuccess) return STLITE_ECUDA;
-  return cuda_status(launch_gather(c.p, budget, io, c.st));
+  return cuda_status(launch_gather(c.p, io, c.st));
 }
 
 }  // namespace
@@ -366,7 +368,7 @@ stlite_status stlite_gate_frames(const stlite_shape* shape, const stlite_frames*
   if (e != cudaSuccess) return STLITE_ECUDA;
   SelectArgs a = {};
   a.mode = kSelGate;
-  a.budget = budget;
+  a.budget[0] = budget;
   a.nchunk = c.plan.nchunk;
   a.tsg_enable = 1;
   a.rho_part = c.view<const float>(c.plan.rho_part);
@@ -406,7 +408,7 @@ stlite_status stlite_select_topk(const stlite_shape* shape, const stlite_frames*
   if (budget < 1 || budget > c.p.n) return STLITE_EINVAL;
   SelectArgs a = {};
   a.mode = kSelTopk;
-  a.budget = budget;
+  a.budget[0] = budget;
   a.css_enable = params->css_enable ? 1 : 0;
   a.alpha = params->alpha;
   select_variants(a, params, c.p);
@@ -428,8 +430,9 @@ stlite_status stlite_compact(const stlite_shape* shape, int32_t budget, const in
     return STLITE_EINVAL;
   if (budget < 1 || budget > shape->n_tokens) return STLITE_EINVAL;
   const Problem p = to_problem(shape, 1);
-  const LayerPtrs io = single_layer(nullptr, k, v, k_out, v_out, const_cast<int32_t*>(idx));
-  return cuda_status(launch_gather(p, budget, io, static_cast<cudaStream_t>(stream)));
+  LayerPtrs io = single_layer(nullptr, k, v, k_out, v_out, const_cast<int32_t*>(idx));
+  io.budget[0] = budget;
+  return cuda_status(launch_gather(p, io, static_cast<cudaStream_t>(stream)));
 }
 
 stlite_status stlite_compress_layer(const stlite_shape* shape, const stlite_frames* frames,
@@ -441,25 +444,27 @@ stlite_status stlite_compress_layer(const stlite_shape* shape, const stlite_fram
   return stlite_compress_layers(shape, frames, params, 1, &io, budget_out, ws, ws_bytes, stream);
 }
 
-stlite_status stlite_compress_layers(const stlite_shape* shape, const stlite_frames* frames,
-                                     const stlite_params* params, int32_t n_layers,
-                                     const stlite_layer_io* layers, int32_t* budget_out, void* ws,
-                                     size_t ws_bytes, void* stream) {
-  if (n_layers < 1 || !layers) return STLITE_EINVAL;
+}  // extern "C"
+
+namespace {
+
+// Algorithm 1 over n_layers layers, layer l keeping budgets[l] tokens per
+// KV head; every budget is checked before anything is enqueued.
+stlite_status compress_layers_impl(const stlite_shape* shape, const stlite_frames* frames,
+                                   const stlite_params* params, int32_t n_layers,
+                                   const stlite_layer_io* layers, const int32_t* budgets, void* ws,
+                                   size_t ws_bytes, void* stream) {
   Ctx c;
   stlite_status s = prepare(shape, frames, ws, ws_bytes, n_layers, stream, &c);
   if (s != STLITE_OK) return s;
-  if ((s = check_params(params)) != STLITE_OK) return s;
   for (int l = 0; l < n_layers; ++l) {
     const stlite_layer_io& x = layers[l];
     if (!x.q || !x.k || !x.v || !x.k_out || !x.v_out || !x.idx_out) return STLITE_EINVAL;
     if (!aligned16(x.q) || !aligned16(x.k) || !aligned16(x.v) || !aligned16(x.k_out) ||
         !aligned16(x.v_out) || !aligned16(x.idx_out))
       return STLITE_EINVAL;
+    if (budgets[l] < 1 || budgets[l] > c.p.n) return STLITE_EINVAL;
   }
-  const int32_t budget = stlite_budget(c.p.n, params->beta, params->k_override);
-  if (budget < 1) return STLITE_EINVAL;
-  if (budget_out) *budget_out = budget;
   // one launch per stage for up to kMaxLayers layers at a time
   for (int l0 = 0; l0 < n_layers; l0 += kMaxLayers) {
     const int L = n_layers - l0 < kMaxLayers ? n_layers - l0 : kMaxLayers;
@@ -476,9 +481,80 @@ stlite_status stlite_compress_layers(const stlite_shape* shape, const stlite_fra
       io.k_out[l] = x.k_out;
       io.v_out[l] = x.v_out;
       io.idx[l] = x.idx_out;
+      io.budget[l] = budgets[l0 + l];
     }
-    if ((s = compress_batch(cb, params, io, budget)) != STLITE_OK) return s;
+    if ((s = compress_batch(cb, params, io)) != STLITE_OK) return s;
   }
+  return STLITE_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+stlite_status stlite_compress_layers(const stlite_shape* shape, const stlite_frames* frames,
+                                     const stlite_params* params, int32_t n_layers,
+                                     const stlite_layer_io* layers, int32_t* budget_out, void* ws,
+                                     size_t ws_bytes, void* stream) {
+  if (n_layers < 1 || !layers || !shape) return STLITE_EINVAL;
+  stlite_status s = check_params(params);
+  if (s != STLITE_OK) return s;
+  const int32_t budget = stlite_budget(shape->n_tokens, params->beta, params->k_override);
+  if (budget < 1) return STLITE_EINVAL;
+  std::vector<int32_t> budgets((size_t)n_layers, budget);
+  s = compress_layers_impl(shape, frames, params, n_layers, layers, budgets.data(), ws, ws_bytes, stream);
+  if (s == STLITE_OK && budget_out) *budget_out = budget;
+  return s;
+}
+
+stlite_status stlite_compress_layers_budgets(const stlite_shape* shape, const stlite_frames* frames,
+                                             const stlite_params* params, int32_t n_layers,
+                                             const stlite_layer_io* layers, const int32_t* budgets,
+                                             void* ws, size_t ws_bytes, void* stream) {
+  if (n_layers < 1 || !layers || !budgets || !shape) return STLITE_EINVAL;
+  stlite_status s = check_params(params);
+  if (s != STLITE_OK) return s;
+  return compress_layers_impl(shape, frames, params, n_layers, layers, budgets, ws, ws_bytes, stream);
+}
+
+stlite_status stlite_hierarchical_budgets(int32_t n_layers, const double* layer_mass, int64_t total_budget,
+                                          int32_t n_tokens, int32_t* budgets) {
+  if (n_layers < 1 || !layer_mass || !budgets || n_tokens < 1) return STLITE_EINVAL;
+  if (total_budget < n_layers || total_budget > (int64_t)n_layers * n_tokens) return STLITE_EINVAL;
+  double sum = 0.0;
+  for (int l = 0; l < n_layers; ++l) {
+    if (!(layer_mass[l] > 0.0) || !std::isfinite(layer_mass[l])) return STLITE_EINVAL;
+    sum += layer_mass[l];
+  }
+  if (!std::isfinite(sum)) return STLITE_EINVAL;
+  // B(l) = S(l) / sum S * B_total made integer: the budgets in [1, N] adding
+  // up to B_total nearest to the real shares in squared distance.  The
+  // problem is separable and convex, so one-token greedy steps from
+  // clamp(floor(share)) reach the minimiser: add where share - b is largest
+  // (room left), or take where b - share is largest (b > 1); ties go to the
+  // lower layer.
+  std::vector<double> share((size_t)n_layers);
+  std::vector<int64_t> b((size_t)n_layers);
+  int64_t given = 0;
+  for (int l = 0; l < n_layers; ++l) {
+    share[l] = layer_mass[l] / sum * (double)total_budget;
+    const double f = floor(share[l]);
+    b[l] = f < 1.0 ? 1 : f > (double)n_tokens ? n_tokens : (int64_t)f;
+    given += b[l];
+  }
+  for (; given < total_budget; ++given) {
+    int best = -1;
+    for (int l = 0; l < n_layers; ++l)
+      if (b[l] < n_tokens && (best < 0 || share[l] - (double)b[l] > share[best] - (double)b[best])) best = l;
+    ++b[best];
+  }
+  for (; given > total_budget; --given) {
+    int best = -1;
+    for (int l = 0; l < n_layers; ++l)
+      if (b[l] > 1 && (best < 0 || (double)b[l] - share[l] > (double)b[best] - share[best])) best = l;
+    --b[best];
+  }
+  for (int l = 0; l < n_layers; ++l) budgets[l] = (int32_t)b[l];
   return STLITE_OK;
 }
 
@@ -543,11 +619,12 @@ stlite_status stlite_compress_varlen(const stlite_shape* shape, int32_t n_seqs, 
     if ((s = prepare(&ss, &frames[i], ws, ws_bytes, 1, stream, &c)) != STLITE_OK) return s;
     const int32_t b = stlite_budget(ss.n_tokens, params->beta, params->k_override);
     const size_t t0 = (size_t)cu_seqlens[i];
-    const LayerPtrs io =
+    LayerPtrs io =
         single_layer(static_cast<const uint8_t*>(q) + i * qseq, static_cast<const uint8_t*>(k) + t0 * row,
                      static_cast<const uint8_t*>(v) + t0 * row, static_cast<uint8_t*>(k_out) + cum * row,
                      static_cast<uint8_t*>(v_out) + cum * row, idx_out + (size_t)shape->n_kv_heads * cum);
-    if ((s = compress_batch(c, params, io, b)) != STLITE_OK) return s;
+    io.budget[0] = b;
+    if ((s = compress_batch(c, params, io)) != STLITE_OK) return s;
     cum += (size_t)b;
     if (cu_budget_out) cu_budget_out[i + 1] = (int32_t)cum;
   }

@@ -36,6 +36,7 @@ struct LayerPtrs {
   void* k_out[kMaxLayers];
   void* v_out[kMaxLayers];
   int32_t* idx[kMaxLayers];
+  int32_t budget[kMaxLayers];  // kept tokens per head of each layer
 };
 
 // A per-layer buffer: layer l starts `stride` bytes after layer l-1.
@@ -151,7 +152,7 @@ constexpr int kTsgCosine = 0, kTsgDot = 1, kTsgNegL2 = 2;
 
 struct SelectArgs {
   int mode;
-  int budget;
+  int budget[kMaxLayers];  // per layer
   int nchunk;
   int tsg_enable;
   int css_enable;
@@ -177,8 +178,8 @@ cudaError_t launch_select(const Problem& p, const FrameTable& ft, const SelectAr
 int select_max_tokens();
 
 // k_out[l][r][h][:] = k_l[idx[l][h][r]][h][:] and the same for v (idx, k,
-// v, k_out, v_out from io).
-cudaError_t launch_gather(const Problem& p, int budget, const LayerPtrs& io, cudaStream_t st);
+// v, k_out, v_out and the budget from io).
+cudaError_t launch_gather(const Problem& p, const LayerPtrs& io, cudaStream_t st);
 
 // 3-D TMA map (d, head, row) over a bf16 [n][hkv][128] tensor with boxes of
 // 64 x 1 x rows and the 128-byte swizzle.

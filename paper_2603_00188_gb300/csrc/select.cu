@@ -255,7 +255,7 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
         tau = a.tsg_fixed_tau;  // fixed-threshold control: no selection
       } else {
         uint32_t need;
-        const uint32_t kt = cluster_select_desc(cl, keys, len, (uint32_t)min(a.budget, pool), sh, pass, &need);
+        const uint32_t kt = cluster_select_desc(cl, keys, len, (uint32_t)min(a.budget[l], pool), sh, pass, &need);
         tau = key_float(~kt);
       }
     }
@@ -306,7 +306,7 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
         });
     __syncthreads();
     uint32_t need;
-    const uint32_t T = cluster_select_desc(cl, keys, len, (uint32_t)a.budget, sh, pass, &need);
+    const uint32_t T = cluster_select_desc(cl, keys, len, (uint32_t)a.budget[l], sh, pass, &need);
     // Ordered compaction.  Thread tid owns the contiguous run [r0, r1) of
     // this CTA's keys (odd run length: conflict-free shared reads); one
     // block scan gives its (greater, equal) counts before the run, the
@@ -338,7 +338,7 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
     }
     __syncthreads();
     uint32_t gt_before = sh.bcast[2] + (ex & 0xffffu), eq_before = sh.bcast[3] + (ex >> 16);
-    int32_t* out = a.idx[l] + (size_t)h * a.budget;
+    int32_t* out = a.idx[l] + (size_t)h * a.budget[l];
     // kept: every key > T, and the first `need` keys == T in index order;
     // a kept token's slot = kept tokens before it
     for (int i = r0; i < r1; ++i) {
@@ -417,9 +417,9 @@ cudaError_t launch_select(const Problem& p, const FrameTable& ft, const SelectAr
 // one output row (coalesced stores, whole 16-byte source vectors).
 // grid.y = layer.
 template <int CPR>
-__global__ void __launch_bounds__(256) k_gather(const __grid_constant__ LayerPtrs io, int n, int hkv,
-                                                int budget) {
+__global__ void __launch_bounds__(256) k_gather(const __grid_constant__ LayerPtrs io, int n, int hkv) {
   const int l = blockIdx.y;
+  const int budget = io.budget[l];
   const int32_t* idx = io.idx[l];
   const uint4* k = static_cast<const uint4*>(io.k[l]);
   const uint4* v = static_cast<const uint4*>(io.v[l]);
@@ -459,9 +459,11 @@ __global__ void __launch_bounds__(256) k_gather(const __grid_constant__ LayerPtr
   }
 }
 
-cudaError_t launch_gather(const Problem& p, int budget, const LayerPtrs& io, cudaStream_t st) {
+cudaError_t launch_gather(const Problem& p, const LayerPtrs& io, cudaStream_t st) {
   const int cpr = p.dtype == kBF16 ? kD * 2 / 16 : kD * 4 / 16;
-  long long total = (long long)budget * p.hkv * cpr;
+  int bmax = 1;
+  for (int l = 0; l < p.L; ++l) bmax = io.budget[l] > bmax ? io.budget[l] : bmax;
+  long long total = (long long)bmax * p.hkv * cpr;
   long long blocks = (total + 1023) / 1024;
   long long cap = (152 * 8 + p.L - 1) / p.L;
   if (blocks > cap) blocks = cap;
@@ -469,9 +471,9 @@ cudaError_t launch_gather(const Problem& p, int budget, const LayerPtrs& io, cud
   TimingScope ts("gather", st);
   dim3 grid((unsigned)blocks, p.L);
   if (cpr == 16)
-    k_gather<16><<<grid, 256, 0, st>>>(io, p.n, p.hkv, budget);
+    k_gather<16><<<grid, 256, 0, st>>>(io, p.n, p.hkv);
   else
-    k_gather<32><<<grid, 256, 0, st>>>(io, p.n, p.hkv, budget);
+    k_gather<32><<<grid, 256, 0, st>>>(io, p.n, p.hkv);
   return cudaGetLastError();
 }
 

@@ -28,7 +28,8 @@ EXPORTED = ("stlite_budget", "stlite_workspace_size", "stlite_score", "stlite_ga
             "stlite_spatial_saliency", "stlite_select_topk", "stlite_compact",
             "stlite_compress_layer", "stlite_device_status", "stlite_timing_enable", "stlite_timing_read",
             "stlite_status_string", "stlite_score_noalloc", "stlite_compress_layers", "stlite_compress_varlen",
-            "stlite_workspace_size_varlen", "stlite_decode_attention", "stlite_decode_workspace_size")
+            "stlite_workspace_size_varlen", "stlite_decode_attention", "stlite_decode_workspace_size",
+            "stlite_compress_layers_budgets", "stlite_hierarchical_budgets")
 
 
 class Shape(ctypes.Structure):
@@ -93,6 +94,11 @@ _sig = {
                                           ctypes.POINTER(ctypes.c_size_t)]),
     "stlite_decode_attention": (_S, [ctypes.POINTER(Shape), _P, _P, _P, _P, _P, ctypes.c_size_t, _P]),
     "stlite_decode_workspace_size": (_S, [ctypes.POINTER(Shape), ctypes.POINTER(ctypes.c_size_t)]),
+    "stlite_compress_layers_budgets": (_S, [ctypes.POINTER(Shape), ctypes.POINTER(Frames), ctypes.POINTER(Params),
+                                            ctypes.c_int32, ctypes.POINTER(LayerIO), ctypes.POINTER(ctypes.c_int32),
+                                            _P, ctypes.c_size_t, _P]),
+    "stlite_hierarchical_budgets": (_S, [ctypes.c_int32, ctypes.POINTER(ctypes.c_double), ctypes.c_int64,
+                                         ctypes.c_int32, ctypes.POINTER(ctypes.c_int32)]),
 }
 for _name, (_res, _args) in _sig.items():
     _f = getattr(_lib, _name)
@@ -235,6 +241,31 @@ def stlite_compress_layers(layers, frames, params, ws, stream=None) -> int:
                                        arr, ctypes.byref(b), _ptr(ws), ws.numel(), _stream(stream)),
            "stlite_compress_layers")
     return int(b.value)
+
+
+def stlite_compress_layers_budgets(layers, frames, params, budgets, ws, stream=None):
+    """As stlite_compress_layers with layer l keeping budgets[l] tokens per
+    KV head (k_out / v_out of layer l: [budgets[l]][Hkv][d], idx_out:
+    [Hkv][budgets[l]])."""
+    q0, k0 = layers[0][0], layers[0][1]
+    sh = make_shape(q0, k0)
+    fs = _frames(frames)
+    arr = (LayerIO * len(layers))(*[LayerIO(*(t.data_ptr() for t in lay)) for lay in layers])
+    bud = (ctypes.c_int32 * len(layers))(*[int(b) for b in budgets])
+    _check(_lib.stlite_compress_layers_budgets(ctypes.byref(sh), ctypes.byref(fs.c), ctypes.byref(params),
+                                               len(layers), arr, bud, _ptr(ws), ws.numel(), _stream(stream)),
+           "stlite_compress_layers_budgets")
+
+
+def stlite_hierarchical_budgets(layer_mass, total_budget: int, n_tokens: int) -> list:
+    """B^(l) = S^(l) / sum S * B_total as integers adding up to B_total
+    (floor plus largest remainder, clamped to [1, n_tokens])."""
+    n = len(layer_mass)
+    mass = (ctypes.c_double * n)(*[float(x) for x in layer_mass])
+    out = (ctypes.c_int32 * n)()
+    _check(_lib.stlite_hierarchical_budgets(n, mass, int(total_budget), int(n_tokens), out),
+           "stlite_hierarchical_budgets")
+    return list(out)
 
 
 def _varlen_args(cu_seqlens, frames_list):

@@ -122,3 +122,63 @@ def test_varlen_validation(st):
     bad = [st.FrameSpec([0], [10], [11]), fr[1], fr[2]]
     with pytest.raises(st.StliteError):
         st.stlite_workspace_size_varlen(sh, [0, 100, 200, 300], bad, prm)
+
+
+def _mass_cases():
+    rng = np.random.default_rng(31)
+    cases = [([1.0, 2.0, 3.0, 4.0], 100, 1000), ([1.0] * 28, 28 * 4718, 23592), ([5.0, 1.0, 1.0], 10, 4),
+             ([1e-9, 1.0, 1.0, 1e-9], 9, 5), ([1.0] * 3, 7, 3), ([100.0, 1.0], 2, 1)]
+    for _ in range(200):
+        n_layers = int(rng.integers(1, 33))
+        n_tokens = int(rng.integers(1, 2000))
+        kind = rng.integers(0, 3)
+        if kind == 0:  # near-uniform: the paper's GUI regime (CV about 1%)
+            mass = 1.0 + 0.013 * rng.standard_normal(n_layers)
+        elif kind == 1:  # pyramid-shaped, shallow layers heavier
+            mass = np.linspace(3.0, 0.5, n_layers) * rng.uniform(0.9, 1.1, n_layers)
+        else:  # heavy-tailed: forces clamping at 1 and at N
+            mass = rng.lognormal(0.0, 3.0, n_layers)
+        total = int(rng.integers(n_layers, n_layers * n_tokens + 1))
+        cases.append((list(mass), total, n_tokens))
+    return cases
+
+
+def test_hierarchical_budgets_match_oracle(st):
+    """The host helper reaches the oracle's integer budgets exactly."""
+    for mass, total, n_tokens in _mass_cases():
+        got = st.stlite_hierarchical_budgets(mass, total, n_tokens)
+        assert got == oracle.hierarchical_budgets(mass, total, n_tokens), (mass, total, n_tokens)
+        assert sum(got) == total and min(got) >= 1 and max(got) <= n_tokens
+
+
+def test_hierarchical_budgets_reject(st):
+    for mass, total, n_tokens in [([], 4, 10), ([1.0, 0.0], 4, 10), ([1.0, -1.0], 4, 10),
+                                  ([1.0, float("nan")], 4, 10), ([1.0, float("inf")], 4, 10),
+                                  ([1.0, 1.0], 1, 10), ([1.0, 1.0], 21, 10), ([1.0], 1, 0),
+                                  ([1e308, 1e308], 4, 10)]:
+        with pytest.raises(st.StliteError):
+            st.stlite_hierarchical_budgets(mass, total, n_tokens)
+
+
+def test_compress_layers_budgets_reject_before_launch(st):
+    """Per-layer budgets outside [1, N] and NULL arrays are refused on the host."""
+    lib = st._lib
+    sh = _shape(st)
+    fr = st.FrameSpec([0, 30], [4, 5], [5, 6])
+    prm = st.make_params(0.2)
+    need = st.stlite_workspace_size(sh, fr, prm)
+    good = 0x10000
+    lay = (st.LayerIO * 2)(st.LayerIO(*([good] * 6)), st.LayerIO(*([good] * 6)))
+    P = ctypes.c_void_p
+    for bud in ([20, 0], [20, 101], [-1, 20]):
+        arr = (ctypes.c_int32 * 2)(*bud)
+        assert lib.stlite_compress_layers_budgets(ctypes.byref(sh), ctypes.byref(fr.c), ctypes.byref(prm), 2, lay,
+                                                  arr, P(good), 2 * need, None) == st.STLITE_EINVAL
+    arr = (ctypes.c_int32 * 2)(20, 30)
+    assert lib.stlite_compress_layers_budgets(ctypes.byref(sh), ctypes.byref(fr.c), ctypes.byref(prm), 2, lay,
+                                              None, P(good), 2 * need, None) == st.STLITE_EINVAL
+    assert lib.stlite_compress_layers_budgets(ctypes.byref(sh), ctypes.byref(fr.c), ctypes.byref(prm), 2, lay,
+                                              arr, P(good), 2 * need - 1, None) == st.STLITE_EWORKSPACE
+    bad = (st.LayerIO * 2)(st.LayerIO(*([good] * 6)), st.LayerIO(*([good] * 5 + [good + 8])))
+    assert lib.stlite_compress_layers_budgets(ctypes.byref(sh), ctypes.byref(fr.c), ctypes.byref(prm), 2, bad,
+                                              arr, P(good), 2 * need, None) == st.STLITE_EINVAL

@@ -597,3 +597,79 @@ def test_uniform_base_prior():
     b = out["budget"]
     np.testing.assert_array_equal(out["a"], wl.q.shape[0] / wl.n)
     np.testing.assert_array_equal(out["idx"], np.tile(np.arange(b), (2, 1)))
+
+
+# ------------------------------------------- hierarchical per-layer budgets
+
+def test_hierarchical_uniform_mass_is_flat():
+    # equal S^(l): every layer gets B_total / L (the flat allocation of
+    # Sec. 3.3); a remainder goes one token each to the lowest layers
+    assert oracle.hierarchical_budgets([2.5] * 28, 28 * 4718, 23592) == [4718] * 28
+    assert oracle.hierarchical_budgets([1.0] * 4, 10, 100) == [3, 3, 2, 2]
+
+
+def test_hierarchical_exact_proportions():
+    # shares that are whole numbers come back unchanged
+    assert oracle.hierarchical_budgets([1.0, 2.0, 3.0, 4.0], 100, 1000) == [10, 20, 30, 40]
+    assert oracle.hierarchical_budgets([3.0, 1.0], 8, 100) == [6, 2]
+    # scale invariance of B = S / sum S * B_total
+    assert oracle.hierarchical_budgets([0.3, 0.6, 0.9, 1.2], 100, 1000) == [10, 20, 30, 40]
+
+
+def _cost(b, share):
+    return sum((x - s) ** 2 for x, s in zip(b, share))
+
+
+@pytest.mark.parametrize("seed", range(40))
+def test_hierarchical_brute_force_nearest(seed):
+    # tiny problems: the oracle's budgets reach the least squared distance to
+    # the real shares over every integer vector in [1, N]^L adding to B_total
+    rng = np.random.default_rng(1000 + seed)
+    n_layers = int(rng.integers(1, 5))
+    n_tokens = int(rng.integers(1, 7))
+    mass = list(rng.lognormal(0.0, 1.5 if seed % 2 else 0.2, n_layers))
+    total = int(rng.integers(n_layers, n_layers * n_tokens + 1))
+    b = oracle.hierarchical_budgets(mass, total, n_tokens)
+    share = [m / math.fsum(mass) * total for m in mass]
+    assert sum(b) == total and all(1 <= x <= n_tokens for x in b)
+    best = min(_cost(c, share) for c in itertools.product(range(1, n_tokens + 1), repeat=n_layers)
+               if sum(c) == total)
+    assert _cost(b, share) <= best + 1e-9
+
+
+def test_hierarchical_largest_remainder_when_unclamped():
+    # away from the [1, N] bounds every budget is the floor or the ceiling of
+    # its share, and the ceilings go to the largest fractional parts
+    rng = np.random.default_rng(77)
+    for _ in range(50):
+        n_layers = int(rng.integers(2, 29))
+        mass = list(1.0 + 0.05 * rng.standard_normal(n_layers))
+        total = int(rng.integers(100 * n_layers, 1000 * n_layers))
+        b = oracle.hierarchical_budgets(mass, total, 10 ** 6)
+        share = [m / math.fsum(mass) * total for m in mass]
+        frac = [s - math.floor(s) for s in share]
+        up = [l for l in range(n_layers) if b[l] == math.floor(share[l]) + 1]
+        down = [l for l in range(n_layers) if b[l] == math.floor(share[l])]
+        assert len(up) + len(down) == n_layers
+        if up and down:
+            assert min(frac[l] for l in up) >= max(frac[l] for l in down) - 1e-12
+
+
+def test_hierarchical_deviation_bound():
+    # F2 proposition: the budget deviation ratio D = (max B - min B) / mean B
+    # equals (max S - min S) / mean S for real budgets and is at most
+    # sqrt(2L) CV_S; with L = 28 and CV_S = 1.3 % the bound is 9.7 %.
+    # Whole-token budgets move each share by less than one token.
+    assert abs(math.sqrt(56) * 0.013 - 0.097) < 5e-4
+    rng = np.random.default_rng(12)
+    n_layers, n_tokens = 28, 393216
+    total = int(0.2 * n_tokens) * n_layers
+    for cv in (0.013, 0.05, 0.3):
+        mass = 1.0 + cv * rng.standard_normal(n_layers)
+        mu = mass.mean()
+        cv_s = mass.std() / mu
+        b = np.array(oracle.hierarchical_budgets(list(mass), total, n_tokens), dtype=np.float64)
+        d_real = (mass.max() - mass.min()) / mu
+        d_int = (b.max() - b.min()) / (total / n_layers)
+        assert d_real <= math.sqrt(2 * n_layers) * cv_s + 1e-12
+        assert abs(d_int - d_real) <= 2.0 / (total / n_layers) + 1e-9

@@ -302,6 +302,61 @@ def test_compress_layers_more_than_one_launch(st):
     _batched_vs_single(st, wls)
 
 
+# ------------------------------------------- per-layer (hierarchical) budgets
+
+def _budgets_vs_single(st, wls, budgets, oracle_layers=()):
+    """stlite_compress_layers_budgets: layer l equals a single-layer call with
+    k_override = budgets[l] (bit-exact), and the layers in oracle_layers
+    match the oracle's kept sets."""
+    dev = [to_device(wl) for wl in wls]
+    wl0 = wls[0]
+    sh = st.make_shape(dev[0][0], dev[0][1])
+    prm = st.make_params(wl0.beta)
+    H = sh.n_kv_heads
+    outs = []
+    for (q, k, v), b in zip(dev, budgets):
+        ko = torch.empty((b, H, 128), dtype=k.dtype, device="cuda")
+        outs.append((q, k, v, ko, torch.empty_like(ko), torch.empty((H, b), dtype=torch.int32, device="cuda")))
+    ws = torch.zeros(len(wls) * st.stlite_workspace_size(sh, wl0.frames, prm), dtype=torch.uint8, device="cuda")
+    st.stlite_compress_layers_budgets(outs, wl0.frames, prm, budgets, ws)
+    torch.cuda.synchronize()
+    assert st.stlite_device_status(ws) == st.STLITE_OK
+    for l, ((q, k, v), b, (_, _, _, ko2, vo2, i2)) in enumerate(zip(dev, budgets, outs)):
+        ko1, vo1, i1 = st.compress_layer(q, k, v, wl0.frames, beta=wl0.beta, k_override=b)
+        torch.cuda.synchronize()
+        assert torch.equal(i1, i2), l
+        assert torch.equal(ko1, ko2) and torch.equal(vo1, vo2), l
+    for l in oracle_layers:
+        ig, ref = _run_edge(st, wls[l], wl0.beta, k_override=budgets[l])
+        np.testing.assert_array_equal(ig, outs[l][5].cpu().numpy())
+
+
+def test_hierarchical_budgets_from_window_mass(st):
+    # S^(l) = the window score's mass on the prefix keys (all heads), the
+    # budgets B^(l) = S^(l) / sum S * B_total with B_total = L * floor(beta N)
+    wls = [synth.scaled("traj50", 3, seed=s) for s in range(4)]
+    n, w = wls[0].n, wls[0].q.shape[0]
+    mass = []
+    for wl in wls:
+        q, k, _ = to_device(wl)
+        mass.append(float(oracle.abase(exact64(q), exact64(k), threads=THREADS)[:, :n - w].sum()))
+    total = len(wls) * oracle.budget(n, wls[0].beta)
+    budgets = st.stlite_hierarchical_budgets(mass, total, n)
+    assert budgets == oracle.hierarchical_budgets(mass, total, n)
+    assert sum(budgets) == total
+    _budgets_vs_single(st, wls, budgets, oracle_layers=(0, len(wls) - 1))
+
+
+def test_per_layer_budgets_extremes_two_launches(st):
+    # 34 layers (two launches), budgets from 1 to N in a pyramid
+    wls = [synth.trajectory(n_steps=3, gh=5, gw=7, n_text=4, hq=8, hkv=2, w=4, beta=0.3, seed=(810, s))
+           for s in range(34)]
+    n = wls[0].n
+    budgets = [max(1, min(n, int(round(n * (1.0 - l / 33.0))))) for l in range(34)]
+    budgets[5], budgets[20] = 1, n
+    _budgets_vs_single(st, wls, budgets, oracle_layers=(0, 5, 20, 33))
+
+
 # ------------------------------------------------- values in page-locked host memory
 
 def test_host_resident_values(st):
