@@ -54,6 +54,7 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-decode", action="store_true", help="skip the decode-over-the-cache measurement")
+    ap.add_argument("--no-variants", action="store_true", help="skip the ablation-variant step times")
     return ap.parse_args()
 
 
@@ -182,6 +183,8 @@ def kernel_roofline(name: str, t_launch: float, layers: int, budget: int, peaks)
         return d
     if name.startswith("css_phi"):
         work = tok_head * (5 * 4 + 4)              # five dot products in, Phi out
+    elif name.startswith("css_box"):
+        work = kbytes + tok_head * 8               # every key once; Phi and 1/|k| out
     elif name.startswith("select"):
         work = tok_head * 3 * 4 + budget * HKV * 4  # A, Phi, rho in; indices out
     elif name.startswith("gather"):
@@ -442,6 +445,81 @@ def run_gpu(args):
     roof["traffic"] = traffic_for(dom) if L == LAYERS else None
     roof["peak_source"] = peaks["source"] + (" burst" if roof["unit"] == "TFLOP/s" else "")
 
+    # ---- the paper's ablation variants on the same workload: step time of
+    # the whole pass (one graph per variant) and the kernels each one changes
+    variants = None
+    if not args.no_variants:
+        variants = {}
+        rng = np.random.default_rng(2603)
+        mass = 1.0 + 0.013 * rng.standard_normal(L)   # near-uniform layer mass (cross-layer CV about 1.3 %)
+        h_budgets = stlite.stlite_hierarchical_budgets(list(mass), L * budget, N_TOK)
+        h_out = [(torch.empty((b, HKV, D), dtype=torch.bfloat16, device=dev),
+                  torch.empty((b, HKV, D), dtype=torch.bfloat16, device=dev),
+                  torch.empty((HKV, b), dtype=torch.int32, device=dev)) for b in h_budgets]
+        h_io = [(qs[l], ks[l], vs[l]) + h_out[l] for l in range(L)]
+        cases = [("tsg_dot", dict(tsg_metric=stlite.STLITE_TSG_DOT)),
+                 ("tsg_neg_l2", dict(tsg_metric=stlite.STLITE_TSG_NEG_L2)),
+                 ("fixed_tau_0.85", dict(fixed_tau=0.85)),
+                 ("uniform_base", dict(base_scorer=stlite.STLITE_BASE_UNIFORM)),
+                 ("abase_max", dict(abase_norm=stlite.STLITE_ABASE_MAX)),
+                 ("css_3x3_box", None), ("css_5x5", dict(css_size=5)), ("css_7x7", dict(css_size=7)),
+                 ("css_9x9", dict(css_size=9)), ("hierarchical_budgets", dict())]
+        for name, kw in cases:
+            if name == "css_3x3_box":
+                # the method's CSS on the box-sum kernel instead of the tensor cores (staged entry)
+                phi_b = torch.empty((HKV, N_TOK), dtype=torch.float32, device=dev)
+
+                def vstep(st=None):
+                    for l in range(L):
+                        stlite.stlite_spatial_saliency_size(qs[l], ks[l], fs, 3, phi_b, ws, st)
+            elif name == "hierarchical_budgets":
+                def vstep(st=None):
+                    stlite.stlite_compress_layers_budgets(h_io, fs, prm, h_budgets, ws, st)
+            else:
+                prm_v = stlite.make_params(BETA, **kw)
+
+                def vstep(st=None, prm_v=prm_v):
+                    stlite.stlite_compress_layers(layer_io, fs, prm_v, ws, st)
+            with torch.cuda.stream(stream):
+                for _ in range(2):
+                    vstep(stream)
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                vstep(stream)
+            a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            reps = max(5, min(20, args.steps))
+            with torch.cuda.stream(stream):
+                for _ in range(2):
+                    g.replay()
+                a0.record(stream)
+                for _ in range(reps):
+                    g.replay()
+                a1.record(stream)
+            torch.cuda.synchronize()
+            assert stlite.stlite_device_status(ws, stream) == stlite.STLITE_OK
+            stlite.stlite_timing_read()
+            stlite.stlite_timing_enable(True)
+            with torch.cuda.stream(stream):
+                vstep(stream)
+            stream.synchronize()
+            stlite.stlite_timing_enable(False)
+            vk = stlite.stlite_timing_read()
+            entry = dict(ms_per_step=a0.elapsed_time(a1) / reps,
+                         kernels_ms={k: t / c for k, (c, t) in vk.items()})
+            if "css_box" in vk:
+                # the staged entry launches once per layer, the fused pass once for all layers
+                c, t = vk["css_box"]
+                entry["css_box_roofline"] = kernel_roofline("css_box", t / c * 1e-3,
+                                                            1 if name == "css_3x3_box" else L, budget, peaks)
+            if name == "hierarchical_budgets":
+                entry["budgets_min_max"] = [min(h_budgets), max(h_budgets)]
+            variants[name] = entry
+        # the variants overwrote the shared workspace's per-layer results; the
+        # published method's outputs are recomputed for what follows
+        with torch.cuda.stream(stream):
+            step(stream)
+        stream.synchronize()
+
     # ---- consumer: one decode step (a query row per layer) over the full and
     # the compressed caches of all layers, each step one CUDA graph
     decode = None
@@ -597,7 +675,7 @@ def run_gpu(args):
                     roofline=roof, kernels=kernels, gpu_launches=per_step_launches * args.steps,
                     clocks=dict(sm_mhz=clk["sm_mhz"], sm_max_mhz=clk["sm_max_mhz"], reasons=clk["reasons"],
                                 samples=clk["samples"]),
-                    e2e=e2e, cpu_baseline=cpu, decode=decode)
+                    e2e=e2e, cpu_baseline=cpu, decode=decode, variants=variants)
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()

@@ -101,6 +101,7 @@ typedef struct {
  * uniform prior of the base-scoring ablation). */
 typedef enum { STLITE_TSG_COSINE = 0, STLITE_TSG_DOT = 1, STLITE_TSG_NEG_L2 = 2 } stlite_tsg_metric;
 typedef enum { STLITE_BASE_WINDOW = 0, STLITE_BASE_UNIFORM = 1 } stlite_base_scorer;
+typedef enum { STLITE_ABASE_RAW = 0, STLITE_ABASE_MAX = 1 } stlite_abase_norm;
 
 typedef struct {
   double beta;        /* compression ratio in (0, 1]: B = floor(beta * N) (Sec. 2.1) */
@@ -115,6 +116,12 @@ typedef struct {
                           (the fixed-threshold control: pool tokens with rho > tau are gated) */
   float tsg_fixed_tau; /* used when tsg_fixed = 1; finite */
   int32_t base_scorer; /* stlite_base_scorer: A_base of Eq. (2), or A = w/N for every token */
+  int32_t abase_norm;  /* stlite_abase_norm: 0 uses A as Eq. (9) writes it; 1 divides each head's A
+                          by its maximum over the N tokens first (a reading of the scale of A that
+                          the paper's reported A_base values suggest) */
+  int32_t css_size;    /* CSS neighbourhood k x k of Eq. (4): 0 or 3 = the 3 x 3 Moore neighbourhood;
+                          5, 7 or 9 = the neighbourhood-size ablation (all in-grid cells within
+                          Chebyshev distance (k-1)/2, the token itself excluded) */
 } stlite_params;
 
 /* Flat per-layer budget (Sec. 2.1, Algorithm 1 initialisation):
@@ -149,6 +156,17 @@ STLITE_API stlite_status stlite_gate_frames(const stlite_shape* shape, const stl
 STLITE_API stlite_status stlite_spatial_saliency(const stlite_shape* shape, const stlite_frames* frames,
                                       const void* k, float* phi, void* ws, size_t ws_bytes,
                                       void* stream);
+
+/* Step 3 over the size x size neighbourhood (the neighbourhood-size ablation
+ * of the CSS appendix): Phi = 1 - mean cosine to the in-grid cells within
+ * Chebyshev distance (size-1)/2 in the same frame, the token itself
+ * excluded.  size: 3, 5, 7 or 9 (3 is the method's Moore neighbourhood; this
+ * entry computes it through box sums of normalised keys on the CUDA cores,
+ * stlite_spatial_saliency on the tensor cores).  Any grid width.  phi as for
+ * stlite_spatial_saliency; STLITE_EINVAL for another size. */
+STLITE_API stlite_status stlite_spatial_saliency_size(const stlite_shape* shape, const stlite_frames* frames,
+                                                      const void* k, int32_t size, float* phi, void* ws,
+                                                      size_t ws_bytes, void* stream);
 
 /* Step 4, Eq. (9) and Top_B (base_scorer = STLITE_BASE_UNIFORM replaces a_base,
  * which may then be NULL, by w/N for every token): S = a_base for text tokens, S = gate * (a_base +

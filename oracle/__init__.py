@@ -52,9 +52,9 @@ def _load():
         lib.orc_abase.restype = None
         lib.orc_abase.argtypes = [_dp, _dp, _i32, _i32, _i32, _i32, _i32, _i32, _dp]
         lib.orc_css_phi_token.restype = ctypes.c_double
-        lib.orc_css_phi_token.argtypes = [_dp, _i32, _i32, _i32, _i32, _i32, _i32, _i32, _i32]
+        lib.orc_css_phi_token.argtypes = [_dp, _i32, _i32, _i32, _i32, _i32, _i32, _i32, _i32, _i32]
         lib.orc_css_phi.restype = None
-        lib.orc_css_phi.argtypes = [_dp, _i32, _i32, _i32, _i32, _i32, _ip, _ip, _ip, _dp]
+        lib.orc_css_phi.argtypes = [_dp, _i32, _i32, _i32, _i32, _i32, _ip, _ip, _ip, _i32, _dp]
         lib.orc_tsg_rho_token.restype = ctypes.c_double
         lib.orc_tsg_rho_token.argtypes = [_dp, _i32, _i32, _i32, _i32, _i32, _i32, _i32]
         lib.orc_tsg_rho.restype = None
@@ -141,8 +141,11 @@ def abase(q, k, threads: int = 1) -> np.ndarray:
     return out
 
 
-def css_phi(k, frames, threads: int = 1) -> np.ndarray:
-    """Eqs. 4-5: Phi = 1 - mean Moore-neighbour cosine; NaN for text tokens."""
+def css_phi(k, frames, threads: int = 1, size: int = 3) -> np.ndarray:
+    """Eqs. 4-5: Phi = 1 - mean neighbour cosine over the in-grid cells of the
+    size x size neighbourhood (3: the Moore neighbourhood of the method; 5, 7,
+    9: the neighbourhood-size ablation); NaN for text tokens."""
+    assert size in (3, 5, 7, 9)
     lib = _load()
     k = _c64(k)
     n, hkv, d = k.shape
@@ -151,17 +154,18 @@ def css_phi(k, frames, threads: int = 1) -> np.ndarray:
 
     def run(h):
         lib.orc_css_phi(_d(k), n, hkv, d, h, len(off), off.ctypes.data_as(_ip),
-                        gh.ctypes.data_as(_ip), gw.ctypes.data_as(_ip), out[h].ctypes.data_as(_dp))
+                        gh.ctypes.data_as(_ip), gw.ctypes.data_as(_ip), size // 2, out[h].ctypes.data_as(_dp))
 
     _per_head(run, hkv, threads)
     return out
 
 
-def css_phi_token(k, h: int, off: int, gh: int, gw: int, u: int, v: int) -> float:
+def css_phi_token(k, h: int, off: int, gh: int, gw: int, u: int, v: int, size: int = 3) -> float:
     """Phi of the single visual token (u, v) of the frame at ``off``."""
+    assert size in (3, 5, 7, 9)
     k = _c64(k)
     n, hkv, d = k.shape
-    return float(_load().orc_css_phi_token(_d(k), hkv, d, h, off, gh, gw, u, v))
+    return float(_load().orc_css_phi_token(_d(k), hkv, d, h, off, gh, gw, u, v, size // 2))
 
 
 TSG_COSINE, TSG_DOT, TSG_NEG_L2 = 0, 1, 2
@@ -263,15 +267,31 @@ def gather(k, v, idx):
 
 
 BASE_WINDOW, BASE_UNIFORM = 0, 1
+ABASE_RAW, ABASE_MAX = 0, 1
+
+
+def normalise_max(a) -> np.ndarray:
+    """A divided by its maximum over the tokens, per head (rows whose maximum
+    is not positive are left as they are): the reading of A_base's scale that
+    the paper's reported A_base magnitudes suggest."""
+    a = np.asarray(a, dtype=np.float64)
+    out = a.copy()
+    for h in range(a.shape[0]):
+        m = a[h].max()
+        if m > 0:
+            out[h] = a[h] / m
+    return out
 
 
 def compress_layer(q, k, frames, beta: float = 0.2, k_override: int = 0, alpha: float = 1.0,
                    tsg_enable: int = 1, css_enable: int = 1, threads: int = 1, tsg_metric: int = TSG_COSINE,
-                   fixed_tau=None, base_scorer: int = BASE_WINDOW) -> dict:
+                   fixed_tau=None, base_scorer: int = BASE_WINDOW, abase_norm: int = ABASE_RAW,
+                   css_size: int = 3) -> dict:
     """Algorithm 1 for one layer: every stage in the paper's order.  The
     keyword variants are the paper's ablations: TSG similarity metric, a fixed
     gate threshold, and the uniform base prior (A = w/N for every token, the
-    same total as the window score)."""
+    same total as the window score); abase_norm = ABASE_MAX divides A by its
+    per-head maximum before Eq. 9; css_size is the CSS neighbourhood k x k."""
     n = k.shape[0]
     w = q.shape[0]
     b = budget(n, beta, k_override)
@@ -279,7 +299,9 @@ def compress_layer(q, k, frames, beta: float = 0.2, k_override: int = 0, alpha: 
         a = np.full((k.shape[1], n), w / n, dtype=np.float64)
     else:
         a = abase(q, k, threads)
-    phi = css_phi(k, frames, threads)
+    if abase_norm == ABASE_MAX:
+        a = normalise_max(a)
+    phi = css_phi(k, frames, threads, size=css_size)
     if tsg_enable:
         rho = tsg_rho(k, frames, threads, metric=tsg_metric)
     else:

@@ -111,16 +111,19 @@ void orc_abase(const double* q, const double* k, int32_t n, int32_t w, int32_t h
 
 /* --------------------------------------------- CSS saliency (Eqs. 4-5) */
 
-/* Phi for one visual token at (u, v) of frame f, KV head h:
+/* Phi for one visual token at (u, v) of frame f, KV head h (Eqs. 4-5):
  *   H = (1/|N|) sum_{(p,q) in N(u,v)} cos(k_{u,v}, k_{p,q}),  Phi = 1 - H,
- * with N(u,v) the in-grid cells of the 3x3 Moore neighbourhood (reading R3). */
+ * with N(u,v) the in-grid cells of the (2 radius + 1)^2 neighbourhood other
+ * than (u, v) itself: radius 1 is the 3x3 Moore neighbourhood of the method
+ * (reading R3), radius 2-4 the 5x5 to 9x9 kernels of the neighbourhood-size
+ * ablation. */
 double orc_css_phi_token(const double* k, int32_t hkv, int32_t d, int32_t h, int32_t off,
-                         int32_t gh, int32_t gw, int32_t u, int32_t v) {
+                         int32_t gh, int32_t gw, int32_t u, int32_t v, int32_t radius) {
   const double* c = key_row(k, hkv, d, off + u * gw + v, h);
   double sum = 0.0;
   int32_t cnt = 0;
-  for (int32_t du = -1; du <= 1; ++du) {
-    for (int32_t dv = -1; dv <= 1; ++dv) {
+  for (int32_t du = -radius; du <= radius; ++du) {
+    for (int32_t dv = -radius; dv <= radius; ++dv) {
       if (du == 0 && dv == 0) continue;
       int32_t pu = u + du, pv = v + dv;
       if (pu < 0 || pu >= gh || pv < 0 || pv >= gw) continue;
@@ -135,13 +138,13 @@ double orc_css_phi_token(const double* k, int32_t hkv, int32_t d, int32_t h, int
 /* Phi over all tokens of KV head h; text tokens get NaN (reading R7). */
 void orc_css_phi(const double* k, int32_t n, int32_t hkv, int32_t d, int32_t h,
                  int32_t n_frames, const int32_t* off, const int32_t* gh, const int32_t* gw,
-                 double* phi_out) {
+                 int32_t radius, double* phi_out) {
   for (int32_t j = 0; j < n; ++j) phi_out[j] = NAN;
   for (int32_t f = 0; f < n_frames; ++f)
     for (int32_t u = 0; u < gh[f]; ++u)
       for (int32_t v = 0; v < gw[f]; ++v)
         phi_out[off[f] + u * gw[f] + v] =
-            orc_css_phi_token(k, hkv, d, h, off[f], gh[f], gw[f], u, v);
+            orc_css_phi_token(k, hkv, d, h, off[f], gh[f], gw[f], u, v, radius);
 }
 
 /* ----------------------------------------------- TSG redundancy (Eq. 6) */
@@ -305,7 +308,7 @@ void orc_compress_head(const double* q, const double* k, int32_t n, int32_t w, i
                        int32_t tsg_enable, int32_t css_enable, double* a, double* phi,
                        double* rho, uint8_t* gate, double* s, double* tau, int32_t* idx_out) {
   orc_abase(q, k, n, w, hq, hkv, d, h, a);
-  orc_css_phi(k, n, hkv, d, h, n_frames, off, gh, gw, phi);
+  orc_css_phi(k, n, hkv, d, h, n_frames, off, gh, gw, 1, phi);
   if (tsg_enable)
     orc_tsg_rho(k, n, hkv, d, h, n_frames, off, gh, gw, 0, rho);
   else

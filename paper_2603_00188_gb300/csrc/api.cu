@@ -81,6 +81,9 @@ stlite_status check_params(const stlite_params* pr) {
   if (pr->tsg_fixed != 0 && pr->tsg_fixed != 1) return STLITE_EINVAL;
   if (pr->tsg_fixed && !isfinite(pr->tsg_fixed_tau)) return STLITE_EINVAL;
   if (pr->base_scorer != STLITE_BASE_WINDOW && pr->base_scorer != STLITE_BASE_UNIFORM) return STLITE_EINVAL;
+  if (pr->abase_norm != STLITE_ABASE_RAW && pr->abase_norm != STLITE_ABASE_MAX) return STLITE_EINVAL;
+  if (pr->css_size != 0 && pr->css_size != 3 && pr->css_size != 5 && pr->css_size != 7 && pr->css_size != 9)
+    return STLITE_EINVAL;
   return STLITE_OK;
 }
 
@@ -234,8 +237,11 @@ Strided<T> one(T* p) {
 // CSS (Eqs. 4-5) into phi, plus the inverse key norms rn / rn_cur that TSG
 // uses.  bf16 caches whose grids are at most 127 wide take the tensor-core
 // kernel; otherwise the CUDA-core one.
-cudaError_t run_css(const Ctx& c, const LayerPtrs& io, Strided<float> phi) {
+// size: the CSS neighbourhood (0 or 3 = the method's 3x3; 5, 7, 9 = the
+// size ablation, on the box-sum kernel).
+cudaError_t run_css(const Ctx& c, const LayerPtrs& io, Strided<float> phi, int size = 3) {
   Strided<float> rn = c.view<float>(c.plan.rn), rc = c.view<float>(c.plan.rn_cur);
+  if (size > 3) return launch_css_box(c.p, c.ft, io, size, phi, rn, rc, c.plan.cur_pad, c.st);
   if (use_tensor_cores(c.p) && css_umma_supported(c.ft)) {
     const size_t hn4 = (size_t)c.p.hkv * c.p.n * 4;
     Strided<float> dE = c.view<float>(c.plan.dots), dS = c.view<float>(c.plan.dots + hn4);
@@ -277,6 +283,7 @@ void select_variants(SelectArgs& a, const stlite_params* params, const Problem& 
   a.tsg_fixed_tau = params->tsg_fixed_tau;
   a.base_uniform = params->base_scorer == STLITE_BASE_UNIFORM ? 1 : 0;
   a.a_uniform = (float)p.w / (float)p.n;  // the window score's total, spread evenly
+  a.a_norm_max = params->abase_norm == STLITE_ABASE_MAX ? 1 : 0;
 }
 
 // Algorithm 1 for a batch of layers (steps 1-5), every stage one launch.
@@ -289,7 +296,7 @@ stlite_status compress_batch(const Ctx& c, const stlite_params* params, const La
   // norms pass provides them.
   cudaError_t e = cudaSuccess;
   if (params->css_enable)
-    e = run_css(c, io, phi);
+    e = run_css(c, io, phi, params->css_size);
   else if (tsg)
     e = run_norms(c, io);
   if (e == cudaSuccess && tsg) e = run_tsg(c, io, params->tsg_metric);
@@ -388,6 +395,21 @@ stlite_status stlite_spatial_saliency(const stlite_shape* shape, const stlite_fr
   if (!k || !phi || !aligned16(k) || !aligned16(phi)) return STLITE_EINVAL;
   const LayerPtrs io = single_layer(nullptr, k, nullptr, nullptr, nullptr, nullptr);
   cudaError_t e = run_css(c, io, one(phi));
+  if (e == cudaSuccess) e = launch_fill_text_nan(c.p, c.ft, phi, c.st);
+  return cuda_status(e);
+}
+
+stlite_status stlite_spatial_saliency_size(const stlite_shape* shape, const stlite_frames* frames,
+                                           const void* k, int32_t size, float* phi, void* ws, size_t ws_bytes,
+                                           void* stream) {
+  if (size != 3 && size != 5 && size != 7 && size != 9) return STLITE_EINVAL;
+  Ctx c;
+  stlite_status s = prepare(shape, frames, ws, ws_bytes, 1, stream, &c);
+  if (s != STLITE_OK) return s;
+  if (!k || !phi || !aligned16(k) || !aligned16(phi)) return STLITE_EINVAL;
+  const LayerPtrs io = single_layer(nullptr, k, nullptr, nullptr, nullptr, nullptr);
+  cudaError_t e = launch_css_box(c.p, c.ft, io, size, one(phi), c.view<float>(c.plan.rn),
+                                 c.view<float>(c.plan.rn_cur), c.plan.cur_pad, c.st);
   if (e == cudaSuccess) e = launch_fill_text_nan(c.p, c.ft, phi, c.st);
   return cuda_status(e);
 }

@@ -139,6 +139,12 @@ cudaError_t launch_css_umma(const Problem& p, const FrameTable& ft, const LayerP
                             Strided<float> rn, Strided<float> rn_cur, int cur_pad, Strided<float> dE,
                             Strided<float> dS, Strided<float> dSE, Strided<float> dSW, uint32_t* err,
                             cudaStream_t st);
+// CSS over the size x size neighbourhood (size 3, 5, 7 or 9; 3 is the
+// method's Moore neighbourhood) on the CUDA cores, through box sums of the
+// normalised keys; any grid width.  Writes phi, rn and rn_cur as launch_css.
+cudaError_t launch_css_box(const Problem& p, const FrameTable& ft, const LayerPtrs& io, int size,
+                           Strided<float> phi, Strided<float> rn, Strided<float> rn_cur, int cur_pad,
+                           cudaStream_t st);
 // phi[h][j] = NaN for every text token j (one layer).
 cudaError_t launch_fill_text_nan(const Problem& p, const FrameTable& ft, float* phi, cudaStream_t st);
 
@@ -162,6 +168,7 @@ struct SelectArgs {
   float tsg_fixed_tau;
   int base_uniform;    // 1: A = a_uniform for every token instead of a_base
   float a_uniform;
+  int a_norm_max;      // 1: A / max_j A per head before Eq. 9
   Strided<const float> rho_part;  // [nchunk][Hkv][N]
   Strided<const float> rn;        // [Hkv][N]
   Strided<float> rho;             // out [Hkv][N]

@@ -31,7 +31,27 @@ struct SelShared {
   uint32_t bcast[4];
   uint32_t warp_tot[32];
   uint32_t counts[2];     // (greater, equal) of this CTA for the compaction
+  float warp_max[32];
+  float cta_max;          // read by the cluster's other CTAs
 };
+
+// Maximum of v over every thread of the cluster (every CTA must call it).
+__device__ float cluster_max(cg::cluster_group& cl, float v, SelShared& sh) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  if (lane == 0) sh.warp_max[wid] = v;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float m = sh.warp_max[0];
+    for (int w = 1; w < nw; ++w) m = fmaxf(m, sh.warp_max[w]);
+    sh.cta_max = m;
+  }
+  cl.sync();
+  float m = -CUDART_INF_F;
+  for (int r = 0; r < (int)cl.num_blocks(); ++r) m = fmaxf(m, *cl.map_shared_rank(&sh.cta_max, r));
+  return m;
+}
 
 // Exclusive block-wide prefix sum of v; *total receives the block sum.
 __device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* warp_tot,
@@ -277,12 +297,25 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
     float* sc = a.score.at(l) + hn;
     const float alpha = a.css_enable ? a.alpha : 0.f;
     const bool fused = (a.mode & kSelGate) != 0;  // gate decided here from the rho keys
+    // optional A / max_j A (per head): the cluster-wide maximum first
+    float amax = 0.f;
+    if (a.a_norm_max) {
+      if (ab) {
+        float m = 0.f;
+        for (int t = j0 + tid; t < j1; t += blockDim.x) m = fmaxf(m, __ldg(ab + t));
+        amax = cluster_max(cl, m, sh);
+      } else {
+        amax = a.a_uniform;
+      }
+    }
+    const bool a_div = amax > 0.f;
     // Eq. 9: S = A_base for text tokens; for visual tokens S = A_base +
     // alpha * Phi where the gate is open and 0 where it is closed
     for_tokens<2>(
         ft, j0, j1,
         [&](int t, int kind) {
-          const float A = ab ? __ldg(ab + t) : a.a_uniform;
+          float A = ab ? __ldg(ab + t) : a.a_uniform;
+          if (a_div) A = __fdiv_rn(A, amax);
           const float P = (kind != kTokText && alpha != 0.f) ? __ldg(ph + t) : 0.f;
           const float G = (kind != kTokText && !fused && gt != nullptr) ? (float)gt[t] : 1.f;
           return make_float3(A, P, G);

@@ -256,6 +256,185 @@ cudaError_t launch_css(const Problem& p, const FrameTable& ft, const LayerPtrs& 
   return css_launch_t<float>(p, ft, io, phi, rn, rn_cur, cur_pad, st);
 }
 
+// ------------------------------------------------------- CSS, k x k box
+// Eqs. 4-5 over the (2R+1) x (2R+1) neighbourhood (R = 1 is the method's 3x3
+// Moore neighbourhood; R = 2..4 the 5x5..9x9 kernels of the size ablation).
+// With khat_j = k_j / max(|k_j|, 1e-8) the neighbour cosines add up to
+//   sum_{j in N(i)} cos(k_i, k_j) = khat_i . (sum_{j in box(i)} khat_j - khat_i),
+// so a cell needs one box sum of normalised keys, whatever the size, and
+// the box sum separates into row sums and a sum of 2R+1 rows.  A CTA (tile,
+// frame, layer*Hkv + head) stages kBoxRows x kBoxCols output cells plus an
+// R-cell halo (out-of-grid cells as zero keys with rn = 0, so they add
+// nothing); each 16-lane half-warp owns one output column, 8 dimensions per
+// lane, walks the tile's rows once and keeps the last 2R+1 row sums in
+// registers.  rn of a cell uses the same operation sequence as the norms
+// kernel, so both agree bit for bit.
+constexpr int kBoxRows = 8, kBoxCols = 16, kBoxThreads = 256;
+
+template <typename T, int R>
+struct BoxGeom {
+  static constexpr int TH = kBoxRows + 2 * R, TW = kBoxCols + 2 * R, cells = TH * TW;
+  static constexpr int stride = kD * (int)sizeof(T) + 16;  // padded key row
+  static constexpr int smem = cells * stride + cells * 4;
+};
+
+template <typename T, int R>
+__global__ void __launch_bounds__(kBoxThreads) k_css_box(const __grid_constant__ LayerPtrs io,
+                                                         const __grid_constant__ FrameTable ft, int hkv,
+                                                         Strided<float> phi_all, Strided<float> rn_all,
+                                                         Strided<float> rc_all, int cur_pad) {
+  using Gm = BoxGeom<T, R>;
+  constexpr int kChunks = kD * (int)sizeof(T) / 16;
+  constexpr int kPer = 16 / (int)sizeof(T);
+  constexpr int TW = Gm::TW, TH = Gm::TH, D2 = 2 * R + 1;
+  extern __shared__ float4 box_smem[];
+  uint8_t* keys = reinterpret_cast<uint8_t*>(box_smem);
+  float* rn = reinterpret_cast<float*>(keys + (size_t)Gm::cells * Gm::stride);
+  const int f = blockIdx.y, l = blockIdx.z / hkv, h = blockIdx.z % hkv, n = ft.n_tokens;
+  const int tid = threadIdx.x;
+  if (f >= ft.n_frames) return;
+  const int gh = ft.gh[f], gw = ft.gw[f], off = ft.off[f];
+  const int tv = (gw + kBoxCols - 1) / kBoxCols;
+  if ((int)blockIdx.x >= ((gh + kBoxRows - 1) / kBoxRows) * tv) return;
+  const int u0 = ((int)blockIdx.x / tv) * kBoxRows, v0 = ((int)blockIdx.x % tv) * kBoxCols;
+  const T* k = static_cast<const T*>(io.k[l]);
+  // stage: local cell (a, b) = grid cell (u0 - R + a, v0 - R + b)
+  for (int e = tid; e < Gm::cells * kChunks; e += blockDim.x) {
+    const int cell = e / kChunks, ch = e - cell * kChunks;
+    const int u = u0 - R + cell / TW, v = v0 - R + cell % TW;
+    uint8_t* dstp = keys + (size_t)cell * Gm::stride + 16 * ch;
+    if (u < 0 || u >= gh || v < 0 || v >= gw) {
+      *reinterpret_cast<uint4*>(dstp) = make_uint4(0u, 0u, 0u, 0u);
+      continue;
+    }
+    const T* src = k + ((size_t)(off + u * gw + v) * hkv + h) * kD + ch * kPer;
+    const uint32_t dst = static_cast<uint32_t>(__cvta_generic_to_shared(dstp));
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+  }
+  asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+  __syncthreads();
+  // inverse norms (0 outside the grid); the output cells' go to rn / rn_cur
+  for (int cell = tid; cell < Gm::cells; cell += blockDim.x) {
+    const int a = cell / TW, b = cell % TW;
+    const int u = u0 - R + a, v = v0 - R + b;
+    float r = 0.f;
+    if (u >= 0 && u < gh && v >= 0 && v < gw) {
+      const uint8_t* p0 = keys + (size_t)cell * Gm::stride;
+      float sn = 0.f;
+#pragma unroll 4
+      for (int c = 0; c < kChunks; ++c) {
+        float x[kPer];
+        unpack16<T>(*reinterpret_cast<const uint4*>(p0 + 16 * c), x);
+#pragma unroll
+        for (int t = 0; t < kPer; ++t) sn = fmaf(x[t], x[t], sn);
+      }
+      r = 1.0f / fmaxf(sqrtf(sn), 1e-8f);
+      if (a >= R && a < R + kBoxRows && b >= R && b < R + kBoxCols) {
+        const int j = off + u * gw + v;
+        rn_all.at(l)[(size_t)h * n + j] = r;
+        if (f == ft.n_frames - 1) rc_all.at(l)[(size_t)h * cur_pad + (j - off)] = r;
+      }
+    }
+    rn[cell] = r;
+  }
+  __syncthreads();
+  // box sums: lane group (16 lanes) = output column, 8 dimensions per lane
+  const int dg = tid & 15, col = tid >> 4;
+  const int v = v0 + col;
+  float* phi = phi_all.at(l);
+  auto load8 = [&](int cell, float (&x)[8]) {
+    const uint8_t* p0 = keys + (size_t)cell * Gm::stride + dg * 8 * (int)sizeof(T);
+#pragma unroll
+    for (int c = 0; c < 8 / kPer; ++c) {
+      float y[kPer];
+      unpack16<T>(*reinterpret_cast<const uint4*>(p0 + 16 * c), y);
+#pragma unroll
+      for (int t = 0; t < kPer; ++t) x[c * kPer + t] = y[t];
+    }
+  };
+  float ring[D2][8];
+#pragma unroll
+  for (int a = 0; a < TH; ++a) {
+    float hs[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) hs[e] = 0.f;
+#pragma unroll
+    for (int dv = 0; dv < D2; ++dv) {
+      const int cell = a * TW + col + dv;
+      const float r = rn[cell];
+      float x[8];
+      load8(cell, x);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) hs[e] = fmaf(r, x[e], hs[e]);
+    }
+#pragma unroll
+    for (int e = 0; e < 8; ++e) ring[a % D2][e] = hs[e];
+    if (a >= 2 * R) {
+      const int o = a - 2 * R;  // output row of the tile
+      const int cell = (o + R) * TW + col + R;
+      const float ri = rn[cell];
+      float x[8];
+      load8(cell, x);
+      float dot = 0.f;
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        float s = ring[0][e];
+#pragma unroll
+        for (int q = 1; q < D2; ++q) s += ring[q][e];
+        const float kh = ri * x[e];
+        dot = fmaf(kh, s - kh, dot);
+      }
+#pragma unroll
+      for (int m = 8; m > 0; m >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, m);
+      const int u = u0 + o;
+      if (dg == 0 && u < gh && v < gw) {
+        const int nu = min(u + R, gh - 1) - max(u - R, 0) + 1;
+        const int nv = min(v + R, gw - 1) - max(v - R, 0) + 1;
+        const int cnt = nu * nv - 1;
+        phi[(size_t)h * n + off + u * gw + v] = cnt ? 1.0f - dot / (float)cnt : 0.0f;
+      }
+    }
+  }
+}
+
+template <typename T, int R>
+static cudaError_t css_box_t(const Problem& p, const FrameTable& ft, const LayerPtrs& io, Strided<float> phi,
+                             Strided<float> rn, Strided<float> rn_cur, int cur_pad, cudaStream_t st) {
+  using Gm = BoxGeom<T, R>;
+  cudaError_t e = cudaFuncSetAttribute(k_css_box<T, R>, cudaFuncAttributeMaxDynamicSharedMemorySize, Gm::smem);
+  if (e != cudaSuccess) return e;
+  int tiles = 1;
+  for (int f = 0; f < ft.n_frames; ++f) {
+    const int t = ((ft.gh[f] + kBoxRows - 1) / kBoxRows) * ((ft.gw[f] + kBoxCols - 1) / kBoxCols);
+    tiles = t > tiles ? t : tiles;
+  }
+  TimingScope ts("css_box", st);
+  dim3 grid((unsigned)tiles, (unsigned)(ft.n_frames > 0 ? ft.n_frames : 1), (unsigned)(p.L * p.hkv));
+  k_css_box<T, R><<<grid, kBoxThreads, Gm::smem, st>>>(io, ft, p.hkv, phi, rn, rn_cur, cur_pad);
+  return cudaGetLastError();
+}
+
+template <typename T>
+static cudaError_t css_box_r(int radius, const Problem& p, const FrameTable& ft, const LayerPtrs& io,
+                             Strided<float> phi, Strided<float> rn, Strided<float> rn_cur, int cur_pad,
+                             cudaStream_t st) {
+  switch (radius) {
+    case 1: return css_box_t<T, 1>(p, ft, io, phi, rn, rn_cur, cur_pad, st);
+    case 2: return css_box_t<T, 2>(p, ft, io, phi, rn, rn_cur, cur_pad, st);
+    case 3: return css_box_t<T, 3>(p, ft, io, phi, rn, rn_cur, cur_pad, st);
+    case 4: return css_box_t<T, 4>(p, ft, io, phi, rn, rn_cur, cur_pad, st);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+cudaError_t launch_css_box(const Problem& p, const FrameTable& ft, const LayerPtrs& io, int size,
+                           Strided<float> phi, Strided<float> rn, Strided<float> rn_cur, int cur_pad,
+                           cudaStream_t st) {
+  if (ft.n_frames == 0) return cudaSuccess;
+  if (p.dtype == kBF16) return css_box_r<__nv_bfloat16>(size / 2, p, ft, io, phi, rn, rn_cur, cur_pad, st);
+  return css_box_r<float>(size / 2, p, ft, io, phi, rn, rn_cur, cur_pad, st);
+}
+
 cudaError_t launch_fill_text_nan(const Problem& p, const FrameTable& ft, float* phi, cudaStream_t st) {
   long long tot = (long long)p.n * p.hkv;
   long long blocks = (tot + 255) / 256;

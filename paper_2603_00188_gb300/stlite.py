@@ -29,7 +29,7 @@ EXPORTED = ("stlite_budget", "stlite_workspace_size", "stlite_score", "stlite_ga
             "stlite_compress_layer", "stlite_device_status", "stlite_timing_enable", "stlite_timing_read",
             "stlite_status_string", "stlite_score_noalloc", "stlite_compress_layers", "stlite_compress_varlen",
             "stlite_workspace_size_varlen", "stlite_decode_attention", "stlite_decode_workspace_size",
-            "stlite_compress_layers_budgets", "stlite_hierarchical_budgets")
+            "stlite_compress_layers_budgets", "stlite_hierarchical_budgets", "stlite_spatial_saliency_size")
 
 
 class Shape(ctypes.Structure):
@@ -46,11 +46,13 @@ class Frames(ctypes.Structure):
 class Params(ctypes.Structure):
     _fields_ = [("beta", ctypes.c_double), ("k_override", ctypes.c_int32), ("alpha", ctypes.c_float),
                 ("tsg_enable", ctypes.c_int32), ("css_enable", ctypes.c_int32), ("tsg_metric", ctypes.c_int32),
-                ("tsg_fixed", ctypes.c_int32), ("tsg_fixed_tau", ctypes.c_float), ("base_scorer", ctypes.c_int32)]
+                ("tsg_fixed", ctypes.c_int32), ("tsg_fixed_tau", ctypes.c_float), ("base_scorer", ctypes.c_int32),
+                ("abase_norm", ctypes.c_int32), ("css_size", ctypes.c_int32)]
 
 
 STLITE_TSG_COSINE, STLITE_TSG_DOT, STLITE_TSG_NEG_L2 = 0, 1, 2
 STLITE_BASE_WINDOW, STLITE_BASE_UNIFORM = 0, 1
+STLITE_ABASE_RAW, STLITE_ABASE_MAX = 0, 1
 
 
 class LayerIO(ctypes.Structure):
@@ -97,6 +99,8 @@ _sig = {
     "stlite_compress_layers_budgets": (_S, [ctypes.POINTER(Shape), ctypes.POINTER(Frames), ctypes.POINTER(Params),
                                             ctypes.c_int32, ctypes.POINTER(LayerIO), ctypes.POINTER(ctypes.c_int32),
                                             _P, ctypes.c_size_t, _P]),
+    "stlite_spatial_saliency_size": (_S, [ctypes.POINTER(Shape), ctypes.POINTER(Frames), _P, ctypes.c_int32, _P, _P,
+                                          ctypes.c_size_t, _P]),
     "stlite_hierarchical_budgets": (_S, [ctypes.c_int32, ctypes.POINTER(ctypes.c_double), ctypes.c_int64,
                                          ctypes.c_int32, ctypes.POINTER(ctypes.c_int32)]),
 }
@@ -155,12 +159,14 @@ def _frames(frames) -> FrameSpec:
 
 
 def make_params(beta=0.2, k_override=0, alpha=1.0, tsg_enable=1, css_enable=1, tsg_metric=STLITE_TSG_COSINE,
-                fixed_tau=None, base_scorer=STLITE_BASE_WINDOW) -> Params:
-    """Parameters of the pass; the last three select the paper's ablation
-    variants (TSG similarity metric, a fixed gate threshold, the uniform base
-    prior) and default to the method as published."""
+                fixed_tau=None, base_scorer=STLITE_BASE_WINDOW, abase_norm=STLITE_ABASE_RAW, css_size=3) -> Params:
+    """Parameters of the pass; the keywords after css_enable select the
+    paper's ablation variants (TSG similarity metric, a fixed gate threshold,
+    the uniform base prior, A_base divided by its maximum, the CSS
+    neighbourhood size) and default to the method as published."""
     return Params(float(beta), int(k_override), float(alpha), int(tsg_enable), int(css_enable), int(tsg_metric),
-                  0 if fixed_tau is None else 1, 0.0 if fixed_tau is None else float(fixed_tau), int(base_scorer))
+                  0 if fixed_tau is None else 1, 0.0 if fixed_tau is None else float(fixed_tau), int(base_scorer),
+                  int(abase_norm), int(css_size))
 
 
 # ----------------------------------------------------------------- entries
@@ -202,6 +208,13 @@ def stlite_spatial_saliency(q, k, frames, phi, ws, stream=None):
     fs = _frames(frames)
     _check(_lib.stlite_spatial_saliency(ctypes.byref(sh), ctypes.byref(fs.c), _ptr(k), _ptr(phi), _ptr(ws),
                                         ws.numel(), _stream(stream)), "stlite_spatial_saliency")
+
+
+def stlite_spatial_saliency_size(q, k, frames, size, phi, ws, stream=None):
+    sh = make_shape(q, k)
+    fs = _frames(frames)
+    _check(_lib.stlite_spatial_saliency_size(ctypes.byref(sh), ctypes.byref(fs.c), _ptr(k), int(size), _ptr(phi),
+                                             _ptr(ws), ws.numel(), _stream(stream)), "stlite_spatial_saliency_size")
 
 
 def stlite_select_topk(q, k, frames, params, a_base, phi, gate, budget, idx, score_out, ws, stream=None):
@@ -355,11 +368,13 @@ def stlite_timing_read() -> dict:
 # ------------------------------------------------------- convenience layer
 
 def compress_layer(q, k, v, frames, beta=0.2, k_override=0, alpha=1.0, tsg_enable=1, css_enable=1,
-                   ws=None, stream=None, tsg_metric=STLITE_TSG_COSINE, fixed_tau=None, base_scorer=STLITE_BASE_WINDOW):
+                   ws=None, stream=None, tsg_metric=STLITE_TSG_COSINE, fixed_tau=None, base_scorer=STLITE_BASE_WINDOW,
+                   abase_norm=STLITE_ABASE_RAW, css_size=3):
     """Allocates outputs (and a workspace if none is given) and runs
     stlite_compress_layer.  Returns (k_out, v_out, idx)."""
     fs = _frames(frames)
-    params = make_params(beta, k_override, alpha, tsg_enable, css_enable, tsg_metric, fixed_tau, base_scorer)
+    params = make_params(beta, k_override, alpha, tsg_enable, css_enable, tsg_metric, fixed_tau, base_scorer,
+                         abase_norm, css_size)
     sh = make_shape(q, k)
     b = stlite_budget(sh.n_tokens, beta, k_override)
     if b < 1:

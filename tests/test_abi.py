@@ -182,3 +182,24 @@ def test_compress_layers_budgets_reject_before_launch(st):
     bad = (st.LayerIO * 2)(st.LayerIO(*([good] * 6)), st.LayerIO(*([good] * 5 + [good + 8])))
     assert lib.stlite_compress_layers_budgets(ctypes.byref(sh), ctypes.byref(fr.c), ctypes.byref(prm), 2, bad,
                                               arr, P(good), 2 * need, None) == st.STLITE_EINVAL
+
+
+def test_variant_params_validation(st):
+    """CSS sizes other than 0/3/5/7/9 and unknown A_base scalings are refused
+    on the host, in the fused and in the staged entry points."""
+    lib = st._lib
+    sh = _shape(st)
+    fr = st.FrameSpec([0, 30], [4, 5], [5, 6])
+    need = st.stlite_workspace_size(sh, fr, st.make_params(0.2))
+    good = ctypes.c_void_p(0x10000)
+    for kw in (dict(css_size=4), dict(css_size=11), dict(css_size=-3), dict(abase_norm=2), dict(abase_norm=-1)):
+        prm = st.make_params(0.2, **kw)
+        assert lib.stlite_compress_layer(ctypes.byref(sh), ctypes.byref(fr.c), ctypes.byref(prm), good, good, good,
+                                         good, good, good, None, good, need, None) == st.STLITE_EINVAL, kw
+    for size in (0, 1, 4, 11):
+        assert lib.stlite_spatial_saliency_size(ctypes.byref(sh), ctypes.byref(fr.c), good, size, good, good, need,
+                                                None) == st.STLITE_EINVAL
+    assert lib.stlite_spatial_saliency_size(ctypes.byref(sh), ctypes.byref(fr.c), good, 5, good, good, need - 1,
+                                            None) == st.STLITE_EWORKSPACE
+    for size in (0, 3, 5, 7, 9):
+        assert st.stlite_workspace_size(sh, fr, st.make_params(0.2, css_size=size, abase_norm=1)) == need

@@ -673,3 +673,95 @@ def test_hierarchical_deviation_bound():
         d_int = (b.max() - b.min()) / (total / n_layers)
         assert d_real <= math.sqrt(2 * n_layers) * cv_s + 1e-12
         assert abs(d_int - d_real) <= 2.0 / (total / n_layers) + 1e-9
+
+
+# ------------------------------------- CSS neighbourhood size (5x5 .. 9x9)
+
+def _alt_sum(lo, hi):
+    # sum of (-1)^t for t in [lo, hi]
+    return sum((-1) ** t for t in range(lo, hi + 1))
+
+
+@pytest.mark.parametrize("size", [3, 5, 7, 9])
+def test_css_size_checkerboard_closed_form(size):
+    # keys +-e by the checkerboard: cos = (-1)^(du + dv), so the neighbour sum
+    # factorises into two alternating sums over the in-grid offsets, minus
+    # the cell itself
+    gh, gw, r = 11, 13, size // 2
+    k = np.zeros((gh * gw, 1, 4))
+    for u in range(gh):
+        for v in range(gw):
+            k[u * gw + v, 0, 2] = (-1) ** (u + v)
+    phi = oracle.css_phi(k, frames_of((0, gh, gw)), size=size)[0].reshape(gh, gw)
+    for u in range(gh):
+        for v in range(gw):
+            du0, du1 = -min(r, u), min(r, gh - 1 - u)
+            dv0, dv1 = -min(r, v), min(r, gw - 1 - v)
+            cnt = (du1 - du0 + 1) * (dv1 - dv0 + 1) - 1
+            expect = 1 - (_alt_sum(du0, du1) * _alt_sum(dv0, dv1) - 1) / cnt
+            assert abs(phi[u, v] - expect) < 1e-13, (size, u, v)
+
+
+@pytest.mark.parametrize("size", [5, 7, 9])
+def test_css_size_equal_orthonormal_and_rectangle(size):
+    rng = np.random.default_rng(size)
+    # equal keys: Phi = 0; distinct basis vectors: Phi = 1
+    k = np.repeat(rng.standard_normal((1, 2, 16)), 42, axis=0)
+    np.testing.assert_allclose(oracle.css_phi(k, frames_of((0, 6, 7)), size=size), 0.0, atol=1e-13)
+    gh, gw, d = 6, 9, 64
+    k = np.eye(d)[: gh * gw][:, None, :] * rng.uniform(0.5, 3.0, size=(gh * gw, 1, 1))
+    np.testing.assert_allclose(oracle.css_phi(k, frames_of((0, gh, gw)), size=size), 1.0, atol=1e-14)
+    # planted 3x4 rectangle of one key on the orthonormal background:
+    # Phi = 1 - (#rectangle cells in the window, self excluded) / |N|
+    r = np.zeros(d); r[-1] = 1.7
+    rect = [(u, v) for u in range(1, 4) for v in range(2, 6)]
+    for (u, v) in rect:
+        k[u * gw + v, 0] = r
+    phi = oracle.css_phi(k, frames_of((0, gh, gw)), size=size)[0].reshape(gh, gw)
+    rad = size // 2
+    for u in range(gh):
+        for v in range(gw):
+            nb = [(u + a, v + b) for a in range(-rad, rad + 1) for b in range(-rad, rad + 1)
+                  if (a or b) and 0 <= u + a < gh and 0 <= v + b < gw]
+            expect = 1 - sum((p in rect) for p in nb) / len(nb) if (u, v) in rect else 1.0
+            assert abs(phi[u, v] - expect) < 1e-14, (size, u, v)
+
+
+def test_css_size_edges():
+    rng = np.random.default_rng(9)
+    k = rng.standard_normal((20, 1, 8))
+    # 1x1 grid: no neighbour at any size
+    for size in (5, 9):
+        assert oracle.css_phi(k, frames_of((4, 1, 1)), size=size)[0][4] == 0.0
+    # a 1x4 strip with a 9x9 kernel: every other cell of the strip is a neighbour
+    k2 = np.zeros((4, 1, 2)); k2[:, 0] = [[1, 0], [0, 1], [1, 1], [1, -1]]
+    p = oracle.css_phi(k2, frames_of((0, 1, 4)), size=9)[0]
+    s = 1 / math.sqrt(2)
+    np.testing.assert_allclose(p, [1 - (0 + s + s) / 3, 1 - (0 + s - s) / 3, 1 - (s + s + 0) / 3,
+                                   1 - (s - s + 0) / 3], atol=1e-15)
+    # size 3 through the size argument is the method's Moore neighbourhood
+    np.testing.assert_array_equal(oracle.css_phi(k, frames_of((0, 4, 5)), size=3),
+                                  oracle.css_phi(k, frames_of((0, 4, 5))))
+
+
+# ------------------------------------------------ A_base scaled by its maximum
+
+def test_abase_max_normalisation():
+    wl = _tiny_traj(seed=3)
+    q, k, fr = wl.q, wl.k, wl.frames
+    ref = oracle.compress_layer(q, k, fr, beta=0.3)
+    nrm = oracle.compress_layer(q, k, fr, beta=0.3, abase_norm=oracle.ABASE_MAX)
+    # every head's largest A becomes exactly 1, the order of A is unchanged
+    np.testing.assert_array_equal(nrm["a"].max(axis=1), 1.0)
+    for h in range(k.shape[1]):
+        np.testing.assert_array_equal(np.argsort(nrm["a"][h], kind="stable"), np.argsort(ref["a"][h], kind="stable"))
+    # without CSS and TSG, S = A: a positive scale leaves the kept set alone
+    a = oracle.compress_layer(q, k, fr, beta=0.3, tsg_enable=0, css_enable=0)
+    b = oracle.compress_layer(q, k, fr, beta=0.3, tsg_enable=0, css_enable=0, abase_norm=oracle.ABASE_MAX)
+    np.testing.assert_array_equal(a["idx"], b["idx"])
+    # equal keys: A is uniform, so A / max A = 1 and S = 1 for every token
+    # (CSS and TSG off): the first B tokens by index
+    kk = np.repeat(k[:1], k.shape[0], axis=0)
+    u = oracle.compress_layer(q, kk, fr, beta=0.3, tsg_enable=0, css_enable=0, abase_norm=oracle.ABASE_MAX)
+    np.testing.assert_array_equal(u["s"], 1.0)
+    np.testing.assert_array_equal(u["idx"], np.tile(np.arange(u["budget"]), (k.shape[1], 1)))

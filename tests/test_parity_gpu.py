@@ -508,3 +508,63 @@ def test_variant_uniform_base(st, name):
     # uniform base prior: A = w/N for every token (the score passes are skipped)
     wl = WORKLOADS[name]()
     _run_edge(st, wl, wl.beta, base_scorer=1)
+
+
+@pytest.mark.parametrize("size", [3, 5, 7, 9])
+@pytest.mark.parametrize("name", ["uitars_3f", "traj50_4f", "tiny_ref_fp32"])
+def test_css_size_phi(st, name, size):
+    # CSS over the size x size neighbourhood (box-sum kernel), element by
+    # element against the oracle; uitars has 64-column grids
+    wl = WORKLOADS[name]()
+    q, k, v = to_device(wl)
+    sh = st.make_shape(q, k)
+    ws = st.workspace(sh, wl.frames)
+    phi = torch.empty((sh.n_kv_heads, sh.n_tokens), dtype=torch.float32, device="cuda")
+    st.stlite_spatial_saliency_size(q, k, wl.frames, size, phi, ws)
+    torch.cuda.synchronize()
+    assert st.stlite_device_status(ws) == st.STLITE_OK
+    ref = oracle.css_phi(exact64(k), wl.frames, threads=THREADS, size=size)
+    pg = phi.cpu().numpy()
+    vis = visual_mask(wl.n, wl.frames)
+    assert np.isnan(pg[:, ~vis]).all()
+    assert_within(pg[:, vis], ref[:, vis], cos_bound(ref[:, vis]), "Phi")
+
+
+def test_css_size_ragged_grids(st):
+    # 1x1, 1xW, Hx1 and odd grids separated by text, fp32 and bf16
+    rng = np.random.default_rng(44)
+    n, hq, hkv, w = 700, 8, 2, 5
+    q = rng.standard_normal((w, hq, 128), dtype=np.float32)
+    k = rng.standard_normal((n, hkv, 128), dtype=np.float32)
+    k[300:340] = k[200:240] + 0.05 * rng.standard_normal((40, hkv, 128), dtype=np.float32)
+    v = rng.standard_normal((n, hkv, 128), dtype=np.float32)
+    frames = (np.array([2, 5, 40, 200, 300, 400], np.int32), np.array([1, 1, 23, 5, 5, 17], np.int32),
+              np.array([1, 30, 1, 8, 8, 17], np.int32))
+    wl = synth.Workload("ragged_css", q, k, v, *frames, beta=0.2)
+    for dtype in ("bf16", "f32"):
+        wl.dtype = dtype
+        qd, kd, _ = to_device(wl)
+        ws = st.workspace(st.make_shape(qd, kd), wl.frames)
+        for size in (3, 5, 9):
+            phi = torch.empty((hkv, n), dtype=torch.float32, device="cuda")
+            st.stlite_spatial_saliency_size(qd, kd, wl.frames, size, phi, ws)
+            torch.cuda.synchronize()
+            ref = oracle.css_phi(exact64(kd), wl.frames, size=size)
+            vis = visual_mask(n, wl.frames)
+            assert_within(phi.cpu().numpy()[:, vis], ref[:, vis], cos_bound(ref[:, vis]), "Phi")
+
+
+@pytest.mark.parametrize("size", [5, 9])
+@pytest.mark.parametrize("name", ["traj50_4f", "tiny_ref_fp32"])
+def test_variant_css_size(st, name, size):
+    # the neighbourhood-size ablation end to end
+    wl = WORKLOADS[name]()
+    _run_edge(st, wl, wl.beta, css_size=size)
+
+
+@pytest.mark.parametrize("name", ["traj50_4f", "small_3f", "tiny_ref_fp32"])
+def test_variant_abase_max(st, name):
+    # A_base divided by its per-head maximum before Eq. 9
+    wl = WORKLOADS[name]()
+    _run_edge(st, wl, wl.beta, abase_norm=1)
+    _run_edge(st, wl, wl.beta, abase_norm=1, base_scorer=1)
