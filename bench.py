@@ -55,6 +55,7 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-decode", action="store_true", help="skip the decode-over-the-cache measurement")
     ap.add_argument("--no-variants", action="store_true", help="skip the ablation-variant step times")
+    ap.add_argument("--no-trajectory", action="store_true", help="skip the per-step trajectory sweep")
     return ap.parse_args()
 
 
@@ -520,6 +521,50 @@ def run_gpu(args):
             step(stream)
         stream.synchronize()
 
+    # ---- per-step use across the trajectory: at agent step t the prompt holds
+    # frames 0..t-1 (t * 1072 tokens), and all 28 layers are compressed once
+    # the step's prefill is done; one graph per step length
+    trajectory = None
+    if not args.no_trajectory:
+        trajectory = []
+        step_tok = GH * GW + N_TEXT
+        for t in (1, 2, 5, 10, 20, 30, 40, 50):
+            n_t = t * step_tok
+            fr = wls[0].frames
+            fs_t = stlite.FrameSpec(fr[0][:t], fr[1][:t], fr[2][:t])
+            b_t = stlite.stlite_budget(n_t, BETA)
+            prm_t = stlite.make_params(BETA)
+            sh_t = stlite.make_shape(qs[0], ks[0][:n_t])
+            assert stlite.stlite_workspace_size(sh_t, fs_t, prm_t) <= ws_layer
+            ix_t = torch.empty((L, HKV, b_t), dtype=torch.int32, device=dev)
+            io_t = [(qs[l], ks[l][:n_t], vs[l][:n_t], kos[l][:b_t], vos[l][:b_t], ix_t[l]) for l in range(L)]
+
+            def tstep(st=None, io_t=io_t, fs_t=fs_t, prm_t=prm_t):
+                stlite.stlite_compress_layers(io_t, fs_t, prm_t, ws, st)
+            with torch.cuda.stream(stream):
+                for _ in range(2):
+                    tstep(stream)
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                tstep(stream)
+            a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            reps = max(5, min(20, args.steps))
+            with torch.cuda.stream(stream):
+                for _ in range(2):
+                    g.replay()
+                a0.record(stream)
+                for _ in range(reps):
+                    g.replay()
+                a1.record(stream)
+            torch.cuda.synchronize()
+            assert stlite.stlite_device_status(ws, stream) == stlite.STLITE_OK
+            t_ms = a0.elapsed_time(a1) / reps
+            trajectory.append(dict(frames=t, n_tokens=n_t, budget=b_t, ms_per_step=t_ms,
+                                   value=n_t * L / (t_ms * 1e-3), unit=UNIT))
+        with torch.cuda.stream(stream):
+            step(stream)
+        stream.synchronize()
+
     # ---- consumer: one decode step (a query row per layer) over the full and
     # the compressed caches of all layers, each step one CUDA graph
     decode = None
@@ -675,7 +720,7 @@ def run_gpu(args):
                     roofline=roof, kernels=kernels, gpu_launches=per_step_launches * args.steps,
                     clocks=dict(sm_mhz=clk["sm_mhz"], sm_max_mhz=clk["sm_max_mhz"], reasons=clk["reasons"],
                                 samples=clk["samples"]),
-                    e2e=e2e, cpu_baseline=cpu, decode=decode, variants=variants)
+                    e2e=e2e, cpu_baseline=cpu, decode=decode, variants=variants, trajectory=trajectory)
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
