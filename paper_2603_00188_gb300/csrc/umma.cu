@@ -230,26 +230,39 @@ __global__ void __launch_bounds__(kThreads, 1)
           float m[8];
 #pragma unroll
           for (int i = 0; i < 8; ++i) m[i] = -CUDART_INF_F;
-#pragma unroll 1
-          for (int c = 0; c < 4; ++c) {
-            float v[64];
-            tmem_ld64(tbase + c * 64, v);
+          auto reduce = [&](const uint32_t (&v)[64], int c) {
             const float4* r4 = reinterpret_cast<const float4*>(rg + c * 64);
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
               const float4 r = r4[i];
+              const float v0 = __uint_as_float(v[4 * i]), v1 = __uint_as_float(v[4 * i + 1]);
+              const float v2 = __uint_as_float(v[4 * i + 2]), v3 = __uint_as_float(v[4 * i + 3]);
               float p0, p1, p2, p3;
               if (METRIC == kTsgNegL2) {
-                fma2(v[4 * i], v[4 * i + 1], 2.f, 2.f, r.x, r.y, p0, p1);
-                fma2(v[4 * i + 2], v[4 * i + 3], 2.f, 2.f, r.z, r.w, p2, p3);
+                fma2(v0, v1, 2.f, 2.f, r.x, r.y, p0, p1);
+                fma2(v2, v3, 2.f, 2.f, r.z, r.w, p2, p3);
               } else {
-                mul2(v[4 * i], v[4 * i + 1], r.x, r.y, p0, p1);
-                mul2(v[4 * i + 2], v[4 * i + 3], r.z, r.w, p2, p3);
+                mul2(v0, v1, r.x, r.y, p0, p1);
+                mul2(v2, v3, r.z, r.w, p2, p3);
               }
               m[(2 * i) & 7] = max3(m[(2 * i) & 7], p0, p1);
               m[(2 * i + 1) & 7] = max3(m[(2 * i + 1) & 7], p2, p3);
             }
-          }
+          };
+          // two register sets: chunk c + 1 loads while chunk c is reduced
+          uint32_t b0[64], b1[64];
+          tmem_ld64_issue(tbase, b0);
+          tmem_ld64_wait(b0);
+          tmem_ld64_issue(tbase + 64, b1);
+          reduce(b0, 0);
+          tmem_ld64_wait_after(b1, m);
+          tmem_ld64_issue(tbase + 128, b0);
+          reduce(b1, 1);
+          tmem_ld64_wait_after(b0, m);
+          tmem_ld64_issue(tbase + 192, b1);
+          reduce(b0, 2);
+          tmem_ld64_wait_after(b1, m);
+          reduce(b1, 3);
           mx = fmaxf(fmaxf(max3(m[0], m[1], m[2]), max3(m[3], m[4], m[5])), fmaxf(m[6], m[7]));
         } else {
           // ragged stage: columns past the frame carry rn = NaN, ignored by fmaxf

@@ -91,7 +91,9 @@ def test_entry_points_reject_before_launch(st):
     mis = P(0x10008)          # not 16-byte aligned
     assert lib.stlite_score(ctypes.byref(sh), None, good, good, good, need, None) == st.STLITE_EINVAL
     assert lib.stlite_score(ctypes.byref(sh), mis, good, good, good, need, None) == st.STLITE_EINVAL
-    assert lib.stlite_score(ctypes.byref(sh), good, good, good, good, need - 1, None) == st.STLITE_EWORKSPACE
+    # stlite_score takes no frames: its workspace is the frame-less size
+    need_score = st.stlite_workspace_size(sh, st.FrameSpec([], [], []), prm)
+    assert lib.stlite_score(ctypes.byref(sh), good, good, good, good, need_score - 1, None) == st.STLITE_EWORKSPACE
     assert lib.stlite_gate_frames(ctypes.byref(sh), ctypes.byref(fr.c), good, 0, good, good, good, good,
                                   need, None) == st.STLITE_EINVAL
     bad_prm = st.make_params(beta=0.0)
