@@ -172,35 +172,46 @@ __global__ void __launch_bounds__(kDecThreads, 2) k_decode_split(const T* __rest
 // ---------------------------------------------------------------------------
 // bf16 caches: key and value tiles of 64 cached rows stream through a ring of
 // shared-memory stages by TMA (128-byte swizzle, the layout of the tensor-core
-// kernels); warp 16 issues the copies, warps 0-15 consume each tile in three
-// phases separated by a named barrier, each key and value element read once
-// per tile:
-//   1. scores: thread (row t = tid % 64, slice sl = tid / 64) dots dimensions
-//      16 sl .. 16 sl + 15 of its row's key with every query head of the
-//      group (a warp's lanes share the slice, so query reads are broadcasts);
-//      the eight slices' partial scores are summed through shared memory;
-//   2. online softmax: warp w updates (max, sum) of query head w and turns
-//      the tile's scores into probabilities;
-//   3. values: thread (dimension pair dp = tid % 64, row slice ts = tid / 64)
-//      accumulates p * v over rows ts, ts + 8, ... for every query head; the
-//      eight row slices are summed once, after the last tile.
-// Scores and probabilities are kept row-slice-major: entry (g, t) at
-// g * 64 + (t % 8) * 8 + t / 8.
-// Every mbarrier wait is made by one thread and its outcome shared through
-// shared memory after the named barrier, so all consumer warps take the same
-// path and always meet at every barrier.
+// kernels).  The sixteen warps form four independent groups of four: group i
+// takes tiles i, i + 4, ... (so it always uses stage i), issues its own
+// copies (the next tile's as soon as the current one is consumed), keeps its
+// own online (max, sum) per query head and meets only its own named barrier,
+// so the groups' copy and barrier latencies overlap one another's work.  A
+// group consumes a tile in three phases:
+//   1. scores: thread (row t = id % 64, half sl = id / 64) dots dimensions
+//      64 sl .. 64 sl + 63 of its row's key with every query head of the
+//      group (a warp's lanes share the half, so query reads are broadcasts);
+//      the two halves' partial scores are summed through shared memory;
+//   2. online softmax: warp w of the group updates (max, sum) of query heads
+//      w, w + 4, ... and turns the tile's scores into probabilities;
+//   3. values: thread (dimension pair dp = id % 64, row parity ts = id / 64)
+//      accumulates p * v over rows ts, ts + 2, ... for every query head.
+// Scores and probabilities are kept parity-major: entry (g, t) at
+// g * 64 + (t % 2) * 32 + t / 2.  The groups and row parities are merged
+// once, after the last tile.  Every mbarrier wait is made by the thread that
+// issued the copy and its outcome shared through shared memory after the
+// group's barrier, so the group's warps take the same path and always meet
+// there.
 constexpr int kDecTile = 64;                         // cached rows per tile
 constexpr int kDecStages = 4;
 constexpr int kDecHalf = kDecTile * 128;             // one 64-dimension half of a tile: 64 rows x 128 B
 constexpr int kDecStageBytes = 4 * kDecHalf;         // keys (two halves), then values (two halves)
-constexpr int kDecConsumers = 512;                   // warps 0-15
-constexpr int kDecQGroups = kDecConsumers / 64;      // query groups of 64 threads
-constexpr int kDecTmaThreads = kDecConsumers + 32;   // + warp 16 (copies)
+constexpr int kDecGroups = 4;                        // consumer groups (one stage each)
+constexpr int kDecGroupThreads = 128;
+constexpr int kDecConsumers = kDecGroups * kDecGroupThreads;  // warps 0-15
+constexpr int kDecTmaThreads = kDecConsumers;
 constexpr int kDecQPitch = kD + 4;                   // floats per staged query row
+// per group: ps [GM][64], part [2][GM][64], m, l, a [GM], the wait flag (+3 pad)
+__host__ __device__ constexpr int dec_group_floats(int gm) { return 3 * gm * kDecTile + 3 * gm + 4; }
 constexpr int kDecTmaSmem = 1024 + kDecStages * kDecStageBytes + kDecMaxG * kDecQPitch * 4 +
-                            9 * kDecMaxG * kDecTile * 4 + 3 * kDecMaxG * 4 + 128;
+                            kDecGroups * dec_group_floats(kDecMaxG) * 4 + 128;
+static_assert(kDecStages == kDecGroups, "group i always uses stage i");
+static_assert(kDecGroups * 2 * kDecMaxG * kD * 4 <= kDecStages * kDecStageBytes, "merge buffer fits the stages");
 
-__device__ __forceinline__ void consumer_sync() { asm volatile("bar.sync 1, 512;" ::: "memory"); }
+__device__ __forceinline__ void group_sync(int gi) {
+  asm volatile("bar.sync %0, 128;" ::"r"(1 + gi) : "memory");
+}
+__device__ __forceinline__ void consumer_sync() { asm volatile("bar.sync 5, 512;" ::: "memory"); }
 
 // Element e (0..127) of row t of a swizzled [2][64][128 B] tile.
 __device__ __forceinline__ uint32_t tile_off(int t, int e) {
@@ -218,121 +229,129 @@ __global__ void __launch_bounds__(kDecTmaThreads, 1)
   const int split = blockIdx.x, h = blockIdx.y, r = blockIdx.z;
   const int G = hq / hkv;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  constexpr int GF = dec_group_floats(GM);
   float* qs = reinterpret_cast<float*>(sm + kDecStages * kDecStageBytes);  // [GM][kDecQPitch]
-  float* ps = qs + GM * kDecQPitch;                                           // [GM][64]
-  float* part = ps + GM * kDecTile;                                          // [8][GM][64]
-  float* st_m = part + 8 * GM * kDecTile;
-  float* st_l = st_m + GM;
-  float* st_a = st_l + GM;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(st_a + GM + (GM & 1));      // 8-byte aligned
-  const uint32_t b_full = smem_u32(&bars[0]), b_empty = smem_u32(&bars[kDecStages]);
-  volatile uint32_t* flag = reinterpret_cast<volatile uint32_t*>(&bars[2 * kDecStages]);
-  volatile uint32_t* abort_flag = flag + 1;
+  float* gscr = qs + GM * kDecQPitch;                                        // [groups][GF]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(gscr + kDecGroups * GF);     // 8-byte aligned
+  const uint32_t b_full = smem_u32(&bars[0]);
+  volatile uint32_t* abort_flag = reinterpret_cast<volatile uint32_t*>(&bars[kDecStages]);
   const uint32_t s0 = smem_u32(sm);
   const int j0 = min(n, split * per), j1 = min(n, j0 + per);
   const int ntiles = (j1 - j0 + kDecTile - 1) / kDecTile;
 
   if (tid == 0) {
-    for (int i = 0; i < kDecStages; ++i) {
-      mbar_init(b_full + 8 * i, 1);
-      mbar_init(b_empty + 8 * i, 1);
-    }
+    for (int i = 0; i < kDecStages; ++i) mbar_init(b_full + 8 * i, 1);
     *abort_flag = 0u;
     fence_mbar_init();
   }
-  // query rows of the group, times log2(e)/sqrt(d); running (max, sum)
+  // query rows of the group, times log2(e)/sqrt(d); every group's running
+  // (max, sum)
   const float scale = kDecLog2e * rsqrtf((float)kD);
   for (int e = tid; e < G * kD; e += kDecTmaThreads)
     qs[(e / kD) * kDecQPitch + e % kD] = __bfloat162float(q[((size_t)r * hq + h * G) * kD + e]) * scale;
-  for (int g = tid; g < GM; g += kDecTmaThreads) {
-    st_m[g] = -CUDART_INF_F;
-    st_l[g] = 0.f;
+  for (int e = tid; e < kDecGroups * GM; e += kDecTmaThreads) {
+    float* st = gscr + (e / GM) * GF + 3 * GM * kDecTile;
+    st[e % GM] = -CUDART_INF_F;  // m
+    st[GM + e % GM] = 0.f;       // l
   }
   __syncthreads();
-
-  if (warp == kDecConsumers / 32) {
-    if (lane == 0) {
-      int issued[kDecStages] = {0, 0, 0, 0};
-      for (int it = 0; it < ntiles; ++it) {
-        const int s = it % kDecStages;
-        if (!mbar_wait(b_empty + 8 * s, ((uint32_t)(it / kDecStages) & 1u) ^ 1u, err, abort_flag)) break;
-        const uint32_t dst = s0 + s * kDecStageBytes;
-        const int row = j0 + it * kDecTile;
-        mbar_arrive_expect_tx(b_full + 8 * s, (uint32_t)kDecStageBytes);
-        tma_load_3d(dst, &kmap, b_full + 8 * s, 0, h, row);
-        tma_load_3d(dst + kDecHalf, &kmap, b_full + 8 * s, 64, h, row);
-        tma_load_3d(dst + 2 * kDecHalf, &vmap, b_full + 8 * s, 0, h, row);
-        tma_load_3d(dst + 3 * kDecHalf, &vmap, b_full + 8 * s, 64, h, row);
-        ++issued[s];
-      }
-      if (*abort_flag)  // drain copies still in flight before the CTA exits
-        for (int s = 0; s < kDecStages; ++s)
-          if (issued[s]) mbar_wait_drain(b_full + 8 * s, (uint32_t)(issued[s] - 1) & 1u);
-    }
-    return;
-  }
+  (void)warp;
+  (void)lane;
+  // keys and values of tile it into stage it % kDecStages (one thread)
+  auto issue = [&](int it) {
+    const int s = it % kDecStages;
+    const uint32_t dst = s0 + s * kDecStageBytes;
+    const int row = j0 + it * kDecTile;
+    mbar_arrive_expect_tx(b_full + 8 * s, (uint32_t)kDecStageBytes);
+    tma_load_3d(dst, &kmap, b_full + 8 * s, 0, h, row);
+    tma_load_3d(dst + kDecHalf, &kmap, b_full + 8 * s, 64, h, row);
+    tma_load_3d(dst + 2 * kDecHalf, &vmap, b_full + 8 * s, 0, h, row);
+    tma_load_3d(dst + 3 * kDecHalf, &vmap, b_full + 8 * s, 64, h, row);
+  };
 
   // ---------------------------------------------------------- consumers
-  float o[GM][2];  // dimensions 2*dp, 2*dp + 1 over this thread's row slice
+  const int gi = tid / kDecGroupThreads, id = tid % kDecGroupThreads, wl = id >> 5;
+  if (id == 0 && gi < ntiles) issue(gi);
+  float* ps = gscr + gi * GF;              // [GM][64] scores, then probabilities
+  float* part = ps + GM * kDecTile;        // [2][GM][64] half-row partial scores
+  float* st_m = part + 2 * GM * kDecTile;  // running max, sum, and this tile's rescale
+  float* st_l = st_m + GM;
+  float* st_a = st_l + GM;
+  volatile uint32_t* flag = reinterpret_cast<volatile uint32_t*>(st_a + GM);
+  float o[GM][2];  // dimensions 2*dp, 2*dp + 1 over this thread's row parity
 #pragma unroll
   for (int g = 0; g < GM; ++g) o[g][0] = o[g][1] = 0.f;
-  const int dp = tid & 63, ts = tid >> 6;   // phase 3 roles
-  const int t1 = tid & 63, sl = tid >> 6;   // phase 1 roles
-  for (int it = 0; it < ntiles; ++it) {
+  const int dp = id & 63, ts = id >> 6;   // phase 3 roles
+  const int t1 = id & 63, sl = id >> 6;   // phase 1 roles
+  for (int it = gi; it < ntiles; it += kDecGroups) {
     const int s = it % kDecStages;
-    if (tid == 0) *flag = mbar_wait(b_full + 8 * s, (uint32_t)(it / kDecStages) & 1u, err, abort_flag) ? 1u : 0u;
-    consumer_sync();
-    if (*flag == 0u) break;  // the same value for every consumer thread
+    const uint32_t par = (uint32_t)(it / kDecStages) & 1u;
+    if (id == 0) {
+      const bool ok = mbar_wait(b_full + 8 * s, par, err, abort_flag);
+      if (!ok) mbar_wait_drain(b_full + 8 * s, par);  // the copy in flight ends before the CTA does
+      *flag = ok ? 1u : 0u;
+    }
+    group_sync(gi);
+    if (*flag == 0u) break;  // the same value for every thread of the group
     const uint8_t* kt = sm + s * kDecStageBytes;
     const uint8_t* vt = kt + 2 * kDecHalf;
     const int base = j0 + it * kDecTile;
-    // phase 1: row t1, dimensions 16 sl .. 16 sl + 15, every query head
+    // phase 1: row t1, dimensions 64 sl .. 64 sl + 63 in two quarters of
+    // 32, every query head
     {
-      float kf[16];
+      float acc[GM];
 #pragma unroll
-      for (int m = 0; m < 2; ++m) {
-        const uint4 u = *reinterpret_cast<const uint4*>(kt + tile_off(t1, 16 * sl + 8 * m));
-        const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+      for (int g = 0; g < GM; ++g) acc[g] = 0.f;
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          kf[8 * m + 2 * i] = __uint_as_float(w4[i] << 16);
-          kf[8 * m + 2 * i + 1] = __uint_as_float(w4[i] & 0xffff0000u);
-        }
-      }
+      for (int qq = 0; qq < 2; ++qq) {
+        const int d0 = 64 * sl + 32 * qq;
+        float kf[32];
 #pragma unroll
-      for (int g = 0; g < GM; ++g) {
-        if (g < G) {
-          float x0 = 0.f, x1 = 0.f;
+        for (int m = 0; m < 4; ++m) {
+          const uint4 u = *reinterpret_cast<const uint4*>(kt + tile_off(t1, d0 + 8 * m));
+          const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            const float4 a = *reinterpret_cast<const float4*>(qs + g * kDecQPitch + 16 * sl + 4 * j);
-            float& x = (j & 1) ? x1 : x0;
-            x = fmaf(kf[4 * j], a.x, fmaf(kf[4 * j + 1], a.y, fmaf(kf[4 * j + 2], a.z, fmaf(kf[4 * j + 3], a.w, x))));
+          for (int i = 0; i < 4; ++i) {
+            kf[8 * m + 2 * i] = __uint_as_float(w4[i] << 16);
+            kf[8 * m + 2 * i + 1] = __uint_as_float(w4[i] & 0xffff0000u);
           }
-          part[(sl * GM + g) * kDecTile + t1] = x0 + x1;
+        }
+#pragma unroll
+        for (int g = 0; g < GM; ++g) {
+          if (g < G) {
+            float x0 = 0.f, x1 = 0.f;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              const float4 a = *reinterpret_cast<const float4*>(qs + g * kDecQPitch + d0 + 4 * j);
+              float& x = (j & 1) ? x1 : x0;
+              x = fmaf(kf[4 * j], a.x, fmaf(kf[4 * j + 1], a.y, fmaf(kf[4 * j + 2], a.z, fmaf(kf[4 * j + 3], a.w, x))));
+            }
+            acc[g] += x0 + x1;
+          }
         }
       }
-    }
-    consumer_sync();
-    // phase 1b: sum the slices; scores of rows past the range are -inf
-    for (int e = tid; e < G * kDecTile; e += kDecConsumers) {
-      const int g = e / kDecTile, t = e % kDecTile;
-      float x = 0.f;
 #pragma unroll
-      for (int q8 = 0; q8 < 8; ++q8) x += part[(q8 * GM + g) * kDecTile + t];
-      ps[g * kDecTile + (t & 7) * 8 + (t >> 3)] = base + t < j1 ? x : -CUDART_INF_F;
+      for (int g = 0; g < GM; ++g)
+        if (g < G) part[(sl * GM + g) * kDecTile + t1] = acc[g];
     }
-    consumer_sync();
-    // phase 2: online softmax of query head g over the tile's 64 rows
-    for (int g = warp; g < G; g += kDecConsumers / 32) {
-      const int i0 = (lane & 7) * 8 + (lane >> 3), i1 = i0 + 4;  // rows lane and lane + 32
-      const float x0 = ps[g * kDecTile + i0], x1 = ps[g * kDecTile + i1];
+    group_sync(gi);
+    // phase 1b: sum the halves; scores of rows past the range are -inf
+    for (int e = id; e < G * kDecTile; e += kDecGroupThreads) {
+      const int g = e / kDecTile, t = e % kDecTile;
+      const float x = part[g * kDecTile + t] + part[(GM + g) * kDecTile + t];
+      ps[g * kDecTile + (t & 1) * 32 + (t >> 1)] = base + t < j1 ? x : -CUDART_INF_F;
+    }
+    group_sync(gi);
+    // phase 2: online softmax of query head g over the tile's 64 rows (any
+    // two positions per lane: the order of rows does not matter here)
+    for (int g = wl; g < G; g += kDecGroupThreads / 32) {
+      const float x0 = ps[g * kDecTile + lane], x1 = ps[g * kDecTile + lane + 32];
       const float mo = st_m[g];
       const float mn = fmaxf(mo, warp_max(fmaxf(x0, x1)));
       const float p0 = weight(x0, mn), p1 = weight(x1, mn);
       const float sum = warp_sum(p0 + p1);
-      ps[g * kDecTile + i0] = p0;
-      ps[g * kDecTile + i1] = p1;
+      ps[g * kDecTile + lane] = p0;
+      ps[g * kDecTile + lane + 32] = p1;
       if (lane == 0) {
         const float a = weight(mo, mn);
         st_a[g] = a;
@@ -340,51 +359,76 @@ __global__ void __launch_bounds__(kDecTmaThreads, 1)
         st_m[g] = mn;
       }
     }
-    consumer_sync();
-    // phase 3: rows ts + 8 k, dimensions 2 dp and 2 dp + 1, every query head
-    {
-      float2 vv[8];
+    group_sync(gi);
+    // phase 3: rows ts + 2 k, dimensions 2 dp and 2 dp + 1, every query head,
+    // in two halves of 16 rows
 #pragma unroll
-      for (int k = 0; k < 8; ++k) {
-        const uint32_t w = *reinterpret_cast<const uint32_t*>(vt + tile_off(ts + 8 * k, 2 * dp));
+    for (int g = 0; g < GM; ++g)
+      if (g < G) {
+        const float a = st_a[g];
+        o[g][0] *= a;
+        o[g][1] *= a;
+      }
+#pragma unroll
+    for (int hh = 0; hh < 2; ++hh) {
+      float2 vv[16];
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {
+        const uint32_t w = *reinterpret_cast<const uint32_t*>(vt + tile_off(ts + 2 * (16 * hh + k), 2 * dp));
         vv[k] = make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
       }
 #pragma unroll
       for (int g = 0; g < GM; ++g) {
         if (g < G) {
-          const float a = st_a[g];
-          const float4 pa = *reinterpret_cast<const float4*>(ps + g * kDecTile + ts * 8);
-          const float4 pb = *reinterpret_cast<const float4*>(ps + g * kDecTile + ts * 8 + 4);
-          const float pp[8] = {pa.x, pa.y, pa.z, pa.w, pb.x, pb.y, pb.z, pb.w};
-          float y0 = o[g][0] * a, y1 = o[g][1] * a;
+          float y0 = o[g][0], y1 = o[g][1], z0 = 0.f, z1 = 0.f;
 #pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            y0 = fmaf(pp[k], vv[k].x, y0);
-            y1 = fmaf(pp[k], vv[k].y, y1);
+          for (int k4 = 0; k4 < 4; ++k4) {
+            const float4 pk = *reinterpret_cast<const float4*>(ps + g * kDecTile + ts * 32 + 16 * hh + 4 * k4);
+            y0 = fmaf(pk.x, vv[4 * k4].x, y0);
+            y1 = fmaf(pk.x, vv[4 * k4].y, y1);
+            z0 = fmaf(pk.y, vv[4 * k4 + 1].x, z0);
+            z1 = fmaf(pk.y, vv[4 * k4 + 1].y, z1);
+            y0 = fmaf(pk.z, vv[4 * k4 + 2].x, y0);
+            y1 = fmaf(pk.z, vv[4 * k4 + 2].y, y1);
+            z0 = fmaf(pk.w, vv[4 * k4 + 3].x, z0);
+            z1 = fmaf(pk.w, vv[4 * k4 + 3].y, z1);
           }
-          o[g][0] = y0;
-          o[g][1] = y1;
+          o[g][0] = y0 + z0;
+          o[g][1] = y1 + z1;
         }
       }
     }
-    consumer_sync();  // every consumer is done with this stage
-    if (tid == 0) mbar_arrive(b_empty + 8 * s);
+    // the group is done with this stage: its reads are ordered before the
+    // next copy into it
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    group_sync(gi);
+    if (id == 0 && it + kDecGroups < ntiles) issue(it + kDecGroups);
   }
-  // sum the eight row slices (through the first stage buffer, now idle),
-  // then write this split's partial per query head
-  float* red = reinterpret_cast<float*>(sm);  // [8 slices][GM][128]
+  // merge the groups and row parities (through the stage buffers, idle once
+  // every group has finished), then write this split's partial per query head
+  consumer_sync();
+  float* red = reinterpret_cast<float*>(sm);  // [groups][2 parities][GM][128]
 #pragma unroll
   for (int g = 0; g < GM; ++g)
-    if (g < G) *reinterpret_cast<float2*>(red + ((size_t)ts * GM + g) * kD + 2 * dp) = make_float2(o[g][0], o[g][1]);
+    if (g < G)
+      *reinterpret_cast<float2*>(red + (((size_t)gi * 2 + ts) * GM + g) * kD + 2 * dp) = make_float2(o[g][0], o[g][1]);
   consumer_sync();
   for (int e = tid; e < G * kD; e += kDecConsumers) {
     const int g = e / kD, c = e % kD;
-    float x = 0.f;
+    float M = -CUDART_INF_F;
 #pragma unroll
-    for (int q8 = 0; q8 < 8; ++q8) x += red[((size_t)q8 * GM + g) * kD + c];
+    for (int q4 = 0; q4 < kDecGroups; ++q4) M = fmaxf(M, gscr[q4 * GF + 3 * GM * kDecTile + g]);
+    float O = 0.f, L = 0.f;
+#pragma unroll
+    for (int q4 = 0; q4 < kDecGroups; ++q4) {
+      const float* st = gscr + q4 * GF + 3 * GM * kDecTile;
+      const float w = weight(st[g], M);
+      L = fmaf(st[GM + g], w, L);
+      O = fmaf(red[(((size_t)q4 * 2 + 0) * GM + g) * kD + c] + red[(((size_t)q4 * 2 + 1) * GM + g) * kD + c], w, O);
+    }
     const size_t slot = ((size_t)split * gridDim.z + r) * hq + h * G + g;
-    part_o[slot * kD + c] = x;
-    if (c == 0) part_ml[slot] = make_float2(st_m[g], st_l[g]);
+    part_o[slot * kD + c] = O;
+    if (c == 0) part_ml[slot] = make_float2(M, L);
   }
 }
 
