@@ -173,45 +173,42 @@ __global__ void __launch_bounds__(kDecThreads, 2) k_decode_split(const T* __rest
 // bf16 caches: key and value tiles of 64 cached rows stream through a ring of
 // shared-memory stages by TMA (128-byte swizzle, the layout of the tensor-core
 // kernels).  The sixteen warps form four independent groups of four: group i
-// takes tiles i, i + 4, ... (so it always uses stage i), issues its own
-// copies (the next tile's as soon as the current one is consumed), keeps its
-// own online (max, sum) per query head and meets only its own named barrier,
-// so the groups' copy and barrier latencies overlap one another's work.  A
-// group consumes a tile in three phases:
-//   1. scores: thread (row t = id % 64, half sl = id / 64) dots dimensions
-//      64 sl .. 64 sl + 63 of its row's key with every query head of the
-//      group (a warp's lanes share the half, so query reads are broadcasts);
-//      the two halves' partial scores are summed through shared memory;
-//   2. online softmax: warp w of the group updates (max, sum) of query heads
-//      w, w + 4, ... and turns the tile's scores into probabilities;
-//   3. values: thread (dimension pair dp = id % 64, row parity ts = id / 64)
-//      accumulates p * v over rows ts, ts + 2, ... for every query head.
-// Scores and probabilities are kept parity-major: entry (g, t) at
-// g * 64 + (t % 2) * 32 + t / 2.  The groups and row parities are merged
-// once, after the last tile.  Every mbarrier wait is made by the thread that
-// issued the copy and its outcome shared through shared memory after the
-// group's barrier, so the group's warps take the same path and always meet
-// there.
+// takes tiles i, i + 4, ... (so it always uses stage i) and issues its own
+// copies, the next tile's as soon as the current one is consumed.  Warp j of
+// a group owns rows 16 j .. 16 j + 15 of every tile and keeps its own online
+// (max, sum) per query head, so a tile needs one group barrier (the release
+// of its stage).  Both products run on the warp's tensor cores (mma.sync
+// m16n8k16, bf16 inputs, fp32 accumulation):
+//   scores  S (16 rows x 8 heads) = K (16 x 128) Q^T, the query fragments
+//           held in registers for the whole kernel, the key fragments read
+//           from the swizzled stage by ldmatrix;
+//   values  O^T (128 dims x 8 heads) += V^T P^T, V^T read by ldmatrix.trans,
+//           P passed through shared memory as P = hi + lo, two bf16 parts
+//           (about 16 bits of the fp32 probabilities).
+// The sixteen warps' states merge once, after the last tile.  Every mbarrier
+// wait is made by the thread that issued the copy and its outcome shared
+// through shared memory after the group's barrier, so the group's warps take
+// the same path and always meet there.
 constexpr int kDecTile = 64;                         // cached rows per tile
 constexpr int kDecStages = 4;
 constexpr int kDecHalf = kDecTile * 128;             // one 64-dimension half of a tile: 64 rows x 128 B
 constexpr int kDecStageBytes = 4 * kDecHalf;         // keys (two halves), then values (two halves)
 constexpr int kDecGroups = 4;                        // consumer groups (one stage each)
 constexpr int kDecGroupThreads = 128;
-constexpr int kDecConsumers = kDecGroups * kDecGroupThreads;  // warps 0-15
-constexpr int kDecTmaThreads = kDecConsumers;
-constexpr int kDecQPitch = kD + 4;                   // floats per staged query row
-// per group: ps [GM][64], part [2][GM][64], m, l, a [GM], the wait flag (+3 pad)
-__host__ __device__ constexpr int dec_group_floats(int gm) { return 3 * gm * kDecTile + 3 * gm + 4; }
-constexpr int kDecTmaSmem = 1024 + kDecStages * kDecStageBytes + kDecMaxG * kDecQPitch * 4 +
-                            kDecGroups * dec_group_floats(kDecMaxG) * 4 + 128;
+constexpr int kDecMmaThreads = kDecGroups * kDecGroupThreads;
+constexpr int kDecMmaWarps = kDecMmaThreads / 32;
+// per warp: P^T as [8 NT heads][16 rows] bf16, high and low parts
+__host__ __device__ constexpr int dec_pt_bytes(int nt) { return 2 * 8 * nt * 16 * 2; }
+// stages, the warps' P^T buffers, (max, sum) of every warp and head, flags
+__host__ __device__ constexpr int dec_mma_smem(int nt) {
+  return 1024 + kDecStages * kDecStageBytes + kDecMmaWarps * dec_pt_bytes(nt) + kDecMmaWarps * 8 * nt * 8 + 128;
+}
 static_assert(kDecStages == kDecGroups, "group i always uses stage i");
-static_assert(kDecGroups * 2 * kDecMaxG * kD * 4 <= kDecStages * kDecStageBytes, "merge buffer fits the stages");
+static_assert(kDecMmaWarps * 16 * kD * 4 <= kDecStages * kDecStageBytes, "merge buffer fits the stages");
 
 __device__ __forceinline__ void group_sync(int gi) {
   asm volatile("bar.sync %0, 128;" ::"r"(1 + gi) : "memory");
 }
-__device__ __forceinline__ void consumer_sync() { asm volatile("bar.sync 5, 512;" ::: "memory"); }
 
 // Element e (0..127) of row t of a swizzled [2][64][128 B] tile.
 __device__ __forceinline__ uint32_t tile_off(int t, int e) {
@@ -219,9 +216,29 @@ __device__ __forceinline__ uint32_t tile_off(int t, int e) {
   return (uint32_t)(kb * kDecHalf + t * 128 + ((c ^ (t & 7)) << 4) + (e & 7) * 2);
 }
 
-template <int GM>
-__global__ void __launch_bounds__(kDecTmaThreads, 1)
-    k_decode_tma(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t (&a)[4]) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(a[0]), "=r"(a[1]), "=r"(a[2]), "=r"(a[3])
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_trans(uint32_t addr, uint32_t (&a)[4]) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(a[0]), "=r"(a[1]), "=r"(a[2]), "=r"(a[3])
+               : "r"(addr));
+}
+// d += a b (m16n8k16, bf16 in, fp32 accumulate)
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// NT: 8-head column tiles of the query group (1 for G <= 8, 2 for G <= 16).
+template <int NT>
+__global__ void __launch_bounds__(kDecMmaThreads, 1)
+    k_decode_mma(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
                  const __nv_bfloat16* __restrict__ q, int n, int hq, int hkv, int per, float* part_o,
                  float2* part_ml, uint32_t* err) {
   extern __shared__ uint8_t dec_raw[];
@@ -229,12 +246,14 @@ __global__ void __launch_bounds__(kDecTmaThreads, 1)
   const int split = blockIdx.x, h = blockIdx.y, r = blockIdx.z;
   const int G = hq / hkv;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  constexpr int GF = dec_group_floats(GM);
-  float* qs = reinterpret_cast<float*>(sm + kDecStages * kDecStageBytes);  // [GM][kDecQPitch]
-  float* gscr = qs + GM * kDecQPitch;                                        // [groups][GF]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(gscr + kDecGroups * GF);     // 8-byte aligned
+  const int gi = warp >> 2, wq = warp & 3, id = tid & (kDecGroupThreads - 1);
+  const int g8 = lane >> 2, t4 = lane & 3;
+  uint8_t* pt_all = sm + kDecStages * kDecStageBytes;                        // [warps][dec_pt_bytes]
+  float2* wml = reinterpret_cast<float2*>(pt_all + kDecMmaWarps * dec_pt_bytes(NT));  // [warps][8 NT]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(wml + kDecMmaWarps * 8 * NT);
   const uint32_t b_full = smem_u32(&bars[0]);
   volatile uint32_t* abort_flag = reinterpret_cast<volatile uint32_t*>(&bars[kDecStages]);
+  volatile uint32_t* flags = abort_flag + 1;  // one per group
   const uint32_t s0 = smem_u32(sm);
   const int j0 = min(n, split * per), j1 = min(n, j0 + per);
   const int ntiles = (j1 - j0 + kDecTile - 1) / kDecTile;
@@ -244,19 +263,7 @@ __global__ void __launch_bounds__(kDecTmaThreads, 1)
     *abort_flag = 0u;
     fence_mbar_init();
   }
-  // query rows of the group, times log2(e)/sqrt(d); every group's running
-  // (max, sum)
-  const float scale = kDecLog2e * rsqrtf((float)kD);
-  for (int e = tid; e < G * kD; e += kDecTmaThreads)
-    qs[(e / kD) * kDecQPitch + e % kD] = __bfloat162float(q[((size_t)r * hq + h * G) * kD + e]) * scale;
-  for (int e = tid; e < kDecGroups * GM; e += kDecTmaThreads) {
-    float* st = gscr + (e / GM) * GF + 3 * GM * kDecTile;
-    st[e % GM] = -CUDART_INF_F;  // m
-    st[GM + e % GM] = 0.f;       // l
-  }
   __syncthreads();
-  (void)warp;
-  (void)lane;
   // keys and values of tile it into stage it % kDecStages (one thread)
   auto issue = [&](int it) {
     const int s = it % kDecStages;
@@ -268,167 +275,155 @@ __global__ void __launch_bounds__(kDecTmaThreads, 1)
     tma_load_3d(dst + 2 * kDecHalf, &vmap, b_full + 8 * s, 0, h, row);
     tma_load_3d(dst + 3 * kDecHalf, &vmap, b_full + 8 * s, 64, h, row);
   };
-
-  // ---------------------------------------------------------- consumers
-  const int gi = tid / kDecGroupThreads, id = tid % kDecGroupThreads, wl = id >> 5;
   if (id == 0 && gi < ntiles) issue(gi);
-  float* ps = gscr + gi * GF;              // [GM][64] scores, then probabilities
-  float* part = ps + GM * kDecTile;        // [2][GM][64] half-row partial scores
-  float* st_m = part + 2 * GM * kDecTile;  // running max, sum, and this tile's rescale
-  float* st_l = st_m + GM;
-  float* st_a = st_l + GM;
-  volatile uint32_t* flag = reinterpret_cast<volatile uint32_t*>(st_a + GM);
-  float o[GM][2];  // dimensions 2*dp, 2*dp + 1 over this thread's row parity
+
+  // B fragments of the scores: query head 8 nt + g8 (zero past the group),
+  // dimensions 16 ks + 2 t4 + {0, 1} and + 8
+  uint32_t qb[8][NT][2];
 #pragma unroll
-  for (int g = 0; g < GM; ++g) o[g][0] = o[g][1] = 0.f;
-  const int dp = id & 63, ts = id >> 6;   // phase 3 roles
-  const int t1 = id & 63, sl = id >> 6;   // phase 1 roles
+  for (int nt = 0; nt < NT; ++nt) {
+    const int head = 8 * nt + g8;
+    const uint32_t* qr = reinterpret_cast<const uint32_t*>(q + ((size_t)r * hq + h * G + (head < G ? head : 0)) * kD);
+#pragma unroll
+    for (int ks = 0; ks < 8; ++ks) {
+      qb[ks][nt][0] = head < G ? __ldg(qr + 8 * ks + t4) : 0u;
+      qb[ks][nt][1] = head < G ? __ldg(qr + 8 * ks + 4 + t4) : 0u;
+    }
+  }
+  const float scale = kDecLog2e * rsqrtf((float)kD);
+  // running state of heads 8 nt + 2 t4 + e; O^T fragments: o[mt][nt][j] is
+  // dimension 16 mt + g8 + 8 (j >> 1), head 8 nt + 2 t4 + (j & 1)
+  float m[NT][2], l[NT][2], o[8][NT][4];
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt) {
+    m[nt][0] = m[nt][1] = -CUDART_INF_F;
+    l[nt][0] = l[nt][1] = 0.f;
+#pragma unroll
+    for (int mt = 0; mt < 8; ++mt) o[mt][nt][0] = o[mt][nt][1] = o[mt][nt][2] = o[mt][nt][3] = 0.f;
+  }
+  uint8_t* pt = pt_all + warp * dec_pt_bytes(NT);  // hi at 0, lo at half
+  __nv_bfloat16* pt_hi = reinterpret_cast<__nv_bfloat16*>(pt);
+  __nv_bfloat16* pt_lo = pt_hi + 8 * NT * 16;
+  const int r0 = 16 * wq;
+
   for (int it = gi; it < ntiles; it += kDecGroups) {
     const int s = it % kDecStages;
     const uint32_t par = (uint32_t)(it / kDecStages) & 1u;
     if (id == 0) {
       const bool ok = mbar_wait(b_full + 8 * s, par, err, abort_flag);
       if (!ok) mbar_wait_drain(b_full + 8 * s, par);  // the copy in flight ends before the CTA does
-      *flag = ok ? 1u : 0u;
+      flags[gi] = ok ? 1u : 0u;
     }
     group_sync(gi);
-    if (*flag == 0u) break;  // the same value for every thread of the group
-    const uint8_t* kt = sm + s * kDecStageBytes;
-    const uint8_t* vt = kt + 2 * kDecHalf;
+    if (flags[gi] == 0u) break;  // the same value for every thread of the group
+    const uint32_t kt = s0 + s * kDecStageBytes, vt = kt + 2 * kDecHalf;
     const int base = j0 + it * kDecTile;
-    // phase 1: row t1, dimensions 64 sl .. 64 sl + 63 in two quarters of
-    // 32, every query head
-    {
-      float acc[GM];
+    // scores of rows r0 + g8 and r0 + g8 + 8, heads 8 nt + 2 t4 + {0, 1}
+    float c[NT][4];
 #pragma unroll
-      for (int g = 0; g < GM; ++g) acc[g] = 0.f;
+    for (int nt = 0; nt < NT; ++nt) c[nt][0] = c[nt][1] = c[nt][2] = c[nt][3] = 0.f;
 #pragma unroll
-      for (int qq = 0; qq < 2; ++qq) {
-        const int d0 = 64 * sl + 32 * qq;
-        float kf[32];
+    for (int ks = 0; ks < 8; ++ks) {
+      uint32_t a[4];
+      ldsm_x4(kt + tile_off(r0 + (lane & 7) + 8 * ((lane >> 3) & 1), 16 * ks + 8 * (lane >> 4)), a);
 #pragma unroll
-        for (int m = 0; m < 4; ++m) {
-          const uint4 u = *reinterpret_cast<const uint4*>(kt + tile_off(t1, d0 + 8 * m));
-          const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+      for (int nt = 0; nt < NT; ++nt) mma_bf16_16816(c[nt], a, qb[ks][nt][0], qb[ks][nt][1]);
+    }
+    const bool va = base + r0 + g8 < j1, vb = base + r0 + g8 + 8 < j1;
+    // online softmax per head over the warp's 16 rows (log2 units)
 #pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            kf[8 * m + 2 * i] = __uint_as_float(w4[i] << 16);
-            kf[8 * m + 2 * i + 1] = __uint_as_float(w4[i] & 0xffff0000u);
-          }
+    for (int nt = 0; nt < NT; ++nt) {
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const int head = 8 * nt + 2 * t4 + e;
+        const float xa = (va && head < G) ? c[nt][e] * scale : -CUDART_INF_F;
+        const float xb = (vb && head < G) ? c[nt][2 + e] * scale : -CUDART_INF_F;
+        float mx = fmaxf(xa, xb);
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
+        const float mn = fmaxf(m[nt][e], mx);
+        const float alpha = weight(m[nt][e], mn);
+        const float pa = weight(xa, mn), pb = weight(xb, mn);
+        float sum = pa + pb;
+        sum += __shfl_xor_sync(0xffffffffu, sum, 4);
+        sum += __shfl_xor_sync(0xffffffffu, sum, 8);
+        sum += __shfl_xor_sync(0xffffffffu, sum, 16);
+        l[nt][e] = l[nt][e] * alpha + sum;
+        m[nt][e] = mn;
+#pragma unroll
+        for (int mt = 0; mt < 8; ++mt) {
+          o[mt][nt][e] *= alpha;
+          o[mt][nt][2 + e] *= alpha;
         }
-#pragma unroll
-        for (int g = 0; g < GM; ++g) {
-          if (g < G) {
-            float x0 = 0.f, x1 = 0.f;
-#pragma unroll
-            for (int j = 0; j < 8; ++j) {
-              const float4 a = *reinterpret_cast<const float4*>(qs + g * kDecQPitch + d0 + 4 * j);
-              float& x = (j & 1) ? x1 : x0;
-              x = fmaf(kf[4 * j], a.x, fmaf(kf[4 * j + 1], a.y, fmaf(kf[4 * j + 2], a.z, fmaf(kf[4 * j + 3], a.w, x))));
-            }
-            acc[g] += x0 + x1;
-          }
-        }
-      }
-#pragma unroll
-      for (int g = 0; g < GM; ++g)
-        if (g < G) part[(sl * GM + g) * kDecTile + t1] = acc[g];
-    }
-    group_sync(gi);
-    // phase 1b: sum the halves; scores of rows past the range are -inf
-    for (int e = id; e < G * kDecTile; e += kDecGroupThreads) {
-      const int g = e / kDecTile, t = e % kDecTile;
-      const float x = part[g * kDecTile + t] + part[(GM + g) * kDecTile + t];
-      ps[g * kDecTile + (t & 1) * 32 + (t >> 1)] = base + t < j1 ? x : -CUDART_INF_F;
-    }
-    group_sync(gi);
-    // phase 2: online softmax of query head g over the tile's 64 rows (any
-    // two positions per lane: the order of rows does not matter here)
-    for (int g = wl; g < G; g += kDecGroupThreads / 32) {
-      const float x0 = ps[g * kDecTile + lane], x1 = ps[g * kDecTile + lane + 32];
-      const float mo = st_m[g];
-      const float mn = fmaxf(mo, warp_max(fmaxf(x0, x1)));
-      const float p0 = weight(x0, mn), p1 = weight(x1, mn);
-      const float sum = warp_sum(p0 + p1);
-      ps[g * kDecTile + lane] = p0;
-      ps[g * kDecTile + lane + 32] = p1;
-      if (lane == 0) {
-        const float a = weight(mo, mn);
-        st_a[g] = a;
-        st_l[g] = st_l[g] * a + sum;
-        st_m[g] = mn;
+        // P^T[head][row] as hi + lo
+        const __nv_bfloat16 ha = __float2bfloat16_rn(pa), hb = __float2bfloat16_rn(pb);
+        pt_hi[head * 16 + g8] = ha;
+        pt_hi[head * 16 + g8 + 8] = hb;
+        pt_lo[head * 16 + g8] = __float2bfloat16_rn(pa - __bfloat162float(ha));
+        pt_lo[head * 16 + g8 + 8] = __float2bfloat16_rn(pb - __bfloat162float(hb));
       }
     }
-    group_sync(gi);
-    // phase 3: rows ts + 2 k, dimensions 2 dp and 2 dp + 1, every query head,
-    // in two halves of 16 rows
+    __syncwarp();
+    // B fragments of the values: P^T rows 2 t4 + {0, 1} (and + 8) of head 8 nt + g8
+    uint32_t bh[NT][2], bl[NT][2];
 #pragma unroll
-    for (int g = 0; g < GM; ++g)
-      if (g < G) {
-        const float a = st_a[g];
-        o[g][0] *= a;
-        o[g][1] *= a;
-      }
+    for (int nt = 0; nt < NT; ++nt) {
+      const int head = 8 * nt + g8;
+      bh[nt][0] = *reinterpret_cast<const uint32_t*>(pt_hi + head * 16 + 2 * t4);
+      bh[nt][1] = *reinterpret_cast<const uint32_t*>(pt_hi + head * 16 + 2 * t4 + 8);
+      bl[nt][0] = *reinterpret_cast<const uint32_t*>(pt_lo + head * 16 + 2 * t4);
+      bl[nt][1] = *reinterpret_cast<const uint32_t*>(pt_lo + head * 16 + 2 * t4 + 8);
+    }
 #pragma unroll
-    for (int hh = 0; hh < 2; ++hh) {
-      float2 vv[16];
+    for (int mt = 0; mt < 8; ++mt) {
+      uint32_t a[4];
+      ldsm_x4_trans(vt + tile_off(r0 + (lane & 7) + 8 * ((lane >> 4) & 1), 16 * mt + 8 * ((lane >> 3) & 1)), a);
 #pragma unroll
-      for (int k = 0; k < 16; ++k) {
-        const uint32_t w = *reinterpret_cast<const uint32_t*>(vt + tile_off(ts + 2 * (16 * hh + k), 2 * dp));
-        vv[k] = make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
-      }
-#pragma unroll
-      for (int g = 0; g < GM; ++g) {
-        if (g < G) {
-          float y0 = o[g][0], y1 = o[g][1], z0 = 0.f, z1 = 0.f;
-#pragma unroll
-          for (int k4 = 0; k4 < 4; ++k4) {
-            const float4 pk = *reinterpret_cast<const float4*>(ps + g * kDecTile + ts * 32 + 16 * hh + 4 * k4);
-            y0 = fmaf(pk.x, vv[4 * k4].x, y0);
-            y1 = fmaf(pk.x, vv[4 * k4].y, y1);
-            z0 = fmaf(pk.y, vv[4 * k4 + 1].x, z0);
-            z1 = fmaf(pk.y, vv[4 * k4 + 1].y, z1);
-            y0 = fmaf(pk.z, vv[4 * k4 + 2].x, y0);
-            y1 = fmaf(pk.z, vv[4 * k4 + 2].y, y1);
-            z0 = fmaf(pk.w, vv[4 * k4 + 3].x, z0);
-            z1 = fmaf(pk.w, vv[4 * k4 + 3].y, z1);
-          }
-          o[g][0] = y0 + z0;
-          o[g][1] = y1 + z1;
-        }
+      for (int nt = 0; nt < NT; ++nt) {
+        mma_bf16_16816(o[mt][nt], a, bh[nt][0], bh[nt][1]);
+        mma_bf16_16816(o[mt][nt], a, bl[nt][0], bl[nt][1]);
       }
     }
+    __syncwarp();  // P^T is rewritten by the next tile
     // the group is done with this stage: its reads are ordered before the
     // next copy into it
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     group_sync(gi);
     if (id == 0 && it + kDecGroups < ntiles) issue(it + kDecGroups);
   }
-  // merge the groups and row parities (through the stage buffers, idle once
-  // every group has finished), then write this split's partial per query head
-  consumer_sync();
-  float* red = reinterpret_cast<float*>(sm);  // [groups][2 parities][GM][128]
+  // merge the sixteen warps (through the stage buffers, idle once every
+  // group has finished), then write this split's partial per query head
+  __syncthreads();
+  float* wo = reinterpret_cast<float*>(sm);  // [warps][8 NT heads][128]
 #pragma unroll
-  for (int g = 0; g < GM; ++g)
-    if (g < G)
-      *reinterpret_cast<float2*>(red + (((size_t)gi * 2 + ts) * GM + g) * kD + 2 * dp) = make_float2(o[g][0], o[g][1]);
-  consumer_sync();
-  for (int e = tid; e < G * kD; e += kDecConsumers) {
-    const int g = e / kD, c = e % kD;
+  for (int nt = 0; nt < NT; ++nt) {
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+      const int head = 8 * nt + 2 * t4 + e;
+      if (g8 == 0) wml[warp * 8 * NT + head] = make_float2(m[nt][e], l[nt][e]);
+#pragma unroll
+      for (int mt = 0; mt < 8; ++mt) {
+        wo[((size_t)warp * 8 * NT + head) * kD + 16 * mt + g8] = o[mt][nt][e];
+        wo[((size_t)warp * 8 * NT + head) * kD + 16 * mt + g8 + 8] = o[mt][nt][2 + e];
+      }
+    }
+  }
+  __syncthreads();
+  for (int e = tid; e < G * kD; e += kDecMmaThreads) {
+    const int g = e / kD, cc = e % kD;
     float M = -CUDART_INF_F;
-#pragma unroll
-    for (int q4 = 0; q4 < kDecGroups; ++q4) M = fmaxf(M, gscr[q4 * GF + 3 * GM * kDecTile + g]);
+    for (int w = 0; w < kDecMmaWarps; ++w) M = fmaxf(M, wml[w * 8 * NT + g].x);
     float O = 0.f, L = 0.f;
-#pragma unroll
-    for (int q4 = 0; q4 < kDecGroups; ++q4) {
-      const float* st = gscr + q4 * GF + 3 * GM * kDecTile;
-      const float w = weight(st[g], M);
-      L = fmaf(st[GM + g], w, L);
-      O = fmaf(red[(((size_t)q4 * 2 + 0) * GM + g) * kD + c] + red[(((size_t)q4 * 2 + 1) * GM + g) * kD + c], w, O);
+    for (int w = 0; w < kDecMmaWarps; ++w) {
+      const float2 ml = wml[w * 8 * NT + g];
+      const float wgt = weight(ml.x, M);
+      L = fmaf(ml.y, wgt, L);
+      O = fmaf(wo[((size_t)w * 8 * NT + g) * kD + cc], wgt, O);
     }
     const size_t slot = ((size_t)split * gridDim.z + r) * hq + h * G + g;
-    part_o[slot * kD + c] = O;
-    if (c == 0) part_ml[slot] = make_float2(M, L);
+    part_o[slot * kD + cc] = O;
+    if (cc == 0) part_ml[slot] = make_float2(M, L);
   }
 }
 
@@ -517,20 +512,18 @@ cudaError_t launch_decode(DType dt, const void* q, const void* k, const void* v,
     CUtensorMap km, vm;
     if ((e = make_row_map(&km, k, n, hkv, kDecTile)) != cudaSuccess) return e;
     if ((e = make_row_map(&vm, v, n, hkv, kDecTile)) != cudaSuccess) return e;
-    auto run = [&](auto gm) {
-      constexpr int GM = decltype(gm)::value;
-      e = cudaFuncSetAttribute(k_decode_tma<GM>, cudaFuncAttributeMaxDynamicSharedMemorySize, kDecTmaSmem);
+    auto run = [&](auto nt) {
+      constexpr int NT = decltype(nt)::value;
+      e = cudaFuncSetAttribute(k_decode_mma<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize, dec_mma_smem(NT));
       if (e != cudaSuccess) return;
-      k_decode_tma<GM><<<grid, kDecTmaThreads, kDecTmaSmem, st>>>(
+      k_decode_mma<NT><<<grid, kDecMmaThreads, dec_mma_smem(NT), st>>>(
           km, vm, static_cast<const __nv_bfloat16*>(q), n, hq, hkv, per, part_o, part_ml, err);
     };
     TimingScope ts("decode_split", st);
-    if (G <= 4)
-      run(std::integral_constant<int, 4>());
-    else if (G <= 8)
-      run(std::integral_constant<int, 8>());
+    if (G <= 8)
+      run(std::integral_constant<int, 1>());
     else
-      run(std::integral_constant<int, 16>());
+      run(std::integral_constant<int, 2>());
   } else {
     const int per = ((n + nsplit - 1) / nsplit + 31) / 32 * 32;
     const size_t smem = (size_t)G * kD * 4 + (size_t)kDecWarps * G * kD * 4 + (size_t)kDecWarps * G * 8;
