@@ -568,3 +568,42 @@ def test_variant_abase_max(st, name):
     wl = WORKLOADS[name]()
     _run_edge(st, wl, wl.beta, abase_norm=1)
     _run_edge(st, wl, wl.beta, abase_norm=1, base_scorer=1)
+
+
+# ----------------------------------------------------------- kernel boundaries
+
+def test_edge_grid_width_limits(st):
+    # 127 columns: the widest grid of the tensor-core CSS band (256 key rows);
+    # 128 columns: the CUDA-core CSS; both against the oracle, bf16 and fp32
+    for gw, seed in ((127, 960), (128, 961), (200, 962)):
+        wl = synth.trajectory(n_steps=3, gh=3, gw=gw, n_text=5, hq=8, hkv=2, w=4, beta=0.2, seed=(seed,))
+        _run_edge(st, wl, 0.2)
+        wl.dtype = "f32"
+        _run_edge(st, wl, 0.2)
+
+
+def test_edge_query_rows_512(st):
+    # R = w G = 512 query rows per KV head, the largest the score passes take
+    wl = synth.trajectory(n_steps=3, gh=6, gw=7, n_text=9, hq=8, hkv=1, w=64, beta=0.25, seed=(963,))
+    _run_edge(st, wl, 0.25)
+
+
+def test_edge_one_query_head_per_group(st):
+    # G = 1: every query head has its own KV head
+    wl = synth.trajectory(n_steps=3, gh=5, gw=9, n_text=3, hq=4, hkv=4, w=16, beta=0.3, seed=(964,))
+    _run_edge(st, wl, 0.3)
+
+
+def test_edge_tiny_caches(st):
+    # one cached token (text only) and a one-token budget
+    rng = np.random.default_rng(965)
+    for n in (1, 2, 3):
+        q = rng.standard_normal((2, 4, 128), dtype=np.float32)
+        k = rng.standard_normal((n, 2, 128), dtype=np.float32)
+        v = rng.standard_normal((n, 2, 128), dtype=np.float32)
+        wl = synth.Workload("tiny%d" % n, q, k, v, np.zeros(0, np.int32), np.zeros(0, np.int32),
+                            np.zeros(0, np.int32), beta=0.5)
+        ig, ref = _run_edge(st, wl, 0.5)
+        assert ig.shape[1] == max(1, n // 2)
+    wl = synth.trajectory(n_steps=2, gh=2, gw=3, n_text=2, hq=4, hkv=2, w=2, beta=0.2, seed=(966,))
+    _run_edge(st, wl, 0.2, k_override=1)
