@@ -56,6 +56,9 @@ def parse():
     ap.add_argument("--no-decode", action="store_true", help="skip the decode-over-the-cache measurement")
     ap.add_argument("--no-variants", action="store_true", help="skip the ablation-variant step times")
     ap.add_argument("--no-trajectory", action="store_true", help="skip the per-step trajectory sweep")
+    ap.add_argument("--workload", default="traj50", choices=["traj50", "uitars", "small_backbone", "long_horizon"],
+                    help="traj50 (default): the 28-layer, 50-step trajectory of the contract line; the others time "
+                         "the remaining configurations (one JSON line of their own)")
     return ap.parse_args()
 
 
@@ -726,10 +729,204 @@ def run_gpu(args):
         dist.destroy_process_group()
 
 
+def run_workload(args):
+    """The other configurations, timed through the same API on one GPU: a
+    1-layer UI-TARS-shaped cache at beta 10-40 %, the batch-8 smaller-backbone
+    shape (28 layers, one packed varlen call per layer) at beta 10 and 40 %,
+    and the long-horizon cache (1 layer and 28 layers) at beta 10 %.  One graph
+    per case; L2 is flushed between timed replays by inputs larger than L2
+    where they are (the 1-layer cases are not, and say so)."""
+    import torch
+    from paper_2603_00188_gb300 import build as pkg_build
+    from paper_2603_00188_gb300 import stlite, synth
+    pkg_build.build()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    peaks = load_peaks()
+    stream = torch.cuda.Stream(device=dev)
+
+    def bf16(x):
+        return torch.from_numpy(x).to(torch.bfloat16).to(dev)
+
+    def timed(step, reps):
+        with torch.cuda.stream(stream):
+            for _ in range(max(3, args.warmup)):
+                step(stream)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            step(stream)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                g.replay()
+            a.record(stream)
+            for _ in range(reps):
+                g.replay()
+            b.record(stream)
+        torch.cuda.synchronize()
+        ms = a.elapsed_time(b) / reps
+        stlite.stlite_timing_read()
+        stlite.stlite_timing_enable(True)
+        with torch.cuda.stream(stream):
+            step(stream)
+        stream.synchronize()
+        stlite.stlite_timing_enable(False)
+        kt = stlite.stlite_timing_read()
+        # per kernel: ms per step (all of the step's launches) and launches
+        return ms, {k: dict(ms_per_step=t, launches=c) for k, (c, t) in kt.items()}
+
+    def tsg_tflops(wls, layers, kernels):
+        # 2 N_hist N_cur d Hkv per layer and sequence, over the TSG launches
+        flop = 0.0
+        for wl in wls:
+            gh, gw = wl.frames[1], wl.frames[2]
+            cur = int(gh[-1] * gw[-1])
+            hist = int((gh[:-1] * gw[:-1]).sum())
+            flop += 2.0 * hist * cur * D * wl.k.shape[1]
+        flop *= layers
+        t = sum(v["ms_per_step"] for k, v in kernels.items() if k.startswith("tsg")) * 1e-3
+        ach = flop / t / 1e12 if t > 0 else 0.0
+        return dict(bound="tensor", achieved=ach, peak=peaks["bf16"], unit="TFLOP/s", frac=ach / peaks["bf16"],
+                    peak_source=peaks["source"] + " burst")
+
+    reps = max(5, min(20, args.steps))
+    runs = []
+    if args.workload == "uitars":
+        for beta in (0.1, 0.2, 0.3, 0.4):
+            wl = synth.uitars_layer(beta=beta)
+            q, k, v = bf16(wl.q), bf16(wl.k), bf16(wl.v)
+            fs = stlite.FrameSpec(*wl.frames)
+            prm = stlite.make_params(beta)
+            sh = stlite.make_shape(q, k)
+            b = stlite.stlite_budget(wl.n, beta)
+            ws = torch.zeros(stlite.stlite_workspace_size(sh, fs, prm), dtype=torch.uint8, device=dev)
+            ko = torch.empty((b, sh.n_kv_heads, D), dtype=torch.bfloat16, device=dev)
+            vo, ix = torch.empty_like(ko), torch.empty((sh.n_kv_heads, b), dtype=torch.int32, device=dev)
+
+            def step(st, q=q, k=k, v=v, fs=fs, prm=prm, ko=ko, vo=vo, ix=ix, ws=ws):
+                stlite.stlite_compress_layer(q, k, v, fs, prm, ko, vo, ix, ws, st)
+            ms, kern = timed(step, reps)
+            runs.append(dict(beta=beta, layers=1, n_tokens=wl.n, budget=b, ms_per_step=ms,
+                             value=wl.n / (ms * 1e-3), kernels=kern, tsg_roofline=tsg_tflops([wl], 1, kern),
+                             l2="one layer's K/V (24 MB) fits in L2: replays may hit L2"))
+    elif args.workload == "small_backbone":
+        L, S = LAYERS, 8
+        # one packed batch of 8 sequences per layer (the data does not depend
+        # on beta, only the budgets do)
+        layers = []
+        for l in range(L):
+            wls = [synth.small_backbone_seq(s, layer=l) for s in range(S)]
+            cu = np.concatenate([[0], np.cumsum([wl.n for wl in wls])]).astype(np.int32)
+            layers.append((wls, cu, torch.stack([bf16(wl.q) for wl in wls]), torch.cat([bf16(wl.k) for wl in wls]),
+                           torch.cat([bf16(wl.v) for wl in wls])))
+        for beta in (0.1, 0.4):
+            prm = stlite.make_params(beta)
+            per_layer = []
+            for (wls, cu, q, k, v) in layers:
+                tot = sum(stlite.stlite_budget(wl.n, beta) for wl in wls)
+                ko = torch.empty((tot, k.shape[1], D), dtype=torch.bfloat16, device=dev)
+                per_layer.append((wls, cu, q, k, v, ko, torch.empty_like(ko),
+                                  torch.empty((k.shape[1] * tot,), dtype=torch.int32, device=dev)))
+            wsb = max(stlite.stlite_workspace_size_varlen(stlite.make_shape(pl[2][0], pl[3]), pl[1],
+                                                          [wl.frames for wl in pl[0]], prm) for pl in per_layer)
+            ws = torch.zeros(wsb, dtype=torch.uint8, device=dev)
+
+            def step(st, per_layer=per_layer, prm=prm, ws=ws):
+                for (wls, cu, q, k, v, ko, vo, ix) in per_layer:
+                    stlite.stlite_compress_varlen(q, k, v, cu, [wl.frames for wl in wls], prm, ko, vo, ix, ws, st)
+            ms, kern = timed(step, reps)
+            ntok = sum(int(pl[1][-1]) for pl in per_layer)
+            runs.append(dict(beta=beta, layers=L, sequences=S, api="stlite_compress_varlen per layer",
+                             n_tokens_per_layer=ntok // L, ms_per_step=ms,
+                             value=ntok / (ms * 1e-3), kernels=kern,
+                             tsg_roofline=tsg_tflops([wl for pl in per_layer for wl in pl[0]], 1, kern),
+                             l2="inputs larger than L2 (%.2f GB K/V per step)" % (
+                                 2 * sum(pl[3].numel() for pl in per_layer) * 2 / 1e9)))
+            del ws
+            # the same step as one stlite_compress_varlen_layers call: every
+            # sequence's 28 layers in one launch per step
+            frames_l = [wl.frames for wl in per_layer[0][0]]
+            wsz = max(stlite.stlite_workspace_size_varlen(stlite.make_shape(pl[2][0], pl[3]), pl[1],
+                                                          [wl.frames for wl in pl[0]], prm) for pl in per_layer)
+            ws3 = torch.zeros(L * wsz, dtype=torch.uint8, device=dev)
+            lay3 = [pl[2:] for pl in per_layer]
+
+            def step3(st, lay3=lay3, cu=per_layer[0][1], frames_l=frames_l, prm=prm, ws3=ws3):
+                stlite.stlite_compress_varlen_layers(lay3, cu, frames_l, prm, ws3, st)
+            ms3, kern3 = timed(step3, reps)
+            runs.append(dict(beta=beta, layers=L, sequences=S, api="stlite_compress_varlen_layers",
+                             n_tokens_per_layer=ntok // L, ms_per_step=ms3, value=ntok / (ms3 * 1e-3), kernels=kern3,
+                             tsg_roofline=tsg_tflops([wl for pl in per_layer for wl in pl[0]], 1, kern3)))
+            del ws3
+            # the same step as one stlite_compress_layers call per sequence
+            # (its 28 layers share the sequence's frame layout): every stage
+            # is one launch over the 28 layers
+            seq_io, seq_ws = [], []
+            for s_ in range(S):
+                wl_s = [per_layer[l][0][s_] for l in range(L)]
+                fr = wl_s[0].frames
+                ios = []
+                for l in range(L):
+                    wls, cu, q, k, v, ko, vo, ix = per_layer[l]
+                    a0, a1 = int(cu[s_]), int(cu[s_ + 1])
+                    b0 = sum(stlite.stlite_budget(int(cu[i + 1] - cu[i]), beta) for i in range(s_))
+                    b_s = stlite.stlite_budget(a1 - a0, beta)
+                    ios.append((q[s_], k[a0:a1], v[a0:a1], ko[b0:b0 + b_s], vo[b0:b0 + b_s],
+                                torch.empty((k.shape[1], b_s), dtype=torch.int32, device=dev)))
+                sh_s = stlite.make_shape(ios[0][0], ios[0][1])
+                seq_ws.append(torch.zeros(L * stlite.stlite_workspace_size(sh_s, stlite.FrameSpec(*fr), prm),
+                                          dtype=torch.uint8, device=dev))
+                seq_io.append((ios, stlite.FrameSpec(*fr)))
+
+            def step2(st, seq_io=seq_io, seq_ws=seq_ws, prm=prm):
+                for (ios, fs_s), ws_s in zip(seq_io, seq_ws):
+                    stlite.stlite_compress_layers(ios, fs_s, prm, ws_s, st)
+            ms2, kern2 = timed(step2, reps)
+            runs.append(dict(beta=beta, layers=L, sequences=S, api="stlite_compress_layers per sequence",
+                             n_tokens_per_layer=ntok // L, ms_per_step=ms2, value=ntok / (ms2 * 1e-3), kernels=kern2,
+                             tsg_roofline=tsg_tflops([wl for pl in per_layer for wl in pl[0]], 1, kern2)))
+            del per_layer, seq_io, seq_ws
+            torch.cuda.empty_cache()
+    else:  # long_horizon
+        distinct = [synth.long_horizon(l) for l in range(4)]
+        for L in (1, LAYERS):
+            # layer l holds a copy of distinct layer l % 4 (its own buffers)
+            q4, k4, v4 = [bf16(wl.q) for wl in distinct], [bf16(wl.k) for wl in distinct], [bf16(wl.v) for wl in distinct]
+            qs = [q4[l % 4] for l in range(L)]
+            ks = [k4[l % 4] if L == 1 else k4[l % 4].clone() for l in range(L)]
+            vs = [v4[l % 4] if L == 1 else v4[l % 4].clone() for l in range(L)]
+            wl0 = distinct[0]
+            fs = stlite.FrameSpec(*wl0.frames)
+            prm = stlite.make_params(wl0.beta)
+            sh = stlite.make_shape(qs[0], ks[0])
+            b = stlite.stlite_budget(wl0.n, wl0.beta)
+            ws = torch.zeros(L * stlite.stlite_workspace_size(sh, fs, prm), dtype=torch.uint8, device=dev)
+            io = []
+            for l in range(L):
+                ko = torch.empty((b, sh.n_kv_heads, D), dtype=torch.bfloat16, device=dev)
+                io.append((qs[l], ks[l], vs[l], ko, torch.empty_like(ko),
+                           torch.empty((sh.n_kv_heads, b), dtype=torch.int32, device=dev)))
+
+            def step(st, io=io, fs=fs, prm=prm, ws=ws):
+                stlite.stlite_compress_layers(io, fs, prm, ws, st)
+            ms, kern = timed(step, reps)
+            runs.append(dict(beta=wl0.beta, layers=L, n_tokens=wl0.n, budget=b, ms_per_step=ms,
+                             value=wl0.n * L / (ms * 1e-3), kernels=kern, tsg_roofline=tsg_tflops([wl0], L, kern),
+                             data="synthetic; 4 distinct layers, repeated" if L > 4 else "synthetic",
+                             l2=("inputs larger than L2 (%.2f GB K/V per step)" % (2 * L * ks[0].numel() * 2 / 1e9))))
+            del io, ws, ks, vs
+            torch.cuda.empty_cache()
+    line = dict(workload=args.workload, metric=METRIC, unit=UNIT, higher_is_better=True, dtype="bf16",
+                data="synthetic", n_gpus=1, runs=runs)
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         run_reference(args)
+    elif args.workload != "traj50":
+        run_workload(args)
     else:
         run_gpu(args)
 

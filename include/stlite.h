@@ -3,8 +3,9 @@
  * ST-Lite per-layer KV-cache compression pass (arXiv 2603.00188, Algorithm 1).
  *
  * One call compresses one layer of one sequence (stlite_compress_layer), a
- * batch of layers of one sequence (stlite_compress_layers), or one layer of
- * a packed batch of sequences (stlite_compress_varlen).  The pass has five steps:
+ * batch of layers of one sequence (stlite_compress_layers), one layer of a
+ * packed batch of sequences (stlite_compress_varlen), or a batch of layers of
+ * a packed batch (stlite_compress_varlen_layers).  The pass has five steps:
  *   1. window scoring       A_base, Sec. 2.1 Eq. (2)
  *   2. TSG redundancy gate  rho, tau, M_time, Sec. 3.2 Eqs. (6)-(8)
  *   3. CSS saliency         Phi, Sec. 3.1 Eqs. (4)-(5)
@@ -296,6 +297,24 @@ STLITE_API stlite_status stlite_compress_varlen(const stlite_shape* shape, int32
                                                 const void* v, void* k_out, void* v_out, int32_t* idx_out,
                                                 int32_t* cu_budget_out, void* ws, size_t ws_bytes,
                                                 void* stream);
+
+/* stlite_compress_varlen over n_layers layers that share the packing
+ * (cu_seqlens, frames): every sequence's layers run together through the
+ * batched-layers path of stlite_compress_layers (one launch per step for up
+ * to 32 layers), the sequences one after another on `stream`.  The result
+ * for every layer equals stlite_compress_varlen's on that layer.
+ * layers: HOST array [n_layers]; entry l holds layer l's packed tensors in
+ *   the layouts of stlite_compress_varlen: q [n_seqs][w][Hq][d], k and v
+ *   [n_tokens][Hkv][d], k_out and v_out [sum_s B_s][Hkv][d], idx_out the
+ *   blocks [Hkv][B_s] one after another.
+ * ws: n_layers times stlite_workspace_size_varlen bytes.  cu_budget_out
+ *   (nullable, HOST) as for stlite_compress_varlen.
+ * Every argument is checked before anything is enqueued. */
+STLITE_API stlite_status stlite_compress_varlen_layers(const stlite_shape* shape, int32_t n_seqs,
+                                                       const int32_t* cu_seqlens, const stlite_frames* frames,
+                                                       const stlite_params* params, int32_t n_layers,
+                                                       const stlite_layer_io* layers, int32_t* cu_budget_out,
+                                                       void* ws, size_t ws_bytes, void* stream);
 
 /* Workspace bytes stlite_compress_varlen needs: the largest of the
  * sequences' stlite_workspace_size. */

@@ -471,20 +471,25 @@ stlite_status stlite_compress_layer(const stlite_shape* shape, const stlite_fram
 namespace {
 
 // Algorithm 1 over n_layers layers, layer l keeping budgets[l] tokens per
-// KV head; every budget is checked before anything is enqueued.
+// KV head; every budget is checked before anything is enqueued.  The pointer
+// checks are skipped for a packed batch's per-sequence offsets (their bases
+// were checked; an index block there starts on a 4-byte boundary, which the
+// kernels' scalar index accesses need).
 stlite_status compress_layers_impl(const stlite_shape* shape, const stlite_frames* frames,
                                    const stlite_params* params, int32_t n_layers,
                                    const stlite_layer_io* layers, const int32_t* budgets, void* ws,
-                                   size_t ws_bytes, void* stream) {
+                                   size_t ws_bytes, void* stream, bool check_pointers = true) {
   Ctx c;
   stlite_status s = prepare(shape, frames, ws, ws_bytes, n_layers, stream, &c);
   if (s != STLITE_OK) return s;
   for (int l = 0; l < n_layers; ++l) {
     const stlite_layer_io& x = layers[l];
-    if (!x.q || !x.k || !x.v || !x.k_out || !x.v_out || !x.idx_out) return STLITE_EINVAL;
-    if (!aligned16(x.q) || !aligned16(x.k) || !aligned16(x.v) || !aligned16(x.k_out) ||
-        !aligned16(x.v_out) || !aligned16(x.idx_out))
-      return STLITE_EINVAL;
+    if (check_pointers) {
+      if (!x.q || !x.k || !x.v || !x.k_out || !x.v_out || !x.idx_out) return STLITE_EINVAL;
+      if (!aligned16(x.q) || !aligned16(x.k) || !aligned16(x.v) || !aligned16(x.k_out) ||
+          !aligned16(x.v_out) || !aligned16(x.idx_out))
+        return STLITE_EINVAL;
+    }
     if (budgets[l] < 1 || budgets[l] > c.p.n) return STLITE_EINVAL;
   }
   // one launch per stage for up to kMaxLayers layers at a time
@@ -647,6 +652,57 @@ stlite_status stlite_compress_varlen(const stlite_shape* shape, int32_t n_seqs, 
                      static_cast<uint8_t*>(v_out) + cum * row, idx_out + (size_t)shape->n_kv_heads * cum);
     io.budget[0] = b;
     if ((s = compress_batch(c, params, io)) != STLITE_OK) return s;
+    cum += (size_t)b;
+    if (cu_budget_out) cu_budget_out[i + 1] = (int32_t)cum;
+  }
+  return STLITE_OK;
+}
+
+stlite_status stlite_compress_varlen_layers(const stlite_shape* shape, int32_t n_seqs, const int32_t* cu_seqlens,
+                                            const stlite_frames* frames, const stlite_params* params,
+                                            int32_t n_layers, const stlite_layer_io* layers,
+                                            int32_t* cu_budget_out, void* ws, size_t ws_bytes, void* stream) {
+  size_t ws_need = 0;
+  stlite_status s = varlen_shapes(shape, n_seqs, cu_seqlens, frames, &ws_need);
+  if (s != STLITE_OK) return s;
+  if ((s = check_params(params)) != STLITE_OK) return s;
+  if (n_layers < 1 || !layers) return STLITE_EINVAL;
+  for (int l = 0; l < n_layers; ++l) {
+    const stlite_layer_io& x = layers[l];
+    if (!x.q || !x.k || !x.v || !x.k_out || !x.v_out || !x.idx_out) return STLITE_EINVAL;
+    if (!aligned16(x.q) || !aligned16(x.k) || !aligned16(x.v) || !aligned16(x.k_out) || !aligned16(x.v_out) ||
+        !aligned16(x.idx_out))
+      return STLITE_EINVAL;
+  }
+  if (!ws || !aligned16(ws)) return STLITE_EINVAL;
+  if (ws_bytes / (size_t)n_layers < ws_need) return STLITE_EWORKSPACE;
+  for (int i = 0; i < n_seqs; ++i)
+    if (stlite_budget(cu_seqlens[i + 1] - cu_seqlens[i], params->beta, params->k_override) < 1)
+      return STLITE_EINVAL;
+  const size_t e = shape->dtype == STLITE_BF16 ? 2 : 4;
+  const size_t row = (size_t)shape->n_kv_heads * shape->head_dim * e;  // one token of k / v
+  const size_t qseq = (size_t)shape->window * shape->n_q_heads * shape->head_dim * e;
+  std::vector<stlite_layer_io> io((size_t)n_layers);
+  size_t cum = 0;
+  if (cu_budget_out) cu_budget_out[0] = 0;
+  for (int i = 0; i < n_seqs; ++i) {
+    stlite_shape ss = *shape;
+    ss.n_tokens = cu_seqlens[i + 1] - cu_seqlens[i];
+    const int32_t b = stlite_budget(ss.n_tokens, params->beta, params->k_override);
+    const size_t t0 = (size_t)cu_seqlens[i];
+    for (int l = 0; l < n_layers; ++l) {
+      const stlite_layer_io& x = layers[l];
+      io[l].q = static_cast<const uint8_t*>(x.q) + i * qseq;
+      io[l].k = static_cast<const uint8_t*>(x.k) + t0 * row;
+      io[l].v = static_cast<const uint8_t*>(x.v) + t0 * row;
+      io[l].k_out = static_cast<uint8_t*>(x.k_out) + cum * row;
+      io[l].v_out = static_cast<uint8_t*>(x.v_out) + cum * row;
+      io[l].idx_out = x.idx_out + (size_t)shape->n_kv_heads * cum;
+    }
+    std::vector<int32_t> budgets((size_t)n_layers, b);
+    if ((s = compress_layers_impl(&ss, &frames[i], params, n_layers, io.data(), budgets.data(), ws, ws_bytes,
+                                  stream, false)) != STLITE_OK)
+      return s;
     cum += (size_t)b;
     if (cu_budget_out) cu_budget_out[i + 1] = (int32_t)cum;
   }

@@ -29,7 +29,8 @@ EXPORTED = ("stlite_budget", "stlite_workspace_size", "stlite_score", "stlite_ga
             "stlite_compress_layer", "stlite_device_status", "stlite_timing_enable", "stlite_timing_read",
             "stlite_status_string", "stlite_score_noalloc", "stlite_compress_layers", "stlite_compress_varlen",
             "stlite_workspace_size_varlen", "stlite_decode_attention", "stlite_decode_workspace_size",
-            "stlite_compress_layers_budgets", "stlite_hierarchical_budgets", "stlite_spatial_saliency_size")
+            "stlite_compress_layers_budgets", "stlite_hierarchical_budgets", "stlite_spatial_saliency_size",
+            "stlite_compress_varlen_layers")
 
 
 class Shape(ctypes.Structure):
@@ -101,6 +102,10 @@ _sig = {
                                             _P, ctypes.c_size_t, _P]),
     "stlite_spatial_saliency_size": (_S, [ctypes.POINTER(Shape), ctypes.POINTER(Frames), _P, ctypes.c_int32, _P, _P,
                                           ctypes.c_size_t, _P]),
+    "stlite_compress_varlen_layers": (_S, [ctypes.POINTER(Shape), ctypes.c_int32, ctypes.POINTER(ctypes.c_int32),
+                                           ctypes.POINTER(Frames), ctypes.POINTER(Params), ctypes.c_int32,
+                                           ctypes.POINTER(LayerIO), ctypes.POINTER(ctypes.c_int32), _P,
+                                           ctypes.c_size_t, _P]),
     "stlite_hierarchical_budgets": (_S, [ctypes.c_int32, ctypes.POINTER(ctypes.c_double), ctypes.c_int64,
                                          ctypes.c_int32, ctypes.POINTER(ctypes.c_int32)]),
 }
@@ -312,6 +317,25 @@ def stlite_compress_varlen(q, k, v, cu_seqlens, frames_list, params, k_out, v_ou
                                        _ptr(q), _ptr(k), _ptr(v), _ptr(k_out), _ptr(v_out), _ptr(idx_out),
                                        cb.ctypes.data_as(ip), _ptr(ws), ws.numel(), _stream(stream)),
            "stlite_compress_varlen")
+    return cb
+
+
+def stlite_compress_varlen_layers(layers, cu_seqlens, frames_list, params, ws, stream=None):
+    """stlite_compress_varlen over several layers of one packed batch: layers
+    is a list of (q, k, v, k_out, v_out, idx_out) per layer, each in the
+    packed layouts of stlite_compress_varlen; ws: n_layers times
+    stlite_workspace_size_varlen bytes.  Returns the budget prefix sums."""
+    n_seqs = len(frames_list)
+    q0, k0 = layers[0][0], layers[0][1]
+    sh = make_shape(q0[0] if q0.dim() == 4 else q0, k0)
+    cu, specs, arr = _varlen_args(cu_seqlens, frames_list)
+    lio = (LayerIO * len(layers))(*[LayerIO(*(t.data_ptr() for t in lay)) for lay in layers])
+    cb = np.zeros(n_seqs + 1, dtype=np.int32)
+    ip = ctypes.POINTER(ctypes.c_int32)
+    _check(_lib.stlite_compress_varlen_layers(ctypes.byref(sh), n_seqs, cu.ctypes.data_as(ip), arr,
+                                              ctypes.byref(params), len(layers), lio, cb.ctypes.data_as(ip),
+                                              _ptr(ws), ws.numel(), _stream(stream)),
+           "stlite_compress_varlen_layers")
     return cb
 
 

@@ -205,3 +205,25 @@ def test_variant_params_validation(st):
                                             None) == st.STLITE_EWORKSPACE
     for size in (0, 3, 5, 7, 9):
         assert st.stlite_workspace_size(sh, fr, st.make_params(0.2, css_size=size, abase_norm=1)) == need
+
+
+def test_varlen_layers_validation(st):
+    """stlite_compress_varlen_layers refuses a short workspace and malformed
+    layer arrays on the host."""
+    lib = st._lib
+    sh = _shape(st, n=300, hq=4, hkv=2, w=4)
+    fr = [st.FrameSpec([0], [5], [8]), st.FrameSpec([10], [4], [6]), st.FrameSpec([], [], [])]
+    prm = st.make_params(0.2)
+    need = st.stlite_workspace_size_varlen(sh, [0, 100, 200, 300], fr, prm)
+    cu, specs, arr = st._varlen_args([0, 100, 200, 300], fr)
+    ip = ctypes.POINTER(ctypes.c_int32)
+    good = 0x10000
+    lay = (st.LayerIO * 2)(st.LayerIO(*([good] * 6)), st.LayerIO(*([good] * 6)))
+    call = lambda layers, n, ws_bytes: lib.stlite_compress_varlen_layers(
+        ctypes.byref(sh), 3, cu.ctypes.data_as(ip), arr, ctypes.byref(prm), n, layers, None,
+        ctypes.c_void_p(good), ws_bytes, None)
+    assert call(lay, 2, 2 * need - 1) == st.STLITE_EWORKSPACE
+    assert call(None, 2, 2 * need) == st.STLITE_EINVAL
+    assert call(lay, 0, 2 * need) == st.STLITE_EINVAL
+    bad = (st.LayerIO * 2)(st.LayerIO(*([good] * 6)), st.LayerIO(*([good] * 5 + [0])))
+    assert call(bad, 2, 2 * need) == st.STLITE_EINVAL

@@ -607,3 +607,47 @@ def test_edge_tiny_caches(st):
         assert ig.shape[1] == max(1, n // 2)
     wl = synth.trajectory(n_steps=2, gh=2, gw=3, n_text=2, hq=4, hkv=2, w=2, beta=0.2, seed=(966,))
     _run_edge(st, wl, 0.2, k_override=1)
+
+
+@pytest.mark.parametrize("beta", [0.1, 0.4])
+def test_varlen_layers_equals_per_layer(st, beta):
+    # a packed batch over several layers in one call equals one packed call
+    # per layer, bit for bit (4 sequences of the batch-8 shape, 3 layers;
+    # at beta = 10 % some sequences' index blocks start on odd offsets)
+    S, L = 4, 3
+    layers = []
+    for l in range(L):
+        wls = [synth.small_backbone_seq(s, layer=l, beta=beta) for s in range(S)]
+        dev = [to_device(wl) for wl in wls]
+        layers.append((wls, dev))
+    wls0 = layers[0][0]
+    cu = np.concatenate([[0], np.cumsum([wl.n for wl in wls0])]).astype(np.int32)
+    frames = [wl.frames for wl in wls0]
+    prm = st.make_params(beta)
+    tot = sum(st.stlite_budget(wl.n, beta) for wl in wls0)
+    packed, single = [], []
+    for wls, dev in layers:
+        q = torch.stack([d[0] for d in dev])
+        k = torch.cat([d[1] for d in dev])
+        v = torch.cat([d[2] for d in dev])
+        H = k.shape[1]
+        mk = lambda: (torch.empty((tot, H, 128), dtype=k.dtype, device="cuda"),
+                      torch.empty((tot, H, 128), dtype=k.dtype, device="cuda"),
+                      torch.empty((H * tot,), dtype=torch.int32, device="cuda"))
+        packed.append((q, k, v) + mk())
+        single.append((q, k, v) + mk())
+    if beta == 0.1:
+        assert any(st.stlite_budget(wl.n, beta) % 2 for wl in wls0)
+    sh = st.make_shape(packed[0][0][0], packed[0][1])
+    wsz = st.stlite_workspace_size_varlen(sh, cu, frames, prm)
+    ws = torch.zeros(L * wsz, dtype=torch.uint8, device="cuda")
+    cb = st.stlite_compress_varlen_layers(packed, cu, frames, prm, ws)
+    ws1 = torch.zeros(wsz, dtype=torch.uint8, device="cuda")
+    for (q, k, v, ko, vo, ix) in single:
+        cb1 = st.stlite_compress_varlen(q, k, v, cu, frames, prm, ko, vo, ix, ws1)
+    torch.cuda.synchronize()
+    assert st.stlite_device_status(ws) == st.STLITE_OK
+    assert list(cb) == list(cb1)
+    for a, b in zip(packed, single):
+        for x, y in zip(a[3:], b[3:]):
+            assert torch.equal(x, y)
