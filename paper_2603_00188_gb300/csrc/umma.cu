@@ -597,18 +597,22 @@ __global__ void __launch_bounds__(kThreads, 1)
 // Window score pass 2.  CTA (x, h): key tiles of 128 tokens are the A operand
 // (M = 128, one key per TMEM lane), Q of head h (NQ = R rounded up to 32
 // rows) is the B operand.  Each thread sums 2^(x_r c + bias_r) over the R
-// query rows of its key.  TMEM: two stages of NQ columns when NQ <= 256
-// (epilogue group g takes the tiles with it % 2 == g), else one stage.
+// query rows of its key.  TMEM: two slots of W columns, so that one item
+// drains while the next one is computed.  An item is a key tile against
+// all NQ query columns (W = NQ <= 256), or against one of nh = 2 column
+// halves (NQ > 256, rounded to 64, W = NQ / 2).
 struct CsLayout {
-  int NQ, nstage, kstages, tmem_cols, q_bytes, off_k, off_bias, off_bar, off_xch, total;
+  int NQ, nh, W, nstage, kstages, tmem_cols, q_bytes, off_k, off_bias, off_bar, off_xch, total;
 };
 constexpr int kCsXchBytes = 2 * 128 * 4 + 64;  // two partial-sum buffers, then xfull[2], xempty[2]
 __host__ __device__ inline CsLayout cs_layout(int R) {
   CsLayout L;
-  L.NQ = (R + 31) & ~31;
-  L.nstage = L.NQ <= 256 ? 2 : 1;
+  L.NQ = R > 256 ? (R + 63) & ~63 : (R + 31) & ~31;
+  L.nh = L.NQ > 256 ? 2 : 1;
+  L.W = L.NQ / L.nh;
+  L.nstage = 2;
   L.tmem_cols = 32;
-  while (L.tmem_cols < L.nstage * L.NQ) L.tmem_cols <<= 1;
+  while (L.tmem_cols < L.nstage * L.W) L.tmem_cols <<= 1;
   L.q_bytes = L.NQ * 256;
   const int fixed = L.q_bytes + L.NQ * 4 + kScoreBarBytes + kCsXchBytes + 1024;
   L.kstages = (kScoreSmemCap - fixed) / 32768;
@@ -622,13 +626,17 @@ __host__ __device__ inline CsLayout cs_layout(int R) {
   return L;
 }
 
+// NH: column halves per key tile (cs_layout's nh), a template parameter so
+// that the one-half loop compiles away.
+template <int NH>
 __global__ void __launch_bounds__(kThreads, 1)
     k_colsum_umma(const __grid_constant__ KMaps maps, const __grid_constant__ LayerPtrs io, Problem p,
                   Strided<float2> part_all, int nsplit, Strided<float> a_all, uint32_t* err) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = align1024(smem_raw);
   const CsLayout L = cs_layout(p.R());
-  const int NQ = L.NQ, nstage = L.nstage, R = p.R(), n = p.n;
+  constexpr int nh = NH;
+  const int NQ = L.NQ, W = L.W, R = p.R(), n = p.n;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int layer = blockIdx.y / p.hkv, h = blockIdx.y % p.hkv;
   const CUtensorMap& kmap = maps.m[layer];
@@ -713,85 +721,101 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      for (int it = 0; it < ntiles; ++it) {
-        const int s = it % S, as = it % nstage;
-        const uint32_t u = (uint32_t)(it / S), ua = (uint32_t)(it / nstage);
+      bool ok = true;
+      for (int it = 0; ok && it < ntiles; ++it) {
+        const int s = it % S;
+        const uint32_t u = (uint32_t)(it / S);
         if (!mbar_wait(b_kfull + 8 * s, u & 1u, err, abort_flag)) break;
-        if (!mbar_wait(b_accempty + 8 * as, (ua & 1u) ^ 1u, err, abort_flag)) break;
-        tc_fence_after();
-        for (int nb = 0; nb < NQ; nb += 256) {
-          const int nn = min(256, NQ - nb);
-          const uint32_t idesc = idesc_bf16(128, nn);
+        // item it*nh + hh: query columns [hh W, hh W + W) into TMEM slot item % 2
+#pragma unroll
+        for (int hh = 0; hh < nh; ++hh) {
+          const int item = it * nh + hh, as = item & 1;
+          if (!mbar_wait(b_accempty + 8 * as, ((uint32_t)(item >> 1) & 1u) ^ 1u, err, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t idesc = idesc_bf16(128, W);
 #pragma unroll
           for (int k = 0; k < 8; ++k) {
             const uint32_t kb = k >> 2, koff = (k & 3) * 32;
             uint64_t ad = desc_sw128(sK + s * 32768 + kb * 16384 + koff);
-            uint64_t bd = desc_sw128(sQ + kb * (NQ * 128) + nb * 128 + koff);
-            umma_bf16(tmem + as * NQ + nb, ad, bd, idesc, k > 0 ? 1u : 0u);
+            uint64_t bd = desc_sw128(sQ + kb * (NQ * 128) + hh * W * 128 + koff);
+            umma_bf16(tmem + as * W, ad, bd, idesc, k > 0 ? 1u : 0u);
           }
+          umma_commit(b_accfull + 8 * as);
         }
-        umma_commit(b_accfull + 8 * as);
+        if (!ok) break;
         umma_commit(b_kempty + 8 * s);
       }
       umma_commit(b_done);
       mbar_wait_drain(b_done, 0);
     }
   } else {
-    // Both groups drain every tile: group 0 the query columns [0, sp),
-    // group 1 [sp, NQ); columns of padded rows carry bias = -inf, so they
-    // add exact zeros.  Group 1 passes its partial sum to group 0 through
-    // a double-buffered shared array (xfull / xempty barriers).
+    // Both groups drain every item: group 0 the item's query columns
+    // [0, sp), group 1 [sp, W); columns of padded rows carry bias = -inf, so
+    // they add exact zeros.  A thread's sum runs over the tile's nh items;
+    // group 1 then passes it to group 0 through a double-buffered shared
+    // array (xfull / xempty barriers).
     const int g = (warp - 2) >> 2, quarter = warp & 3, row = quarter * 32 + lane;
-    const int sp = min(NQ, ((NQ >> 1) + 63) & ~63);
-    const int c0 = g == 0 ? 0 : sp, c1 = g == 0 ? sp : NQ;
+    const int sp = min(W, ((W >> 1) + 63) & ~63);
+    const int c0 = g == 0 ? 0 : sp, c1 = g == 0 ? sp : W;
     const uint32_t lanebase = tmem + ((uint32_t)(quarter * 32) << 16);
-    for (int it = 0; it < ntiles; ++it) {
-      const int as = it % nstage;
-      const uint32_t ua = (uint32_t)(it / nstage);
-      if (!warp_wait(b_accfull + 8 * as, ua & 1u, err, abort_flag)) break;
-      tc_fence_after();
-      const uint32_t tbase = lanebase + as * NQ;
+    bool ok = true;
+    for (int it = 0; ok && it < ntiles; ++it) {
       float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
-      int cb = c0;
+#pragma unroll
+      for (int hh = 0; hh < nh; ++hh) {
+        const int item = it * nh + hh, as = item & 1;
+        if (!warp_wait(b_accfull + 8 * as, (uint32_t)(item >> 1) & 1u, err, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t tbase = lanebase + as * W;
+        const float* bias_h = bias_s + hh * W;
+        int cb = c0;
 #pragma unroll 1
-      for (; cb + 64 <= c1; cb += 64) {
-        float v[64];
-        tmem_ld64(tbase + cb, v);
-        const float4* b4 = reinterpret_cast<const float4*>(bias_s + cb);
-        // three phases over the chunk (exponent arguments, exponentials,
-        // sums), so that independent work separates dependent instructions
+        for (; cb + 64 <= c1; cb += 64) {
+          float v[64];
+          tmem_ld64(tbase + cb, v);
+          const float4* b4 = reinterpret_cast<const float4*>(bias_h + cb);
+          // three phases over the chunk (exponent arguments, exponentials,
+          // sums), so that independent work separates dependent instructions
 #pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const float4 b = b4[i];
-          fma2(v[4 * i], v[4 * i + 1], c, c, b.x, b.y, v[4 * i], v[4 * i + 1]);
-          fma2(v[4 * i + 2], v[4 * i + 3], c, c, b.z, b.w, v[4 * i + 2], v[4 * i + 3]);
+          for (int i = 0; i < 16; ++i) {
+            const float4 b = b4[i];
+            fma2(v[4 * i], v[4 * i + 1], c, c, b.x, b.y, v[4 * i], v[4 * i + 1]);
+            fma2(v[4 * i + 2], v[4 * i + 3], c, c, b.z, b.w, v[4 * i + 2], v[4 * i + 3]);
+          }
+#pragma unroll
+          for (int i = 0; i < 64; ++i) v[i] = ex2_approx(v[i]);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            add2(a0, a1, v[4 * i], v[4 * i + 1]);
+            add2(a2, a3, v[4 * i + 2], v[4 * i + 3]);
+          }
         }
+        if (c1 - cb == 32) {
+          float v[32];
+          tmem_ld32(tbase + cb, v);
+          const float4* b4 = reinterpret_cast<const float4*>(bias_h + cb);
 #pragma unroll
-        for (int i = 0; i < 64; ++i) v[i] = ex2_approx(v[i]);
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          add2(a0, a1, v[4 * i], v[4 * i + 1]);
-          add2(a2, a3, v[4 * i + 2], v[4 * i + 3]);
+          for (int i = 0; i < 8; ++i) {
+            const float4 b = b4[i];
+            float x0, x1, x2, x3;
+            fma2(v[4 * i], v[4 * i + 1], c, c, b.x, b.y, x0, x1);
+            fma2(v[4 * i + 2], v[4 * i + 3], c, c, b.z, b.w, x2, x3);
+            add2(a0, a1, ex2_approx(x0), ex2_approx(x1));
+            add2(a2, a3, ex2_approx(x2), ex2_approx(x3));
+          }
         }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(b_accempty + 8 * as);
       }
-      if (c1 - cb == 32) {
-        float v[32];
-        tmem_ld32(tbase + cb, v);
-        const float4* b4 = reinterpret_cast<const float4*>(bias_s + cb);
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const float4 b = b4[i];
-          float x0, x1, x2, x3;
-          fma2(v[4 * i], v[4 * i + 1], c, c, b.x, b.y, x0, x1);
-          fma2(v[4 * i + 2], v[4 * i + 3], c, c, b.z, b.w, x2, x3);
-          add2(a0, a1, ex2_approx(x0), ex2_approx(x1));
-          add2(a2, a3, ex2_approx(x2), ex2_approx(x3));
-        }
-      }
+      if (!ok) break;
       float acc = (a0 + a1) + (a2 + a3);
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(b_accempty + 8 * as);
       const int xb = it & 1;
       const uint32_t ux = (uint32_t)(it >> 1);
       if (g == 1) {
@@ -1194,8 +1218,8 @@ cudaError_t launch_score_umma(const Problem& p, const LayerPtrs& io, Strided<flo
   if ((e = cudaFuncSetAttribute(rs_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, L1.total)) !=
       cudaSuccess)
     return e;
-  if ((e = cudaFuncSetAttribute(k_colsum_umma, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                L2.total)) != cudaSuccess)
+  auto cs_kernel = L2.nh == 2 ? k_colsum_umma<2> : k_colsum_umma<1>;
+  if ((e = cudaFuncSetAttribute(cs_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, L2.total)) != cudaSuccess)
     return e;
   {
     TimingScope ts("rowstats_umma", st);
@@ -1205,7 +1229,7 @@ cudaError_t launch_score_umma(const Problem& p, const LayerPtrs& io, Strided<flo
   const int tiles = (p.n + 127) / 128;
   const int gx = pick_split(p.L * p.hkv, tiles, sm_count());
   TimingScope ts("colsum_umma", st);
-  k_colsum_umma<<<dim3(gx, p.L * p.hkv), kThreads, L2.total, st>>>(m2, io, p, rowpart, nsplit, a_base, err);
+  cs_kernel<<<dim3(gx, p.L * p.hkv), kThreads, L2.total, st>>>(m2, io, p, rowpart, nsplit, a_base, err);
   return cudaGetLastError();
 }
 
