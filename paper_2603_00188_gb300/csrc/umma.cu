@@ -7,9 +7,11 @@
 //                    softmax probabilities.
 //
 // All three share one structure: warp 0 issues TMA loads of 128-byte-swizzled
-// key tiles, warp 1 issues tcgen05.mma into TMEM (fp32 accumulators), warps
-// 2-9 (two groups of four, one warp per TMEM lane quarter) drain TMEM with
-// tcgen05.ld and run the fp32 epilogue.  Every mbarrier wait is bounded.
+// key tiles, warp 1 issues tcgen05.mma into TMEM (fp32 accumulators), and
+// groups of four warps (one warp per TMEM lane quarter) drain TMEM with
+// tcgen05.ld and run the fp32 epilogue: two groups (warps 2-9) in TSG and
+// the column sums, four (warps 2-17) in the row statistics.  Every mbarrier
+// wait is bounded.
 #include <cudaTypedefs.h>
 
 #include "kernels.cuh"
@@ -307,11 +309,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // =========================================================================
 // Window score pass 1.  CTA (split, h): Q of head h (R rows, MT M-tiles of
-// 128) stays in shared memory as the A operand; key tiles of KN = 256/MT
-// keys stream as the B operand.  TMEM: two stages of MT*KN <= 256 columns;
-// epilogue group g handles the key tiles with it % 2 == g and keeps, per
-// query row, the running max m (raw dot units) and l = sum 2^((x - m) c).
-// The two groups merge at the end; part[h][split][r] = (m c, l).
+// 128) stays in shared memory as the A operand; key tiles of KN keys (256
+// for MT <= 2, else 128) stream as the B operand.  TMEM: two slots of 256
+// columns, one (m-tile, key tile) item each; every epilogue group drains a
+// quarter of each item's keys and keeps, per query row, the running max m
+// (raw dot units) and l = sum 2^((x - m) c).  The groups merge at the end;
+// part[h][split][r] = (m c, l).
 constexpr int kMaxKStages = 4;        // key-tile ring depth (as shared memory allows)
 constexpr int kScoreSmemCap = 200 * 1024;
 
@@ -336,6 +339,13 @@ __device__ __forceinline__ ScoreBars score_bars(uint8_t* base) {
 }
 constexpr int kScoreBarBytes = 128;
 
+// Row-statistics pass: a TMA warp, an MMA warp and kRsGroups epilogue
+// groups of four warps.  With 18 warps, an SM sub-partition holds five of
+// them, so its 64 K registers leave at most 96 per thread.
+constexpr int kRsGroups = 4;
+constexpr int kRsThreads = (2 + 4 * kRsGroups) * 32;
+constexpr int kRsMaxReg = 96;
+
 struct RsLayout {
   int MT, KN, q_bytes, k_stage_bytes, kstages, off_k, off_bar, off_xch, total;
 };
@@ -345,14 +355,15 @@ __host__ __device__ inline RsLayout rs_layout(int R) {
   L.KN = L.MT <= 2 ? 256 : 128;  // keys per tile = MMA N of one (m-tile, key tile) item
   L.q_bytes = L.MT * 128 * 256;
   L.k_stage_bytes = L.KN * 256;
-  const int fixed = L.q_bytes + kScoreBarBytes + L.MT * 128 * 8 + 1024;
+  const int xch = (kRsGroups - 1) * L.MT * 128 * 8;
+  const int fixed = L.q_bytes + kScoreBarBytes + xch + 1024;
   L.kstages = (kScoreSmemCap - fixed) / L.k_stage_bytes;
   if (L.kstages > kMaxKStages) L.kstages = kMaxKStages;
   if (L.kstages < 2) L.kstages = 2;
   L.off_k = L.q_bytes;
   L.off_bar = L.off_k + L.kstages * L.k_stage_bytes;
   L.off_xch = L.off_bar + kScoreBarBytes;
-  L.total = L.off_xch + L.MT * 128 * 8 + 1024;
+  L.total = L.off_xch + xch + 1024;
   return L;
 }
 
@@ -366,13 +377,14 @@ __device__ __forceinline__ void online_merge(float& m, float& l, float m2, float
 }
 
 template <int MT>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __maxnreg__(kRsMaxReg)
     k_rowstats_umma(const __grid_constant__ KMaps maps, const __grid_constant__ LayerPtrs io, Problem p,
                     int nsplit, Strided<float2> part_all, uint32_t* err) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = align1024(smem_raw);
   const RsLayout L = rs_layout(p.R());
   constexpr int KN = MT <= 2 ? 256 : 128;
+  constexpr int CW = KN / kRsGroups;  // key columns per group and item (64 or 32)
   const int R = p.R();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int split = blockIdx.x, layer = blockIdx.y / p.hkv, h = blockIdx.y % p.hkv, n = p.n;
@@ -400,7 +412,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(b_accfull + 8 * i, 1);
-      mbar_init(b_accempty + 8 * i, 8);  // both epilogue groups
+      mbar_init(b_accempty + 8 * i, 4 * kRsGroups);  // every epilogue warp
     }
     mbar_init(b_done, 1);
     *abort_flag = 0u;
@@ -418,11 +430,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = *slot;
 
   // Work items u = t * MT + mt: m-tile mt of Q against key tile t, into
-  // TMEM slot u % 2 (KN columns).  Both epilogue groups drain every item,
-  // group g taking key columns [g*KN/2, (g+1)*KN/2), so that one item drains
-  // while the MMA fills the other slot.  Each group keeps a row state per
-  // m-tile, (running max m in raw dot units, l = sum 2^((x - m) c)); the two
-  // groups' states are merged at the end.
+  // TMEM slot u % 2 (KN columns).  All kRsGroups epilogue groups drain every
+  // item, group g taking key columns [g*CW, (g+1)*CW): four warps per SM
+  // sub-partition hide one another's latencies, and one item drains while
+  // the MMA fills the other slot.  Each group keeps a row state per m-tile,
+  // (running max m in raw dot units, l = sum 2^((x - m) c)); the groups'
+  // states are merged at the end.
   float ms[MT], ls[MT];
 #pragma unroll
   for (int i = 0; i < MT; ++i) {
@@ -479,13 +492,24 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_wait_drain(b_done, 0);
     }
   } else {
-    constexpr int HALF = KN / 2;  // key columns per group and item
-    const uint32_t lanebase = tmem + ((uint32_t)(quarter * 32) << 16) + g * HALF;
+    const uint32_t lanebase = tmem + ((uint32_t)(quarter * 32) << 16) + g * CW;
     for (int u = 0; u < nitems; ++u) {
       const int as = u & 1;
       if (!warp_wait(b_accfull + 8 * as, (uint32_t)(u >> 1) & 1u, err, abort_flag)) break;
       tc_fence_after();
       const int t = u / MT, mt = u % MT;
+      uint32_t b[CW];
+      if constexpr (CW == 64) {
+        tmem_ld64_issue(lanebase + as * 256, b);
+        tmem_ld64_wait(b);
+      } else {
+        tmem_ld32_issue(lanebase + as * 256, b);
+        tmem_wait_regs32(b);
+      }
+      // the item's TMEM columns are in registers: release the slot
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(b_accempty + 8 * as);
       float m = ms[0], l = ls[0];
 #pragma unroll
       for (int i = 1; i < MT; ++i)
@@ -493,71 +517,54 @@ __global__ void __launch_bounds__(kThreads, 1)
           m = ms[i];
           l = ls[i];
         }
-      const int tok = j0 + t * KN + g * HALF;
-      // 64-column chunks in key order; chunk q+1 loads from TMEM while
-      // chunk q is reduced
-      auto online = [&](const uint32_t (&b)[64], int q) {
-        const int kbase = tok + q * 64;
-        const int nv = min(64, j1 - kbase);
-        if (nv <= 0) return;
-        if (nv == 64) {
-          // chunk maximum over four independent chains: chain r starts at
-          // element r and takes pairs 4 + 2r + 8i, 5 + 2r + 8i (i = 0..7)
-          float cm[4];
+      const int nv = min(CW, j1 - (j0 + t * KN + g * CW));
+      if (nv == CW) {
+        // chunk maximum over four independent chains: chain r starts at
+        // element r and takes pairs 4 + 2r + 8i, 5 + 2r + 8i
+        float cm[4];
 #pragma unroll
-          for (int r = 0; r < 4; ++r) cm[r] = __uint_as_float(b[r]);
+        for (int r = 0; r < 4; ++r) cm[r] = __uint_as_float(b[r]);
 #pragma unroll
-          for (int i = 4; i < 64; i += 8) {
+        for (int i = 4; i < CW; i += 8) {
 #pragma unroll
-            for (int r = 0; r < 4; ++r)
-              if (i + 2 * r + 1 < 64)
-                cm[r] = max3(cm[r], __uint_as_float(b[i + 2 * r]), __uint_as_float(b[i + 2 * r + 1]));
-          }
-          const float mn = fmaxf(m, fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3])));
-          const float mnc = mn * c;
-          float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-          // three phases (exponent arguments, exponentials, sums), so that
-          // independent work separates dependent instructions
-          float x[64];
-#pragma unroll
-          for (int i = 0; i < 64; i += 2)
-            fma2(__uint_as_float(b[i]), __uint_as_float(b[i + 1]), c, c, -mnc, -mnc, x[i], x[i + 1]);
-#pragma unroll
-          for (int i = 0; i < 64; ++i) x[i] = ex2_approx(x[i]);
-#pragma unroll
-          for (int i = 0; i < 64; i += 4) {
-            add2(s0, s1, x[i], x[i + 1]);
-            add2(s2, s3, x[i + 2], x[i + 3]);
-          }
-          l = (m == -CUDART_INF_F ? 0.f : l * ex2_approx((m - mn) * c)) + ((s0 + s1) + (s2 + s3));
-          m = mn;
-        } else {
-          float mc = -CUDART_INF_F;
-#pragma unroll
-          for (int i = 0; i < 64; ++i)
-            if (i < nv) mc = fmaxf(mc, __uint_as_float(b[i]));
-          const float mn = fmaxf(m, mc);
-          const float mnc = mn * c;
-          float sacc = 0.f;
-#pragma unroll
-          for (int i = 0; i < 64; ++i)
-            if (i < nv) sacc += ex2_approx(fmaf(__uint_as_float(b[i]), c, -mnc));
-          l = (m == -CUDART_INF_F ? 0.f : l * ex2_approx((m - mn) * c)) + sacc;
-          m = mn;
+          for (int r = 0; r < 4; ++r)
+            if (i + 2 * r + 1 < CW)
+              cm[r] = max3(cm[r], __uint_as_float(b[i + 2 * r]), __uint_as_float(b[i + 2 * r + 1]));
         }
-      };
-      const uint32_t tb = lanebase + as * 256;
-      uint32_t b0[64];
-      tmem_ld64_issue(tb, b0);
-      tmem_ld64_wait(b0);
-      if (HALF == 128) {
-        uint32_t b1[64];
-        tmem_ld64_issue(tb + 64, b1);
-        online(b0, 0);
-        tmem_ld64_wait(b1);
-        online(b1, 1);
-      } else {
-        online(b0, 0);
+        const float mn = fmaxf(m, fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3])));
+        const float mnc = mn * c;
+        float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+        // three phases (exponent arguments, exponentials, sums) in place, so
+        // that independent work separates dependent instructions
+#pragma unroll
+        for (int i = 0; i < CW; i += 2) {
+          float x0, x1;
+          fma2(__uint_as_float(b[i]), __uint_as_float(b[i + 1]), c, c, -mnc, -mnc, x0, x1);
+          b[i] = __float_as_uint(x0);
+          b[i + 1] = __float_as_uint(x1);
+        }
+#pragma unroll
+        for (int i = 0; i < CW; ++i) b[i] = __float_as_uint(ex2_approx(__uint_as_float(b[i])));
+#pragma unroll
+        for (int i = 0; i < CW; i += 4) {
+          add2(s0, s1, __uint_as_float(b[i]), __uint_as_float(b[i + 1]));
+          add2(s2, s3, __uint_as_float(b[i + 2]), __uint_as_float(b[i + 3]));
+        }
+        l = (m == -CUDART_INF_F ? 0.f : l * ex2_approx((m - mn) * c)) + ((s0 + s1) + (s2 + s3));
+        m = mn;
+      } else if (nv > 0) {
+        float mc = -CUDART_INF_F;
+#pragma unroll
+        for (int i = 0; i < CW; ++i)
+          if (i < nv) mc = fmaxf(mc, __uint_as_float(b[i]));
+        const float mn = fmaxf(m, mc);
+        const float mnc = mn * c;
+        float sacc = 0.f;
+#pragma unroll
+        for (int i = 0; i < CW; ++i)
+          if (i < nv) sacc += ex2_approx(fmaf(__uint_as_float(b[i]), c, -mnc));
+        l = (m == -CUDART_INF_F ? 0.f : l * ex2_approx((m - mn) * c)) + sacc;
+        m = mn;
       }
 #pragma unroll
       for (int i = 0; i < MT; ++i)
@@ -565,15 +572,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           ms[i] = m;
           ls[i] = l;
         }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(b_accempty + 8 * as);
     }
   }
-  // merge the two groups' states, then write (m * c, l) per query row
-  if (warp >= 2 && g == 1) {
+  // merge the groups' states, then write (m * c, l) per query row
+  if (warp >= 2 && g > 0) {
 #pragma unroll
-    for (int mt = 0; mt < MT; ++mt) xch[mt * 128 + quarter * 32 + lane] = make_float2(ms[mt], ls[mt]);
+    for (int mt = 0; mt < MT; ++mt)
+      xch[((g - 1) * MT + mt) * 128 + quarter * 32 + lane] = make_float2(ms[mt], ls[mt]);
   }
   tc_fence_before();
   __syncthreads();
@@ -581,9 +586,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
     for (int mt = 0; mt < MT; ++mt) {
       const int row = mt * 128 + quarter * 32 + lane;
-      const float2 o = xch[row];
       float m = ms[mt], l = ls[mt];
-      online_merge(m, l, o.x, o.y, c);
+      for (int o = 1; o < kRsGroups; ++o) {
+        const float2 v = xch[((o - 1) * MT + mt) * 128 + quarter * 32 + lane];
+        online_merge(m, l, v.x, v.y, c);
+      }
       if (row < R) part[((size_t)h * nsplit + split) * R + row] = make_float2(m * c, l);
     }
   }
@@ -1223,7 +1230,7 @@ cudaError_t launch_score_umma(const Problem& p, const LayerPtrs& io, Strided<flo
     return e;
   {
     TimingScope ts("rowstats_umma", st);
-    rs_kernel<<<dim3(nsplit, p.L * p.hkv), kThreads, L1.total, st>>>(m1, io, p, nsplit, rowpart, err);
+    rs_kernel<<<dim3(nsplit, p.L * p.hkv), kRsThreads, L1.total, st>>>(m1, io, p, nsplit, rowpart, err);
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const int tiles = (p.n + 127) / 128;
