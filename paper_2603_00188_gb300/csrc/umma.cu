@@ -339,12 +339,13 @@ __device__ __forceinline__ ScoreBars score_bars(uint8_t* base) {
 }
 constexpr int kScoreBarBytes = 128;
 
-// Row-statistics pass: a TMA warp, an MMA warp and kRsGroups epilogue
+// Window-score passes: a TMA warp, an MMA warp and kScoreGroups epilogue
 // groups of four warps.  With 18 warps, an SM sub-partition holds five of
 // them, so its 64 K registers leave at most 96 per thread.
-constexpr int kRsGroups = 4;
-constexpr int kRsThreads = (2 + 4 * kRsGroups) * 32;
-constexpr int kRsMaxReg = 96;
+constexpr int kScoreGroups = 4;
+constexpr int kScoreThreads = (2 + 4 * kScoreGroups) * 32;
+constexpr int kScoreMaxReg = 96;
+static_assert(kScoreGroups == 4, "the column sums add four partial sums per key");
 
 struct RsLayout {
   int MT, KN, q_bytes, k_stage_bytes, kstages, off_k, off_bar, off_xch, total;
@@ -355,7 +356,7 @@ __host__ __device__ inline RsLayout rs_layout(int R) {
   L.KN = L.MT <= 2 ? 256 : 128;  // keys per tile = MMA N of one (m-tile, key tile) item
   L.q_bytes = L.MT * 128 * 256;
   L.k_stage_bytes = L.KN * 256;
-  const int xch = (kRsGroups - 1) * L.MT * 128 * 8;
+  const int xch = (kScoreGroups - 1) * L.MT * 128 * 8;
   const int fixed = L.q_bytes + kScoreBarBytes + xch + 1024;
   L.kstages = (kScoreSmemCap - fixed) / L.k_stage_bytes;
   if (L.kstages > kMaxKStages) L.kstages = kMaxKStages;
@@ -377,14 +378,14 @@ __device__ __forceinline__ void online_merge(float& m, float& l, float m2, float
 }
 
 template <int MT>
-__global__ void __maxnreg__(kRsMaxReg)
+__global__ void __maxnreg__(kScoreMaxReg)
     k_rowstats_umma(const __grid_constant__ KMaps maps, const __grid_constant__ LayerPtrs io, Problem p,
                     int nsplit, Strided<float2> part_all, uint32_t* err) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = align1024(smem_raw);
   const RsLayout L = rs_layout(p.R());
   constexpr int KN = MT <= 2 ? 256 : 128;
-  constexpr int CW = KN / kRsGroups;  // key columns per group and item (64 or 32)
+  constexpr int CW = KN / kScoreGroups;  // key columns per group and item (64 or 32)
   const int R = p.R();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int split = blockIdx.x, layer = blockIdx.y / p.hkv, h = blockIdx.y % p.hkv, n = p.n;
@@ -412,7 +413,7 @@ __global__ void __maxnreg__(kRsMaxReg)
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(b_accfull + 8 * i, 1);
-      mbar_init(b_accempty + 8 * i, 4 * kRsGroups);  // every epilogue warp
+      mbar_init(b_accempty + 8 * i, 4 * kScoreGroups);  // every epilogue warp
     }
     mbar_init(b_done, 1);
     *abort_flag = 0u;
@@ -430,7 +431,7 @@ __global__ void __maxnreg__(kRsMaxReg)
   const uint32_t tmem = *slot;
 
   // Work items u = t * MT + mt: m-tile mt of Q against key tile t, into
-  // TMEM slot u % 2 (KN columns).  All kRsGroups epilogue groups drain every
+  // TMEM slot u % 2 (KN columns).  All kScoreGroups epilogue groups drain every
   // item, group g taking key columns [g*CW, (g+1)*CW): four warps per SM
   // sub-partition hide one another's latencies, and one item drains while
   // the MMA fills the other slot.  Each group keeps a row state per m-tile,
@@ -587,7 +588,7 @@ __global__ void __maxnreg__(kRsMaxReg)
     for (int mt = 0; mt < MT; ++mt) {
       const int row = mt * 128 + quarter * 32 + lane;
       float m = ms[mt], l = ls[mt];
-      for (int o = 1; o < kRsGroups; ++o) {
+      for (int o = 1; o < kScoreGroups; ++o) {
         const float2 v = xch[((o - 1) * MT + mt) * 128 + quarter * 32 + lane];
         online_merge(m, l, v.x, v.y, c);
       }
@@ -611,7 +612,10 @@ __global__ void __maxnreg__(kRsMaxReg)
 struct CsLayout {
   int NQ, nh, W, nstage, kstages, tmem_cols, q_bytes, off_k, off_bias, off_bar, off_xch, total;
 };
-constexpr int kCsXchBytes = 2 * 128 * 4 + 64;  // two partial-sum buffers, then xfull[2], xempty[2]
+// partial sums [kCsXBuf][kScoreGroups][128 keys] fp32, then the arrival
+// counters [kCsXBuf][4 lane quarters]
+constexpr int kCsXBuf = 3;
+constexpr int kCsXchBytes = kCsXBuf * kScoreGroups * 128 * 4 + kCsXBuf * 4 * 4;
 __host__ __device__ inline CsLayout cs_layout(int R) {
   CsLayout L;
   L.NQ = R > 256 ? (R + 63) & ~63 : (R + 31) & ~31;
@@ -636,7 +640,7 @@ __host__ __device__ inline CsLayout cs_layout(int R) {
 // NH: column halves per key tile (cs_layout's nh), a template parameter so
 // that the one-half loop compiles away.
 template <int NH>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __maxnreg__(kScoreMaxReg)
     k_colsum_umma(const __grid_constant__ KMaps maps, const __grid_constant__ LayerPtrs io, Problem p,
                   Strided<float2> part_all, int nsplit, Strided<float> a_all, uint32_t* err) {
   extern __shared__ uint8_t smem_raw[];
@@ -661,8 +665,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int S = L.kstages;
   const float c = kLog2eF * rsqrtf((float)kD);
   float* xch = reinterpret_cast<float*>(sm + L.off_xch);
-  uint64_t* xbars = reinterpret_cast<uint64_t*>(sm + L.off_xch + 2 * 128 * 4);
-  const uint32_t b_xfull = smem_u32(&xbars[0]), b_xempty = smem_u32(&xbars[2]);
+  uint32_t* xcnt = reinterpret_cast<uint32_t*>(sm + L.off_xch + kCsXBuf * kScoreGroups * 128 * 4);
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < S; ++i) {
@@ -671,10 +674,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(b_accfull + 8 * i, 1);
-      mbar_init(b_accempty + 8 * i, 8);  // both epilogue groups
-      mbar_init(b_xfull + 8 * i, 4);
-      mbar_init(b_xempty + 8 * i, 4);
+      mbar_init(b_accempty + 8 * i, 4 * kScoreGroups);  // every epilogue warp
     }
+    for (int i = 0; i < kCsXBuf * 4; ++i) xcnt[i] = 0u;
     mbar_init(b_done, 1);
     *abort_flag = 0u;
     fence_mbar_init();
@@ -759,14 +761,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_wait_drain(b_done, 0);
     }
   } else {
-    // Both groups drain every item: group 0 the item's query columns
-    // [0, sp), group 1 [sp, W); columns of padded rows carry bias = -inf, so
-    // they add exact zeros.  A thread's sum runs over the tile's nh items;
-    // group 1 then passes it to group 0 through a double-buffered shared
-    // array (xfull / xempty barriers).
+    // Every group drains every item: group g the item's query columns
+    // [c0, c1), at most 64; columns of padded rows carry bias = -inf, so
+    // they add exact zeros.  A thread's sum runs over the tile's nh items.
+    // The groups' partial sums of a tile meet in shared buffer it % kCsXBuf:
+    // each warp adds one to its lane quarter's arrival counter, and the
+    // warp that arrives last (old value 3 mod 4) adds the four partials in
+    // group order and stores A_base.  Nobody waits for the hand-off.  A
+    // buffer is rewritten at tile it + kCsXBuf, which the MMA can only have
+    // produced once every warp has loaded tile it + 1 from TMEM, i.e. has
+    // finished with tile it.
     const int g = (warp - 2) >> 2, quarter = warp & 3, row = quarter * 32 + lane;
-    const int sp = min(W, ((W >> 1) + 63) & ~63);
-    const int c0 = g == 0 ? 0 : sp, c1 = g == 0 ? sp : W;
+    const int gwid = (((W + kScoreGroups - 1) / kScoreGroups) + 31) & ~31;
+    const int c0 = min(W, g * gwid), c1 = min(W, c0 + gwid);
     const uint32_t lanebase = tmem + ((uint32_t)(quarter * 32) << 16);
     bool ok = true;
     for (int it = 0; ok && it < ntiles; ++it) {
@@ -779,14 +786,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         tc_fence_after();
-        const uint32_t tbase = lanebase + as * W;
-        const float* bias_h = bias_s + hh * W;
-        int cb = c0;
-#pragma unroll 1
-        for (; cb + 64 <= c1; cb += 64) {
+        const uint32_t tb = lanebase + as * W + c0;
+        const float4* b4 = reinterpret_cast<const float4*>(bias_s + hh * W + c0);
+        if (c1 - c0 == 64) {
           float v[64];
-          tmem_ld64(tbase + cb, v);
-          const float4* b4 = reinterpret_cast<const float4*>(bias_h + cb);
+          tmem_ld64(tb, v);
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(b_accempty + 8 * as);
           // three phases over the chunk (exponent arguments, exponentials,
           // sums), so that independent work separates dependent instructions
 #pragma unroll
@@ -802,41 +809,45 @@ __global__ void __launch_bounds__(kThreads, 1)
             add2(a0, a1, v[4 * i], v[4 * i + 1]);
             add2(a2, a3, v[4 * i + 2], v[4 * i + 3]);
           }
-        }
-        if (c1 - cb == 32) {
+        } else if (c1 - c0 == 32) {
           float v[32];
-          tmem_ld32(tbase + cb, v);
-          const float4* b4 = reinterpret_cast<const float4*>(bias_h + cb);
+          tmem_ld32(tb, v);
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(b_accempty + 8 * as);
 #pragma unroll
           for (int i = 0; i < 8; ++i) {
             const float4 b = b4[i];
-            float x0, x1, x2, x3;
-            fma2(v[4 * i], v[4 * i + 1], c, c, b.x, b.y, x0, x1);
-            fma2(v[4 * i + 2], v[4 * i + 3], c, c, b.z, b.w, x2, x3);
-            add2(a0, a1, ex2_approx(x0), ex2_approx(x1));
-            add2(a2, a3, ex2_approx(x2), ex2_approx(x3));
+            fma2(v[4 * i], v[4 * i + 1], c, c, b.x, b.y, v[4 * i], v[4 * i + 1]);
+            fma2(v[4 * i + 2], v[4 * i + 3], c, c, b.z, b.w, v[4 * i + 2], v[4 * i + 3]);
           }
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] = ex2_approx(v[i]);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            add2(a0, a1, v[4 * i], v[4 * i + 1]);
+            add2(a2, a3, v[4 * i + 2], v[4 * i + 3]);
+          }
+        } else {
+          __syncwarp();
+          if (lane == 0) mbar_arrive(b_accempty + 8 * as);
         }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(b_accempty + 8 * as);
       }
       if (!ok) break;
-      float acc = (a0 + a1) + (a2 + a3);
-      const int xb = it & 1;
-      const uint32_t ux = (uint32_t)(it >> 1);
-      if (g == 1) {
-        if (!warp_wait(b_xempty + 8 * xb, (ux & 1u) ^ 1u, err, abort_flag)) break;
-        __syncwarp();  // the lanes' accesses follow lane 0's acquire
-        xch[xb * 128 + row] = acc;
-        __syncwarp();
-        if (lane == 0) mbar_arrive(b_xfull + 8 * xb);
-      } else {
-        if (!warp_wait(b_xfull + 8 * xb, ux & 1u, err, abort_flag)) break;
-        __syncwarp();
-        acc += xch[xb * 128 + row];
-        __syncwarp();
-        if (lane == 0) mbar_arrive(b_xempty + 8 * xb);
+      const int xb = it % kCsXBuf;
+      float* xp = xch + xb * (kScoreGroups * 128);
+      xp[g * 128 + row] = (a0 + a1) + (a2 + a3);
+      __syncwarp();
+      uint32_t last = 0u;
+      if (lane == 0) {
+        __threadfence_block();
+        last = (atomicAdd(&xcnt[xb * 4 + quarter], 1u) & 3u) == 3u ? 1u : 0u;
+        __threadfence_block();
+      }
+      last = __shfl_sync(0xffffffffu, last, 0);
+      __syncwarp();
+      if (last) {
+        const float acc = (xp[row] + xp[128 + row]) + (xp[256 + row] + xp[384 + row]);
         const int tok = (blockIdx.x + it * gridDim.x) * 128 + row;
         if (tok < n) a_base[(size_t)h * n + tok] = acc;
       }
@@ -1230,13 +1241,13 @@ cudaError_t launch_score_umma(const Problem& p, const LayerPtrs& io, Strided<flo
     return e;
   {
     TimingScope ts("rowstats_umma", st);
-    rs_kernel<<<dim3(nsplit, p.L * p.hkv), kRsThreads, L1.total, st>>>(m1, io, p, nsplit, rowpart, err);
+    rs_kernel<<<dim3(nsplit, p.L * p.hkv), kScoreThreads, L1.total, st>>>(m1, io, p, nsplit, rowpart, err);
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const int tiles = (p.n + 127) / 128;
   const int gx = pick_split(p.L * p.hkv, tiles, sm_count());
   TimingScope ts("colsum_umma", st);
-  cs_kernel<<<dim3(gx, p.L * p.hkv), kThreads, L2.total, st>>>(m2, io, p, rowpart, nsplit, a_base, err);
+  cs_kernel<<<dim3(gx, p.L * p.hkv), kScoreThreads, L2.total, st>>>(m2, io, p, rowpart, nsplit, a_base, err);
   return cudaGetLastError();
 }
 
