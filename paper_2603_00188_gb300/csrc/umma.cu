@@ -32,17 +32,17 @@ struct KMaps {
   CUtensorMap m[kMaxLayers];
 };
 
-// Q rows of KV head h into shared memory in the K-major 128B-swizzle layout
-// [2 K-halves][rows][128 B]; row r = window row * G + group member; rows past
-// R are zero.
+// Q rows [r0, r0 + rows) of KV head h into shared memory in the K-major
+// 128B-swizzle layout [2 K-halves][rows][128 B]; query row r = window row *
+// G + group member; rows past R are zero.
 __device__ __forceinline__ void load_q_sw128(uint8_t* sq, int rows, const __nv_bfloat16* q,
-                                             const Problem& p, int h) {
+                                             const Problem& p, int h, int r0 = 0) {
   const int G = p.G(), R = p.R();
   for (int e = threadIdx.x; e < rows * 16; e += blockDim.x) {
     int row = e >> 4, c16 = e & 15, kb = c16 >> 3, cc = c16 & 7;
     uint4 val = make_uint4(0, 0, 0, 0);
-    if (row < R) {
-      int wr = row / G, g = row - wr * G;
+    if (r0 + row < R) {
+      int wr = (r0 + row) / G, g = (r0 + row) - wr * G;
       val = __ldg(reinterpret_cast<const uint4*>(q + ((size_t)wr * p.hq + h * G + g) * kD + c16 * 8));
     }
     *reinterpret_cast<uint4*>(sq + (size_t)kb * rows * 128 + row * 128 + ((cc ^ (row & 7)) << 4)) = val;
@@ -308,13 +308,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // =========================================================================
-// Window score pass 1.  CTA (split, h): Q of head h (R rows, MT M-tiles of
-// 128) stays in shared memory as the A operand; key tiles of KN keys (256
-// for MT <= 2, else 128) stream as the B operand.  TMEM: two slots of 256
-// columns, one (m-tile, key tile) item each; every epilogue group drains a
-// quarter of each item's keys and keeps, per query row, the running max m
-// (raw dot units) and l = sum 2^((x - m) c).  The groups merge at the end;
-// part[h][split][r] = (m c, l).
+// Window score pass 1.  CTA (split * NMH + mh, h): query rows [256 mh,
+// 256 mh + 128 MT) of head h (MT <= 2 m-tiles of 128) stay in shared memory
+// as the A operand; key tiles of 256 keys stream as the B operand.  TMEM:
+// two slots of 256 columns, one (m-tile, key tile) item each; every
+// epilogue group drains a quarter of each item's keys and keeps, per query
+// row, the running max m (raw dot units) and l = sum 2^((x - m) c).  The
+// groups merge at the end; part[h][split][r] = (m c, l).
 constexpr int kMaxKStages = 4;        // key-tile ring depth (as shared memory allows)
 constexpr int kScoreSmemCap = 200 * 1024;
 
@@ -347,13 +347,19 @@ constexpr int kScoreThreads = (2 + 4 * kScoreGroups) * 32;
 constexpr int kScoreMaxReg = 96;
 static_assert(kScoreGroups == 4, "the column sums add four partial sums per key");
 
+// NMH CTAs share a key split, each holding MT m-tiles of Q (query rows
+// [256 mh, 256 mh + 128 MT)): for R > 256 two CTAs read the same key tiles
+// at about the same time (adjacent in the grid, so the second read mostly
+// hits L2) instead of one CTA with all of Q, whose 128 KB would leave room
+// only for 128-key tiles.
 struct RsLayout {
-  int MT, KN, q_bytes, k_stage_bytes, kstages, off_k, off_bar, off_xch, total;
+  int MT, NMH, KN, q_bytes, k_stage_bytes, kstages, off_k, off_bar, off_xch, total;
 };
 __host__ __device__ inline RsLayout rs_layout(int R) {
   RsLayout L;
-  L.MT = R <= 128 ? 1 : (R <= 256 ? 2 : 4);
-  L.KN = L.MT <= 2 ? 256 : 128;  // keys per tile = MMA N of one (m-tile, key tile) item
+  L.MT = R <= 128 ? 1 : 2;
+  L.NMH = R <= 256 ? 1 : 2;
+  L.KN = 256;  // keys per tile = MMA N of one (m-tile, key tile) item
   L.q_bytes = L.MT * 128 * 256;
   L.k_stage_bytes = L.KN * 256;
   const int xch = (kScoreGroups - 1) * L.MT * 128 * 8;
@@ -384,11 +390,12 @@ __global__ void __maxnreg__(kScoreMaxReg)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = align1024(smem_raw);
   const RsLayout L = rs_layout(p.R());
-  constexpr int KN = MT <= 2 ? 256 : 128;
-  constexpr int CW = KN / kScoreGroups;  // key columns per group and item (64 or 32)
+  constexpr int KN = 256;
+  constexpr int CW = KN / kScoreGroups;  // key columns per group and item
   const int R = p.R();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int split = blockIdx.x, layer = blockIdx.y / p.hkv, h = blockIdx.y % p.hkv, n = p.n;
+  const int split = blockIdx.x / L.NMH, r0 = (blockIdx.x % L.NMH) * 256;
+  const int layer = blockIdx.y / p.hkv, h = blockIdx.y % p.hkv, n = p.n;
   const CUtensorMap& kmap = maps.m[layer];
   const __nv_bfloat16* q = static_cast<const __nv_bfloat16*>(io.q[layer]);
   float2* part = part_all.at(layer);
@@ -424,7 +431,7 @@ __global__ void __maxnreg__(kScoreMaxReg)
     tmem_alloc(smem_u32(slot), 512);
     tmem_relinquish();
   }
-  load_q_sw128(sm, MT * 128, q, p, h);
+  load_q_sw128(sm, MT * 128, q, p, h, r0);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -500,13 +507,8 @@ __global__ void __maxnreg__(kScoreMaxReg)
       tc_fence_after();
       const int t = u / MT, mt = u % MT;
       uint32_t b[CW];
-      if constexpr (CW == 64) {
-        tmem_ld64_issue(lanebase + as * 256, b);
-        tmem_ld64_wait(b);
-      } else {
-        tmem_ld32_issue(lanebase + as * 256, b);
-        tmem_wait_regs32(b);
-      }
+      tmem_ld64_issue(lanebase + as * 256, b);
+      tmem_ld64_wait(b);
       // the item's TMEM columns are in registers: release the slot
       tc_fence_before();
       __syncwarp();
@@ -586,7 +588,7 @@ __global__ void __maxnreg__(kScoreMaxReg)
   if (warp >= 2 && g == 0) {
 #pragma unroll
     for (int mt = 0; mt < MT; ++mt) {
-      const int row = mt * 128 + quarter * 32 + lane;
+      const int row = r0 + mt * 128 + quarter * 32 + lane;
       float m = ms[mt], l = ls[mt];
       for (int o = 1; o < kScoreGroups; ++o) {
         const float2 v = xch[((o - 1) * MT + mt) * 128 + quarter * 32 + lane];
@@ -1191,7 +1193,8 @@ static int score_tiles(const Problem& p) {
 int score_nsplit_max(const Problem& p) {
   const int slots = p.dtype == kBF16 ? 152 : 2 * 152;
   const int tiles = score_tiles(p);
-  int s = pick_split(p.hkv, tiles, slots);
+  const int nmh = p.dtype == kBF16 ? rs_layout(p.R()).NMH : 1;
+  int s = pick_split(p.hkv * nmh, tiles, slots);
   // at least ~24 key tiles per split, so that a CTA's set-up (Q load,
   // barrier and TMEM set-up, pipeline fill) stays small next to its work
   const int fat = (tiles + 23) / 24;
@@ -1232,7 +1235,7 @@ cudaError_t launch_score_umma(const Problem& p, const LayerPtrs& io, Strided<flo
   cudaError_t e = make_kmaps(&m1, io, p.L, p.n, p.hkv, L1.KN);
   if (e != cudaSuccess) return e;
   if ((e = make_kmaps(&m2, io, p.L, p.n, p.hkv, 128)) != cudaSuccess) return e;
-  auto rs_kernel = L1.MT == 1 ? k_rowstats_umma<1> : (L1.MT == 2 ? k_rowstats_umma<2> : k_rowstats_umma<4>);
+  auto rs_kernel = L1.MT == 1 ? k_rowstats_umma<1> : k_rowstats_umma<2>;
   if ((e = cudaFuncSetAttribute(rs_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, L1.total)) !=
       cudaSuccess)
     return e;
@@ -1241,7 +1244,8 @@ cudaError_t launch_score_umma(const Problem& p, const LayerPtrs& io, Strided<flo
     return e;
   {
     TimingScope ts("rowstats_umma", st);
-    rs_kernel<<<dim3(nsplit, p.L * p.hkv), kScoreThreads, L1.total, st>>>(m1, io, p, nsplit, rowpart, err);
+    rs_kernel<<<dim3(nsplit * L1.NMH, p.L * p.hkv), kScoreThreads, L1.total, st>>>(m1, io, p, nsplit, rowpart,
+                                                                                     err);
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const int tiles = (p.n + 127) / 128;
