@@ -69,6 +69,15 @@ stlite_status build_frames(const stlite_shape* s, const stlite_frames* fr, Frame
     ft->cur_off = ft->off[F - 1];
     ft->cur_len = ft->gh[F - 1] * ft->gw[F - 1];
   }
+  if (F >= 2) {
+    // ragged frames waste the rows of each frame's last tile; spanning tiles
+    // waste the text rows between frames instead: take the fewer tiles
+    ft->tsg_off = ft->off[0];
+    ft->tsg_end = ft->off[F - 2] + ft->gh[F - 2] * ft->gw[F - 2];
+    const int span = (ft->tsg_end - ft->tsg_off + kTsgTile - 1) / kTsgTile;
+    ft->tsg_span = span < ft->tile0[F - 1] ? 1 : 0;
+    ft->tsg_tiles = ft->tsg_span ? span : ft->tile0[F - 1];
+  }
   return STLITE_OK;
 }
 

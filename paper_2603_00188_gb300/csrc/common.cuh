@@ -34,6 +34,13 @@ struct FrameTable {
   int32_t gw[kMaxFrames];
   int32_t tile0[kMaxFrames + 1];
   int32_t ctile0[kMaxFrames + 1];  // first 128-token CSS tile of every frame (all frames)
+  // Row tiles of the tensor-core TSG pass: per historical frame (tile0), or,
+  // when that takes more tiles, 128-token tiles spanning the whole range
+  // [tsg_off, tsg_end) of the historical frames, text tokens included (their
+  // rho slices are never read).
+  int32_t tsg_tiles;
+  int32_t tsg_span;  // 1: spanning tiles
+  int32_t tsg_off, tsg_end;
 };
 
 // Frame holding token j, or -1 for a text token (binary search on offsets).

@@ -59,8 +59,14 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, uint32_
   return __shfl_sync(0xffffffffu, ok, 0) != 0;
 }
 
-// First token of TSG row tile t and the end of its frame's visual span.
+// First token of TSG row tile t and the end of the rows it may write: its
+// frame's visual span, or the whole historical range for spanning tiles.
 __device__ __forceinline__ void tsg_tile(const FrameTable& ft, int t, int& tok0, int& fend) {
+  if (ft.tsg_span) {
+    tok0 = ft.tsg_off + t * kTsgTile;
+    fend = ft.tsg_end;
+    return;
+  }
   int lo = 0, hi = ft.n_frames - 2, f = 0;
   while (lo <= hi) {
     int mid = (lo + hi) >> 1;
@@ -108,7 +114,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const CUtensorMap& kmap = maps.m[l];
   const float* rn_cur = rc_all.at(l) + (size_t)h * cur_pad;  // 16-byte aligned rows
   float* rho_part = rho_all.at(l);
-  const int n_tiles = ft.tile0[ft.n_frames - 1];
+  const int n_tiles = ft.tsg_tiles;
   const int col0 = chunk * 512;
   const int valid = min(512, ft.cur_len - col0);
   const int nst = valid > 256 ? 2 : 1;
@@ -1208,7 +1214,7 @@ cudaError_t launch_tsg_umma(const Problem& p, const FrameTable& ft, const LayerP
                             Strided<const float> rn_cur, int cur_pad, Strided<float> rho_part, int metric,
                             uint32_t* err, cudaStream_t st) {
   if (ft.n_frames < 2) return cudaSuccess;
-  const int n_tiles = ft.tile0[ft.n_frames - 1];
+  const int n_tiles = ft.tsg_tiles;
   if (n_tiles == 0 || ft.cur_len == 0) return cudaSuccess;
   const int nchunk = (ft.cur_len + 511) / 512;
   KMaps local;

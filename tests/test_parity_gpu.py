@@ -588,6 +588,17 @@ def test_edge_query_rows_512(st):
     _run_edge(st, wl, 0.25)
 
 
+def test_edge_query_rows_ragged_second_half(st):
+    # R = 33 x 9 = 297: pass 1 runs two CTAs per key split, the second with
+    # 41 valid rows in its first M-tile and none in its second; pass 2 runs
+    # two column halves of 160 whose last epilogue group has no columns
+    wl = synth.trajectory(n_steps=3, gh=5, gw=6, n_text=7, hq=9, hkv=1, w=33, beta=0.25, seed=(967,))
+    _run_edge(st, wl, 0.25)
+    # R = 129 x 2 = 258: two rows past the one-CTA limit
+    wl = synth.trajectory(n_steps=2, gh=4, gw=5, n_text=3, hq=2, hkv=1, w=129, beta=0.3, seed=(968,))
+    _run_edge(st, wl, 0.3)
+
+
 def test_edge_one_query_head_per_group(st):
     # G = 1: every query head has its own KV head
     wl = synth.trajectory(n_steps=3, gh=5, gw=9, n_text=3, hq=4, hkv=4, w=16, beta=0.3, seed=(964,))
