@@ -48,6 +48,44 @@ def test_decode_matches_oracle(st, w, hq, hkv, n, dtype):
     _close(out.cpu().numpy().astype(np.float64), ref, exact64(v))
 
 
+def test_decode_workspace_reused(st):
+    # one workspace serves many calls, eager and in a replayed graph, and
+    # every call equals a call on a fresh workspace, bit for bit
+    g = torch.Generator().manual_seed(977)
+    w, hq, hkv, n = 2, 28, 4, 3000
+    k = torch.randn((n, hkv, 128), generator=g).to(torch.bfloat16).cuda()
+    v = torch.randn((n, hkv, 128), generator=g).to(torch.bfloat16).cuda()
+    qs = [torch.randn((w, hq, 128), generator=g).to(torch.bfloat16).cuda() for _ in range(3)]
+    sh = st.make_shape(qs[0], k)
+    nbytes = st.stlite_decode_workspace_size(sh)
+    ws = torch.zeros(nbytes, dtype=torch.uint8, device="cuda")
+    outs = []
+    for q in qs + qs:
+        out = torch.empty((w, hq, 128), dtype=torch.float32, device="cuda")
+        st.stlite_decode_attention(q, k, v, out, ws)
+        outs.append(out)
+    torch.cuda.synchronize()
+    for i, q in enumerate(qs):
+        fresh = torch.empty((w, hq, 128), dtype=torch.float32, device="cuda")
+        st.stlite_decode_attention(q, k, v, fresh, torch.zeros(nbytes, dtype=torch.uint8, device="cuda"))
+        torch.cuda.synchronize()
+        assert torch.equal(outs[i], fresh) and torch.equal(outs[i + 3], fresh)
+    out = torch.empty((w, hq, 128), dtype=torch.float32, device="cuda")
+    stream = torch.cuda.Stream()
+    with torch.cuda.stream(stream):
+        st.stlite_decode_attention(qs[1], k, v, out, ws, stream=stream)
+    stream.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        st.stlite_decode_attention(qs[1], k, v, out, ws, stream=stream)
+    for _ in range(4):
+        out.zero_()
+        graph.replay()
+    torch.cuda.synchronize()
+    assert torch.equal(out, outs[1])
+    assert st.stlite_device_status(ws) == st.STLITE_OK
+
+
 def test_decode_over_compressed_cache(st):
     # compress one layer, then decode a probe row over the compacted rows
     wl = synth.scaled("traj50", 4)
