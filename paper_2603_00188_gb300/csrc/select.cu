@@ -162,6 +162,16 @@ __device__ uint32_t cluster_select_desc(cg::cluster_group& cl, const uint32_t* k
   return prefix;
 }
 
+// Warms L2 with the 128-byte lines of x[j0, j1) (one prefetch per line):
+// the token loops then find their inputs in L2 instead of waiting on DRAM
+// once per batch.
+__device__ __forceinline__ void prefetch_l2(const void* x, size_t elem, int j0, int j1) {
+  const char* b = static_cast<const char*>(x);
+  const size_t lo = (size_t)j0 * elem, hi = (size_t)j1 * elem;
+  for (size_t o = (lo & ~(size_t)127) + (size_t)threadIdx.x * 128; o < hi; o += (size_t)blockDim.x * 128)
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(b + o));
+}
+
 // Inputs of one pool token's rho: the row maxima of the TSG slices (folded
 // into four) and 1/|k_i|.
 struct RhoIn {
@@ -237,6 +247,8 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
     const float* rn = a.rn.at(l) + hn;
     const size_t slice = (size_t)p.hkv * n;
     const int nsl = a.nchunk;
+    for (int s = 0; s < nsl; ++s) prefetch_l2(rp + (size_t)s * slice, 4, j0, j1);
+    prefetch_l2(rn, 4, j0, j1);
     // rho of every token: pool tokens from the TSG slices and 1/|k_i|, NaN
     // elsewhere; the selection keys are complements (m-th smallest rho ==
     // m-th largest key), 0 marks a token outside the pool
@@ -270,6 +282,9 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
           keys[t - j0] = kind == kTokPool ? ~float_key(r) : 0u;
         });
     __syncthreads();
+    // the score phase's inputs arrive in L2 while tau is selected
+    if ((a.mode & kSelTopk) && !a.base_uniform) prefetch_l2(a.a_base.at(l) + hn, 4, j0, j1);
+    if ((a.mode & kSelTopk) && a.phi.base && a.css_enable) prefetch_l2(a.phi.at(l) + hn, 4, j0, j1);
     if (gate_sel) {
       if (a.tsg_fixed) {
         tau = a.tsg_fixed_tau;  // fixed-threshold control: no selection
