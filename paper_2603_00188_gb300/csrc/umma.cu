@@ -1083,34 +1083,75 @@ __global__ void __launch_bounds__(kThreads, 1)
 // Phi from the per-token dots: the eight in-grid Moore neighbours of (u, v)
 // are E, W, S, N, SE, NW, SW, NE; W's dot is E of the left neighbour, N's is
 // S of the upper one, NW's is SE of the upper-left one and NE's is SW of the
-// upper-right one.  grid = (cell block, frame, layer*Hkv + head).
+// upper-right one.  A thread takes kPhiRun consecutive cells of one grid
+// row, so that the index arithmetic and the loads of the shared neighbours
+// are done once per run.  grid = (run block, frame, layer*Hkv + head).
+constexpr int kPhiRun = 4;
 __global__ void __launch_bounds__(256) k_css_phi(const __grid_constant__ FrameTable ft, int hkv, CssDots d,
                                                  Strided<float> phi_all) {
   const int f = blockIdx.y, l = blockIdx.z / hkv, h = blockIdx.z % hkv, n = ft.n_tokens;
   if (f >= ft.n_frames) return;
   const int gh = ft.gh[f], gw = ft.gw[f], off = ft.off[f];
-  const int cell = blockIdx.x * blockDim.x + threadIdx.x;
-  if (cell >= gh * gw) return;
+  const int runs = (gw + kPhiRun - 1) / kPhiRun;  // runs per grid row
+  const int slot = blockIdx.x * blockDim.x + threadIdx.x;
+  if (slot >= gh * runs) return;
+  const int u = slot / runs, v0 = (slot - u * runs) * kPhiRun;
   const size_t hn = (size_t)h * n;
   const float* rn = d.rn.at(l) + hn;
   const float* e = d.dE.at(l) + hn;
   const float* s = d.dS.at(l) + hn;
   const float* se = d.dSE.at(l) + hn;
   const float* sw = d.dSW.at(l) + hn;
-  const int u = cell / gw, v = cell - u * gw, j = off + cell;
-  const bool up = u > 0, dn = u + 1 < gh, lf = v > 0, rt = v + 1 < gw;
-  const float r0 = __ldg(rn + j);
-  float sum = 0.f;
-  int cnt = 0;
-  if (rt) { sum += __ldg(e + j) * r0 * __ldg(rn + j + 1); ++cnt; }
-  if (lf) { sum += __ldg(e + j - 1) * __ldg(rn + j - 1) * r0; ++cnt; }
-  if (dn) { sum += __ldg(s + j) * r0 * __ldg(rn + j + gw); ++cnt; }
-  if (up) { sum += __ldg(s + j - gw) * __ldg(rn + j - gw) * r0; ++cnt; }
-  if (dn && rt) { sum += __ldg(se + j) * r0 * __ldg(rn + j + gw + 1); ++cnt; }
-  if (up && lf) { sum += __ldg(se + j - gw - 1) * __ldg(rn + j - gw - 1) * r0; ++cnt; }
-  if (dn && lf) { sum += __ldg(sw + j) * r0 * __ldg(rn + j + gw - 1); ++cnt; }
-  if (up && rt) { sum += __ldg(sw + j - gw + 1) * __ldg(rn + j - gw + 1) * r0; ++cnt; }
-  phi_all.at(l)[hn + j] = cnt ? 1.0f - sum / (float)cnt : 0.0f;
+  const bool up = u > 0, dn = u + 1 < gh;
+  const int j0 = off + u * gw + v0;  // token of cell (u, v0)
+  // columns v0 - 1 .. v0 + kPhiRun of the rows above, at and below: index
+  // c + 1 holds column v0 + c (loads outside the grid are skipped)
+  float ra[kPhiRun + 2], rc[kPhiRun + 2], rb[kPhiRun + 2];
+  float ec[kPhiRun + 1], sa[kPhiRun], sc[kPhiRun], sea[kPhiRun + 1], sec[kPhiRun], swa[kPhiRun + 1], swc[kPhiRun];
+#pragma unroll
+  for (int c = -1; c <= kPhiRun; ++c) {
+    const int v = v0 + c;
+    const bool in = v >= 0 && v < gw;
+    rc[c + 1] = in ? __ldg(rn + j0 + c) : 0.f;
+    ra[c + 1] = in && up ? __ldg(rn + j0 + c - gw) : 0.f;
+    rb[c + 1] = in && dn ? __ldg(rn + j0 + c + gw) : 0.f;
+  }
+#pragma unroll
+  for (int c = -1; c < kPhiRun; ++c) {
+    const int v = v0 + c;
+    const bool in = v >= 0 && v < gw;
+    ec[c + 1] = in ? __ldg(e + j0 + c) : 0.f;                    // E of (u, v)
+    sea[c + 1] = in && up ? __ldg(se + j0 + c - gw) : 0.f;       // SE of (u - 1, v)
+    const bool in2 = v + 2 >= 0 && v + 2 < gw;
+    swa[c + 1] = in2 && up ? __ldg(sw + j0 + c + 2 - gw) : 0.f;  // SW of (u - 1, v + 2)
+  }
+#pragma unroll
+  for (int c = 0; c < kPhiRun; ++c) {
+    const bool in = v0 + c < gw;
+    sa[c] = in && up ? __ldg(s + j0 + c - gw) : 0.f;
+    sc[c] = in && dn ? __ldg(s + j0 + c) : 0.f;
+    sec[c] = in && dn ? __ldg(se + j0 + c) : 0.f;
+    swc[c] = in && dn ? __ldg(sw + j0 + c) : 0.f;
+  }
+  float* phi = phi_all.at(l) + hn;
+#pragma unroll
+  for (int c = 0; c < kPhiRun; ++c) {
+    const int v = v0 + c;
+    if (v >= gw) break;
+    const bool lf = v > 0, rt = v + 1 < gw;
+    const float r0 = rc[c + 1];
+    float sum = 0.f;
+    int cnt = 0;
+    if (rt) { sum += ec[c + 1] * r0 * rc[c + 2]; ++cnt; }
+    if (lf) { sum += ec[c] * rc[c] * r0; ++cnt; }
+    if (dn) { sum += sc[c] * r0 * rb[c + 1]; ++cnt; }
+    if (up) { sum += sa[c] * ra[c + 1] * r0; ++cnt; }
+    if (dn && rt) { sum += sec[c] * r0 * rb[c + 2]; ++cnt; }
+    if (up && lf) { sum += sea[c] * ra[c] * r0; ++cnt; }
+    if (dn && lf) { sum += swc[c] * r0 * rb[c]; ++cnt; }
+    if (up && rt) { sum += swa[c] * ra[c + 2] * r0; ++cnt; }
+    phi[j0 + c] = cnt ? 1.0f - sum / (float)cnt : 0.0f;
+  }
 }
 
 // =========================================================================
@@ -1302,8 +1343,8 @@ cudaError_t launch_css_umma(const Problem& p, const FrameTable& ft, const LayerP
     k_css_umma<<<dim3(gx, p.L * p.hkv), kThreads, geo.smem, st>>>(maps, ft, p.hkv, d, geo, err);
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  int cmax = 1;
-  for (int f = 0; f < ft.n_frames; ++f) cmax = max(cmax, ft.gh[f] * ft.gw[f]);
+  int cmax = 1;  // the most kPhiRun-cell runs of any frame
+  for (int f = 0; f < ft.n_frames; ++f) cmax = max(cmax, ft.gh[f] * ((ft.gw[f] + kPhiRun - 1) / kPhiRun));
   TimingScope ts("css_phi", st);
   k_css_phi<<<dim3((cmax + 255) / 256, ft.n_frames, p.L * p.hkv), 256, 0, st>>>(ft, p.hkv, d, phi);
   return cudaGetLastError();
