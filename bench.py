@@ -271,12 +271,38 @@ def run_reference(args):
 
 # ----------------------------------------------------------------- GPU arm
 
+def _code_only(text: str) -> str:
+    """C/C++/CUDA source without its comments (string and character literals
+    kept) and with every run of white space made one blank, so that editing
+    a comment or reflowing lines does not mark counters as stale."""
+    out, i, n = [], 0, len(text)
+    while i < n:
+        if text.startswith("//", i):
+            j = text.find("\n", i)
+            i = n if j < 0 else j
+        elif text.startswith("/*", i):
+            j = text.find("*/", i + 2)
+            i = n if j < 0 else j + 2
+        elif text[i] in "\"'":
+            q, j = text[i], i + 1
+            while j < n and text[j] != q:
+                j += 2 if text[j] == "\\" else 1
+            out.append(text[i:j + 1])
+            i = j + 1
+        else:
+            out.append(text[i])
+            i += 1
+    return " ".join("".join(out).split())
+
+
 def src_digest():
+    """Digest of the kernel sources (comments excluded) the committed ncu
+    counters must have been taken on."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2603_00188_gb300", "csrc")
     for name in sorted(os.listdir(csrc)):
-        with open(os.path.join(csrc, name), "rb") as f:
-            h.update(name.encode() + f.read())
+        with open(os.path.join(csrc, name), encoding="utf-8") as f:
+            h.update(name.encode() + _code_only(f.read()).encode())
     return h.hexdigest()[:16]
 
 

@@ -612,11 +612,12 @@ __global__ void __maxnreg__(kScoreMaxReg)
 // =========================================================================
 // Window score pass 2.  CTA (x, h): key tiles of 128 tokens are the A operand
 // (M = 128, one key per TMEM lane), Q of head h (NQ = R rounded up to 32
-// rows) is the B operand.  Each thread sums 2^(x_r c + bias_r) over the R
-// query rows of its key.  TMEM: two slots of W columns, so that one item
-// drains while the next one is computed.  An item is a key tile against
-// all NQ query columns (W = NQ <= 256), or against one of nh = 2 column
-// halves (NQ > 256, rounded to 64, W = NQ / 2).
+// rows) is the B operand.  Each epilogue thread sums 2^(x_r c + bias_r) for
+// its key over its group's range of at most 64 query rows; the four groups'
+// partial sums meet in shared memory.  TMEM: two slots of W columns, so that
+// one item drains while the next one is computed.  An item is a key tile
+// against all NQ query columns (W = NQ <= 256), or against one of nh = 2
+// column halves (NQ > 256, rounded to 64, W = NQ / 2).
 struct CsLayout {
   int NQ, nh, W, nstage, kstages, tmem_cols, q_bytes, off_k, off_bias, off_bar, off_xch, total;
 };
