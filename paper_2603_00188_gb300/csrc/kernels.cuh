@@ -107,10 +107,14 @@ cudaError_t launch_score(const Problem& p, const LayerPtrs& io, Strided<float2> 
                          Strided<float> a_base, uint32_t* err, cudaStream_t st);
 cudaError_t launch_score_umma(const Problem& p, const LayerPtrs& io, Strided<float2> rowpart,
                               int nsplit, Strided<float> a_base, uint32_t* err, cudaStream_t st);
-// Key splits of window-score pass 1 for this batch, and the largest value it
-// takes for any batch size (which sizes the workspace).
+// Key splits of window-score pass 1 (the partials it writes per query row);
+// they depend on the shape alone, so that a layer gives the same bits alone
+// or batched.  score_nsplit_max sizes the workspace.
 int score_nsplit(const Problem& p);
 int score_nsplit_max(const Problem& p);
+// Merges pass 1's split partials into the row bias -m_r - log2(G l_r) that
+// follows them in rowpart ([Hkv][R] float per layer).
+void launch_row_bias(const Problem& p, int nsplit, Strided<float2> rowpart, cudaStream_t st);
 
 // TSG partial row maxima: rho_part[l][s][h][i] = max over the current-frame
 // columns of 256-column slice s of k_i.k_j * rn_j, for historical visual

@@ -506,23 +506,37 @@ __global__ void __launch_bounds__(kRsRows) k_rowstats_simt(const __grid_constant
 }
 
 // Merge the splits: bias[h][r] = -m_r - log2(G * l_r), so that
-// 2^(x + bias) = softmax probability / G.  grid.y = layer.
-__global__ void k_row_bias(Problem p, int nsplit, Strided<float2> part_all) {
+// 2^(x + bias) = softmax probability / G.  One thread per row (consecutive
+// rows, coalesced loads), one pass in split order with eight partials in
+// flight: (M, L) <- (max(M, m_s), L 2^(M - M') + l_s 2^(m_s - M')).
+// grid.y = layer.
+__global__ void __launch_bounds__(128) k_row_bias(Problem p, int nsplit, Strided<float2> part_all) {
   const int R = p.R(), l = blockIdx.y;
   const float2* part = part_all.at(l);
   float* bias = reinterpret_cast<float*>(part_all.at(l) + (size_t)p.hkv * nsplit * R);
-  int e = blockIdx.x * blockDim.x + threadIdx.x;
+  const int e = blockIdx.x * blockDim.x + threadIdx.x;
   if (e >= p.hkv * R) return;
-  int h = e / R, r = e - h * R;
+  const int h = e / R, r = e - h * R;
   const float2* pp = part + (size_t)h * nsplit * R + r;
-  float m = -CUDART_INF_F;
-  for (int s = 0; s < nsplit; ++s) m = fmaxf(m, pp[(size_t)s * R].x);
-  float lsum = 0.f;
-  for (int s = 0; s < nsplit; ++s) {
-    float2 v = pp[(size_t)s * R];
-    if (v.y > 0.f) lsum += v.y * exp2f(v.x - m);
+  float m = -CUDART_INF_F, lsum = 0.f;
+  for (int s0 = 0; s0 < nsplit; s0 += 8) {
+    float2 v[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) v[u] = s0 + u < nsplit ? pp[(size_t)(s0 + u) * R] : make_float2(-CUDART_INF_F, 0.f);
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      if (!(v[u].y > 0.f)) continue;
+      const float mn = fmaxf(m, v[u].x);
+      lsum = (lsum > 0.f ? lsum * exp2f(m - mn) : 0.f) + v[u].y * exp2f(v[u].x - mn);
+      m = mn;
+    }
   }
   bias[e] = -m - log2f((float)p.G() * lsum);
+}
+
+void launch_row_bias(const Problem& p, int nsplit, Strided<float2> rowpart, cudaStream_t st) {
+  const int rows = p.hkv * p.R();
+  k_row_bias<<<dim3((rows + 127) / 128, p.L), 128, 0, st>>>(p, nsplit, rowpart);
 }
 
 // ---------------------------------------------------------- column sums
@@ -605,8 +619,7 @@ cudaError_t launch_score(const Problem& p, const LayerPtrs& io, Strided<float2> 
   if (e != cudaSuccess) return e;
   {
     TimingScope ts("row_bias", st);
-    int tot = p.hkv * p.R();
-    k_row_bias<<<dim3((tot + 127) / 128, p.L), 128, 0, st>>>(p, nsplit, rowpart);
+    launch_row_bias(p, nsplit, rowpart, st);
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   TimingScope ts("colsum_simt", st);

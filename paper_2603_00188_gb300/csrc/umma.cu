@@ -358,6 +358,7 @@ static_assert(kScoreGroups == 4, "the column sums add four partial sums per key"
 // at about the same time (adjacent in the grid, so the second read mostly
 // hits L2) instead of one CTA with all of Q, whose 128 KB would leave room
 // only for 128-key tiles.
+constexpr int kRsXBuf = 3;
 struct RsLayout {
   int MT, NMH, KN, q_bytes, k_stage_bytes, kstages, off_k, off_bar, off_xch, total;
 };
@@ -368,7 +369,9 @@ __host__ __device__ inline RsLayout rs_layout(int R) {
   L.KN = 256;  // keys per tile = MMA N of one (m-tile, key tile) item
   L.q_bytes = L.MT * 128 * 256;
   L.k_stage_bytes = L.KN * 256;
-  const int xch = (kScoreGroups - 1) * L.MT * 128 * 8;
+  // split-end exchange: kRsXBuf buffers of every group's (m, l) per row,
+  // then kRsXBuf x 4 arrival counters
+  const int xch = kRsXBuf * kScoreGroups * L.MT * 128 * 8 + kRsXBuf * 4 * 4;
   const int fixed = L.q_bytes + kScoreBarBytes + xch + 1024;
   L.kstages = (kScoreSmemCap - fixed) / L.k_stage_bytes;
   if (L.kstages > kMaxKStages) L.kstages = kMaxKStages;
@@ -392,7 +395,7 @@ __device__ __forceinline__ void online_merge(float& m, float& l, float m2, float
 template <int MT>
 __global__ void __maxnreg__(kScoreMaxReg)
     k_rowstats_umma(const __grid_constant__ KMaps maps, const __grid_constant__ LayerPtrs io, Problem p,
-                    int nsplit, Strided<float2> part_all, uint32_t* err) {
+                    int nsplit, int cps, Strided<float2> part_all, uint32_t* err) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = align1024(smem_raw);
   const RsLayout L = rs_layout(p.R());
@@ -400,14 +403,18 @@ __global__ void __maxnreg__(kScoreMaxReg)
   constexpr int CW = KN / kScoreGroups;  // key columns per group and item
   const int R = p.R();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int split = blockIdx.x / L.NMH, r0 = (blockIdx.x % L.NMH) * 256;
+  // this CTA's key splits [s0, s0 + cps) of `per_t` tiles each (the last
+  // split of the head may be shorter)
+  const int s0 = (blockIdx.x / L.NMH) * cps, r0 = (blockIdx.x % L.NMH) * 256;
   const int layer = blockIdx.y / p.hkv, h = blockIdx.y % p.hkv, n = p.n;
   const CUtensorMap& kmap = maps.m[layer];
   const __nv_bfloat16* q = static_cast<const __nv_bfloat16*>(io.q[layer]);
   float2* part = part_all.at(layer);
-  const int per = (((n + nsplit - 1) / nsplit) + KN - 1) / KN * KN;
-  const int j0 = split * per, j1 = min(n, j0 + per);
-  const int ntiles = j1 > j0 ? (j1 - j0 + KN - 1) / KN : 0;
+  const int tiles_all = (n + KN - 1) / KN;
+  const int per_t = (tiles_all + nsplit - 1) / nsplit;
+  const int t0 = min(tiles_all, s0 * per_t), t1 = min(tiles_all, (s0 + cps) * per_t);
+  const int j0 = t0 * KN, j1 = n;
+  const int ntiles = t1 - t0;
   const int nitems = ntiles * MT;
   const uint32_t sQ = smem_u32(sm), sK = smem_u32(sm + L.off_k);
   const ScoreBars bb = score_bars(sm + L.off_bar);
@@ -417,6 +424,7 @@ __global__ void __maxnreg__(kScoreMaxReg)
   volatile uint32_t* abort_flag = bb.abort_flag;
   const int S = L.kstages;
   float2* xch = reinterpret_cast<float2*>(sm + L.off_xch);
+  uint32_t* xcnt = reinterpret_cast<uint32_t*>(sm + L.off_xch + kRsXBuf * kScoreGroups * MT * 128 * 8);
   const float c = kLog2eF * rsqrtf((float)kD);
 
   if (threadIdx.x == 0) {
@@ -430,6 +438,7 @@ __global__ void __maxnreg__(kScoreMaxReg)
     }
     mbar_init(b_done, 1);
     *abort_flag = 0u;
+    for (int i = 0; i < kRsXBuf * 4; ++i) xcnt[i] = 0u;
     fence_mbar_init();
     tma_prefetch_desc(&kmap);
   }
@@ -448,8 +457,14 @@ __global__ void __maxnreg__(kScoreMaxReg)
   // item, group g taking key columns [g*CW, (g+1)*CW): four warps per SM
   // sub-partition hide one another's latencies, and one item drains while
   // the MMA fills the other slot.  Each group keeps a row state per m-tile,
-  // (running max m in raw dot units, l = sum 2^((x - m) c)); the groups'
-  // states are merged at the end.
+  // (running max m in raw dot units, l = sum 2^((x - m) c)).  At the end of
+  // every key split each warp parks its states in exchange buffer
+  // (split index in the CTA) % kRsXBuf and counts itself in; the warp that
+  // arrives last for its lane quarter merges the four groups' states in
+  // group order and writes the split's partial.  Nobody waits, and the
+  // partials depend on the shape alone, not on how many splits a CTA takes.
+  // A buffer is rewritten kRsXBuf splits (>= 3 items) later, which the MMA
+  // can only have produced once every warp has finished with it.
   float ms[MT], ls[MT];
 #pragma unroll
   for (int i = 0; i < MT; ++i) {
@@ -507,102 +522,132 @@ __global__ void __maxnreg__(kScoreMaxReg)
     }
   } else {
     const uint32_t lanebase = tmem + ((uint32_t)(quarter * 32) << 16) + g * CW;
+    // Every epilogue warp runs the same item sequence and the same split
+    // flushes (named barrier 1 of the 16 epilogue warps), also after a wait
+    // gave up: the abort flag then makes every later wait return at once.
+    bool live = true;
+    int nflush = 0, tin = 0;  // splits handed over, tiles into the current split
     for (int u = 0; u < nitems; ++u) {
       const int as = u & 1;
-      if (!warp_wait(b_accfull + 8 * as, (uint32_t)(u >> 1) & 1u, err, abort_flag)) break;
-      tc_fence_after();
       const int t = u / MT, mt = u % MT;
-      uint32_t b[CW];
-      tmem_ld64_issue(lanebase + as * 256, b);
-      tmem_ld64_wait(b);
-      // the item's TMEM columns are in registers: release the slot
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(b_accempty + 8 * as);
-      float m = ms[0], l = ls[0];
+      if (live && !warp_wait(b_accfull + 8 * as, (uint32_t)(u >> 1) & 1u, err, abort_flag)) live = false;
+      if (live) {
+        tc_fence_after();
+        uint32_t b[CW];
+        tmem_ld64_issue(lanebase + as * 256, b);
+        tmem_ld64_wait(b);
+        // the item's TMEM columns are in registers: release the slot
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(b_accempty + 8 * as);
+        float m = ms[0], l = ls[0];
 #pragma unroll
-      for (int i = 1; i < MT; ++i)
-        if (mt == i) {
-          m = ms[i];
-          l = ls[i];
+        for (int i = 1; i < MT; ++i)
+          if (mt == i) {
+            m = ms[i];
+            l = ls[i];
+          }
+        const int nv = min(CW, j1 - (j0 + t * KN + g * CW));
+        if (nv == CW) {
+          // chunk maximum over four independent chains: chain r starts at
+          // element r and takes pairs 4 + 2r + 8i, 5 + 2r + 8i
+          float cm[4];
+#pragma unroll
+          for (int r = 0; r < 4; ++r) cm[r] = __uint_as_float(b[r]);
+#pragma unroll
+          for (int i = 4; i < CW; i += 8) {
+#pragma unroll
+            for (int r = 0; r < 4; ++r)
+              if (i + 2 * r + 1 < CW)
+                cm[r] = max3(cm[r], __uint_as_float(b[i + 2 * r]), __uint_as_float(b[i + 2 * r + 1]));
+          }
+          const float mn = fmaxf(m, fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3])));
+          const float mnc = mn * c;
+          float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+          // three phases (exponent arguments, exponentials, sums) in place, so
+          // that independent work separates dependent instructions
+#pragma unroll
+          for (int i = 0; i < CW; i += 2) {
+            float x0, x1;
+            fma2(__uint_as_float(b[i]), __uint_as_float(b[i + 1]), c, c, -mnc, -mnc, x0, x1);
+            b[i] = __float_as_uint(x0);
+            b[i + 1] = __float_as_uint(x1);
+          }
+#pragma unroll
+          for (int i = 0; i < CW; ++i) b[i] = __float_as_uint(ex2_approx(__uint_as_float(b[i])));
+#pragma unroll
+          for (int i = 0; i < CW; i += 4) {
+            add2(s0, s1, __uint_as_float(b[i]), __uint_as_float(b[i + 1]));
+            add2(s2, s3, __uint_as_float(b[i + 2]), __uint_as_float(b[i + 3]));
+          }
+          l = (m == -CUDART_INF_F ? 0.f : l * ex2_approx((m - mn) * c)) + ((s0 + s1) + (s2 + s3));
+          m = mn;
+        } else if (nv > 0) {
+          float mc = -CUDART_INF_F;
+#pragma unroll
+          for (int i = 0; i < CW; ++i)
+            if (i < nv) mc = fmaxf(mc, __uint_as_float(b[i]));
+          const float mn = fmaxf(m, mc);
+          const float mnc = mn * c;
+          float sacc = 0.f;
+#pragma unroll
+          for (int i = 0; i < CW; ++i)
+            if (i < nv) sacc += ex2_approx(fmaf(__uint_as_float(b[i]), c, -mnc));
+          l = (m == -CUDART_INF_F ? 0.f : l * ex2_approx((m - mn) * c)) + sacc;
+          m = mn;
         }
-      const int nv = min(CW, j1 - (j0 + t * KN + g * CW));
-      if (nv == CW) {
-        // chunk maximum over four independent chains: chain r starts at
-        // element r and takes pairs 4 + 2r + 8i, 5 + 2r + 8i
-        float cm[4];
 #pragma unroll
-        for (int r = 0; r < 4; ++r) cm[r] = __uint_as_float(b[r]);
-#pragma unroll
-        for (int i = 4; i < CW; i += 8) {
-#pragma unroll
-          for (int r = 0; r < 4; ++r)
-            if (i + 2 * r + 1 < CW)
-              cm[r] = max3(cm[r], __uint_as_float(b[i + 2 * r]), __uint_as_float(b[i + 2 * r + 1]));
-        }
-        const float mn = fmaxf(m, fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3])));
-        const float mnc = mn * c;
-        float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-        // three phases (exponent arguments, exponentials, sums) in place, so
-        // that independent work separates dependent instructions
-#pragma unroll
-        for (int i = 0; i < CW; i += 2) {
-          float x0, x1;
-          fma2(__uint_as_float(b[i]), __uint_as_float(b[i + 1]), c, c, -mnc, -mnc, x0, x1);
-          b[i] = __float_as_uint(x0);
-          b[i + 1] = __float_as_uint(x1);
-        }
-#pragma unroll
-        for (int i = 0; i < CW; ++i) b[i] = __float_as_uint(ex2_approx(__uint_as_float(b[i])));
-#pragma unroll
-        for (int i = 0; i < CW; i += 4) {
-          add2(s0, s1, __uint_as_float(b[i]), __uint_as_float(b[i + 1]));
-          add2(s2, s3, __uint_as_float(b[i + 2]), __uint_as_float(b[i + 3]));
-        }
-        l = (m == -CUDART_INF_F ? 0.f : l * ex2_approx((m - mn) * c)) + ((s0 + s1) + (s2 + s3));
-        m = mn;
-      } else if (nv > 0) {
-        float mc = -CUDART_INF_F;
-#pragma unroll
-        for (int i = 0; i < CW; ++i)
-          if (i < nv) mc = fmaxf(mc, __uint_as_float(b[i]));
-        const float mn = fmaxf(m, mc);
-        const float mnc = mn * c;
-        float sacc = 0.f;
-#pragma unroll
-        for (int i = 0; i < CW; ++i)
-          if (i < nv) sacc += ex2_approx(fmaf(__uint_as_float(b[i]), c, -mnc));
-        l = (m == -CUDART_INF_F ? 0.f : l * ex2_approx((m - mn) * c)) + sacc;
-        m = mn;
+        for (int i = 0; i < MT; ++i)
+          if (mt == i) {
+            ms[i] = m;
+            ls[i] = l;
+          }
       }
+      // end of a key split: hand the states over (see above) and start over
+      // (the CTA's tiles start on a split boundary)
+      if (mt == MT - 1) ++tin;
+      if (mt == MT - 1 && (tin == per_t || t + 1 == ntiles)) {
+        const int split = s0 + nflush, xb = nflush % kRsXBuf;
+        ++nflush;
+        tin = 0;
+        float2* xp = xch + (size_t)xb * kScoreGroups * MT * 128;
 #pragma unroll
-      for (int i = 0; i < MT; ++i)
-        if (mt == i) {
-          ms[i] = m;
-          ls[i] = l;
+        for (int i = 0; i < MT; ++i) xp[(g * MT + i) * 128 + quarter * 32 + lane] = make_float2(ms[i], ls[i]);
+        __syncwarp();
+        uint32_t last = 0u;
+        if (lane == 0) {
+          // release the warp's states (cumulative over the __syncwarp) and
+          // acquire the other groups' ones with the same atomic
+          uint32_t old;
+          asm volatile("atom.acq_rel.cta.shared::cta.add.u32 %0, [%1], 1;"
+                       : "=r"(old) : "r"(smem_u32(&xcnt[xb * 4 + quarter])) : "memory");
+          last = (old & 3u) == 3u ? 1u : 0u;
         }
-    }
-  }
-  // merge the groups' states, then write (m * c, l) per query row
-  if (warp >= 2 && g > 0) {
+        last = __shfl_sync(0xffffffffu, last, 0);
+        __syncwarp();
+        if (last) {
 #pragma unroll
-    for (int mt = 0; mt < MT; ++mt)
-      xch[((g - 1) * MT + mt) * 128 + quarter * 32 + lane] = make_float2(ms[mt], ls[mt]);
+          for (int i = 0; i < MT; ++i) {
+            const int row = r0 + i * 128 + quarter * 32 + lane;
+            const float2 v0 = xp[i * 128 + quarter * 32 + lane];
+            float m = v0.x, l = v0.y;
+            for (int o = 1; o < kScoreGroups; ++o) {
+              const float2 v = xp[(o * MT + i) * 128 + quarter * 32 + lane];
+              online_merge(m, l, v.x, v.y, c);
+            }
+            if (row < R) part[((size_t)h * nsplit + split) * R + row] = make_float2(m * c, l);
+          }
+        }
+#pragma unroll
+        for (int i = 0; i < MT; ++i) {
+          ms[i] = -CUDART_INF_F;
+          ls[i] = 0.f;
+        }
+      }
+    }
   }
   tc_fence_before();
   __syncthreads();
-  if (warp >= 2 && g == 0) {
-#pragma unroll
-    for (int mt = 0; mt < MT; ++mt) {
-      const int row = r0 + mt * 128 + quarter * 32 + lane;
-      float m = ms[mt], l = ls[mt];
-      for (int o = 1; o < kScoreGroups; ++o) {
-        const float2 v = xch[((o - 1) * MT + mt) * 128 + quarter * 32 + lane];
-        online_merge(m, l, v.x, v.y, c);
-      }
-      if (row < R) part[((size_t)h * nsplit + split) * R + row] = make_float2(m * c, l);
-    }
-  }
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, 512);
@@ -696,23 +741,11 @@ __global__ void __maxnreg__(kScoreMaxReg)
     tmem_relinquish();
   }
   load_q_sw128(sm, NQ, q, p, h);
-  // merge pass 1's per-split row statistics: bias_r = -m_r - log2(G l_r), so
-  // that 2^(x c + bias_r) is the softmax probability divided by G
-  for (int r = threadIdx.x; r < NQ; r += blockDim.x) {
-    float b = -CUDART_INF_F;
-    if (r < R) {
-      const float2* pp = part + (size_t)h * nsplit * R + r;
-      float m = -CUDART_INF_F;
-      for (int s = 0; s < nsplit; ++s) m = fmaxf(m, pp[(size_t)s * R].x);
-      float l = 0.f;
-      for (int s = 0; s < nsplit; ++s) {
-        const float2 v = pp[(size_t)s * R];
-        if (v.y > 0.f) l += v.y * exp2f(v.x - m);
-      }
-      b = -m - log2f((float)p.G() * l);
-    }
-    bias_s[r] = b;
-  }
+  // pass 1's merged row statistics: bias_r = -m_r - log2(G l_r), so that
+  // 2^(x c + bias_r) is the softmax probability divided by G (padded rows
+  // get -inf and add exact zeros)
+  const float* bias_g = reinterpret_cast<const float*>(part + (size_t)p.hkv * nsplit * R) + (size_t)h * R;
+  for (int r = threadIdx.x; r < NQ; r += blockDim.x) bias_s[r] = r < R ? bias_g[r] : -CUDART_INF_F;
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -1239,14 +1272,19 @@ static int score_tiles(const Problem& p) {
 }
 
 int score_nsplit_max(const Problem& p) {
-  const int slots = p.dtype == kBF16 ? 152 : 2 * 152;
   const int tiles = score_tiles(p);
-  const int nmh = p.dtype == kBF16 ? rs_layout(p.R()).NMH : 1;
-  int s = pick_split(p.hkv * nmh, tiles, slots);
-  // at least ~24 key tiles per split, so that a CTA's set-up (Q load,
-  // barrier and TMEM set-up, pipeline fill) stays small next to its work
-  const int fat = (tiles + 23) / 24;
-  if (p.dtype == kBF16 && s > fat) s = fat;
+  if (p.dtype == kBF16) {
+    // bf16: enough splits that one layer alone fills one wave of a nominal
+    // 152-SM GB300, every split non-empty; a batch of layers runs several
+    // splits per CTA (the partials stay those of the shape)
+    const int nmh = rs_layout(p.R()).NMH;
+    int target = (152 + p.hkv * nmh - 1) / (p.hkv * nmh);
+    if (target > tiles) target = tiles;
+    if (target < 1) target = 1;
+    const int per_t = (tiles + target - 1) / target;
+    return (tiles + per_t - 1) / per_t;
+  }
+  int s = pick_split(p.hkv, tiles, 2 * 152);
   return s < 1 ? 1 : s;
 }
 
@@ -1292,8 +1330,18 @@ cudaError_t launch_score_umma(const Problem& p, const LayerPtrs& io, Strided<flo
     return e;
   {
     TimingScope ts("rowstats_umma", st);
-    rs_kernel<<<dim3(nsplit * L1.NMH, p.L * p.hkv), kScoreThreads, L1.total, st>>>(m1, io, p, nsplit, rowpart,
-                                                                                     err);
+    // CTAs per (layer, head, row half): whole waves for the batch, each
+    // taking cps consecutive splits
+    const int cph0 = pick_split(p.L * p.hkv * L1.NMH, nsplit, sm_count());
+    const int cps = (nsplit + cph0 - 1) / cph0;
+    const int cph = (nsplit + cps - 1) / cps;
+    rs_kernel<<<dim3(cph * L1.NMH, p.L * p.hkv), kScoreThreads, L1.total, st>>>(m1, io, p, nsplit, cps, rowpart,
+                                                                               err);
+  }
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  {
+    TimingScope ts("row_bias", st);
+    launch_row_bias(p, nsplit, rowpart, st);
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const int tiles = (p.n + 127) / 128;
