@@ -185,7 +185,17 @@ def kernel_roofline(name: str, t_launch: float, layers: int, budget: int, peaks)
             d["mufu"] = dict(achieved=ex, peak=mufu_peak_texp(peaks), unit="Texp/s",
                              frac=ex / mufu_peak_texp(peaks))
         return d
-    if name.startswith("css_phi"):
+    if name.startswith("row_bias"):
+        # window-score pass 1's split partials in, one bias per query row out;
+        # the split count follows the library's rule for this shape (one
+        # layer's splits fill one wave of 152 SMs, every split non-empty)
+        rows = HKV * W * (HQ // HKV)
+        tiles = (N_TOK + 255) // 256
+        target = min(tiles, (152 + HKV - 1) // HKV)
+        per_t = (tiles + target - 1) // target
+        nsplit = (tiles + per_t - 1) // per_t
+        work = rows * nsplit * 8 + rows * 4
+    elif name.startswith("css_phi"):
         work = tok_head * (5 * 4 + 4)              # five dot products in, Phi out
     elif name.startswith("css_box"):
         work = kbytes + tok_head * 8               # every key once; Phi and 1/|k| out
