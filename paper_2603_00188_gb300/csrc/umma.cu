@@ -61,22 +61,15 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, uint32_
 
 // First token of TSG row tile t and the end of the rows it may write: its
 // frame's visual span, or the whole historical range for spanning tiles.
-__device__ __forceinline__ void tsg_tile(const FrameTable& ft, int t, int& tok0, int& fend) {
+// For a loop whose tiles only grow: f carries the frame of the previous
+// tile (start it at 0).
+__device__ __forceinline__ void tsg_tile_next(const FrameTable& ft, int t, int& f, int& tok0, int& fend) {
   if (ft.tsg_span) {
     tok0 = ft.tsg_off + t * kTsgTile;
     fend = ft.tsg_end;
     return;
   }
-  int lo = 0, hi = ft.n_frames - 2, f = 0;
-  while (lo <= hi) {
-    int mid = (lo + hi) >> 1;
-    if (ft.tile0[mid] <= t) {
-      f = mid;
-      lo = mid + 1;
-    } else {
-      hi = mid - 1;
-    }
-  }
+  while (f + 1 < ft.n_frames - 1 && ft.tile0[f + 1] <= t) ++f;
   tok0 = ft.off[f] + (t - ft.tile0[f]) * kTsgTile;
   fend = ft.off[f] + ft.gh[f] * ft.gw[f];
 }
@@ -171,13 +164,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int rb = 0; rb < 4; ++rb)
           tma_load_3d(sB + kb * 65536 + rb * 16384, &kmap, b_bfull, kb * 64, h,
                       ft.cur_off + col0 + rb * 128);
-      int it = 0, issued[kTsgAStages] = {0, 0, 0};
+      int it = 0, issued[kTsgAStages] = {0, 0, 0}, tf = 0;
       for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++it) {
         const int s = it % kTsgAStages;
         const uint32_t u = (uint32_t)(it / kTsgAStages);
         if (!mbar_wait(b_aempty + 8 * s, (u & 1u) ^ 1u, err, abort_flag)) break;
         int tok0, fend;
-        tsg_tile(ft, t, tok0, fend);
+        tsg_tile_next(ft, t, tf, tok0, fend);
         mbar_arrive_expect_tx(b_afull + 8 * s, 32768);
         tma_load_3d(sA + s * 32768, &kmap, b_afull + 8 * s, 0, h, tok0);
         tma_load_3d(sA + s * 32768 + 16384, &kmap, b_afull + 8 * s, 64, h, tok0);
@@ -227,7 +220,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int valid_g = min(256, valid - g * 256);
       const uint32_t tbase = tmem + ((uint32_t)(quarter * 32) << 16) + g * 256;
       const float* rg = rn_s + g * 256;
-      int it = 0;
+      int it = 0, tf = 0;
       for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++it) {
         if (!warp_wait(b_accfull + 8 * g, (uint32_t)it & 1u, err, abort_flag)) break;
         tc_fence_after();
@@ -300,7 +293,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(b_accempty + 8 * g);
         int tok0, fend;
-        tsg_tile(ft, t, tok0, fend);
+        tsg_tile_next(ft, t, tf, tok0, fend);
         const int tok = tok0 + quarter * 32 + lane;
         if (tok < fend) rho_part[((size_t)(2 * chunk + g) * hkv + h) * n + tok] = mx;
       }
@@ -934,18 +927,12 @@ struct CssDots {
   int cur_pad;
 };
 
-__device__ __forceinline__ void css_tile(const FrameTable& ft, int t, int& f, int& t0) {
-  int lo = 0, hi = ft.n_frames - 1;
-  f = 0;
-  while (lo <= hi) {
-    const int mid = (lo + hi) >> 1;
-    if (ft.ctile0[mid] <= t) {
-      f = mid;
-      lo = mid + 1;
-    } else {
-      hi = mid - 1;
-    }
-  }
+// Frame f and first token t0 of CSS tile t (the tiles of frame f are
+// ctile0[f] .. ctile0[f+1]-1), for a loop whose tiles only grow: f carries
+// the frame of the previous tile (start it at 0), so a step costs a
+// comparison or two instead of a search.
+__device__ __forceinline__ void css_tile_next(const FrameTable& ft, int t, int& f, int& t0) {
+  while (f + 1 < ft.n_frames && ft.ctile0[f + 1] <= t) ++f;
   t0 = ft.off[f] + (t - ft.ctile0[f]) * 128;
 }
 
@@ -1001,12 +988,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       int issued[kCssMaxStages] = {0, 0, 0, 0};
+      int f = 0;
       for (int it = 0; it < ntiles; ++it) {
         const int s = it % S;
         const uint32_t u = (uint32_t)(it / S);
         if (!mbar_wait(b_kempty + 8 * s, (u & 1u) ^ 1u, err, abort_flag)) break;
-        int f, t0;
-        css_tile(ft, blockIdx.x + it * gridDim.x, f, t0);
+        int t0;
+        css_tile_next(ft, blockIdx.x + it * gridDim.x, f, t0);
         const int nbox = (((128 + ft.gw[f] + 1 + 15) & ~15) + 63) / 64;  // 64-row boxes covering NB rows
         mbar_arrive_expect_tx(b_kfull + 8 * s, (uint32_t)(2 * nbox * 64 * 128));
         for (int kb = 0; kb < 2; ++kb)
@@ -1021,13 +1009,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 1) {
     if (lane == 0) {
+      int f = 0;
       for (int it = 0; it < ntiles; ++it) {
         const int s = it % S, as = it & 1;
         if (!mbar_wait(b_kfull + 8 * s, (uint32_t)(it / S) & 1u, err, abort_flag)) break;
         if (!mbar_wait(b_accempty + 8 * as, ((uint32_t)(it >> 1) & 1u) ^ 1u, err, abort_flag)) break;
         tc_fence_after();
-        int f, t0;
-        css_tile(ft, blockIdx.x + it * gridDim.x, f, t0);
+        int t0;
+        css_tile_next(ft, blockIdx.x + it * gridDim.x, f, t0);
         const int nb = (128 + ft.gw[f] + 1 + 15) & ~15;
         const uint32_t idesc = idesc_bf16(128, nb);
 #pragma unroll
@@ -1052,12 +1041,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     float* se_o = out.dSE.at(l) + (size_t)h * n;
     float* sw_o = out.dSW.at(l) + (size_t)h * n;
     float* rc_o = out.rn_cur.at(l) + (size_t)h * out.cur_pad;
+    int f = 0;
     for (int it = g; it < ntiles; it += 2) {
       const uint32_t ua = (uint32_t)(it >> 1);
       if (!warp_wait(b_accfull + 8 * g, ua & 1u, err, abort_flag)) break;
       tc_fence_after();
-      int f, t0;
-      css_tile(ft, blockIdx.x + it * gridDim.x, f, t0);
+      int t0;
+      css_tile_next(ft, blockIdx.x + it * gridDim.x, f, t0);
       const int gw = ft.gw[f];
       const int dd[5] = {0, 1, gw - 1, gw, gw + 1};
       float val[5] = {0.f, 0.f, 0.f, 0.f, 0.f};
