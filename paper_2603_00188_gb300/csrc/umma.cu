@@ -469,9 +469,11 @@ __global__ void __maxnreg__(kScoreMaxReg)
   if (warp == 0) {
     if (lane == 0) {
       int issued[kMaxKStages] = {0, 0, 0, 0};
-      for (int it = 0; it < ntiles; ++it) {
-        const int s = it % S;
-        const uint32_t u = (uint32_t)(it / S);
+      int ks = 0;        // stage of tile it (it % S), counted instead of divided
+      uint32_t kp = 0u;  // passes over the ring (it / S)
+      for (int it = 0; it < ntiles; ++it, ks = ks + 1 == S ? 0 : ks + 1, kp += ks == 0u ? 1u : 0u) {
+        const int s = ks;
+        const uint32_t u = kp;
         if (!mbar_wait(b_kempty + 8 * s, (u & 1u) ^ 1u, err, abort_flag)) break;
         const int tok = j0 + it * KN;
         mbar_arrive_expect_tx(b_kfull + 8 * s, (uint32_t)L.k_stage_bytes);
@@ -487,10 +489,11 @@ __global__ void __maxnreg__(kScoreMaxReg)
     if (lane == 0) {
       const uint32_t idesc = idesc_bf16(128, KN);
       bool ok = true;
-      int u = 0;
-      for (int it = 0; ok && it < ntiles; ++it) {
-        const int s = it % S;
-        if (!mbar_wait(b_kfull + 8 * s, (uint32_t)(it / S) & 1u, err, abort_flag)) break;
+      int u = 0, ks = 0;
+      uint32_t kp = 0u;
+      for (int it = 0; ok && it < ntiles; ++it, ks = ks + 1 == S ? 0 : ks + 1, kp += ks == 0u ? 1u : 0u) {
+        const int s = ks;
+        if (!mbar_wait(b_kfull + 8 * s, kp & 1u, err, abort_flag)) break;
         for (int mt = 0; mt < MT; ++mt, ++u) {
           const int as = u & 1;
           if (!mbar_wait(b_accempty + 8 * as, ((uint32_t)(u >> 1) & 1u) ^ 1u, err, abort_flag)) {
@@ -749,9 +752,11 @@ __global__ void __maxnreg__(kScoreMaxReg)
   if (warp == 0) {
     if (lane == 0) {
       int issued[kMaxKStages] = {0, 0, 0, 0};
-      for (int it = 0; it < ntiles; ++it) {
-        const int s = it % S;
-        const uint32_t u = (uint32_t)(it / S);
+      int ks = 0;
+      uint32_t kp = 0u;
+      for (int it = 0; it < ntiles; ++it, ks = ks + 1 == S ? 0 : ks + 1, kp += ks == 0u ? 1u : 0u) {
+        const int s = ks;
+        const uint32_t u = kp;
         if (!mbar_wait(b_kempty + 8 * s, (u & 1u) ^ 1u, err, abort_flag)) break;
         const int tok = (blockIdx.x + it * gridDim.x) * 128;
         mbar_arrive_expect_tx(b_kfull + 8 * s, 32768);
@@ -766,9 +771,11 @@ __global__ void __maxnreg__(kScoreMaxReg)
   } else if (warp == 1) {
     if (lane == 0) {
       bool ok = true;
-      for (int it = 0; ok && it < ntiles; ++it) {
-        const int s = it % S;
-        const uint32_t u = (uint32_t)(it / S);
+      int ks = 0;
+      uint32_t kp = 0u;
+      for (int it = 0; ok && it < ntiles; ++it, ks = ks + 1 == S ? 0 : ks + 1, kp += ks == 0u ? 1u : 0u) {
+        const int s = ks;
+        const uint32_t u = kp;
         if (!mbar_wait(b_kfull + 8 * s, u & 1u, err, abort_flag)) break;
         // item it*nh + hh: query columns [hh W, hh W + W) into TMEM slot item % 2
 #pragma unroll
@@ -988,10 +995,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       int issued[kCssMaxStages] = {0, 0, 0, 0};
-      int f = 0;
-      for (int it = 0; it < ntiles; ++it) {
-        const int s = it % S;
-        const uint32_t u = (uint32_t)(it / S);
+      int f = 0, ks = 0;
+      uint32_t kp = 0u;
+      for (int it = 0; it < ntiles; ++it, ks = ks + 1 == S ? 0 : ks + 1, kp += ks == 0u ? 1u : 0u) {
+        const int s = ks;
+        const uint32_t u = kp;
         if (!mbar_wait(b_kempty + 8 * s, (u & 1u) ^ 1u, err, abort_flag)) break;
         int t0;
         css_tile_next(ft, blockIdx.x + it * gridDim.x, f, t0);
@@ -1009,10 +1017,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      int f = 0;
-      for (int it = 0; it < ntiles; ++it) {
-        const int s = it % S, as = it & 1;
-        if (!mbar_wait(b_kfull + 8 * s, (uint32_t)(it / S) & 1u, err, abort_flag)) break;
+      int f = 0, ks = 0;
+      uint32_t kp = 0u;
+      for (int it = 0; it < ntiles; ++it, ks = ks + 1 == S ? 0 : ks + 1, kp += ks == 0u ? 1u : 0u) {
+        const int s = ks, as = it & 1;
+        if (!mbar_wait(b_kfull + 8 * s, kp & 1u, err, abort_flag)) break;
         if (!mbar_wait(b_accempty + 8 * as, ((uint32_t)(it >> 1) & 1u) ^ 1u, err, abort_flag)) break;
         tc_fence_after();
         int t0;
