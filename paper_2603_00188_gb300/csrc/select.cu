@@ -435,22 +435,34 @@ cudaError_t launch_select(const Problem& p, const FrameTable& ft, const SelectAr
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg;
   cudaLaunchAttribute attr[1];
-  int cl = 0;
+  int cl = 0, fit8 = 0;
   long long best = 0;
+  const long long units = (long long)p.L * p.hkv;
   for (int c = 1; c <= kSelMaxCluster; c <<= 1) {
     const int ch = (p.n + c - 1) / c;
     if (ch > kSelMaxChunk) continue;
     select_config(&cfg, attr, p, c, st);
     int fit = 0;
     if ((e = cudaOccupancyMaxActiveClusters(&fit, k_select, &cfg)) != cudaSuccess) return e;
+    if (c == kSelMaxCluster) fit8 = fit;
     if (fit < 1) continue;
-    const long long units = (long long)p.L * p.hkv;
     const long long est = (units + fit - 1) / fit * ch;
     if (cl == 0 || est < best) {
       cl = c;
       best = est;
     }
   }
+  // A few (layer, head) problems (one layer, a small batch) leave most SMs
+  // idle even with clusters of 8: clusters of 16 (non-portable) halve each
+  // CTA's tokens.  Only then, so that batches keep their portable shape.
+  if (cl == kSelMaxCluster && units <= fit8 &&
+      cudaFuncSetAttribute(k_select, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess) {
+    const int c = 2 * kSelMaxCluster;
+    select_config(&cfg, attr, p, c, st);
+    int fit = 0;
+    if (cudaOccupancyMaxActiveClusters(&fit, k_select, &cfg) == cudaSuccess && fit >= units) cl = c;
+  }
+  (void)cudaGetLastError();  // a refused non-portable query leaves no error behind
   if (cl == 0) return cudaErrorNotSupported;
   select_config(&cfg, attr, p, cl, st);
   TimingScope ts(a.mode & kSelGate ? (a.mode & kSelTopk ? "select_gate_topk" : "select_gate") : "select_topk", st);
