@@ -452,10 +452,15 @@ cudaError_t launch_select(const Problem& p, const FrameTable& ft, const SelectAr
       best = est;
     }
   }
-  // A few (layer, head) problems (one layer, a small batch) leave most SMs
-  // idle even with clusters of 8: clusters of 16 (non-portable) halve each
-  // CTA's tokens.  Only then, so that batches keep their portable shape.
-  if (cl == kSelMaxCluster && units <= fit8 &&
+  // A few (layer, head) problems (one layer, a couple of layers) leave most
+  // SMs idle even with clusters of 8: clusters of 16 (non-portable) halve
+  // each CTA's tokens.  Only while they take at most one CTA per SM (the
+  // 16-CTA barriers cost more once CTAs share SMs), so that batches keep
+  // their portable shape.
+  int nsm = 0, dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    nsm = 0;
+  if (cl == kSelMaxCluster && units <= fit8 && units * 2 * kSelMaxCluster <= nsm &&
       cudaFuncSetAttribute(k_select, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess) {
     const int c = 2 * kSelMaxCluster;
     select_config(&cfg, attr, p, c, st);
