@@ -192,7 +192,7 @@ def kernel_roofline(name: str, t_launch: float, layers: int, budget: int, peaks)
         rows = HKV * W * (HQ // HKV)
         tiles = (N_TOK + 255) // 256
         target = min(tiles, (152 + HKV - 1) // HKV)
-        per_t = (tiles + target - 1) // target
+        per_t = max(2, (tiles + target - 1) // target)
         nsplit = (tiles + per_t - 1) // per_t
         work = rows * nsplit * 8 + rows * 4
     elif name.startswith("css_phi"):

@@ -1276,11 +1276,14 @@ int score_nsplit_max(const Problem& p) {
     // bf16: enough splits that one layer alone fills one wave of a nominal
     // 152-SM GB300, every split non-empty; a batch of layers runs several
     // splits per CTA (the partials stay those of the shape)
+    // (at least two tiles per split: a one-tile split hands its partial over
+    // after every tile and doubles the partials the row-bias pass merges)
     const int nmh = rs_layout(p.R()).NMH;
     int target = (152 + p.hkv * nmh - 1) / (p.hkv * nmh);
     if (target > tiles) target = tiles;
     if (target < 1) target = 1;
-    const int per_t = (tiles + target - 1) / target;
+    int per_t = (tiles + target - 1) / target;
+    if (per_t < 2) per_t = 2;
     return (tiles + per_t - 1) / per_t;
   }
   int s = pick_split(p.hkv, tiles, 2 * 152);
