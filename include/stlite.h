@@ -232,9 +232,10 @@ typedef struct {
 
 /* Algorithm 1 for n_layers layers of one sequence (one frame layout, one
  * budget), each layer compressed independently with its own window queries;
- * the result for every layer equals stlite_compress_layer's.  Every step
- * runs as one launch covering up to 32 layers at a time, so small per-layer
- * stages (the selections, the compaction) fill the GPU.  layers: HOST array
+ * the result for every layer equals stlite_compress_layer's.  Each kernel
+ * launch covers up to 32 layers at a time (with TSG and CSS on, eight
+ * launches per batch of up to 32 layers), so small per-layer stages (the
+ * selections, the compaction) fill the GPU.  layers: HOST array
  * [n_layers].  ws: n_layers times stlite_workspace_size() bytes (layer l uses
  * the l-th slice; the first word of the whole workspace is the error word).
  * budget_out (nullable, HOST) receives B. */
@@ -300,7 +301,7 @@ STLITE_API stlite_status stlite_compress_varlen(const stlite_shape* shape, int32
 
 /* stlite_compress_varlen over n_layers layers that share the packing
  * (cu_seqlens, frames): every sequence's layers run together through the
- * batched-layers path of stlite_compress_layers (one launch per step for up
+ * batched-layers path of stlite_compress_layers (each kernel launch covers up
  * to 32 layers), the sequences one after another on `stream`.  The result
  * for every layer equals stlite_compress_varlen's on that layer.
  * layers: HOST array [n_layers]; entry l holds layer l's packed tensors in
