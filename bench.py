@@ -305,29 +305,64 @@ def _code_only(text: str) -> str:
     return " ".join("".join(out).split())
 
 
-def src_digest():
-    """Digest of the kernel sources (comments excluded) the committed ncu
-    counters must have been taken on."""
+CSRC = os.path.join(ROOT, "paper_2603_00188_gb300", "csrc")
+
+# The translation units each step kernel is built from, on top of the shared
+# headers and the host planning in api.cu (frame tables, workspace plan):
+# a code change there changes what the kernel does, a change elsewhere does
+# not.  The row-bias pass also depends on umma.cu, whose launcher picks the
+# number of row-statistics splits it merges.
+KERNEL_UNITS = {
+    "tsg_umma": ("umma.cu",),
+    "rowstats_umma": ("umma.cu",),
+    "colsum_umma": ("umma.cu",),
+    "css_umma": ("umma.cu",),
+    "css_phi": ("umma.cu",),
+    "row_bias": ("simt.cu", "umma.cu"),
+    "select_gate_topk": ("select.cu",),
+    "gather": ("select.cu",),
+}
+SHARED_UNITS = ("api.cu", "common.cuh", "kernels.cuh", "ptx.cuh")
+
+
+def _digest(names, read):
     h = hashlib.sha256()
-    csrc = os.path.join(ROOT, "paper_2603_00188_gb300", "csrc")
-    for name in sorted(os.listdir(csrc)):
-        with open(os.path.join(csrc, name), encoding="utf-8") as f:
-            h.update(name.encode() + _code_only(f.read()).encode())
+    for name in sorted(names):
+        h.update(name.encode() + _code_only(read(name)).encode())
     return h.hexdigest()[:16]
+
+
+def _read_csrc(name):
+    with open(os.path.join(CSRC, name), encoding="utf-8") as f:
+        return f.read()
+
+
+def src_digest(read=_read_csrc):
+    """Digest of all kernel sources (comments excluded)."""
+    return _digest(os.listdir(CSRC), read)
+
+
+def kernel_digest(kernel: str, read=_read_csrc):
+    """Digest of the sources (comments excluded) that `kernel` is built from:
+    the committed ncu counters of that kernel must have been taken on them."""
+    return _digest(KERNEL_UNITS[kernel] + SHARED_UNITS, read)
 
 
 def traffic_for(kernel: str):
     """Per-launch DRAM bytes of `kernel` from the committed ncu summary, if it
-    was taken on the current sources."""
+    was taken on the kernel's current sources."""
     p = os.path.join(ROOT, "profiles", "ncu_traffic.json")
     if not os.path.exists(p):
         return None
     with open(p) as f:
         d = json.load(f)
-    if d.get("src_digest") != src_digest():
-        return None
     e = d.get("kernels", {}).get(kernel)
-    return None if e is None else e.get("dram_bytes_per_launch_full")
+    if e is None:
+        return None
+    want = e.get("src_digest")
+    if want is None:
+        return e.get("dram_bytes_per_launch_full") if d.get("src_digest") == src_digest() else None
+    return e.get("dram_bytes_per_launch_full") if want == kernel_digest(kernel) else None
 
 
 # ------------------------------------------------------- critical hit rate

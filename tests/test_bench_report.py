@@ -36,18 +36,43 @@ def test_code_only_drops_comments_and_layout(bench):
 
 
 def test_committed_traffic_is_reported_only_for_its_sources(bench):
-    # the bench reports the committed ncu traffic while the kernel code is the
-    # one it was taken on, and nothing (null) once the kernels have changed
+    # the bench reports a kernel's committed ncu traffic while the code of
+    # the units it is built from is the code the counters were taken on, and
+    # nothing (null) once they have changed
     with open(os.path.join(ROOT, "profiles", "ncu_traffic.json")) as f:
         d = json.load(f)
-    names = ("tsg_umma", "rowstats_umma", "row_bias", "colsum_umma", "css_umma", "css_phi", "gather",
-             "select_gate_topk")
-    for name in names:
-        assert d["kernels"][name]["dram_bytes_per_launch_full"] > 0
-    current = d["src_digest"] == bench.src_digest()
-    for name in names:
-        got = bench.traffic_for(name)
-        assert got == (d["kernels"][name]["dram_bytes_per_launch_full"] if current else None)
+    assert set(d["kernels"]) == set(bench.KERNEL_UNITS)
+    for name, e in d["kernels"].items():
+        assert e["dram_bytes_per_launch_full"] > 0
+        current = e["src_digest"] == bench.kernel_digest(name)
+        assert bench.traffic_for(name) == (e["dram_bytes_per_launch_full"] if current else None)
+
+
+def test_kernel_digest_follows_its_own_units(bench):
+    # a code change in one translation unit stales the counters of the
+    # kernels built from it and of no other; a comment change stales none
+    def edited(unit, old, new):
+        def read(name):
+            text = bench._read_csrc(name)
+            if name == unit:
+                assert old in text
+                text = text.replace(old, new, 1)
+            return text
+        return read
+
+    base = {k: bench.kernel_digest(k) for k in bench.KERNEL_UNITS}
+    code = edited("select.cu", "k_gather(", "k_gather2(")
+    for k in bench.KERNEL_UNITS:
+        changed = bench.kernel_digest(k, code) != base[k]
+        assert changed == ("select.cu" in bench.KERNEL_UNITS[k]), k
+    code = edited("umma.cu", "k_css_phi(", "k_css_phi2(")
+    for k in bench.KERNEL_UNITS:
+        changed = bench.kernel_digest(k, code) != base[k]
+        assert changed == ("umma.cu" in bench.KERNEL_UNITS[k]), k
+    shared = edited("common.cuh", "struct FrameTable", "struct FrameTable2")
+    assert all(bench.kernel_digest(k, shared) != base[k] for k in bench.KERNEL_UNITS)
+    comment = edited("select.cu", "k_gather(", "k_gather(/* a comment */")
+    assert all(bench.kernel_digest(k, comment) == base[k] for k in bench.KERNEL_UNITS)
 
 
 def test_kernel_roofline_units(bench):
