@@ -87,3 +87,24 @@ def test_kernel_roofline_units(bench):
     # the row-bias pass moves a fraction of a key pass
     assert (bench.kernel_roofline("row_bias", t, 1, 10720, peaks)["achieved"]
             < 0.01 * bench.kernel_roofline("rowstats_umma", t, 1, 10720, peaks)["achieved"])
+
+
+def test_reference_arm_line():
+    # `bench.py --impl reference` times the oracle on the host and prints one
+    # JSON line in the bench's own metric, unit and workload
+    import subprocess
+    out = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
+                          "--steps", "1", "--warmup", "0"], cwd=ROOT, capture_output=True, text=True,
+                         timeout=600)
+    assert out.returncode == 0, out.stderr[-2000:]
+    lines = [l for l in out.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["value"] > 0 and d["higher_is_better"] is True
+    assert d["metric"].startswith("KV tokens compressed/sec") and d["unit"] == "tokens/s/layer"
+    assert d["config"]["layers"] == 28 and d["config"]["n_tokens"] == 53600
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"] and cb["sample"]
+    e = d["e2e"]
+    assert e["value"] == d["value"] and e["unit"] == d["unit"]
+    assert e["h2d_bytes_per_step"] == 0 and e["d2h_bytes_per_step"] == 0
