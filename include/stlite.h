@@ -205,16 +205,21 @@ STLITE_API stlite_status stlite_compress_layer(const stlite_shape* shape, const 
  * counterpart: this is a deployment convenience.  Its scratch (an error word
  * and the per-split softmax row statistics) is one fixed 2 MiB device array
  * inside the library, which every GPU that loads the library holds until
- * exit; problems whose scratch, 256 + Hkv*S*w*G*8 + Hkv*w*G*4 bytes (S = the
- * library's key splits, at most ceil(304/Hkv)), exceeds it are rejected with
- * STLITE_EUNSUPPORTED.  The call allocates nothing.  Its first call on each
- * device resolves that device's scratch address (cudaGetSymbolAddress), so
- * make the first call on a device before any stream capture.  All calls
- * share the array, which keeps the last call's contents (each call clears
- * its error word; the statistics are fully rewritten): calls that overlap on
- * the GPU -- issued to one device on different streams, or from several
- * threads -- race on it.  Kernel timeouts of this path are not reported (its
- * error word is internal).
+ * exit.  A problem needs 256 + Hkv*S*w*G*8 + Hkv*w*G*4 bytes of it, where S,
+ * the key splits of the first softmax pass, is at most max(4,
+ * 4*ceil(304/Hkv)); a problem beyond 2 MiB is rejected with
+ * STLITE_EUNSUPPORTED (checked after the shape limits of stlite_score and
+ * before the pointers, so no launch is attempted).  The call allocates
+ * nothing.  The array's address is resolved (cudaGetSymbolAddress) on the
+ * first call on each device, and again on the first call after the current
+ * context changed (cudaDeviceReset, another context made current), so make
+ * that first call before any stream capture.  All calls share the array,
+ * which keeps the last call's contents (each call clears its error word; the
+ * statistics are fully rewritten): calls that overlap on the GPU -- issued to
+ * one device on different streams, or from several threads -- race on it.
+ * A bounded wait of its kernels that ran out is recorded in the array's
+ * error word, which stlite_device_status(NULL, ...) reads on the current
+ * device; read it before the next call clears it.
  * q, k, a_base: as for stlite_score. */
 STLITE_API stlite_status stlite_score_noalloc(const stlite_shape* shape, const void* q, const void* k,
                                               float* a_base, void* stream);
@@ -345,7 +350,9 @@ STLITE_API stlite_status stlite_decode_workspace_size(const stlite_shape* shape,
 /* Reads and clears the workspace's device error word (synchronises `stream`).
  * *status receives STLITE_OK, STLITE_ETIMEOUT if a kernel's bounded wait ran
  * out since the last read, or STLITE_ECUDA if a kernel found its launch
- * configuration unusable (it then returned without touching its outputs). */
+ * configuration unusable (it then returned without touching its outputs).
+ * ws = NULL reads the error word of stlite_score_noalloc's fixed scratch on
+ * the current device instead. */
 STLITE_API stlite_status stlite_device_status(void* ws, void* stream, stlite_status* status);
 
 /* Per-kernel timing (instrumentation; not part of Algorithm 1).

@@ -22,23 +22,6 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-stlite_status check_shape(const stlite_shape* s) {
-  if (!s) return STLITE_EINVAL;
-  if (s->n_tokens < 1 || s->n_q_heads < 1 || s->n_kv_heads < 1 || s->window < 1 ||
-      s->head_dim < 1)
-    return STLITE_EINVAL;
-  if (s->n_q_heads % s->n_kv_heads != 0) return STLITE_EINVAL;
-  if (s->dtype != STLITE_BF16 && s->dtype != STLITE_F32) return STLITE_EINVAL;
-  if (s->head_dim != STLITE_HEAD_DIM) return STLITE_EUNSUPPORTED;
-  if (s->window > 256) return STLITE_EUNSUPPORTED;
-  const long long R = (long long)s->window * (s->n_q_heads / s->n_kv_heads);
-  if (R > 512) return STLITE_EUNSUPPORTED;
-  if ((long long)s->n_tokens * s->n_kv_heads > (1LL << 30)) return STLITE_EUNSUPPORTED;
-  if (s->n_tokens > select_max_tokens()) return STLITE_EUNSUPPORTED;
-  if (s->n_kv_heads > 4096) return STLITE_EUNSUPPORTED;
-  return STLITE_OK;
-}
-
 stlite_status build_frames(const stlite_shape* s, const stlite_frames* fr, FrameTable* ft) {
   memset(ft, 0, sizeof(*ft));
   ft->n_tokens = s->n_tokens;
@@ -114,6 +97,25 @@ stlite_status cuda_status(cudaError_t e) { return e == cudaSuccess ? STLITE_OK :
 }  // namespace
 
 namespace stl {
+
+// Shape checks shared by every entry point (the kernels' index arithmetic
+// relies on these limits).
+stlite_status check_shape(const stlite_shape* s) {
+  if (!s) return STLITE_EINVAL;
+  if (s->n_tokens < 1 || s->n_q_heads < 1 || s->n_kv_heads < 1 || s->window < 1 ||
+      s->head_dim < 1)
+    return STLITE_EINVAL;
+  if (s->n_q_heads % s->n_kv_heads != 0) return STLITE_EINVAL;
+  if (s->dtype != STLITE_BF16 && s->dtype != STLITE_F32) return STLITE_EINVAL;
+  if (s->head_dim != STLITE_HEAD_DIM) return STLITE_EUNSUPPORTED;
+  if (s->window > 256) return STLITE_EUNSUPPORTED;
+  const long long R = (long long)s->window * (s->n_q_heads / s->n_kv_heads);
+  if (R > 512) return STLITE_EUNSUPPORTED;
+  if ((long long)s->n_tokens * s->n_kv_heads > (1LL << 30)) return STLITE_EUNSUPPORTED;
+  if (s->n_tokens > select_max_tokens()) return STLITE_EUNSUPPORTED;
+  if (s->n_kv_heads > 4096) return STLITE_EUNSUPPORTED;
+  return STLITE_OK;
+}
 
 // One layer's workspace region; regions of consecutive layers follow each
 // other.  Every buffer is 256-byte aligned.
@@ -748,7 +750,12 @@ stlite_status stlite_decode_attention(const stlite_shape* shape, const void* q, 
 }
 
 stlite_status stlite_device_status(void* ws, void* stream, stlite_status* status) {
-  if (!ws || !status || !aligned16(ws)) return STLITE_EINVAL;
+  if (!status || (ws && !aligned16(ws))) return STLITE_EINVAL;
+  if (!ws) {  // the error word of stlite_score_noalloc's fixed scratch on the current device
+    uint32_t* word = nullptr;
+    if (noalloc_error_word(&word) != cudaSuccess) return STLITE_ECUDA;
+    ws = word;
+  }
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   uint32_t word = 0;
   if (cudaMemcpyAsync(&word, ws, 4, cudaMemcpyDeviceToHost, st) != cudaSuccess) return STLITE_ECUDA;

@@ -9,6 +9,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "../../include/stlite.h"
 #include "common.cuh"
 
 namespace stl {
@@ -55,6 +56,11 @@ inline Strided<T> strided(T* base, size_t stride) {
   s.stride = stride;
   return s;
 }
+
+// Shape limits shared by every entry point: STLITE_OK, or the status the
+// call returns (N, heads and window within the ranges the kernels' index
+// arithmetic and the selection's on-chip capacity assume).
+stlite_status check_shape(const stlite_shape* s);
 
 // ---- workspace plan (byte offsets into one layer's workspace region) ------
 struct WsPlan {
@@ -195,6 +201,11 @@ cudaError_t launch_gather(const Problem& p, const LayerPtrs& io, cudaStream_t st
 // 3-D TMA map (d, head, row) over a bf16 [n][hkv][128] tensor with boxes of
 // 64 x 1 x rows and the 128-byte swizzle.
 cudaError_t make_row_map(CUtensorMap* m, const void* base, int n, int hkv, int rows);
+
+// ---- fixed scratch of stlite_score_noalloc ---------------------------------
+// Device address of that array's error word on the current device (and
+// context), resolved as stlite_score_noalloc does.
+cudaError_t noalloc_error_word(uint32_t** word);
 
 // ---- consumer: decode attention over a (compressed) cache -----------------
 constexpr int kDecMaxG = 16;  // query heads per KV head

@@ -22,23 +22,73 @@ constexpr int kMaxDevices = 64;
 // symbol: the device address comes from cudaGetSymbolAddress below.
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kScratchBytes];
 
+// The resolved address of each device's array, with the context it belongs
+// to: the array is part of the library's module, which is loaded into each
+// context anew (after cudaDeviceReset, or when another context is current),
+// possibly at another address.  A call whose current context differs from
+// the cached one resolves the address again.
+struct ScratchSlot {
+  unsigned long long ctx_id;
+  void* addr;
+};
 std::mutex g_setup_mu;
-void* g_scratch_addr[kMaxDevices] = {};
+ScratchSlot g_slot[kMaxDevices] = {};
 
-// Once per device, with that device current: resolve the scratch address.
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
+typedef CUresult (*CtxGetIdFn)(CUcontext, unsigned long long*);
+
+bool driver_fns(CtxGetCurrentFn* get_current, CtxGetIdFn* get_id) {
+  static CtxGetCurrentFn cur = nullptr;
+  static CtxGetIdFn id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult qr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &qr) == cudaSuccess &&
+        qr == cudaDriverEntryPointSuccess)
+      cur = reinterpret_cast<CtxGetCurrentFn>(p);
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &qr) == cudaSuccess &&
+        qr == cudaDriverEntryPointSuccess)
+      id = reinterpret_cast<CtxGetIdFn>(p);
+  });
+  *get_current = cur;
+  *get_id = id;
+  return cur && id;
+}
+
+// The identifier of the context current on this thread (0 if none is).
+cudaError_t current_ctx_id(unsigned long long* out) {
+  CtxGetCurrentFn get_current;
+  CtxGetIdFn get_id;
+  if (!driver_fns(&get_current, &get_id)) return cudaErrorNotSupported;
+  CUcontext ctx = nullptr;
+  if (get_current(&ctx) != CUDA_SUCCESS) return cudaErrorDeviceUninitialized;
+  *out = 0;
+  if (ctx && get_id(ctx, out) != CUDA_SUCCESS) return cudaErrorDeviceUninitialized;
+  return cudaSuccess;
+}
+
+// Set-up, with the device current: resolve the array's address once per
+// device and context (cudaGetSymbolAddress, return code checked).
 cudaError_t scratch_address(void** out) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  unsigned long long ctx = 0;
+  if ((e = current_ctx_id(&ctx)) != cudaSuccess) return e;
   std::lock_guard<std::mutex> lk(g_setup_mu);
-  if (!g_scratch_addr[dev]) {
+  if (ctx == 0 || !g_slot[dev].addr || g_slot[dev].ctx_id != ctx) {
     void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);  // makes the device's primary context current if none was
     if (e != cudaSuccess) return e;
-    g_scratch_addr[dev] = p;
+    if ((e = current_ctx_id(&ctx)) != cudaSuccess) return e;
+    if (ctx == 0) return cudaErrorDeviceUninitialized;
+    g_slot[dev].ctx_id = ctx;
+    g_slot[dev].addr = p;
   }
-  *out = g_scratch_addr[dev];
+  *out = g_slot[dev].addr;
   return cudaSuccess;
 }
 
@@ -46,16 +96,24 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 }  // namespace
 
+namespace stl {
+
+cudaError_t noalloc_error_word(uint32_t** word) {
+  void* base = nullptr;
+  cudaError_t e = scratch_address(&base);
+  if (e == cudaSuccess) *word = static_cast<uint32_t*>(base);
+  return e;
+}
+
+}  // namespace stl
+
 extern "C" stlite_status stlite_score_noalloc(const stlite_shape* s, const void* q, const void* k,
                                               float* a_base, void* stream) {
-  if (!s || !q || !k || !a_base) return STLITE_EINVAL;
-  if (!aligned16(q) || !aligned16(k) || !aligned16(a_base)) return STLITE_EINVAL;
-  if (s->n_tokens < 1 || s->n_q_heads < 1 || s->n_kv_heads < 1 || s->window < 1 || s->head_dim < 1)
-    return STLITE_EINVAL;
-  if (s->n_q_heads % s->n_kv_heads != 0) return STLITE_EINVAL;
-  if (s->dtype != STLITE_BF16 && s->dtype != STLITE_F32) return STLITE_EINVAL;
-  if (s->head_dim != STLITE_HEAD_DIM || s->window > 256) return STLITE_EUNSUPPORTED;
-  if ((long long)s->window * (s->n_q_heads / s->n_kv_heads) > 512) return STLITE_EUNSUPPORTED;
+  // the shape limits of stlite_score, then the fixed scratch's capacity, then
+  // the pointers: a problem too large for the array is refused whatever the
+  // pointers are
+  stlite_status status = check_shape(s);
+  if (status != STLITE_OK) return status;
   Problem p;
   p.n = s->n_tokens;
   p.hq = s->n_q_heads;
@@ -68,6 +126,8 @@ extern "C" stlite_status stlite_score_noalloc(const stlite_shape* s, const void*
   const WsPlan plan = plan_workspace(p, ft);
   const size_t stats = (size_t)p.hkv * plan.nsplit * p.R() * 8 + (size_t)p.hkv * p.R() * 4;
   if (kErrBytes + stats > kScratchBytes) return STLITE_EUNSUPPORTED;  // beyond the fixed scratch
+  if (!q || !k || !a_base) return STLITE_EINVAL;
+  if (!aligned16(q) || !aligned16(k) || !aligned16(a_base)) return STLITE_EINVAL;
   void* base = nullptr;
   if (scratch_address(&base) != cudaSuccess) return STLITE_ECUDA;
   cudaStream_t st = static_cast<cudaStream_t>(stream);

@@ -363,6 +363,8 @@ def decode_attention(q, k, v, stream=None):
 
 
 def stlite_device_status(ws, stream=None) -> int:
+    """Reads and clears a workspace's device error word; ws=None reads the
+    error word of stlite_score_noalloc's fixed scratch on the current device."""
     st = ctypes.c_int32(0)
     _check(_lib.stlite_device_status(_ptr(ws), _stream(stream), ctypes.byref(st)), "stlite_device_status")
     return int(st.value)

@@ -21,6 +21,22 @@ def st():
     return stlite
 
 
+@pytest.fixture(scope="module")
+def good():
+    """A 16-byte-aligned address the rejection tests pass where a tensor is
+    expected: a real 32 MiB device allocation (larger than any buffer these
+    shapes describe) when a CUDA device is present, so that no unmapped
+    address could reach a kernel even if a host check regressed; without a
+    device, where nothing can launch, a stand-in value."""
+    import torch
+    if torch.cuda.is_available():
+        buf = torch.zeros(32 << 20, dtype=torch.uint8, device="cuda")
+        yield buf.data_ptr()
+        del buf
+    else:
+        yield 0x10000
+
+
 def header_functions():
     text = open(os.path.join(ROOT, "include", "stlite.h")).read()
     return sorted(set(re.findall(r"STLITE_API\s+[\w\s\*]+?\b(stlite_\w+)\s*\(", text)))
@@ -79,7 +95,7 @@ def test_workspace_size_and_validation(st):
         assert e.value.status == code
 
 
-def test_entry_points_reject_before_launch(st):
+def test_entry_points_reject_before_launch(st, good):
     """Malformed pointers and sizes are refused on the host (no GPU needed)."""
     lib = st._lib
     sh = _shape(st)
@@ -87,8 +103,8 @@ def test_entry_points_reject_before_launch(st):
     prm = st.make_params(0.2)
     need = st.stlite_workspace_size(sh, fr, prm)
     P = ctypes.c_void_p
-    good = P(0x10000)
-    mis = P(0x10008)          # not 16-byte aligned
+    mis = P(good + 8)          # not 16-byte aligned
+    good = P(good)
     assert lib.stlite_score(ctypes.byref(sh), None, good, good, good, need, None) == st.STLITE_EINVAL
     assert lib.stlite_score(ctypes.byref(sh), mis, good, good, good, need, None) == st.STLITE_EINVAL
     # stlite_score takes no frames: its workspace is the frame-less size
@@ -162,14 +178,13 @@ def test_hierarchical_budgets_reject(st):
             st.stlite_hierarchical_budgets(mass, total, n_tokens)
 
 
-def test_compress_layers_budgets_reject_before_launch(st):
+def test_compress_layers_budgets_reject_before_launch(st, good):
     """Per-layer budgets outside [1, N] and NULL arrays are refused on the host."""
     lib = st._lib
     sh = _shape(st)
     fr = st.FrameSpec([0, 30], [4, 5], [5, 6])
     prm = st.make_params(0.2)
     need = st.stlite_workspace_size(sh, fr, prm)
-    good = 0x10000
     lay = (st.LayerIO * 2)(st.LayerIO(*([good] * 6)), st.LayerIO(*([good] * 6)))
     P = ctypes.c_void_p
     for bud in ([20, 0], [20, 101], [-1, 20]):
@@ -186,14 +201,14 @@ def test_compress_layers_budgets_reject_before_launch(st):
                                               arr, P(good), 2 * need, None) == st.STLITE_EINVAL
 
 
-def test_variant_params_validation(st):
+def test_variant_params_validation(st, good):
     """CSS sizes other than 0/3/5/7/9 and unknown A_base scalings are refused
     on the host, in the fused and in the staged entry points."""
     lib = st._lib
     sh = _shape(st)
     fr = st.FrameSpec([0, 30], [4, 5], [5, 6])
     need = st.stlite_workspace_size(sh, fr, st.make_params(0.2))
-    good = ctypes.c_void_p(0x10000)
+    good = ctypes.c_void_p(good)
     for kw in (dict(css_size=4), dict(css_size=11), dict(css_size=-3), dict(abase_norm=2), dict(abase_norm=-1)):
         prm = st.make_params(0.2, **kw)
         assert lib.stlite_compress_layer(ctypes.byref(sh), ctypes.byref(fr.c), ctypes.byref(prm), good, good, good,
@@ -207,7 +222,7 @@ def test_variant_params_validation(st):
         assert st.stlite_workspace_size(sh, fr, st.make_params(0.2, css_size=size, abase_norm=1)) == need
 
 
-def test_varlen_layers_validation(st):
+def test_varlen_layers_validation(st, good):
     """stlite_compress_varlen_layers refuses a short workspace and malformed
     layer arrays on the host."""
     lib = st._lib
@@ -217,7 +232,6 @@ def test_varlen_layers_validation(st):
     need = st.stlite_workspace_size_varlen(sh, [0, 100, 200, 300], fr, prm)
     cu, specs, arr = st._varlen_args([0, 100, 200, 300], fr)
     ip = ctypes.POINTER(ctypes.c_int32)
-    good = 0x10000
     lay = (st.LayerIO * 2)(st.LayerIO(*([good] * 6)), st.LayerIO(*([good] * 6)))
     call = lambda layers, n, ws_bytes: lib.stlite_compress_varlen_layers(
         ctypes.byref(sh), 3, cu.ctypes.data_as(ip), arr, ctypes.byref(prm), n, layers, None,
@@ -227,3 +241,56 @@ def test_varlen_layers_validation(st):
     assert call(lay, 0, 2 * need) == st.STLITE_EINVAL
     bad = (st.LayerIO * 2)(st.LayerIO(*([good] * 6)), st.LayerIO(*([good] * 5 + [0])))
     assert call(bad, 2, 2 * need) == st.STLITE_EINVAL
+
+
+NOALLOC_SCRATCH = 2 << 20
+
+
+def _noalloc_need(hkv, r, splits):
+    return 256 + hkv * splits * r * 8 + hkv * r * 4
+
+
+@pytest.mark.parametrize("n,hq,hkv,w,dt", [
+    (53600, 28, 4, 32, 0), (132800, 28, 4, 64, 0), (20960, 12, 2, 16, 0), (1152, 28, 4, 32, 1),
+    (5000, 400, 400, 1, 1), (5000, 400, 400, 1, 0), (100000, 64, 64, 8, 1), (100000, 64, 64, 8, 0),
+    (100000, 256, 16, 32, 1), (100000, 256, 16, 32, 0), (300, 8, 1, 64, 1), (64, 4096, 1024, 128, 0),
+    (64, 4096, 1024, 128, 1), (5000, 1024, 1024, 1, 1), (100000, 1024, 512, 1, 0)])
+def test_noalloc_scratch_bound(st, n, hq, hkv, w, dt):
+    """The no-workspace window score's capacity rule, checked on the host: a
+    shape whose scratch fits in the fixed 2 MiB even with the documented
+    largest split count, S = max(4, 4 ceil(304 / Hkv)), passes the capacity
+    check (and then fails only on the NULL pointers given here); a shape that
+    does not fit even with one split is refused as unsupported.  Nothing can
+    launch: the pointers are NULL."""
+    sh = st.Shape(n, hq, hkv, 128, w, dt)
+    r = w * (hq // hkv)
+    s_max = max(4, 4 * (-(-304 // hkv)))
+    got = st._lib.stlite_score_noalloc(ctypes.byref(sh), None, None, None, None)
+    if _noalloc_need(hkv, r, s_max) <= NOALLOC_SCRATCH:
+        assert got == st.STLITE_EINVAL
+    elif _noalloc_need(hkv, r, 1) > NOALLOC_SCRATCH:
+        assert got == st.STLITE_EUNSUPPORTED
+    else:
+        assert got in (st.STLITE_EINVAL, st.STLITE_EUNSUPPORTED)
+
+
+def test_noalloc_shape_limits_match_score(st):
+    """stlite_score_noalloc applies the same shape limits as stlite_score
+    (both refuse before looking at any pointer)."""
+    for sh, code in [(st.Shape(100, 5, 2, 128, 4, 0), st.STLITE_EINVAL),
+                     (st.Shape(100, 4, 2, 64, 4, 0), st.STLITE_EUNSUPPORTED),
+                     (st.Shape(100, 4, 2, 128, 300, 0), st.STLITE_EUNSUPPORTED),
+                     (st.Shape(100, 4 * 5000, 5000, 128, 1, 1), st.STLITE_EUNSUPPORTED),
+                     (st.Shape(1 << 29, 4, 4, 128, 1, 1), st.STLITE_EUNSUPPORTED),
+                     (st.Shape(0, 4, 2, 128, 4, 0), st.STLITE_EINVAL)]:
+        assert st._lib.stlite_score_noalloc(ctypes.byref(sh), None, None, None, None) == code
+        assert st._lib.stlite_score(ctypes.byref(sh), None, None, None, None, 0, None) == code
+
+
+def test_device_status_without_scratch_argument(st):
+    """stlite_device_status(NULL, ...) reads the no-workspace scratch; a NULL
+    status pointer or a misaligned workspace is refused on the host."""
+    lib = st._lib
+    assert lib.stlite_device_status(None, None, None) == st.STLITE_EINVAL
+    status = ctypes.c_int32(0)
+    assert lib.stlite_device_status(ctypes.c_void_p(0x10008), None, ctypes.byref(status)) == st.STLITE_EINVAL
