@@ -212,17 +212,35 @@ def kernel_roofline(name: str, t_launch: float, layers: int, budget: int, peaks)
 
 # --------------------------------------------------------------- oracle arm
 
+def bench_config(layers: int, budget: int, world: int) -> dict:
+    """The workload description both arms print (same keys and values)."""
+    return dict(workload=WORKLOAD, layers=layers, n_tokens=N_TOK, frames=N_STEPS, grid="%dx%d" % (GH, GW),
+                text_per_step=N_TEXT, q_heads=HQ, kv_heads=HKV, head_dim=D, window=W, beta=BETA,
+                budget=budget, l2="inputs larger than L2 (%.2f GB K/V per step)" %
+                (2 * layers * N_TOK * HKV * D * 2 / 1e9),
+                timing="CUDA graph of one step (one stlite_compress_layers call), replayed",
+                parallelism="dp%d" % world)
+
+
+def bf16_inputs(wl):
+    """The workload's q and k as the bf16 values the GPU arm computes on,
+    exactly converted to float64 for the oracle."""
+    import torch
+    q = torch.from_numpy(wl.q).to(torch.bfloat16).to(torch.float64).numpy()
+    k = torch.from_numpy(wl.k).to(torch.bfloat16).to(torch.float64).numpy()
+    return q, k
+
+
 def oracle_sample(wl, pool_stride: int = 16, q_heads: int = HQ // HKV):
-    """Times the oracle on KV head 0 of one layer: the window score of
-    `q_heads` of the head's G query heads, CSS, the TSG threshold and gate,
-    integrated score and top-B in full, and rho on every pool_stride-th
-    historical token.  Returns the seconds extrapolated to the whole layer
-    (all query heads, every historical token, all KV heads), the measured
-    seconds, and a description of the sample."""
+    """Times the oracle single-threaded on KV head 0 of one layer: the
+    window score of `q_heads` of the head's G query heads, CSS, the TSG
+    threshold and gate, integrated score and top-B in full, and rho on every
+    pool_stride-th historical token.  Returns the seconds extrapolated to the
+    whole layer (all query heads, every historical token, all KV heads), the
+    measured seconds, and a description of the sample."""
     import oracle
     G = HQ // HKV
-    q64 = wl.q.astype(np.float64)
-    k64 = wl.k.astype(np.float64)
+    q64, k64 = bf16_inputs(wl)
     off, gh, gw = wl.frames
     b = oracle.budget(wl.n, wl.beta)
     kh = np.ascontiguousarray(k64[:, :1])
@@ -232,11 +250,9 @@ def oracle_sample(wl, pool_stride: int = 16, q_heads: int = HQ // HKV):
     t1 = time.perf_counter()
     phi = oracle.css_phi(kh, wl.frames)
     t2 = time.perf_counter()
-    pool = np.concatenate([np.arange(o, o + x * y) for o, x, y in zip(off[:-1], gh[:-1], gw[:-1])])
+    pool = oracle.pool_tokens(wl.frames)
     sample = pool[::pool_stride]
-    rho = np.full((1, wl.n), np.nan)
-    for i in sample:
-        rho[0, i] = oracle.tsg_rho_token(kh, 0, int(i), wl.frames)
+    rho = oracle.tsg_rho(kh, wl.frames, tokens=sample)
     t3 = time.perf_counter()
     rho[0, pool] = np.nan_to_num(rho[0, pool], nan=0.5)   # unsampled tokens: placeholder values
     tau, gate, _ = oracle.tsg_gate(rho, wl.frames, b)
@@ -244,37 +260,80 @@ def oracle_sample(wl, pool_stride: int = 16, q_heads: int = HQ // HKV):
     oracle.topk(s, b)
     t4 = time.perf_counter()
     per_head = (t1 - t0) * (G / q_heads) + (t2 - t1) + (t3 - t2) * (len(pool) / len(sample)) + (t4 - t3)
-    note = ("oracle on KV head 0 of one layer: window score of %d/%d query heads, CSS, gate and top-B in "
-            "full, rho on 1/%d of the %d historical tokens; extrapolated to all query heads, all historical "
+    note = ("oracle on 1 thread, KV head 0 of one layer: window score of %d/%d query heads, CSS, gate and top-B "
+            "in full, rho on 1/%d of the %d historical tokens; extrapolated to all query heads, all historical "
             "tokens and %d KV heads" % (q_heads, G, pool_stride, len(pool), HKV))
     return per_head * HKV, t4 - t0, note
 
 
+def oracle_layer(wl, threads: int, pool_stride: int = 1):
+    """Times the oracle on one whole layer (all KV heads and query heads) on
+    `threads` host threads: window score, CSS, rho on every pool_stride-th
+    historical token (all of them at stride 1), threshold, gate, integrated
+    score and top-B.  Returns the seconds for the whole layer (rho's time
+    scaled by the pool fraction when strided), the measured seconds, and a
+    description."""
+    import oracle
+    q64, k64 = bf16_inputs(wl)
+    b = oracle.budget(wl.n, wl.beta)
+    t0 = time.perf_counter()
+    a = oracle.abase(q64, k64, threads=threads)
+    t1 = time.perf_counter()
+    phi = oracle.css_phi(k64, wl.frames, threads=threads)
+    t2 = time.perf_counter()
+    pool = oracle.pool_tokens(wl.frames)
+    sample = pool[::pool_stride]
+    rho = oracle.tsg_rho(k64, wl.frames, threads=threads, tokens=sample)
+    t3 = time.perf_counter()
+    if pool_stride > 1:
+        rho[:, pool] = np.nan_to_num(rho[:, pool], nan=0.5)   # unsampled tokens: placeholder values
+    tau, gate, _ = oracle.tsg_gate(rho, wl.frames, b)
+    s = oracle.combine(a, phi, gate, wl.frames)
+    oracle.topk(s, b)
+    t4 = time.perf_counter()
+    est = (t1 - t0) + (t2 - t1) + (t3 - t2) * (len(pool) / len(sample)) + (t4 - t3)
+    if pool_stride == 1:
+        note = ("oracle on %d threads, one whole layer (all %d KV heads and %d query heads, rho of all %d "
+                "historical tokens), nothing extrapolated" % (threads, HKV, HQ, len(pool)))
+    else:
+        note = ("oracle on %d threads, one layer (all %d KV heads and %d query heads) with rho on 1/%d of the %d "
+                "historical tokens; rho's time scaled to the whole pool" % (threads, HKV, HQ, pool_stride,
+                                                                         len(pool)))
+    return est, t4 - t0, note
+
+
 def run_reference(args):
-    _, rank, _ = dist_env()
+    """The reference arm: the oracle, as it stands, on the host cores.  Each
+    step is one bounded sample of the workload (one layer with rho on 1/16 of
+    the pool, all host threads); the line reports the seconds really
+    measured per step and the throughput extrapolated from them."""
+    world, rank, _ = dist_env()
     if rank != 0:   # under torchrun rank 0 alone times the oracle; the others exit 0
         return
     sys.stdout.flush()
-    from paper_2603_00188_gb300 import synth
     import oracle
     oracle.build()
-    vals = []
-    note = ""
+    threads = oracle.host_threads()
     wls = gen_layers(2, seed=0)
-    for wl in wls:   # the bf16-rounded inputs the GPU arm sees
-        import torch
-        wl.q = torch.from_numpy(wl.q).to(torch.bfloat16).float().numpy()
-        wl.k = torch.from_numpy(wl.k).to(torch.bfloat16).float().numpy()
+    stride = 16
+    vals, measured = [], []
+    note = ""
     for step in range(args.warmup + args.steps):
-        t_layer, _, note = oracle_sample(wls[step % len(wls)], pool_stride=256, q_heads=1)
+        t_layer, t_raw, note = oracle_layer(wls[step % len(wls)], threads, pool_stride=stride)
         if step >= args.warmup:
             vals.append(N_TOK / t_layer)
+            measured.append(t_raw)
     value = statistics.mean(vals)
+    ms_step = 1e3 * statistics.mean(measured)
+    budget = oracle.budget(N_TOK, BETA)
     line = dict(impl="reference", metric=METRIC, value=value, unit=UNIT, n_gpus=args.gpus, steps=args.steps,
-                warmup=args.warmup, ms_per_step=1e3 * N_TOK * LAYERS / value, higher_is_better=True,
-                scaling="weak", vs_baseline=None, dtype="f64", data="synthetic",
-                config=dict(workload=WORKLOAD, layers=LAYERS, n_tokens=N_TOK, beta=BETA),
-                cpu_baseline=dict(value=value, unit=UNIT, cores=1, kind="oracle", sample=note),
+                warmup=args.warmup, ms_per_step=ms_step, higher_is_better=True, scaling="weak", vs_baseline=None,
+                dtype="f64", data="synthetic", config=bench_config(LAYERS, budget, max(world, args.gpus)),
+                extrapolated=True, measured_s=round(sum(measured), 3),
+                step_note="each step is one bounded sample (%s); value = N / the layer time extrapolated from "
+                          "it, ms_per_step = the sample's measured time" % note,
+                cpu_baseline=dict(value=value, unit=UNIT, cores=threads, kind="oracle", sample=note,
+                                  measured_s=round(sum(measured), 3)),
                 e2e=dict(value=value, unit=UNIT, h2d_bytes_per_step=0, d2h_bytes_per_step=0))
     print(json.dumps(line), flush=True)
 
@@ -769,22 +828,21 @@ def run_gpu(args):
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         import oracle
         oracle.build()
-        wl0 = wls[0]
-        wl0.q, wl0.k = host[0][0].float().numpy(), host[0][1].float().numpy()   # the bf16 inputs
-        t_layer, t_raw, note = oracle_sample(wl0, pool_stride=16)
-        cpu = dict(value=N_TOK / t_layer, unit=UNIT, cores=1, kind="oracle", sample=note,
-                   measured_s=round(t_raw, 2))
+        threads = oracle.host_threads()
+        # all host threads: one whole layer, nothing extrapolated
+        t_all, t_all_raw, note_all = oracle_layer(wls[0], threads, pool_stride=1)
+        # one thread: a sample of one KV head, extrapolated to the layer
+        t_one, t_one_raw, note_one = oracle_sample(wls[0], pool_stride=16)
+        cpu = dict(value=N_TOK / t_all, unit=UNIT, cores=threads, kind="oracle", sample=note_all,
+                   measured_s=round(t_all_raw, 2),
+                   single_core=dict(value=N_TOK / t_one, unit=UNIT, cores=1, sample=note_one,
+                                    measured_s=round(t_one_raw, 2), extrapolated=True))
 
     if rank == 0:
         line = dict(metric=METRIC, value=value, unit=UNIT, n_gpus=world, steps=args.steps, warmup=args.warmup,
                     ms_per_step=ms, higher_is_better=True, scaling="weak", vs_baseline=None, dtype="bf16",
                     data="synthetic",
-                    config=dict(workload=WORKLOAD, layers=L, n_tokens=N_TOK, frames=N_STEPS, grid="%dx%d" % (GH, GW),
-                                text_per_step=N_TEXT, q_heads=HQ, kv_heads=HKV, head_dim=D, window=W, beta=BETA,
-                                budget=budget, l2="inputs larger than L2 (%.2f GB K/V per step)" %
-                                (2 * L * N_TOK * HKV * D * 2 / 1e9),
-                                timing="CUDA graph of one step (one stlite_compress_layers call), replayed",
-                                parallelism="dp%d" % world),
+                    config=bench_config(L, budget, world),
                     hbm=dict(achieved_gbs=alg_bytes_per_layer(budget) * L / (ms * 1e-3) / 1e9,
                              peak_gbs=peaks["hbm"],
                              frac=alg_bytes_per_layer(budget) * L / (ms * 1e-3) / 1e9 / peaks["hbm"],

@@ -51,6 +51,10 @@ def _load():
         lib.orc_budget.argtypes = [_i32, ctypes.c_double, _i32]
         lib.orc_abase.restype = None
         lib.orc_abase.argtypes = [_dp, _dp, _i32, _i32, _i32, _i32, _i32, _i32, _dp]
+        lib.orc_abase_qhead.restype = None
+        lib.orc_abase_qhead.argtypes = [_dp, _dp, _i32, _i32, _i32, _i32, _i32, _i32, _dp]
+        lib.orc_tsg_rho_tokens.restype = None
+        lib.orc_tsg_rho_tokens.argtypes = [_dp, _i32, _i32, _i32, _ip, _i32, _i32, _i32, _i32, _dp]
         lib.orc_css_phi_token.restype = ctypes.c_double
         lib.orc_css_phi_token.argtypes = [_dp, _i32, _i32, _i32, _i32, _i32, _i32, _i32, _i32, _i32]
         lib.orc_css_phi.restype = None
@@ -87,12 +91,27 @@ def _frames(frames):
 
 
 def _per_head(fn, hkv, threads):
-    if threads and threads > 1 and hkv > 1:
-        with ThreadPoolExecutor(max_workers=min(threads, hkv)) as ex:
-            list(ex.map(fn, range(hkv)))
+    _run_tasks(fn, list(range(hkv)), threads)
+
+
+def _run_tasks(fn, tasks, threads):
+    """Runs fn on every task, on `threads` threads (the C calls release the
+    GIL); each task writes its own slice of the output, so the result does
+    not depend on the thread count."""
+    if threads and threads > 1 and len(tasks) > 1:
+        with ThreadPoolExecutor(max_workers=min(threads, len(tasks))) as ex:
+            list(ex.map(fn, tasks))
     else:
-        for h in range(hkv):
-            fn(h)
+        for t in tasks:
+            fn(t)
+
+
+def host_threads() -> int:
+    """Threads this process may run on (its CPU affinity)."""
+    try:
+        return len(os.sched_getaffinity(0))
+    except (AttributeError, OSError):
+        return os.cpu_count() or 1
 
 
 def budget(n: int, beta: float, k_override: int = 0) -> int:
@@ -126,18 +145,41 @@ def hierarchical_budgets(layer_mass, total_budget: int, n_tokens: int) -> list:
 
 
 def abase(q, k, threads: int = 1) -> np.ndarray:
-    """Eq. 2 window score per KV head (mean over the G query heads of a group)."""
+    """Eq. 2 window score per KV head (mean over the G query heads of a group):
+    each query head's sum over the window rows of its softmax rows is one
+    task (``orc_abase_qhead``), and A[h] = (1/G) * the sum of its group's
+    partials in query-head order."""
     lib = _load()
     q, k = _c64(q), _c64(k)
     w, hq, d = q.shape
     n, hkv, d2 = k.shape
     assert d == d2 and hq % hkv == 0
+    G = hq // hkv
+    part = np.zeros((hq, n), dtype=np.float64)
+
+    def run(g):
+        lib.orc_abase_qhead(_d(q), _d(k), n, w, hq, hkv, d, g, part[g].ctypes.data_as(_dp))
+
+    _run_tasks(run, list(range(hq)), threads)
     out = np.zeros((hkv, n), dtype=np.float64)
+    for h in range(hkv):
+        for g in range(h * G, (h + 1) * G):
+            out[h] += part[g]
+        out[h] /= G
+    return out
 
-    def run(h):
+
+def abase_per_head(q, k) -> np.ndarray:
+    """Eq. 2 computed head by head in one pass (``orc_abase``: the G query
+    heads and w rows of a group accumulated into A directly); the same
+    quantity as ``abase``, kept as a cross-check of its task split."""
+    lib = _load()
+    q, k = _c64(q), _c64(k)
+    w, hq, d = q.shape
+    n, hkv, d2 = k.shape
+    out = np.zeros((hkv, n), dtype=np.float64)
+    for h in range(hkv):
         lib.orc_abase(_d(q), _d(k), n, w, hq, hkv, d, h, out[h].ctypes.data_as(_dp))
-
-    _per_head(run, hkv, threads)
     return out
 
 
@@ -171,21 +213,62 @@ def css_phi_token(k, h: int, off: int, gh: int, gw: int, u: int, v: int, size: i
 TSG_COSINE, TSG_DOT, TSG_NEG_L2 = 0, 1, 2
 
 
-def tsg_rho(k, frames, threads: int = 1, metric: int = TSG_COSINE) -> np.ndarray:
+def pool_tokens(frames) -> np.ndarray:
+    """The historical pool T_pool: the visual tokens of frames 0..F-2, ascending."""
+    off, gh, gw = _frames(frames)
+    if len(off) < 2:
+        return np.zeros(0, np.int32)
+    return np.concatenate([np.arange(o, o + a * b, dtype=np.int32) for o, a, b in
+                           zip(off[:-1], gh[:-1], gw[:-1])])
+
+
+def tsg_rho(k, frames, threads: int = 1, metric: int = TSG_COSINE, chunk: int = 2048,
+            tokens=None) -> np.ndarray:
     """Eq. 6: rho_i = max similarity to the current frame (cosine; or, for the
     similarity-metric ablation, dot product / negative squared L2 distance);
-    NaN outside the pool."""
+    NaN outside the pool.  The pool (visual tokens of frames 0..F-2) is cut
+    into runs of `chunk` tokens per KV head, one task each
+    (``orc_tsg_rho_tokens``), so that every host core can take part.
+    ``tokens`` (a subset of the pool) restricts the computation to those
+    tokens; every other entry is NaN."""
+    lib = _load()
+    k = _c64(k)
+    n, hkv, d = k.shape
+    off, gh, gw = _frames(frames)
+    out = np.full((hkv, n), np.nan, dtype=np.float64)
+    if len(off) < 2:
+        return out
+    pool = pool_tokens(frames)
+    if tokens is not None:
+        tokens = np.asarray(tokens, dtype=np.int32)
+        assert np.isin(tokens, pool).all(), "tokens outside the historical pool"
+        pool = tokens
+    cur_off, cur_len = int(off[-1]), int(gh[-1] * gw[-1])
+    tasks = [(h, c) for h in range(hkv) for c in range(0, len(pool), chunk)]
+
+    def run(t):
+        h, c = t
+        tok = np.ascontiguousarray(pool[c:c + chunk])
+        vals = np.zeros(len(tok), dtype=np.float64)
+        lib.orc_tsg_rho_tokens(_d(k), hkv, d, h, tok.ctypes.data_as(_ip), len(tok), cur_off, cur_len,
+                               int(metric), vals.ctypes.data_as(_dp))
+        out[h, tok] = vals
+
+    _run_tasks(run, tasks, threads)
+    return out
+
+
+def tsg_rho_per_head(k, frames, metric: int = TSG_COSINE) -> np.ndarray:
+    """Eq. 6 in one pass per KV head over the frames (``orc_tsg_rho``); the
+    same quantity as ``tsg_rho``, kept as a cross-check of its task split."""
     lib = _load()
     k = _c64(k)
     n, hkv, d = k.shape
     off, gh, gw = _frames(frames)
     out = np.zeros((hkv, n), dtype=np.float64)
-
-    def run(h):
+    for h in range(hkv):
         lib.orc_tsg_rho(_d(k), n, hkv, d, h, len(off), off.ctypes.data_as(_ip),
                         gh.ctypes.data_as(_ip), gw.ctypes.data_as(_ip), int(metric), out[h].ctypes.data_as(_dp))
-
-    _per_head(run, hkv, threads)
     return out
 
 

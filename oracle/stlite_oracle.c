@@ -109,6 +109,31 @@ void orc_abase(const double* q, const double* k, int32_t n, int32_t w, int32_t h
   free(logit);
 }
 
+/* The inner sum of Eq. 2 for the single query head g: partial[j] =
+ * sum_{r < w} softmax_j(q_{r,g} . k_{j,h} / sqrt(d)), h = g / G (not yet
+ * divided by G).  A_base of KV head h is the mean of these partials over
+ * the G query heads of its group (reading R1); the test drivers run the
+ * query heads on separate threads and add the partials afterwards. */
+void orc_abase_qhead(const double* q, const double* k, int32_t n, int32_t w, int32_t hq,
+                     int32_t hkv, int32_t d, int32_t g, double* partial) {
+  int32_t G = hq / hkv, h = g / G;
+  double inv_sqrt_d = 1.0 / sqrt((double)d);
+  double* logit = (double*)malloc(sizeof(double) * (size_t)(n > 0 ? n : 1));
+  for (int32_t j = 0; j < n; ++j) partial[j] = 0.0;
+  for (int32_t r = 0; r < w; ++r) {
+    const double* qrow = q + ((size_t)r * hq + g) * d;
+    double mx = -INFINITY;
+    for (int32_t j = 0; j < n; ++j) {
+      logit[j] = dot(qrow, key_row(k, hkv, d, j, h), d) * inv_sqrt_d;
+      if (logit[j] > mx) mx = logit[j];
+    }
+    double z = 0.0;
+    for (int32_t j = 0; j < n; ++j) z += exp(logit[j] - mx);
+    for (int32_t j = 0; j < n; ++j) partial[j] += exp(logit[j] - mx) / z;
+  }
+  free(logit);
+}
+
 /* --------------------------------------------- CSS saliency (Eqs. 4-5) */
 
 /* Phi for one visual token at (u, v) of frame f, KV head h (Eqs. 4-5):
@@ -172,6 +197,16 @@ double orc_tsg_rho_token(const double* k, int32_t hkv, int32_t d, int32_t h, int
     if (c > best) best = c;
   }
   return best;
+}
+
+/* rho of the listed tokens (each a member of the historical pool) against
+ * the current frame [cur_off, cur_off + cur_len): the per-token step of
+ * Algorithm 1's ComputeScores, for test drivers that spread the pool over
+ * threads. */
+void orc_tsg_rho_tokens(const double* k, int32_t hkv, int32_t d, int32_t h, const int32_t* tok,
+                        int32_t count, int32_t cur_off, int32_t cur_len, int32_t metric, double* out) {
+  for (int32_t t = 0; t < count; ++t)
+    out[t] = orc_tsg_rho_token(k, hkv, d, h, tok[t], cur_off, cur_len, metric);
 }
 
 /* rho for every token of the historical pool T_pool (visual tokens of frames

@@ -89,7 +89,7 @@ def test_kernel_roofline_units(bench):
             < 0.01 * bench.kernel_roofline("rowstats_umma", t, 1, 10720, peaks)["achieved"])
 
 
-def test_reference_arm_line():
+def test_reference_arm_line(bench):
     # `bench.py --impl reference` times the oracle on the host and prints one
     # JSON line in the bench's own metric, unit and workload
     import subprocess
@@ -103,8 +103,16 @@ def test_reference_arm_line():
     assert d["impl"] == "reference" and d["value"] > 0 and d["higher_is_better"] is True
     assert d["metric"].startswith("KV tokens compressed/sec") and d["unit"] == "tokens/s/layer"
     assert d["config"]["layers"] == 28 and d["config"]["n_tokens"] == 53600
+    # the same workload description as the GPU arm's line
+    assert d["config"] == bench.bench_config(28, 10720, 1)
+    # the timing claimed is the timing measured: steps x ms_per_step is the
+    # measured time of the timed samples, and the value is extrapolated from it
+    assert d["steps"] == 1 and d["extrapolated"] is True
+    assert abs(d["steps"] * d["ms_per_step"] - 1e3 * d["measured_s"]) <= 1.0
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"] and cb["sample"]
+    import oracle
+    assert cb["cores"] == oracle.host_threads()
     e = d["e2e"]
     assert e["value"] == d["value"] and e["unit"] == d["unit"]
     assert e["h2d_bytes_per_step"] == 0 and e["d2h_bytes_per_step"] == 0

@@ -765,3 +765,34 @@ def test_abase_max_normalisation():
     u = oracle.compress_layer(q, kk, fr, beta=0.3, tsg_enable=0, css_enable=0, abase_norm=oracle.ABASE_MAX)
     np.testing.assert_array_equal(u["s"], 1.0)
     np.testing.assert_array_equal(u["idx"], np.tile(np.arange(u["budget"]), (k.shape[1], 1)))
+
+
+# ------------------------------------------- task splits of the oracle drivers
+
+@pytest.mark.parametrize("threads", [1, 3])
+def test_abase_task_split_matches_single_pass(threads):
+    # Eq. 2 (reading R1): the per-query-head partials summed per group equal
+    # the group accumulated in one pass, whatever the thread count; the two
+    # differ only in the order of the fp64 additions.
+    wl = synth.scaled("long", 2, beta=0.1)
+    q, k = wl.q[:, :8].astype(np.float64), wl.k[:2000, :1].astype(np.float64)
+    a1 = oracle.abase(q, k, threads=threads)
+    a2 = oracle.abase_per_head(q, k)
+    np.testing.assert_allclose(a1, a2, rtol=1e-12, atol=0)
+    np.testing.assert_allclose(a1.sum(1), q.shape[0], rtol=1e-12)
+
+
+@pytest.mark.parametrize("threads,chunk", [(1, 2048), (4, 97), (3, 1)])
+def test_rho_task_split_matches_single_pass(threads, chunk):
+    # Eq. 6: the pool cut into token runs (ragged last run, one-token runs)
+    # gives exactly the per-head pass's values, NaN outside the pool.
+    wl = synth.scaled("traj50", 3)
+    k = wl.k.astype(np.float64)
+    r1 = oracle.tsg_rho(k, wl.frames, threads=threads, chunk=chunk)
+    r2 = oracle.tsg_rho_per_head(k, wl.frames)
+    np.testing.assert_array_equal(np.isnan(r1), np.isnan(r2))
+    np.testing.assert_array_equal(r1[~np.isnan(r1)], r2[~np.isnan(r2)])
+    for metric in (oracle.TSG_DOT, oracle.TSG_NEG_L2):
+        np.testing.assert_array_equal(
+            np.nan_to_num(oracle.tsg_rho(k, wl.frames, threads=threads, chunk=chunk, metric=metric), nan=7.0),
+            np.nan_to_num(oracle.tsg_rho_per_head(k, wl.frames, metric=metric), nan=7.0))
