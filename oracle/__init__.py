@@ -53,6 +53,8 @@ def _load():
         lib.orc_abase.argtypes = [_dp, _dp, _i32, _i32, _i32, _i32, _i32, _i32, _dp]
         lib.orc_abase_qhead.restype = None
         lib.orc_abase_qhead.argtypes = [_dp, _dp, _i32, _i32, _i32, _i32, _i32, _i32, _dp]
+        lib.orc_prompt_qhead.restype = None
+        lib.orc_prompt_qhead.argtypes = [_dp, _dp, _i32, _i32, _i32, _i32, _i32, _i32, _dp]
         lib.orc_tsg_rho_tokens.restype = None
         lib.orc_tsg_rho_tokens.argtypes = [_dp, _i32, _i32, _i32, _ip, _i32, _i32, _i32, _i32, _dp]
         lib.orc_css_phi_token.restype = ctypes.c_double
@@ -180,6 +182,42 @@ def abase_per_head(q, k) -> np.ndarray:
     out = np.zeros((hkv, n), dtype=np.float64)
     for h in range(hkv):
         lib.orc_abase(_d(q), _d(k), n, w, hq, hkv, d, h, out[h].ctypes.data_as(_dp))
+    return out
+
+
+PROMPT_FULL, PROMPT_MEAN = 0, 1
+
+
+def prompt_abase(q_prompt, k, mode: int = PROMPT_MEAN, threads: int = 1) -> np.ndarray:
+    """Prompt-wide base scores of the base-scoring ablation (appendix
+    "Sensitivity to the Base Attention Scoring Function").  q_prompt
+    [n_q, Hq, d] are the query rows of the last n_q cached positions, each
+    attending causally (keys up to its own position).  PROMPT_FULL (the
+    full-attention "snapshot" base): A[h][j] = (1/G) sum over the group's query
+    heads and every prompt row of its softmax probability of key j.
+    PROMPT_MEAN (Mean Attention, 1D average pooling over the prompt): the same
+    sum divided by the number of prompt rows that attend to j."""
+    lib = _load()
+    q, k = _c64(q_prompt), _c64(k)
+    n_q, hq, d = q.shape
+    n, hkv, d2 = k.shape
+    assert d == d2 and hq % hkv == 0 and 1 <= n_q <= n
+    G = hq // hkv
+    part = np.zeros((hq, n), dtype=np.float64)
+
+    def run(g):
+        lib.orc_prompt_qhead(_d(q), _d(k), n, n_q, hq, hkv, d, g, part[g].ctypes.data_as(_dp))
+
+    _run_tasks(run, list(range(hq)), threads)
+    out = np.zeros((hkv, n), dtype=np.float64)
+    for h in range(hkv):
+        for g in range(h * G, (h + 1) * G):
+            out[h] += part[g]
+        out[h] /= G
+    if mode == PROMPT_MEAN:
+        j = np.arange(n)
+        count = np.minimum(n_q, n - j).astype(np.float64)   # rows r with n - n_q + r >= j
+        out /= count[None, :]
     return out
 
 

@@ -134,6 +134,37 @@ void orc_abase_qhead(const double* q, const double* k, int32_t n, int32_t w, int
   free(logit);
 }
 
+/* Prompt-wide base scores (appendix "Sensitivity to the Base Attention
+ * Scoring Function": the Mean Attention base and the full-attention
+ * "snapshot" base), partial sum of the single query head g.  The last n_q
+ * cached positions are the prompt's query rows: row r sits at position
+ * p_r = n - n_q + r and, as in the model's causal prefill, attends to the
+ * keys j <= p_r only (reading R18):
+ *   partial[j] = sum_{r : p_r >= j} softmax_{j' <= p_r}(q_{r,g} . k_{j',h} / sqrt(d))_j,
+ * h = g / G.  The full-attention base of KV head h is the mean of these
+ * partials over its G query heads; the Mean Attention base divides that by
+ * the number of prompt rows that attend to j (reading R19). */
+void orc_prompt_qhead(const double* q, const double* k, int32_t n, int32_t n_q, int32_t hq,
+                      int32_t hkv, int32_t d, int32_t g, double* partial) {
+  int32_t G = hq / hkv, h = g / G;
+  double inv_sqrt_d = 1.0 / sqrt((double)d);
+  double* logit = (double*)malloc(sizeof(double) * (size_t)(n > 0 ? n : 1));
+  for (int32_t j = 0; j < n; ++j) partial[j] = 0.0;
+  for (int32_t r = 0; r < n_q; ++r) {
+    const int32_t pos = n - n_q + r;  /* keys 0..pos are visible */
+    const double* qrow = q + ((size_t)r * hq + g) * d;
+    double mx = -INFINITY;
+    for (int32_t j = 0; j <= pos; ++j) {
+      logit[j] = dot(qrow, key_row(k, hkv, d, j, h), d) * inv_sqrt_d;
+      if (logit[j] > mx) mx = logit[j];
+    }
+    double z = 0.0;
+    for (int32_t j = 0; j <= pos; ++j) z += exp(logit[j] - mx);
+    for (int32_t j = 0; j <= pos; ++j) partial[j] += exp(logit[j] - mx) / z;
+  }
+  free(logit);
+}
+
 /* --------------------------------------------- CSS saliency (Eqs. 4-5) */
 
 /* Phi for one visual token at (u, v) of frame f, KV head h (Eqs. 4-5):

@@ -796,3 +796,99 @@ def test_rho_task_split_matches_single_pass(threads, chunk):
         np.testing.assert_array_equal(
             np.nan_to_num(oracle.tsg_rho(k, wl.frames, threads=threads, chunk=chunk, metric=metric), nan=7.0),
             np.nan_to_num(oracle.tsg_rho_per_head(k, wl.frames, metric=metric), nan=7.0))
+
+
+# ------------------------------- prompt-wide base scores (base-scoring ablation)
+
+@pytest.mark.parametrize("n,n_q", [(9, 9), (12, 5), (7, 1)])
+def test_prompt_equal_keys_harmonic(n, n_q):
+    # Mean Attention / full-attention bases (appendix on the base scoring
+    # function), causal reading R18: with every key equal, prompt row r (at
+    # position p = n - n_q + r) spreads 1/(p+1) over keys 0..p, so the full
+    # base is C_j = sum_{p >= max(j, n - n_q)} 1/(p + 1) (harmonic numbers)
+    # and the mean base divides by the rows that see j.  A flipped mask or a
+    # missing 1/G would change both.
+    rng = np.random.default_rng(5)
+    d, hq, hkv = 8, 4, 2
+    q = rng.standard_normal((n_q, hq, d))
+    k = np.ones((n, hkv, d))
+    full = oracle.prompt_abase(q, k, oracle.PROMPT_FULL)
+    mean = oracle.prompt_abase(q, k, oracle.PROMPT_MEAN)
+    for j in range(n):
+        c = sum(1.0 / (p + 1) for p in range(max(j, n - n_q), n))
+        cnt = min(n_q, n - j)
+        np.testing.assert_allclose(full[:, j], c, rtol=1e-13)
+        np.testing.assert_allclose(mean[:, j], c / cnt, rtol=1e-13)
+
+
+def test_prompt_single_row_is_textbook_softmax():
+    # n_q = 1: the last position sees every key, so the full base is one
+    # softmax row: q = e_0, k_j = sqrt(d) x_j e_0 gives softmax(x).
+    d, n = 16, 6
+    x = np.array([0.5, -2.0, 1.5, 0.25, -0.75, 3.0])
+    q = np.zeros((1, 1, d)); q[0, 0, 0] = 1.0
+    k = np.zeros((n, 1, d)); k[:, 0, 0] = math.sqrt(d) * x
+    z = sum(math.exp(t) for t in x)
+    want = [math.exp(t) / z for t in x]
+    np.testing.assert_allclose(oracle.prompt_abase(q, k, oracle.PROMPT_FULL)[0], want, rtol=1e-13)
+    np.testing.assert_allclose(oracle.prompt_abase(q, k, oracle.PROMPT_MEAN)[0], want, rtol=1e-13)
+
+
+def test_prompt_dominant_key_sees_only_later_rows():
+    # a key with an overwhelming logit takes all the mass of every row at or
+    # after its position and none of the rows before it (causality): its full
+    # base is the number of rows that see it and its mean base is 1.
+    d, n = 8, 10
+    q = np.zeros((n, 1, d)); q[:, 0, 0] = 1.0
+    k = np.zeros((n, 1, d)); k[:, 0, 1] = 1.0
+    js = 4
+    k[js, 0, 0] = 400.0 * math.sqrt(d)
+    full = oracle.prompt_abase(q, k, oracle.PROMPT_FULL)[0]
+    mean = oracle.prompt_abase(q, k, oracle.PROMPT_MEAN)[0]
+    np.testing.assert_allclose(full[js], n - js, rtol=1e-12)
+    np.testing.assert_allclose(mean[js], 1.0, rtol=1e-12)
+    # rows before js see keys 0..p uniformly (all logits 0 there)
+    for j in range(js):
+        np.testing.assert_allclose(full[j], sum(1.0 / (p + 1) for p in range(j, js)), rtol=1e-12)
+    np.testing.assert_allclose(full[js + 1:], 0.0, atol=1e-100)
+
+
+def test_prompt_mass_and_library_softmax():
+    # every prompt row's probabilities sum to one (sum_j C_j = n_q), and the
+    # full base equals torch's softmax over causally masked logits, summed
+    # over rows and averaged over the group's query heads
+    import torch
+    rng = np.random.default_rng(11)
+    n, n_q, hq, hkv, d = 40, 23, 6, 2, 16
+    q = rng.standard_normal((n_q, hq, d))
+    k = rng.standard_normal((n, hkv, d))
+    full = oracle.prompt_abase(q, k, oracle.PROMPT_FULL, threads=3)
+    mean = oracle.prompt_abase(q, k, oracle.PROMPT_MEAN)
+    np.testing.assert_allclose(full.sum(1), n_q, rtol=1e-12)
+    cnt = np.minimum(n_q, n - np.arange(n))
+    np.testing.assert_allclose((mean * cnt).sum(1), n_q, rtol=1e-12)
+    G = hq // hkv
+    qt, kt = torch.from_numpy(q), torch.from_numpy(k)
+    pos = torch.arange(n - n_q, n)[:, None]
+    mask = torch.arange(n)[None, :] > pos                      # [n_q, n]
+    for h in range(hkv):
+        acc = torch.zeros(n, dtype=torch.float64)
+        for g in range(h * G, (h + 1) * G):
+            logits = qt[:, g] @ kt[:, h].T / math.sqrt(d)
+            acc += torch.softmax(logits.masked_fill(mask, float("-inf")), dim=1).sum(0)
+        np.testing.assert_allclose(full[h], (acc / G).numpy(), rtol=1e-12, atol=1e-15)
+
+
+def test_prompt_gqa_grouping():
+    # only the owning KV head's keys move its scores
+    rng = np.random.default_rng(2)
+    n, hq, hkv, d = 15, 6, 3, 8
+    q = rng.standard_normal((n, hq, d))
+    k = rng.standard_normal((n, hkv, d))
+    a = oracle.prompt_abase(q, k, oracle.PROMPT_MEAN)
+    k2 = k.copy()
+    k2[:, 1] = rng.standard_normal((n, d))
+    b = oracle.prompt_abase(q, k2, oracle.PROMPT_MEAN)
+    np.testing.assert_array_equal(a[0], b[0])
+    np.testing.assert_array_equal(a[2], b[2])
+    assert not np.allclose(a[1], b[1])
