@@ -328,6 +328,33 @@ STLITE_API stlite_status stlite_workspace_size_varlen(const stlite_shape* shape,
                                                       const int32_t* cu_seqlens, const stlite_frames* frames,
                                                       const stlite_params* params, size_t* bytes);
 
+/* Prompt-wide base scores of the base-scoring ablation (appendix
+ * "Sensitivity to the Base Attention Scoring Function"): instead of the w
+ * window queries of Eq. (2), every query row of the prompt votes.  The
+ * n_prompt rows q_prompt [n_prompt][Hq][d] are the queries of the last
+ * n_prompt cached positions (n_prompt = N: the whole prompt); the row at
+ * position p attends, as in the model's causal prefill, to the keys
+ * j <= p.  With C[h][j] = (1/G) sum over the group's query heads and the
+ * prompt rows of their softmax probability of key j:
+ *   STLITE_PROMPT_FULL  a_base = C (the full-attention "snapshot" base);
+ *   STLITE_PROMPT_MEAN  a_base = C / (number of prompt rows that attend to
+ *                       j, min(n_prompt, N - j)) (Mean Attention: attention
+ *                       averaged over the prompt).
+ * a_base (device float [Hkv][N]) then takes the place of the window score
+ * in stlite_select_topk.  bf16 only (STLITE_EUNSUPPORTED for fp32), G <=
+ * 128; shape->window is not used (any valid value).  The work is that of
+ * the prompt's causal attention, twice (row statistics, then column sums).
+ * ws: at least stlite_prompt_workspace_size bytes, zero-filled before its
+ * first use (its first word is the device error word of
+ * stlite_device_status). */
+typedef enum { STLITE_PROMPT_FULL = 0, STLITE_PROMPT_MEAN = 1 } stlite_prompt_base;
+STLITE_API stlite_status stlite_prompt_score(const stlite_shape* shape, int32_t n_prompt, int32_t base,
+                                             const void* q_prompt, const void* k, float* a_base, void* ws,
+                                             size_t ws_bytes, void* stream);
+
+/* Workspace bytes of stlite_prompt_score. */
+STLITE_API stlite_status stlite_prompt_workspace_size(const stlite_shape* shape, int32_t n_prompt, size_t* bytes);
+
 /* Consumer of the compressed cache: attention of query rows over a KV cache,
  * the operation a decoder runs for every generated token (the paper's
  * efficiency study compares decode latency with the full and the compressed

@@ -720,6 +720,42 @@ stlite_status stlite_compress_varlen_layers(const stlite_shape* shape, int32_t n
   return STLITE_OK;
 }
 
+// Prompt-wide base scores (Mean Attention / full-attention bases).
+static stlite_status check_prompt(const stlite_shape* shape, int32_t n_prompt, int32_t base) {
+  stlite_status s = check_shape(shape);
+  if (s != STLITE_OK) return s;
+  if (n_prompt < 1 || n_prompt > shape->n_tokens) return STLITE_EINVAL;
+  if (base != STLITE_PROMPT_FULL && base != STLITE_PROMPT_MEAN) return STLITE_EINVAL;
+  if (shape->dtype != STLITE_BF16) return STLITE_EUNSUPPORTED;
+  if (shape->n_q_heads / shape->n_kv_heads > 128) return STLITE_EUNSUPPORTED;
+  return STLITE_OK;
+}
+
+static size_t prompt_ws_bytes(const stlite_shape* shape, int32_t n_prompt) {
+  return 256 + prompt_bias_bytes(shape->n_tokens, n_prompt, shape->n_q_heads, shape->n_kv_heads);
+}
+
+stlite_status stlite_prompt_workspace_size(const stlite_shape* shape, int32_t n_prompt, size_t* bytes) {
+  if (!bytes) return STLITE_EINVAL;
+  stlite_status s = check_prompt(shape, n_prompt, STLITE_PROMPT_FULL);
+  if (s != STLITE_OK) return s;
+  *bytes = prompt_ws_bytes(shape, n_prompt);
+  return STLITE_OK;
+}
+
+stlite_status stlite_prompt_score(const stlite_shape* shape, int32_t n_prompt, int32_t base, const void* q_prompt,
+                                  const void* k, float* a_base, void* ws, size_t ws_bytes, void* stream) {
+  stlite_status s = check_prompt(shape, n_prompt, base);
+  if (s != STLITE_OK) return s;
+  if (!q_prompt || !k || !a_base || !ws) return STLITE_EINVAL;
+  if (!aligned16(q_prompt) || !aligned16(k) || !aligned16(a_base) || !aligned16(ws)) return STLITE_EINVAL;
+  if (ws_bytes < prompt_ws_bytes(shape, n_prompt)) return STLITE_EWORKSPACE;
+  uint8_t* w = static_cast<uint8_t*>(ws);
+  return cuda_status(launch_prompt_score(q_prompt, k, shape->n_tokens, n_prompt, shape->n_q_heads,
+                                         shape->n_kv_heads, base, a_base, reinterpret_cast<float*>(w + 256),
+                                         reinterpret_cast<uint32_t*>(w), static_cast<cudaStream_t>(stream)));
+}
+
 // Decode attention over a (compressed) cache.
 static stlite_status check_decode(const stlite_shape* shape) {
   stlite_status s = check_shape(shape);

@@ -30,7 +30,7 @@ EXPORTED = ("stlite_budget", "stlite_workspace_size", "stlite_score", "stlite_ga
             "stlite_status_string", "stlite_score_noalloc", "stlite_compress_layers", "stlite_compress_varlen",
             "stlite_workspace_size_varlen", "stlite_decode_attention", "stlite_decode_workspace_size",
             "stlite_compress_layers_budgets", "stlite_hierarchical_budgets", "stlite_spatial_saliency_size",
-            "stlite_compress_varlen_layers")
+            "stlite_compress_varlen_layers", "stlite_prompt_score", "stlite_prompt_workspace_size")
 
 
 class Shape(ctypes.Structure):
@@ -54,6 +54,7 @@ class Params(ctypes.Structure):
 STLITE_TSG_COSINE, STLITE_TSG_DOT, STLITE_TSG_NEG_L2 = 0, 1, 2
 STLITE_BASE_WINDOW, STLITE_BASE_UNIFORM = 0, 1
 STLITE_ABASE_RAW, STLITE_ABASE_MAX = 0, 1
+STLITE_PROMPT_FULL, STLITE_PROMPT_MEAN = 0, 1
 
 
 class LayerIO(ctypes.Structure):
@@ -108,6 +109,9 @@ _sig = {
                                            ctypes.c_size_t, _P]),
     "stlite_hierarchical_budgets": (_S, [ctypes.c_int32, ctypes.POINTER(ctypes.c_double), ctypes.c_int64,
                                          ctypes.c_int32, ctypes.POINTER(ctypes.c_int32)]),
+    "stlite_prompt_score": (_S, [ctypes.POINTER(Shape), ctypes.c_int32, ctypes.c_int32, _P, _P, _P, _P,
+                                 ctypes.c_size_t, _P]),
+    "stlite_prompt_workspace_size": (_S, [ctypes.POINTER(Shape), ctypes.c_int32, ctypes.POINTER(ctypes.c_size_t)]),
 }
 for _name, (_res, _args) in _sig.items():
     _f = getattr(_lib, _name)
@@ -360,6 +364,40 @@ def decode_attention(q, k, v, stream=None):
     out = torch.empty(q.shape, dtype=torch.float32, device=k.device)
     stlite_decode_attention(q, k, v, out, ws, stream)
     return out
+
+
+def prompt_shape(q_prompt, k) -> Shape:
+    """Shape of a prompt-wide score call: the window field is unused (1)."""
+    n_q, hq, d = q_prompt.shape
+    n, hkv, d2 = k.shape
+    if d != d2:
+        raise ValueError("q and k head_dim differ")
+    dt = {torch.bfloat16: STLITE_BF16, torch.float32: STLITE_F32}[k.dtype]
+    return Shape(n, hq, hkv, d, 1, dt)
+
+
+def stlite_prompt_workspace_size(shape: Shape, n_prompt: int) -> int:
+    out = ctypes.c_size_t()
+    _check(_lib.stlite_prompt_workspace_size(ctypes.byref(shape), int(n_prompt), ctypes.byref(out)),
+           "stlite_prompt_workspace_size")
+    return int(out.value)
+
+
+def stlite_prompt_score(q_prompt, k, base, a_base, ws, stream=None):
+    """Prompt-wide base scores (STLITE_PROMPT_FULL / STLITE_PROMPT_MEAN) of
+    the n_prompt = q_prompt.shape[0] rows of the last positions."""
+    sh = prompt_shape(q_prompt, k)
+    _check(_lib.stlite_prompt_score(ctypes.byref(sh), int(q_prompt.shape[0]), int(base), _ptr(q_prompt), _ptr(k),
+                                    _ptr(a_base), _ptr(ws), ws.numel(), _stream(stream)), "stlite_prompt_score")
+
+
+def prompt_score(q_prompt, k, base=STLITE_PROMPT_MEAN, stream=None):
+    """Allocates the output and a workspace and runs stlite_prompt_score."""
+    sh = prompt_shape(q_prompt, k)
+    ws = torch.zeros(stlite_prompt_workspace_size(sh, q_prompt.shape[0]), dtype=torch.uint8, device=k.device)
+    a = torch.empty((sh.n_kv_heads, sh.n_tokens), dtype=torch.float32, device=k.device)
+    stlite_prompt_score(q_prompt, k, base, a, ws, stream)
+    return a, ws
 
 
 def stlite_device_status(ws, stream=None) -> int:
