@@ -648,6 +648,61 @@ def run_gpu(args):
             if name == "hierarchical_budgets":
                 entry["budgets_min_max"] = [min(h_budgets), max(h_budgets)]
             variants[name] = entry
+        # the prompt-wide bases (Mean Attention, full attention): every one of
+        # the N prompt positions' query rows votes (causal), the work of the
+        # prompt's attention twice, so one layer (layer 0) is timed: prompt
+        # score, CSS, gate, Eq. 9 and Top-B on that base, compaction
+        gq = torch.Generator().manual_seed(2604)
+        q_prompt = torch.randn((N_TOK, HQ, D), generator=gq).to(torch.bfloat16).to(dev)
+        shp = stlite.prompt_shape(q_prompt, ks[0])
+        ws_p = torch.zeros(stlite.stlite_prompt_workspace_size(shp, N_TOK), dtype=torch.uint8, device=dev)
+        a_p = torch.empty((HKV, N_TOK), dtype=torch.float32, device=dev)
+        phi_p, rho_p = torch.empty_like(a_p), torch.empty_like(a_p)
+        tau_p = torch.empty((HKV,), dtype=torch.float32, device=dev)
+        gate_p = torch.empty((HKV, N_TOK), dtype=torch.uint8, device=dev)
+        for name, base in (("mean_attention_base", stlite.STLITE_PROMPT_MEAN),
+                           ("full_attention_base", stlite.STLITE_PROMPT_FULL)):
+            def pstep(st=None, base=base):
+                stlite.stlite_prompt_score(q_prompt, ks[0], base, a_p, ws_p, st)
+                stlite.stlite_spatial_saliency(qs[0], ks[0], fs, phi_p, ws, st)
+                stlite.stlite_gate_frames(qs[0], ks[0], fs, budget, rho_p, tau_p, gate_p, ws, st)
+                stlite.stlite_select_topk(qs[0], ks[0], fs, prm, a_p, phi_p, gate_p, budget, idxs[0], None, ws, st)
+                stlite.stlite_compact(qs[0], ks[0], vs[0], budget, idxs[0], kos[0], vos[0], st)
+            with torch.cuda.stream(stream):
+                pstep(stream)
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                pstep(stream)
+            a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            reps = 5
+            with torch.cuda.stream(stream):
+                g.replay()
+                a0.record(stream)
+                for _ in range(reps):
+                    g.replay()
+                a1.record(stream)
+            torch.cuda.synchronize()
+            assert stlite.stlite_device_status(ws_p, stream) == stlite.STLITE_OK
+            stlite.stlite_timing_read()
+            stlite.stlite_timing_enable(True)
+            with torch.cuda.stream(stream):
+                pstep(stream)
+            stream.synchronize()
+            stlite.stlite_timing_enable(False)
+            vk = stlite.stlite_timing_read()
+            pass_flop = 2.0 * (N_TOK * (N_TOK + 1) / 2) * D * HQ   # one causal QK^T over the prompt
+            entry = dict(ms_per_layer=a0.elapsed_time(a1) / reps, layers_timed=1, prompt_rows=N_TOK,
+                         kernels_ms={k: t / c for k, (c, t) in vk.items()})
+            for kname in ("prompt_rowstats", "prompt_colsum"):
+                if kname in vk:
+                    c, t = vk[kname]
+                    ach = pass_flop / (t / c * 1e-3) / 1e12
+                    entry[kname + "_roofline"] = dict(bound="tensor", achieved=ach, peak=peaks["bf16"],
+                                                      unit="TFLOP/s", frac=ach / peaks["bf16"],
+                                                      work="2*(N(N+1)/2)*d*Hq = %.4g FLOP (causal half)" %
+                                                           pass_flop)
+            variants[name] = entry
+        del q_prompt, ws_p
         # the variants overwrote the shared workspace's per-layer results; the
         # published method's outputs are recomputed for what follows
         with torch.cuda.stream(stream):
@@ -820,9 +875,55 @@ def run_gpu(args):
         for l in (0, L - 1):
             assert torch.equal(last["h_out"][l][2], idxs[l].cpu())
             assert torch.equal(last["h_out"][l][1], vos[l].cpu())
+        # the host link alone, measured on the same buffers: the step's input
+        # bytes host -> device (q, k and as many bytes of v as the kept rows)
+        # and its output bytes device -> host, each direction alone and both
+        # at once (the floor of a step that moves them)
+        S = sets[0]
+        hv = [host[l][2].view(-1)[:kept_v // 2] for l in range(L)]
+        dv = torch.empty(kept_v // 2, dtype=torch.bfloat16, device=dev)
+
+        def h2d():
+            with torch.cuda.stream(cp_in):
+                for l in range(L):
+                    S["q"][l].copy_(host[l][0], non_blocking=True)
+                    S["k"][l].copy_(host[l][1], non_blocking=True)
+                    dv.copy_(hv[l], non_blocking=True)
+
+        def d2h():
+            with torch.cuda.stream(cp_out):
+                for l in range(L):
+                    S["h_out"][l][0].copy_(S["ko"][l], non_blocking=True)
+                    S["h_out"][l][1].copy_(S["vo"][l], non_blocking=True)
+                    S["h_out"][l][2].copy_(S["ix"][l], non_blocking=True)
+
+        def link_ms(fns, reps=3):
+            best = None
+            for _ in range(reps):
+                torch.cuda.synchronize()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(cp_in)
+                cp_out.wait_stream(cp_in)
+                for fn in fns:
+                    fn()
+                cp_in.wait_stream(cp_out)
+                e1.record(cp_in)
+                torch.cuda.synchronize()
+                t = e0.elapsed_time(e1)
+                best = t if best is None else min(best, t)
+            return best
+
+        t_in, t_out, t_both = link_ms([h2d]), link_ms([d2h]), link_ms([h2d, d2h])
+        link = dict(h2d_gbs=bi / (t_in * 1e-3) / 1e9, d2h_gbs=bo / (t_out * 1e-3) / 1e9,
+                    h2d_ms=t_in, d2h_ms=t_out, both_directions_ms=t_both,
+                    floor_ms=t_both, e2e_over_floor=ms_e2e / t_both,
+                    note="cudaMemcpyAsync of the step's bytes from and to page-locked host memory, best of 3; "
+                         "floor = both directions at once")
         e2e = dict(value=job_throughput(world, L, ms_e2e), unit=UNIT, h2d_bytes_per_step=bi,
-                   d2h_bytes_per_step=bo, ms_per_step=ms_e2e,
-                   note="q and k copied; v read in place from page-locked host memory (kept rows only)")
+                   d2h_bytes_per_step=bo, ms_per_step=ms_e2e, host_link=link,
+                   note="q and k copied host -> device by torch (cudaMemcpyAsync on a copy stream) before the "
+                        "library call; v read by the compaction kernel in place from page-locked host memory "
+                        "(kept rows only); k_out, v_out, idx copied back by torch")
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
