@@ -759,13 +759,21 @@ def run_gpu(args):
     if not args.no_decode:
         probes = [qs[l][-1:].contiguous() for l in range(L)]    # the last window row as the next query
         dsh = stlite.make_shape(probes[0], ks[0])
-        dws = torch.zeros(stlite.stlite_decode_workspace_size(dsh), dtype=torch.uint8, device=dev)
+        dws = torch.zeros(max(stlite.stlite_decode_workspace_size(dsh),
+                              stlite.stlite_decode_layers_workspace_size(dsh, L)), dtype=torch.uint8, device=dev)
         douts = [torch.empty((1, HQ, D), dtype=torch.float32, device=dev) for _ in range(L)]
 
-        def decode_ms(kk, vv):
+        def decode_ms(kk, vv, batched=True):
+            # batched: one stlite_decode_attention_layers call for all layers;
+            # else one stlite_decode_attention call per layer
+            io = [(probes[l], kk[l], vv[l], douts[l]) for l in range(L)]
+
             def one():
-                for l in range(L):
-                    stlite.stlite_decode_attention(probes[l], kk[l], vv[l], douts[l], dws, stream)
+                if batched:
+                    stlite.stlite_decode_attention_layers(io, dws, stream)
+                else:
+                    for l in range(L):
+                        stlite.stlite_decode_attention(probes[l], kk[l], vv[l], douts[l], dws, stream)
             with torch.cuda.stream(stream):
                 for _ in range(3):
                     one()
@@ -786,6 +794,8 @@ def run_gpu(args):
 
         t_full = decode_ms(ks, vs)
         t_comp = decode_ms(kos, vos)
+        t_full_1 = decode_ms(ks, vs, batched=False)
+        t_comp_1 = decode_ms(kos, vos, batched=False)
         assert stlite.stlite_device_status(dws, stream) == stlite.STLITE_OK
         # critical hit rate of the same probe rows: mean over layers and KV heads
         chr_ = torch.stack([gpu_critical_hit_rate(stlite, probes[l], ks[l], idxs[l], stream) for l in range(L)])
@@ -797,9 +807,12 @@ def run_gpu(args):
                       compressed_gbs=budget * row * L / (t_comp * 1e-3) / 1e9,
                       peak_gbs=peaks["hbm"],
                       critical_hit_rate=float(chr_.mean()), critical_hit_rate_min=float(chr_.min()),
+                      per_layer_calls=dict(full_us_per_step=t_full_1 * 1e3, compressed_us_per_step=t_comp_1 * 1e3),
                       note="one query row per layer (the last window row) attends over every cached row (keys and "
-                           "values read once); full = N rows, compressed = the B kept rows; critical hit rate = "
-                           "share of that probe's B most-attended tokens kept (synthetic inputs)")
+                           "values read once), all layers in one stlite_decode_attention_layers call "
+                           "(per_layer_calls: one stlite_decode_attention call per layer); full = N rows, "
+                           "compressed = the B kept rows; critical hit rate = share of that probe's B "
+                           "most-attended tokens kept (synthetic inputs)")
 
     # ---- end to end: host (pinned) inputs -> device -> compress -> host outputs.
     # Q and K of every layer are copied to the device (every stage reads all

@@ -374,6 +374,31 @@ STLITE_API stlite_status stlite_decode_attention(const stlite_shape* shape, cons
 /* Workspace bytes of stlite_decode_attention for this shape. */
 STLITE_API stlite_status stlite_decode_workspace_size(const stlite_shape* shape, size_t* bytes);
 
+/* One layer's tensors for stlite_decode_attention_layers (device pointers,
+ * layouts as for stlite_decode_attention). */
+typedef struct {
+  const void* q; /* [w][Hq][d] */
+  const void* k; /* [n][Hkv][d] */
+  const void* v; /* [n][Hkv][d] */
+  float* out;    /* [w][Hq][d] fp32 */
+} stlite_decode_io;
+
+/* stlite_decode_attention for n_layers layers of one shape at once (the
+ * decode step of a whole model over its per-layer caches): one launch of the
+ * split kernel and one of the split merge per batch of up to 32 layers, the
+ * splits sized so that the batch fills whole waves of the GPU.  Each layer's
+ * result equals stlite_decode_attention's up to fp32 rounding (the splits
+ * group the sums differently).  layers: HOST array [n_layers]; ws: at least
+ * stlite_decode_layers_workspace_size bytes, zero-filled before its first
+ * use (first word: the device error word). */
+STLITE_API stlite_status stlite_decode_attention_layers(const stlite_shape* shape, int32_t n_layers,
+                                                        const stlite_decode_io* layers, void* ws, size_t ws_bytes,
+                                                        void* stream);
+
+/* Workspace bytes of stlite_decode_attention_layers. */
+STLITE_API stlite_status stlite_decode_layers_workspace_size(const stlite_shape* shape, int32_t n_layers,
+                                                             size_t* bytes);
+
 /* Reads and clears the workspace's device error word (synchronises `stream`).
  * *status receives STLITE_OK, STLITE_ETIMEOUT if a kernel's bounded wait ran
  * out since the last read, or STLITE_ECUDA if a kernel found its launch

@@ -768,7 +768,7 @@ stlite_status stlite_decode_workspace_size(const stlite_shape* shape, size_t* by
   if (!bytes) return STLITE_EINVAL;
   stlite_status s = check_decode(shape);
   if (s != STLITE_OK) return s;
-  *bytes = decode_workspace_bytes(shape->n_tokens, shape->n_q_heads, shape->n_kv_heads, shape->window);
+  *bytes = decode_workspace_bytes(shape->n_tokens, shape->n_q_heads, shape->n_kv_heads, shape->window, 1);
   return STLITE_OK;
 }
 
@@ -778,11 +778,70 @@ stlite_status stlite_decode_attention(const stlite_shape* shape, const void* q, 
   if (s != STLITE_OK) return s;
   if (!q || !k || !v || !out || !ws) return STLITE_EINVAL;
   if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(out) || !aligned16(ws)) return STLITE_EINVAL;
-  if (ws_bytes < decode_workspace_bytes(shape->n_tokens, shape->n_q_heads, shape->n_kv_heads, shape->window))
+  if (ws_bytes < decode_workspace_bytes(shape->n_tokens, shape->n_q_heads, shape->n_kv_heads, shape->window, 1))
     return STLITE_EWORKSPACE;
-  return cuda_status(launch_decode(shape->dtype == STLITE_BF16 ? kBF16 : kF32, q, k, v, shape->n_tokens,
-                                   shape->n_q_heads, shape->n_kv_heads, shape->window, out, ws,
+  DecBatch b;
+  memset(&b, 0, sizeof(b));
+  b.q[0] = q;
+  b.k[0] = k;
+  b.v[0] = v;
+  b.out[0] = out;
+  return cuda_status(launch_decode(shape->dtype == STLITE_BF16 ? kBF16 : kF32, b, 1, shape->n_tokens,
+                                   shape->n_q_heads, shape->n_kv_heads, shape->window, ws,
                                    static_cast<cudaStream_t>(stream)));
+}
+
+// The launches of a call run batches of kMaxLayers layers and then the rest;
+// the batch size sets the splits, so the workspace is the larger need.
+static size_t decode_layers_bytes(const stlite_shape* shape, int32_t n_layers) {
+  size_t need = 0;
+  const int full = n_layers >= kMaxLayers ? kMaxLayers : 0, rest = n_layers % kMaxLayers;
+  for (int L : {full, rest})
+    if (L > 0) {
+      const size_t b =
+          decode_workspace_bytes(shape->n_tokens, shape->n_q_heads, shape->n_kv_heads, shape->window, L);
+      if (b > need) need = b;
+    }
+  return need;
+}
+
+stlite_status stlite_decode_layers_workspace_size(const stlite_shape* shape, int32_t n_layers, size_t* bytes) {
+  if (!bytes || n_layers < 1) return STLITE_EINVAL;
+  stlite_status s = check_decode(shape);
+  if (s != STLITE_OK) return s;
+  *bytes = decode_layers_bytes(shape, n_layers);
+  return STLITE_OK;
+}
+
+stlite_status stlite_decode_attention_layers(const stlite_shape* shape, int32_t n_layers,
+                                             const stlite_decode_io* layers, void* ws, size_t ws_bytes,
+                                             void* stream) {
+  stlite_status s = check_decode(shape);
+  if (s != STLITE_OK) return s;
+  if (n_layers < 1 || !layers || !ws || !aligned16(ws)) return STLITE_EINVAL;
+  for (int l = 0; l < n_layers; ++l) {
+    const stlite_decode_io& x = layers[l];
+    if (!x.q || !x.k || !x.v || !x.out) return STLITE_EINVAL;
+    if (!aligned16(x.q) || !aligned16(x.k) || !aligned16(x.v) || !aligned16(x.out)) return STLITE_EINVAL;
+  }
+  if (ws_bytes < decode_layers_bytes(shape, n_layers)) return STLITE_EWORKSPACE;
+  // up to kMaxLayers layers per launch; the batches share the workspace
+  for (int l0 = 0; l0 < n_layers; l0 += kMaxLayers) {
+    const int L = n_layers - l0 < kMaxLayers ? n_layers - l0 : kMaxLayers;
+    DecBatch b;
+    memset(&b, 0, sizeof(b));
+    for (int l = 0; l < L; ++l) {
+      b.q[l] = layers[l0 + l].q;
+      b.k[l] = layers[l0 + l].k;
+      b.v[l] = layers[l0 + l].v;
+      b.out[l] = layers[l0 + l].out;
+    }
+    if ((s = cuda_status(launch_decode(shape->dtype == STLITE_BF16 ? kBF16 : kF32, b, L, shape->n_tokens,
+                                       shape->n_q_heads, shape->n_kv_heads, shape->window, ws,
+                                       static_cast<cudaStream_t>(stream)))) != STLITE_OK)
+      return s;
+  }
+  return STLITE_OK;
 }
 
 stlite_status stlite_device_status(void* ws, void* stream, stlite_status* status) {

@@ -52,11 +52,16 @@ __device__ __forceinline__ float weight(float a, float m) { return a == -CUDART_
 // Dynamic shared memory: qs[G][128] (query rows times log2(e)/sqrt(d)), then
 // per warp o[G][128] and (m, l)[G].
 template <typename T, int GM>
-__global__ void __launch_bounds__(kDecThreads, 2) k_decode_split(const T* __restrict__ q, const T* __restrict__ k,
-                                                              const T* __restrict__ v, int n, int hq, int hkv,
-                                                              int per, float* part_o, float2* part_ml) {
+__global__ void __launch_bounds__(kDecThreads, 2) k_decode_split(const __grid_constant__ DecBatch b, int w, int n,
+                                                              int hq, int hkv, int per, float* part_o_all,
+                                                              float2* part_ml_all) {
   extern __shared__ float4 dec_smem[];
-  const int split = blockIdx.x, h = blockIdx.y, r = blockIdx.z, nsplit = gridDim.x;
+  const int split = blockIdx.x, h = blockIdx.y, r = blockIdx.z % w, layer = blockIdx.z / w, nsplit = gridDim.x;
+  const T* __restrict__ q = static_cast<const T*>(b.q[layer]);
+  const T* __restrict__ k = static_cast<const T*>(b.k[layer]);
+  const T* __restrict__ v = static_cast<const T*>(b.v[layer]);
+  float* part_o = part_o_all + (size_t)layer * nsplit * w * hq * kD;
+  float2* part_ml = part_ml_all + (size_t)layer * nsplit * w * hq;
   const int G = hq / hkv;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   float* qs = reinterpret_cast<float*>(dec_smem);
@@ -162,11 +167,10 @@ __global__ void __launch_bounds__(kDecThreads, 2) k_decode_split(const T* __rest
       L = fmaf(wml[w * G + g].y, a, L);
       O = fmaf(wo[((size_t)w * G + g) * kD + c], a, O);
     }
-    const size_t slot = ((size_t)split * gridDim.z + r) * hq + h * G + g;
+    const size_t slot = ((size_t)split * w + r) * hq + h * G + g;
     part_o[slot * kD + c] = O;
     if (c == 0) part_ml[slot] = make_float2(M, L);
   }
-  (void)nsplit;
 }
 
 // ---------------------------------------------------------------------------
@@ -189,6 +193,12 @@ __global__ void __launch_bounds__(kDecThreads, 2) k_decode_split(const T* __rest
 // wait is made by the thread that issued the copy and its outcome shared
 // through shared memory after the group's barrier, so the group's warps take
 // the same path and always meet there.
+// Per-layer tensor maps of a batched decode launch.
+struct DecMaps {
+  CUtensorMap k[kMaxLayers];
+  CUtensorMap v[kMaxLayers];
+};
+
 constexpr int kDecTile = 64;                         // cached rows per tile
 constexpr int kDecStages = 4;
 constexpr int kDecHalf = kDecTile * 128;             // one 64-dimension half of a tile: 64 rows x 128 B
@@ -238,12 +248,16 @@ __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a
 // NT: 8-head column tiles of the query group (1 for G <= 8, 2 for G <= 16).
 template <int NT>
 __global__ void __launch_bounds__(kDecMmaThreads, 1)
-    k_decode_mma(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
-                 const __nv_bfloat16* __restrict__ q, int n, int hq, int hkv, int per, float* part_o,
-                 float2* part_ml, uint32_t* err) {
+    k_decode_mma(const __grid_constant__ DecMaps maps, const __grid_constant__ DecBatch b, int w, int n, int hq,
+                 int hkv, int per, float* part_o_all, float2* part_ml_all, uint32_t* err) {
   extern __shared__ uint8_t dec_raw[];
   uint8_t* sm = dec_raw + ((1024u - (smem_u32(dec_raw) & 1023u)) & 1023u);
-  const int split = blockIdx.x, h = blockIdx.y, r = blockIdx.z;
+  const int split = blockIdx.x, h = blockIdx.y, r = blockIdx.z % w, layer = blockIdx.z / w;
+  const CUtensorMap& kmap = maps.k[layer];
+  const CUtensorMap& vmap = maps.v[layer];
+  const __nv_bfloat16* __restrict__ q = static_cast<const __nv_bfloat16*>(b.q[layer]);
+  float* part_o = part_o_all + (size_t)layer * gridDim.x * w * hq * kD;
+  float2* part_ml = part_ml_all + (size_t)layer * gridDim.x * w * hq;
   const int G = hq / hkv;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int gi = warp >> 2, wq = warp & 3, id = tid & (kDecGroupThreads - 1);
@@ -421,7 +435,7 @@ __global__ void __launch_bounds__(kDecMmaThreads, 1)
       L = fmaf(ml.y, wgt, L);
       O = fmaf(wo[((size_t)w * 8 * NT + g) * kD + cc], wgt, O);
     }
-    const size_t slot = ((size_t)split * gridDim.z + r) * hq + h * G + g;
+    const size_t slot = ((size_t)split * w + r) * hq + h * G + g;
     part_o[slot * kD + cc] = O;
     if (cc == 0) part_ml[slot] = make_float2(M, L);
   }
@@ -432,12 +446,15 @@ __global__ void __launch_bounds__(kDecMmaThreads, 1)
 // once in shared memory, then every thread sums its dimension over the splits
 // with eight partial loads in flight.
 constexpr int kDecMaxSplits = 1024;
-__global__ void __launch_bounds__(kD) k_decode_combine(const float* part_o, const float2* part_ml, int nsplit,
-                                                       int hq, int w, float* out) {
+__global__ void __launch_bounds__(kD) k_decode_combine(const __grid_constant__ DecBatch b, const float* part_o_all,
+                                                       const float2* part_ml_all, int nsplit, int hq, int w) {
   __shared__ float wts[kDecMaxSplits];
   __shared__ float red[kD / 32];
   __shared__ float bc[2];
-  const int g = blockIdx.x, r = blockIdx.y, c = threadIdx.x, lane = c & 31, wp = c >> 5;
+  const int g = blockIdx.x, r = blockIdx.y % w, layer = blockIdx.y / w, c = threadIdx.x, lane = c & 31, wp = c >> 5;
+  const float* part_o = part_o_all + (size_t)layer * nsplit * w * hq * kD;
+  const float2* part_ml = part_ml_all + (size_t)layer * nsplit * w * hq;
+  float* out = b.out[layer];
   float mx = -CUDART_INF_F;
   for (int s = c; s < nsplit; s += kD) mx = fmaxf(mx, part_ml[((size_t)s * w + r) * hq + g].x);
   mx = warp_max(mx);
@@ -480,44 +497,66 @@ __global__ void __launch_bounds__(kD) k_decode_combine(const float* part_o, cons
   out[((size_t)r * hq + g) * kD + c] = O / bc[1];
 }
 
-int decode_splits(int n, int hkv, int w) {
+int decode_splits(int n, int hkv, int w, int layers) {
   int dev = 0, sms = 152;
   if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  // one wave of one CTA per SM, each with at least 256 cached rows
-  long long s = ((long long)sms + (long long)hkv * w - 1) / ((long long)hkv * w);
-  const long long cap = (n + 255) / 256;
-  if (s > cap) s = cap;
-  if (s > kDecMaxSplits) s = kDecMaxSplits;
-  if (s < 1) s = 1;
-  return (int)s;
+  const long long cap0 = (n + 255) / 256;  // at least 256 cached rows per split
+  const long long cap = cap0 < kDecMaxSplits ? cap0 : kDecMaxSplits;
+  if (layers <= 1) {
+    // one layer: one wave of one CTA per SM
+    long long s = ((long long)sms + (long long)hkv * w - 1) / ((long long)hkv * w);
+    if (s > cap) s = cap;
+    if (s < 1) s = 1;
+    return (int)s;
+  }
+  // a batch of layers: the split count whose CTAs fill whole waves best
+  // (among fills within 2 % the fewest CTAs)
+  const long long units = (long long)layers * hkv * w;
+  long long smax = 4 * ((sms + units - 1) / units);
+  if (smax < 4) smax = 4;
+  if (smax > cap) smax = cap;
+  long long best = 1;
+  double best_eff = 0.0;
+  for (long long s = 1; s <= smax; ++s) {
+    const long long ctas = units * s, waves = (ctas + sms - 1) / sms;
+    const double eff = (double)ctas / (double)(waves * sms);
+    if (eff > best_eff + 0.02) {
+      best = s;
+      best_eff = eff;
+    }
+  }
+  return (int)best;
 }
 
-// Workspace: the error word (first 256 bytes), then the split partials.
-size_t decode_workspace_bytes(int n, int hq, int hkv, int w) {
-  const size_t slots = (size_t)decode_splits(n, hkv, w) * w * hq;
+// Workspace: the error word (first 256 bytes), then every layer's split
+// partials.
+size_t decode_workspace_bytes(int n, int hq, int hkv, int w, int layers) {
+  const size_t slots = (size_t)layers * decode_splits(n, hkv, w, layers) * w * hq;
   return 256 + slots * kD * sizeof(float) + slots * sizeof(float2);
 }
 
-cudaError_t launch_decode(DType dt, const void* q, const void* k, const void* v, int n, int hq, int hkv, int w,
-                          float* out, void* ws, cudaStream_t st) {
-  const int nsplit = decode_splits(n, hkv, w);
+cudaError_t launch_decode(DType dt, const DecBatch& b, int layers, int n, int hq, int hkv, int w, void* ws,
+                          cudaStream_t st) {
+  const int nsplit = decode_splits(n, hkv, w, layers);
   uint32_t* err = static_cast<uint32_t*>(ws);
   float* part_o = reinterpret_cast<float*>(static_cast<uint8_t*>(ws) + 256);
-  float2* part_ml = reinterpret_cast<float2*>(part_o + (size_t)nsplit * w * hq * kD);
+  float2* part_ml = reinterpret_cast<float2*>(part_o + (size_t)layers * nsplit * w * hq * kD);
   const int G = hq / hkv;
-  dim3 grid(nsplit, hkv, w);
+  dim3 grid(nsplit, hkv, w * layers);
   cudaError_t e = cudaSuccess;
   if (dt == kBF16) {
     const int per = ((n + nsplit - 1) / nsplit + kDecTile - 1) / kDecTile * kDecTile;
-    CUtensorMap km, vm;
-    if ((e = make_row_map(&km, k, n, hkv, kDecTile)) != cudaSuccess) return e;
-    if ((e = make_row_map(&vm, v, n, hkv, kDecTile)) != cudaSuccess) return e;
+    DecMaps maps;
+    for (int l = 0; l < layers; ++l) {
+      if ((e = make_row_map(&maps.k[l], b.k[l], n, hkv, kDecTile)) != cudaSuccess) return e;
+      if ((e = make_row_map(&maps.v[l], b.v[l], n, hkv, kDecTile)) != cudaSuccess) return e;
+    }
     auto run = [&](auto nt) {
       constexpr int NT = decltype(nt)::value;
       e = cudaFuncSetAttribute(k_decode_mma<NT>, cudaFuncAttributeMaxDynamicSharedMemorySize, dec_mma_smem(NT));
       if (e != cudaSuccess) return;
-      k_decode_mma<NT><<<grid, kDecMmaThreads, dec_mma_smem(NT), st>>>(
-          km, vm, static_cast<const __nv_bfloat16*>(q), n, hq, hkv, per, part_o, part_ml, err);
+      k_decode_mma<NT><<<grid, kDecMmaThreads, dec_mma_smem(NT), st>>>(maps, b, w, n, hq, hkv, per, part_o,
+                                                                       part_ml, err);
     };
     TimingScope ts("decode_split", st);
     if (G <= 8)
@@ -531,10 +570,7 @@ cudaError_t launch_decode(DType dt, const void* q, const void* k, const void* v,
       constexpr int GM = decltype(gm)::value;
       e = cudaFuncSetAttribute(k_decode_split<float, GM>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
       if (e != cudaSuccess) return;
-      k_decode_split<float, GM><<<grid, kDecThreads, smem, st>>>(static_cast<const float*>(q),
-                                                                 static_cast<const float*>(k),
-                                                                 static_cast<const float*>(v), n, hq, hkv, per,
-                                                                 part_o, part_ml);
+      k_decode_split<float, GM><<<grid, kDecThreads, smem, st>>>(b, w, n, hq, hkv, per, part_o, part_ml);
     };
     TimingScope ts("decode_split", st);
     if (G <= 4)
@@ -547,7 +583,7 @@ cudaError_t launch_decode(DType dt, const void* q, const void* k, const void* v,
   if (e != cudaSuccess) return e;
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   TimingScope ts("decode_combine", st);
-  k_decode_combine<<<dim3(hq, w), kD, 0, st>>>(part_o, part_ml, nsplit, hq, w, out);
+  k_decode_combine<<<dim3(hq, w * layers), kD, 0, st>>>(b, part_o, part_ml, nsplit, hq, w);
   return cudaGetLastError();
 }
 

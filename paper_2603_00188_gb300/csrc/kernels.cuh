@@ -218,10 +218,19 @@ cudaError_t noalloc_error_word(uint32_t** word);
 
 // ---- consumer: decode attention over a (compressed) cache -----------------
 constexpr int kDecMaxG = 16;  // query heads per KV head
-int decode_splits(int n, int hkv, int w);
-size_t decode_workspace_bytes(int n, int hq, int hkv, int w);
-// out [w][hq][128] fp32; q [w][hq][128], k/v [n][hkv][128] of dtype dt.
-cudaError_t launch_decode(DType dt, const void* q, const void* k, const void* v, int n, int hq, int hkv, int w,
-                          float* out, void* ws, cudaStream_t st);
+// Per-layer tensors of one decode launch (up to kMaxLayers layers).
+struct DecBatch {
+  const void* q[kMaxLayers];  // [w][hq][128]
+  const void* k[kMaxLayers];  // [n][hkv][128]
+  const void* v[kMaxLayers];
+  float* out[kMaxLayers];     // [w][hq][128] fp32
+};
+// Cache splits per (layer, KV head, query row): one layer fills one wave;
+// a batch of layers takes the count that fills whole waves best.
+int decode_splits(int n, int hkv, int w, int layers);
+size_t decode_workspace_bytes(int n, int hq, int hkv, int w, int layers);
+// Every layer of the batch: out = attention of q over (k, v), dtype dt.
+cudaError_t launch_decode(DType dt, const DecBatch& b, int layers, int n, int hq, int hkv, int w, void* ws,
+                          cudaStream_t st);
 
 }  // namespace stl

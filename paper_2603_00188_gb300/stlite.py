@@ -30,7 +30,8 @@ EXPORTED = ("stlite_budget", "stlite_workspace_size", "stlite_score", "stlite_ga
             "stlite_status_string", "stlite_score_noalloc", "stlite_compress_layers", "stlite_compress_varlen",
             "stlite_workspace_size_varlen", "stlite_decode_attention", "stlite_decode_workspace_size",
             "stlite_compress_layers_budgets", "stlite_hierarchical_budgets", "stlite_spatial_saliency_size",
-            "stlite_compress_varlen_layers", "stlite_prompt_score", "stlite_prompt_workspace_size")
+            "stlite_compress_varlen_layers", "stlite_prompt_score", "stlite_prompt_workspace_size",
+            "stlite_decode_attention_layers", "stlite_decode_layers_workspace_size")
 
 
 class Shape(ctypes.Structure):
@@ -60,6 +61,10 @@ STLITE_PROMPT_FULL, STLITE_PROMPT_MEAN = 0, 1
 class LayerIO(ctypes.Structure):
     _fields_ = [("q", ctypes.c_void_p), ("k", ctypes.c_void_p), ("v", ctypes.c_void_p),
                 ("k_out", ctypes.c_void_p), ("v_out", ctypes.c_void_p), ("idx_out", ctypes.c_void_p)]
+
+
+class DecodeIO(ctypes.Structure):
+    _fields_ = [("q", ctypes.c_void_p), ("k", ctypes.c_void_p), ("v", ctypes.c_void_p), ("out", ctypes.c_void_p)]
 
 
 class KernelTime(ctypes.Structure):
@@ -112,6 +117,10 @@ _sig = {
     "stlite_prompt_score": (_S, [ctypes.POINTER(Shape), ctypes.c_int32, ctypes.c_int32, _P, _P, _P, _P,
                                  ctypes.c_size_t, _P]),
     "stlite_prompt_workspace_size": (_S, [ctypes.POINTER(Shape), ctypes.c_int32, ctypes.POINTER(ctypes.c_size_t)]),
+    "stlite_decode_attention_layers": (_S, [ctypes.POINTER(Shape), ctypes.c_int32, ctypes.POINTER(DecodeIO), _P,
+                                            ctypes.c_size_t, _P]),
+    "stlite_decode_layers_workspace_size": (_S, [ctypes.POINTER(Shape), ctypes.c_int32,
+                                                 ctypes.POINTER(ctypes.c_size_t)]),
 }
 for _name, (_res, _args) in _sig.items():
     _f = getattr(_lib, _name)
@@ -398,6 +407,32 @@ def prompt_score(q_prompt, k, base=STLITE_PROMPT_MEAN, stream=None):
     a = torch.empty((sh.n_kv_heads, sh.n_tokens), dtype=torch.float32, device=k.device)
     stlite_prompt_score(q_prompt, k, base, a, ws, stream)
     return a, ws
+
+
+def stlite_decode_layers_workspace_size(shape: Shape, n_layers: int) -> int:
+    out = ctypes.c_size_t()
+    _check(_lib.stlite_decode_layers_workspace_size(ctypes.byref(shape), int(n_layers), ctypes.byref(out)),
+           "stlite_decode_layers_workspace_size")
+    return int(out.value)
+
+
+def stlite_decode_attention_layers(layers, ws, stream=None):
+    """layers: list of (q, k, v, out) device tensors, one tuple per layer
+    (same shapes)."""
+    sh = make_shape(layers[0][0], layers[0][1])
+    arr = (DecodeIO * len(layers))(*[DecodeIO(*(t.data_ptr() for t in lay)) for lay in layers])
+    _check(_lib.stlite_decode_attention_layers(ctypes.byref(sh), len(layers), arr, _ptr(ws), ws.numel(),
+                                               _stream(stream)), "stlite_decode_attention_layers")
+
+
+def decode_attention_layers(qs, ks, vs, stream=None):
+    """Allocates the outputs and the workspace and runs
+    stlite_decode_attention_layers over the layers' (q, k, v)."""
+    sh = make_shape(qs[0], ks[0])
+    ws = torch.zeros(stlite_decode_layers_workspace_size(sh, len(qs)), dtype=torch.uint8, device=ks[0].device)
+    outs = [torch.empty(q.shape, dtype=torch.float32, device=ks[0].device) for q in qs]
+    stlite_decode_attention_layers(list(zip(qs, ks, vs, outs)), ws, stream)
+    return outs, ws
 
 
 def stlite_device_status(ws, stream=None) -> int:

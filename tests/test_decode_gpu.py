@@ -107,3 +107,53 @@ def test_decode_rejects(st):
     k = torch.zeros((10, 1, 128), dtype=torch.bfloat16, device="cuda")
     with pytest.raises(st.StliteError):
         st.decode_attention(q, k, k)                  # 32 query heads per KV head > 16
+
+
+@pytest.mark.parametrize("layers,w,hq,hkv,n,dtype", [(28, 1, 28, 4, 3000, torch.bfloat16),
+                                                      (5, 2, 12, 2, 1001, torch.bfloat16),
+                                                      (34, 1, 8, 2, 300, torch.bfloat16),
+                                                      (3, 1, 16, 1, 77, torch.bfloat16),
+                                                      (4, 2, 12, 2, 513, torch.float32)])
+def test_decode_layers_match_oracle(st, layers, w, hq, hkv, n, dtype):
+    """The layer-batched decode (one launch pair per batch of up to 32
+    layers; 34 layers take two) against the oracle layer by layer, and
+    against the single-layer call within fp32 rounding."""
+    g = torch.Generator().manual_seed(layers * 131 + n)
+    qs = [torch.randn((w, hq, 128), generator=g).to(dtype).cuda() for _ in range(layers)]
+    ks = [torch.randn((n, hkv, 128), generator=g).to(dtype).cuda() for _ in range(layers)]
+    vs = [torch.randn((n, hkv, 128), generator=g).to(dtype).cuda() for _ in range(layers)]
+    outs, ws = st.decode_attention_layers(qs, ks, vs)
+    torch.cuda.synchronize()
+    assert st.stlite_device_status(ws) == st.STLITE_OK
+    for l in sorted({0, layers // 2, layers - 1}):
+        ref = oracle.decode_attention(exact64(qs[l]), exact64(ks[l]), exact64(vs[l]))
+        _close(outs[l].cpu().numpy().astype(np.float64), ref, exact64(vs[l]))
+    for l in range(layers):
+        one = st.decode_attention(qs[l], ks[l], vs[l])
+        torch.cuda.synchronize()
+        _close(outs[l].cpu().numpy().astype(np.float64), one.cpu().numpy().astype(np.float64), exact64(vs[l]))
+
+
+def test_decode_layers_in_graph(st):
+    """The batched call replays in a CUDA graph with the same bits."""
+    g = torch.Generator().manual_seed(5)
+    qs = [torch.randn((1, 28, 128), generator=g).to(torch.bfloat16).cuda() for _ in range(6)]
+    ks = [torch.randn((2000, 4, 128), generator=g).to(torch.bfloat16).cuda() for _ in range(6)]
+    vs = [torch.randn((2000, 4, 128), generator=g).to(torch.bfloat16).cuda() for _ in range(6)]
+    outs, ws = st.decode_attention_layers(qs, ks, vs)
+    torch.cuda.synchronize()
+    ref = [o.clone() for o in outs]
+    stream = torch.cuda.Stream()
+    graph = torch.cuda.CUDAGraph()
+    io = list(zip(qs, ks, vs, outs))
+    with torch.cuda.stream(stream):
+        st.stlite_decode_attention_layers(io, ws, stream)
+    stream.synchronize()
+    with torch.cuda.graph(graph, stream=stream):
+        st.stlite_decode_attention_layers(io, ws, stream)
+    for o in outs:
+        o.zero_()
+    graph.replay()
+    torch.cuda.synchronize()
+    for o, r in zip(outs, ref):
+        assert torch.equal(o, r)
