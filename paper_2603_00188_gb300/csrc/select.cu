@@ -221,6 +221,46 @@ __device__ __forceinline__ void for_tokens(const FrameTable& ft, int j0, int j1,
   }
 }
 
+// The same visit in groups of four consecutive tokens t0 .. t0 + 3 (t0 =
+// j0 + 4 (tid + k B)), for 128-bit loads and stores: j0, j1 and every row
+// base are multiples of four tokens.  kinds[e] is the kind of t0 + e.
+template <class Load4, class Use4>
+__device__ __forceinline__ void for_tokens4(const FrameTable& ft, int j0, int j1, Load4 load4, Use4 use4) {
+  const int B = blockDim.x, F = ft.n_frames;
+  const int first = j0 + 4 * (int)threadIdx.x;
+  int f = -1, lo = 0, hi = F - 1;
+  while (lo <= hi) {  // last frame starting at or before the thread's first token
+    const int mid = (lo + hi) >> 1;
+    if (ft.off[mid] <= first) {
+      f = mid;
+      lo = mid + 1;
+    } else {
+      hi = mid - 1;
+    }
+  }
+  for (int t0 = first; t0 < j1; t0 += 4 * B) {
+    int kinds[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int t = t0 + e;
+      while (f + 1 < F && ft.off[f + 1] <= t) ++f;
+      const bool vis = f >= 0 && t < ft.off[f] + ft.gh[f] * ft.gw[f];
+      kinds[e] = vis ? (f + 1 < F ? kTokPool : kTokCur) : kTokText;
+    }
+    const auto v = load4(t0, kinds);
+    use4(t0, kinds, v);
+  }
+}
+
+struct RhoIn4 {
+  float4 s[4];
+  float4 rn;
+};
+struct ScoreIn4 {
+  float4 A, P;
+  uint32_t G;  // four gate bytes
+};
+
 __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __grid_constant__ FrameTable ft,
                                                         SelectArgs a) {
   extern __shared__ uint32_t keys[];
@@ -228,8 +268,9 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
   cg::cluster_group cl = cg::this_cluster();
   const int ncta = (int)cl.num_blocks(), c = (int)cl.block_rank();
   const int l = blockIdx.y / p.hkv, h = blockIdx.y % p.hkv, n = p.n, tid = threadIdx.x;
-  const int chunk = (n + ncta - 1) / ncta;
+  const int chunk = ((n + ncta - 1) / ncta + 3) & ~3;  // four-token groups never straddle two CTAs
   const int j0 = min(n, c * chunk), j1 = min(n, j0 + chunk), len = j1 - j0;
+  const bool vec = (n & 3) == 0;  // every row base [Hkv][N] is 16-byte aligned
   const size_t hn = (size_t)h * n;
   const int F = ft.n_frames;
   int pass = 0;
@@ -251,7 +292,50 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
     prefetch_l2(rn, 4, j0, j1);
     // rho of every token: pool tokens from the TSG slices and 1/|k_i|, NaN
     // elsewhere; the selection keys are complements (m-th smallest rho ==
-    // m-th largest key), 0 marks a token outside the pool
+    // m-th largest key), 0 marks a token outside the pool.  Finish Eq. 6
+    // with the row's own term: times 1/|k_i| (cosine), nothing (dot), minus
+    // |k_i|^2 (negative squared L2).
+    auto finish = [&](float m, float rnv) {
+      return a.tsg_metric == kTsgCosine ? m * rnv : (a.tsg_metric == kTsgDot ? m : m - 1.f / (rnv * rnv));
+    };
+    if (vec) {
+      for_tokens4(
+          ft, j0, j1,
+          [&](int t0, const int (&kinds)[4]) {
+            RhoIn4 r;
+            const float ninf = -CUDART_INF_F;
+#pragma unroll
+            for (int s = 0; s < 4; ++s) r.s[s] = make_float4(ninf, ninf, ninf, ninf);
+            r.rn = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (kinds[0] == kTokPool || kinds[1] == kTokPool || kinds[2] == kTokPool || kinds[3] == kTokPool) {
+              const float* src = rp + t0;
+#pragma unroll
+              for (int s = 0; s < 4; ++s)
+                if (s < nsl) r.s[s] = __ldg(reinterpret_cast<const float4*>(src + (size_t)s * slice));
+              for (int s = 4; s < nsl; ++s) {
+                const float4 x = __ldg(reinterpret_cast<const float4*>(src + (size_t)s * slice));
+                r.s[3] = make_float4(fmaxf(r.s[3].x, x.x), fmaxf(r.s[3].y, x.y), fmaxf(r.s[3].z, x.z),
+                                     fmaxf(r.s[3].w, x.w));
+              }
+              r.rn = __ldg(reinterpret_cast<const float4*>(rn + t0));
+            }
+            return r;
+          },
+          [&](int t0, const int (&kinds)[4], const RhoIn4& v) {
+            const float m0 = fmaxf(fmaxf(v.s[0].x, v.s[1].x), fmaxf(v.s[2].x, v.s[3].x));
+            const float m1 = fmaxf(fmaxf(v.s[0].y, v.s[1].y), fmaxf(v.s[2].y, v.s[3].y));
+            const float m2 = fmaxf(fmaxf(v.s[0].z, v.s[1].z), fmaxf(v.s[2].z, v.s[3].z));
+            const float m3 = fmaxf(fmaxf(v.s[0].w, v.s[1].w), fmaxf(v.s[2].w, v.s[3].w));
+            const float r0 = kinds[0] == kTokPool ? finish(m0, v.rn.x) : CUDART_NAN_F;
+            const float r1 = kinds[1] == kTokPool ? finish(m1, v.rn.y) : CUDART_NAN_F;
+            const float r2 = kinds[2] == kTokPool ? finish(m2, v.rn.z) : CUDART_NAN_F;
+            const float r3 = kinds[3] == kTokPool ? finish(m3, v.rn.w) : CUDART_NAN_F;
+            *reinterpret_cast<float4*>(rho + t0) = make_float4(r0, r1, r2, r3);
+            *reinterpret_cast<uint4*>(keys + (t0 - j0)) =
+                make_uint4(kinds[0] == kTokPool ? ~float_key(r0) : 0u, kinds[1] == kTokPool ? ~float_key(r1) : 0u,
+                           kinds[2] == kTokPool ? ~float_key(r2) : 0u, kinds[3] == kTokPool ? ~float_key(r3) : 0u);
+          });
+    } else
     for_tokens<2>(
         ft, j0, j1,
         [&](int t, int kind) {
@@ -272,12 +356,8 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
           return r;
         },
         [&](int t, int kind, const RhoIn& v) {
-          // finish Eq. 6 with the row's own term: times 1/|k_i| (cosine),
-          // nothing (dot), minus |k_i|^2 (negative squared L2)
           const float m = fmaxf(fmaxf(v.s[0], v.s[1]), fmaxf(v.s[2], v.s[3]));
-          const float own = a.tsg_metric == kTsgCosine ? m * v.rn
-                            : (a.tsg_metric == kTsgDot ? m : m - 1.f / (v.rn * v.rn));
-          const float r = kind == kTokPool ? own : CUDART_NAN_F;
+          const float r = kind == kTokPool ? finish(m, v.rn) : CUDART_NAN_F;
           rho[t] = r;
           keys[t - j0] = kind == kTokPool ? ~float_key(r) : 0u;
         });
@@ -326,6 +406,51 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
     const bool a_div = amax > 0.f;
     // Eq. 9: S = A_base for text tokens; for visual tokens S = A_base +
     // alpha * Phi where the gate is open and 0 where it is closed
+    auto score_of = [&](int t, int kind, float A, float P, float G) {
+      float s;
+      if (kind == kTokText) {
+        s = A + 0.0f;
+        if (fused) gate[t] = 1;
+      } else {
+        bool g = G != 0.f;
+        if (fused) {
+          g = !(kind == kTokPool && gate_sel) || key_float(~keys[t - j0]) <= tau;
+          gate[t] = g ? 1 : 0;
+        }
+        const float x = alpha != 0.f ? __fmaf_rn(alpha, P, A) : A;
+        s = (g ? x : 0.f) + 0.0f;
+      }
+      return s;
+    };
+    if (vec) {
+      for_tokens4(
+          ft, j0, j1,
+          [&](int t0, const int (&kinds)[4]) {
+            ScoreIn4 v;
+            v.A = ab ? __ldg(reinterpret_cast<const float4*>(ab + t0))
+                     : make_float4(a.a_uniform, a.a_uniform, a.a_uniform, a.a_uniform);
+            if (a_div)
+              v.A = make_float4(__fdiv_rn(v.A.x, amax), __fdiv_rn(v.A.y, amax), __fdiv_rn(v.A.z, amax),
+                                __fdiv_rn(v.A.w, amax));
+            const bool vis = kinds[0] != kTokText || kinds[1] != kTokText || kinds[2] != kTokText ||
+                             kinds[3] != kTokText;
+            v.P = (vis && alpha != 0.f) ? __ldg(reinterpret_cast<const float4*>(ph + t0)) : make_float4(0.f, 0.f, 0.f, 0.f);
+            v.G = (vis && !fused && gt != nullptr) ? __ldg(reinterpret_cast<const uint32_t*>(gt + t0)) : 0x01010101u;
+            return v;
+          },
+          [&](int t0, const int (&kinds)[4], const ScoreIn4& v) {
+            const float s0 = score_of(t0, kinds[0], v.A.x, kinds[0] != kTokText ? v.P.x : 0.f, (float)(v.G & 0xffu));
+            const float s1 = score_of(t0 + 1, kinds[1], v.A.y, kinds[1] != kTokText ? v.P.y : 0.f,
+                                      (float)((v.G >> 8) & 0xffu));
+            const float s2 = score_of(t0 + 2, kinds[2], v.A.z, kinds[2] != kTokText ? v.P.z : 0.f,
+                                      (float)((v.G >> 16) & 0xffu));
+            const float s3 = score_of(t0 + 3, kinds[3], v.A.w, kinds[3] != kTokText ? v.P.w : 0.f,
+                                      (float)(v.G >> 24));
+            *reinterpret_cast<float4*>(sc + t0) = make_float4(s0, s1, s2, s3);
+            *reinterpret_cast<uint4*>(keys + (t0 - j0)) =
+                make_uint4(float_key(s0), float_key(s1), float_key(s2), float_key(s3));
+          });
+    } else
     for_tokens<2>(
         ft, j0, j1,
         [&](int t, int kind) {
@@ -336,19 +461,7 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
           return make_float3(A, P, G);
         },
         [&](int t, int kind, float3 v) {
-          float s;
-          if (kind == kTokText) {
-            s = v.x + 0.0f;
-            if (fused) gate[t] = 1;
-          } else {
-            bool g = v.z != 0.f;
-            if (fused) {
-              g = !(kind == kTokPool && gate_sel) || key_float(~keys[t - j0]) <= tau;
-              gate[t] = g ? 1 : 0;
-            }
-            const float x = alpha != 0.f ? __fmaf_rn(alpha, v.y, v.x) : v.x;
-            s = (g ? x : 0.f) + 0.0f;
-          }
+          const float s = score_of(t, kind, v.x, v.y, v.z);
           sc[t] = s;
           keys[t - j0] = float_key(s);
         });
@@ -410,7 +523,7 @@ static void select_config(cudaLaunchConfig_t* cfg, cudaLaunchAttribute* attr, co
   *cfg = cudaLaunchConfig_t{};
   cfg->gridDim = dim3(cl, p.L * p.hkv, 1);
   cfg->blockDim = dim3(kSelThreads, 1, 1);
-  cfg->dynamicSmemBytes = (size_t)((p.n + cl - 1) / cl) * 4;
+  cfg->dynamicSmemBytes = (size_t)(((p.n + cl - 1) / cl + 3) & ~3) * 4;
   cfg->stream = st;
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = cl;
@@ -439,7 +552,7 @@ cudaError_t launch_select(const Problem& p, const FrameTable& ft, const SelectAr
   long long best = 0;
   const long long units = (long long)p.L * p.hkv;
   for (int c = 1; c <= kSelMaxCluster; c <<= 1) {
-    const int ch = (p.n + c - 1) / c;
+    const int ch = ((p.n + c - 1) / c + 3) & ~3;
     if (ch > kSelMaxChunk) continue;
     select_config(&cfg, attr, p, c, st);
     int fit = 0;
