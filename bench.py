@@ -56,7 +56,10 @@ def parse():
     ap.add_argument("--no-decode", action="store_true", help="skip the decode-over-the-cache measurement")
     ap.add_argument("--no-variants", action="store_true", help="skip the ablation-variant step times")
     ap.add_argument("--no-trajectory", action="store_true", help="skip the per-step trajectory sweep")
-    ap.add_argument("--workload", default="traj50", choices=["traj50", "uitars", "small_backbone", "long_horizon"],
+    ap.add_argument("--prompt-rows", type=int, default=0,
+                    help="--workload mean_attention: prompt query rows (0 = the whole cache)")
+    ap.add_argument("--workload", default="traj50",
+                    choices=["traj50", "uitars", "small_backbone", "long_horizon", "mean_attention"],
                     help="traj50 (default): the 28-layer, 50-step trajectory of the contract line; the others time "
                          "the remaining configurations (one JSON line of their own)")
     return ap.parse_args()
@@ -1130,6 +1133,32 @@ def run_workload(args):
                              tsg_roofline=tsg_tflops([wl for pl in per_layer for wl in pl[0]], 1, kern2)))
             del per_layer, seq_io, seq_ws
             torch.cuda.empty_cache()
+    elif args.workload == "mean_attention":
+        # the prompt-wide bases of the base-scoring ablation on one layer of
+        # the 50-step trajectory: every prompt position's query rows vote
+        wl = synth.trajectory_50(0)
+        k = bf16(wl.k)
+        n_prompt = args.prompt_rows if args.prompt_rows > 0 else wl.n
+        gq = torch.Generator().manual_seed(2604)
+        qp = torch.randn((n_prompt, HQ, D), generator=gq).to(torch.bfloat16).to(dev)
+        shp = stlite.prompt_shape(qp, k)
+        ws = torch.zeros(stlite.stlite_prompt_workspace_size(shp, n_prompt), dtype=torch.uint8, device=dev)
+        a = torch.empty((HKV, wl.n), dtype=torch.float32, device=dev)
+        n0 = wl.n - n_prompt
+        pass_flop = 2.0 * (n_prompt * n0 + n_prompt * (n_prompt + 1) / 2) * D * HQ   # causal QK^T of the rows
+        for name, base in (("mean_attention", stlite.STLITE_PROMPT_MEAN), ("full_attention", stlite.STLITE_PROMPT_FULL)):
+            def step(st, base=base):
+                stlite.stlite_prompt_score(qp, k, base, a, ws, st)
+            ms, kern = timed(step, max(3, min(10, args.steps)))
+            roof = {}
+            for kname in ("prompt_rowstats", "prompt_colsum"):
+                if kname in kern:
+                    ach = pass_flop / (kern[kname]["ms_per_step"] * 1e-3) / 1e12
+                    roof[kname] = dict(bound="tensor", achieved=ach, peak=peaks["bf16"], unit="TFLOP/s",
+                                       frac=ach / peaks["bf16"], peak_source=peaks["source"] + " burst")
+            runs.append(dict(base=name, layers=1, n_tokens=wl.n, prompt_rows=n_prompt, ms_per_step=ms,
+                             value=wl.n / (ms * 1e-3), kernels=kern, roofline=roof,
+                             work="2*(causal pairs)*d*Hq = %.4g FLOP per pass" % pass_flop))
     else:  # long_horizon
         distinct = [synth.long_horizon(l) for l in range(4)]
         for L in (1, LAYERS):
