@@ -407,6 +407,16 @@ STLITE_API stlite_status stlite_decode_layers_workspace_size(const stlite_shape*
  * the current device instead. */
 STLITE_API stlite_status stlite_device_status(void* ws, void* stream, stlite_status* status);
 
+/* Diagnostic of the failure path (not part of Algorithm 1): one kernel waits,
+ * through the bounded wait every tensor-core kernel of the library uses, on
+ * a barrier that nothing completes.  After limit_ns (1 us .. 2 s) of
+ * %globaltimer the wait gives up, records STLITE_ETIMEOUT in the workspace
+ * error word and the kernel returns: stlite_device_status(ws) then reports
+ * STLITE_ETIMEOUT, and the context stays usable for later calls.  Nothing
+ * faults and nothing hangs.  ws: at least 16 bytes of device memory whose
+ * first word is the error word (any workspace of this library qualifies). */
+STLITE_API stlite_status stlite_selftest_wait_timeout(void* ws, int64_t limit_ns, void* stream);
+
 /* Per-kernel timing (instrumentation; not part of Algorithm 1).
  * stlite_timing_enable(1) makes every later launch by this library, on a
  * stream that is not being captured into a graph, record a pair of CUDA

@@ -47,15 +47,16 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
 
 // Waits for the phase of parity `parity` to complete.  Gives up (returns
 // false) when the CTA-wide abort flag is raised by another role, or after
-// kWaitLimitNs, in which case it raises the flag and records kErrTimeout.
+// limit_ns (kWaitLimitNs in every kernel), in which case it raises the flag
+// and records kErrTimeout.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint32_t* err,
-                                          volatile uint32_t* abort_flag) {
+                                          volatile uint32_t* abort_flag, uint64_t limit_ns = kWaitLimitNs) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_timer_ns();
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*abort_flag) return false;
-    if (global_timer_ns() - t0 > kWaitLimitNs) {
+    if (global_timer_ns() - t0 > limit_ns) {
       *abort_flag = 1u;
       record_error(err, kErrTimeout);
       return false;

@@ -31,7 +31,8 @@ EXPORTED = ("stlite_budget", "stlite_workspace_size", "stlite_score", "stlite_ga
             "stlite_workspace_size_varlen", "stlite_decode_attention", "stlite_decode_workspace_size",
             "stlite_compress_layers_budgets", "stlite_hierarchical_budgets", "stlite_spatial_saliency_size",
             "stlite_compress_varlen_layers", "stlite_prompt_score", "stlite_prompt_workspace_size",
-            "stlite_decode_attention_layers", "stlite_decode_layers_workspace_size")
+            "stlite_decode_attention_layers", "stlite_decode_layers_workspace_size",
+            "stlite_selftest_wait_timeout")
 
 
 class Shape(ctypes.Structure):
@@ -117,6 +118,7 @@ _sig = {
     "stlite_prompt_score": (_S, [ctypes.POINTER(Shape), ctypes.c_int32, ctypes.c_int32, _P, _P, _P, _P,
                                  ctypes.c_size_t, _P]),
     "stlite_prompt_workspace_size": (_S, [ctypes.POINTER(Shape), ctypes.c_int32, ctypes.POINTER(ctypes.c_size_t)]),
+    "stlite_selftest_wait_timeout": (_S, [_P, ctypes.c_int64, _P]),
     "stlite_decode_attention_layers": (_S, [ctypes.POINTER(Shape), ctypes.c_int32, ctypes.POINTER(DecodeIO), _P,
                                             ctypes.c_size_t, _P]),
     "stlite_decode_layers_workspace_size": (_S, [ctypes.POINTER(Shape), ctypes.c_int32,
@@ -433,6 +435,13 @@ def decode_attention_layers(qs, ks, vs, stream=None):
     outs = [torch.empty(q.shape, dtype=torch.float32, device=ks[0].device) for q in qs]
     stlite_decode_attention_layers(list(zip(qs, ks, vs, outs)), ws, stream)
     return outs, ws
+
+
+def stlite_selftest_wait_timeout(ws, limit_ns: int, stream=None):
+    """Runs the failure-path diagnostic: a bounded wait that runs out after
+    limit_ns and records STLITE_ETIMEOUT in ws's error word."""
+    _check(_lib.stlite_selftest_wait_timeout(_ptr(ws), int(limit_ns), _stream(stream)),
+           "stlite_selftest_wait_timeout")
 
 
 def stlite_device_status(ws, stream=None) -> int:
