@@ -341,9 +341,10 @@ STLITE_API stlite_status stlite_workspace_size_varlen(const stlite_shape* shape,
  *                       j, min(n_prompt, N - j)) (Mean Attention: attention
  *                       averaged over the prompt).
  * a_base (device float [Hkv][N]) then takes the place of the window score
- * in stlite_select_topk.  bf16 only (STLITE_EUNSUPPORTED for fp32), G <=
- * 128; shape->window is not used (any valid value).  The work is that of
- * the prompt's causal attention, twice (row statistics, then column sums).
+ * in stlite_select_topk.  bf16 caches run on the tensor cores, fp32 caches
+ * on the CUDA cores; G <= 128; shape->window is not used (any valid value).
+ * The work is that of the prompt's causal attention, twice (row statistics,
+ * then column sums).
  * ws: at least stlite_prompt_workspace_size bytes, zero-filled before its
  * first use (its first word is the device error word of
  * stlite_device_status). */

@@ -726,7 +726,6 @@ static stlite_status check_prompt(const stlite_shape* shape, int32_t n_prompt, i
   if (s != STLITE_OK) return s;
   if (n_prompt < 1 || n_prompt > shape->n_tokens) return STLITE_EINVAL;
   if (base != STLITE_PROMPT_FULL && base != STLITE_PROMPT_MEAN) return STLITE_EINVAL;
-  if (shape->dtype != STLITE_BF16) return STLITE_EUNSUPPORTED;
   if (shape->n_q_heads / shape->n_kv_heads > 128) return STLITE_EUNSUPPORTED;
   return STLITE_OK;
 }
@@ -751,7 +750,8 @@ stlite_status stlite_prompt_score(const stlite_shape* shape, int32_t n_prompt, i
   if (!aligned16(q_prompt) || !aligned16(k) || !aligned16(a_base) || !aligned16(ws)) return STLITE_EINVAL;
   if (ws_bytes < prompt_ws_bytes(shape, n_prompt)) return STLITE_EWORKSPACE;
   uint8_t* w = static_cast<uint8_t*>(ws);
-  return cuda_status(launch_prompt_score(q_prompt, k, shape->n_tokens, n_prompt, shape->n_q_heads,
+  return cuda_status(launch_prompt_score(shape->dtype == STLITE_BF16 ? kBF16 : kF32, q_prompt, k, shape->n_tokens,
+                                         n_prompt, shape->n_q_heads,
                                          shape->n_kv_heads, base, a_base, reinterpret_cast<float*>(w + 256),
                                          reinterpret_cast<uint32_t*>(w), static_cast<cudaStream_t>(stream)));
 }

@@ -205,10 +205,10 @@ cudaError_t make_row_map(CUtensorMap* m, const void* base, int n, int hkv, int r
 // ---- prompt-wide base scores (base-scoring ablation) -----------------------
 // a_out [hkv][n] fp32 = the full-attention base (mode 0) or the Mean
 // Attention base (mode 1) of the nq prompt rows q [nq][hq][128] (the last nq
-// positions, causal) over k [n][hkv][128], bf16.  bias: prompt_bias_bytes of
-// scratch (per-row softmax statistics).
+// positions, causal) over k [n][hkv][128], bf16 (tensor cores) or fp32 (CUDA
+// cores).  bias: prompt_bias_bytes of scratch (per-row softmax statistics).
 size_t prompt_bias_bytes(int n, int nq, int hq, int hkv);
-cudaError_t launch_prompt_score(const void* q, const void* k, int n, int nq, int hq, int hkv, int mode,
+cudaError_t launch_prompt_score(DType dt, const void* q, const void* k, int n, int nq, int hq, int hkv, int mode,
                                 float* a_out, float* bias, uint32_t* err, cudaStream_t st);
 
 // ---- fixed scratch of stlite_score_noalloc ---------------------------------

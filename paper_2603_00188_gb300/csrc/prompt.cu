@@ -456,6 +456,123 @@ __global__ void __maxnreg__(kPrMaxReg)
   }
 }
 
+// ---- fp32 caches: the same two passes on the CUDA cores --------------------
+// Pass 1: one CTA of 128 threads per (query row, KV head); each thread keeps
+// an online (max, sum of 2^(x c - max c)) over its strided keys j <= pos, and
+// the block merges the threads' states in a fixed order.
+constexpr int kPrSimtRows = 128;
+__global__ void __launch_bounds__(kPrSimtRows) k_prompt_rowstats_simt(const float* __restrict__ q,
+                                                                     const float* __restrict__ k, PromptArgs a,
+                                                                     float* bias) {
+  __shared__ float qs[kD];
+  __shared__ float2 st[kPrSimtRows];
+  const int row = blockIdx.x, h = blockIdx.y, tid = threadIdx.x;
+  const int prel = row / a.G, gq = row - prel * a.G;
+  const int pos = a.n - a.nq + prel;
+  const float c = kPrLog2e * rsqrtf((float)kD);
+  qs[tid] = q[((size_t)prel * a.hq + h * a.G + gq) * kD + tid];
+  __syncthreads();
+  float m = -CUDART_INF_F, l = 0.f;
+  for (int j = tid; j <= pos; j += kPrSimtRows) {
+    const float4* kr = reinterpret_cast<const float4*>(k + ((size_t)j * a.hkv + h) * kD);
+    float d = 0.f;
+#pragma unroll 8
+    for (int e = 0; e < kD / 4; ++e) {
+      const float4 kv = __ldg(kr + e);
+      d = fmaf(kv.x, qs[4 * e], d);
+      d = fmaf(kv.y, qs[4 * e + 1], d);
+      d = fmaf(kv.z, qs[4 * e + 2], d);
+      d = fmaf(kv.w, qs[4 * e + 3], d);
+    }
+    const float x = d * c;
+    if (x > m) {
+      l = (m == -CUDART_INF_F ? 0.f : l * exp2f(m - x)) + 1.f;
+      m = x;
+    } else {
+      l += exp2f(x - m);
+    }
+  }
+  st[tid] = make_float2(m, l);
+  __syncthreads();
+  if (tid == 0) {
+    float mm = -CUDART_INF_F, ll = 0.f;
+    for (int t = 0; t < kPrSimtRows; ++t) {
+      const float2 s = st[t];
+      const float mn = fmaxf(mm, s.x);
+      if (mn == -CUDART_INF_F) continue;
+      ll = (mm == -CUDART_INF_F ? 0.f : ll * exp2f(mm - mn)) + (s.x == -CUDART_INF_F ? 0.f : s.y * exp2f(s.x - mn));
+      mm = mn;
+    }
+    const size_t at = ((size_t)h * a.n_ch + prel / a.p2) * a.crp + (size_t)(prel % a.p2) * a.G + gq;
+    bias[at] = -mm - log2f((float)a.G * ll);
+  }
+}
+
+// Pass 2: one CTA of 256 threads per (32-key tile, KV head).  The tile's keys
+// and, in turn, tiles of query rows (with their biases) sit in shared
+// memory (32-row tiles); thread t sums 2^(x c + bias_r) for key t % 32 over rows t / 32 + 8 i
+// that attend to it, and the eight partial sums of a key are added in a
+// fixed order.
+constexpr int kPrSimtKeys = 32, kPrSimtRowTile = 32, kPrSimtThreads = 256;
+__global__ void __launch_bounds__(kPrSimtThreads) k_prompt_colsum_simt(const float* __restrict__ q,
+                                                                      const float* __restrict__ k, PromptArgs a,
+                                                                      const float* bias, float* a_out) {
+  __shared__ float ks[kPrSimtKeys][kD + 1];
+  __shared__ float qs[kPrSimtRowTile][kD + 1];
+  __shared__ float bs[kPrSimtRowTile];
+  __shared__ float part[kPrSimtThreads];
+  const int h = blockIdx.y, tid = threadIdx.x, j0 = blockIdx.x * kPrSimtKeys;
+  const int kk = tid % kPrSimtKeys, rsub = tid / kPrSimtKeys;
+  const int j = j0 + kk;
+  const int p_first = a.n - a.nq;
+  const float c = kPrLog2e * rsqrtf((float)kD);
+  for (int e = tid; e < kPrSimtKeys * kD; e += kPrSimtThreads) {
+    const int r = e / kD, d = e % kD;
+    ks[r][d] = j0 + r < a.n ? k[((size_t)(j0 + r) * a.hkv + h) * kD + d] : 0.f;
+  }
+  const int rows = a.nq * a.G;
+  const int r_start = j0 <= p_first ? 0 : (j0 - p_first) * a.G;  // rows before it see no key of the tile
+  float acc = 0.f;
+  for (int r0 = r_start; r0 < rows; r0 += kPrSimtRowTile) {
+    __syncthreads();
+    for (int e = tid; e < kPrSimtRowTile * kD; e += kPrSimtThreads) {
+      const int r = e / kD, d = e % kD, row = r0 + r;
+      float v = 0.f;
+      if (row < rows) {
+        const int prel = row / a.G, gq = row - prel * a.G;
+        v = q[((size_t)prel * a.hq + h * a.G + gq) * kD + d];
+      }
+      qs[r][d] = v;
+    }
+    for (int r = tid; r < kPrSimtRowTile; r += kPrSimtThreads) {
+      const int row = r0 + r;
+      float b = -CUDART_INF_F;
+      if (row < rows) {
+        const int prel = row / a.G, gq = row - prel * a.G;
+        b = bias[((size_t)h * a.n_ch + prel / a.p2) * a.crp + (size_t)(prel % a.p2) * a.G + gq];
+      }
+      bs[r] = b;
+    }
+    __syncthreads();
+    for (int r = rsub; r < kPrSimtRowTile; r += kPrSimtThreads / kPrSimtKeys) {
+      const int row = r0 + r;
+      if (row >= rows || p_first + row / a.G < j) continue;  // past the rows, or before key j
+      float d = 0.f;
+#pragma unroll 8
+      for (int e = 0; e < kD; ++e) d = fmaf(ks[kk][e], qs[r][e], d);
+      acc += exp2f(fmaf(d, c, bs[r]));
+    }
+  }
+  part[tid] = acc;
+  __syncthreads();
+  if (rsub == 0 && j < a.n) {
+    float s = 0.f;
+    for (int t = 0; t < kPrSimtThreads / kPrSimtKeys; ++t) s += part[t * kPrSimtKeys + kk];
+    if (a.mode == 1) s /= (float)min(a.nq, a.n - j);
+    a_out[(size_t)h * a.n + j] = s;
+  }
+}
+
 // ---- host --------------------------------------------------------------
 
 namespace {
@@ -511,10 +628,32 @@ size_t prompt_bias_bytes(int n, int nq, int hq, int hkv) {
   return (size_t)hkv * a.n_ch * a.crp * 4;
 }
 
-cudaError_t launch_prompt_score(const void* q, const void* k, int n, int nq, int hq, int hkv, int mode,
+cudaError_t launch_prompt_score(DType dt, const void* q, const void* k, int n, int nq, int hq, int hkv, int mode,
                                 float* a_out, float* bias, uint32_t* err, cudaStream_t st) {
   const PromptArgs a = prompt_args(n, nq, hq, hkv, mode);
   if (a.p1 < 1) return cudaErrorNotSupported;
+  if (dt == kF32) {
+    const size_t nbias = (size_t)hkv * a.n_ch * a.crp;
+    const size_t blocks = (nbias + 255) / 256;
+    cudaError_t e;
+    {
+      TimingScope ts("prompt_bias_fill", st);
+      k_prompt_bias_fill<<<(unsigned)(blocks < 1024 ? blocks : 1024), 256, 0, st>>>(bias, nbias);
+    }
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    const float* qf = static_cast<const float*>(q);
+    const float* kf = static_cast<const float*>(k);
+    {
+      TimingScope ts("prompt_rowstats_simt", st);
+      k_prompt_rowstats_simt<<<dim3((unsigned)(nq * a.G), hkv), kPrSimtRows, 0, st>>>(qf, kf, a, bias);
+    }
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    TimingScope ts("prompt_colsum_simt", st);
+    k_prompt_colsum_simt<<<dim3((unsigned)((n + kPrSimtKeys - 1) / kPrSimtKeys), hkv), kPrSimtThreads, 0, st>>>(
+        qf, kf, a, bias, a_out);
+    (void)err;
+    return cudaGetLastError();
+  }
   PromptMaps maps;
   cudaError_t e = make_prompt_qmap(&maps.q1, q, nq, hq, a.G, a.p1);
   if (e == cudaSuccess) e = make_prompt_qmap(&maps.q2, q, nq, hq, a.G, a.p2);

@@ -2,7 +2,8 @@
 full-attention bases) through the C ABI against the fp64 oracle: every
 element of A within the window score's tolerance, for prompts covering the
 whole cache and its last n_prompt positions (ragged m-tiles and chunks),
-group sizes 7, 6 and 1, Gaussian and heavy-tailed keys; the row-mass
+group sizes 7, 6 and 1, Gaussian and heavy-tailed keys, bf16 caches (tensor
+cores) and fp32 caches (CUDA cores); the row-mass
 invariant; bit-identical repeated calls; and the kept set of the method run
 on this base (Eq. 9 with A replaced, then Top-B) against the oracle's.
 """
@@ -26,6 +27,9 @@ CASES = {
                                            seed=(77,)), None),
     "last_7": (lambda: synth.scaled("small", 2, beta=0.4), 7),
     "last_1": (lambda: synth.scaled("traj50", 2), 1),
+    # fp32 caches (CUDA-core passes): the tiny reference, whole and partial prompts
+    "fp32_tiny_all": (lambda: synth.tiny_ref(), None),
+    "fp32_tiny_last333": (lambda: synth.tiny_ref(), 333),
 }
 
 
@@ -48,7 +52,8 @@ def prompt_rows(wl, q_all, n_prompt):
     qp = rng.standard_normal((npr, q_all.shape[1], q_all.shape[2])).astype(np.float32)
     w = min(npr, q_all.shape[0])
     qp[npr - w:] = q_all[q_all.shape[0] - w:]
-    return torch.from_numpy(qp).to(torch.bfloat16).cuda()
+    dt = torch.float32 if wl.dtype == "f32" else torch.bfloat16
+    return torch.from_numpy(qp).to(dt).cuda()
 
 
 def load(name):
@@ -88,7 +93,7 @@ def test_prompt_score(st, name, base):
     assert torch.equal(a, a2)
 
 
-@pytest.mark.parametrize("name", ["traj50_4f_all", "small_3f_all", "long_2f_last777"])
+@pytest.mark.parametrize("name", ["traj50_4f_all", "small_3f_all", "long_2f_last777", "fp32_tiny_all"])
 def test_method_on_prompt_base(st, name):
     """Eq. 9 and Top-B with the Mean Attention base in place of the window
     score (CSS and TSG unchanged): kept sets against the oracle's pipeline."""
@@ -124,13 +129,12 @@ def test_method_on_prompt_base(st, name):
 
 
 def test_prompt_rejects(st):
-    """fp32 caches and prompts longer than the cache are refused on the host."""
-    k = torch.zeros((64, 2, 128), dtype=torch.float32, device="cuda")
-    qp = torch.zeros((64, 4, 128), dtype=torch.float32, device="cuda")
+    """Groups of more than 128 query heads and prompts longer than the cache
+    are refused on the host."""
+    kb = torch.zeros((64, 1, 128), dtype=torch.bfloat16, device="cuda")
     with pytest.raises(st.StliteError) as e:
-        st.prompt_score(qp, k)
+        st.prompt_score(torch.zeros((64, 256, 128), dtype=torch.bfloat16, device="cuda"), kb)
     assert e.value.status == st.STLITE_EUNSUPPORTED
-    kb = k.to(torch.bfloat16)
     with pytest.raises(st.StliteError) as e:
         st.prompt_score(torch.zeros((65, 4, 128), dtype=torch.bfloat16, device="cuda"), kb)
     assert e.value.status == st.STLITE_EINVAL
