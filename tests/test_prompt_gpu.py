@@ -138,3 +138,28 @@ def test_prompt_rejects(st):
     with pytest.raises(st.StliteError) as e:
         st.prompt_score(torch.zeros((65, 4, 128), dtype=torch.bfloat16, device="cuda"), kb)
     assert e.value.status == st.STLITE_EINVAL
+
+
+def test_prompt_full_size_bench_layer(st):
+    """The bench's full-size case: layer 0 of the 50-step trajectory (N =
+    53,600) with the whole prompt voting.  The oracle cannot redo 10 TFLOP,
+    so: every row's mass is one (sum_j C_j = N per head); the Mean Attention
+    base times the rows that see a key equals the full base; and the last 64
+    keys, which only the last 64 prompt rows can see, equal the oracle's
+    scores of those 64 rows exactly as defined (same rows, same keys)."""
+    wl = synth.trajectory_50(0)
+    k = torch.from_numpy(wl.k).to(torch.bfloat16).cuda()
+    qp = prompt_rows(wl, wl.q, None)
+    n, H = wl.n, k.shape[1]
+    full, _ = st.prompt_score(qp, k, st.STLITE_PROMPT_FULL)
+    mean, ws = st.prompt_score(qp, k, st.STLITE_PROMPT_MEAN)
+    torch.cuda.synchronize()
+    assert st.stlite_device_status(ws) == st.STLITE_OK
+    f, m = full.cpu().numpy().astype(np.float64), mean.cpu().numpy().astype(np.float64)
+    np.testing.assert_allclose(f.sum(1), n, rtol=1e-4)
+    count = np.minimum(n, n - np.arange(n)).astype(np.float64)
+    np.testing.assert_allclose(m * count, f, rtol=2e-6, atol=0)
+    tail = 64
+    ora = oracle.prompt_abase(exact64(qp[n - tail:]), exact64(k), oracle.PROMPT_FULL, threads=oracle.host_threads())
+    for h in range(H):
+        assert_within(f[h, n - tail:], ora[h, n - tail:], a_bound(ora[h, n - tail:]), "full base, last keys, head %d" % h)
