@@ -329,6 +329,7 @@ stlite_status compress_batch(const Ctx& c, const stlite_params* params, const La
   a.a_base = c.view<const float>(c.plan.a_base);
   a.phi = params->css_enable ? c.view<const float>(c.plan.phi) : strided<const float>(nullptr, 0);
   a.score = c.view<float>(c.plan.score);
+  a.write_stages = 0;  // rho, gate and S stay on chip: only the indices leave
   for (int l = 0; l < c.p.L; ++l) a.idx[l] = io.idx[l];
   if ((e = launch_select(c.p, c.ft, a, c.st)) != cudaSuccess) return STLITE_ECUDA;
   return cuda_status(launch_gather(c.p, io, c.st));
@@ -394,6 +395,7 @@ stlite_status stlite_gate_frames(const stlite_shape* shape, const stlite_frames*
   a.rho = one(rho);
   a.tau = one(tau);
   a.gate = one(gate);
+  a.write_stages = 1;
   return cuda_status(launch_select(c.p, c.ft, a, c.st));
 }
 
@@ -450,6 +452,7 @@ stlite_status stlite_select_topk(const stlite_shape* shape, const stlite_frames*
   a.gate = one(const_cast<uint8_t*>(gate));
   a.score = score_out ? one(score_out) : c.view<float>(c.plan.score);
   a.idx[0] = idx;
+  a.write_stages = 1;
   return cuda_status(launch_select(c.p, c.ft, a, c.st));
 }
 

@@ -179,6 +179,7 @@ struct SelectArgs {
   int base_uniform;    // 1: A = a_uniform for every token instead of a_base
   float a_uniform;
   int a_norm_max;      // 1: A / max_j A per head before Eq. 9
+  int write_stages;    // 1: write rho, gate and score (the staged outputs); 0: only tau and the indices
   Strided<const float> rho_part;  // [nchunk][Hkv][N]
   Strided<const float> rn;        // [Hkv][N]
   Strided<float> rho;             // out [Hkv][N]

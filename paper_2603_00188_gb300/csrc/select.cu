@@ -20,7 +20,7 @@ namespace cg = cooperative_groups;
 
 namespace stl {
 
-constexpr int kSelThreads = 512;
+constexpr int kSelThreads = 512;  // two per histogram bin in the radix passes
 constexpr int kSelMaxCluster = 8;
 constexpr int kSelMaxChunk = 49152;  // keys per CTA held in shared memory (192 KB)
 
@@ -28,11 +28,14 @@ struct SelShared {
   uint32_t whist[kSelThreads / 32][256];  // per-warp histograms
   uint32_t hist[2][256];  // this CTA's histogram, double-buffered by pass parity
   uint32_t tot[256];      // cluster-wide histogram of the current pass
+  uint32_t dig[2][2];     // (digit, count above it), double-buffered by pass parity
   uint32_t bcast[4];
   uint32_t warp_tot[32];
   uint32_t counts[2];     // (greater, equal) of this CTA for the compaction
   float warp_max[32];
   float cta_max;          // read by the cluster's other CTAs
+  int32_t fr_off[kMaxFrames + 1];  // first token of every frame; fr_off[F] = INT_MAX
+  int32_t fr_vend[kMaxFrames];     // end of every frame's visual span
 };
 
 // Maximum of v over every thread of the cluster (every CTA must call it).
@@ -83,7 +86,14 @@ __device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* w
 
 // k-th largest (1-indexed) key over the whole cluster; key 0 marks an empty
 // slot.  Returns the key T; *need_out = how many keys equal to T belong to
-// the top k.
+// the top k.  Per pass: per-warp histograms, one block barrier, the CTA's
+// histogram (two threads per bin), one cluster barrier, the cluster's
+// histogram (two threads per bin, each reading half of the CTAs), one block
+// barrier, the digit found by warp 0, one block barrier.  The CTA histogram
+// and the digit broadcast are double-buffered by pass parity, so that no
+// barrier is needed before the next pass rewrites them: a buffer is
+// rewritten two passes later, after every thread has passed the barriers
+// that follow its last read.
 __device__ uint32_t cluster_select_desc(cg::cluster_group& cl, const uint32_t* keys, int len,
                                         uint32_t k, SelShared& sh, int& pass,
                                         uint32_t* need_out) {
@@ -91,6 +101,7 @@ __device__ uint32_t cluster_select_desc(cg::cluster_group& cl, const uint32_t* k
   const int tid = threadIdx.x, lane = tid & 31, nw = blockDim.x >> 5, wid = tid >> 5;
   const int ncta = (int)cl.num_blocks();
   uint32_t* wh = sh.whist[wid];
+  const int bin = tid >> 1, half = tid & 1;  // 512 threads: two per bin
   for (int shift = 24; shift >= 0; shift -= 8, ++pass) {
     uint32_t* hb = sh.hist[pass & 1];
     for (int b = lane; b < 256; b += 32) wh[b] = 0u;
@@ -111,24 +122,30 @@ __device__ uint32_t cluster_select_desc(cg::cluster_group& cl, const uint32_t* k
       if (key != 0u && (key & mask) == prefix) atomicAdd(&wh[(key >> shift) & 255u], 1u);
     }
     __syncthreads();
-    for (int b = tid; b < 256; b += blockDim.x) {
+    {
       uint32_t t = 0;
+      const int w0 = half * (nw >> 1), w1 = w0 + (nw >> 1);
 #pragma unroll 8
-      for (int w = 0; w < nw; ++w) t += sh.whist[w][b];
-      hb[b] = t;
+      for (int w = w0; w < w1; ++w) t += sh.whist[w][bin];
+      t += __shfl_xor_sync(0xffffffffu, t, 1);
+      if (half == 0) hb[bin] = t;
     }
     cl.sync();
-    for (int b = tid; b < 256; b += blockDim.x) {
+    {
       uint32_t t = 0;
-      for (int r0 = 0; r0 < ncta; r0 += 4) {  // four remote reads in flight
+      for (int r0 = half; r0 < ncta; r0 += 8) {  // four remote reads in flight
         uint32_t v[4];
 #pragma unroll
-        for (int r = 0; r < 4; ++r) v[r] = r0 + r < ncta ? cl.map_shared_rank(hb, r0 + r)[b] : 0u;
+        for (int r = 0; r < 4; ++r) v[r] = r0 + 2 * r < ncta ? cl.map_shared_rank(hb, r0 + 2 * r)[bin] : 0u;
         t += (v[0] + v[1]) + (v[2] + v[3]);
       }
-      sh.tot[b] = t;
+      t += __shfl_xor_sync(0xffffffffu, t, 1);
+      if (half == 0) sh.tot[bin] = t;
     }
     __syncthreads();
+    // warp 0: lane L holds bins 8L .. 8L+7; the digit is the bin where the
+    // count of larger keys first reaches need
+    uint32_t* dg = sh.dig[pass & 1];
     if (tid < 32) {
       uint32_t c[8], s = 0;
 #pragma unroll
@@ -146,17 +163,16 @@ __device__ uint32_t cluster_select_desc(cg::cluster_group& cl, const uint32_t* k
 #pragma unroll
       for (int b = 7; b >= 0; --b) {
         if (above < need && need <= above + c[b]) {
-          sh.bcast[0] = (uint32_t)(lane * 8 + b);
-          sh.bcast[1] = above;
+          dg[0] = (uint32_t)(lane * 8 + b);
+          dg[1] = above;
         }
         above += c[b];
       }
     }
     __syncthreads();
-    need -= sh.bcast[1];
-    prefix |= sh.bcast[0] << shift;
+    need -= dg[1];
+    prefix |= dg[0] << shift;
     mask |= 0xffu << shift;
-    __syncthreads();
   }
   *need_out = need;
   return prefix;
@@ -184,23 +200,31 @@ constexpr int kTokText = 0;  // not inside any frame's visual span
 constexpr int kTokPool = 1;  // visual token of a historical frame (the TSG pool)
 constexpr int kTokCur = 2;   // visual token of the current (last) frame
 
-// Visits the tokens j0 + threadIdx.x + k * blockDim.x of [j0, j1) in
-// batches of U per thread: load(t, kind) runs for the whole batch before
-// use(t, kind, value) runs for any of it, so the batch's memory latencies
-// overlap.  Each thread tracks the frame of its (increasing) tokens.
-template <int U, class Load, class Use>
-__device__ __forceinline__ void for_tokens(const FrameTable& ft, int j0, int j1, Load load, Use use) {
-  const int B = blockDim.x, F = ft.n_frames;
-  int f = -1, lo = 0, hi = F - 1;
-  while (lo <= hi) {  // last frame starting at or before j0
+// Last frame starting at or before token t (-1: none), on the shared copy
+// of the frame table.
+__device__ __forceinline__ int frame_at(const SelShared& sh, int F, int t) {
+  int lo = 0, hi = F - 1, f = -1;
+  while (lo <= hi) {
     const int mid = (lo + hi) >> 1;
-    if (ft.off[mid] <= j0) {
+    if (sh.fr_off[mid] <= t) {
       f = mid;
       lo = mid + 1;
     } else {
       hi = mid - 1;
     }
   }
+  return f;
+}
+
+// Visits the tokens j0 + threadIdx.x + k * blockDim.x of [j0, j1) in
+// batches of U per thread: load(t, kind) runs for the whole batch before
+// use(t, kind, value) runs for any of it, so the batch's memory latencies
+// overlap.  Each thread tracks the frame of its (increasing) tokens in the
+// shared copy of the frame table (fr_off ends with INT_MAX).
+template <int U, class Load, class Use>
+__device__ __forceinline__ void for_tokens(const SelShared& sh, int F, int j0, int j1, Load load, Use use) {
+  const int B = blockDim.x;
+  int f = frame_at(sh, F, j0 + (int)threadIdx.x);
   for (int base = j0 + (int)threadIdx.x; base < j1; base += U * B) {
     int kind[U];
     decltype(load(0, 0)) v[U];
@@ -209,8 +233,8 @@ __device__ __forceinline__ void for_tokens(const FrameTable& ft, int j0, int j1,
       const int t = base + u * B;
       kind[u] = -1;
       if (t < j1) {
-        while (f + 1 < F && ft.off[f + 1] <= t) ++f;
-        const bool vis = f >= 0 && t < ft.off[f] + ft.gh[f] * ft.gw[f];
+        while (sh.fr_off[f + 1] <= t) ++f;
+        const bool vis = f >= 0 && t < sh.fr_vend[f];
         kind[u] = vis ? (f + 1 < F ? kTokPool : kTokCur) : kTokText;
         v[u] = load(t, kind[u]);
       }
@@ -223,29 +247,28 @@ __device__ __forceinline__ void for_tokens(const FrameTable& ft, int j0, int j1,
 
 // The same visit in groups of four consecutive tokens t0 .. t0 + 3 (t0 =
 // j0 + 4 (tid + k B)), for 128-bit loads and stores: j0, j1 and every row
-// base are multiples of four tokens.  kinds[e] is the kind of t0 + e.
+// base are multiples of four tokens.  kinds[e] is the kind of t0 + e (one
+// comparison for a group inside one visual span or text run).
 template <class Load4, class Use4>
-__device__ __forceinline__ void for_tokens4(const FrameTable& ft, int j0, int j1, Load4 load4, Use4 use4) {
-  const int B = blockDim.x, F = ft.n_frames;
-  const int first = j0 + 4 * (int)threadIdx.x;
-  int f = -1, lo = 0, hi = F - 1;
-  while (lo <= hi) {  // last frame starting at or before the thread's first token
-    const int mid = (lo + hi) >> 1;
-    if (ft.off[mid] <= first) {
-      f = mid;
-      lo = mid + 1;
-    } else {
-      hi = mid - 1;
-    }
-  }
-  for (int t0 = first; t0 < j1; t0 += 4 * B) {
+__device__ __forceinline__ void for_tokens4(const SelShared& sh, int F, int j0, int j1, Load4 load4, Use4 use4) {
+  const int B = blockDim.x;
+  int f = frame_at(sh, F, j0 + 4 * (int)threadIdx.x);
+  for (int t0 = j0 + 4 * (int)threadIdx.x; t0 < j1; t0 += 4 * B) {
     int kinds[4];
+    while (sh.fr_off[f + 1] <= t0) ++f;
+    const int vend = f >= 0 ? sh.fr_vend[f] : -1, next = sh.fr_off[f + 1];
+    if (t0 + 3 < vend || (t0 >= vend && t0 + 3 < next)) {  // one kind for the group
+      const int k = t0 < vend ? (f + 1 < F ? kTokPool : kTokCur) : kTokText;
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      const int t = t0 + e;
-      while (f + 1 < F && ft.off[f + 1] <= t) ++f;
-      const bool vis = f >= 0 && t < ft.off[f] + ft.gh[f] * ft.gw[f];
-      kinds[e] = vis ? (f + 1 < F ? kTokPool : kTokCur) : kTokText;
+      for (int e = 0; e < 4; ++e) kinds[e] = k;
+    } else {  // the group straddles a span or frame boundary
+      int fe = f;
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int t = t0 + e;
+        while (sh.fr_off[fe + 1] <= t) ++fe;
+        kinds[e] = fe >= 0 && t < sh.fr_vend[fe] ? (fe + 1 < F ? kTokPool : kTokCur) : kTokText;
+      }
     }
     const auto v = load4(t0, kinds);
     use4(t0, kinds, v);
@@ -276,6 +299,12 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
   int pass = 0;
   int pool = 0;
   for (int f = 0; f + 1 < F; ++f) pool += ft.gh[f] * ft.gw[f];
+  // the frame table in shared memory for the token loops' frame tracking
+  for (int f = tid; f <= F; f += blockDim.x) {
+    sh.fr_off[f] = f < F ? ft.off[f] : 0x7fffffff;
+    if (f < F) sh.fr_vend[f] = ft.off[f] + ft.gh[f] * ft.gw[f];
+  }
+  __syncthreads();
   // tau comes from a selection only when there is a pool and TSG is on;
   // otherwise tau = NaN and every gate stays open
   const bool gate_sel = (a.mode & kSelGate) && pool > 0 && a.tsg_enable;
@@ -300,7 +329,7 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
     };
     if (vec) {
       for_tokens4(
-          ft, j0, j1,
+          sh, F, j0, j1,
           [&](int t0, const int (&kinds)[4]) {
             RhoIn4 r;
             const float ninf = -CUDART_INF_F;
@@ -330,14 +359,14 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
             const float r1 = kinds[1] == kTokPool ? finish(m1, v.rn.y) : CUDART_NAN_F;
             const float r2 = kinds[2] == kTokPool ? finish(m2, v.rn.z) : CUDART_NAN_F;
             const float r3 = kinds[3] == kTokPool ? finish(m3, v.rn.w) : CUDART_NAN_F;
-            *reinterpret_cast<float4*>(rho + t0) = make_float4(r0, r1, r2, r3);
+            if (a.write_stages) *reinterpret_cast<float4*>(rho + t0) = make_float4(r0, r1, r2, r3);
             *reinterpret_cast<uint4*>(keys + (t0 - j0)) =
                 make_uint4(kinds[0] == kTokPool ? ~float_key(r0) : 0u, kinds[1] == kTokPool ? ~float_key(r1) : 0u,
                            kinds[2] == kTokPool ? ~float_key(r2) : 0u, kinds[3] == kTokPool ? ~float_key(r3) : 0u);
           });
     } else
     for_tokens<2>(
-        ft, j0, j1,
+        sh, F, j0, j1,
         [&](int t, int kind) {
           // independent loads (no max between them), so that all of a
           // batch's slices are in flight together
@@ -358,7 +387,7 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
         [&](int t, int kind, const RhoIn& v) {
           const float m = fmaxf(fmaxf(v.s[0], v.s[1]), fmaxf(v.s[2], v.s[3]));
           const float r = kind == kTokPool ? finish(m, v.rn) : CUDART_NAN_F;
-          rho[t] = r;
+          if (a.write_stages) rho[t] = r;
           keys[t - j0] = kind == kTokPool ? ~float_key(r) : 0u;
         });
     __syncthreads();
@@ -378,7 +407,7 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
     if (!(a.mode & kSelTopk)) {
       // gate only: Eq. 8 on the pool, open elsewhere
       for_tokens<2>(
-          ft, j0, j1, [&](int, int) { return 0; },
+          sh, F, j0, j1, [&](int, int) { return 0; },
           [&](int t, int kind, int) {
             gate[t] = (kind == kTokPool && gate_sel) ? (key_float(~keys[t - j0]) <= tau ? 1 : 0) : 1;
           });
@@ -410,12 +439,12 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
       float s;
       if (kind == kTokText) {
         s = A + 0.0f;
-        if (fused) gate[t] = 1;
+        if (fused && a.write_stages) gate[t] = 1;
       } else {
         bool g = G != 0.f;
         if (fused) {
           g = !(kind == kTokPool && gate_sel) || key_float(~keys[t - j0]) <= tau;
-          gate[t] = g ? 1 : 0;
+          if (a.write_stages) gate[t] = g ? 1 : 0;
         }
         const float x = alpha != 0.f ? __fmaf_rn(alpha, P, A) : A;
         s = (g ? x : 0.f) + 0.0f;
@@ -424,7 +453,7 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
     };
     if (vec) {
       for_tokens4(
-          ft, j0, j1,
+          sh, F, j0, j1,
           [&](int t0, const int (&kinds)[4]) {
             ScoreIn4 v;
             v.A = ab ? __ldg(reinterpret_cast<const float4*>(ab + t0))
@@ -446,13 +475,13 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
                                       (float)((v.G >> 16) & 0xffu));
             const float s3 = score_of(t0 + 3, kinds[3], v.A.w, kinds[3] != kTokText ? v.P.w : 0.f,
                                       (float)(v.G >> 24));
-            *reinterpret_cast<float4*>(sc + t0) = make_float4(s0, s1, s2, s3);
+            if (a.write_stages) *reinterpret_cast<float4*>(sc + t0) = make_float4(s0, s1, s2, s3);
             *reinterpret_cast<uint4*>(keys + (t0 - j0)) =
                 make_uint4(float_key(s0), float_key(s1), float_key(s2), float_key(s3));
           });
     } else
     for_tokens<2>(
-        ft, j0, j1,
+        sh, F, j0, j1,
         [&](int t, int kind) {
           float A = ab ? __ldg(ab + t) : a.a_uniform;
           if (a_div) A = __fdiv_rn(A, amax);
@@ -462,7 +491,7 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
         },
         [&](int t, int kind, float3 v) {
           const float s = score_of(t, kind, v.x, v.y, v.z);
-          sc[t] = s;
+          if (a.write_stages) sc[t] = s;
           keys[t - j0] = float_key(s);
         });
     __syncthreads();
