@@ -287,20 +287,20 @@ def test_noalloc_shape_limits_match_score(st):
         assert st._lib.stlite_score(ctypes.byref(sh), None, None, None, None, 0, None) == code
 
 
-def test_device_status_without_scratch_argument(st):
+def test_device_status_without_scratch_argument(st, good):
     """stlite_device_status(NULL, ...) reads the no-workspace scratch; a NULL
     status pointer or a misaligned workspace is refused on the host."""
     lib = st._lib
     assert lib.stlite_device_status(None, None, None) == st.STLITE_EINVAL
     status = ctypes.c_int32(0)
-    assert lib.stlite_device_status(ctypes.c_void_p(0x10008), None, ctypes.byref(status)) == st.STLITE_EINVAL
+    assert lib.stlite_device_status(ctypes.c_void_p(good + 8), None, ctypes.byref(status)) == st.STLITE_EINVAL
 
 
-def test_selftest_validation_on_host(st):
+def test_selftest_validation_on_host(st, good):
     """The failure-path diagnostic refuses a NULL or misaligned error word and
     limits outside 1 us .. 2 s before launching anything."""
     lib = st._lib
     assert lib.stlite_selftest_wait_timeout(None, 10_000_000, None) == st.STLITE_EINVAL
-    assert lib.stlite_selftest_wait_timeout(ctypes.c_void_p(0x10008), 10_000_000, None) == st.STLITE_EINVAL
+    assert lib.stlite_selftest_wait_timeout(ctypes.c_void_p(good + 8), 10_000_000, None) == st.STLITE_EINVAL
     for limit in (0, 999, 2_000_000_001):
-        assert lib.stlite_selftest_wait_timeout(ctypes.c_void_p(0x10000), limit, None) == st.STLITE_EINVAL
+        assert lib.stlite_selftest_wait_timeout(ctypes.c_void_p(good), limit, None) == st.STLITE_EINVAL
