@@ -654,18 +654,22 @@ __global__ void __maxnreg__(kScoreMaxReg)
 // Window score pass 2.  CTA (x, h): key tiles of 128 tokens are the A operand
 // (M = 128, one key per TMEM lane), Q of head h (NQ = R rounded up to 32
 // rows) is the B operand.  Each epilogue thread sums 2^(x_r c + bias_r) for
-// its key over its group's range of at most 64 query rows; the four groups'
-// partial sums meet in shared memory.  TMEM: two slots of W columns, so that
+// its key over its group's range of at most 64 query rows; a merge warp adds
+// the four groups' partial sums and stores A_base.  TMEM: two slots of W columns, so that
 // one item drains while the next one is computed.  An item is a key tile
 // against all NQ query columns (W = NQ <= 256), or against one of nh = 2
 // column halves (NQ > 256, rounded to 64, W = NQ / 2).
 struct CsLayout {
   int NQ, nh, W, nstage, kstages, tmem_cols, q_bytes, off_k, off_bias, off_bar, off_xch, total;
 };
-// partial sums [kCsXBuf][kScoreGroups][128 keys] fp32, then the arrival
-// counters [kCsXBuf][4 lane quarters]
+// partial sums [kCsXBuf][kScoreGroups][128 keys] fp32, then the mbarriers
+// xfull[kCsXBuf] (every epilogue warp has parked its partials) and
+// xfree[kCsXBuf] (the merge warp has summed them)
 constexpr int kCsXBuf = 3;
-constexpr int kCsXchBytes = kCsXBuf * kScoreGroups * 128 * 4 + kCsXBuf * 4 * 4;
+constexpr int kCsXchBytes = kCsXBuf * kScoreGroups * 128 * 4 + kCsXBuf * 2 * 8;
+// Column sums add a merge warp (warp 2 + 4 kScoreGroups) to the score
+// passes' TMA, MMA and epilogue warps: 19 warps at 96 registers.
+constexpr int kCsThreads = kScoreThreads + 32;
 __host__ __device__ inline CsLayout cs_layout(int R) {
   CsLayout L;
   L.NQ = R > 256 ? (R + 63) & ~63 : (R + 31) & ~31;
@@ -715,7 +719,8 @@ __global__ void __maxnreg__(kScoreMaxReg)
   const int S = L.kstages;
   const float c = kLog2eF * rsqrtf((float)kD);
   float* xch = reinterpret_cast<float*>(sm + L.off_xch);
-  uint32_t* xcnt = reinterpret_cast<uint32_t*>(sm + L.off_xch + kCsXBuf * kScoreGroups * 128 * 4);
+  const uint32_t b_xfull = smem_u32(sm + L.off_xch + kCsXBuf * kScoreGroups * 128 * 4);
+  const uint32_t b_xfree = b_xfull + 8 * kCsXBuf;
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < S; ++i) {
@@ -726,7 +731,10 @@ __global__ void __maxnreg__(kScoreMaxReg)
       mbar_init(b_accfull + 8 * i, 1);
       mbar_init(b_accempty + 8 * i, 4 * kScoreGroups);  // every epilogue warp
     }
-    for (int i = 0; i < kCsXBuf * 4; ++i) xcnt[i] = 0u;
+    for (int i = 0; i < kCsXBuf; ++i) {
+      mbar_init(b_xfull + 8 * i, 4 * kScoreGroups);
+      mbar_init(b_xfree + 8 * i, 1);
+    }
     mbar_init(b_done, 1);
     *abort_flag = 0u;
     fence_mbar_init();
@@ -802,22 +810,21 @@ __global__ void __maxnreg__(kScoreMaxReg)
       umma_commit(b_done);
       mbar_wait_drain(b_done, 0);
     }
-  } else {
+  } else if (warp < 2 + 4 * kScoreGroups) {
     // Every group drains every item: group g the item's query columns
     // [c0, c1), at most 64; columns of padded rows carry bias = -inf, so
     // they add exact zeros.  A thread's sum runs over the tile's nh items.
-    // The groups' partial sums of a tile meet in shared buffer it % kCsXBuf:
-    // each warp adds one to its lane quarter's arrival counter, and the
-    // warp that arrives last (old value 3 mod 4) adds the four partials in
-    // group order and stores A_base.  Nobody waits for the hand-off.  A
-    // buffer is rewritten at tile it + kCsXBuf, which the MMA can only have
-    // produced once every warp has loaded tile it + 1 from TMEM, i.e. has
-    // finished with tile it.
+    // The groups' partial sums of a tile go to shared buffer it % kCsXBuf
+    // (once the merge warp has released that buffer's previous tile), and
+    // every warp arrives on the buffer's xfull barrier; the merge warp adds
+    // them.  The drain of the next item does not wait for the sum.
     const int g = (warp - 2) >> 2, quarter = warp & 3, row = quarter * 32 + lane;
     const int gwid = (((W + kScoreGroups - 1) / kScoreGroups) + 31) & ~31;
     const int c0 = min(W, g * gwid), c1 = min(W, c0 + gwid);
     const uint32_t lanebase = tmem + ((uint32_t)(quarter * 32) << 16);
     bool ok = true;
+    int xb = 0;         // exchange buffer of tile it (it % kCsXBuf), counted
+    uint32_t xu = 0u;   // uses of that buffer so far (it / kCsXBuf)
     for (int it = 0; ok && it < ntiles; ++it) {
       float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
 #pragma unroll
@@ -876,22 +883,35 @@ __global__ void __maxnreg__(kScoreMaxReg)
         }
       }
       if (!ok) break;
-      const int xb = it % kCsXBuf;
-      float* xp = xch + xb * (kScoreGroups * 128);
-      xp[g * 128 + row] = (a0 + a1) + (a2 + a3);
+      if (xu > 0 && !warp_wait(b_xfree + 8 * xb, (xu - 1u) & 1u, err, abort_flag)) break;
+      xch[xb * (kScoreGroups * 128) + g * 128 + row] = (a0 + a1) + (a2 + a3);
       __syncwarp();
-      uint32_t last = 0u;
-      if (lane == 0) {
-        __threadfence_block();
-        last = (atomicAdd(&xcnt[xb * 4 + quarter], 1u) & 3u) == 3u ? 1u : 0u;
-        __threadfence_block();
+      if (lane == 0) mbar_arrive(b_xfull + 8 * xb);
+      if (++xb == kCsXBuf) {
+        xb = 0;
+        ++xu;
       }
-      last = __shfl_sync(0xffffffffu, last, 0);
+    }
+  } else {
+    // Merge warp: A_base of tile it = the four groups' partials added in
+    // group order, stored by lanes on consecutive keys; then the buffer is
+    // released for tile it + kCsXBuf.
+    int xb = 0;
+    uint32_t xu = 0u;
+    for (int it = 0; it < ntiles; ++it) {
+      if (!warp_wait(b_xfull + 8 * xb, xu & 1u, err, abort_flag)) break;
+      const float* xp = xch + xb * (kScoreGroups * 128);
+      const int tok0 = (blockIdx.x + it * gridDim.x) * 128;
+#pragma unroll
+      for (int r = lane; r < 128; r += 32) {
+        const float acc = (xp[r] + xp[128 + r]) + (xp[256 + r] + xp[384 + r]);
+        if (tok0 + r < n) a_base[(size_t)h * n + tok0 + r] = acc;
+      }
       __syncwarp();
-      if (last) {
-        const float acc = (xp[row] + xp[128 + row]) + (xp[256 + row] + xp[384 + row]);
-        const int tok = (blockIdx.x + it * gridDim.x) * 128 + row;
-        if (tok < n) a_base[(size_t)h * n + tok] = acc;
+      if (lane == 0) mbar_arrive(b_xfree + 8 * xb);
+      if (++xb == kCsXBuf) {
+        xb = 0;
+        ++xu;
       }
     }
   }
@@ -1349,7 +1369,7 @@ cudaError_t launch_score_umma(const Problem& p, const LayerPtrs& io, Strided<flo
   const int tiles = (p.n + 127) / 128;
   const int gx = pick_split(p.L * p.hkv, tiles, sm_count());
   TimingScope ts("colsum_umma", st);
-  cs_kernel<<<dim3(gx, p.L * p.hkv), kScoreThreads, L2.total, st>>>(m2, io, p, rowpart, nsplit, a_base, err);
+  cs_kernel<<<dim3(gx, p.L * p.hkv), kCsThreads, L2.total, st>>>(m2, io, p, rowpart, nsplit, a_base, err);
   return cudaGetLastError();
 }
 
