@@ -28,7 +28,7 @@ struct SelShared {
   uint32_t whist[kSelThreads / 32][256];  // per-warp histograms
   uint32_t hist[2][256];  // this CTA's histogram, double-buffered by pass parity
   uint32_t tot[256];      // cluster-wide histogram of the current pass
-  uint32_t dig[2][2];     // (digit, count above it), double-buffered by pass parity
+  uint32_t dig[2][3];     // (digit, count above it, count in it), double-buffered by pass parity
   uint32_t bcast[4];
   uint32_t warp_tot[32];
   uint32_t counts[2];     // (greater, equal) of this CTA for the compaction
@@ -93,10 +93,15 @@ __device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* w
 // and the digit broadcast are double-buffered by pass parity, so that no
 // barrier is needed before the next pass rewrites them: a buffer is
 // rewritten two passes later, after every thread has passed the barriers
-// that follow its last read.
+// that follow its last read.  early: the caller needs only the top-k set,
+// not the k-th key itself, so the select may stop once the chosen bin holds
+// exactly the keys still needed (all of them belong to the top k); it then
+// returns the bin's lower bound minus one with *need_out = 0, which selects
+// the same set.  Every CTA of the cluster takes that decision on the same
+// cluster histogram.
 __device__ uint32_t cluster_select_desc(cg::cluster_group& cl, const uint32_t* keys, int len,
                                         uint32_t k, SelShared& sh, int& pass,
-                                        uint32_t* need_out) {
+                                        uint32_t* need_out, bool early) {
   uint32_t prefix = 0, mask = 0, need = k;
   const int tid = threadIdx.x, lane = tid & 31, nw = blockDim.x >> 5, wid = tid >> 5;
   const int ncta = (int)cl.num_blocks();
@@ -165,6 +170,7 @@ __device__ uint32_t cluster_select_desc(cg::cluster_group& cl, const uint32_t* k
         if (above < need && need <= above + c[b]) {
           dg[0] = (uint32_t)(lane * 8 + b);
           dg[1] = above;
+          dg[2] = c[b];
         }
         above += c[b];
       }
@@ -173,6 +179,11 @@ __device__ uint32_t cluster_select_desc(cg::cluster_group& cl, const uint32_t* k
     need -= dg[1];
     prefix |= dg[0] << shift;
     mask |= 0xffu << shift;
+    if (early && shift > 0 && dg[2] == need && prefix != 0u) {
+      ++pass;  // the parity sequence of the double buffers goes on
+      *need_out = 0u;
+      return prefix - 1u;
+    }
   }
   *need_out = need;
   return prefix;
@@ -309,6 +320,7 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
   // otherwise tau = NaN and every gate stays open
   const bool gate_sel = (a.mode & kSelGate) && pool > 0 && a.tsg_enable;
   float tau = CUDART_NAN_F;
+  uint32_t kt_gate = 0u;  // gate: rho <= tau, i.e. key (~float_key(rho)) >= kt_gate
   uint8_t* gate = a.gate.base ? a.gate.at(l) + hn : nullptr;
 
   if (a.mode & kSelGate) {
@@ -397,10 +409,13 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
     if (gate_sel) {
       if (a.tsg_fixed) {
         tau = a.tsg_fixed_tau;  // fixed-threshold control: no selection
+        kt_gate = ~float_key(tau);
       } else {
+        // the fused call needs only the gated set; the staged call reports tau
         uint32_t need;
-        const uint32_t kt = cluster_select_desc(cl, keys, len, (uint32_t)min(a.budget[l], pool), sh, pass, &need);
-        tau = key_float(~kt);
+        kt_gate = cluster_select_desc(cl, keys, len, (uint32_t)min(a.budget[l], pool), sh, pass, &need,
+                                      !a.write_stages);
+        tau = key_float(~kt_gate);
       }
     }
     if (c == 0 && tid == 0) a.tau.at(l)[h] = tau;
@@ -409,7 +424,7 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
       for_tokens<2>(
           sh, F, j0, j1, [&](int, int) { return 0; },
           [&](int t, int kind, int) {
-            gate[t] = (kind == kTokPool && gate_sel) ? (key_float(~keys[t - j0]) <= tau ? 1 : 0) : 1;
+            gate[t] = (kind == kTokPool && gate_sel) ? (keys[t - j0] >= kt_gate ? 1 : 0) : 1;
           });
     }
   }
@@ -443,7 +458,7 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
       } else {
         bool g = G != 0.f;
         if (fused) {
-          g = !(kind == kTokPool && gate_sel) || key_float(~keys[t - j0]) <= tau;
+          g = !(kind == kTokPool && gate_sel) || keys[t - j0] >= kt_gate;
           if (a.write_stages) gate[t] = g ? 1 : 0;
         }
         const float x = alpha != 0.f ? __fmaf_rn(alpha, P, A) : A;
@@ -496,7 +511,7 @@ __global__ void __launch_bounds__(kSelThreads, 4) k_select(Problem p, const __gr
         });
     __syncthreads();
     uint32_t need;
-    const uint32_t T = cluster_select_desc(cl, keys, len, (uint32_t)a.budget[l], sh, pass, &need);
+    const uint32_t T = cluster_select_desc(cl, keys, len, (uint32_t)a.budget[l], sh, pass, &need, true);
     // Ordered compaction.  Thread tid owns the contiguous run [r0, r1) of
     // this CTA's keys (odd run length: conflict-free shared reads); one
     // block scan gives its (greater, equal) counts before the run, the
