@@ -1161,30 +1161,86 @@ __global__ void __launch_bounds__(256) k_css_phi(const __grid_constant__ FrameTa
   // c + 1 holds column v0 + c (loads outside the grid are skipped)
   float ra[kPhiRun + 2], rc[kPhiRun + 2], rb[kPhiRun + 2];
   float ec[kPhiRun + 1], sa[kPhiRun], sc[kPhiRun], sea[kPhiRun + 1], sec[kPhiRun], swa[kPhiRun + 1], swc[kPhiRun];
+  static_assert(kPhiRun == 4, "the vector path loads a run as one float4");
+  // 16-byte loads of the run's columns when every row of the arrays and the
+  // frame's rows start on a 16-byte boundary (N, the frame offset and the
+  // grid width multiples of four); v0 + 3 < gw then holds as well
+  if ((n & 3) == 0 && (off & 3) == 0 && (gw & 3) == 0) {
+    auto ld4 = [](const float* p) { return __ldg(reinterpret_cast<const float4*>(p)); };
+    auto put4 = [](float* d, float4 x) {
+      d[0] = x.x;
+      d[1] = x.y;
+      d[2] = x.z;
+      d[3] = x.w;
+    };
+    const bool lf0 = v0 > 0, rt4 = v0 + kPhiRun < gw;
+    put4(rc + 1, ld4(rn + j0));
+    rc[0] = lf0 ? __ldg(rn + j0 - 1) : 0.f;
+    rc[5] = rt4 ? __ldg(rn + j0 + 4) : 0.f;
+    put4(ec + 1, ld4(e + j0));
+    ec[0] = lf0 ? __ldg(e + j0 - 1) : 0.f;
+    if (up) {
+      put4(ra + 1, ld4(rn + j0 - gw));
+      ra[0] = lf0 ? __ldg(rn + j0 - gw - 1) : 0.f;
+      ra[5] = rt4 ? __ldg(rn + j0 - gw + 4) : 0.f;
+      put4(sea + 1, ld4(se + j0 - gw));
+      sea[0] = lf0 ? __ldg(se + j0 - gw - 1) : 0.f;
+      put4(sa, ld4(s + j0 - gw));
+      // SW of (u - 1, v + 2) for c = -1 .. 3: columns v0 + 1 .. v0 + 5
+      const float4 w0 = ld4(sw + j0 - gw);
+      const float4 w1 = rt4 ? ld4(sw + j0 - gw + 4) : make_float4(0.f, 0.f, 0.f, 0.f);
+      swa[0] = w0.y;
+      swa[1] = w0.z;
+      swa[2] = w0.w;
+      swa[3] = w1.x;
+      swa[4] = w1.y;
+    } else {
 #pragma unroll
-  for (int c = -1; c <= kPhiRun; ++c) {
-    const int v = v0 + c;
-    const bool in = v >= 0 && v < gw;
-    rc[c + 1] = in ? __ldg(rn + j0 + c) : 0.f;
-    ra[c + 1] = in && up ? __ldg(rn + j0 + c - gw) : 0.f;
-    rb[c + 1] = in && dn ? __ldg(rn + j0 + c + gw) : 0.f;
-  }
+      for (int i = 0; i < kPhiRun + 2; ++i) ra[i] = 0.f;
 #pragma unroll
-  for (int c = -1; c < kPhiRun; ++c) {
-    const int v = v0 + c;
-    const bool in = v >= 0 && v < gw;
-    ec[c + 1] = in ? __ldg(e + j0 + c) : 0.f;                    // E of (u, v)
-    sea[c + 1] = in && up ? __ldg(se + j0 + c - gw) : 0.f;       // SE of (u - 1, v)
-    const bool in2 = v + 2 >= 0 && v + 2 < gw;
-    swa[c + 1] = in2 && up ? __ldg(sw + j0 + c + 2 - gw) : 0.f;  // SW of (u - 1, v + 2)
-  }
+      for (int i = 0; i < kPhiRun + 1; ++i) sea[i] = swa[i] = 0.f;
 #pragma unroll
-  for (int c = 0; c < kPhiRun; ++c) {
-    const bool in = v0 + c < gw;
-    sa[c] = in && up ? __ldg(s + j0 + c - gw) : 0.f;
-    sc[c] = in && dn ? __ldg(s + j0 + c) : 0.f;
-    sec[c] = in && dn ? __ldg(se + j0 + c) : 0.f;
-    swc[c] = in && dn ? __ldg(sw + j0 + c) : 0.f;
+      for (int i = 0; i < kPhiRun; ++i) sa[i] = 0.f;
+    }
+    if (dn) {
+      put4(rb + 1, ld4(rn + j0 + gw));
+      rb[0] = lf0 ? __ldg(rn + j0 + gw - 1) : 0.f;
+      rb[5] = rt4 ? __ldg(rn + j0 + gw + 4) : 0.f;
+      put4(sc, ld4(s + j0));
+      put4(sec, ld4(se + j0));
+      put4(swc, ld4(sw + j0));
+    } else {
+#pragma unroll
+      for (int i = 0; i < kPhiRun + 2; ++i) rb[i] = 0.f;
+#pragma unroll
+      for (int i = 0; i < kPhiRun; ++i) sc[i] = sec[i] = swc[i] = 0.f;
+    }
+  } else {
+#pragma unroll
+    for (int c = -1; c <= kPhiRun; ++c) {
+      const int v = v0 + c;
+      const bool in = v >= 0 && v < gw;
+      rc[c + 1] = in ? __ldg(rn + j0 + c) : 0.f;
+      ra[c + 1] = in && up ? __ldg(rn + j0 + c - gw) : 0.f;
+      rb[c + 1] = in && dn ? __ldg(rn + j0 + c + gw) : 0.f;
+    }
+#pragma unroll
+    for (int c = -1; c < kPhiRun; ++c) {
+      const int v = v0 + c;
+      const bool in = v >= 0 && v < gw;
+      ec[c + 1] = in ? __ldg(e + j0 + c) : 0.f;                    // E of (u, v)
+      sea[c + 1] = in && up ? __ldg(se + j0 + c - gw) : 0.f;       // SE of (u - 1, v)
+      const bool in2 = v + 2 >= 0 && v + 2 < gw;
+      swa[c + 1] = in2 && up ? __ldg(sw + j0 + c + 2 - gw) : 0.f;  // SW of (u - 1, v + 2)
+    }
+#pragma unroll
+    for (int c = 0; c < kPhiRun; ++c) {
+      const bool in = v0 + c < gw;
+      sa[c] = in && up ? __ldg(s + j0 + c - gw) : 0.f;
+      sc[c] = in && dn ? __ldg(s + j0 + c) : 0.f;
+      sec[c] = in && dn ? __ldg(se + j0 + c) : 0.f;
+      swc[c] = in && dn ? __ldg(sw + j0 + c) : 0.f;
+    }
   }
   float* phi = phi_all.at(l) + hn;
 #pragma unroll
