@@ -510,33 +510,56 @@ __global__ void __launch_bounds__(kRsRows) k_rowstats_simt(const __grid_constant
 // rows, coalesced loads), one pass in split order with eight partials in
 // flight: (M, L) <- (max(M, m_s), L 2^(M - M') + l_s 2^(m_s - M')).
 // grid.y = layer.
+// Folds one split partial (m2, l2) into (m, l): the running max in log2
+// units and the sum of 2^(x - max).  Symmetric in its two arguments, bit for
+// bit (max and a two-term sum commute).
+__device__ __forceinline__ void fold_partial(float& m, float& l, float m2, float l2) {
+  if (!(l2 > 0.f)) return;
+  if (!(l > 0.f)) {
+    m = m2;
+    l = l2;
+    return;
+  }
+  const float mn = fmaxf(m, m2);
+  l = l * exp2f(m - mn) + l2 * exp2f(m2 - mn);
+  m = mn;
+}
+
+// Four lanes per query row: lane q folds splits q, q + 4, q + 8, ... (eight
+// loads in flight), then the four lanes' states are folded pairwise with
+// shuffles, so every lane holds the same bits and lane 0 writes the bias.
+// The order depends on the split count alone.
 __global__ void __launch_bounds__(128) k_row_bias(Problem p, int nsplit, Strided<float2> part_all) {
   const int R = p.R(), l = blockIdx.y;
   const float2* part = part_all.at(l);
   float* bias = reinterpret_cast<float*>(part_all.at(l) + (size_t)p.hkv * nsplit * R);
-  const int e = blockIdx.x * blockDim.x + threadIdx.x;
-  if (e >= p.hkv * R) return;
-  const int h = e / R, r = e - h * R;
-  const float2* pp = part + (size_t)h * nsplit * R + r;
+  const int e4 = blockIdx.x * blockDim.x + threadIdx.x;
+  const int e = e4 >> 2, q = e4 & 3;
+  const bool live = e < p.hkv * R;
   float m = -CUDART_INF_F, lsum = 0.f;
-  for (int s0 = 0; s0 < nsplit; s0 += 8) {
-    float2 v[8];
+  if (live) {
+    const int h = e / R, r = e - h * R;
+    const float2* pp = part + (size_t)h * nsplit * R + r;
+    for (int s0 = q; s0 < nsplit; s0 += 32) {
+      float2 v[8];
 #pragma unroll
-    for (int u = 0; u < 8; ++u) v[u] = s0 + u < nsplit ? pp[(size_t)(s0 + u) * R] : make_float2(-CUDART_INF_F, 0.f);
+      for (int u = 0; u < 8; ++u)
+        v[u] = s0 + 4 * u < nsplit ? pp[(size_t)(s0 + 4 * u) * R] : make_float2(-CUDART_INF_F, 0.f);
 #pragma unroll
-    for (int u = 0; u < 8; ++u) {
-      if (!(v[u].y > 0.f)) continue;
-      const float mn = fmaxf(m, v[u].x);
-      lsum = (lsum > 0.f ? lsum * exp2f(m - mn) : 0.f) + v[u].y * exp2f(v[u].x - mn);
-      m = mn;
+      for (int u = 0; u < 8; ++u) fold_partial(m, lsum, v[u].x, v[u].y);
     }
   }
-  bias[e] = -m - log2f((float)p.G() * lsum);
+#pragma unroll
+  for (int o = 1; o < 4; o <<= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, m, o), l2 = __shfl_xor_sync(0xffffffffu, lsum, o);
+    fold_partial(m, lsum, m2, l2);
+  }
+  if (live && q == 0) bias[e] = -m - log2f((float)p.G() * lsum);
 }
 
 void launch_row_bias(const Problem& p, int nsplit, Strided<float2> rowpart, cudaStream_t st) {
   const int rows = p.hkv * p.R();
-  k_row_bias<<<dim3((rows + 127) / 128, p.L), 128, 0, st>>>(p, nsplit, rowpart);
+  k_row_bias<<<dim3((4 * rows + 127) / 128, p.L), 128, 0, st>>>(p, nsplit, rowpart);
 }
 
 // ---------------------------------------------------------- column sums
