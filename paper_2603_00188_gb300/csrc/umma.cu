@@ -884,6 +884,7 @@ __global__ void __maxnreg__(kScoreMaxReg)
       }
       if (!ok) break;
       if (xu > 0 && !warp_wait(b_xfree + 8 * xb, (xu - 1u) & 1u, err, abort_flag)) break;
+      __syncwarp();  // every lane's store follows lane 0's acquire
       xch[xb * (kScoreGroups * 128) + g * 128 + row] = (a0 + a1) + (a2 + a3);
       __syncwarp();
       if (lane == 0) mbar_arrive(b_xfull + 8 * xb);
