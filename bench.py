@@ -401,7 +401,7 @@ def _read_csrc(name):
 
 def src_digest(read=_read_csrc):
     """Digest of all kernel sources (comments excluded)."""
-    return _digest(os.listdir(CSRC), read)
+    return _digest([n for n in os.listdir(CSRC) if n.endswith((".cu", ".cuh", ".h"))], read)
 
 
 def kernel_digest(kernel: str, read=_read_csrc):
