@@ -148,6 +148,14 @@ WsPlan plan_workspace(const Problem& p, const FrameTable& ft) {
   return w;
 }
 
+// The second stream of a call and its fork / join events (see aux_stream).
+struct AuxStream {
+  unsigned long long ctx_id;
+  cudaStream_t s;
+  cudaEvent_t ev[2];
+};
+AuxStream* aux_stream(cudaStream_t st);
+
 // ---- per-kernel timing ----------------------------------------------------
 namespace {
 struct TimingRecord {
@@ -191,6 +199,84 @@ TimingScope::~TimingScope() {
   if (!stop || cudaEventRecord(stop, st_) != cudaSuccess) return;
   std::lock_guard<std::mutex> lk(g_timing_mu);
   g_records.push_back({name_, start_, stop});
+}
+
+namespace {
+// cuCtxGetCurrent and cuCtxGetId through the runtime's driver entry points
+// (no link against the driver library).
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
+typedef CUresult (*CtxGetIdFn)(CUcontext, unsigned long long*);
+
+bool driver_fns(CtxGetCurrentFn* get_current, CtxGetIdFn* get_id) {
+  static CtxGetCurrentFn cur = nullptr;
+  static CtxGetIdFn id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult qr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &qr) == cudaSuccess &&
+        qr == cudaDriverEntryPointSuccess)
+      cur = reinterpret_cast<CtxGetCurrentFn>(p);
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &qr) == cudaSuccess &&
+        qr == cudaDriverEntryPointSuccess)
+      id = reinterpret_cast<CtxGetIdFn>(p);
+  });
+  *get_current = cur;
+  *get_id = id;
+  return cur && id;
+}
+}  // namespace
+
+cudaError_t current_ctx_id(unsigned long long* out) {
+  CtxGetCurrentFn get_current;
+  CtxGetIdFn get_id;
+  if (!driver_fns(&get_current, &get_id)) return cudaErrorNotSupported;
+  CUcontext ctx = nullptr;
+  if (get_current(&ctx) != CUDA_SUCCESS) return cudaErrorDeviceUninitialized;
+  *out = 0;
+  if (ctx && get_id(ctx, out) != CUDA_SUCCESS) return cudaErrorDeviceUninitialized;
+  return cudaSuccess;
+}
+
+// ---- a second stream for the independent stages of one call ----------------
+// The window score (step 1) does not depend on CSS and TSG (steps 2-3): a
+// call runs it on a second stream, forked from and joined back into the
+// caller's with events, so that SMs that one chain's last wave leaves idle
+// take the other chain's work.  The second stream and its events
+// belong to the calling host thread and device (a thread enqueues its calls
+// in order, so one set of events serves them all); they are made outside
+// graph capture only, and again when the device's context has changed (the
+// old handles went with the old context).  While per-kernel timing is on,
+// every launch stays on the caller's stream, so that each kernel is timed
+// alone.
+namespace {
+constexpr int kMaxAuxDevices = 64;
+thread_local AuxStream t_aux[kMaxAuxDevices];
+}  // namespace
+
+AuxStream* aux_stream(cudaStream_t st) {
+  if (g_timing_on.load(std::memory_order_relaxed)) return nullptr;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxAuxDevices) return nullptr;
+  unsigned long long ctx = 0;
+  if (current_ctx_id(&ctx) != cudaSuccess || ctx == 0) return nullptr;
+  AuxStream& x = t_aux[dev];
+  if (x.s && x.ctx_id == ctx) return &x;
+  if (stream_capturing(st)) return nullptr;
+  AuxStream n = {};
+  n.ctx_id = ctx;
+  bool ok = cudaStreamCreateWithFlags(&n.s, cudaStreamNonBlocking) == cudaSuccess;
+  for (int i = 0; ok && i < 2; ++i) ok = cudaEventCreateWithFlags(&n.ev[i], cudaEventDisableTiming) == cudaSuccess;
+  if (!ok) {
+    for (int i = 0; i < 2; ++i)
+      if (n.ev[i]) cudaEventDestroy(n.ev[i]);
+    if (n.s) cudaStreamDestroy(n.s);
+    (void)cudaGetLastError();
+    return nullptr;
+  }
+  x = n;
+  return &x;
 }
 
 }  // namespace stl
@@ -298,20 +384,35 @@ void select_variants(SelectArgs& a, const stlite_params* params, const Problem& 
 }
 
 // Algorithm 1 for a batch of layers (steps 1-5), every stage one launch.
-// Layer l keeps io.budget[l] tokens per KV head.
+// Layer l keeps io.budget[l] tokens per KV head.  With a second stream
+// (aux_stream), step 1 runs on it beside steps 2-3: CSS and TSG are enqueued
+// first, so that they take the SMs first and the window score fills those
+// their last waves leave idle (the other order measured slower).
 stlite_status compress_batch(const Ctx& c, const stlite_params* params, const LayerPtrs& io) {
   const bool tsg = params->tsg_enable && c.ft.n_frames >= 2;
+  const bool window = params->base_scorer == STLITE_BASE_WINDOW;
   Strided<float> a_base = c.view<float>(c.plan.a_base);
   Strided<float> phi = c.view<float>(c.plan.phi);
+  AuxStream* x = window && (params->css_enable || tsg) ? aux_stream(c.st) : nullptr;
+  cudaError_t e = cudaSuccess;
+  if (x) {
+    e = cudaEventRecord(x->ev[0], c.st);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(x->s, x->ev[0], 0);
+  }
   // CSS also produces the inverse key norms TSG needs; without CSS a plain
   // norms pass provides them.
-  cudaError_t e = cudaSuccess;
-  if (params->css_enable)
+  if (e == cudaSuccess && params->css_enable)
     e = run_css(c, io, phi, params->css_size);
-  else if (tsg)
+  else if (e == cudaSuccess && tsg)
     e = run_norms(c, io);
   if (e == cudaSuccess && tsg) e = run_tsg(c, io, params->tsg_metric);
-  if (e == cudaSuccess && params->base_scorer == STLITE_BASE_WINDOW) e = run_score(c, io, a_base);
+  if (e == cudaSuccess && window) {
+    Ctx cs = c;
+    if (x) cs.st = x->s;
+    e = run_score(cs, io, a_base);
+  }
+  if (e == cudaSuccess && x) e = cudaEventRecord(x->ev[1], x->s);
+  if (e == cudaSuccess && x) e = cudaStreamWaitEvent(c.st, x->ev[1], 0);
   if (e != cudaSuccess) return STLITE_ECUDA;
   SelectArgs a = {};
   a.mode = (tsg ? kSelGate : 0) | kSelTopk;

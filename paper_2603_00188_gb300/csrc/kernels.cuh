@@ -199,6 +199,11 @@ int select_max_tokens();
 // v, k_out, v_out and the budget from io).
 cudaError_t launch_gather(const Problem& p, const LayerPtrs& io, cudaStream_t st);
 
+// The identifier of the context current on this thread (0 if none is):
+// caches of per-context handles compare it to tell a context re-created
+// (cudaDeviceReset, another context made current) from the one they saw.
+cudaError_t current_ctx_id(unsigned long long* out);
+
 // 3-D TMA map (d, head, row) over a bf16 [n][hkv][128] tensor with boxes of
 // 64 x 1 x rows and the 128-byte swizzle.
 cudaError_t make_row_map(CUtensorMap* m, const void* base, int n, int hkv, int rows);

@@ -34,41 +34,6 @@ struct ScratchSlot {
 std::mutex g_setup_mu;
 ScratchSlot g_slot[kMaxDevices] = {};
 
-typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
-typedef CUresult (*CtxGetIdFn)(CUcontext, unsigned long long*);
-
-bool driver_fns(CtxGetCurrentFn* get_current, CtxGetIdFn* get_id) {
-  static CtxGetCurrentFn cur = nullptr;
-  static CtxGetIdFn id = nullptr;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult qr;
-    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &qr) == cudaSuccess &&
-        qr == cudaDriverEntryPointSuccess)
-      cur = reinterpret_cast<CtxGetCurrentFn>(p);
-    p = nullptr;
-    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &qr) == cudaSuccess &&
-        qr == cudaDriverEntryPointSuccess)
-      id = reinterpret_cast<CtxGetIdFn>(p);
-  });
-  *get_current = cur;
-  *get_id = id;
-  return cur && id;
-}
-
-// The identifier of the context current on this thread (0 if none is).
-cudaError_t current_ctx_id(unsigned long long* out) {
-  CtxGetCurrentFn get_current;
-  CtxGetIdFn get_id;
-  if (!driver_fns(&get_current, &get_id)) return cudaErrorNotSupported;
-  CUcontext ctx = nullptr;
-  if (get_current(&ctx) != CUDA_SUCCESS) return cudaErrorDeviceUninitialized;
-  *out = 0;
-  if (ctx && get_id(ctx, out) != CUDA_SUCCESS) return cudaErrorDeviceUninitialized;
-  return cudaSuccess;
-}
-
 // Set-up, with the device current: resolve the array's address once per
 // device and context (cudaGetSymbolAddress, return code checked).
 cudaError_t scratch_address(void** out) {
@@ -77,13 +42,13 @@ cudaError_t scratch_address(void** out) {
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
   unsigned long long ctx = 0;
-  if ((e = current_ctx_id(&ctx)) != cudaSuccess) return e;
+  if ((e = stl::current_ctx_id(&ctx)) != cudaSuccess) return e;
   std::lock_guard<std::mutex> lk(g_setup_mu);
   if (ctx == 0 || !g_slot[dev].addr || g_slot[dev].ctx_id != ctx) {
     void* p = nullptr;
     e = cudaGetSymbolAddress(&p, g_noalloc_scratch);  // makes the device's primary context current if none was
     if (e != cudaSuccess) return e;
-    if ((e = current_ctx_id(&ctx)) != cudaSuccess) return e;
+    if ((e = stl::current_ctx_id(&ctx)) != cudaSuccess) return e;
     if (ctx == 0) return cudaErrorDeviceUninitialized;
     g_slot[dev].ctx_id = ctx;
     g_slot[dev].addr = p;
