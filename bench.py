@@ -877,14 +877,20 @@ def run_gpu(args):
         f0.record(cp_in)
         stream.wait_stream(cp_in)
         cp_out.wait_stream(cp_in)
+        # the end of every step (its last read-back), for the spread of the
+        # intervals between steps: the host link sees other traffic of the
+        # machine, and a step or two that stall for tens of ms raise the mean
+        ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
         for it in range(args.steps):
             e2e_step(it)
+            ends[it].record(cp_out)
         stream.wait_stream(cp_out)
         stream.wait_stream(cp_in)
         f1.record(stream)
         torch.cuda.synchronize()
         barrier()
         ms_e2e = f0.elapsed_time(f1) / args.steps
+        gaps = sorted(ends[i - 1].elapsed_time(ends[i]) for i in range(1, args.steps))
         ms_e2e = max_over_ranks(ms_e2e, dev, world)
         # the host copies hold the device results of the last step
         last = sets[(args.steps - 1) % 2]
@@ -935,8 +941,10 @@ def run_gpu(args):
                     floor_ms=t_both, e2e_over_floor=ms_e2e / t_both,
                     note="cudaMemcpyAsync of the step's bytes from and to page-locked host memory, best of 3; "
                          "floor = both directions at once")
+        spread = dict(min=gaps[0], median=statistics.median(gaps), max=gaps[-1],
+                      note="ms between the ends of consecutive steps (last read-back), rank 0") if gaps else None
         e2e = dict(value=job_throughput(world, L, ms_e2e), unit=UNIT, h2d_bytes_per_step=bi,
-                   d2h_bytes_per_step=bo, ms_per_step=ms_e2e, host_link=link,
+                   d2h_bytes_per_step=bo, ms_per_step=ms_e2e, step_interval_ms=spread, host_link=link,
                    note="q and k copied host -> device by torch (cudaMemcpyAsync on a copy stream) before the "
                         "library call; v read by the compaction kernel in place from page-locked host memory "
                         "(kept rows only); k_out, v_out, idx copied back by torch")

@@ -64,14 +64,6 @@ __device__ __forceinline__ uint8_t* pr_align1024(uint8_t* p) {
   return p + ((1024u - (a & 1023u)) & 1023u);
 }
 
-// Lane 0 polls; the verdict is broadcast so the warp leaves converged.
-__device__ __forceinline__ bool pr_warp_wait(uint32_t bar, uint32_t parity, uint32_t* err,
-                                             volatile uint32_t* abort_flag) {
-  int ok = 1;
-  if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, err, abort_flag) ? 1 : 0;
-  return __shfl_sync(0xffffffffu, ok, 0) != 0;
-}
-
 // Contiguous global -> shared copy completing on `bar` (16-byte aligned
 // addresses, size a multiple of 16).
 __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
@@ -212,7 +204,7 @@ __global__ void __maxnreg__(kPrMaxReg)
     float m = -CUDART_INF_F, l = 0.f;
     for (int it = 0; it < ntiles; ++it) {
       const int as = it & 1;
-      if (!pr_warp_wait(b_accfull + 8 * as, (uint32_t)(it >> 1) & 1u, err, abort_flag)) break;
+      if (!warp_wait(b_accfull + 8 * as, (uint32_t)(it >> 1) & 1u, err, abort_flag)) break;
       tc_fence_after();
       float v[64];
       tmem_ld64(lanebase + as * 256, v);
@@ -401,7 +393,7 @@ __global__ void __maxnreg__(kPrMaxReg)
     int ks = 0;
     for (int it = 0; it < nitems; ++it, ks = ks + 1 == kP2Stages ? 0 : ks + 1) {
       const int as = it & 1;
-      if (!pr_warp_wait(b_accfull + 8 * as, (uint32_t)(it >> 1) & 1u, err, abort_flag)) break;
+      if (!warp_wait(b_accfull + 8 * as, (uint32_t)(it >> 1) & 1u, err, abort_flag)) break;
       tc_fence_after();
       float v[64];
       tmem_ld64(lanebase + as * 256, v);

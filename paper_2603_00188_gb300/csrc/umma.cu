@@ -50,15 +50,6 @@ __device__ __forceinline__ void load_q_sw128(uint8_t* sq, int rows, const __nv_b
   fence_proxy_async_smem();
 }
 
-// Lane 0 polls the barrier; the verdict is broadcast so that the whole warp
-// leaves converged (the tcgen05.ld that follows is .sync.aligned).
-__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, uint32_t* err,
-                                          volatile uint32_t* abort_flag) {
-  int ok = 1;
-  if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, err, abort_flag) ? 1 : 0;
-  return __shfl_sync(0xffffffffu, ok, 0) != 0;
-}
-
 // First token of TSG row tile t and the end of the rows it may write: its
 // frame's visual span, or the whole historical range for spanning tiles.
 // For a loop whose tiles only grow: f carries the frame of the previous
