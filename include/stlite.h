@@ -43,11 +43,12 @@
  *   launches, without synchronising; outputs are valid once the stream has
  *   reached that point.  No call allocates device memory.  The fused calls
  *   (stlite_compress_layer, stlite_compress_layers[_budgets],
- *   stlite_compress_varlen[_layers]) run the window score on a second stream
- *   beside CSS and TSG, forked from `stream` by an event and joined back into
- *   it by another before the selection, so that each call is still ordered
- *   on `stream` alone (and is captured into a graph as one fork and join).
- *   That stream (non-blocking, default priority) and its two events are
+ *   stlite_compress_varlen[_layers]) run the window score, and the last
+ *   kernel of the tensor-core CSS, on a second stream beside TSG, forked from
+ *   `stream` by an event and joined back into it by another before the
+ *   selection, so that each call is still ordered on `stream` alone (and is
+ *   captured into a graph as one fork and join).
+ *   That stream (non-blocking, default priority) and its three events are
  *   created on the first fused call of each host thread on each device, and
  *   again after the device's context changed, and are kept until the process
  *   exits; a call made during stream capture before them runs every stage on

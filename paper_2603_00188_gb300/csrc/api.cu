@@ -148,11 +148,12 @@ WsPlan plan_workspace(const Problem& p, const FrameTable& ft) {
   return w;
 }
 
-// The second stream of a call and its fork / join events (see aux_stream).
+// The second stream of a call and its events: fork, join, CSS dots done
+// (see aux_stream).
 struct AuxStream {
   unsigned long long ctx_id;
   cudaStream_t s;
-  cudaEvent_t ev[2];
+  cudaEvent_t ev[3];
 };
 AuxStream* aux_stream(cudaStream_t st);
 
@@ -240,10 +241,10 @@ cudaError_t current_ctx_id(unsigned long long* out) {
 }
 
 // ---- a second stream for the independent stages of one call ----------------
-// The window score (step 1) does not depend on CSS and TSG (steps 2-3): a
-// call runs it on a second stream, forked from and joined back into the
-// caller's with events, so that SMs that one chain's last wave leaves idle
-// take the other chain's work.  The second stream and its events
+// The window score (step 1) does not depend on CSS and TSG (steps 2-3), nor
+// TSG on CSS's Phi: a call runs the score and Phi on a second stream, forked
+// from and joined back into the caller's with events, so that SMs that one
+// chain's last wave leaves idle take the other chain's work.  The second stream and its events
 // belong to the calling host thread and device (a thread enqueues its calls
 // in order, so one set of events serves them all); they are made outside
 // graph capture only, and again when the device's context has changed (the
@@ -267,9 +268,9 @@ AuxStream* aux_stream(cudaStream_t st) {
   AuxStream n = {};
   n.ctx_id = ctx;
   bool ok = cudaStreamCreateWithFlags(&n.s, cudaStreamNonBlocking) == cudaSuccess;
-  for (int i = 0; ok && i < 2; ++i) ok = cudaEventCreateWithFlags(&n.ev[i], cudaEventDisableTiming) == cudaSuccess;
+  for (int i = 0; ok && i < 3; ++i) ok = cudaEventCreateWithFlags(&n.ev[i], cudaEventDisableTiming) == cudaSuccess;
   if (!ok) {
-    for (int i = 0; i < 2; ++i)
+    for (int i = 0; i < 3; ++i)
       if (n.ev[i]) cudaEventDestroy(n.ev[i]);
     if (n.s) cudaStreamDestroy(n.s);
     (void)cudaGetLastError();
@@ -336,16 +337,30 @@ Strided<T> one(T* p) {
 // kernel; otherwise the CUDA-core one.
 // size: the CSS neighbourhood (0 or 3 = the method's 3x3; 5, 7, 9 = the
 // size ablation, on the box-sum kernel).
-cudaError_t run_css(const Ctx& c, const LayerPtrs& io, Strided<float> phi, int size = 3) {
+// defer_phi: the tensor-core CSS leaves Phi to a later run_css_phi and sets
+// *deferred (the other kernels produce Phi themselves).
+cudaError_t run_css(const Ctx& c, const LayerPtrs& io, Strided<float> phi, int size = 3, bool defer_phi = false,
+                    bool* deferred = nullptr) {
   Strided<float> rn = c.view<float>(c.plan.rn), rc = c.view<float>(c.plan.rn_cur);
+  if (deferred) *deferred = false;
   if (size > 3) return launch_css_box(c.p, c.ft, io, size, phi, rn, rc, c.plan.cur_pad, c.st);
   if (use_tensor_cores(c.p) && css_umma_supported(c.ft)) {
+    if (defer_phi && deferred) *deferred = true;
     const size_t hn4 = (size_t)c.p.hkv * c.p.n * 4;
     Strided<float> dE = c.view<float>(c.plan.dots), dS = c.view<float>(c.plan.dots + hn4);
     Strided<float> dSE = c.view<float>(c.plan.dots + 2 * hn4), dSW = c.view<float>(c.plan.dots + 3 * hn4);
-    return launch_css_umma(c.p, c.ft, io, phi, rn, rc, c.plan.cur_pad, dE, dS, dSE, dSW, c.err, c.st);
+    return launch_css_umma(c.p, c.ft, io, phi, rn, rc, c.plan.cur_pad, dE, dS, dSE, dSW, c.err, c.st,
+                           !(defer_phi && deferred));
   }
   return launch_css(c.p, c.ft, io, phi, rn, rc, c.plan.cur_pad, c.st);
+}
+
+// Phi of a deferred tensor-core CSS (its dots written), on stream st.
+cudaError_t run_css_phi(const Ctx& c, Strided<float> phi, cudaStream_t st) {
+  const size_t hn4 = (size_t)c.p.hkv * c.p.n * 4;
+  return launch_css_phi(c.p, c.ft, phi, c.view<float>(c.plan.rn), c.view<float>(c.plan.rn_cur), c.plan.cur_pad,
+                        c.view<float>(c.plan.dots), c.view<float>(c.plan.dots + hn4),
+                        c.view<float>(c.plan.dots + 2 * hn4), c.view<float>(c.plan.dots + 3 * hn4), st);
 }
 
 // The inverse norms alone: from the CSS kernel when that is the tensor-core
@@ -387,7 +402,10 @@ void select_variants(SelectArgs& a, const stlite_params* params, const Problem& 
 // Layer l keeps io.budget[l] tokens per KV head.  With a second stream
 // (aux_stream), step 1 runs on it beside steps 2-3: CSS and TSG are enqueued
 // first, so that they take the SMs first and the window score fills those
-// their last waves leave idle (the other order measured slower).
+// their last waves leave idle (the other order measured slower).  TSG needs
+// CSS's inverse norms but not Phi, so with the tensor-core CSS its second
+// kernel (Phi from the dots) goes last on the second stream, after an event
+// that marks the dots done: TSG starts as soon as the dots are written.
 stlite_status compress_batch(const Ctx& c, const stlite_params* params, const LayerPtrs& io) {
   const bool tsg = params->tsg_enable && c.ft.n_frames >= 2;
   const bool window = params->base_scorer == STLITE_BASE_WINDOW;
@@ -401,15 +419,22 @@ stlite_status compress_batch(const Ctx& c, const stlite_params* params, const La
   }
   // CSS also produces the inverse key norms TSG needs; without CSS a plain
   // norms pass provides them.
-  if (e == cudaSuccess && params->css_enable)
-    e = run_css(c, io, phi, params->css_size);
-  else if (e == cudaSuccess && tsg)
+  bool late_phi = false;
+  if (e == cudaSuccess && params->css_enable) {
+    e = run_css(c, io, phi, params->css_size, x != nullptr, &late_phi);
+    if (e == cudaSuccess && late_phi) e = cudaEventRecord(x->ev[2], c.st);
+  } else if (e == cudaSuccess && tsg) {
     e = run_norms(c, io);
+  }
   if (e == cudaSuccess && tsg) e = run_tsg(c, io, params->tsg_metric);
   if (e == cudaSuccess && window) {
     Ctx cs = c;
     if (x) cs.st = x->s;
     e = run_score(cs, io, a_base);
+  }
+  if (e == cudaSuccess && late_phi) {
+    e = cudaStreamWaitEvent(x->s, x->ev[2], 0);
+    if (e == cudaSuccess) e = run_css_phi(c, phi, x->s);
   }
   if (e == cudaSuccess && x) e = cudaEventRecord(x->ev[1], x->s);
   if (e == cudaSuccess && x) e = cudaStreamWaitEvent(c.st, x->ev[1], 0);

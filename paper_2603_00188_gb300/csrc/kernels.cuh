@@ -148,7 +148,12 @@ bool css_umma_supported(const FrameTable& ft);
 cudaError_t launch_css_umma(const Problem& p, const FrameTable& ft, const LayerPtrs& io, Strided<float> phi,
                             Strided<float> rn, Strided<float> rn_cur, int cur_pad, Strided<float> dE,
                             Strided<float> dS, Strided<float> dSE, Strided<float> dSW, uint32_t* err,
-                            cudaStream_t st);
+                            cudaStream_t st,
+                            bool with_phi = true);
+// Phi of the CSS dots (the second kernel of launch_css_umma, on its own).
+cudaError_t launch_css_phi(const Problem& p, const FrameTable& ft, Strided<float> phi, Strided<float> rn,
+                           Strided<float> rn_cur, int cur_pad, Strided<float> dE, Strided<float> dS,
+                           Strided<float> dSE, Strided<float> dSW, cudaStream_t st);
 // CSS over the size x size neighbourhood (size 3, 5, 7 or 9; 3 is the
 // method's Moore neighbourhood) on the CUDA cores, through box sums of the
 // normalised keys; any grid width.  Writes phi, rn and rn_cur as launch_css.

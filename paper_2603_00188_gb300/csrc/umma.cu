@@ -1430,7 +1430,7 @@ bool css_umma_supported(const FrameTable& ft) {
 cudaError_t launch_css_umma(const Problem& p, const FrameTable& ft, const LayerPtrs& io, Strided<float> phi,
                             Strided<float> rn, Strided<float> rn_cur, int cur_pad, Strided<float> dE,
                             Strided<float> dS, Strided<float> dSE, Strided<float> dSW, uint32_t* err,
-                            cudaStream_t st) {
+                            cudaStream_t st, bool with_phi) {
   const int tiles = ft.ctile0[ft.n_frames];
   if (tiles == 0) return cudaSuccess;
   KMaps maps;
@@ -1462,6 +1462,21 @@ cudaError_t launch_css_umma(const Problem& p, const FrameTable& ft, const LayerP
     k_css_umma<<<dim3(gx, p.L * p.hkv), kThreads, geo.smem, st>>>(maps, ft, p.hkv, d, geo, err);
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  return with_phi ? launch_css_phi(p, ft, phi, rn, rn_cur, cur_pad, dE, dS, dSE, dSW, st) : cudaSuccess;
+}
+
+cudaError_t launch_css_phi(const Problem& p, const FrameTable& ft, Strided<float> phi, Strided<float> rn,
+                           Strided<float> rn_cur, int cur_pad, Strided<float> dE, Strided<float> dS,
+                           Strided<float> dSE, Strided<float> dSW, cudaStream_t st) {
+  if (ft.ctile0[ft.n_frames] == 0) return cudaSuccess;
+  CssDots d;
+  d.rn = rn;
+  d.dE = dE;
+  d.dS = dS;
+  d.dSE = dSE;
+  d.dSW = dSW;
+  d.rn_cur = rn_cur;
+  d.cur_pad = cur_pad;
   int cmax = 1;  // the most kPhiRun-cell runs of any frame
   for (int f = 0; f < ft.n_frames; ++f) cmax = max(cmax, ft.gh[f] * ((ft.gw[f] + kPhiRun - 1) / kPhiRun));
   TimingScope ts("css_phi", st);
