@@ -213,18 +213,30 @@ __global__ void __maxnreg__(kPrMaxReg)
       if (lane == 0) mbar_arrive(b_accempty + 8 * as);
       const int key0 = it * 256 + g * 64;
       if (key0 + 63 <= pa) {
-        // every row of the tile sees all 64 keys
-        float mx = v[0];
+        // every row of the tile sees all 64 keys.  The maximum over four
+        // independent max3 chains (exact in any order); then exponent
+        // arguments, exponentials and sums in three phases with packed
+        // fp32x2 operations (each lane of a pair rounds as the scalar op)
+        float cm[4];
 #pragma unroll
-        for (int i = 1; i < 64; ++i) mx = fmaxf(mx, v[i]);
+        for (int r = 0; r < 4; ++r) cm[r] = v[r];
+#pragma unroll
+        for (int i = 4; i < 64; i += 8) {
+#pragma unroll
+          for (int r = 0; r < 4; ++r)
+            if (i + 2 * r + 1 < 64) cm[r] = max3(cm[r], v[i + 2 * r], v[i + 2 * r + 1]);
+        }
+        const float mx = fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3]));
         const float mn = fmaxf(m, mx), mnc = mn * c;
         float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
 #pragma unroll
+        for (int i = 0; i < 64; i += 2) fma2(v[i], v[i + 1], c, c, -mnc, -mnc, v[i], v[i + 1]);
+#pragma unroll
+        for (int i = 0; i < 64; ++i) v[i] = ex2_approx(v[i]);
+#pragma unroll
         for (int i = 0; i < 64; i += 4) {
-          s0 += ex2_approx(fmaf(v[i], c, -mnc));
-          s1 += ex2_approx(fmaf(v[i + 1], c, -mnc));
-          s2 += ex2_approx(fmaf(v[i + 2], c, -mnc));
-          s3 += ex2_approx(fmaf(v[i + 3], c, -mnc));
+          add2(s0, s1, v[i], v[i + 1]);
+          add2(s2, s3, v[i + 2], v[i + 3]);
         }
         l = (m == -CUDART_INF_F ? 0.f : l * ex2_approx((m - mn) * c)) + ((s0 + s1) + (s2 + s3));
         m = mn;
@@ -404,14 +416,20 @@ __global__ void __maxnreg__(kPrMaxReg)
       const int p0 = p_first + (cstart + it) * a.p2;
       float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
       if (p0 >= j0 + 127) {
-        // every row of the chunk sees every key of the tile
+        // every row of the chunk sees every key of the tile: exponent
+        // arguments, exponentials and sums in three phases, packed fp32x2
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           const float4 b = b4[i];
-          s0 += ex2_approx(fmaf(v[4 * i], c, b.x));
-          s1 += ex2_approx(fmaf(v[4 * i + 1], c, b.y));
-          s2 += ex2_approx(fmaf(v[4 * i + 2], c, b.z));
-          s3 += ex2_approx(fmaf(v[4 * i + 3], c, b.w));
+          fma2(v[4 * i], v[4 * i + 1], c, c, b.x, b.y, v[4 * i], v[4 * i + 1]);
+          fma2(v[4 * i + 2], v[4 * i + 3], c, c, b.z, b.w, v[4 * i + 2], v[4 * i + 3]);
+        }
+#pragma unroll
+        for (int i = 0; i < 64; ++i) v[i] = ex2_approx(v[i]);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          add2(s0, s1, v[4 * i], v[4 * i + 1]);
+          add2(s2, s3, v[4 * i + 2], v[4 * i + 3]);
         }
       } else {
         const int colmin = max(0, (j - p0) * a.G) - g * 64;  // first visible column of the group's 64
