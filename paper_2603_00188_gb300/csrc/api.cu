@@ -244,13 +244,13 @@ cudaError_t current_ctx_id(unsigned long long* out) {
 // The window score (step 1) does not depend on CSS and TSG (steps 2-3), nor
 // TSG on CSS's Phi: a call runs the score and Phi on a second stream, forked
 // from and joined back into the caller's with events, so that SMs that one
-// chain's last wave leaves idle take the other chain's work.  The second stream and its events
-// belong to the calling host thread and device (a thread enqueues its calls
-// in order, so one set of events serves them all); they are made outside
-// graph capture only, and again when the device's context has changed (the
-// old handles went with the old context).  While per-kernel timing is on,
-// every launch stays on the caller's stream, so that each kernel is timed
-// alone.
+// chain's last wave leaves idle take the other chain's work.  The second
+// stream and its events belong to the calling host thread and device (a
+// thread enqueues its calls in order, so one set of events serves them all);
+// they are made outside graph capture only, and again when the device's
+// context has changed (the old handles went with the old context).  While
+// per-kernel timing is on, every launch stays on the caller's stream, so
+// that each kernel is timed alone.
 namespace {
 constexpr int kMaxAuxDevices = 64;
 thread_local AuxStream t_aux[kMaxAuxDevices];
