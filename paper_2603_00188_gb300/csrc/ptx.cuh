@@ -66,9 +66,9 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint32_
 
 // mbar_wait for a whole warp, which leaves it converged (a tcgen05.ld that
 // follows is .sync.aligned).  Every lane tries the barrier once, and a warp
-// vote takes the verdict: when the phase is already complete, the usual case
+// vote decides: when the phase is already complete, the usual case
 // in the epilogues, no lane branches apart.  Otherwise lane 0 waits with the
-// bounded loop and the verdict is broadcast.  (The earlier form, lane 0
+// bounded loop and the outcome is broadcast.  (The earlier form, lane 0
 // alone polling inside a branch, cost the column sums 8 % and TSG 2 %.)
 __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, uint32_t* err,
                                           volatile uint32_t* abort_flag) {
