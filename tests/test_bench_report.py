@@ -75,6 +75,22 @@ def test_kernel_digest_follows_its_own_units(bench):
     assert all(bench.kernel_digest(k, comment) == base[k] for k in bench.KERNEL_UNITS)
 
 
+def test_src_digest_reads_source_files_only(bench, tmp_path, monkeypatch):
+    # whatever else lands beside the sources (a cache folder of a Python
+    # helper, an editor's backup) neither breaks nor changes the digest
+    (tmp_path / "a.cu").write_text("int a;\n")
+    (tmp_path / "b.cuh").write_text("int b;\n")
+    monkeypatch.setattr(bench, "CSRC", str(tmp_path))
+    read = lambda name: (tmp_path / name).read_text()
+    base = bench.src_digest(read)
+    (tmp_path / "__pycache__").mkdir()
+    (tmp_path / "notes.txt").write_text("x")
+    (tmp_path / "a.cu~").write_text("int z;\n")
+    assert bench.src_digest(read) == base
+    (tmp_path / "c.cu").write_text("int c;\n")
+    assert bench.src_digest(read) != base
+
+
 def test_kernel_roofline_units(bench):
     peaks = {"hbm": 6783.5, "bf16": 1910.3, "bf16_sus": 1704.3, "sm_mhz": 2070.0}
     t = 1e-3
