@@ -143,14 +143,15 @@ cudaError_t launch_css(const Problem& p, const FrameTable& ft, const LayerPtrs& 
                        cudaStream_t st);
 // Tensor-core CSS (bf16, every grid at most 127 wide): per-token squared-norm
 // and E/S/SE/SW dots on the tensor cores, then Phi; writes rn and rn_cur as
-// launch_css does.
+// launch_css does.  with_phi = false stops after the dots (rn and rn_cur
+// written), for a later launch_css_phi on the same dots.
 bool css_umma_supported(const FrameTable& ft);
 cudaError_t launch_css_umma(const Problem& p, const FrameTable& ft, const LayerPtrs& io, Strided<float> phi,
                             Strided<float> rn, Strided<float> rn_cur, int cur_pad, Strided<float> dE,
                             Strided<float> dS, Strided<float> dSE, Strided<float> dSW, uint32_t* err,
-                            cudaStream_t st,
-                            bool with_phi = true);
-// Phi of the CSS dots (the second kernel of launch_css_umma, on its own).
+                            cudaStream_t st, bool with_phi = true);
+// Phi of the CSS dots (the second kernel of launch_css_umma, on its own;
+// the caller orders it after the dots are written).
 cudaError_t launch_css_phi(const Problem& p, const FrameTable& ft, Strided<float> phi, Strided<float> rn,
                            Strided<float> rn_cur, int cur_pad, Strided<float> dE, Strided<float> dS,
                            Strided<float> dSE, Strided<float> dSW, cudaStream_t st);
