@@ -253,7 +253,29 @@ cudaError_t current_ctx_id(unsigned long long* out) {
 // that each kernel is timed alone.
 namespace {
 constexpr int kMaxAuxDevices = 64;
-thread_local AuxStream t_aux[kMaxAuxDevices];
+// The calling thread's second streams, one per device, released when the
+// thread exits: only while the context they were made in is still the
+// device's current one (a stream with work still queued is released by
+// CUDA once that work is done).
+struct AuxSlots {
+  AuxStream slot[kMaxAuxDevices] = {};
+  ~AuxSlots() {
+    int cur = -1;
+    if (cudaGetDevice(&cur) != cudaSuccess) return;
+    for (int d = 0; d < kMaxAuxDevices; ++d) {
+      AuxStream& x = slot[d];
+      if (!x.s || cudaSetDevice(d) != cudaSuccess) continue;
+      unsigned long long ctx = 0;
+      if (current_ctx_id(&ctx) != cudaSuccess || ctx != x.ctx_id) continue;
+      for (cudaEvent_t e : x.ev)
+        if (e) cudaEventDestroy(e);
+      cudaStreamDestroy(x.s);
+    }
+    cudaSetDevice(cur);
+    (void)cudaGetLastError();
+  }
+};
+thread_local AuxSlots t_aux;
 }  // namespace
 
 AuxStream* aux_stream(cudaStream_t st) {
@@ -262,7 +284,7 @@ AuxStream* aux_stream(cudaStream_t st) {
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxAuxDevices) return nullptr;
   unsigned long long ctx = 0;
   if (current_ctx_id(&ctx) != cudaSuccess || ctx == 0) return nullptr;
-  AuxStream& x = t_aux[dev];
+  AuxStream& x = t_aux.slot[dev];
   if (x.s && x.ctx_id == ctx) return &x;
   if (stream_capturing(st)) return nullptr;
   AuxStream n = {};

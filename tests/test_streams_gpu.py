@@ -1,15 +1,18 @@
 """The fused call's schedule does not change its results.
 
-stlite_compress_layers runs the window score on a second stream beside CSS
-and TSG (forked from and joined back into the caller's stream), except while
+stlite_compress_layers runs the window score and CSS's Phi kernel on a
+second stream beside CSS and TSG (forked from and joined back into the
+caller's stream), except while
 per-kernel timing is on, and except for a call captured into a graph before
 its host thread has made an uncaptured call on the device; those run every
 stage on the caller's stream.  Every kernel's arithmetic is deterministic,
 so all of these schedules must give the same indices and the same compacted
 rows, bit for bit: eager with the fork, eager serialised, replayed from a
-graph captured with the fork, and replayed from a graph captured first on a
-fresh host thread.  The workload is the bench's: the 50-step trajectory,
-N = 53,600 tokens, four layers in one call.
+graph captured with the fork, replayed from a graph captured first on a
+fresh host thread, and enqueued by threads that exit at once (releasing
+their second streams with the work still queued) between calls of the main
+thread.  The workload is the bench's: the 50-step trajectory, N = 53,600
+tokens, four layers in one call.
 """
 import threading
 
@@ -132,3 +135,31 @@ def test_first_call_under_capture_on_a_new_thread(st, case):
     if "err" in res:
         raise res["err"]
     same(res["out"], eager(st, case, timing=True))
+
+
+def test_threads_that_exit_release_their_streams(st, case):
+    # each worker enqueues a forked call (creating its second stream) and
+    # exits without waiting, which releases that stream with its work still
+    # queued; the main thread's calls go on with their own
+    ref = eager(st, case, timing=True)
+    pending, outs = [], []
+
+    def run():
+        io, ws, out = outputs(case)
+        stream = torch.cuda.Stream()
+        with torch.cuda.stream(stream):
+            st.stlite_compress_layers(io, case["frames"], case["prm"], ws, stream)
+        pending.append((out, ws, stream))
+
+    for _ in range(3):
+        t = threading.Thread(target=run)
+        t.start()
+        t.join()
+        outs.append(eager(st, case, timing=False))
+    assert len(pending) == 3
+    for out, ws, stream in pending:
+        stream.synchronize()
+        assert st.stlite_device_status(ws, stream) == st.STLITE_OK
+        outs.append(out)
+    for o in outs:
+        same(o, ref)
