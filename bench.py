@@ -221,7 +221,8 @@ def bench_config(layers: int, budget: int, world: int) -> dict:
                 text_per_step=N_TEXT, q_heads=HQ, kv_heads=HKV, head_dim=D, window=W, beta=BETA,
                 budget=budget, l2="inputs larger than L2 (%.2f GB K/V per step)" %
                 (2 * layers * N_TOK * HKV * D * 2 / 1e9),
-                timing="CUDA graph of one step (one stlite_compress_layers call), replayed",
+                timing=("CUDA graph of one step (one stlite_compress_layers call: window score and Phi on the "
+                        "call's second stream, joined before the selection), replayed"),
                 parallelism="dp%d" % world)
 
 
