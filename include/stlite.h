@@ -50,9 +50,10 @@
  *   captured into a graph as one fork and join).
  *   That stream (non-blocking, default priority) and its three events are
  *   created on the first fused call of each host thread on each device, and
- *   again after the device's context changed, and are released when the
- *   thread exits; a call made during stream capture before them runs every
- *   stage on `stream`, as every call does while per-kernel timing is on.
+ *   again after the device's context changed; those of the device current
+ *   when the thread exits are released then (others stay until the process
+ *   exits).  A call made during stream capture before them runs every stage
+ *   on `stream`, as every call does while per-kernel timing is on.
  * Errors.  All arguments are validated on the host before anything is
  *   enqueued; a failed check returns STLITE_EINVAL / STLITE_EUNSUPPORTED /
  *   STLITE_EWORKSPACE and enqueues nothing.  A launch failure returns

@@ -253,25 +253,23 @@ cudaError_t current_ctx_id(unsigned long long* out) {
 // that each kernel is timed alone.
 namespace {
 constexpr int kMaxAuxDevices = 64;
-// The calling thread's second streams, one per device, released when the
-// thread exits: only while the context they were made in is still the
-// device's current one (a stream with work still queued is released by
-// CUDA once that work is done).
+// The calling thread's second streams, one per device.  When the thread
+// exits, the one of the device then current is released if the context it
+// was made in is still current there (a stream with work still queued is
+// released by CUDA once that work is done).  Nothing here makes a device or
+// context current: after a reset that would create a context only to find
+// the handles gone.
 struct AuxSlots {
   AuxStream slot[kMaxAuxDevices] = {};
   ~AuxSlots() {
-    int cur = -1;
-    if (cudaGetDevice(&cur) != cudaSuccess) return;
-    for (int d = 0; d < kMaxAuxDevices; ++d) {
-      AuxStream& x = slot[d];
-      if (!x.s || cudaSetDevice(d) != cudaSuccess) continue;
-      unsigned long long ctx = 0;
-      if (current_ctx_id(&ctx) != cudaSuccess || ctx != x.ctx_id) continue;
-      for (cudaEvent_t e : x.ev)
-        if (e) cudaEventDestroy(e);
-      cudaStreamDestroy(x.s);
-    }
-    cudaSetDevice(cur);
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxAuxDevices) return;
+    AuxStream& x = slot[dev];
+    unsigned long long ctx = 0;
+    if (!x.s || current_ctx_id(&ctx) != cudaSuccess || ctx != x.ctx_id) return;
+    for (cudaEvent_t e : x.ev)
+      if (e) cudaEventDestroy(e);
+    cudaStreamDestroy(x.s);
     (void)cudaGetLastError();
   }
 };
